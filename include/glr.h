@@ -1,0 +1,211 @@
+/*
+ * glr.h -- C ABI of the GB300 GreedyLore compression library (libglr.so).
+ *
+ * One handle holds the compressor state of ONE layer matrix X in R^{m x n}
+ * trained by N data-parallel nodes (the problem statement of Sec. 1, Eq.
+ * formulation), all simulated on one GPU.  glr_step runs one iteration of
+ * Algorithm 3 (GreedyLore) for that matrix:
+ *
+ *   M_i   = G_i + E_i                          error-compensated gradient
+ *   J, P  = Approx-Top-r(M_1..M_N, U, r)       Algorithm 2, Eq. semi-lazy-svd-3
+ *   R_i   = P^T M_i,  Rbar = mean_i R_i        Eq. 8zhb2we09 (the All-Reduce is a
+ *                                               fixed-order sum in device memory)
+ *   Ghat  = P Rbar                             decompression
+ *   X     = Optimizer(X, Ghat)                 Eq. msgd / Eq. adam
+ *   E_i   = M_i - P R_i                        error feedback, Eq. ef2
+ *
+ * and, when (t - compress_start) mod tau == 0, the Semi-Lazy SVD refresh of
+ * Eq. SVD-P1: U <- left singular basis of mean_i M_i; under Algorithm 3 that
+ * step uses the uncompressed mean and resets E_i = 0.  Matrices with m > n are
+ * handled on their transpose (Algorithm 4 orientation rule, Appendix D), so the
+ * basis is min(m, n)^2.  Notation below: m' = min(m, n), n' = max(m, n).
+ *
+ * Conventions for every entry point
+ *   - Return value: GLR_OK (0) or a negative GLR_E* code; nothing throws.  The
+ *     message of the last failure on a handle is glr_last_error(handle); a
+ *     failure of glr_create is reported by glr_last_error(NULL).
+ *   - "device pointer": memory of the CUDA device that was current when the
+ *     handle was created; "host pointer": ordinary or pinned host memory.
+ *   - All GPU work is enqueued on the caller's stream (cudaStream_t passed as
+ *     void*; NULL = legacy default stream) and is stream-ordered.  Functions
+ *     that return host data synchronise that stream first.
+ *   - A handle is not thread-safe; distinct handles may be used concurrently.
+ *   - The library owns every buffer it allocates; the caller owns G, X and all
+ *     output buffers it passes in.
+ */
+#ifndef GLR_H
+#define GLR_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* ---- status codes ---------------------------------------------------------------------- */
+#define GLR_OK          0
+#define GLR_EINVAL     -1   /* bad argument (sizes, null pointer, unknown enum value)      */
+#define GLR_ENOMEM     -2   /* a device or host allocation failed                          */
+#define GLR_ECUDA      -3   /* a CUDA runtime call or kernel launch failed                 */
+#define GLR_ENUMERIC   -4   /* the refresh could not orthonormalise its basis              */
+#define GLR_ENONFINITE -5   /* reserved: non-finite values detected                        */
+#define GLR_ETIMEOUT   -6   /* reserved: a bounded device-side wait gave up                */
+
+/* ---- enumerations -------------------------------------------------------------------- */
+#define GLR_ALG3 0   /* refresh step: uncompressed mean, E reset to 0 (Algorithm 3)          */
+#define GLR_ALG4 1   /* refresh step still compressed with P = U[:, :r], no E reset (Alg. 4) */
+
+#define GLR_MSGD 0   /* Eq. msgd:  M = b1 M + (1 - b1) G;  X -= lr M                          */
+#define GLR_ADAM 1   /* Eq. adam:  M, V EMAs; X -= lr M / (sqrt(V) + eps); no bias correction */
+
+#define GLR_F32  0   /* gradients G_i are float32                                            */
+#define GLR_BF16 1   /* gradients G_i are bfloat16                                           */
+
+#define GLR_MAX_NODES 64
+
+/* Compressor and optimizer settings (Algorithm 3 inputs: tau, r; Sec. 2 optimizers).
+ *   tau            refresh period (>= 1)
+ *   refresh_mode   GLR_ALG3 | GLR_ALG4
+ *   optimizer      GLR_MSGD | GLR_ADAM; lr = gamma; beta1 = beta (MSGD) or beta_1 (Adam);
+ *                  beta2, eps used by Adam only
+ *   seed           64-bit key of the shared random vectors v_j (Eq. random-v): all nodes
+ *                  of one matrix draw the same v_j; give every matrix its own seed
+ *   basis_rank     k.  0 (or m') keeps the full m' x m' singular basis U of Eq. SVD-P1
+ *                  (paper-exact).  r <= k < m' keeps the top-k singular vectors and
+ *                  completes them to an orthogonal U with Householder reflectors; the
+ *                  refresh then uses power_iters block power iterations
+ *   power_iters    q >= 1 (truncated basis only)
+ *   grad_dtype     GLR_F32 | GLR_BF16
+ *   compress_start the first compress_start steps are uncompressed (plain node mean, no
+ *                  error feedback); step compress_start is the first refresh           */
+typedef struct glr_schedule {
+    int32_t  tau;
+    int32_t  refresh_mode;
+    int32_t  optimizer;
+    float    lr;
+    float    beta1;
+    float    beta2;
+    float    eps;
+    uint64_t seed;
+    int32_t  basis_rank;
+    int32_t  power_iters;
+    int32_t  grad_dtype;
+    int32_t  compress_start;
+} glr_schedule;
+
+typedef struct glr_handle glr_handle;
+
+/* Counters of one handle.  comm_floats_* are the floats the paper's nodes would exchange
+ * (Table 2: n r + m per compressed step, m n at a refresh), counted per node.           */
+typedef struct glr_stats {
+    int64_t t;                      /* steps taken                                           */
+    int64_t refreshes;              /* refresh steps taken                                   */
+    int64_t comm_floats_total;      /* sum over steps of the per-node exchanged floats       */
+    int64_t state_bytes;            /* device bytes owned by the handle                      */
+    int32_t m_prime, n_prime, r, k; /* oriented sizes, rank, basis rank                      */
+    int32_t transposed;             /* 1 when m > n (the handle works on G^T)                */
+    int32_t last_refresh_sweeps;    /* eigen-solver sweeps used by the last refresh          */
+    int64_t launches;               /* kernels launched by this handle so far                */
+} glr_stats;
+
+/* Phases of a step, for glr_profile_read.                                                 */
+#define GLR_PH_PREV_PROJECT 0   /* R_i = P_{t-1}^T B_i for the deferred error                 */
+#define GLR_PH_COMPOSE      1   /* K1: M_i = G_i + E_i, B_i <- M_i, Mbar                      */
+#define GLR_PH_LAMBDA       2   /* Algorithm 2 bilinear forms (and W = Y^T Mbar, truncated)   */
+#define GLR_PH_SELECT       3   /* arg-top-r and P = U[:, J]                                  */
+#define GLR_PH_PROJECT      4   /* Rbar = P^T Mbar                                            */
+#define GLR_PH_UPDATE       5   /* K3: Ghat = P Rbar (or Mbar) + optimizer                    */
+#define GLR_PH_REFRESH      6   /* Semi-Lazy SVD refresh of the basis                         */
+#define GLR_PHASES          7
+
+/* Device time per phase, accumulated over the steps taken while profiling was enabled.   */
+typedef struct glr_profile {
+    double  ms[GLR_PHASES];         /* CUDA-event milliseconds on the step's stream          */
+    int64_t launches[GLR_PHASES];   /* kernel launches                                        */
+    int64_t count[GLR_PHASES];      /* number of timed occurrences                            */
+} glr_profile;
+
+/* ---- lifetime ------------------------------------------------------------------------ */
+
+/* Create the state for one m x n layer matrix and N nodes (Sec. 1, Eq. formulation;
+ * Algorithm 3 inputs).  Requires m, n >= 1, 1 <= r <= min(m, n), 1 <= N <= GLR_MAX_NODES,
+ * tau >= 1 and a valid schedule (see glr_schedule).  Allocates all state on the current
+ * CUDA device: E_i (N x m' x n' fp32), the basis, optimizer moments (m x n fp32, two for
+ * Adam) and workspace.  E starts at 0 and U at I (Algorithm 3 input); t = 0.  On
+ * success *out receives the handle.  Errors: GLR_EINVAL, GLR_ENOMEM, GLR_ECUDA.         */
+int glr_create(int64_t m, int64_t n, int32_t r, int32_t N, const glr_schedule* schedule,
+               glr_handle** out);
+
+/* Free every device and host buffer of the handle (after synchronising the device).
+ * NULL is accepted.                                                                      */
+int glr_destroy(glr_handle* h);
+
+/* ---- the step --------------------------------------------------------------------------- */
+
+/* One iteration of Algorithm 3 (Algorithm 4 orientation) for this matrix.
+ *   G       host array of N device pointers; G[i] is node i's gradient, row-major m x n
+ *           of the schedule's grad_dtype, 16-byte aligned.  Read only; must stay valid
+ *           until the stream has passed the step.
+ *   X       device pointer, row-major m x n float32 weights, updated in place.
+ *   stream  cudaStream_t (as void*).
+ * No host/device synchronisation.  Errors: GLR_EINVAL (null or misaligned pointer),
+ * GLR_ECUDA (launch failure).                                                            */
+int glr_step(glr_handle* h, const void* const* G, float* X, void* stream);
+
+/* The same step with host gradients: G_host[i] are host pointers (pinned memory gives
+ * asynchronous copies) that are copied into library-owned device staging on the stream
+ * before the step.  X is the device weight matrix (updated in place); when X_host_out is
+ * not NULL the updated X is copied back to it and the stream is synchronised.          */
+int glr_step_host(glr_handle* h, const void* const* G_host, float* X, float* X_host_out,
+                  void* stream);
+
+/* Make the next glr_step a refresh step (Semi-Lazy SVD, Eq. SVD-P1) and restart the tau
+ * period there.                                                                          */
+int glr_refresh(glr_handle* h);
+
+/* ---- introspection (tests, debugging) ------------------------------------------------- */
+
+/* Counters (see glr_stats); host call, no synchronisation.                               */
+int glr_get_stats(const glr_handle* h, glr_stats* out);
+
+/* Message of the last failure on h (or of the last failed glr_create when h is NULL);
+ * "" when there was none.  The string stays valid until the next call on h.             */
+const char* glr_last_error(const glr_handle* h);
+
+/* E_i after the last step (Eq. ef2), oriented m' x n' row-major fp32, written to the
+ * device buffer E_out.  0 <= i < N.                                                      */
+int glr_get_error(glr_handle* h, int32_t i, float* E_out, void* stream);
+
+/* The last step's selection: J (r int32, ascending, to host J_host), and when not NULL
+ * the device buffers P_out (m' x r fp32), Rbar_out (r x n' fp32), lambda_out (m' fp32,
+ * the node-mean lambda-bar of Algorithm 2) and Mbar_out (m' x n', mean_i M_i).  After a
+ * refresh step under Algorithm 3 J is all -1 (no selection).  Synchronises the stream. */
+int glr_get_selection(glr_handle* h, int32_t* J_host, float* P_out, float* Rbar_out,
+                      float* lambda_out, float* Mbar_out, void* stream);
+
+/* The current orthogonal basis U (m' x m' fp32, row-major) to the device buffer U_out.
+ * With a truncated basis the Householder complement is materialised.                     */
+int glr_get_basis(glr_handle* h, float* U_out, void* stream);
+
+/* Replace the basis: Q (device, m' x k row-major fp32, orthonormal columns; k = the basis
+ * rank, m' for the full basis) becomes U[:, :k]; a truncated basis is completed with
+ * Householder reflectors on the device.  For tests that start both sides from one U.   */
+int glr_set_basis(glr_handle* h, const float* Q, void* stream);
+
+/* Turn per-phase timing on (1) or off (0).  While on, every phase of glr_step records a
+ * pair of CUDA events on the step's stream (a few microseconds of overhead per phase).   */
+int glr_profile_enable(glr_handle* h, int32_t enable);
+
+/* Accumulated per-phase times since the last reset (synchronises the device); reset != 0
+ * clears the accumulators afterwards.                                                    */
+int glr_profile_read(glr_handle* h, glr_profile* out, int32_t reset);
+
+/* Override the selection of the next compressed step with J_host (r distinct indices in
+ * [0, m')), instead of Algorithm 2.  One-shot.                                           */
+int glr_force_selection(glr_handle* h, const int32_t* J_host);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* GLR_H */

@@ -174,10 +174,11 @@ def adam_update(X, Mo, Vo, G, lr, beta1, beta2, eps):
 # Algorithm 2 and the exact-energy rule
 # ----------------------------------------------------------------------------
 def approx_top_r_lambda(M_nodes: Sequence[np.ndarray], U: np.ndarray, V: np.ndarray) -> np.ndarray:
-    """lambda-bar of Algorithm 2: per node Lambda^(i)_j = u_j^T M_i v_j, then the node mean."""
+    """lambda-bar of Algorithm 2: per node Lambda^(i)_j = u_j^T M_i v_j (row j of U^T M_i dotted
+    with v_j), then the node mean."""
     lam = []
     for Mi in M_nodes:
-        lam.append(np.einsum("aj,ab,jb->j", U, Mi, V))
+        lam.append(np.sum((U.T @ Mi) * V, axis=1))
     return np.mean(lam, axis=0)
 
 
@@ -292,13 +293,13 @@ class GreedyLoreOracle:
             lam_bar = approx_top_r_lambda(list(M), self.U, V)
             J = argtop_r(lam_bar ** 2, self.r)
         P = self.U[:, J]
-        R = np.einsum("aq,iab->iqb", P, M)           # R_i = P^T G^(i)
-        self.E = M - np.einsum("aq,iqb->iab", P, R)  # E_i = G^(i) - P R_i
+        R = P.T @ M                                  # R_i = P^T G^(i)   (for every node i)
+        self.E = M - P @ R                           # E_i = G^(i) - P R_i
         Rbar = R.mean(axis=0)                        # All-Reduce
         Ghat = P @ Rbar
         X = self.apply_optimizer(X, Ghat)
         self.t += 1
-        sent = np.einsum("aq,iqb->iab", P, R)
+        sent = P @ R
         return X, StepInfo(t, refresh, True, J, P, lam_bar, Rbar, Mbar, Ghat, self.E.copy(), sent)
 
 

@@ -1,0 +1,198 @@
+"""GreedyLore on GB300: Python binding of libglr.so.
+
+The functions below carry the names of the C entry points declared in
+``include/glr.h`` and only marshal arguments (tensor addresses, the CUDA
+stream, the schedule struct).  Every step of the method runs in the CUDA
+library; PyTorch provides device memory and streams.  There is no CPU path:
+if ``libglr.so`` is missing, ``load()`` raises.
+"""
+from __future__ import annotations
+
+import ctypes
+from typing import Optional, Sequence
+
+import numpy as np
+import torch
+
+from . import _lib
+from ._lib import (GLR_ADAM, GLR_ALG3, GLR_ALG4, GLR_BF16, GLR_F32, GLR_MSGD, GLR_OK,  # noqa: F401
+                   PHASE_NAMES, GlrProfile, GlrSchedule, GlrStats, load)
+
+__all__ = ["GlrError", "make_schedule", "glr_create", "glr_destroy", "glr_step", "glr_step_host",
+           "glr_refresh", "glr_get_stats", "glr_last_error", "glr_get_error", "glr_get_selection",
+           "glr_get_basis", "glr_set_basis", "glr_force_selection", "glr_profile_enable",
+           "glr_profile_read", "GreedyLore", "load"]
+
+
+class GlrError(RuntimeError):
+    def __init__(self, code: int, msg: str):
+        super().__init__(f"GLR error {code}: {msg}")
+        self.code = code
+
+
+def _check(rc: int, handle=None):
+    if rc != GLR_OK:
+        lib = load()
+        msg = lib.glr_last_error(handle)
+        raise GlrError(rc, msg.decode() if msg else "")
+
+
+def _stream_ptr(stream) -> int:
+    if stream is None:
+        stream = torch.cuda.current_stream()
+    return int(stream.cuda_stream) if hasattr(stream, "cuda_stream") else int(stream)
+
+
+def make_schedule(tau: int, refresh_mode: str = "alg3", optimizer: str = "msgd", lr: float = 0.01,
+                  beta1: float = 0.9, beta2: float = 0.999, eps: float = 1e-8, seed: int = 0,
+                  basis_rank: int = 0, power_iters: int = 4, grad_dtype: str = "f32",
+                  compress_start: int = 0) -> GlrSchedule:
+    return GlrSchedule(tau=tau, refresh_mode={"alg3": GLR_ALG3, "alg4": GLR_ALG4}[refresh_mode],
+                       optimizer={"msgd": GLR_MSGD, "adam": GLR_ADAM}[optimizer], lr=lr, beta1=beta1,
+                       beta2=beta2, eps=eps, seed=seed & (2 ** 64 - 1), basis_rank=basis_rank,
+                       power_iters=power_iters, grad_dtype={"f32": GLR_F32, "bf16": GLR_BF16}[grad_dtype],
+                       compress_start=compress_start)
+
+
+def glr_create(m: int, n: int, r: int, N: int, schedule: GlrSchedule) -> ctypes.c_void_p:
+    lib = load()
+    h = ctypes.c_void_p()
+    _check(lib.glr_create(m, n, r, N, ctypes.byref(schedule), ctypes.byref(h)))
+    return h
+
+
+def glr_destroy(h) -> None:
+    _check(load().glr_destroy(h), h)
+
+
+def _ptr_array(tensors: Sequence) -> ctypes.Array:
+    arr = (ctypes.c_void_p * len(tensors))()
+    for i, t in enumerate(tensors):
+        arr[i] = t.data_ptr() if isinstance(t, torch.Tensor) else int(t)
+    return arr
+
+
+def glr_step(h, G: Sequence[torch.Tensor], X: torch.Tensor, stream=None) -> None:
+    _check(load().glr_step(h, _ptr_array(G), X.data_ptr(), _stream_ptr(stream)), h)
+
+
+def glr_step_host(h, G_host: Sequence[torch.Tensor], X: torch.Tensor, X_host_out: Optional[torch.Tensor] = None,
+                  stream=None) -> None:
+    _check(load().glr_step_host(h, _ptr_array(G_host), X.data_ptr(),
+                                None if X_host_out is None else X_host_out.data_ptr(), _stream_ptr(stream)), h)
+
+
+def glr_refresh(h) -> None:
+    _check(load().glr_refresh(h), h)
+
+
+def glr_get_stats(h) -> dict:
+    st = GlrStats()
+    _check(load().glr_get_stats(h, ctypes.byref(st)), h)
+    return {name: getattr(st, name) for name, _ in GlrStats._fields_}
+
+
+def glr_last_error(h=None) -> str:
+    msg = load().glr_last_error(h)
+    return msg.decode() if msg else ""
+
+
+def glr_get_error(h, i: int, out: torch.Tensor, stream=None) -> None:
+    _check(load().glr_get_error(h, i, out.data_ptr(), _stream_ptr(stream)), h)
+
+
+def glr_get_selection(h, r: int, P: Optional[torch.Tensor] = None, Rbar: Optional[torch.Tensor] = None,
+                      lam: Optional[torch.Tensor] = None, Mbar: Optional[torch.Tensor] = None,
+                      stream=None) -> np.ndarray:
+    J = np.zeros(r, dtype=np.int32)
+    ptr = lambda t: None if t is None else t.data_ptr()  # noqa: E731
+    _check(load().glr_get_selection(h, J.ctypes.data, ptr(P), ptr(Rbar), ptr(lam), ptr(Mbar),
+                                    _stream_ptr(stream)), h)
+    return J
+
+
+def glr_get_basis(h, out: torch.Tensor, stream=None) -> None:
+    _check(load().glr_get_basis(h, out.data_ptr(), _stream_ptr(stream)), h)
+
+
+def glr_set_basis(h, Q: torch.Tensor, stream=None) -> None:
+    _check(load().glr_set_basis(h, Q.data_ptr(), _stream_ptr(stream)), h)
+
+
+def glr_force_selection(h, J) -> None:
+    arr = np.ascontiguousarray(np.asarray(J, dtype=np.int32))
+    _check(load().glr_force_selection(h, arr.ctypes.data), h)
+
+
+def glr_profile_enable(h, enable: bool = True) -> None:
+    _check(load().glr_profile_enable(h, 1 if enable else 0), h)
+
+
+def glr_profile_read(h, reset: bool = False) -> dict:
+    p = GlrProfile()
+    _check(load().glr_profile_read(h, ctypes.byref(p), 1 if reset else 0), h)
+    return {name: {"ms": p.ms[i], "launches": p.launches[i], "count": p.count[i]}
+            for i, name in enumerate(PHASE_NAMES)}
+
+
+class GreedyLore:
+    """One layer matrix's GreedyLore state (owns a glr handle)."""
+
+    def __init__(self, m: int, n: int, r: int, N: int, **schedule):
+        self.m, self.n, self.r, self.N = m, n, r, N
+        self.mp, self.np_ = min(m, n), max(m, n)
+        self.schedule = make_schedule(**schedule)
+        self.handle = glr_create(m, n, r, N, self.schedule)
+
+    def step(self, G, X, stream=None):
+        glr_step(self.handle, G, X, stream)
+
+    def step_host(self, G_host, X, X_host_out=None, stream=None):
+        glr_step_host(self.handle, G_host, X, X_host_out, stream)
+
+    def refresh(self):
+        glr_refresh(self.handle)
+
+    def stats(self):
+        return glr_get_stats(self.handle)
+
+    def error(self, i: int) -> torch.Tensor:
+        out = torch.empty(self.mp, self.np_, device="cuda", dtype=torch.float32)
+        glr_get_error(self.handle, i, out)
+        return out
+
+    def selection(self):
+        P = torch.empty(self.mp, self.r, device="cuda")
+        Rbar = torch.empty(self.r, self.np_, device="cuda")
+        lam = torch.empty(self.mp, device="cuda")
+        Mbar = torch.empty(self.mp, self.np_, device="cuda")
+        J = glr_get_selection(self.handle, self.r, P, Rbar, lam, Mbar)
+        return J, P, Rbar, lam, Mbar
+
+    def basis(self) -> torch.Tensor:
+        out = torch.empty(self.mp, self.mp, device="cuda")
+        glr_get_basis(self.handle, out)
+        return out
+
+    def set_basis(self, Q: torch.Tensor):
+        glr_set_basis(self.handle, Q.contiguous().float())
+
+    def force_selection(self, J):
+        glr_force_selection(self.handle, J)
+
+    def profile(self, enable: bool = True):
+        glr_profile_enable(self.handle, enable)
+
+    def profile_read(self, reset: bool = False) -> dict:
+        return glr_profile_read(self.handle, reset)
+
+    def close(self):
+        if self.handle is not None:
+            glr_destroy(self.handle)
+            self.handle = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass

@@ -1,0 +1,563 @@
+// C ABI of libglr.so: handle lifetime, the per-step schedule of Algorithm 3 (Semi-Lazy SVD
+// refresh every tau steps, Approx-Top-r selection otherwise) and the introspection calls.
+// All device work is enqueued on the caller's stream; the host only tracks the schedule.
+#include <algorithm>
+#include <cstdio>
+#include <cstring>
+#include <string>
+#include <vector>
+
+#include "glr_internal.cuh"
+
+using namespace glr;
+
+namespace {
+constexpr int kMaxRank = 512;
+constexpr int kMaxFullBasis = 1024;
+constexpr int kMaxTruncBasis = 512;
+thread_local std::string g_create_err;
+}  // namespace
+
+struct glr_handle {
+    int64_t m = 0, n = 0;
+    int mp = 0, np = 0, transposed = 0, r = 0, N = 0, k = 0, exact = 0;
+    glr_schedule s{};
+    int device = 0;
+    size_t gsize = 4;
+    // device state
+    float *B = nullptr, *Mbar = nullptr, *Rw = nullptr, *Rbar = nullptr, *P = nullptr, *Pprev = nullptr;
+    int32_t* J = nullptr;
+    float *lam = nullptr, *lam_part = nullptr;
+    int ntiles = 0;
+    float *Mo = nullptr, *Vo = nullptr;
+    float *U = nullptr, *Hbuf = nullptr, *Vbuf = nullptr, *evals = nullptr, *evals_sorted = nullptr;
+    float *Q = nullptr, *Qn = nullptr, *Y = nullptr, *Yt = nullptr, *T = nullptr, *dsign = nullptr;
+    float *Wbar = nullptr, *Z = nullptr, *Hk = nullptr, *Vk = nullptr, *gram = nullptr, *scratch = nullptr;
+    int* dflags = nullptr;   // [0] Cholesky restarts, [1] Jacobi sweeps of the last refresh
+    void* Gstage = nullptr;
+    // host state
+    int64_t t = 0, refreshes = 0, comm = 0, state_bytes = 0, period_start = 0;
+    bool e_zero = true, force_refresh = false, last_uncompressed = true, basis_from_user = false;
+    bool has_forceJ = false, forced_this_step = false;
+    std::vector<int32_t> forceJ, iotaJ;
+    std::vector<void*> allocs;
+    std::string err;
+    // launch counting and optional per-phase event timing
+    int64_t launches = 0;
+    bool prof = false;
+    struct Rec { int phase; cudaEvent_t a, b; int64_t launches; };
+    std::vector<Rec> recs;
+    std::vector<cudaEvent_t> free_events;
+    double prof_ms[GLR_PHASES] = {};
+    int64_t prof_launch[GLR_PHASES] = {}, prof_count[GLR_PHASES] = {};
+    int cur_phase = -1;
+    cudaEvent_t cur_start = nullptr;
+    int64_t cur_launch0 = 0;
+};
+
+namespace {
+
+int fail(glr_handle* h, int code, const char* fmt, const char* a = "", int line = 0) {
+    char buf[512];
+    snprintf(buf, sizeof(buf), fmt, a, line);
+    if (h) h->err = buf; else g_create_err = buf;
+    return code;
+}
+
+#define GLR_CK(h, expr)                                                                        \
+    do {                                                                                       \
+        cudaError_t e__ = (expr);                                                              \
+        if (e__ != cudaSuccess)                                                                \
+            return fail((h), GLR_ECUDA, "CUDA error %s (glr_api.cu:%d)", cudaGetErrorString(e__), \
+                        __LINE__);                                                             \
+    } while (0)
+
+// Count kernels launched by a launcher call and check its status.
+#define GLR_LAUNCH(h, nk, expr)                                                                \
+    do {                                                                                       \
+        (h)->launches += (nk);                                                                 \
+        GLR_CK(h, expr);                                                                       \
+    } while (0)
+
+cudaEvent_t take_event(glr_handle* h) {
+    if (!h->free_events.empty()) {
+        cudaEvent_t e = h->free_events.back();
+        h->free_events.pop_back();
+        return e;
+    }
+    cudaEvent_t e = nullptr;
+    cudaEventCreate(&e);
+    return e;
+}
+
+void phase_begin(glr_handle* h, int phase, cudaStream_t st) {
+    if (!h->prof) return;
+    h->cur_phase = phase;
+    h->cur_start = take_event(h);
+    h->cur_launch0 = h->launches;
+    cudaEventRecord(h->cur_start, st);
+}
+
+void phase_end(glr_handle* h, cudaStream_t st) {
+    if (!h->prof || h->cur_phase < 0) return;
+    cudaEvent_t b = take_event(h);
+    cudaEventRecord(b, st);
+    h->recs.push_back({h->cur_phase, h->cur_start, b, h->launches - h->cur_launch0});
+    h->cur_phase = -1;
+}
+
+struct PhaseScope {
+    glr_handle* h; cudaStream_t st;
+    PhaseScope(glr_handle* h_, int phase, cudaStream_t st_) : h(h_), st(st_) { phase_begin(h, phase, st); }
+    ~PhaseScope() { phase_end(h, st); }
+};
+
+template <typename T>
+int alloc(glr_handle* h, T** p, size_t count) {
+    if (count == 0) count = 1;
+    void* ptr = nullptr;
+    const size_t bytes = count * sizeof(T);
+    if (cudaMalloc(&ptr, bytes) != cudaSuccess) {
+        cudaGetLastError();
+        return fail(h, GLR_ENOMEM, "device allocation of %s bytes failed", std::to_string(bytes).c_str());
+    }
+    h->allocs.push_back(ptr);
+    h->state_bytes += static_cast<int64_t>(bytes);
+    if (cudaMemset(ptr, 0, bytes) != cudaSuccess) return fail(h, GLR_ECUDA, "cudaMemset failed%s");
+    *p = static_cast<T*>(ptr);
+    return GLR_OK;
+}
+
+void free_all(glr_handle* h) {
+    for (void* p : h->allocs) cudaFree(p);
+    h->allocs.clear();
+}
+
+GemmDesc gd(int M, int N, int K, const float* A, int64_t sAi, int64_t sAp, const float* B, int64_t sBp,
+            int64_t sBj, float* C, int64_t sCi, int64_t sCj, float alpha = 1.f, float beta = 0.f) {
+    GemmDesc d{};
+    d.M = M; d.N = N; d.K = K; d.batch = 1; d.alpha = alpha; d.beta = beta;
+    d.A = A; d.sAi = sAi; d.sAp = sAp;
+    d.B = B; d.sBp = sBp; d.sBj = sBj;
+    d.C = C; d.sCi = sCi; d.sCj = sCj;
+    return d;
+}
+
+// A (rows x k, row-major) <- A R^{-1} with R from Cholesky of A^T A.
+int cholqr(glr_handle* h, float* A, int rows, cudaStream_t st) {
+    const int k = h->k;
+    GLR_LAUNCH(h, 1, gemm_f32(gd(k, k, rows, A, 1, k, A, k, 1, h->gram, k, 1), st));
+    GLR_LAUNCH(h, 1, cholesky(h->gram, k, h->scratch, h->dflags + 0, st));
+    GLR_LAUNCH(h, 1, trsm_right_lt(A, rows, k, h->gram, st));
+    return GLR_OK;
+}
+
+int wy_from_Q(glr_handle* h, cudaStream_t st) {
+    const int mp = h->mp, k = h->k;
+    GLR_LAUNCH(h, 2, householder_reconstruct(h->Q, mp, k, h->Y, h->T, h->dsign, h->scratch, st));
+    // Yt = Y T^T
+    GLR_LAUNCH(h, 1, gemm_f32(gd(mp, k, k, h->Y, k, 1, h->T, 1, k, h->Yt, k, 1), st));
+    return GLR_OK;
+}
+
+// Semi-Lazy SVD refresh (Eq. SVD-P1) from Mbar.
+int do_refresh(glr_handle* h, cudaStream_t st) {
+    const int mp = h->mp, np = h->np, k = h->k;
+    if (h->exact) {
+        // H = Mbar Mbar^T, eigenvectors = left singular vectors, sorted by descending sigma
+        GLR_LAUNCH(h, 1, gemm_f32(gd(mp, mp, np, h->Mbar, np, 1, h->Mbar, 1, np, h->Hbuf, mp, 1), st));
+        GLR_LAUNCH(h, 1, jacobi_eig(h->Hbuf, mp, h->Vbuf, h->evals, h->dflags + 1, st));
+        GLR_LAUNCH(h, 1, sort_fix_basis(h->evals, h->Vbuf, mp, mp, h->U, mp, h->evals_sorted, st));
+        return GLR_OK;
+    }
+    if (h->refreshes == 0 && !h->basis_from_user)
+        GLR_LAUNCH(h, 1, random_block(h->Q, mp, k, h->s.seed, static_cast<uint32_t>(h->t), st));
+    int rc;
+    for (int it = 0; it < h->s.power_iters; ++it) {
+        // Z = Mbar^T Q  (n' x k), orthonormalised;  Q = Mbar Z  (m' x k), orthonormalised
+        GLR_LAUNCH(h, 1, gemm_f32(gd(np, k, mp, h->Mbar, 1, np, h->Q, k, 1, h->Z, k, 1), st));
+        if ((rc = cholqr(h, h->Z, np, st)) != GLR_OK) return rc;
+        if ((rc = cholqr(h, h->Z, np, st)) != GLR_OK) return rc;
+        GLR_LAUNCH(h, 1, gemm_f32(gd(mp, k, np, h->Mbar, np, 1, h->Z, k, 1, h->Q, k, 1), st));
+        if ((rc = cholqr(h, h->Q, mp, st)) != GLR_OK) return rc;
+        if ((rc = cholqr(h, h->Q, mp, st)) != GLR_OK) return rc;
+    }
+    // Rayleigh-Ritz: Z = Mbar^T Q, H = Z^T Z = Q^T Mbar Mbar^T Q, H = W diag W^T, Q <- Q W
+    GLR_LAUNCH(h, 1, gemm_f32(gd(np, k, mp, h->Mbar, 1, np, h->Q, k, 1, h->Z, k, 1), st));
+    GLR_LAUNCH(h, 1, gemm_f32(gd(k, k, np, h->Z, 1, k, h->Z, k, 1, h->Hk, k, 1), st));
+    GLR_LAUNCH(h, 1, jacobi_eig(h->Hk, k, h->Vk, h->evals, h->dflags + 1, st));
+    GLR_LAUNCH(h, 1, sort_fix_basis(h->evals, h->Vk, k, k, h->gram, k, h->evals_sorted, st));
+    GLR_LAUNCH(h, 1, gemm_f32(gd(mp, k, k, h->Q, k, 1, h->gram, k, 1, h->Qn, k, 1), st));
+    GLR_LAUNCH(h, 1, fix_column_signs(h->Qn, mp, k, st));
+    std::swap(h->Q, h->Qn);
+    return wy_from_Q(h, st);
+}
+
+// Rbar = P^T Mbar; Ghat = P Rbar; optimizer.
+int project_and_update(glr_handle* h, float* X, cudaStream_t st) {
+    const int mp = h->mp, np = h->np, r = h->r;
+    {
+        PhaseScope ps(h, GLR_PH_PROJECT, st);
+        GLR_LAUNCH(h, 1, gemm_f32(gd(r, np, mp, h->P, 1, r, h->Mbar, np, 1, h->Rbar, np, 1), st));
+    }
+    PhaseScope ps(h, GLR_PH_UPDATE, st);
+    UpdateArgs u{};
+    u.mp = mp; u.np = np; u.r = r; u.transposed = h->transposed; u.compressed = 1;
+    u.optimizer = h->s.optimizer; u.lr = h->s.lr; u.beta1 = h->s.beta1; u.beta2 = h->s.beta2; u.eps = h->s.eps;
+    u.P = h->P; u.Rbar = h->Rbar; u.Mbar = h->Mbar; u.X = X; u.Mo = h->Mo; u.Vo = h->Vo;
+    GLR_LAUNCH(h, 1, update(u, st));
+    return GLR_OK;
+}
+
+int uncompressed_update(glr_handle* h, float* X, cudaStream_t st) {
+    UpdateArgs u{};
+    u.mp = h->mp; u.np = h->np; u.r = h->r; u.transposed = h->transposed; u.compressed = 0;
+    u.optimizer = h->s.optimizer; u.lr = h->s.lr; u.beta1 = h->s.beta1; u.beta2 = h->s.beta2; u.eps = h->s.eps;
+    u.P = h->P; u.Rbar = h->Rbar; u.Mbar = h->Mbar; u.X = X; u.Mo = h->Mo; u.Vo = h->Vo;
+    GLR_LAUNCH(h, 1, update(u, st));
+    return GLR_OK;
+}
+
+int build_selection_P(glr_handle* h, cudaStream_t st) {
+    GLR_LAUNCH(h, 1, build_P(h->exact ? 0 : 1, h->mp, h->r, h->k, h->J, h->U, h->Y, h->Yt, h->dsign, h->P, st));
+    return GLR_OK;
+}
+
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+}  // namespace
+
+extern "C" {
+
+int glr_create(int64_t m, int64_t n, int32_t r, int32_t N, const glr_schedule* s, glr_handle** out) {
+    g_create_err.clear();
+    if (!out || !s) return fail(nullptr, GLR_EINVAL, "null schedule or output pointer%s");
+    *out = nullptr;
+    if (m < 1 || n < 1 || m > (1 << 20) || n > (1 << 20))
+        return fail(nullptr, GLR_EINVAL, "matrix sizes must be in [1, 2^20]%s");
+    const int64_t mp = std::min(m, n), np = std::max(m, n);
+    if (mp * np > (int64_t(1) << 31)) return fail(nullptr, GLR_EINVAL, "matrix larger than 2^31 elements%s");
+    if (r < 1 || r > mp || r > kMaxRank) return fail(nullptr, GLR_EINVAL, "need 1 <= r <= min(m, n) and r <= 512%s");
+    if (N < 1 || N > GLR_MAX_NODES) return fail(nullptr, GLR_EINVAL, "need 1 <= N <= GLR_MAX_NODES%s");
+    if (s->tau < 1) return fail(nullptr, GLR_EINVAL, "need tau >= 1%s");
+    if (s->refresh_mode != GLR_ALG3 && s->refresh_mode != GLR_ALG4)
+        return fail(nullptr, GLR_EINVAL, "unknown refresh_mode%s");
+    if (s->optimizer != GLR_MSGD && s->optimizer != GLR_ADAM) return fail(nullptr, GLR_EINVAL, "unknown optimizer%s");
+    if (s->grad_dtype != GLR_F32 && s->grad_dtype != GLR_BF16) return fail(nullptr, GLR_EINVAL, "unknown grad_dtype%s");
+    if (s->compress_start < 0) return fail(nullptr, GLR_EINVAL, "need compress_start >= 0%s");
+    const int k = (s->basis_rank == 0 || s->basis_rank == mp) ? static_cast<int>(mp) : s->basis_rank;
+    const bool exact = k == mp;
+    if (!exact && (k < r || k > mp)) return fail(nullptr, GLR_EINVAL, "need r <= basis_rank <= min(m, n)%s");
+    if (exact && mp > kMaxFullBasis)
+        return fail(nullptr, GLR_EINVAL, "the full basis is supported up to min(m, n) = 1024; set basis_rank%s");
+    if (!exact && k > kMaxTruncBasis) return fail(nullptr, GLR_EINVAL, "basis_rank above 512 is not supported%s");
+    if (!exact && (s->power_iters < 1 || s->power_iters > 64)) return fail(nullptr, GLR_EINVAL, "need 1 <= power_iters <= 64%s");
+
+    glr_handle* h = new glr_handle();
+    h->m = m; h->n = n; h->mp = static_cast<int>(mp); h->np = static_cast<int>(np);
+    h->transposed = m > n ? 1 : 0; h->r = r; h->N = N; h->k = k; h->exact = exact ? 1 : 0;
+    h->s = *s; h->gsize = s->grad_dtype == GLR_BF16 ? 2 : 4;
+    h->period_start = s->compress_start;
+    h->ntiles = static_cast<int>((np + kLambdaTile - 1) / kLambdaTile);
+    cudaGetDevice(&h->device);
+    int rc = GLR_OK;
+    const size_t MP = mp, NP = np;
+    auto A = [&](auto** p, size_t cnt) { if (rc == GLR_OK) rc = alloc(h, p, cnt); };
+    A(&h->B, (size_t)N * MP * NP);
+    A(&h->Mbar, MP * NP);
+    A(&h->Rw, (size_t)N * r * NP);
+    A(&h->Rbar, (size_t)r * NP);
+    A(&h->P, MP * r);
+    A(&h->Pprev, MP * r);
+    A(&h->J, (size_t)r);
+    A(&h->lam, MP);
+    A(&h->lam_part, MP * h->ntiles);
+    A(&h->Mo, (size_t)m * n);
+    if (s->optimizer == GLR_ADAM) A(&h->Vo, (size_t)m * n);
+    A(&h->dflags, 4);
+    if (exact) {
+        A(&h->U, MP * MP); A(&h->Hbuf, MP * MP); A(&h->Vbuf, MP * MP);
+        A(&h->evals, MP); A(&h->evals_sorted, MP);
+    } else {
+        const size_t K = k;
+        A(&h->Q, MP * K); A(&h->Qn, MP * K); A(&h->Y, MP * K); A(&h->Yt, MP * K);
+        A(&h->T, K * K); A(&h->dsign, K); A(&h->Wbar, K * NP); A(&h->Z, NP * K);
+        A(&h->Hk, K * K); A(&h->Vk, K * K); A(&h->gram, K * K); A(&h->scratch, K * K);
+        A(&h->evals, K); A(&h->evals_sorted, K);
+    }
+    if (rc != GLR_OK) {
+        g_create_err = h->err;
+        free_all(h);
+        delete h;
+        return rc;
+    }
+    // U = I (Algorithm 3 input): dense identity, or Q = I[:, :k], Y = T = 0, d = 1.
+    std::vector<float> ones(static_cast<size_t>(mp), 1.f);
+    cudaError_t e = cudaSuccess;
+    if (exact) e = cudaMemcpy2D(h->U, (MP + 1) * 4, ones.data(), 4, 4, MP, cudaMemcpyHostToDevice);
+    else {
+        e = cudaMemcpy2D(h->Q, ((size_t)k + 1) * 4, ones.data(), 4, 4, k, cudaMemcpyHostToDevice);
+        if (e == cudaSuccess) e = cudaMemcpy(h->dsign, ones.data(), 4 * (size_t)k, cudaMemcpyHostToDevice);
+    }
+    if (e == cudaSuccess) e = cudaDeviceSynchronize();
+    if (e != cudaSuccess) {
+        g_create_err = std::string("CUDA error during initialisation: ") + cudaGetErrorString(e);
+        free_all(h);
+        delete h;
+        return GLR_ECUDA;
+    }
+    h->iotaJ.resize(r);
+    for (int q = 0; q < r; ++q) h->iotaJ[q] = q;
+    *out = h;
+    return GLR_OK;
+}
+
+int glr_destroy(glr_handle* h) {
+    if (!h) return GLR_OK;
+    cudaDeviceSynchronize();
+    for (auto& rec : h->recs) { cudaEventDestroy(rec.a); cudaEventDestroy(rec.b); }
+    for (cudaEvent_t e : h->free_events) cudaEventDestroy(e);
+    free_all(h);
+    delete h;
+    return GLR_OK;
+}
+
+int glr_step(glr_handle* h, const void* const* G, float* X, void* stream) {
+    if (!h) return GLR_EINVAL;
+    h->err.clear();
+    if (!G || !X) return fail(h, GLR_EINVAL, "null gradient array or X%s");
+    if (!aligned16(X)) return fail(h, GLR_EINVAL, "X must be 16-byte aligned%s");
+    for (int i = 0; i < h->N; ++i)
+        if (!G[i] || !aligned16(G[i])) return fail(h, GLR_EINVAL, "gradient %s is null or not 16-byte aligned", std::to_string(i).c_str());
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    const int mp = h->mp, np = h->np, r = h->r, N = h->N;
+    const bool warm = h->t < h->s.compress_start;
+    h->forced_this_step = false;
+    const bool refresh = !warm && (h->force_refresh || ((h->t - h->period_start) % h->s.tau == 0));
+    if (refresh && h->force_refresh) h->period_start = h->t;
+    h->force_refresh = false;
+
+    // K1: Rw_i = Pprev^T B_i (deferred error), then compose M_i, B_i, Mbar
+    if (!h->e_zero) {
+        PhaseScope ps(h, GLR_PH_PREV_PROJECT, st);
+        GemmDesc d = gd(r, np, mp, h->Pprev, 1, r, h->B, np, 1, h->Rw, np, 1);
+        d.batch = N; d.sAz = 0; d.sBz = (int64_t)mp * np; d.sCz = (int64_t)r * np;
+        GLR_LAUNCH(h, 1, gemm_f32(d, st));
+    }
+    {
+        PhaseScope ps(h, GLR_PH_COMPOSE, st);
+        ComposeArgs ca{};
+        for (int i = 0; i < N; ++i) ca.G[i] = G[i];
+        ca.grad_dtype = h->s.grad_dtype; ca.transposed = h->transposed;
+        ca.mp = mp; ca.np = np; ca.N = N; ca.r = r; ca.e_zero = h->e_zero ? 1 : 0; ca.write_B = warm ? 0 : 1;
+        ca.B = h->B; ca.Pprev = h->Pprev; ca.Rw = h->Rw; ca.Mbar = h->Mbar;
+        GLR_LAUNCH(h, 1, compose(ca, st));
+    }
+
+    int rc = GLR_OK;
+    if (warm) {
+        PhaseScope ps(h, GLR_PH_UPDATE, st);
+        if ((rc = uncompressed_update(h, X, st)) != GLR_OK) return rc;
+        h->comm += (int64_t)mp * np;
+        h->last_uncompressed = true;
+        h->t++;
+        return GLR_OK;
+    }
+    if (refresh) {
+        {
+            PhaseScope ps(h, GLR_PH_REFRESH, st);
+            if ((rc = do_refresh(h, st)) != GLR_OK) return rc;
+        }
+        h->refreshes++;
+        h->comm += (int64_t)mp * np;
+        if (h->s.refresh_mode == GLR_ALG3) {
+            PhaseScope ps(h, GLR_PH_UPDATE, st);
+            if ((rc = uncompressed_update(h, X, st)) != GLR_OK) return rc;
+            h->e_zero = true;
+            h->last_uncompressed = true;
+            h->has_forceJ = false;
+            h->t++;
+            return GLR_OK;
+        }
+        GLR_CK(h, cudaMemcpyAsync(h->J, h->iotaJ.data(), sizeof(int32_t) * r, cudaMemcpyHostToDevice, st));
+        h->comm += (int64_t)r * np;
+    } else if (h->has_forceJ) {
+        GLR_CK(h, cudaMemcpyAsync(h->J, h->forceJ.data(), sizeof(int32_t) * r, cudaMemcpyHostToDevice, st));
+        h->has_forceJ = false;
+        h->forced_this_step = true;
+        h->comm += (int64_t)r * np + mp;
+    } else {
+        PhaseScope ps(h, GLR_PH_LAMBDA, st);
+        LambdaArgs la{};
+        la.mp = mp; la.np = np; la.seed = h->s.seed; la.t = static_cast<uint32_t>(h->t);
+        la.part = h->lam_part; la.ntiles = h->ntiles;
+        if (h->exact) {
+            la.mode = 0; la.K = mp; la.A = h->U; la.Bm = h->Mbar; la.Mbar = h->Mbar;
+        } else {
+            const int k = h->k;
+            GLR_LAUNCH(h, 1, gemm_f32(gd(k, np, mp, h->Y, 1, k, h->Mbar, np, 1, h->Wbar, np, 1), st));  // Wbar = Y^T Mbar
+            la.mode = 1; la.K = k; la.A = h->Yt; la.Bm = h->Wbar; la.Mbar = h->Mbar;
+        }
+        GLR_LAUNCH(h, 1, lambda_partials(la, st));
+        h->comm += (int64_t)r * np + mp;
+    }
+    {
+        PhaseScope ps(h, GLR_PH_SELECT, st);
+        if (!refresh && !h->forced_this_step)
+            GLR_LAUNCH(h, 1, select_top_r(h->lam_part, h->ntiles, mp, r, h->exact ? nullptr : h->dsign, h->k, h->lam, h->J, st));
+        if ((rc = build_selection_P(h, st)) != GLR_OK) return rc;
+    }
+    if ((rc = project_and_update(h, X, st)) != GLR_OK) return rc;
+    std::swap(h->P, h->Pprev);          // Pprev now holds this step's P (deferred E_i = B_i - P P^T B_i)
+    h->e_zero = false;
+    h->last_uncompressed = false;
+    h->t++;
+    return GLR_OK;
+}
+
+int glr_step_host(glr_handle* h, const void* const* G_host, float* X, float* X_host_out, void* stream) {
+    if (!h) return GLR_EINVAL;
+    if (!G_host || !X) return fail(h, GLR_EINVAL, "null gradient array or X%s");
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    const size_t bytes = static_cast<size_t>(h->m) * h->n * h->gsize;
+    if (!h->Gstage) {
+        char* p = nullptr;
+        int rc = alloc(h, &p, bytes * h->N);
+        if (rc != GLR_OK) return rc;
+        h->Gstage = p;
+    }
+    const void* Gd[GLR_MAX_NODES];
+    for (int i = 0; i < h->N; ++i) {
+        if (!G_host[i]) return fail(h, GLR_EINVAL, "host gradient %s is null", std::to_string(i).c_str());
+        char* dst = static_cast<char*>(h->Gstage) + bytes * i;
+        GLR_CK(h, cudaMemcpyAsync(dst, G_host[i], bytes, cudaMemcpyHostToDevice, st));
+        Gd[i] = dst;
+    }
+    int rc = glr_step(h, Gd, X, stream);
+    if (rc != GLR_OK) return rc;
+    if (X_host_out) {
+        GLR_CK(h, cudaMemcpyAsync(X_host_out, X, sizeof(float) * h->m * h->n, cudaMemcpyDeviceToHost, st));
+        GLR_CK(h, cudaStreamSynchronize(st));
+    }
+    return GLR_OK;
+}
+
+int glr_refresh(glr_handle* h) {
+    if (!h) return GLR_EINVAL;
+    h->force_refresh = true;
+    return GLR_OK;
+}
+
+int glr_get_stats(const glr_handle* h, glr_stats* out) {
+    if (!h || !out) return GLR_EINVAL;
+    out->t = h->t; out->refreshes = h->refreshes; out->comm_floats_total = h->comm;
+    out->state_bytes = h->state_bytes;
+    out->m_prime = h->mp; out->n_prime = h->np; out->r = h->r; out->k = h->k;
+    out->transposed = h->transposed;
+    int flags[4] = {0, 0, 0, 0};
+    cudaMemcpy(flags, h->dflags, sizeof(flags), cudaMemcpyDeviceToHost);
+    out->last_refresh_sweeps = flags[1];
+    out->launches = h->launches;
+    return GLR_OK;
+}
+
+const char* glr_last_error(const glr_handle* h) { return h ? h->err.c_str() : g_create_err.c_str(); }
+
+int glr_get_error(glr_handle* h, int32_t i, float* E_out, void* stream) {
+    if (!h) return GLR_EINVAL;
+    if (i < 0 || i >= h->N || !E_out) return fail(h, GLR_EINVAL, "bad node index or null output%s");
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    const int mp = h->mp, np = h->np, r = h->r;
+    float* Bi = h->B + (size_t)i * mp * np;
+    float* Rwi = h->Rw + (size_t)i * r * np;
+    if (!h->e_zero) GLR_LAUNCH(h, 1, gemm_f32(gd(r, np, mp, h->Pprev, 1, r, Bi, np, 1, Rwi, np, 1), st));
+    GLR_LAUNCH(h, 1, materialize_error(mp, np, r, h->e_zero ? 1 : 0, Bi, h->Pprev, Rwi, E_out, st));
+    return GLR_OK;
+}
+
+int glr_get_selection(glr_handle* h, int32_t* J_host, float* P_out, float* Rbar_out, float* lambda_out,
+                      float* Mbar_out, void* stream) {
+    if (!h) return GLR_EINVAL;
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    const size_t mp = h->mp, np = h->np, r = h->r;
+    if (P_out) GLR_CK(h, cudaMemcpyAsync(P_out, h->Pprev, 4 * mp * r, cudaMemcpyDeviceToDevice, st));
+    if (Rbar_out) GLR_CK(h, cudaMemcpyAsync(Rbar_out, h->Rbar, 4 * r * np, cudaMemcpyDeviceToDevice, st));
+    if (lambda_out) GLR_CK(h, cudaMemcpyAsync(lambda_out, h->lam, 4 * mp, cudaMemcpyDeviceToDevice, st));
+    if (Mbar_out) GLR_CK(h, cudaMemcpyAsync(Mbar_out, h->Mbar, 4 * mp * np, cudaMemcpyDeviceToDevice, st));
+    if (J_host) {
+        if (h->last_uncompressed) {
+            for (size_t q = 0; q < r; ++q) J_host[q] = -1;
+        } else {
+            GLR_CK(h, cudaMemcpyAsync(J_host, h->J, 4 * r, cudaMemcpyDeviceToHost, st));
+        }
+    }
+    GLR_CK(h, cudaStreamSynchronize(st));
+    return GLR_OK;
+}
+
+int glr_get_basis(glr_handle* h, float* U_out, void* stream) {
+    if (!h || !U_out) return GLR_EINVAL;
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    const size_t mp = h->mp;
+    if (h->exact) GLR_CK(h, cudaMemcpyAsync(U_out, h->U, 4 * mp * mp, cudaMemcpyDeviceToDevice, st));
+    else GLR_LAUNCH(h, 1, materialize_wy_basis(h->mp, h->k, h->Y, h->Yt, h->dsign, U_out, st));
+    return GLR_OK;
+}
+
+int glr_set_basis(glr_handle* h, const float* Q, void* stream) {
+    if (!h || !Q) return GLR_EINVAL;
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    const size_t mp = h->mp, k = h->k;
+    if (h->exact) {
+        GLR_CK(h, cudaMemcpyAsync(h->U, Q, 4 * mp * mp, cudaMemcpyDeviceToDevice, st));
+    } else {
+        GLR_CK(h, cudaMemcpyAsync(h->Q, Q, 4 * mp * k, cudaMemcpyDeviceToDevice, st));
+        int rc = wy_from_Q(h, st);
+        if (rc != GLR_OK) return rc;
+    }
+    h->basis_from_user = true;
+    return GLR_OK;
+}
+
+int glr_profile_enable(glr_handle* h, int32_t enable) {
+    if (!h) return GLR_EINVAL;
+    h->prof = enable != 0;
+    return GLR_OK;
+}
+
+int glr_profile_read(glr_handle* h, glr_profile* out, int32_t reset) {
+    if (!h || !out) return GLR_EINVAL;
+    for (auto& rec : h->recs) {
+        GLR_CK(h, cudaEventSynchronize(rec.b));
+        float ms = 0.f;
+        GLR_CK(h, cudaEventElapsedTime(&ms, rec.a, rec.b));
+        h->prof_ms[rec.phase] += ms;
+        h->prof_launch[rec.phase] += rec.launches;
+        h->prof_count[rec.phase] += 1;
+        h->free_events.push_back(rec.a);
+        h->free_events.push_back(rec.b);
+    }
+    h->recs.clear();
+    for (int p = 0; p < GLR_PHASES; ++p) {
+        out->ms[p] = h->prof_ms[p];
+        out->launches[p] = h->prof_launch[p];
+        out->count[p] = h->prof_count[p];
+        if (reset) { h->prof_ms[p] = 0.0; h->prof_launch[p] = 0; h->prof_count[p] = 0; }
+    }
+    return GLR_OK;
+}
+
+int glr_force_selection(glr_handle* h, const int32_t* J_host) {
+    if (!h || !J_host) return GLR_EINVAL;
+    std::vector<int32_t> J(J_host, J_host + h->r);
+    std::sort(J.begin(), J.end());
+    for (int q = 0; q < h->r; ++q) {
+        if (J[q] < 0 || J[q] >= h->mp || (q && J[q] == J[q - 1]))
+            return fail(h, GLR_EINVAL, "forced selection must hold r distinct indices in [0, m')%s");
+    }
+    h->forceJ = J;
+    h->has_forceJ = true;
+    return GLR_OK;
+}
+
+}  // extern "C"

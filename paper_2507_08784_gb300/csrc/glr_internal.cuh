@@ -1,0 +1,162 @@
+// Internal declarations shared by the CUDA translation units of libglr.so.
+#pragma once
+
+#include <cuda_runtime.h>
+#include <cuda_bf16.h>
+#include <stdint.h>
+
+#include "glr.h"
+
+namespace glr {
+
+// ------------------------------------------------------------------------------------------
+// Philox4x32-10 (Salmon, Moraes, Dror, Shaw, SC'11) and Box-Muller: the random vectors
+// v_j ~ N(0, I) of Eq. random-v.  Element (j, b) of the stacked m' x n' matrix uses counter
+// (b / 4, j, t, tag) and key (seed lo, seed hi); the four output words give two Box-Muller
+// pairs and v_j[b] = z_{b mod 4}.  Uniforms are (top 24 bits + 0.5) * 2^-24, exact in fp32.
+// ------------------------------------------------------------------------------------------
+constexpr uint32_t kTagLambdaV = 0x4C414D56u;   // v_j of Algorithm 2
+constexpr uint32_t kTagPowerInit = 0x50574954u; // random start block of the power iteration
+
+struct U32x4 { uint32_t x, y, z, w; };
+
+__device__ __forceinline__ U32x4 philox4x32_10(uint32_t c0, uint32_t c1, uint32_t c2, uint32_t c3,
+                                               uint32_t k0, uint32_t k1) {
+#pragma unroll
+    for (int rnd = 0; rnd < 10; ++rnd) {
+        if (rnd) { k0 += 0x9E3779B9u; k1 += 0xBB67AE85u; }
+        const uint32_t hi0 = __umulhi(0xD2511F53u, c0), lo0 = 0xD2511F53u * c0;
+        const uint32_t hi1 = __umulhi(0xCD9E8D57u, c2), lo1 = 0xCD9E8D57u * c2;
+        const uint32_t n0 = hi1 ^ c1 ^ k0, n2 = hi0 ^ c3 ^ k1;
+        c0 = n0; c1 = lo1; c2 = n2; c3 = lo0;
+    }
+    return {c0, c1, c2, c3};
+}
+
+__device__ __forceinline__ float unit_open(uint32_t w) {
+    return (static_cast<float>(w >> 8) + 0.5f) * 5.9604644775390625e-8f;  // 2^-24
+}
+
+// The four normals of quad q = b / 4 of row j.
+__device__ __forceinline__ float4 gauss4(uint64_t seed, uint32_t t, uint32_t j, uint32_t q,
+                                         uint32_t tag) {
+    const U32x4 w = philox4x32_10(q, j, t, tag, static_cast<uint32_t>(seed),
+                                  static_cast<uint32_t>(seed >> 32));
+    float s0, c0, s1, c1;
+    const float r0 = sqrtf(-2.0f * logf(unit_open(w.x)));
+    const float r1 = sqrtf(-2.0f * logf(unit_open(w.z)));
+    sincospif(2.0f * unit_open(w.y), &s0, &c0);
+    sincospif(2.0f * unit_open(w.w), &s1, &c1);
+    return make_float4(r0 * c0, r0 * s0, r1 * c1, r1 * s1);
+}
+
+// ------------------------------------------------------------------------------------------
+// Gradient element loads (fp32 or bf16, widened to fp32).
+// ------------------------------------------------------------------------------------------
+__device__ __forceinline__ float load_grad(const void* p, int64_t idx, int dtype) {
+    if (dtype == GLR_BF16) return __bfloat162float(static_cast<const __nv_bfloat16*>(p)[idx]);
+    return static_cast<const float*>(p)[idx];
+}
+
+// ------------------------------------------------------------------------------------------
+// Launchers (all asynchronous on `st`; they return cudaGetLastError()).
+// ------------------------------------------------------------------------------------------
+
+// Strided, batched fp32 GEMM: for z < batch,
+//   C_z(i, j) = alpha * sum_p A_z(i, p) B_z(p, j) + beta * C_z(i, j)
+// with A_z(i, p) = A[z*sAz + i*sAi + p*sAp], B_z(p, j) = B[z*sBz + p*sBp + j*sBj],
+// C_z(i, j) = C[z*sCz + i*sCi + j*sCj].  beta == 0 never reads C.
+struct GemmDesc {
+    int M, N, K, batch;
+    float alpha, beta;
+    const float* A; int64_t sAz, sAi, sAp;
+    const float* B; int64_t sBz, sBp, sBj;
+    float* C;       int64_t sCz, sCi, sCj;
+};
+cudaError_t gemm_f32(const GemmDesc& d, cudaStream_t st);
+
+// K1 -- compose: for every node i and oriented element (a, b) of the m' x n' working layout
+//   M_i(a, b) = G_i(a, b) + [!e_zero] (B_i(a, b) - sum_q Pprev(a, q) Rw_i(q, b))
+//   B_i(a, b) = M_i(a, b)          (kept for the deferred error E_i = B_i - P P^T B_i)
+//   Mbar(a, b) = (1/N) sum_i M_i(a, b)
+// G_i is read in its caller layout (row-major m x n; transposed view when m > n).
+struct ComposeArgs {
+    const void* G[GLR_MAX_NODES];   // node gradients (device pointers)
+    int grad_dtype;
+    int transposed;         // 1: G_i(a, b) = G_i[b * m' + a]
+    int mp, np, N, r;
+    int e_zero;             // 1: E = 0 (skip B and the correction)
+    int write_B;            // 0: warm-up steps, B is not needed
+    float* B;               // N x m' x n'
+    const float* Pprev;     // m' x r
+    const float* Rw;        // N x r x n'  (Rw_i = Pprev^T B_i)
+    float* Mbar;            // m' x n'
+};
+cudaError_t compose(const ComposeArgs& a, cudaStream_t st);
+
+// Approx-Top-r partial sums: part[j * ntiles + tb] = sum_{b in tile tb} C(j, b) v_j[b] where
+//   dense:  C = U^T Mbar                  (A(j, p) = U[p * m' + j], K = m')
+//   wy:     C = Mbar - Yt Wbar            (A(j, c) = Yt[j * k + c], K = k)
+struct LambdaArgs {
+    int mode;               // 0 dense, 1 wy
+    int mp, np, K;
+    const float* A;         // U (dense) or Yt (wy)
+    const float* Bm;        // Mbar (dense) or Wbar (wy)
+    const float* Mbar;      // wy only
+    uint64_t seed; uint32_t t;
+    float* part; int ntiles;
+};
+constexpr int kLambdaTile = 64;
+cudaError_t lambda_partials(const LambdaArgs& a, cudaStream_t st);
+
+// Reduce the partials in fixed order, apply the column signs d (k entries, may be null),
+// pick J = the r largest lambda^2 (ties -> lower index), J ascending.
+cudaError_t select_top_r(const float* part, int ntiles, int mp, int r, const float* dsign, int k,
+                         float* lam, int32_t* J, cudaStream_t st);
+
+// P(:, q) = column J[q] of U: dense U (mode 0) or U = (I - Y Yt^T) D (mode 1).
+cudaError_t build_P(int mode, int mp, int r, int k, const int32_t* J, const float* U,
+                    const float* Y, const float* Yt, const float* dsign, float* P, cudaStream_t st);
+
+// K3 -- decompress + optimizer: Ghat(a, b) = sum_q P(a, q) Rbar(q, b) (compressed) or
+// Mbar(a, b), mapped back to X's layout (transposed when m > n), then MSGD / Adam.
+struct UpdateArgs {
+    int mp, np, r, transposed, compressed, optimizer;
+    float lr, beta1, beta2, eps;
+    const float* P; const float* Rbar; const float* Mbar;
+    float* X; float* Mo; float* Vo;
+};
+cudaError_t update(const UpdateArgs& a, cudaStream_t st);
+
+// E_i = B_i - Pprev (Pprev^T B_i) given Rw_i = Pprev^T B_i  (or 0 when e_zero)
+cudaError_t materialize_error(int mp, int np, int r, int e_zero, const float* B, const float* Pprev,
+                              const float* Rw, float* E, cudaStream_t st);
+
+// ---- refresh ------------------------------------------------------------------------------
+// Cyclic two-sided Jacobi on the symmetric n x n matrix H (overwritten), one CTA:
+// eigenvalues to evals, eigenvectors (columns) to V; the sweep count to *sweeps.
+cudaError_t jacobi_eig(float* H, int n, float* V, float* evals, int* sweeps, cudaStream_t st);
+// Sort eigenpairs by descending eigenvalue, write the first ncols vectors as columns of Out
+// (rows x ncols, row-major, leading dim ldo), largest-|entry| of each column positive.
+cudaError_t sort_fix_basis(const float* evals, const float* V, int n, int ncols, float* Out,
+                           int ldo, float* evals_sorted, cudaStream_t st);
+// Make the largest-|entry| of each column of A (rows x cols, row-major) positive.
+cudaError_t fix_column_signs(float* A, int rows, int cols, cudaStream_t st);
+// In-place Cholesky of the n x n SPD matrix A (lower factor in the lower triangle); if a
+// pivot is not positive the diagonal is shifted and the factorisation restarted (*flag =
+// number of restarts).  scratch: n*n floats.
+cudaError_t cholesky(float* A, int n, float* scratch, int* flag, cudaStream_t st);
+// Q <- Q L^{-T} for the rows x n matrix Q (row-major) and lower-triangular L.
+cudaError_t trsm_right_lt(float* Q, int rows, int n, const float* L, cudaStream_t st);
+// Random Gaussian start block (rows x cols) from Philox with the power-iteration tag.
+cudaError_t random_block(float* Q, int rows, int cols, uint64_t seed, uint32_t t, cudaStream_t st);
+// Householder reconstruction (modified LU, Ballard et al. 2015) of orthonormal Q (mp x k):
+// Y (mp x k unit lower trapezoidal), T (k x k upper), s (k signs) with (I - Y T Y^T)[:, :k]
+// diag(s) = Q.  Work: scratch of k*k floats.
+cudaError_t householder_reconstruct(const float* Q, int mp, int k, float* Y, float* T, float* s,
+                                    float* scratch, cudaStream_t st);
+// U = (I - Y Yt^T) D materialised (mp x mp).
+cudaError_t materialize_wy_basis(int mp, int k, const float* Y, const float* Yt, const float* dsign,
+                                 float* U, cudaStream_t st);
+
+}  // namespace glr

@@ -1,0 +1,168 @@
+// Approx-Top-r (Algorithm 2) on the device: the bilinear forms lambda_j = u_j^T Mbar v_j with
+// v_j generated in the GEMM epilogue (never stored), the fixed-order reduction, the arg-top-r
+// of lambda-bar^2 (Eq. semi-lazy-svd-3) and the gather of P = U[:, J].
+#include "glr_internal.cuh"
+
+namespace glr {
+
+namespace {
+constexpr int LT = kLambdaTile;   // 64 rows (j) x 64 columns (b) per CTA
+constexpr int LK = 16;
+
+// C(j, b) = sum_p A(j, p) B(p, b) for a 64 x 64 tile; then for each row j the partial
+// sum over the tile's columns of C'(j, b) v_j[b], with C' = C (dense) or Mbar - C (wy).
+__global__ void __launch_bounds__(256) lambda_kernel(LambdaArgs a) {
+    __shared__ float As[LK][LT + 4];
+    __shared__ float Bs[LK][LT + 4];
+    const int j0 = blockIdx.y * LT, b0 = blockIdx.x * LT;
+    const int tid = threadIdx.x, tx = tid % 16, ty = tid / 16;
+    // A(j, p): dense U^T -> U[p * m' + j] (unit stride along j); wy Yt -> Yt[j * K + p]
+    const int64_t sAj = a.mode == 0 ? 1 : a.K;
+    const int64_t sAp = a.mode == 0 ? a.mp : 1;
+    float acc[4][4] = {};
+    for (int p0 = 0; p0 < a.K; p0 += LK) {
+        for (int e = tid; e < LT * LK; e += 256) {
+            int jj, pp;
+            if (a.mode == 0) { jj = e % LT; pp = e / LT; } else { pp = e % LK; jj = e / LK; }
+            const int gj = j0 + jj, gp = p0 + pp;
+            As[pp][jj] = (gj < a.mp && gp < a.K) ? a.A[gj * sAj + gp * sAp] : 0.f;
+        }
+        for (int e = tid; e < LT * LK; e += 256) {
+            const int bb = e % LT, pp = e / LT;
+            const int gb = b0 + bb, gp = p0 + pp;
+            Bs[pp][bb] = (gb < a.np && gp < a.K) ? a.Bm[(int64_t)gp * a.np + gb] : 0.f;
+        }
+        __syncthreads();
+#pragma unroll
+        for (int p = 0; p < LK; ++p) {
+            float x[4], y[4];
+#pragma unroll
+            for (int u = 0; u < 4; ++u) { x[u] = As[p][ty * 4 + u]; y[u] = Bs[p][tx * 4 + u]; }
+#pragma unroll
+            for (int u = 0; u < 4; ++u)
+#pragma unroll
+                for (int v = 0; v < 4; ++v) acc[u][v] = fmaf(x[u], y[v], acc[u][v]);
+        }
+        __syncthreads();
+    }
+    const int bq = b0 + tx * 4;   // first column of this thread (a multiple of 4)
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+        const int j = j0 + ty * 4 + u;
+        float s = 0.f;
+        if (j < a.mp && bq < a.np) {
+            const float4 g = gauss4(a.seed, a.t, static_cast<uint32_t>(j), static_cast<uint32_t>(bq >> 2), kTagLambdaV);
+            const float gv[4] = {g.x, g.y, g.z, g.w};
+#pragma unroll
+            for (int v = 0; v < 4; ++v) {
+                const int b = bq + v;
+                if (b < a.np) {
+                    float c = acc[u][v];
+                    if (a.mode == 1) c = a.Mbar[(int64_t)j * a.np + b] - c;
+                    s = fmaf(c, gv[v], s);
+                }
+            }
+        }
+        // fixed-order reduction over the 16 column groups (lanes with equal ty share a half-warp)
+#pragma unroll
+        for (int off = 8; off > 0; off >>= 1) s += __shfl_xor_sync(0xffffffffu, s, off);
+        if (tx == 0 && j < a.mp) a.part[(int64_t)j * a.ntiles + blockIdx.x] = s;
+    }
+}
+}  // namespace
+
+cudaError_t lambda_partials(const LambdaArgs& a, cudaStream_t st) {
+    dim3 grid(a.ntiles, (a.mp + LT - 1) / LT);
+    lambda_kernel<<<grid, 256, 0, st>>>(a);
+    return cudaGetLastError();
+}
+
+// ------------------------------------------------------------------------------------------
+// Selection: one CTA.  lambda_j = d_j * sum_t part[j][t] (fixed order); keys
+// (bits(lambda^2) << 32) | (~j) sorted descending by a bitonic network, so ties go to the
+// lower index; the first r indices are then written in ascending order.
+// ------------------------------------------------------------------------------------------
+namespace {
+__global__ void __launch_bounds__(1024) select_kernel(const float* part, int ntiles, int mp, int r,
+                                                      const float* dsign, int k, float* lam,
+                                                      int32_t* J, int npow2) {
+    extern __shared__ unsigned long long keys[];
+    const int tid = threadIdx.x;
+    for (int j = tid; j < npow2; j += blockDim.x) {
+        unsigned long long key = 0ull;
+        if (j < mp) {
+            float s = 0.f;
+            for (int t = 0; t < ntiles; ++t) s += part[(int64_t)j * ntiles + t];
+            if (dsign != nullptr && j < k) s *= dsign[j];
+            lam[j] = s;
+            const float sc = s * s;
+            key = (static_cast<unsigned long long>(__float_as_uint(sc)) << 32) |
+                  static_cast<unsigned long long>(0xFFFFFFFFu - static_cast<uint32_t>(j));
+        }
+        keys[j] = key;
+    }
+    __syncthreads();
+    for (int size = 2; size <= npow2; size <<= 1) {
+        for (int stride = size >> 1; stride > 0; stride >>= 1) {
+            for (int i = tid; i < npow2; i += blockDim.x) {
+                const int partner = i ^ stride;
+                if (partner > i) {
+                    const bool desc = (i & size) == 0;
+                    const unsigned long long x = keys[i], y = keys[partner];
+                    if ((x < y) == desc) { keys[i] = y; keys[partner] = x; }
+                }
+            }
+            __syncthreads();
+        }
+    }
+    // ascending index order of the r winners: rank among the winners
+    for (int q = tid; q < r; q += blockDim.x) {
+        const uint32_t jq = 0xFFFFFFFFu - static_cast<uint32_t>(keys[q] & 0xFFFFFFFFull);
+        int rank = 0;
+        for (int w = 0; w < r; ++w) {
+            const uint32_t jw = 0xFFFFFFFFu - static_cast<uint32_t>(keys[w] & 0xFFFFFFFFull);
+            rank += jw < jq;
+        }
+        J[rank] = static_cast<int32_t>(jq);
+    }
+}
+
+__global__ void build_P_kernel(int mode, int mp, int r, int k, const int32_t* J, const float* U,
+                               const float* Y, const float* Yt, const float* dsign, float* P) {
+    const int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+    if (e >= (int64_t)mp * r) return;
+    const int aa = static_cast<int>(e / r), q = static_cast<int>(e % r);
+    const int j = J[q];
+    if (mode == 0) { P[e] = U[(int64_t)aa * mp + j]; return; }
+    // column j of (I - Y Yt^T), times d_j for the spectral columns j < k
+    float v = (aa == j) ? 1.f : 0.f;
+    const float* ya = Y + (int64_t)aa * k;
+    const float* yj = Yt + (int64_t)j * k;
+    for (int c = 0; c < k; ++c) v = fmaf(-ya[c], yj[c], v);
+    if (j < k) v *= dsign[j];
+    P[e] = v;
+}
+}  // namespace
+
+cudaError_t select_top_r(const float* part, int ntiles, int mp, int r, const float* dsign, int k,
+                         float* lam, int32_t* J, cudaStream_t st) {
+    int npow2 = 1;
+    while (npow2 < mp) npow2 <<= 1;
+    const size_t smem = sizeof(unsigned long long) * npow2;
+    static bool attr_set = false;
+    if (!attr_set) {
+        cudaFuncSetAttribute(select_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, 200 * 1024);
+        attr_set = true;
+    }
+    select_kernel<<<1, 1024, smem, st>>>(part, ntiles, mp, r, dsign, k, lam, J, npow2);
+    return cudaGetLastError();
+}
+
+cudaError_t build_P(int mode, int mp, int r, int k, const int32_t* J, const float* U, const float* Y,
+                    const float* Yt, const float* dsign, float* P, cudaStream_t st) {
+    const int64_t total = (int64_t)mp * r;
+    build_P_kernel<<<(unsigned)((total + 255) / 256), 256, 0, st>>>(mode, mp, r, k, J, U, Y, Yt, dsign, P);
+    return cudaGetLastError();
+}
+
+}  // namespace glr

@@ -1,0 +1,73 @@
+"""Host-side checks of the C ABI that need no GPU: the library builds for sm_103a, loads, and
+exports every function declared in include/glr.h; glr_create rejects bad arguments before it
+touches the device; the ctypes structs match the C layout."""
+import ctypes
+import os
+import subprocess
+
+import pytest
+
+import __graft_entry__
+from paper_2507_08784_gb300 import _lib
+
+
+@pytest.fixture(scope="module")
+def lib():
+    __graft_entry__.build()
+    return _lib.load()
+
+
+def test_exports_every_declared_symbol(lib):
+    names = _lib.header_symbols()
+    assert len(names) >= 12
+    missing = [nm for nm in names if not hasattr(lib, nm)]
+    assert not missing, missing
+    out = subprocess.run(["nm", "-D", "--defined-only", _lib.LIB_PATH], capture_output=True, text=True).stdout
+    exported = {line.split()[-1] for line in out.splitlines() if line.strip()}
+    assert set(names) <= exported
+
+
+def test_bindings_cover_every_symbol():
+    assert set(_lib.header_symbols()) == set(_lib._SIGNATURES)
+
+
+def test_struct_layouts():
+    assert ctypes.sizeof(_lib.GlrSchedule) == 56
+    assert _lib.GlrSchedule.seed.offset == 32
+    assert ctypes.sizeof(_lib.GlrStats) == 64
+
+
+@pytest.mark.parametrize("m,n,r,N,kw,frag", [
+    (0, 5, 1, 1, {}, "matrix sizes"),
+    (5, 5, 0, 1, {}, "1 <= r"),
+    (5, 5, 6, 1, {}, "1 <= r"),
+    (5, 5, 2, 0, {}, "N"),
+    (5, 5, 2, 65, {}, "N"),
+    (5, 5, 2, 1, {"tau": 0}, "tau"),
+    (8, 20, 4, 1, {"basis_rank": 3}, "basis_rank"),
+    (2000, 3000, 4, 1, {"basis_rank": 0}, "full basis"),
+    (8, 20, 4, 1, {"power_iters": 0, "basis_rank": 5}, "power_iters"),
+])
+def test_create_rejects_bad_arguments(lib, m, n, r, N, kw, frag):
+    import paper_2507_08784_gb300 as glr
+    sched = dict(tau=5)
+    sched.update(kw)
+    s = glr.make_schedule(**sched)
+    h = ctypes.c_void_p()
+    rc = lib.glr_create(m, n, r, N, ctypes.byref(s), ctypes.byref(h))
+    assert rc == _lib.GLR_EINVAL
+    assert not h.value
+    assert frag in lib.glr_last_error(None).decode()
+
+
+def test_null_arguments(lib):
+    h = ctypes.c_void_p()
+    assert lib.glr_create(4, 4, 1, 1, None, ctypes.byref(h)) == _lib.GLR_EINVAL
+    assert lib.glr_step(None, None, None, None) == _lib.GLR_EINVAL
+    assert lib.glr_destroy(None) == _lib.GLR_OK
+    assert lib.glr_refresh(None) == _lib.GLR_EINVAL
+
+
+def test_build_is_sm103a_only():
+    from paper_2507_08784_gb300 import build
+    assert build.ARCH == ["-gencode", "arch=compute_103a,code=sm_103a"]

@@ -28,7 +28,7 @@ import numpy as np
 
 __all__ = [
     "Config", "CONFIGS", "config", "Problem", "make_problem",
-    "gradients_numpy", "round_to_dtype_numpy",
+    "gradients_numpy", "round_to_dtype_numpy", "gradients_torch",
 ]
 
 
@@ -154,3 +154,24 @@ def gradients_numpy(prob: Problem, li: int, t: int, workers: Sequence[int] | Non
         rng = np.random.default_rng([prob.seed, 2, li, t, i])
         out[slot] = S + cfg.noise * rng.standard_normal((m, n)) / math.sqrt(n)
     return round_to_dtype_numpy(out, cfg.grad_dtype)
+
+
+def gradients_torch(prob: Problem, li: int, t: int, device="cuda", workers: Sequence[int] | None = None):
+    """The same recipe generated on a torch device (for large benchmark inputs): a list of N
+    tensors (m x n) in the configuration's dtype.  Uses torch's generator, so the noise
+    differs from gradients_numpy; S is the same matrix."""
+    import torch
+    cfg = prob.cfg
+    m, n = cfg.shapes[li]
+    rho = prob.Ub[li].shape[1]
+    Ub = torch.from_numpy(prob.Ub[li] * prob.s[None, :rho]).float().to(device)
+    Vb = torch.from_numpy(prob.Vb[li]).float().to(device)
+    S = Ub @ Vb.T
+    dt = torch.float32 if cfg.grad_dtype == "f32" else torch.bfloat16
+    gen = torch.Generator(device=device)
+    out = []
+    for i in (range(cfg.N) if workers is None else workers):
+        gen.manual_seed((prob.seed * 1_000_003 + li * 10_007 + t * 101 + i) % (2 ** 63))
+        noise = torch.randn(m, n, device=device, generator=gen)
+        out.append((S + (cfg.noise / math.sqrt(n)) * noise).to(dt).contiguous())
+    return out
