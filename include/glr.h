@@ -205,6 +205,31 @@ int glr_profile_read(glr_handle* h, glr_profile* out, int32_t reset);
  * [0, m')), instead of Algorithm 2.  One-shot.                                           */
 int glr_force_selection(glr_handle* h, const int32_t* J_host);
 
+/* ---- selection without device allocation ------------------------------------------------ */
+
+/* The Approx-Top-r selection (the lambda-bar and J that glr_step computes for a full basis)
+ * for callers that cannot let a library allocate device memory: frameworks that own the GPU
+ * through their own caching allocator and forbid raw cudaMalloc from other libraries,
+ * services that reserve all memory at start-up and allow no allocation on the hot path, and
+ * code that must not risk the device synchronisation cudaMalloc/cudaFree can cause.  The
+ * paper has no counterpart: this is a deployment variant, not a step of the method.
+ *   U           device, m' x m' row-major fp32 orthogonal basis (columns u_j)
+ *   Mbar        device, m' x n' row-major fp32 node-mean gradient
+ *   seed, t     key and step of the shared random vectors v_j (same stream as glr_step)
+ *   lambda_out  device, m' fp32: lambda-bar_j = u_j^T Mbar v_j
+ *   J_out       device, r int32: the r largest lambda-bar^2 (ties to the lower index),
+ *               ascending
+ * Allocates nothing: the per-tile partial sums live in a fixed 4 MiB array inside the
+ * library (2^20 floats; every GPU that loads the library holds it until the process exits).
+ * Sizes with m' * ceil(n'/64) > 2^20 are rejected with GLR_EINVAL and a message in
+ * glr_last_error(NULL).  The first call on each device looks up the array's device address
+ * (cudaGetSymbolAddress) with that device current; make that first call before any stream
+ * capture.  Every call shares the one array and overwrites the partial sums it uses, so
+ * calls that overlap on the GPU (other streams, other threads) race: serialise them.
+ * Asynchronous on `stream`.  Errors: GLR_EINVAL, GLR_ECUDA.                              */
+int glr_select_noalloc(int32_t m_prime, int32_t n_prime, int32_t r, const float* U, const float* Mbar,
+                       uint64_t seed, int64_t t, float* lambda_out, int32_t* J_out, void* stream);
+
 #ifdef __cplusplus
 }
 #endif

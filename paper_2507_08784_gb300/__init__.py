@@ -21,7 +21,7 @@ from ._lib import (GLR_ADAM, GLR_ALG3, GLR_ALG4, GLR_BF16, GLR_F32, GLR_MSGD, GL
 __all__ = ["GlrError", "make_schedule", "glr_create", "glr_destroy", "glr_step", "glr_step_host",
            "glr_refresh", "glr_get_stats", "glr_last_error", "glr_get_error", "glr_get_selection",
            "glr_get_basis", "glr_set_basis", "glr_force_selection", "glr_profile_enable",
-           "glr_profile_read", "GreedyLore", "load"]
+           "glr_profile_read", "glr_select_noalloc", "GreedyLore", "load"]
 
 
 class GlrError(RuntimeError):
@@ -133,6 +133,14 @@ def glr_profile_read(h, reset: bool = False) -> dict:
     _check(load().glr_profile_read(h, ctypes.byref(p), 1 if reset else 0), h)
     return {name: {"ms": p.ms[i], "launches": p.launches[i], "count": p.count[i]}
             for i, name in enumerate(PHASE_NAMES)}
+
+
+def glr_select_noalloc(U: torch.Tensor, Mbar: torch.Tensor, seed: int, t: int, r: int,
+                       lambda_out: torch.Tensor, J_out: torch.Tensor, stream=None) -> None:
+    """Approx-Top-r selection into caller buffers; the library allocates nothing (see glr.h)."""
+    mp, np_ = Mbar.shape
+    _check(load().glr_select_noalloc(mp, np_, r, U.data_ptr(), Mbar.data_ptr(), seed & (2 ** 64 - 1), t,
+                                     lambda_out.data_ptr(), J_out.data_ptr(), _stream_ptr(stream)))
 
 
 class GreedyLore:

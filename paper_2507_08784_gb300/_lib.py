@@ -86,6 +86,9 @@ _SIGNATURES = {
     "glr_force_selection": (ctypes.c_int, [ctypes.c_void_p, ctypes.c_void_p]),
     "glr_profile_enable": (ctypes.c_int, [ctypes.c_void_p, ctypes.c_int32]),
     "glr_profile_read": (ctypes.c_int, [ctypes.c_void_p, ctypes.POINTER(GlrProfile), ctypes.c_int32]),
+    "glr_select_noalloc": (ctypes.c_int, [ctypes.c_int32, ctypes.c_int32, ctypes.c_int32, ctypes.c_void_p,
+                                          ctypes.c_void_p, ctypes.c_uint64, ctypes.c_int64, ctypes.c_void_p,
+                                          ctypes.c_void_p, ctypes.c_void_p]),
 }
 
 _lib = None

@@ -227,6 +227,8 @@ bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) ==
 
 }  // namespace
 
+void glr::set_global_error(const char* msg) { g_create_err = msg ? msg : ""; }
+
 extern "C" {
 
 int glr_create(int64_t m, int64_t n, int32_t r, int32_t N, const glr_schedule* s, glr_handle** out) {

@@ -159,4 +159,7 @@ cudaError_t householder_reconstruct(const float* Q, int mp, int k, float* Y, flo
 cudaError_t materialize_wy_basis(int mp, int k, const float* Y, const float* Yt, const float* dsign,
                                  float* U, cudaStream_t st);
 
+// Message reported by glr_last_error(NULL) for entry points that have no handle.
+void set_global_error(const char* msg);
+
 }  // namespace glr
