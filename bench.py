@@ -120,10 +120,9 @@ def make_handles(glr, cfg, basis_rank):
 
 
 def run_steps(hs, gsets, X, t0, K):
+    import paper_2507_08784_gb300 as glr
     for s in range(K):
-        G = gsets[(t0 + s) % len(gsets)]
-        for h, g, x in zip(hs, G, X):
-            h.step(g, x)
+        glr.glr_step_group(hs, gsets[(t0 + s) % len(gsets)], X)
 
 
 def timed(torch, fn):

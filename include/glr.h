@@ -153,6 +153,15 @@ int glr_destroy(glr_handle* h);
  * GLR_ECUDA (launch failure).                                                            */
 int glr_step(glr_handle* h, const void* const* G, float* X, void* stream);
 
+/* One step of several handles at once (typically every layer matrix of a model), with the
+ * streaming passes of all of them batched into shared kernel launches.  handles[j] gets the
+ * gradient pointer array G[j] (N_j device pointers, as in glr_step) and the weights X[j].
+ * Equivalent to calling glr_step on each handle in turn (same results); handles must be
+ * distinct and on the current device.  Failures are reported by glr_last_error of the
+ * offending handle, or glr_last_error(NULL) for malformed arrays.                        */
+int glr_step_group(glr_handle* const* handles, int32_t count, const void* const* const* G, float* const* X,
+                   void* stream);
+
 /* The same step with host gradients: G_host[i] are host pointers (pinned memory gives
  * asynchronous copies) that are copied into library-owned device staging on the stream
  * before the step.  X is the device weight matrix (updated in place); when X_host_out is

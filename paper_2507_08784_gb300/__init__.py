@@ -18,7 +18,7 @@ from . import _lib
 from ._lib import (GLR_ADAM, GLR_ALG3, GLR_ALG4, GLR_BF16, GLR_F32, GLR_MSGD, GLR_OK,  # noqa: F401
                    PHASE_NAMES, GlrProfile, GlrSchedule, GlrStats, load)
 
-__all__ = ["GlrError", "make_schedule", "glr_create", "glr_destroy", "glr_step", "glr_step_host",
+__all__ = ["GlrError", "make_schedule", "glr_create", "glr_destroy", "glr_step", "glr_step_group", "glr_step_host",
            "glr_refresh", "glr_get_stats", "glr_last_error", "glr_get_error", "glr_get_selection",
            "glr_get_basis", "glr_set_basis", "glr_force_selection", "glr_profile_enable",
            "glr_profile_read", "glr_select_noalloc", "GreedyLore", "load"]
@@ -74,6 +74,17 @@ def _ptr_array(tensors: Sequence) -> ctypes.Array:
 
 def glr_step(h, G: Sequence[torch.Tensor], X: torch.Tensor, stream=None) -> None:
     _check(load().glr_step(h, _ptr_array(G), X.data_ptr(), _stream_ptr(stream)), h)
+
+
+def glr_step_group(handles: Sequence, G: Sequence[Sequence[torch.Tensor]], X: Sequence[torch.Tensor],
+                   stream=None) -> None:
+    """One step of several handles with batched launches (see glr.h)."""
+    n = len(handles)
+    hs = (ctypes.c_void_p * n)(*[h.handle if isinstance(h, GreedyLore) else h for h in handles])
+    gp = [_ptr_array(g) for g in G]
+    garr = (ctypes.c_void_p * n)(*[ctypes.addressof(a) for a in gp])
+    xarr = (ctypes.c_void_p * n)(*[x.data_ptr() for x in X])
+    _check(load().glr_step_group(hs, n, garr, xarr, _stream_ptr(stream)))
 
 
 def glr_step_host(h, G_host: Sequence[torch.Tensor], X: torch.Tensor, X_host_out: Optional[torch.Tensor] = None,

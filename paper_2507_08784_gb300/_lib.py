@@ -73,6 +73,8 @@ _SIGNATURES = {
                                   ctypes.POINTER(GlrSchedule), ctypes.POINTER(ctypes.c_void_p)]),
     "glr_destroy": (ctypes.c_int, [ctypes.c_void_p]),
     "glr_step": (ctypes.c_int, [ctypes.c_void_p, _c_void_pp, ctypes.c_void_p, ctypes.c_void_p]),
+    "glr_step_group": (ctypes.c_int, [ctypes.c_void_p, ctypes.c_int32, ctypes.c_void_p, ctypes.c_void_p,
+                                      ctypes.c_void_p]),
     "glr_step_host": (ctypes.c_int, [ctypes.c_void_p, _c_void_pp, ctypes.c_void_p, ctypes.c_void_p,
                                      ctypes.c_void_p]),
     "glr_refresh": (ctypes.c_int, [ctypes.c_void_p]),

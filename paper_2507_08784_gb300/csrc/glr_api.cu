@@ -28,12 +28,14 @@ struct glr_handle {
     float *B = nullptr, *Mbar = nullptr, *Rw = nullptr, *Rbar = nullptr, *P = nullptr, *Pprev = nullptr;
     int32_t* J = nullptr;
     float *lam = nullptr, *lam_part = nullptr;
-    int ntiles = 0;
+    int ntiles = 0;                 // lambda tiles of the first-path kernel (64 columns)
+    int fused = 0, BN = 0, nstrips = 0;   // fused strip kernels: strip width, strips per matrix
     float *Mo = nullptr, *Vo = nullptr;
     float *U = nullptr, *Hbuf = nullptr, *Vbuf = nullptr, *evals = nullptr, *evals_sorted = nullptr;
     float *Q = nullptr, *Qn = nullptr, *Y = nullptr, *Yt = nullptr, *T = nullptr, *dsign = nullptr;
     float *Wbar = nullptr, *Z = nullptr, *Hk = nullptr, *Vk = nullptr, *gram = nullptr, *scratch = nullptr;
     int* dflags = nullptr;   // [0] Cholesky restarts, [1] Jacobi sweeps of the last refresh
+    float* gemm_ws = nullptr;   // split-K partial tiles of the refresh GEMMs
     void* Gstage = nullptr;
     // host state
     int64_t t = 0, refreshes = 0, comm = 0, state_bytes = 0, period_start = 0;
@@ -133,9 +135,13 @@ void free_all(glr_handle* h) {
     h->allocs.clear();
 }
 
+thread_local float* g_ws = nullptr;   // split-K workspace of the handle being stepped
+
 GemmDesc gd(int M, int N, int K, const float* A, int64_t sAi, int64_t sAp, const float* B, int64_t sBp,
             int64_t sBj, float* C, int64_t sCi, int64_t sCj, float alpha = 1.f, float beta = 0.f) {
     GemmDesc d{};
+    d.ws = g_ws;
+    d.ws_floats = g_ws ? kGemmWsFloats : 0;
     d.M = M; d.N = N; d.K = K; d.batch = 1; d.alpha = alpha; d.beta = beta;
     d.A = A; d.sAi = sAi; d.sAp = sAp;
     d.B = B; d.sBp = sBp; d.sBj = sBj;
@@ -163,6 +169,8 @@ int wy_from_Q(glr_handle* h, cudaStream_t st) {
 // Semi-Lazy SVD refresh (Eq. SVD-P1) from Mbar.
 int do_refresh(glr_handle* h, cudaStream_t st) {
     const int mp = h->mp, np = h->np, k = h->k;
+    g_ws = h->gemm_ws;
+    struct Reset { ~Reset() { g_ws = nullptr; } } reset_ws;
     if (h->exact) {
         // H = Mbar Mbar^T, eigenvectors = left singular vectors, sorted by descending sigma
         GLR_LAUNCH(h, 1, gemm_f32(gd(mp, mp, np, h->Mbar, np, 1, h->Mbar, 1, np, h->Hbuf, mp, 1), st));
@@ -261,6 +269,20 @@ int glr_create(int64_t m, int64_t n, int32_t r, int32_t N, const glr_schedule* s
     h->s = *s; h->gsize = s->grad_dtype == GLR_BF16 ? 2 : 4;
     h->period_start = s->compress_start;
     h->ntiles = static_cast<int>((np + kLambdaTile - 1) / kLambdaTile);
+    {
+        // The fused strip kernels keep a whole m' x BN strip (and P) in shared memory and move
+        // rows with 16-byte cp.async: they need m' <= 2048, 16-byte row pitches and room for P.
+        const int BN = mp <= 512 ? 32 : mp <= 1024 ? 16 : mp <= 2048 ? 8 : 0;
+        const int gsz = s->grad_dtype == GLR_BF16 ? 2 : 4;
+        const bool rows16 = (np % 4 == 0) && (h->transposed ? (mp * gsz) % 16 == 0 : (np * gsz) % 16 == 0);
+        const size_t lim = 227 * 1024;
+        if (BN && rows16 && stream_smem_bytes((int)mp, r, k, BN, gsz, h->transposed, exact ? 0 : 1) <= lim &&
+            update_smem_bytes((int)mp, r, BN) <= lim) {
+            h->fused = 1;
+            h->BN = BN;
+            h->nstrips = static_cast<int>((np + BN - 1) / BN);
+        }
+    }
     cudaGetDevice(&h->device);
     int rc = GLR_OK;
     const size_t MP = mp, NP = np;
@@ -273,10 +295,11 @@ int glr_create(int64_t m, int64_t n, int32_t r, int32_t N, const glr_schedule* s
     A(&h->Pprev, MP * r);
     A(&h->J, (size_t)r);
     A(&h->lam, MP);
-    A(&h->lam_part, MP * h->ntiles);
+    A(&h->lam_part, MP * std::max(h->ntiles, h->nstrips));
     A(&h->Mo, (size_t)m * n);
     if (s->optimizer == GLR_ADAM) A(&h->Vo, (size_t)m * n);
     A(&h->dflags, 4);
+    A(&h->gemm_ws, (size_t)kGemmWsFloats);
     if (exact) {
         A(&h->U, MP * MP); A(&h->Hbuf, MP * MP); A(&h->Vbuf, MP * MP);
         A(&h->evals, MP); A(&h->evals_sorted, MP);
@@ -324,71 +347,165 @@ int glr_destroy(glr_handle* h) {
     return GLR_OK;
 }
 
-int glr_step(glr_handle* h, const void* const* G, float* X, void* stream) {
-    if (!h) return GLR_EINVAL;
+}  // extern "C"
+
+namespace {
+
+struct StepPlan {
+    glr_handle* h = nullptr;
+    const void* const* G = nullptr;
+    float* X = nullptr;
+    bool warm = false, refresh = false, forced = false, lam_fused = false, compressed = false;
+};
+
+int check_step_args(glr_handle* h, const void* const* G, float* X) {
     h->err.clear();
     if (!G || !X) return fail(h, GLR_EINVAL, "null gradient array or X%s");
     if (!aligned16(X)) return fail(h, GLR_EINVAL, "X must be 16-byte aligned%s");
     for (int i = 0; i < h->N; ++i)
-        if (!G[i] || !aligned16(G[i])) return fail(h, GLR_EINVAL, "gradient %s is null or not 16-byte aligned", std::to_string(i).c_str());
-    cudaStream_t st = static_cast<cudaStream_t>(stream);
-    const int mp = h->mp, np = h->np, r = h->r, N = h->N;
-    const bool warm = h->t < h->s.compress_start;
-    h->forced_this_step = false;
-    const bool refresh = !warm && (h->force_refresh || ((h->t - h->period_start) % h->s.tau == 0));
-    if (refresh && h->force_refresh) h->period_start = h->t;
-    h->force_refresh = false;
+        if (!G[i] || !aligned16(G[i]))
+            return fail(h, GLR_EINVAL, "gradient %s is null or not 16-byte aligned", std::to_string(i).c_str());
+    return GLR_OK;
+}
 
-    // K1: Rw_i = Pprev^T B_i (deferred error), then compose M_i, B_i, Mbar
+// This step's place in the schedule of Algorithm 3: warm-up (uncompressed), refresh
+// ((t - start) mod tau == 0, Semi-Lazy SVD), or a compressed step (Approx-Top-r).
+void plan_step(StepPlan& p) {
+    glr_handle* h = p.h;
+    p.warm = h->t < h->s.compress_start;
+    p.refresh = !p.warm && (h->force_refresh || ((h->t - h->period_start) % h->s.tau == 0));
+    if (p.refresh && h->force_refresh) h->period_start = h->t;
+    h->force_refresh = false;
+    p.forced = !p.warm && !p.refresh && h->has_forceJ;
+    p.lam_fused = h->fused && !h->exact && !p.warm && !p.refresh && !p.forced;
+    p.compressed = !p.warm && !(p.refresh && h->s.refresh_mode == GLR_ALG3);
+    h->forced_this_step = p.forced;
+}
+
+// K1 with the first-path kernels: R_w,i = P_prev^T B_i, then compose.
+int compose_unfused(StepPlan& p, cudaStream_t st) {
+    glr_handle* h = p.h;
+    const int mp = h->mp, np = h->np, r = h->r, N = h->N;
     if (!h->e_zero) {
         PhaseScope ps(h, GLR_PH_PREV_PROJECT, st);
         GemmDesc d = gd(r, np, mp, h->Pprev, 1, r, h->B, np, 1, h->Rw, np, 1);
         d.batch = N; d.sAz = 0; d.sBz = (int64_t)mp * np; d.sCz = (int64_t)r * np;
         GLR_LAUNCH(h, 1, gemm_f32(d, st));
     }
-    {
-        PhaseScope ps(h, GLR_PH_COMPOSE, st);
-        ComposeArgs ca{};
-        for (int i = 0; i < N; ++i) ca.G[i] = G[i];
-        ca.grad_dtype = h->s.grad_dtype; ca.transposed = h->transposed;
-        ca.mp = mp; ca.np = np; ca.N = N; ca.r = r; ca.e_zero = h->e_zero ? 1 : 0; ca.write_B = warm ? 0 : 1;
-        ca.B = h->B; ca.Pprev = h->Pprev; ca.Rw = h->Rw; ca.Mbar = h->Mbar;
-        GLR_LAUNCH(h, 1, compose(ca, st));
-    }
+    PhaseScope ps(h, GLR_PH_COMPOSE, st);
+    ComposeArgs ca{};
+    for (int i = 0; i < N; ++i) ca.G[i] = p.G[i];
+    ca.grad_dtype = h->s.grad_dtype; ca.transposed = h->transposed;
+    ca.mp = mp; ca.np = np; ca.N = N; ca.r = r; ca.e_zero = h->e_zero ? 1 : 0; ca.write_B = p.warm ? 0 : 1;
+    ca.B = h->B; ca.Pprev = h->Pprev; ca.Rw = h->Rw; ca.Mbar = h->Mbar;
+    GLR_LAUNCH(h, 1, compose(ca, st));
+    return GLR_OK;
+}
 
-    int rc = GLR_OK;
-    if (warm) {
-        PhaseScope ps(h, GLR_PH_UPDATE, st);
-        if ((rc = uncompressed_update(h, X, st)) != GLR_OK) return rc;
-        h->comm += (int64_t)mp * np;
-        h->last_uncompressed = true;
-        h->t++;
-        return GLR_OK;
+// Work per strip CTA (rows x nodes): larger first so the grouped grid ends evenly.
+bool heavier(const StepPlan* a, const StepPlan* b) {
+    const int64_t wa = (int64_t)a->h->mp * a->h->N, wb = (int64_t)b->h->mp * b->h->N;
+    return wa != wb ? wa > wb : a->h < b->h;
+}
+
+// K1 fused and grouped: one launch per (strip width, gradient dtype) bucket and chunk.
+int compose_fused(std::vector<StepPlan*>& plans, cudaStream_t st) {
+    std::vector<StepPlan*> todo(plans);
+    std::stable_sort(todo.begin(), todo.end(), heavier);
+    while (!todo.empty()) {
+        const int BN = todo.front()->h->BN, dt = todo.front()->h->s.grad_dtype;
+        StreamGroup g{};
+        g.BN = BN; g.grad_dtype = dt;
+        size_t smem = 0;
+        std::vector<StepPlan*> rest;
+        for (StepPlan* p : todo) {
+            glr_handle* h = p->h;
+            if (h->BN != BN || h->s.grad_dtype != dt || g.nmat == kGroupMax ||
+                g.nmat + 0 >= kGroupMax || (int)(g.nmat ? g.mat[g.nmat - 1].g_off + g.mat[g.nmat - 1].N : 0) + h->N > kGroupPtrs) {
+                rest.push_back(p);
+                continue;
+            }
+            StreamMat& M = g.mat[g.nmat];
+            M.mp = h->mp; M.np = h->np; M.N = h->N; M.r = h->r; M.k = h->k;
+            M.transposed = h->transposed; M.e_zero = h->e_zero ? 1 : 0; M.write_B = p->warm ? 0 : 1;
+            M.lam = p->lam_fused ? 1 : 0;
+            M.g_off = g.nmat ? g.mat[g.nmat - 1].g_off + g.mat[g.nmat - 1].N : 0;
+            M.strip0 = g.total_strips; M.nstrips = h->nstrips;
+            M.B = h->B; M.Pprev = h->Pprev; M.Mbar = h->Mbar;
+            M.Y = h->Y; M.Yt = h->Yt; M.part = h->lam_part;
+            M.seed = h->s.seed; M.t = static_cast<uint32_t>(h->t);
+            for (int i = 0; i < h->N; ++i) g.G[M.g_off + i] = p->G[i];
+            g.total_strips += h->nstrips;
+            smem = std::max(smem, stream_smem_bytes(h->mp, h->r, h->k, BN, (int)h->gsize, h->transposed, M.lam));
+            g.nmat++;
+        }
+        glr_handle* h0 = todo.front()->h;
+        {
+            PhaseScope ps(h0, GLR_PH_COMPOSE, st);
+            GLR_LAUNCH(h0, 1, stream_group(g, smem, st));
+        }
+        todo.swap(rest);
     }
-    if (refresh) {
+    return GLR_OK;
+}
+
+// K3 fused and grouped.
+int update_fused(std::vector<StepPlan*>& plans, cudaStream_t st) {
+    std::vector<StepPlan*> todo(plans);
+    std::stable_sort(todo.begin(), todo.end(), heavier);
+    while (!todo.empty()) {
+        glr_handle* h0 = todo.front()->h;
+        const int BN = h0->BN;
+        UpdateGroup g{};
+        g.BN = BN; g.optimizer = h0->s.optimizer;
+        g.lr = h0->s.lr; g.beta1 = h0->s.beta1; g.beta2 = h0->s.beta2; g.eps = h0->s.eps;
+        size_t smem = 0;
+        std::vector<StepPlan*> rest;
+        for (StepPlan* p : todo) {
+            glr_handle* h = p->h;
+            if (h->BN != BN || h->s.optimizer != g.optimizer || h->s.lr != g.lr || h->s.beta1 != g.beta1 ||
+                h->s.beta2 != g.beta2 || h->s.eps != g.eps || g.nmat == kGroupMax) {
+                rest.push_back(p);
+                continue;
+            }
+            UpdateMat& M = g.mat[g.nmat];
+            M.mp = h->mp; M.np = h->np; M.r = h->r; M.transposed = h->transposed; M.compressed = p->compressed ? 1 : 0;
+            M.strip0 = g.total_strips; M.nstrips = h->nstrips;
+            M.P = h->P; M.Rbar = h->Rbar; M.Mbar = h->Mbar; M.X = p->X; M.Mo = h->Mo; M.Vo = h->Vo;
+            g.total_strips += h->nstrips;
+            smem = std::max(smem, update_smem_bytes(h->mp, h->r, BN));
+            g.nmat++;
+        }
+        {
+            PhaseScope ps(h0, GLR_PH_UPDATE, st);
+            GLR_LAUNCH(h0, 1, update_group(g, smem, st));
+        }
+        todo.swap(rest);
+    }
+    return GLR_OK;
+}
+
+// Between K1 and K3: refresh, or Approx-Top-r selection and P.
+int select_phase(StepPlan& p, cudaStream_t st) {
+    glr_handle* h = p.h;
+    const int mp = h->mp, np = h->np, r = h->r;
+    int rc = GLR_OK;
+    if (p.warm) return GLR_OK;
+    if (p.refresh) {
         {
             PhaseScope ps(h, GLR_PH_REFRESH, st);
             if ((rc = do_refresh(h, st)) != GLR_OK) return rc;
         }
         h->refreshes++;
         h->comm += (int64_t)mp * np;
-        if (h->s.refresh_mode == GLR_ALG3) {
-            PhaseScope ps(h, GLR_PH_UPDATE, st);
-            if ((rc = uncompressed_update(h, X, st)) != GLR_OK) return rc;
-            h->e_zero = true;
-            h->last_uncompressed = true;
-            h->has_forceJ = false;
-            h->t++;
-            return GLR_OK;
-        }
+        if (h->s.refresh_mode == GLR_ALG3) return GLR_OK;
         GLR_CK(h, cudaMemcpyAsync(h->J, h->iotaJ.data(), sizeof(int32_t) * r, cudaMemcpyHostToDevice, st));
         h->comm += (int64_t)r * np;
-    } else if (h->has_forceJ) {
+    } else if (p.forced) {
         GLR_CK(h, cudaMemcpyAsync(h->J, h->forceJ.data(), sizeof(int32_t) * r, cudaMemcpyHostToDevice, st));
         h->has_forceJ = false;
-        h->forced_this_step = true;
         h->comm += (int64_t)r * np + mp;
-    } else {
+    } else if (!p.lam_fused) {
         PhaseScope ps(h, GLR_PH_LAMBDA, st);
         LambdaArgs la{};
         la.mp = mp; la.np = np; la.seed = h->s.seed; la.t = static_cast<uint32_t>(h->t);
@@ -402,19 +519,114 @@ int glr_step(glr_handle* h, const void* const* G, float* X, void* stream) {
         }
         GLR_LAUNCH(h, 1, lambda_partials(la, st));
         h->comm += (int64_t)r * np + mp;
+    } else {
+        h->comm += (int64_t)r * np + mp;
     }
-    {
-        PhaseScope ps(h, GLR_PH_SELECT, st);
-        if (!refresh && !h->forced_this_step)
-            GLR_LAUNCH(h, 1, select_top_r(h->lam_part, h->ntiles, mp, r, h->exact ? nullptr : h->dsign, h->k, h->lam, h->J, st));
-        if ((rc = build_selection_P(h, st)) != GLR_OK) return rc;
-    }
-    if ((rc = project_and_update(h, X, st)) != GLR_OK) return rc;
-    std::swap(h->P, h->Pprev);          // Pprev now holds this step's P (deferred E_i = B_i - P P^T B_i)
-    h->e_zero = false;
-    h->last_uncompressed = false;
-    h->t++;
     return GLR_OK;
+}
+
+// arg-top-r (unless J was supplied) and P = U[:, J] for every compressed matrix, grouped.
+int select_P_grouped(std::vector<StepPlan>& plans, cudaStream_t st) {
+    SelectGroup g{};
+    glr_handle* h0 = nullptr;
+    auto flush = [&]() -> int {
+        if (g.nmat == 0) return GLR_OK;
+        PhaseScope ps(h0, GLR_PH_SELECT, st);
+        GLR_LAUNCH(h0, 1, select_group(g, st));
+        g = SelectGroup{};
+        h0 = nullptr;
+        return GLR_OK;
+    };
+    for (StepPlan& p : plans) {
+        if (!p.compressed) continue;
+        glr_handle* h = p.h;
+        if (!h0) h0 = h;
+        SelectMat& M = g.mat[g.nmat++];
+        M.part = h->lam_part; M.ntiles = p.lam_fused ? h->nstrips : h->ntiles;
+        M.mp = h->mp; M.r = h->r; M.k = h->k; M.mode = h->exact ? 0 : 1;
+        M.do_select = (!p.refresh && !p.forced) ? 1 : 0;
+        M.dsign = h->exact ? nullptr : h->dsign; M.lam = h->lam; M.J = h->J;
+        M.U = h->U; M.Y = h->Y; M.Yt = h->Yt; M.P = h->P;
+        if (g.nmat == kGroupMax) {
+            int rc = flush();
+            if (rc != GLR_OK) return rc;
+        }
+    }
+    return flush();
+}
+
+int update_unfused(StepPlan& p, cudaStream_t st) {
+    if (!p.compressed) {
+        PhaseScope ps(p.h, GLR_PH_UPDATE, st);
+        return uncompressed_update(p.h, p.X, st);
+    }
+    return project_and_update(p.h, p.X, st);
+}
+
+void finish_step(StepPlan& p) {
+    glr_handle* h = p.h;
+    if (p.warm) {
+        h->comm += (int64_t)h->mp * h->np;
+        h->last_uncompressed = true;
+    } else if (!p.compressed) {
+        h->e_zero = true;
+        h->last_uncompressed = true;
+        h->has_forceJ = false;
+    } else {
+        std::swap(h->P, h->Pprev);      // Pprev now holds this step's P (deferred E_i = B_i - P P^T B_i)
+        h->e_zero = false;
+        h->last_uncompressed = false;
+    }
+    h->t++;
+}
+
+int step_group(std::vector<StepPlan>& plans, cudaStream_t st) {
+    std::vector<StepPlan*> fused, unfused;
+    for (StepPlan& p : plans) {
+        plan_step(p);
+        (p.h->fused ? fused : unfused).push_back(&p);
+    }
+    int rc;
+    if (!fused.empty() && (rc = compose_fused(fused, st)) != GLR_OK) return rc;
+    for (StepPlan* p : unfused)
+        if ((rc = compose_unfused(*p, st)) != GLR_OK) return rc;
+    for (StepPlan& p : plans)
+        if ((rc = select_phase(p, st)) != GLR_OK) return rc;
+    if ((rc = select_P_grouped(plans, st)) != GLR_OK) return rc;
+    if (!fused.empty() && (rc = update_fused(fused, st)) != GLR_OK) return rc;
+    for (StepPlan* p : unfused)
+        if ((rc = update_unfused(*p, st)) != GLR_OK) return rc;
+    for (StepPlan& p : plans) finish_step(p);
+    return GLR_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+int glr_step(glr_handle* h, const void* const* G, float* X, void* stream) {
+    if (!h) return GLR_EINVAL;
+    int rc = check_step_args(h, G, X);
+    if (rc != GLR_OK) return rc;
+    std::vector<StepPlan> plans(1);
+    plans[0].h = h; plans[0].G = G; plans[0].X = X;
+    return step_group(plans, static_cast<cudaStream_t>(stream));
+}
+
+int glr_step_group(glr_handle* const* handles, int32_t count, const void* const* const* G, float* const* X,
+                   void* stream) {
+    if (!handles || count < 1 || !G || !X) return fail(nullptr, GLR_EINVAL, "null arrays or count < 1%s");
+    std::vector<StepPlan> plans(count);
+    for (int j = 0; j < count; ++j) {
+        glr_handle* h = handles[j];
+        if (!h) return fail(nullptr, GLR_EINVAL, "null handle in the group%s");
+        for (int l = 0; l < j; ++l)
+            if (handles[l] == h) return fail(nullptr, GLR_EINVAL, "a handle appears twice in the group%s");
+        int rc = check_step_args(h, G[j], X[j]);
+        if (rc != GLR_OK) return rc;
+        plans[j].h = h; plans[j].G = G[j]; plans[j].X = X[j];
+    }
+    return step_group(plans, static_cast<cudaStream_t>(stream));
 }
 
 int glr_step_host(glr_handle* h, const void* const* G_host, float* X, float* X_host_out, void* stream) {

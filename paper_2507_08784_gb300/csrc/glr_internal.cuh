@@ -50,6 +50,8 @@ __device__ __forceinline__ float4 gauss4(uint64_t seed, uint32_t t, uint32_t j, 
     return make_float4(r0 * c0, r0 * s0, r1 * c1, r1 * s1);
 }
 
+constexpr int kGroupMax = 32;          // matrices per grouped launch
+
 // ------------------------------------------------------------------------------------------
 // Gradient element loads (fp32 or bf16, widened to fp32).
 // ------------------------------------------------------------------------------------------
@@ -65,14 +67,18 @@ __device__ __forceinline__ float load_grad(const void* p, int64_t idx, int dtype
 // Strided, batched fp32 GEMM: for z < batch,
 //   C_z(i, j) = alpha * sum_p A_z(i, p) B_z(p, j) + beta * C_z(i, j)
 // with A_z(i, p) = A[z*sAz + i*sAi + p*sAp], B_z(p, j) = B[z*sBz + p*sBp + j*sBj],
-// C_z(i, j) = C[z*sCz + i*sCi + j*sCj].  beta == 0 never reads C.
+// C_z(i, j) = C[z*sCz + i*sCi + j*sCj].  beta == 0 never reads C.  When few output tiles
+// face a long K (the tall-skinny products of the refresh) and a workspace is given, K is split
+// across CTAs whose partial tiles are summed afterwards in fixed order (no atomics).
 struct GemmDesc {
     int M, N, K, batch;
     float alpha, beta;
     const float* A; int64_t sAz, sAi, sAp;
     const float* B; int64_t sBz, sBp, sBj;
     float* C;       int64_t sCz, sCi, sCj;
+    float* ws = nullptr; int64_t ws_floats = 0;   // split-K workspace (optional)
 };
+constexpr int64_t kGemmWsFloats = int64_t(1) << 20;
 cudaError_t gemm_f32(const GemmDesc& d, cudaStream_t st);
 
 // K1 -- compose: for every node i and oriented element (a, b) of the m' x n' working layout
@@ -94,7 +100,7 @@ struct ComposeArgs {
 };
 cudaError_t compose(const ComposeArgs& a, cudaStream_t st);
 
-// Approx-Top-r partial sums: part[j * ntiles + tb] = sum_{b in tile tb} C(j, b) v_j[b] where
+// Approx-Top-r partial sums: part[tb * m' + j] = sum_{b in tile tb} C(j, b) v_j[b] where
 //   dense:  C = U^T Mbar                  (A(j, p) = U[p * m' + j], K = m')
 //   wy:     C = Mbar - Yt Wbar            (A(j, c) = Yt[j * k + c], K = k)
 struct LambdaArgs {
@@ -113,6 +119,20 @@ cudaError_t lambda_partials(const LambdaArgs& a, cudaStream_t st);
 // pick J = the r largest lambda^2 (ties -> lower index), J ascending.
 cudaError_t select_top_r(const float* part, int ntiles, int mp, int r, const float* dsign, int k,
                          float* lam, int32_t* J, cudaStream_t st);
+
+// One CTA per matrix: lambda-bar from the partials (when do_select), J = arg-top-r, and
+// P(:, q) = column J[q] of U (dense U, mode 0, or U = (I - Y Yt^T) D, mode 1).  r <= 1024.
+struct SelectMat {
+    const float* part; int ntiles;
+    int mp, r, k, mode, do_select;
+    const float* dsign; float* lam; int32_t* J;
+    const float* U; const float* Y; const float* Yt; float* P;
+};
+struct SelectGroup {
+    int nmat;
+    SelectMat mat[kGroupMax];
+};
+cudaError_t select_group(const SelectGroup& g, cudaStream_t st);
 
 // P(:, q) = column J[q] of U: dense U (mode 0) or U = (I - Y Yt^T) D (mode 1).
 cudaError_t build_P(int mode, int mp, int r, int k, const int32_t* J, const float* U,
@@ -158,6 +178,49 @@ cudaError_t householder_reconstruct(const float* Q, int mp, int k, float* Y, flo
 // U = (I - Y Yt^T) D materialised (mp x mp).
 cudaError_t materialize_wy_basis(int mp, int k, const float* Y, const float* Yt, const float* dsign,
                                  float* U, cudaStream_t st);
+
+// ------------------------------------------------------------------------------------------
+// Fused, grouped streaming kernels (one launch for every matrix of a group).  A CTA owns a
+// strip of BN columns of one matrix's oriented m' x n' layout and all of its m' rows.
+// ------------------------------------------------------------------------------------------
+constexpr int kGroupPtrs = 512;        // node gradient pointers per grouped launch
+constexpr int kFusedThreads = 512;
+constexpr int kFusedMaxEpt = 32;       // strip elements per thread: m' * BN <= 512 * 32
+
+struct StreamMat {
+    int mp, np, N, r, k;
+    int transposed, e_zero, write_B, lam;   // lam: truncated-basis lambda partials in the epilogue
+    int g_off;                              // first gradient pointer of this matrix in StreamGroup::G
+    int strip0, nstrips;                    // CTAs [strip0, strip0 + nstrips) work on this matrix
+    float* B; const float* Pprev; float* Mbar;
+    const float* Y; const float* Yt; float* part;   // part: nstrips x m' lambda partial sums
+    uint64_t seed; uint32_t t;
+};
+struct StreamGroup {
+    int nmat, grad_dtype, total_strips, BN;
+    StreamMat mat[kGroupMax];
+    const void* G[kGroupPtrs];
+};
+// K1 fused: per strip and node, R = Pprev^T B_i (deferred error), M_i = G_i + B_i - Pprev R,
+// B_i <- M_i, Mbar; with lam = 1 also W = Y^T Mbar_strip and the lambda partial sums of
+// (Mbar - Yt W) against v_j over the strip's columns.
+cudaError_t stream_group(const StreamGroup& g, size_t smem_bytes, cudaStream_t st);
+size_t stream_smem_bytes(int mp, int r, int k, int BN, int gsize, int transposed, int lam);
+
+struct UpdateMat {
+    int mp, np, r, transposed, compressed;
+    int strip0, nstrips;
+    const float* P; float* Rbar; const float* Mbar;
+    float* X; float* Mo; float* Vo;
+};
+struct UpdateGroup {
+    int nmat, total_strips, BN, optimizer;
+    float lr, beta1, beta2, eps;
+    UpdateMat mat[kGroupMax];
+};
+// K3 fused: Rbar_strip = P^T Mbar_strip, Ghat = P Rbar (or Mbar), MSGD / Adam on X.
+cudaError_t update_group(const UpdateGroup& g, size_t smem_bytes, cudaStream_t st);
+size_t update_smem_bytes(int mp, int r, int BN);
 
 // Message reported by glr_last_error(NULL) for entry points that have no handle.
 void set_global_error(const char* msg);

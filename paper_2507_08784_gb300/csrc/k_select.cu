@@ -66,7 +66,7 @@ __global__ void __launch_bounds__(256) lambda_kernel(LambdaArgs a) {
         // fixed-order reduction over the 16 column groups (lanes with equal ty share a half-warp)
 #pragma unroll
         for (int off = 8; off > 0; off >>= 1) s += __shfl_xor_sync(0xffffffffu, s, off);
-        if (tx == 0 && j < a.mp) a.part[(int64_t)j * a.ntiles + blockIdx.x] = s;
+        if (tx == 0 && j < a.mp) a.part[(int64_t)blockIdx.x * a.mp + j] = s;
     }
 }
 }  // namespace
@@ -92,7 +92,7 @@ __global__ void __launch_bounds__(1024) select_kernel(const float* part, int nti
         unsigned long long key = 0ull;
         if (j < mp) {
             float s = 0.f;
-            for (int t = 0; t < ntiles; ++t) s += part[(int64_t)j * ntiles + t];
+            for (int t = 0; t < ntiles; ++t) s += part[(int64_t)t * mp + j];   // coalesced over j
             if (dsign != nullptr && j < k) s *= dsign[j];
             lam[j] = s;
             const float sc = s * s;
@@ -143,6 +143,91 @@ __global__ void build_P_kernel(int mode, int mp, int r, int k, const int32_t* J,
     P[e] = v;
 }
 }  // namespace
+
+// ------------------------------------------------------------------------------------------
+// Grouped selection: one CTA per matrix reduces its partials, runs the arg-top-r (unless J
+// was supplied) and builds P = U[:, J] for its matrix.
+// ------------------------------------------------------------------------------------------
+namespace {
+__global__ void __launch_bounds__(1024) select_group_kernel(const __grid_constant__ SelectGroup g) {
+    extern __shared__ unsigned long long keys[];
+    const SelectMat& M = g.mat[blockIdx.x];
+    const int tid = threadIdx.x, mp = M.mp, r = M.r;
+    __shared__ int32_t Js[1024];
+    if (M.do_select) {
+        int npow2 = 1;
+        while (npow2 < mp) npow2 <<= 1;
+        for (int j = tid; j < npow2; j += blockDim.x) {
+            unsigned long long key = 0ull;
+            if (j < mp) {
+                float s = 0.f;
+                for (int t = 0; t < M.ntiles; ++t) s += M.part[(int64_t)t * mp + j];
+                if (M.dsign != nullptr && j < M.k) s *= M.dsign[j];
+                M.lam[j] = s;
+                key = (static_cast<unsigned long long>(__float_as_uint(s * s)) << 32) |
+                      static_cast<unsigned long long>(0xFFFFFFFFu - static_cast<uint32_t>(j));
+            }
+            keys[j] = key;
+        }
+        __syncthreads();
+        for (int size = 2; size <= npow2; size <<= 1) {
+            for (int stride = size >> 1; stride > 0; stride >>= 1) {
+                for (int i = tid; i < npow2; i += blockDim.x) {
+                    const int partner = i ^ stride;
+                    if (partner > i) {
+                        const bool desc = (i & size) == 0;
+                        const unsigned long long x = keys[i], y = keys[partner];
+                        if ((x < y) == desc) { keys[i] = y; keys[partner] = x; }
+                    }
+                }
+                __syncthreads();
+            }
+        }
+        for (int q = tid; q < r; q += blockDim.x) {
+            const uint32_t jq = 0xFFFFFFFFu - static_cast<uint32_t>(keys[q] & 0xFFFFFFFFull);
+            int rank = 0;
+            for (int w = 0; w < r; ++w)
+                rank += (0xFFFFFFFFu - static_cast<uint32_t>(keys[w] & 0xFFFFFFFFull)) < jq;
+            M.J[rank] = static_cast<int32_t>(jq);
+            Js[rank] = static_cast<int32_t>(jq);
+        }
+    } else {
+        for (int q = tid; q < r; q += blockDim.x) Js[q] = M.J[q];
+    }
+    __syncthreads();
+    const int k = M.k;
+    for (int e = tid; e < mp * r; e += blockDim.x) {
+        const int aa = e / r, q = e % r;
+        const int j = Js[q];
+        float v;
+        if (M.mode == 0) {
+            v = M.U[(int64_t)aa * mp + j];
+        } else {
+            v = (aa == j) ? 1.f : 0.f;
+            const float* ya = M.Y + (int64_t)aa * k;
+            const float* yj = M.Yt + (int64_t)j * k;
+            for (int c = 0; c < k; ++c) v = fmaf(-ya[c], yj[c], v);
+            if (j < k) v *= M.dsign[j];
+        }
+        M.P[e] = v;
+    }
+}
+}  // namespace
+
+cudaError_t select_group(const SelectGroup& g, cudaStream_t st) {
+    if (g.nmat <= 0) return cudaSuccess;
+    int maxmp = 1;
+    for (int i = 0; i < g.nmat; ++i) maxmp = g.mat[i].mp > maxmp ? g.mat[i].mp : maxmp;
+    int npow2 = 1;
+    while (npow2 < maxmp) npow2 <<= 1;
+    static bool attr_set = false;
+    if (!attr_set) {
+        cudaFuncSetAttribute(select_group_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, 200 * 1024);
+        attr_set = true;
+    }
+    select_group_kernel<<<g.nmat, 1024, sizeof(unsigned long long) * npow2, st>>>(g);
+    return cudaGetLastError();
+}
 
 cudaError_t select_top_r(const float* part, int ntiles, int mp, int r, const float* dsign, int k,
                          float* lam, int32_t* J, cudaStream_t st) {

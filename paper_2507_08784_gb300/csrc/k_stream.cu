@@ -13,10 +13,11 @@ namespace glr {
 namespace {
 constexpr int GB_M = 64, GB_N = 64, GB_K = 16;
 
-__global__ void __launch_bounds__(256) gemm_f32_kernel(GemmDesc d) {
+__global__ void __launch_bounds__(256) gemm_f32_kernel(GemmDesc d, int kchunk) {
     __shared__ float As[GB_K][GB_M + 4];
     __shared__ float Bs[GB_K][GB_N + 4];
-    const int z = blockIdx.z;
+    const bool split = kchunk > 0;                  // blockIdx.z = K slice (batch == 1)
+    const int z = split ? 0 : blockIdx.z;
     const float* A = d.A + z * d.sAz;
     const float* B = d.B + z * d.sBz;
     float* C = d.C + z * d.sCz;
@@ -25,18 +26,20 @@ __global__ void __launch_bounds__(256) gemm_f32_kernel(GemmDesc d) {
     float acc[4][4] = {};
     const bool a_i_unit = d.sAi == 1;
     const bool b_j_unit = d.sBj == 1;
-    for (int p0 = 0; p0 < d.K; p0 += GB_K) {
+    const int kbeg = split ? blockIdx.z * kchunk : 0;
+    const int kend = split ? min(d.K, kbeg + kchunk) : d.K;
+    for (int p0 = kbeg; p0 < kend; p0 += GB_K) {
         for (int e = tid; e < GB_M * GB_K; e += 256) {
             int ii, pp;
             if (a_i_unit) { ii = e % GB_M; pp = e / GB_M; } else { pp = e % GB_K; ii = e / GB_K; }
             const int gi = i0 + ii, gp = p0 + pp;
-            As[pp][ii] = (gi < d.M && gp < d.K) ? A[gi * d.sAi + gp * d.sAp] : 0.f;
+            As[pp][ii] = (gi < d.M && gp < kend) ? A[gi * d.sAi + gp * d.sAp] : 0.f;
         }
         for (int e = tid; e < GB_N * GB_K; e += 256) {
             int jj, pp;
             if (b_j_unit) { jj = e % GB_N; pp = e / GB_N; } else { pp = e % GB_K; jj = e / GB_K; }
             const int gj = j0 + jj, gp = p0 + pp;
-            Bs[pp][jj] = (gj < d.N && gp < d.K) ? B[gp * d.sBp + gj * d.sBj] : 0.f;
+            Bs[pp][jj] = (gj < d.N && gp < kend) ? B[gp * d.sBp + gj * d.sBj] : 0.f;
         }
         __syncthreads();
 #pragma unroll
@@ -59,18 +62,53 @@ __global__ void __launch_bounds__(256) gemm_f32_kernel(GemmDesc d) {
         for (int v = 0; v < 4; ++v) {
             const int gj = j0 + tx * 4 + v;
             if (gj >= d.N) continue;
+            if (split) {
+                d.ws[((int64_t)blockIdx.z * d.M + gi) * d.N + gj] = acc[u][v];
+                continue;
+            }
             float* c = C + gi * d.sCi + gj * d.sCj;
             const float val = d.alpha * acc[u][v];
             *c = d.beta == 0.f ? val : fmaf(d.beta, *c, val);
         }
     }
 }
+
+// C = alpha * sum_z ws[z] + beta * C, slices added in order.
+__global__ void gemm_splitk_reduce(GemmDesc d, int splits) {
+    const int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+    if (e >= (int64_t)d.M * d.N) return;
+    const int i = static_cast<int>(e / d.N), j = static_cast<int>(e % d.N);
+    float acc = 0.f;
+    for (int zz = 0; zz < splits; ++zz) acc += d.ws[(int64_t)zz * d.M * d.N + e];
+    float* c = d.C + i * d.sCi + j * d.sCj;
+    const float val = d.alpha * acc;
+    *c = d.beta == 0.f ? val : fmaf(d.beta, *c, val);
+}
 }  // namespace
 
 cudaError_t gemm_f32(const GemmDesc& d, cudaStream_t st) {
     if (d.M <= 0 || d.N <= 0 || d.batch <= 0) return cudaSuccess;
+    const int tiles = ((d.N + GB_N - 1) / GB_N) * ((d.M + GB_M - 1) / GB_M);
+    int splits = 1;
+    if (d.batch == 1 && d.ws && tiles < 148 && d.K >= 512) {
+        splits = d.K / 256;
+        splits = splits < 296 / tiles ? splits : 296 / tiles;
+        const int64_t fit = d.ws_floats / ((int64_t)d.M * d.N);
+        splits = (int64_t)splits < fit ? splits : (int)fit;
+    }
+    if (splits > 1) {
+        const int kchunk = ((d.K + splits - 1) / splits + GB_K - 1) / GB_K * GB_K;
+        splits = (d.K + kchunk - 1) / kchunk;
+        dim3 grid((d.N + GB_N - 1) / GB_N, (d.M + GB_M - 1) / GB_M, splits);
+        gemm_f32_kernel<<<grid, 256, 0, st>>>(d, kchunk);
+        cudaError_t e = cudaGetLastError();
+        if (e != cudaSuccess) return e;
+        const int64_t total = (int64_t)d.M * d.N;
+        gemm_splitk_reduce<<<(unsigned)((total + 255) / 256), 256, 0, st>>>(d, splits);
+        return cudaGetLastError();
+    }
     dim3 grid((d.N + GB_N - 1) / GB_N, (d.M + GB_M - 1) / GB_M, d.batch);
-    gemm_f32_kernel<<<grid, 256, 0, st>>>(d);
+    gemm_f32_kernel<<<grid, 256, 0, st>>>(d, 0);
     return cudaGetLastError();
 }
 

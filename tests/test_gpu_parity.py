@@ -197,3 +197,34 @@ def test_step_host_matches_device_step():
         assert torch.equal(Xa.cpu(), Xh)
     a.close()
     b.close()
+
+
+@pytest.mark.parametrize("basis_rank", [0, 16])
+def test_step_group_equals_single_steps(basis_rank):
+    """glr_step_group batches the streaming kernels of every matrix into shared launches; the
+    results must be bit-identical to stepping each handle alone."""
+    import torch
+    import paper_2507_08784_gb300 as glr
+    cfg = W.config("cfg2_resnet")
+    prob = W.make_problem(cfg)
+    shapes = list(cfg.shapes) + [(130, 96)]          # plus a transposed matrix
+    kw = dict(tau=3, optimizer="msgd", lr=cfg.lr, beta1=cfg.beta1, basis_rank=basis_rank)
+    solo = [glr.GreedyLore(m, n, cfg.r, cfg.N, seed=50 + j, **kw) for j, (m, n) in enumerate(shapes)]
+    grp = [glr.GreedyLore(m, n, cfg.r, cfg.N, seed=50 + j, **kw) for j, (m, n) in enumerate(shapes)]
+    Xs = [torch.zeros(m, n, device="cuda") for m, n in shapes]
+    Xg = [torch.zeros(m, n, device="cuda") for m, n in shapes]
+    gen = torch.Generator(device="cuda").manual_seed(7)
+    for t in range(5):
+        G = [[torch.randn(m, n, device="cuda", generator=gen) for _ in range(cfg.N)] for m, n in shapes]
+        for h, g, x in zip(solo, G, Xs):
+            h.step(g, x)
+        glr.glr_step_group(grp, G, Xg)
+        torch.cuda.synchronize()
+        for j in range(len(shapes)):
+            assert torch.equal(Xs[j], Xg[j]), (t, j)
+            Ja, *_ = solo[j].selection()
+            Jb, *_ = grp[j].selection()
+            assert np.array_equal(Ja, Jb)
+            assert torch.equal(solo[j].error(0), grp[j].error(0))
+    for h in solo + grp:
+        h.close()
