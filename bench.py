@@ -137,6 +137,21 @@ def timed(torch, fn):
     return a.elapsed_time(b)
 
 
+def timed_steps(torch, hs, gsets, X, t0, K):
+    """K steps with a CUDA event after each one (events on the launching stream); returns the
+    total and the per-step milliseconds."""
+    st = torch.cuda.current_stream()
+    evs = [torch.cuda.Event(enable_timing=True) for _ in range(K + 1)]
+    torch.cuda.synchronize()
+    evs[0].record(st)
+    for s in range(K):
+        run_steps(hs, gsets, X, t0 + s, 1)
+        evs[s + 1].record(st)
+    torch.cuda.synchronize()
+    per = [evs[s].elapsed_time(evs[s + 1]) for s in range(K)]
+    return evs[0].elapsed_time(evs[K]), per
+
+
 def bench_mode(torch, glr, cfg, prob, basis_rank, K, Wm, dist_ctx, gsets):
     """Time K steps (after Wm warm-up steps) for one basis mode; returns a dict."""
     hs = make_handles(glr, cfg, basis_rank)
@@ -146,8 +161,13 @@ def bench_mode(torch, glr, cfg, prob, basis_rank, K, Wm, dist_ctx, gsets):
     l0 = sum(h.stats()["launches"] for h in hs)
     t_first = Wm
     dist_ctx.barrier()
-    ms = timed(torch, lambda: run_steps(hs, gsets, X, t_first, K))
+    ms, per = timed_steps(torch, hs, gsets, X, t_first, K)
     ms = dist_ctx.max(ms)
+    is_ref = [(t_first + s) % cfg.tau == 0 for s in range(K)]
+    nonref = [p for p, f in zip(per, is_ref) if not f]
+    ref = [p for p, f in zip(per, is_ref) if f]
+    nonref_ms = statistics.median(nonref) if nonref else None
+    refresh_step_ms = statistics.mean(ref) if ref else None
     launches = sum(h.stats()["launches"] for h in hs) - l0
     refreshes = sum(1 for t in range(t_first, t_first + K) if t % cfg.tau == 0)
     # second pass with per-phase CUDA events (same schedule continued) for the kernel breakdown
@@ -170,7 +190,8 @@ def bench_mode(torch, glr, cfg, prob, basis_rank, K, Wm, dist_ctx, gsets):
     for h in hs:
         h.close()
     return {"ms": ms, "launches": launches, "refreshes": refreshes, "ms_prof": ms_prof,
-            "phases": phases, "compose_bytes": compose_bytes, "refresh_in_prof": refresh_in_prof}
+            "phases": phases, "compose_bytes": compose_bytes, "refresh_in_prof": refresh_in_prof,
+            "nonrefresh_step_ms": nonref_ms, "refresh_step_ms": refresh_step_ms}
 
 
 def bench_e2e(torch, glr, cfg, K, Wm, dist_ctx):
@@ -332,8 +353,8 @@ def main():
     dominant = max(ph, key=lambda k: ph[k]["ms"])
     compose = ph["compose"]
     compose_gbs = main_run["compose_bytes"] / (compose["ms"] / 1e3) / 1e9 if compose["ms"] else None
-    refresh_ms = ph["refresh"]["ms"] / max(main_run["refresh_in_prof"], 1)
-    nonrefresh = main_run["ms_prof"] - ph["refresh"]["ms"]
+    nonrefresh_ms = main_run["nonrefresh_step_ms"]
+    refresh_extra_ms = (main_run["refresh_step_ms"] - nonrefresh_ms) if main_run["refresh_step_ms"] else None
     step_bytes = algorithmic_bytes(cfg, False)
     traffic = None
     tr_path = os.path.join(ROOT, "profiles", "compose_cfg2_traffic.json")
@@ -356,14 +377,19 @@ def main():
                      "algorithmic_bytes_per_launch_avg": compose_launch_bytes,
                      "dominant_phase": dominant},
         "step_roofline": {"algorithmic_bytes_per_step": step_bytes,
-                          "achieved_gbs_nonrefresh": step_bytes / ((nonrefresh / K) / 1e3) / 1e9,
-                          "frac_nonrefresh": step_bytes / ((nonrefresh / K) / 1e3) / 1e9 / hbm_peak},
-        "refresh_ms_all_matrices": refresh_ms,
+                          "nonrefresh_step_ms_median": nonrefresh_ms,
+                          "achieved_gbs_nonrefresh": step_bytes / (nonrefresh_ms / 1e3) / 1e9,
+                          "frac_nonrefresh": step_bytes / (nonrefresh_ms / 1e3) / 1e9 / hbm_peak,
+                          "grad_elems_per_s_nonrefresh": elems / (nonrefresh_ms / 1e3)},
+        "refresh_ms_all_matrices": refresh_extra_ms,
+        "refresh_ms_per_layer": refresh_extra_ms / len(cfg.shapes) if refresh_extra_ms else None,
         "phases_ms_per_step": {k: v["ms"] / K for k, v in ph.items()},
         "phase_launches": {k: v["launches"] for k, v in ph.items()},
         "paper_exact_basis": {"value": ctx.world * elems * K / (exact_run["ms"] / 1e3),
                               "ms_per_step": exact_run["ms"] / K,
-                              "refresh_ms_all_matrices": exact_run["phases"]["refresh"]["ms"] / max(exact_run["refresh_in_prof"], 1),
+                              "nonrefresh_step_ms_median": exact_run["nonrefresh_step_ms"],
+                              "refresh_ms_all_matrices": (exact_run["refresh_step_ms"] - exact_run["nonrefresh_step_ms"])
+                              if exact_run["refresh_step_ms"] else None,
                               "phases_ms_per_step": {k: v["ms"] / K for k, v in exact_run["phases"].items()}},
         "e2e": {"value": ctx.world * elems * args.e2e_steps / (e2e["ms"] / 1e3), "unit": UNIT,
                 "h2d_bytes_per_step": e2e["h2d"], "d2h_bytes_per_step": e2e["d2h"]},

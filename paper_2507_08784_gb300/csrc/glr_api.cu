@@ -30,12 +30,16 @@ struct glr_handle {
     float *lam = nullptr, *lam_part = nullptr;
     int ntiles = 0;                 // lambda tiles of the first-path kernel (64 columns)
     int fused = 0, BN = 0, nstrips = 0;   // fused strip kernels: strip width, strips per matrix
+    int mma = 0;                          // compose on the tensor cores (k_mma.cu)
     float *Mo = nullptr, *Vo = nullptr;
     float *U = nullptr, *Hbuf = nullptr, *Vbuf = nullptr, *evals = nullptr, *evals_sorted = nullptr;
     float *Q = nullptr, *Qn = nullptr, *Y = nullptr, *Yt = nullptr, *T = nullptr, *dsign = nullptr;
     float *Wbar = nullptr, *Z = nullptr, *Hk = nullptr, *Vk = nullptr, *gram = nullptr, *scratch = nullptr;
+    float *YT = nullptr, *YtT = nullptr;   // k x transposed_pitch(m') copies of Y and Yt for the fused kernel
     int* dflags = nullptr;   // [0] Cholesky restarts, [1] Jacobi sweeps of the last refresh
     float* gemm_ws = nullptr;   // split-K partial tiles of the refresh GEMMs
+    cudaStream_t rstream = nullptr;            // side stream of this handle's refresh
+    cudaEvent_t rfork = nullptr, rdone = nullptr;
     void* Gstage = nullptr;
     // host state
     int64_t t = 0, refreshes = 0, comm = 0, state_bytes = 0, period_start = 0;
@@ -163,6 +167,9 @@ int wy_from_Q(glr_handle* h, cudaStream_t st) {
     GLR_LAUNCH(h, 2, householder_reconstruct(h->Q, mp, k, h->Y, h->T, h->dsign, h->scratch, st));
     // Yt = Y T^T
     GLR_LAUNCH(h, 1, gemm_f32(gd(mp, k, k, h->Y, k, 1, h->T, 1, k, h->Yt, k, 1), st));
+    // transposed copies (k x tp, zero-padded) for the fused compose kernel's lambda epilogue
+    GLR_LAUNCH(h, 1, transpose_pad(h->YT, transposed_pitch(mp), h->Y, mp, k, st));
+    GLR_LAUNCH(h, 1, transpose_pad(h->YtT, transposed_pitch(mp), h->Yt, mp, k, st));
     return GLR_OK;
 }
 
@@ -182,14 +189,14 @@ int do_refresh(glr_handle* h, cudaStream_t st) {
         GLR_LAUNCH(h, 1, random_block(h->Q, mp, k, h->s.seed, static_cast<uint32_t>(h->t), st));
     int rc;
     for (int it = 0; it < h->s.power_iters; ++it) {
-        // Z = Mbar^T Q  (n' x k), orthonormalised;  Q = Mbar Z  (m' x k), orthonormalised
+        // Z = Mbar^T Q (n' x k) and Q = Mbar Z (m' x k), each re-orthonormalised by CholeskyQR
+        // (one pass keeps the block well conditioned; the span is what the iteration needs)
         GLR_LAUNCH(h, 1, gemm_f32(gd(np, k, mp, h->Mbar, 1, np, h->Q, k, 1, h->Z, k, 1), st));
-        if ((rc = cholqr(h, h->Z, np, st)) != GLR_OK) return rc;
         if ((rc = cholqr(h, h->Z, np, st)) != GLR_OK) return rc;
         GLR_LAUNCH(h, 1, gemm_f32(gd(mp, k, np, h->Mbar, np, 1, h->Z, k, 1, h->Q, k, 1), st));
         if ((rc = cholqr(h, h->Q, mp, st)) != GLR_OK) return rc;
-        if ((rc = cholqr(h, h->Q, mp, st)) != GLR_OK) return rc;
     }
+    if ((rc = cholqr(h, h->Q, mp, st)) != GLR_OK) return rc;   // CholeskyQR2: orthonormal to rounding
     // Rayleigh-Ritz: Z = Mbar^T Q, H = Z^T Z = Q^T Mbar Mbar^T Q, H = W diag W^T, Q <- Q W
     GLR_LAUNCH(h, 1, gemm_f32(gd(np, k, mp, h->Mbar, 1, np, h->Q, k, 1, h->Z, k, 1), st));
     GLR_LAUNCH(h, 1, gemm_f32(gd(k, k, np, h->Z, 1, k, h->Z, k, 1, h->Hk, k, 1), st));
@@ -271,16 +278,26 @@ int glr_create(int64_t m, int64_t n, int32_t r, int32_t N, const glr_schedule* s
     h->ntiles = static_cast<int>((np + kLambdaTile - 1) / kLambdaTile);
     {
         // The fused strip kernels keep a whole m' x BN strip (and P) in shared memory and move
-        // rows with 16-byte cp.async: they need m' <= 2048, 16-byte row pitches and room for P.
-        const int BN = mp <= 512 ? 32 : mp <= 1024 ? 16 : mp <= 2048 ? 8 : 0;
+        // rows in 16-byte vectors: they need m' <= 2048, rows of a multiple of 4 elements and
+        // room for P.
+        const int BN = mp <= 512 ? 32 : mp <= 1024 ? 16 : mp <= 2048 ? 8 : mp <= 4096 ? 4 : 0;
         const int gsz = s->grad_dtype == GLR_BF16 ? 2 : 4;
-        const bool rows16 = (np % 4 == 0) && (h->transposed ? (mp * gsz) % 16 == 0 : (np * gsz) % 16 == 0);
+        const bool rows16 = (np % 4 == 0) && (!h->transposed || mp % 4 == 0);
         const size_t lim = 227 * 1024;
-        if (BN && rows16 && stream_smem_bytes((int)mp, r, k, BN, gsz, h->transposed, exact ? 0 : 1) <= lim &&
+        const bool fits_threads = BN && (int64_t)r * BN / 4 <= kUpdateThreads &&
+                                  (int64_t)std::max(r, exact ? 0 : k) * BN / 4 <= kFusedThreads;
+        if (BN && rows16 && fits_threads &&
+            stream_smem_bytes((int)mp, r, k, BN, gsz, h->transposed, exact ? 0 : 1) <= lim &&
             update_smem_bytes((int)mp, r, BN) <= lim) {
             h->fused = 1;
             h->BN = BN;
             h->nstrips = static_cast<int>((np + BN - 1) / BN);
+            if (mma_stream_eligible((int)mp, (int)np, r, k, exact ? 0 : 1, h->transposed, gsz) &&
+                (int64_t)r * kMmaStrip / 4 <= kUpdateThreads && update_smem_bytes((int)mp, r, kMmaStrip) <= lim) {
+                h->mma = 1;
+                h->BN = kMmaStrip;
+                h->nstrips = static_cast<int>((np + kMmaStrip - 1) / kMmaStrip);
+            }
         }
     }
     cudaGetDevice(&h->device);
@@ -309,6 +326,8 @@ int glr_create(int64_t m, int64_t n, int32_t r, int32_t N, const glr_schedule* s
         A(&h->T, K * K); A(&h->dsign, K); A(&h->Wbar, K * NP); A(&h->Z, NP * K);
         A(&h->Hk, K * K); A(&h->Vk, K * K); A(&h->gram, K * K); A(&h->scratch, K * K);
         A(&h->evals, K); A(&h->evals_sorted, K);
+        A(&h->YT, K * transposed_pitch(static_cast<int>(mp)));
+        A(&h->YtT, K * transposed_pitch(static_cast<int>(mp)));
     }
     if (rc != GLR_OK) {
         g_create_err = h->err;
@@ -331,6 +350,14 @@ int glr_create(int64_t m, int64_t n, int32_t r, int32_t N, const glr_schedule* s
         delete h;
         return GLR_ECUDA;
     }
+    if (cudaStreamCreateWithFlags(&h->rstream, cudaStreamNonBlocking) != cudaSuccess ||
+        cudaEventCreateWithFlags(&h->rfork, cudaEventDisableTiming) != cudaSuccess ||
+        cudaEventCreateWithFlags(&h->rdone, cudaEventDisableTiming) != cudaSuccess) {
+        g_create_err = "could not create the refresh stream";
+        free_all(h);
+        delete h;
+        return GLR_ECUDA;
+    }
     h->iotaJ.resize(r);
     for (int q = 0; q < r; ++q) h->iotaJ[q] = q;
     *out = h;
@@ -342,6 +369,9 @@ int glr_destroy(glr_handle* h) {
     cudaDeviceSynchronize();
     for (auto& rec : h->recs) { cudaEventDestroy(rec.a); cudaEventDestroy(rec.b); }
     for (cudaEvent_t e : h->free_events) cudaEventDestroy(e);
+    if (h->rstream) cudaStreamDestroy(h->rstream);
+    if (h->rfork) cudaEventDestroy(h->rfork);
+    if (h->rdone) cudaEventDestroy(h->rdone);
     free_all(h);
     delete h;
     return GLR_OK;
@@ -413,14 +443,14 @@ int compose_fused(std::vector<StepPlan*>& plans, cudaStream_t st) {
     std::vector<StepPlan*> todo(plans);
     std::stable_sort(todo.begin(), todo.end(), heavier);
     while (!todo.empty()) {
-        const int BN = todo.front()->h->BN, dt = todo.front()->h->s.grad_dtype;
+        const int BN = todo.front()->h->BN, dt = todo.front()->h->s.grad_dtype, mma = todo.front()->h->mma;
         StreamGroup g{};
         g.BN = BN; g.grad_dtype = dt;
         size_t smem = 0;
         std::vector<StepPlan*> rest;
         for (StepPlan* p : todo) {
             glr_handle* h = p->h;
-            if (h->BN != BN || h->s.grad_dtype != dt || g.nmat == kGroupMax ||
+            if (h->BN != BN || h->s.grad_dtype != dt || h->mma != mma || g.nmat == kGroupMax ||
                 g.nmat + 0 >= kGroupMax || (int)(g.nmat ? g.mat[g.nmat - 1].g_off + g.mat[g.nmat - 1].N : 0) + h->N > kGroupPtrs) {
                 rest.push_back(p);
                 continue;
@@ -432,17 +462,18 @@ int compose_fused(std::vector<StepPlan*>& plans, cudaStream_t st) {
             M.g_off = g.nmat ? g.mat[g.nmat - 1].g_off + g.mat[g.nmat - 1].N : 0;
             M.strip0 = g.total_strips; M.nstrips = h->nstrips;
             M.B = h->B; M.Pprev = h->Pprev; M.Mbar = h->Mbar;
-            M.Y = h->Y; M.Yt = h->Yt; M.part = h->lam_part;
+            M.YT = h->YT; M.YtT = h->YtT; M.part = h->lam_part;
             M.seed = h->s.seed; M.t = static_cast<uint32_t>(h->t);
             for (int i = 0; i < h->N; ++i) g.G[M.g_off + i] = p->G[i];
             g.total_strips += h->nstrips;
-            smem = std::max(smem, stream_smem_bytes(h->mp, h->r, h->k, BN, (int)h->gsize, h->transposed, M.lam));
+            smem = std::max(smem, mma ? mma_stream_smem_bytes(h->mp, h->r, h->k, h->exact ? 0 : 1, (int)h->gsize, h->transposed)
+                                      : stream_smem_bytes(h->mp, h->r, h->k, BN, (int)h->gsize, h->transposed, M.lam));
             g.nmat++;
         }
         glr_handle* h0 = todo.front()->h;
         {
             PhaseScope ps(h0, GLR_PH_COMPOSE, st);
-            GLR_LAUNCH(h0, 1, stream_group(g, smem, st));
+            GLR_LAUNCH(h0, 1, mma ? stream_group_mma(g, smem, st) : stream_group(g, smem, st));
         }
         todo.swap(rest);
     }
@@ -492,10 +523,6 @@ int select_phase(StepPlan& p, cudaStream_t st) {
     int rc = GLR_OK;
     if (p.warm) return GLR_OK;
     if (p.refresh) {
-        {
-            PhaseScope ps(h, GLR_PH_REFRESH, st);
-            if ((rc = do_refresh(h, st)) != GLR_OK) return rc;
-        }
         h->refreshes++;
         h->comm += (int64_t)mp * np;
         if (h->s.refresh_mode == GLR_ALG3) return GLR_OK;
@@ -532,7 +559,7 @@ int select_P_grouped(std::vector<StepPlan>& plans, cudaStream_t st) {
     auto flush = [&]() -> int {
         if (g.nmat == 0) return GLR_OK;
         PhaseScope ps(h0, GLR_PH_SELECT, st);
-        GLR_LAUNCH(h0, 1, select_group(g, st));
+        GLR_LAUNCH(h0, 2, select_group(g, st));
         g = SelectGroup{};
         h0 = nullptr;
         return GLR_OK;
@@ -590,8 +617,25 @@ int step_group(std::vector<StepPlan>& plans, cudaStream_t st) {
     if (!fused.empty() && (rc = compose_fused(fused, st)) != GLR_OK) return rc;
     for (StepPlan* p : unfused)
         if ((rc = compose_unfused(*p, st)) != GLR_OK) return rc;
+    // Refreshes (Semi-Lazy SVD) of different matrices are independent: each runs on its
+    // handle's side stream after the compose pass, overlapping the others and the selection
+    // work of the non-refreshing matrices; the main stream joins them before P is built.
+    std::vector<glr_handle*> refreshing;
+    for (StepPlan& p : plans) {
+        if (!p.refresh) continue;
+        glr_handle* h = p.h;
+        GLR_CK(h, cudaEventRecord(h->rfork, st));
+        GLR_CK(h, cudaStreamWaitEvent(h->rstream, h->rfork, 0));
+        {
+            PhaseScope ps(h, GLR_PH_REFRESH, h->rstream);
+            if ((rc = do_refresh(h, h->rstream)) != GLR_OK) return rc;
+        }
+        GLR_CK(h, cudaEventRecord(h->rdone, h->rstream));
+        refreshing.push_back(h);
+    }
     for (StepPlan& p : plans)
         if ((rc = select_phase(p, st)) != GLR_OK) return rc;
+    for (glr_handle* h : refreshing) GLR_CK(h, cudaStreamWaitEvent(st, h->rdone, 0));
     if ((rc = select_P_grouped(plans, st)) != GLR_OK) return rc;
     if (!fused.empty() && (rc = update_fused(fused, st)) != GLR_OK) return rc;
     for (StepPlan* p : unfused)

@@ -184,8 +184,10 @@ cudaError_t materialize_wy_basis(int mp, int k, const float* Y, const float* Yt,
 // strip of BN columns of one matrix's oriented m' x n' layout and all of its m' rows.
 // ------------------------------------------------------------------------------------------
 constexpr int kGroupPtrs = 512;        // node gradient pointers per grouped launch
-constexpr int kFusedThreads = 512;
-constexpr int kFusedMaxEpt = 32;       // strip elements per thread: m' * BN <= 512 * 32
+constexpr int kFusedThreads = 1024;    // K1: one 4 x 4 block per thread, so m' <= 4096 * 4 / BN
+constexpr int kUpdateThreads = 256;    // K3
+constexpr int kMmaThreads = 512;       // K1 on the tensor cores (k_mma.cu)
+constexpr int kMmaMaxRows = 512;       // 16 warps x 2 m-tiles x 16 rows
 
 struct StreamMat {
     int mp, np, N, r, k;
@@ -193,7 +195,7 @@ struct StreamMat {
     int g_off;                              // first gradient pointer of this matrix in StreamGroup::G
     int strip0, nstrips;                    // CTAs [strip0, strip0 + nstrips) work on this matrix
     float* B; const float* Pprev; float* Mbar;
-    const float* Y; const float* Yt; float* part;   // part: nstrips x m' lambda partial sums
+    const float* YT; const float* YtT; float* part;   // Y^T, Yt^T (k x transposed_pitch(m')); part: nstrips x m'
     uint64_t seed; uint32_t t;
 };
 struct StreamGroup {
@@ -206,6 +208,17 @@ struct StreamGroup {
 // (Mbar - Yt W) against v_j over the strip's columns.
 cudaError_t stream_group(const StreamGroup& g, size_t smem_bytes, cudaStream_t st);
 size_t stream_smem_bytes(int mp, int r, int k, int BN, int gsize, int transposed, int lam);
+// Row pitch of the k x m' transposed copies (YT, YtT and the shared P^T of the FFMA kernel):
+// 16-byte rows covering m' rounded up to 16; consecutive rows start 4 (or 20) banks apart.
+__host__ __device__ __forceinline__ int transposed_pitch(int mp) { return ((mp + 15) & ~15) + 4; }
+// K1 with its rank-r products on the tensor cores (3xTF32 mma.sync): strips of 16 columns,
+// m' <= 512, r <= 16, truncated basis k <= 32 with k % 8 == 0.
+constexpr int kMmaStrip = 16;
+bool mma_stream_eligible(int mp, int np, int r, int k, int lam, int transposed, int gsize);
+size_t mma_stream_smem_bytes(int mp, int r, int k, int lam, int gsize, int transposed);
+cudaError_t stream_group_mma(const StreamGroup& g, size_t smem_bytes, cudaStream_t st);
+// dst (cols x tp) = src^T for row-major src (rows x cols), entries a >= rows set to 0.
+cudaError_t transpose_pad(float* dst, int tp, const float* src, int rows, int cols, cudaStream_t st);
 
 struct UpdateMat {
     int mp, np, r, transposed, compressed;

@@ -152,47 +152,59 @@ namespace {
 __global__ void __launch_bounds__(1024) select_group_kernel(const __grid_constant__ SelectGroup g) {
     extern __shared__ unsigned long long keys[];
     const SelectMat& M = g.mat[blockIdx.x];
-    const int tid = threadIdx.x, mp = M.mp, r = M.r;
+    const int tid = threadIdx.x, mp = M.mp, r = M.r, nth = blockDim.x;
     __shared__ int32_t Js[1024];
     if (M.do_select) {
         int npow2 = 1;
         while (npow2 < mp) npow2 <<= 1;
-        for (int j = tid; j < npow2; j += blockDim.x) {
-            unsigned long long key = 0ull;
-            if (j < mp) {
-                float s = 0.f;
-                for (int t = 0; t < M.ntiles; ++t) s += M.part[(int64_t)t * mp + j];
-                if (M.dsign != nullptr && j < M.k) s *= M.dsign[j];
-                M.lam[j] = s;
-                key = (static_cast<unsigned long long>(__float_as_uint(s * s)) << 32) |
-                      static_cast<unsigned long long>(0xFFFFFFFFu - static_cast<uint32_t>(j));
-            }
-            keys[j] = key;
-        }
+        // lambda-bar was reduced from the partials by lambda_reduce_kernel
+        for (int j = tid; j < npow2; j += nth)
+            keys[j] = j < mp ? (static_cast<unsigned long long>(__float_as_uint(M.lam[j] * M.lam[j])) << 32) |
+                                   static_cast<unsigned long long>(0xFFFFFFFFu - static_cast<uint32_t>(j))
+                             : 0ull;
         __syncthreads();
-        for (int size = 2; size <= npow2; size <<= 1) {
-            for (int stride = size >> 1; stride > 0; stride >>= 1) {
-                for (int i = tid; i < npow2; i += blockDim.x) {
-                    const int partner = i ^ stride;
-                    if (partner > i) {
-                        const bool desc = (i & size) == 0;
-                        const unsigned long long x = keys[i], y = keys[partner];
-                        if ((x < y) == desc) { keys[i] = y; keys[partner] = x; }
-                    }
-                }
-                __syncthreads();
+        if (mp <= 1024) {
+            // keys are distinct: j is among the r largest iff fewer than r keys exceed it
+            __shared__ unsigned char win[1024];
+            for (int j = tid; j < mp; j += nth) {
+                const unsigned long long kj = keys[j];
+                int above = 0;
+                for (int w = 0; w < mp; ++w) above += keys[w] > kj;
+                win[j] = above < r ? 1 : 0;
             }
-        }
-        for (int q = tid; q < r; q += blockDim.x) {
-            const uint32_t jq = 0xFFFFFFFFu - static_cast<uint32_t>(keys[q] & 0xFFFFFFFFull);
-            int rank = 0;
-            for (int w = 0; w < r; ++w)
-                rank += (0xFFFFFFFFu - static_cast<uint32_t>(keys[w] & 0xFFFFFFFFull)) < jq;
-            M.J[rank] = static_cast<int32_t>(jq);
-            Js[rank] = static_cast<int32_t>(jq);
+            __syncthreads();
+            for (int j = tid; j < mp; j += nth) {
+                if (!win[j]) continue;
+                int pos = 0;
+                for (int w = 0; w < j; ++w) pos += win[w];
+                M.J[pos] = j;
+                Js[pos] = j;
+            }
+        } else {
+            for (int size = 2; size <= npow2; size <<= 1) {
+                for (int stride = size >> 1; stride > 0; stride >>= 1) {
+                    for (int i = tid; i < npow2; i += nth) {
+                        const int partner = i ^ stride;
+                        if (partner > i) {
+                            const bool desc = (i & size) == 0;
+                            const unsigned long long x = keys[i], y = keys[partner];
+                            if ((x < y) == desc) { keys[i] = y; keys[partner] = x; }
+                        }
+                    }
+                    __syncthreads();
+                }
+            }
+            for (int q = tid; q < r; q += nth) {
+                const uint32_t jq = 0xFFFFFFFFu - static_cast<uint32_t>(keys[q] & 0xFFFFFFFFull);
+                int rank = 0;
+                for (int w = 0; w < r; ++w)
+                    rank += (0xFFFFFFFFu - static_cast<uint32_t>(keys[w] & 0xFFFFFFFFull)) < jq;
+                M.J[rank] = static_cast<int32_t>(jq);
+                Js[rank] = static_cast<int32_t>(jq);
+            }
         }
     } else {
-        for (int q = tid; q < r; q += blockDim.x) Js[q] = M.J[q];
+        for (int q = tid; q < r; q += nth) Js[q] = M.J[q];
     }
     __syncthreads();
     const int k = M.k;
@@ -214,8 +226,37 @@ __global__ void __launch_bounds__(1024) select_group_kernel(const __grid_constan
 }
 }  // namespace
 
+// lambda-bar_j = d_j * sum_t part[t][j]: block (x, matrix) covers 32 consecutive j (lanes)
+// with its 32 warps taking every 32nd tile; the warp sums are added in warp order.
+__global__ void __launch_bounds__(1024) lambda_reduce_kernel(const __grid_constant__ SelectGroup g) {
+    const SelectMat& M = g.mat[blockIdx.y];
+    if (!M.do_select) return;
+    const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
+    const int j = blockIdx.x * 32 + lane;
+    if (blockIdx.x * 32 >= M.mp) return;
+    __shared__ float red[32][33];
+    float sum = 0.f;
+    if (j < M.mp)
+        for (int t = w; t < M.ntiles; t += 32) sum += M.part[(int64_t)t * M.mp + j];
+    red[w][lane] = sum;
+    __syncthreads();
+    if (w == 0 && j < M.mp) {
+        float tot = 0.f;
+        for (int ww = 0; ww < 32; ++ww) tot += red[ww][lane];
+        if (M.dsign != nullptr && j < M.k) tot *= M.dsign[j];
+        M.lam[j] = tot;
+    }
+}
+
 cudaError_t select_group(const SelectGroup& g, cudaStream_t st) {
     if (g.nmat <= 0) return cudaSuccess;
+    {
+        int maxmp = 1;
+        for (int i = 0; i < g.nmat; ++i) maxmp = g.mat[i].mp > maxmp ? g.mat[i].mp : maxmp;
+        lambda_reduce_kernel<<<dim3((maxmp + 31) / 32, g.nmat), 1024, 0, st>>>(g);
+        cudaError_t e = cudaGetLastError();
+        if (e != cudaSuccess) return e;
+    }
     int maxmp = 1;
     for (int i = 0; i < g.nmat; ++i) maxmp = g.mat[i].mp > maxmp ? g.mat[i].mp : maxmp;
     int npow2 = 1;

@@ -228,3 +228,14 @@ def test_step_group_equals_single_steps(basis_rank):
             assert torch.equal(solo[j].error(0), grp[j].error(0))
     for h in solo + grp:
         h.close()
+
+
+@pytest.mark.parametrize("m,n,dtype,k", [(640, 1280, "f32", 16), (1280, 640, "bf16", 0), (1024, 256, "bf16", 16),
+                                         (256, 1024, "f32", 0), (96, 2048, "f32", 8)])
+def test_fused_kernel_shapes_lockstep(m, n, dtype, k):
+    """Aligned shapes that take the fused kernels: m' > 512 runs the FFMA strip kernel, m' <= 512
+    the tensor-core (3xTF32 mma.sync) strip kernel; transposed and bf16 gradients included."""
+    g = _synthetic(m, n, 3, 24, lambda j: 1.0 / j, 0.05, 40 + m, dtype=dtype)
+    reps = lockstep(m, n, 6, 3, 5, g, dtype=dtype, tau=3, optimizer="msgd", lr=0.05, beta1=0.9, seed=6,
+                    basis_rank=k)
+    _assert_reports(reps)
