@@ -36,6 +36,7 @@ struct glr_handle {
     float *Q = nullptr, *Qn = nullptr, *Y = nullptr, *Yt = nullptr, *T = nullptr, *dsign = nullptr;
     float *Wbar = nullptr, *Z = nullptr, *Hk = nullptr, *Vk = nullptr, *gram = nullptr, *scratch = nullptr;
     float *YT = nullptr, *YtT = nullptr;   // k x transposed_pitch(m') copies of Y and Yt for the fused kernel
+    float *YF = nullptr, *YtF = nullptr;   // Y and Yt in fragment order for the tensor-core kernel
     int* dflags = nullptr;   // [0] Cholesky restarts, [1] Jacobi sweeps of the last refresh
     float* gemm_ws = nullptr;   // split-K partial tiles of the refresh GEMMs
     cudaStream_t rstream = nullptr;            // side stream of this handle's refresh
@@ -170,6 +171,10 @@ int wy_from_Q(glr_handle* h, cudaStream_t st) {
     // transposed copies (k x tp, zero-padded) for the fused compose kernel's lambda epilogue
     GLR_LAUNCH(h, 1, transpose_pad(h->YT, transposed_pitch(mp), h->Y, mp, k, st));
     GLR_LAUNCH(h, 1, transpose_pad(h->YtT, transposed_pitch(mp), h->Yt, mp, k, st));
+    if (h->mma) {
+        GLR_LAUNCH(h, 1, pack_frag(h->YF, h->Y, mp, k, k, 0, st));
+        GLR_LAUNCH(h, 1, pack_frag(h->YtF, h->Yt, mp, k, k, 1, st));
+    }
     return GLR_OK;
 }
 
@@ -328,6 +333,10 @@ int glr_create(int64_t m, int64_t n, int32_t r, int32_t N, const glr_schedule* s
         A(&h->evals, K); A(&h->evals_sorted, K);
         A(&h->YT, K * transposed_pitch(static_cast<int>(mp)));
         A(&h->YtT, K * transposed_pitch(static_cast<int>(mp)));
+        if (h->mma) {
+            const size_t frag = ((MP + 7) & ~size_t(7)) * ((K + 7) & ~size_t(7));
+            A(&h->YF, frag); A(&h->YtF, frag);
+        }
     }
     if (rc != GLR_OK) {
         g_create_err = h->err;
@@ -450,7 +459,8 @@ int compose_fused(std::vector<StepPlan*>& plans, cudaStream_t st) {
         std::vector<StepPlan*> rest;
         for (StepPlan* p : todo) {
             glr_handle* h = p->h;
-            if (h->BN != BN || h->s.grad_dtype != dt || h->mma != mma || g.nmat == kGroupMax ||
+            if (h->BN != BN || h->s.grad_dtype != dt || h->mma != mma ||
+                (mma && mma_stream_nq(h->r) != mma_stream_nq(todo.front()->h->r)) || g.nmat == kGroupMax ||
                 g.nmat + 0 >= kGroupMax || (int)(g.nmat ? g.mat[g.nmat - 1].g_off + g.mat[g.nmat - 1].N : 0) + h->N > kGroupPtrs) {
                 rest.push_back(p);
                 continue;
@@ -462,7 +472,7 @@ int compose_fused(std::vector<StepPlan*>& plans, cudaStream_t st) {
             M.g_off = g.nmat ? g.mat[g.nmat - 1].g_off + g.mat[g.nmat - 1].N : 0;
             M.strip0 = g.total_strips; M.nstrips = h->nstrips;
             M.B = h->B; M.Pprev = h->Pprev; M.Mbar = h->Mbar;
-            M.YT = h->YT; M.YtT = h->YtT; M.part = h->lam_part;
+            M.YT = h->YT; M.YtT = h->YtT; M.YF = h->YF; M.YtF = h->YtF; M.part = h->lam_part;
             M.seed = h->s.seed; M.t = static_cast<uint32_t>(h->t);
             for (int i = 0; i < h->N; ++i) g.G[M.g_off + i] = p->G[i];
             g.total_strips += h->nstrips;

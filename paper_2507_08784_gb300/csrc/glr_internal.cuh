@@ -187,7 +187,6 @@ constexpr int kGroupPtrs = 512;        // node gradient pointers per grouped lau
 constexpr int kFusedThreads = 1024;    // K1: one 4 x 4 block per thread, so m' <= 4096 * 4 / BN
 constexpr int kUpdateThreads = 256;    // K3
 constexpr int kMmaThreads = 512;       // K1 on the tensor cores (k_mma.cu)
-constexpr int kMmaMaxRows = 512;       // 16 warps x 2 m-tiles x 16 rows
 
 struct StreamMat {
     int mp, np, N, r, k;
@@ -196,6 +195,7 @@ struct StreamMat {
     int strip0, nstrips;                    // CTAs [strip0, strip0 + nstrips) work on this matrix
     float* B; const float* Pprev; float* Mbar;
     const float* YT; const float* YtT; float* part;   // Y^T, Yt^T (k x transposed_pitch(m')); part: nstrips x m'
+    const float* YF; const float* YtF;                // Y, Yt in the tensor-core kernel's fragment order
     uint64_t seed; uint32_t t;
 };
 struct StreamGroup {
@@ -212,11 +212,16 @@ size_t stream_smem_bytes(int mp, int r, int k, int BN, int gsize, int transposed
 // 16-byte rows covering m' rounded up to 16; consecutive rows start 4 (or 20) banks apart.
 __host__ __device__ __forceinline__ int transposed_pitch(int mp) { return ((mp + 15) & ~15) + 4; }
 // K1 with its rank-r products on the tensor cores (3xTF32 mma.sync): strips of 16 columns,
-// m' <= 512, r <= 16, truncated basis k <= 32 with k % 8 == 0.
+// m' <= 512 for r <= 8 and m' <= 256 for r <= 16, truncated basis k <= 32.  One launch takes
+// matrices of one mma_stream_nq(r) only.
 constexpr int kMmaStrip = 16;
+int mma_stream_nq(int r);
 bool mma_stream_eligible(int mp, int np, int r, int k, int lam, int transposed, int gsize);
 size_t mma_stream_smem_bytes(int mp, int r, int k, int lam, int gsize, int transposed);
 cudaError_t stream_group_mma(const StreamGroup& g, size_t smem_bytes, cudaStream_t st);
+// src (rows x cols, row-major, leading dimension ld) in the tensor-core kernel's fragment order
+// (up8(rows) x up8(cols) floats, zero-padded); form 0 for Y, form 1 for Yt.
+cudaError_t pack_frag(float* dst, const float* src, int rows, int cols, int ld, int form, cudaStream_t st);
 // dst (cols x tp) = src^T for row-major src (rows x cols), entries a >= rows set to 0.
 cudaError_t transpose_pad(float* dst, int tp, const float* src, int rows, int cols, cudaStream_t st);
 

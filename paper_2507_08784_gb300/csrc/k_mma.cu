@@ -1,21 +1,36 @@
-// K1 on the tensor cores: the fused compose pass of k_fused.cu with its two rank-r products
-// done by warp-level TF32 MMA (mma.sync m16n8k8) in the 3xTF32 form (each fp32 operand x is
-// split into x_hi = tf32(x) and x_lo = tf32(x - x_hi); a*b ~ a_hi b_hi + a_hi b_lo + a_lo b_hi,
-// accumulated in fp32, which keeps fp32-level accuracy).  The products are tiny (K or N = r),
-// so the tensor pipe is far from busy: the point is to replace ~4r FFMA (plus operand loads and
-// index arithmetic) per node-element with a handful of MMA instructions per warp.
+// K1 on the tensor cores: the fused compose pass with its two rank-r products done by warp-level
+// TF32 MMA (mma.sync m16n8k8) in the 3xTF32 form (each fp32 operand x is split into
+// x_hi = tf32(x) and x_lo = tf32(x - x_hi); a*b ~ a_hi b_hi + a_hi b_lo + a_lo b_hi, accumulated in
+// fp32, which keeps fp32-level accuracy).  The products are tiny (K or N = r), so the tensor pipe
+// is far from busy: the point is to replace ~2r FFMA (plus operand loads and index arithmetic)
+// per node-element with a few MMA instructions per warp.
 //
 // Per CTA: one strip of 16 columns x all m' (<= 512) rows of one matrix; 16 warps.  A 3-slot
-// cp.async ring holds node i's B and G strips while nodes i+1 and i+2 are in flight.
+// cp.async ring holds node i's B and G strips while nodes i+1 and i+2 are in flight; after the
+// last node the two free slots receive Y and Yt for the truncated-basis lambda epilogue.
 //   node i:  R_i^T (16 x r) = B_i,strip^T P_prev        K = m' split over the warps
 //            C (m' x 16)    = P_prev R_i                 K = r
-//            M_i = G_i + B_i - C;  B_i <- M_i;  acc += M_i
+//            M_i = G_i + (B_i - C);  B_i <- M_i;  acc += M_i
 //   epilogue: Mbar, and for a truncated basis the Approx-Top-r partial sums of
 //            (Mbar - Yt (Y^T Mbar)) v_j over the strip (the same two products with Y, Yt).
+//
 // Fragment layouts (PTX ISA, mma.m16n8k8 .tf32): with g = lane / 4, t = lane % 4,
 //   A (16 x 8): a0 (g, t), a1 (g + 8, t), a2 (g, t + 4), a3 (g + 8, t + 4)
 //   B (8 x 8):  b0 (t, g), b1 (t + 4, g)
 //   C (16 x 8): c0 (g, 2t), c1 (g, 2t + 1), c2 (g + 8, 2t), c3 (g + 8, 2t + 1)
+// Both products are computed transposed, with M = the strip's 16 columns, and their indices are
+// relabelled so that one lane owns the same four elements of every operand: in each 8-row group
+// the lane owns rows t, t + 4 and strip columns 2g, 2g + 1,
+//   e0 = (t, 2g)   e1 = (t, 2g + 1)   e2 = (t + 4, 2g)   e3 = (t + 4, 2g + 1).
+//   R^T = B^T P   (M = columns, K = rows, N = q): M index m <-> column 2 (m % 8) + m / 8, K index
+//                 k <-> row k.  A fragment = (e0, e1, e2, e3); B fragment P(t, q), P(t + 4, q).
+//   C^T = R^T P^T (M = columns, K = q, N = rows): N index n <-> row n / 2 + 4 (n % 2), K index k
+//                 <-> q = 2 (k % 4) + k / 4.  C fragment = (e0, e2, e1, e3); its A fragment is
+//                 the R^T C fragment in the order (c0, c2, c1, c3); B fragment P(row, 2t),
+//                 P(row, 2t + 1) with row = g / 2 + 4 (g % 2).
+// Sums over K are order-free, so the relabelling changes nothing but the rounding order.  B is
+// read from shared memory once per node for both products, P's fragments are loaded once per
+// strip into registers, and no operand is re-staged between the products.
 #include "glr_internal.cuh"
 
 namespace glr {
@@ -25,7 +40,6 @@ namespace {
 constexpr int T = kMmaThreads;         // 512 threads = 16 warps
 constexpr int NW = T / 32;
 constexpr int SW = 16;                 // strip width (columns)
-constexpr int RP = SW + 8;             // pitch of R / W in shared memory: conflict-free B fragments
 
 __device__ __forceinline__ uint32_t to_tf32(float x) {
     uint32_t r;
@@ -74,102 +88,13 @@ __device__ __forceinline__ void cp_async_wait() {
 
 __host__ __device__ __forceinline__ int up8(int x) { return (x + 7) & ~7; }
 __host__ __device__ __forceinline__ int up16(int x) { return (x + 15) & ~15; }
-// Pitch of the transposed r x m' copy of P: = 8 (mod 32) so the A-fragment loads hit 32 banks.
-__host__ __device__ __forceinline__ int mma_pt(int mp) { return ((mp + 31) & ~31) + 8; }
 __host__ __device__ __forceinline__ size_t a16(size_t x) { return (x + 15) & ~size_t(15); }
 
-__device__ __forceinline__ float2 ldg2(const float* p) { return __ldcs(reinterpret_cast<const float2*>(p)); }
-__device__ __forceinline__ float2 ldg2(const __nv_bfloat16* p) {
-    const __nv_bfloat162 v = __ldcs(reinterpret_cast<const __nv_bfloat162*>(p));
-    return __bfloat1622float2(v);
-}
-template <typename GT> __device__ __forceinline__ float ldg1(const GT* p);
-template <> __device__ __forceinline__ float ldg1<float>(const float* p) { return __ldcs(p); }
-template <> __device__ __forceinline__ float ldg1<__nv_bfloat16>(const __nv_bfloat16* p) {
-    return __bfloat162float(__ldcs(p));
-}
-
-// Strips are 16 columns wide; a strip row is 64 bytes = four 16-byte chunks.  B strips are
-// stored with chunk c of row a at position c ^ (2 * ((a >> 1) & 1)), which makes the A-fragment
-// loads of the R^T product (rows k0 + t, t < 4, columns g and g + 8) hit 32 distinct banks.
+// Strip rows are 64 bytes = four 16-byte chunks.  fp32 strips (B, and G when it is fp32) store
+// chunk c of row a at position c ^ (2 * ((a >> 1) & 1)), which makes the 8-byte loads of a lane's
+// (row t or t + 4, columns 2g, 2g + 1) hit 32 distinct banks per half-warp.
 __device__ __forceinline__ int sw_elem(int a, int c) {
     return a * SW + 4 * ((c >> 2) ^ (((a >> 1) & 1) << 1)) + (c & 3);
-}
-
-// R^T (16 x RQ) = S^T P: S the m' x 16 swizzled strip, P given transposed (Pt, RQ x pt, rows
-// q >= r zero), K = m' split over the warps (warp w takes k-steps w, w + NW, ...).  The warp
-// partials are added in warp order into out (RQ x RP).  Ends with __syncthreads.
-template <bool GLOBAL_P>
-__device__ __forceinline__ void rt_product(const float* S, const float* Pt, int pt, int mp16, int RQ, float* part,
-                                           float* out) {
-    const int w = threadIdx.x >> 5, lane = threadIdx.x & 31, g = lane >> 2, t = lane & 3;
-    const int nq = RQ / 8;             // 1..4 n-tiles over q
-    float d[4][4];
-#pragma unroll
-    for (int j = 0; j < 4; ++j)
-#pragma unroll
-        for (int e = 0; e < 4; ++e) d[j][e] = 0.f;
-    // A fragment addresses: rows k0 + t and k0 + t + 4 share the swizzle of row t (k0 % 8 == 0)
-    const int swt = ((t >> 1) & 1) << 1;
-    const int oa0 = t * SW + 4 * ((g >> 2) ^ swt) + (g & 3);          // (k0 + t, g)
-    const int oa1 = t * SW + 4 * (((g >> 2) + 2) ^ swt) + (g & 3);    // (k0 + t, g + 8)
-    const float* sk = S + (w * 8) * SW;
-    const float* pk = Pt + g * pt + w * 8 + t;
-    const int kstep = NW * 8;
-    for (int k0 = w * 8; k0 < mp16; k0 += kstep, sk += kstep * SW, pk += kstep) {
-        const FragA A = frag_a(sk[oa0], sk[oa1], sk[oa0 + 4 * SW], sk[oa1 + 4 * SW]);
-#pragma unroll
-        for (int nt = 0; nt < 4; ++nt) {
-            if (nt < nq) {
-                const float* prow = pk + nt * 8 * pt;
-                const FragB B = GLOBAL_P ? frag_b(__ldg(prow), __ldg(prow + 4)) : frag_b(prow[0], prow[4]);
-                mma3(d[nt], A, B);
-            }
-        }
-    }
-    float* mine = part + w * (RQ * SW) + (2 * t) * SW + g;
-#pragma unroll
-    for (int nt = 0; nt < 4; ++nt) {
-        if (nt < nq) {
-            float* m = mine + nt * 8 * SW;
-            m[0] = d[nt][0];
-            m[SW] = d[nt][1];
-            m[8] = d[nt][2];
-            m[SW + 8] = d[nt][3];
-        }
-    }
-    __syncthreads();
-    for (int o = threadIdx.x; o < RQ * SW; o += T) {
-        const float* pp = part + o;
-        float acc = 0.f;
-#pragma unroll 4
-        for (int ww = 0; ww < NW; ++ww, pp += RQ * SW) acc += *pp;
-        out[(o / SW) * RP + (o % SW)] = acc;
-    }
-    __syncthreads();
-}
-
-// C fragments of P R for m-tile m0 (rows m0..m0+15) and the two 8-column tiles: c[nt][e],
-// K = RQ (columns of P, zero beyond r).  R is RQ x RP.
-template <bool GLOBAL_P>
-__device__ __forceinline__ void c_product(const float* Pt, int pt, const float* R, int RQ, int m0, float (&c)[2][4]) {
-    const int lane = threadIdx.x & 31, g = lane >> 2, t = lane & 3;
-#pragma unroll
-    for (int nt = 0; nt < 2; ++nt)
-#pragma unroll
-        for (int e = 0; e < 4; ++e) c[nt][e] = 0.f;
-    const float* p0 = Pt + t * pt + m0 + g;
-    const float* rr = R + t * RP + g;
-    for (int kq = 0; kq < RQ; kq += 8, p0 += 8 * pt, rr += 8 * RP) {
-        const float* p1 = p0 + 4 * pt;
-        const FragA A = GLOBAL_P ? frag_a(__ldg(p0), __ldg(p0 + 8), __ldg(p1), __ldg(p1 + 8))
-                                 : frag_a(p0[0], p0[8], p1[0], p1[8]);
-#pragma unroll
-        for (int nt = 0; nt < 2; ++nt) {
-            const FragB B = frag_b(rr[nt * 8], rr[4 * RP + nt * 8]);
-            mma3(c[nt], A, B);
-        }
-    }
 }
 
 // Ring stage layout: [B strip: mp16 x 16 fp32, swizzled][G strip: mp16 x 16 (gradient dtype),
@@ -179,9 +104,45 @@ __host__ __device__ __forceinline__ int g_tpitch(int mp16, int gsize) { return m
 __host__ __device__ __forceinline__ size_t stage_g_bytes(int mp16, int gsize, int transposed) {
     return a16(transposed ? (size_t)SW * g_tpitch(mp16, gsize) * gsize : (size_t)mp16 * SW * gsize);
 }
+// Warp partials of a 16 x (8 NT) product: one float4 per lane and n-tile; the pitch between
+// warps is = 8 (mod 32) floats so the quarter-sums of the reduction hit distinct banks.
+__host__ __device__ __forceinline__ int part_pitch(int NT) { return NT * 128 + 8; }
 
-template <typename GT>
+// tot[o] = sum over the 16 warps of part[w][o], o < NT * 128, in a fixed order: four threads
+// per output each add four warps (w = q, q + 4, q + 8, q + 12), then two xor-shuffles.
+__device__ __forceinline__ void reduce_warps(const float* part, int pitch, int NT, float* tot) {
+    const int nout = NT * 128;
+    for (int base = 0; base < nout * 4; base += T) {
+        const int idx = base + threadIdx.x, o = idx >> 2, q = idx & 3;
+        float a = 0.f;
+        if (o < nout) {
+            const float* p = part + q * pitch + o;
+            a = ((p[0] + p[4 * pitch]) + p[8 * pitch]) + p[12 * pitch];
+        }
+        a += __shfl_xor_sync(0xffffffffu, a, 1);
+        a += __shfl_xor_sync(0xffffffffu, a, 2);
+        if (q == 0 && o < nout) tot[o] = a;
+    }
+}
+
+template <typename GT> struct GradPair;
+template <> struct GradPair<float> {
+    // (row a, columns 2g, 2g + 1) of a row-major swizzled fp32 strip
+    static __device__ __forceinline__ float2 row(const float* Gs, int a, int c) {
+        return *reinterpret_cast<const float2*>(Gs + sw_elem(a, c));
+    }
+};
+template <> struct GradPair<__nv_bfloat16> {
+    static __device__ __forceinline__ float2 row(const __nv_bfloat16* Gs, int a, int c) {
+        return __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(Gs + a * SW + c));
+    }
+};
+
+// NQ = ceil(r / 8) n-tiles over q; each warp owns up to GPW = 4 / NQ groups of 8 rows
+// (group w + 16 j), so m' <= 128 GPW.
+template <typename GT, int NQ>
 __global__ void __launch_bounds__(T, 1) stream_mma_kernel(const __grid_constant__ StreamGroup g) {
+    constexpr int GPW = 4 / NQ;
     extern __shared__ __align__(16) unsigned char smem[];
     int mi = 0;
     while (mi + 1 < g.nmat && blockIdx.x >= static_cast<unsigned>(g.mat[mi + 1].strip0)) ++mi;
@@ -189,19 +150,22 @@ __global__ void __launch_bounds__(T, 1) stream_mma_kernel(const __grid_constant_
     const int s = blockIdx.x - M.strip0;
     const int b0 = s * SW;
     const int mp = M.mp, np = M.np, r = M.r, N = M.N;
-    const int mp16 = up16(mp), RQ = up8(r), pt = mma_pt(mp);
+    const int mp16 = up16(mp), ng = up8(mp) >> 3;
     const int tid = threadIdx.x, w = tid >> 5, lane = tid & 31, gg = lane >> 2, t = lane & 3;
     constexpr int GS = sizeof(GT);
     constexpr int EPC = 16 / GS;                      // gradient elements per 16-byte chunk
     const bool trans = M.transposed != 0;
     const int gpt = g_tpitch(mp16, GS);
     const size_t sb = stage_b_bytes(mp16), sg = stage_g_bytes(mp16, GS, trans), stage = sb + sg;
+    const int KT = M.lam ? up8(M.k) >> 3 : 0;        // n-tiles of the lambda epilogue
+    const int pitch = part_pitch(NQ > KT ? NQ : KT);
     unsigned char* ring = smem;
-    float* Pt = reinterpret_cast<float*>(smem + 3 * stage);
-    float* Rs = Pt + a16((size_t)RQ * pt * 4) / 4;
-    float* Rpart = Rs + a16((size_t)32 * RP * 4) / 4;
+    float* part = reinterpret_cast<float*>(smem + 3 * stage);
+    float* tot = part + NW * pitch;
     const bool corr = !M.e_zero;
     const GT* const* Gp = reinterpret_cast<const GT* const*>(g.G + M.g_off);
+    const int c2 = 2 * gg;                            // the lane's first strip column
+    const bool colok = b0 + c2 < np;                  // n' % 4 == 0: both columns or neither
 
     // ---- per-thread staging plan (fixed for all nodes): up to 4 chunks of B and 4 of G -------
     int boff[4], bdst[4], goff[4], gdst[4];
@@ -233,7 +197,7 @@ __global__ void __launch_bounds__(T, 1) stream_mma_kernel(const __grid_constant_
             constexpr int CPR = SW / EPC;
             const int ga = c / CPR, gch = c % CPR, gcol = b0 + gch * EPC;
             goff[j] = ga * np + gcol;
-            gdst[j] = ga * SW + gch * EPC;
+            gdst[j] = GS == 4 ? ga * SW + 4 * (gch ^ (((ga >> 1) & 1) << 1)) : ga * SW + gch * EPC;
             if (c < mp * CPR) {
                 if (gcol < np) gmask |= 1u << j;
                 else for (int st = 0; st < 3; ++st)
@@ -242,7 +206,8 @@ __global__ void __launch_bounds__(T, 1) stream_mma_kernel(const __grid_constant_
             }
         }
     }
-    // rows mp..mp16 of every B strip and every (non-transposed) G strip stay zero
+    // rows mp..mp16 of every B strip and every (non-transposed) G strip stay zero; transposed
+    // matrices have m' % 8 == 0, so their row groups never reach past m'
     for (int a = mp + (tid >> 4); a < mp16; a += T / SW) {
         const int c = tid & (SW - 1);
 #pragma unroll
@@ -251,220 +216,295 @@ __global__ void __launch_bounds__(T, 1) stream_mma_kernel(const __grid_constant_
             if (!trans) reinterpret_cast<GT*>(ring + st * stage + sb)[a * SW + c] = GT(0.f);
         }
     }
-    if (corr)
-        for (int q = 0; q < RQ; ++q)
-            for (int a = tid; a < pt; a += T) Pt[q * pt + a] = (q < r && a < mp) ? M.Pprev[a * r + q] : 0.f;
 
-    auto stage_node = [&](int i) {
-        if (i < N) {
-            unsigned char* base = ring + (size_t)(i % 3) * stage;
+    // ring item j: node j's B (unless E = 0) and G strips; with the lambda epilogue, items N and
+    // N + 1 are the fragment-ordered Y and Yt (up8(m') x 8 KT floats each)
+    auto stage_item = [&](int j) {
+        if (j < N) {
+            unsigned char* base = ring + (size_t)(j % 3) * stage;
             if (corr) {
                 float* dst = reinterpret_cast<float*>(base);
-                const float* src = M.B + (int64_t)i * mp * np;
+                const float* src = M.B + (int64_t)j * mp * np;
 #pragma unroll
-                for (int j = 0; j < 4; ++j)
-                    if (bmask & (1u << j)) cp_async16(dst + bdst[j], src + boff[j]);
+                for (int q = 0; q < 4; ++q)
+                    if (bmask & (1u << q)) cp_async16(dst + bdst[q], src + boff[q]);
             }
             GT* dst = reinterpret_cast<GT*>(base + sb);
-            const GT* src = Gp[i];
+            const GT* src = Gp[j];
 #pragma unroll
-            for (int j = 0; j < 4; ++j)
-                if (gmask & (1u << j)) cp_async16(dst + gdst[j], src + goff[j]);
+            for (int q = 0; q < 4; ++q)
+                if (gmask & (1u << q)) cp_async16(dst + gdst[q], src + goff[q]);
+        } else if (j < N + 2 && KT) {
+            float* dst = reinterpret_cast<float*>(ring + (size_t)(j % 3) * stage);
+            const float* src = j == N ? M.YF : M.YtF;
+            const int nch = ng * KT * 16;             // 64 floats per (group, n-tile)
+            for (int c = tid; c < nch; c += T) cp_async16(dst + 4 * c, src + 4 * c);
         }
         cp_async_commit();
     };
-    stage_node(0);
-    stage_node(1);
+    stage_item(0);
+    stage_item(1);
 
-    // ---- per-lane fragment geometry (fixed for all nodes) ------------------------------------
-    const int ntiles_m = mp16 / 16;
-    const int swz = ((gg >> 1) & 1) << 1;             // swizzle of rows m0 + gg (+8): m0 % 16 == 0
-    int soff[2], goffc[2], colv[2];                  // per n-tile: swizzled column offset, G column, global column
+    // ---- P_prev fragments of the lane's row groups, once per strip ----------------------------
+    const int prow = (gg >> 1) + 4 * (gg & 1);      // C^T = R^T P^T: N index g -> row
+    FragB prt[GPW][NQ], pcb[GPW][NQ];
 #pragma unroll
-    for (int nt = 0; nt < 2; ++nt) {
-        const int bl = nt * 8 + 2 * t;
-        soff[nt] = 4 * ((bl >> 2) ^ swz) + (bl & 3);
-        goffc[nt] = trans ? bl * gpt : bl;
-        colv[nt] = b0 + bl;
+    for (int j = 0; j < GPW; ++j) {
+        const int G8 = w + NW * j;
+        const int ra = 8 * G8 + t, rc = 8 * G8 + prow;
+#pragma unroll
+        for (int nt = 0; nt < NQ; ++nt) {
+            const int q = 8 * nt + gg, q0 = 8 * nt + 2 * t;
+            const bool use = corr && G8 < ng;
+            const float* P = M.Pprev;
+            prt[j][nt] = frag_b(use && q < r && ra < mp ? __ldg(P + ra * r + q) : 0.f,
+                                use && q < r && ra + 4 < mp ? __ldg(P + (ra + 4) * r + q) : 0.f);
+            pcb[j][nt] = frag_b(use && q0 < r && rc < mp ? __ldg(P + rc * r + q0) : 0.f,
+                                use && q0 + 1 < r && rc < mp ? __ldg(P + rc * r + q0 + 1) : 0.f);
+        }
     }
-    int rowoff[2][2];                                 // global row offsets a * n' of (u, h)
-#pragma unroll
-    for (int u = 0; u < 2; ++u)
-#pragma unroll
-        for (int h = 0; h < 2; ++h) rowoff[u][h] = ((w + u * NW) * 16 + gg + 8 * h) * np;
 
-    float acc[2][2][4];
+    float acc[GPW][4];
 #pragma unroll
-    for (int u = 0; u < 2; ++u)
+    for (int j = 0; j < GPW; ++j)
 #pragma unroll
-        for (int nt = 0; nt < 2; ++nt)
-#pragma unroll
-            for (int e = 0; e < 4; ++e) acc[u][nt][e] = 0.f;
+        for (int e = 0; e < 4; ++e) acc[j][e] = 0.f;
 
     for (int i = 0; i < N; ++i) {
-        stage_node(i + 2);                 // ring slot (i+2)%3 was released by node i-1
-        cp_async_wait<2>();                // node i has landed; nodes i+1, i+2 may be in flight
-        __syncthreads();
+        cp_async_wait<1>();                // node i has landed; item i + 1 may be in flight
+        __syncthreads();                   // ... for every thread; node i - 1 is finished
+        stage_item(i + 2);                 // into the slot node i - 1 used
         const unsigned char* base = ring + (size_t)(i % 3) * stage;
         const float* S = reinterpret_cast<const float*>(base);
         const GT* Gs = reinterpret_cast<const GT*>(base + sb);
-        if (corr) rt_product<false>(S, Pt, pt, mp16, RQ, Rpart, Rs);
-        float* Bi = M.B + (int64_t)i * mp * np;
+        if (corr) {                        // warp partials of R_i^T = B_i^T P_prev
+            float d[NQ][4];
 #pragma unroll
-        for (int u = 0; u < 2; ++u) {
-            const int mt = w + u * NW;
-            if (mt < ntiles_m) {
-                const int m0 = mt * 16;
-                float c[2][4];
-                if (corr) c_product<false>(Pt, pt, Rs, RQ, m0, c);
+            for (int nt = 0; nt < NQ; ++nt)
 #pragma unroll
-                for (int h = 0; h < 2; ++h) {
-                    const int a = m0 + gg + 8 * h;
-                    if (a < mp) {
-                        const float* Sa = S + a * SW;
-                        const GT* Ga = trans ? Gs + a : Gs + a * SW;
-                        float* Ba = Bi + rowoff[u][h];
+                for (int e = 0; e < 4; ++e) d[nt][e] = 0.f;
 #pragma unroll
-                        for (int nt = 0; nt < 2; ++nt) {
-                            if (colv[nt] < np) {
-                                const GT* gp = Ga + goffc[nt];
-                                float m0v = static_cast<float>(gp[0]);
-                                float m1v = static_cast<float>(trans ? gp[gpt] : gp[1]);
-                                if (corr) {
-                                    const float2 bv = *reinterpret_cast<const float2*>(Sa + soff[nt]);
-                                    m0v += bv.x - c[nt][2 * h];
-                                    m1v += bv.y - c[nt][2 * h + 1];
-                                }
-                                if (M.write_B) __stcs(reinterpret_cast<float2*>(Ba + colv[nt]), make_float2(m0v, m1v));
-                                acc[u][nt][2 * h] += m0v;
-                                acc[u][nt][2 * h + 1] += m1v;
-                            }
-                        }
-                    }
+            for (int j = 0; j < GPW; ++j) {
+                const int G8 = w + NW * j;
+                if (G8 < ng) {
+                    const int ra = 8 * G8 + t;
+                    const float2 x0 = *reinterpret_cast<const float2*>(S + sw_elem(ra, c2));
+                    const float2 x1 = *reinterpret_cast<const float2*>(S + sw_elem(ra + 4, c2));
+                    const FragA A = frag_a(x0.x, x0.y, x1.x, x1.y);
+#pragma unroll
+                    for (int nt = 0; nt < NQ; ++nt) mma3(d[nt], A, prt[j][nt]);
                 }
             }
+#pragma unroll
+            for (int nt = 0; nt < NQ; ++nt)
+                *reinterpret_cast<float4*>(part + w * pitch + (nt * 32 + lane) * 4) =
+                    make_float4(d[nt][0], d[nt][1], d[nt][2], d[nt][3]);
         }
         __syncthreads();
+        FragA RA[NQ];
+        if (corr) {
+            reduce_warps(part, pitch, NQ, tot);
+            __syncthreads();
+#pragma unroll
+            for (int nt = 0; nt < NQ; ++nt) {
+                const float4 R = *reinterpret_cast<const float4*>(tot + (nt * 32 + lane) * 4);
+                RA[nt] = frag_a(R.x, R.z, R.y, R.w);
+            }
+        }
+        float* Bi = M.B + (int64_t)i * mp * np + b0 + c2;
+#pragma unroll
+        for (int j = 0; j < GPW; ++j) {
+            const int G8 = w + NW * j;
+            if (G8 < ng) {
+                const int ra = 8 * G8 + t, rb = ra + 4;
+                float c[4] = {0.f, 0.f, 0.f, 0.f};
+                float2 x0 = make_float2(0.f, 0.f), x1 = make_float2(0.f, 0.f);
+                if (corr) {
+#pragma unroll
+                    for (int nt = 0; nt < NQ; ++nt) mma3(c, RA[nt], pcb[j][nt]);
+                    x0 = *reinterpret_cast<const float2*>(S + sw_elem(ra, c2));
+                    x1 = *reinterpret_cast<const float2*>(S + sw_elem(rb, c2));
+                }
+                float2 g0, g1;
+                if (trans) {
+                    g0 = make_float2(static_cast<float>(Gs[c2 * gpt + ra]), static_cast<float>(Gs[(c2 + 1) * gpt + ra]));
+                    g1 = make_float2(static_cast<float>(Gs[c2 * gpt + rb]), static_cast<float>(Gs[(c2 + 1) * gpt + rb]));
+                } else {
+                    g0 = GradPair<GT>::row(Gs, ra, c2);
+                    g1 = GradPair<GT>::row(Gs, rb, c2);
+                }
+                const float m0 = g0.x + (x0.x - c[0]);       // M = G + E, E = B - P_prev R
+                const float m1 = g0.y + (x0.y - c[2]);
+                const float m2 = g1.x + (x1.x - c[1]);
+                const float m3 = g1.y + (x1.y - c[3]);
+                if (M.write_B && colok) {
+                    if (ra < mp) __stcs(reinterpret_cast<float2*>(Bi + (int64_t)ra * np), make_float2(m0, m1));
+                    if (rb < mp) __stcs(reinterpret_cast<float2*>(Bi + (int64_t)rb * np), make_float2(m2, m3));
+                }
+                acc[j][0] += m0; acc[j][1] += m1; acc[j][2] += m2; acc[j][3] += m3;
+            }
+        }
     }
     cp_async_wait<0>();
     const float invN = 1.0f / static_cast<float>(N);
+    float* Mb = M.Mbar + b0 + c2;
 #pragma unroll
-    for (int u = 0; u < 2; ++u)
+    for (int j = 0; j < GPW; ++j) {
+        const int G8 = w + NW * j;
 #pragma unroll
-        for (int nt = 0; nt < 2; ++nt)
-#pragma unroll
-            for (int e = 0; e < 4; ++e) acc[u][nt][e] *= invN;
-#pragma unroll
-    for (int u = 0; u < 2; ++u) {
-        const int mt = w + u * NW;
-#pragma unroll
-        for (int h = 0; h < 2; ++h) {
-            const int a = mt * 16 + gg + 8 * h;
-            if (mt < ntiles_m && a < mp)
-#pragma unroll
-                for (int nt = 0; nt < 2; ++nt)
-                    if (colv[nt] < np)
-                        *reinterpret_cast<float2*>(M.Mbar + rowoff[u][h] + colv[nt]) =
-                            make_float2(acc[u][nt][2 * h], acc[u][nt][2 * h + 1]);
+        for (int e = 0; e < 4; ++e) acc[j][e] *= invN;
+        const int ra = 8 * G8 + t, rb = ra + 4;
+        if (G8 < ng && colok) {
+            if (ra < mp) *reinterpret_cast<float2*>(Mb + (int64_t)ra * np) = make_float2(acc[j][0], acc[j][1]);
+            if (rb < mp) *reinterpret_cast<float2*>(Mb + (int64_t)rb * np) = make_float2(acc[j][2], acc[j][3]);
         }
     }
-    if (!M.lam) return;
+    if (!KT) return;
 
     // ---- truncated-basis Approx-Top-r partial sums: (Mbar - Yt (Y^T Mbar)) v_j ------------------
-    const int k = M.k, KQ = up8(k), tp = transposed_pitch(mp);
-    float* Ms = reinterpret_cast<float*>(ring);              // Mbar strip (swizzled, rows >= mp zero)
-    float* Wp = reinterpret_cast<float*>(ring + stage);      // warp partials of W^T (ring slots 1-2)
-    float* Ws = Rs;                                          // W = Y^T Mbar_strip (KQ x RP)
+    __syncthreads();                                         // Y, Yt landed for every thread
+    const float* YF = reinterpret_cast<const float*>(ring + (size_t)(N % 3) * stage);
+    const float* YtF = reinterpret_cast<const float*>(ring + (size_t)((N + 1) % 3) * stage);
+    {
+        float d[4][4];
 #pragma unroll
-    for (int u = 0; u < 2; ++u) {
-        const int mt = w + u * NW;
-        if (mt < ntiles_m) {
+        for (int nt = 0; nt < 4; ++nt)
 #pragma unroll
-            for (int h = 0; h < 2; ++h) {
-                const int a = mt * 16 + gg + 8 * h;
+            for (int e = 0; e < 4; ++e) d[nt][e] = 0.f;
 #pragma unroll
-                for (int nt = 0; nt < 2; ++nt)
-                    *reinterpret_cast<float2*>(Ms + a * SW + soff[nt]) =
-                        colv[nt] < np && a < mp ? make_float2(acc[u][nt][2 * h], acc[u][nt][2 * h + 1])
-                                                : make_float2(0.f, 0.f);
+        for (int j = 0; j < GPW; ++j) {
+            const int G8 = w + NW * j;
+            if (G8 < ng) {
+                const FragA A = frag_a(acc[j][0], acc[j][1], acc[j][2], acc[j][3]);
+#pragma unroll
+                for (int nt = 0; nt < 4; ++nt)
+                    if (nt < KT) {
+                        const float2 y = *reinterpret_cast<const float2*>(YF + (G8 * KT + nt) * 64 + 2 * lane);
+                        mma3(d[nt], A, frag_b(y.x, y.y));
+                    }
             }
         }
+#pragma unroll
+        for (int nt = 0; nt < 4; ++nt)
+            if (nt < KT)
+                *reinterpret_cast<float4*>(part + w * pitch + (nt * 32 + lane) * 4) =
+                    make_float4(d[nt][0], d[nt][1], d[nt][2], d[nt][3]);
     }
     __syncthreads();
-    rt_product<true>(Ms, M.YT, tp, mp16, KQ, Wp, Ws);        // W^T = Mbar_strip^T Y
-    float rows[2][2] = {{0.f, 0.f}, {0.f, 0.f}};
+    reduce_warps(part, pitch, KT, tot);                      // W^T = Mbar_strip^T Y
+    __syncthreads();
+    FragA WA[4];
 #pragma unroll
-    for (int u = 0; u < 2; ++u) {
-        const int mt = w + u * NW;
-        const int m0 = mt * 16;
-        float c[2][4] = {};
-        if (mt < ntiles_m) c_product<true>(M.YtT, tp, Ws, KQ, m0, c);
+    for (int nt = 0; nt < 4; ++nt)
+        if (nt < KT) {
+            const float4 W = *reinterpret_cast<const float4*>(tot + (nt * 32 + lane) * 4);
+            WA[nt] = frag_a(W.x, W.z, W.y, W.w);
+        }
+    const bool odd = (gg & 1) != 0;
 #pragma unroll
-        for (int h = 0; h < 2; ++h) {
-            const int a = m0 + gg + 8 * h;
-            // the 32 lanes draw the 32 distinct quads (row gg, quad lane & 3) of this row block;
-            // each lane then fetches the two values of its own columns
-            const float4 vq = gauss4(M.seed, M.t, static_cast<uint32_t>(a), static_cast<uint32_t>((b0 >> 2) + t),
-                                     kTagLambdaV);
+    for (int j = 0; j < GPW; ++j) {
+        const int G8 = w + NW * j;                           // warp-uniform: shuffles below are safe
+        if (G8 < ng) {
+            float c[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
-            for (int nt = 0; nt < 2; ++nt) {
-                const int src = (lane & ~3) | (nt * 2 + (t >> 1));
-                const float vx = __shfl_sync(0xffffffffu, vq.x, src), vy = __shfl_sync(0xffffffffu, vq.y, src);
-                const float vz = __shfl_sync(0xffffffffu, vq.z, src), vw = __shfl_sync(0xffffffffu, vq.w, src);
-                const bool hi = (t & 1) != 0;            // columns 2, 3 of the quad
-                const float v0 = hi ? vz : vx, v1 = hi ? vw : vy;
-                if (mt < ntiles_m && a < mp && colv[nt] < np) {
-                    const float2 mv = *reinterpret_cast<const float2*>(Ms + a * SW + soff[nt]);
-                    rows[u][h] += (mv.x - c[nt][2 * h]) * v0 + (mv.y - c[nt][2 * h + 1]) * v1;
+            for (int nt = 0; nt < 4; ++nt)
+                if (nt < KT) {
+                    const float2 y = *reinterpret_cast<const float2*>(YtF + (G8 * KT + nt) * 64 + 2 * lane);
+                    mma3(c, WA[nt], frag_b(y.x, y.y));
                 }
+            const float d0 = acc[j][0] - c[0], d1 = acc[j][1] - c[2];
+            const float d2 = acc[j][2] - c[1], d3 = acc[j][3] - c[3];
+            // v_j: the 32 lanes draw the 32 quads (row, 4 columns) of the group once each: lane
+            // (g, t) draws row t + 4 (g % 2), quad g / 2, keeps the half it needs and trades the
+            // other half with lane g ^ 1
+            const int ra = 8 * G8 + t;
+            const float4 vq = gauss4(M.seed, M.t, static_cast<uint32_t>(ra + 4 * (gg & 1)),
+                                     static_cast<uint32_t>((b0 >> 2) + (gg >> 1)), kTagLambdaV);
+            const float q0 = __shfl_xor_sync(0xffffffffu, odd ? vq.x : vq.z, 4);
+            const float q1 = __shfl_xor_sync(0xffffffffu, odd ? vq.y : vq.w, 4);
+            const float v0 = odd ? q0 : vq.x, v1 = odd ? q1 : vq.y;     // row t
+            const float v2 = odd ? vq.z : q0, v3 = odd ? vq.w : q1;     // row t + 4
+            float pa = colok ? d0 * v0 + d1 * v1 : 0.f;
+            float pb = colok ? d2 * v2 + d3 * v3 : 0.f;
+#pragma unroll
+            for (int x = 4; x < 32; x <<= 1) {
+                pa += __shfl_xor_sync(0xffffffffu, pa, x);
+                pb += __shfl_xor_sync(0xffffffffu, pb, x);
+            }
+            if (gg == 0) {
+                if (ra < mp) M.part[(int64_t)s * mp + ra] = pa;
+                if (ra + 4 < mp) M.part[(int64_t)s * mp + ra + 4] = pb;
             }
         }
     }
-    // the 4 lanes of a group (t = 0..3) hold one row's partial sums
-#pragma unroll
-    for (int u = 0; u < 2; ++u)
-#pragma unroll
-        for (int h = 0; h < 2; ++h) {
-            float v = rows[u][h];
-            v += __shfl_xor_sync(0xffffffffu, v, 1);
-            v += __shfl_xor_sync(0xffffffffu, v, 2);
-            const int mt = w + u * NW;
-            const int a = mt * 16 + gg + 8 * h;
-            if (t == 0 && mt < ntiles_m && a < mp) M.part[(int64_t)s * mp + a] = v;
-        }
+}
+
+// dst = src (rows x cols, row-major, ld) in fragment order, up8(rows) x up8(cols) floats:
+// block (group G8, n-tile nt) holds 64 floats, lane L's pair at 2L, 2L + 1.
+//   form 0 (B fragment of X^T Y):  src(8 G8 + t, 8 nt + g), src(8 G8 + t + 4, 8 nt + g)
+//   form 1 (B fragment of W Y^T): src(8 G8 + row, 8 nt + 2t), src(8 G8 + row, 8 nt + 2t + 1),
+//                                  row = g / 2 + 4 (g % 2)
+__global__ void pack_frag_kernel(float* dst, const float* src, int rows, int cols, int ld, int form) {
+    const int KT = up8(cols) >> 3;
+    const int total = up8(rows) * KT * 8;
+    for (int idx = blockIdx.x * blockDim.x + threadIdx.x; idx < total; idx += gridDim.x * blockDim.x) {
+        const int blk = idx >> 6, L = (idx >> 1) & 31, e = idx & 1;
+        const int G8 = blk / KT, nt = blk % KT, g = L >> 2, t = L & 3;
+        int row, col;
+        if (form == 0) { row = 8 * G8 + t + 4 * e; col = 8 * nt + g; }
+        else { row = 8 * G8 + (g >> 1) + 4 * (g & 1); col = 8 * nt + 2 * t + e; }
+        dst[idx] = row < rows && col < cols ? src[(int64_t)row * ld + col] : 0.f;
+    }
 }
 
 }  // namespace
 
+int mma_stream_nq(int r) { return (r + 7) / 8; }
+
 bool mma_stream_eligible(int mp, int np, int r, int k, int lam, int transposed, int gsize) {
-    if (mp > kMmaMaxRows || r > 16 || (lam && (k > 32 || k % 8 != 0))) return false;
-    if (np % 4 != 0 || (transposed && mp % 8 != 0)) return false;   // 16-byte chunks of G rows
+    const int NQ = mma_stream_nq(r), ng = up8(mp) / 8;
+    if (NQ < 1 || NQ > 2 || (ng + NW - 1) / NW > 4 / NQ) return false;   // groups per warp
+    if (lam && (k < 1 || k > 32)) return false;
+    if (np % 4 != 0 || (transposed && mp % 8 != 0)) return false;      // 16-byte chunks of G rows
     return mma_stream_smem_bytes(mp, r, k, lam, gsize, transposed) <= 227 * 1024;
 }
 
 size_t mma_stream_smem_bytes(int mp, int r, int k, int lam, int gsize, int transposed) {
-    const int mp16 = up16(mp), RQ = up8(r), pt = mma_pt(mp), KQ = up8(k);
+    const int mp16 = up16(mp), NQ = mma_stream_nq(r), KT = lam ? up8(k) / 8 : 0;
     const size_t stage = stage_b_bytes(mp16) + stage_g_bytes(mp16, gsize, transposed);
-    if (lam && (size_t)NW * KQ * SW * 4 > 2 * stage) return ~size_t(0);   // W partials use ring slots 1-2
-    return 3 * stage + a16((size_t)RQ * pt * 4) + a16((size_t)32 * RP * 4) + a16((size_t)NW * RQ * SW * 4);
+    if (lam && (size_t)up8(mp) * KT * 8 * 4 > stage) return ~size_t(0);   // Y, Yt use ring slots
+    const int NT = NQ > KT ? NQ : KT;
+    return 3 * stage + (size_t)NW * part_pitch(NT) * 4 + (size_t)NT * 128 * 4;
 }
 
-template <typename GT>
+template <typename GT, int NQ>
 static cudaError_t launch_mma(const StreamGroup& g, size_t smem, cudaStream_t st) {
     static bool set = false;
     if (!set) {
-        cudaError_t e = cudaFuncSetAttribute(stream_mma_kernel<GT>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+        cudaError_t e = cudaFuncSetAttribute(stream_mma_kernel<GT, NQ>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                              227 * 1024);
         if (e != cudaSuccess) return e;
         set = true;
     }
-    stream_mma_kernel<GT><<<g.total_strips, T, smem, st>>>(g);
+    stream_mma_kernel<GT, NQ><<<g.total_strips, T, smem, st>>>(g);
     return cudaGetLastError();
 }
 
 cudaError_t stream_group_mma(const StreamGroup& g, size_t smem, cudaStream_t st) {
     if (g.total_strips <= 0) return cudaSuccess;
-    return g.grad_dtype == GLR_BF16 ? launch_mma<__nv_bfloat16>(g, smem, st) : launch_mma<float>(g, smem, st);
+    const int NQ = mma_stream_nq(g.mat[0].r);
+    for (int i = 1; i < g.nmat; ++i)
+        if (mma_stream_nq(g.mat[i].r) != NQ) return cudaErrorInvalidValue;
+    if (g.grad_dtype == GLR_BF16)
+        return NQ == 1 ? launch_mma<__nv_bfloat16, 1>(g, smem, st) : launch_mma<__nv_bfloat16, 2>(g, smem, st);
+    return NQ == 1 ? launch_mma<float, 1>(g, smem, st) : launch_mma<float, 2>(g, smem, st);
+}
+
+cudaError_t pack_frag(float* dst, const float* src, int rows, int cols, int ld, int form, cudaStream_t st) {
+    const int total = up8(rows) * up8(cols);
+    if (total <= 0) return cudaSuccess;
+    pack_frag_kernel<<<(total + 255) / 256, 256, 0, st>>>(dst, src, rows, cols, ld, form);
+    return cudaGetLastError();
 }
 
 }  // namespace glr
