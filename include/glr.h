@@ -50,7 +50,7 @@ extern "C" {
 #define GLR_ECUDA      -3   /* a CUDA runtime call or kernel launch failed                 */
 #define GLR_ENUMERIC   -4   /* the refresh could not orthonormalise its basis              */
 #define GLR_ENONFINITE -5   /* reserved: non-finite values detected                        */
-#define GLR_ETIMEOUT   -6   /* reserved: a bounded device-side wait gave up                */
+#define GLR_ETIMEOUT   -6   /* a bounded device-side wait gave up (reported by glr_get_stats) */
 
 /* ---- enumerations -------------------------------------------------------------------- */
 #define GLR_ALG3 0   /* refresh step: uncompressed mean, E reset to 0 (Algorithm 3)          */
@@ -175,7 +175,10 @@ int glr_refresh(glr_handle* h);
 
 /* ---- introspection (tests, debugging) ------------------------------------------------- */
 
-/* Counters (see glr_stats); host call, no synchronisation.                               */
+/* Counters (see glr_stats).  Reads the handle's device flags with a blocking copy, so it
+ * waits for work already queued on the device.  Returns GLR_ETIMEOUT (with out filled) when a
+ * bounded wait inside a compose kernel of this handle's launches has given up since creation:
+ * the results of those steps are not valid.                                               */
 int glr_get_stats(const glr_handle* h, glr_stats* out);
 
 /* Message of the last failure on h (or of the last failed glr_create when h is NULL);

@@ -31,13 +31,18 @@ struct glr_handle {
     int ntiles = 0;                 // lambda tiles of the first-path kernel (64 columns)
     int fused = 0, BN = 0, nstrips = 0;   // fused strip kernels: strip width, strips per matrix
     int mma = 0;                          // compose on the tensor cores (k_mma.cu)
+    int tma = 0;                          // ... with its ring filled by tile copies
+    CUtensorMap Bmap{};                   // tile-copy descriptor of B (n' x m' x N)
+    struct GMap { const void* ptr; CUtensorMap map; };
+    std::vector<GMap> gmaps;              // per node: the descriptors of its last two gradient buffers
     float *Mo = nullptr, *Vo = nullptr;
     float *U = nullptr, *Hbuf = nullptr, *Vbuf = nullptr, *evals = nullptr, *evals_sorted = nullptr;
     float *Q = nullptr, *Qn = nullptr, *Y = nullptr, *Yt = nullptr, *T = nullptr, *dsign = nullptr;
     float *Wbar = nullptr, *Z = nullptr, *Hk = nullptr, *Vk = nullptr, *gram = nullptr, *scratch = nullptr;
     float *YT = nullptr, *YtT = nullptr;   // k x transposed_pitch(m') copies of Y and Yt for the fused kernel
     float *YF = nullptr, *YtF = nullptr;   // Y and Yt in fragment order for the tensor-core kernel
-    int* dflags = nullptr;   // [0] Cholesky restarts, [1] Jacobi sweeps of the last refresh
+    int* dflags = nullptr;   // [0] Cholesky restarts, [1] Jacobi sweeps of the last refresh,
+                             // [2] bounded device waits of the compose kernel that gave up
     float* gemm_ws = nullptr;   // split-K partial tiles of the refresh GEMMs
     cudaStream_t rstream = nullptr;            // side stream of this handle's refresh
     cudaEvent_t rfork = nullptr, rdone = nullptr;
@@ -138,6 +143,49 @@ int alloc(glr_handle* h, T** p, size_t count) {
 void free_all(glr_handle* h) {
     for (void* p : h->allocs) cudaFree(p);
     h->allocs.clear();
+}
+
+// cuTensorMapEncodeTiled from the driver, looked up once through the runtime (no libcuda link).
+using EncodeTiledFn = CUresult (*)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
+                                   const cuuint64_t*, const cuuint32_t*, const cuuint32_t*, CUtensorMapInterleave,
+                                   CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+EncodeTiledFn encode_fn() {
+    static EncodeTiledFn fn = [] {
+        void* p = nullptr;
+        cudaDriverEntryPointQueryResult q{};
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) != cudaSuccess ||
+            q != cudaDriverEntryPointSuccess)
+            p = nullptr;
+        return reinterpret_cast<EncodeTiledFn>(p);
+    }();
+    return fn;
+}
+
+// Row-major (rows x cols) matrices, `depth` of them back to back, read in boxes of 16 columns x
+// mma_tma_box_rows(rows) rows; fp32 with the 64-byte swizzle, bf16 with the 32-byte one.
+bool encode_strip_map(CUtensorMap* map, const void* base, int rows, int cols, int depth, int gsize) {
+    EncodeTiledFn fn = encode_fn();
+    if (!fn) return false;
+    const cuuint64_t dims[3] = {(cuuint64_t)cols, (cuuint64_t)rows, (cuuint64_t)depth};
+    const cuuint64_t strides[2] = {(cuuint64_t)cols * gsize, (cuuint64_t)cols * gsize * rows};
+    const cuuint32_t box[3] = {16, (cuuint32_t)mma_tma_box_rows(rows), 1};
+    const cuuint32_t estr[3] = {1, 1, 1};
+    return fn(map, gsize == 2 ? CU_TENSOR_MAP_DATA_TYPE_BFLOAT16 : CU_TENSOR_MAP_DATA_TYPE_FLOAT32, depth > 1 ? 3 : 2,
+              const_cast<void*>(base), dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+              gsize == 2 ? CU_TENSOR_MAP_SWIZZLE_32B : CU_TENSOR_MAP_SWIZZLE_64B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+              CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+// The descriptor of node i's gradient buffer, re-encoded only when the buffer changes.
+bool gradient_map(glr_handle* h, int i, const void* ptr, CUtensorMap* out) {
+    glr_handle::GMap* slots = &h->gmaps[2 * (size_t)i];
+    for (int q = 0; q < 2; ++q)
+        if (slots[q].ptr == ptr) { *out = slots[q].map; return true; }
+    slots[1] = slots[0];
+    if (!encode_strip_map(&slots[0].map, ptr, h->mp, h->np, 1, (int)h->gsize)) { slots[0].ptr = nullptr; return false; }
+    slots[0].ptr = ptr;
+    *out = slots[0].map;
+    return true;
 }
 
 thread_local float* g_ws = nullptr;   // split-K workspace of the handle being stepped
@@ -367,6 +415,11 @@ int glr_create(int64_t m, int64_t n, int32_t r, int32_t N, const glr_schedule* s
         delete h;
         return GLR_ECUDA;
     }
+    if (h->mma && mma_stream_tma_eligible((int)mp, (int)np, r, k, exact ? 0 : 1, h->transposed, (int)h->gsize) &&
+        encode_strip_map(&h->Bmap, h->B, (int)mp, (int)np, N, 4)) {
+        h->tma = 1;
+        h->gmaps.assign(2 * (size_t)N, glr_handle::GMap{nullptr, CUtensorMap{}});
+    }
     h->iotaJ.resize(r);
     for (int q = 0; q < r; ++q) h->iotaJ[q] = q;
     *out = h;
@@ -451,17 +504,20 @@ bool heavier(const StepPlan* a, const StepPlan* b) {
 int compose_fused(std::vector<StepPlan*>& plans, cudaStream_t st) {
     std::vector<StepPlan*> todo(plans);
     std::stable_sort(todo.begin(), todo.end(), heavier);
+    static thread_local TmaMaps maps;      // ~20 KiB: kept off the stack
     while (!todo.empty()) {
-        const int BN = todo.front()->h->BN, dt = todo.front()->h->s.grad_dtype, mma = todo.front()->h->mma;
+        glr_handle* f = todo.front()->h;
+        const int BN = f->BN, dt = f->s.grad_dtype, mma = f->mma, tma = f->tma;
+        const int gmax = tma ? kTmaGMax : kGroupPtrs;
         StreamGroup g{};
-        g.BN = BN; g.grad_dtype = dt;
+        g.BN = BN; g.grad_dtype = dt; g.err = f->dflags + 2;
         size_t smem = 0;
         std::vector<StepPlan*> rest;
         for (StepPlan* p : todo) {
             glr_handle* h = p->h;
-            if (h->BN != BN || h->s.grad_dtype != dt || h->mma != mma ||
-                (mma && mma_stream_nq(h->r) != mma_stream_nq(todo.front()->h->r)) || g.nmat == kGroupMax ||
-                g.nmat + 0 >= kGroupMax || (int)(g.nmat ? g.mat[g.nmat - 1].g_off + g.mat[g.nmat - 1].N : 0) + h->N > kGroupPtrs) {
+            const int used = g.nmat ? g.mat[g.nmat - 1].g_off + g.mat[g.nmat - 1].N : 0;
+            if (h->BN != BN || h->s.grad_dtype != dt || h->mma != mma || h->tma != tma ||
+                (mma && mma_stream_nq(h->r) != mma_stream_nq(f->r)) || g.nmat == kGroupMax || used + h->N > gmax) {
                 rest.push_back(p);
                 continue;
             }
@@ -469,21 +525,28 @@ int compose_fused(std::vector<StepPlan*>& plans, cudaStream_t st) {
             M.mp = h->mp; M.np = h->np; M.N = h->N; M.r = h->r; M.k = h->k;
             M.transposed = h->transposed; M.e_zero = h->e_zero ? 1 : 0; M.write_B = p->warm ? 0 : 1;
             M.lam = p->lam_fused ? 1 : 0;
-            M.g_off = g.nmat ? g.mat[g.nmat - 1].g_off + g.mat[g.nmat - 1].N : 0;
+            M.g_off = used;
             M.strip0 = g.total_strips; M.nstrips = h->nstrips;
             M.B = h->B; M.Pprev = h->Pprev; M.Mbar = h->Mbar;
             M.YT = h->YT; M.YtT = h->YtT; M.YF = h->YF; M.YtF = h->YtF; M.part = h->lam_part;
             M.seed = h->s.seed; M.t = static_cast<uint32_t>(h->t);
             for (int i = 0; i < h->N; ++i) g.G[M.g_off + i] = p->G[i];
+            if (tma) {
+                maps.B[g.nmat] = h->Bmap;
+                for (int i = 0; i < h->N; ++i)
+                    if (!gradient_map(h, i, p->G[i], &maps.G[M.g_off + i]))
+                        return fail(h, GLR_ECUDA, "could not describe gradient %s for tile copies",
+                                    std::to_string(i).c_str());
+            }
             g.total_strips += h->nstrips;
-            smem = std::max(smem, mma ? mma_stream_smem_bytes(h->mp, h->r, h->k, h->exact ? 0 : 1, (int)h->gsize, h->transposed)
+            smem = std::max(smem, mma ? mma_stream_smem_bytes(h->mp, h->r, h->k, h->exact ? 0 : 1, (int)h->gsize,
+                                                              h->transposed, tma)
                                       : stream_smem_bytes(h->mp, h->r, h->k, BN, (int)h->gsize, h->transposed, M.lam));
             g.nmat++;
         }
-        glr_handle* h0 = todo.front()->h;
         {
-            PhaseScope ps(h0, GLR_PH_COMPOSE, st);
-            GLR_LAUNCH(h0, 1, mma ? stream_group_mma(g, smem, st) : stream_group(g, smem, st));
+            PhaseScope ps(f, GLR_PH_COMPOSE, st);
+            GLR_LAUNCH(f, 1, mma ? stream_group_mma(g, tma ? &maps : nullptr, smem, st) : stream_group(g, smem, st));
         }
         todo.swap(rest);
     }
@@ -726,7 +789,7 @@ int glr_get_stats(const glr_handle* h, glr_stats* out) {
     cudaMemcpy(flags, h->dflags, sizeof(flags), cudaMemcpyDeviceToHost);
     out->last_refresh_sweeps = flags[1];
     out->launches = h->launches;
-    return GLR_OK;
+    return flags[2] ? GLR_ETIMEOUT : GLR_OK;
 }
 
 const char* glr_last_error(const glr_handle* h) { return h ? h->err.c_str() : g_create_err.c_str(); }

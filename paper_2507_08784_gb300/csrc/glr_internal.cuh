@@ -1,6 +1,7 @@
 // Internal declarations shared by the CUDA translation units of libglr.so.
 #pragma once
 
+#include <cuda.h>
 #include <cuda_runtime.h>
 #include <cuda_bf16.h>
 #include <stdint.h>
@@ -200,8 +201,17 @@ struct StreamMat {
 };
 struct StreamGroup {
     int nmat, grad_dtype, total_strips, BN;
+    int* err;                               // bounded device waits that gave up are counted here
     StreamMat mat[kGroupMax];
     const void* G[kGroupPtrs];
+};
+// Tile-copy descriptors of the tensor-core K1 launch: B of each matrix (3-D: n' x m' x N) and
+// each node gradient (2-D: n' x m'), boxes of 16 columns x mma_tma_box_rows(m') rows.  Passed
+// by value as a kernel parameter (with StreamGroup under the 32 KiB parameter limit).
+constexpr int kTmaGMax = 128;
+struct TmaMaps {
+    CUtensorMap B[kGroupMax];
+    CUtensorMap G[kTmaGMax];
 };
 // K1 fused: per strip and node, R = Pprev^T B_i (deferred error), M_i = G_i + B_i - Pprev R,
 // B_i <- M_i, Mbar; with lam = 1 also W = Y^T Mbar_strip and the lambda partial sums of
@@ -213,12 +223,15 @@ size_t stream_smem_bytes(int mp, int r, int k, int BN, int gsize, int transposed
 __host__ __device__ __forceinline__ int transposed_pitch(int mp) { return ((mp + 15) & ~15) + 4; }
 // K1 with its rank-r products on the tensor cores (3xTF32 mma.sync): strips of 16 columns,
 // m' <= 512 for r <= 8 and m' <= 256 for r <= 16, truncated basis k <= 32.  One launch takes
-// matrices of one mma_stream_nq(r) only.
+// matrices of one mma_stream_nq(r) only.  With `maps` the ring is filled by tile copies (G read
+// in its stored orientation, n' x gsize a multiple of 16 bytes), else by cp.async.
 constexpr int kMmaStrip = 16;
 int mma_stream_nq(int r);
 bool mma_stream_eligible(int mp, int np, int r, int k, int lam, int transposed, int gsize);
-size_t mma_stream_smem_bytes(int mp, int r, int k, int lam, int gsize, int transposed);
-cudaError_t stream_group_mma(const StreamGroup& g, size_t smem_bytes, cudaStream_t st);
+bool mma_stream_tma_eligible(int mp, int np, int r, int k, int lam, int transposed, int gsize);
+size_t mma_stream_smem_bytes(int mp, int r, int k, int lam, int gsize, int transposed, int tma);
+int mma_tma_box_rows(int mp);
+cudaError_t stream_group_mma(const StreamGroup& g, const TmaMaps* maps, size_t smem_bytes, cudaStream_t st);
 // src (rows x cols, row-major, leading dimension ld) in the tensor-core kernel's fragment order
 // (up8(rows) x up8(cols) floats, zero-padded); form 0 for Y, form 1 for Yt.
 cudaError_t pack_frag(float* dst, const float* src, int rows, int cols, int ld, int form, cudaStream_t st);

@@ -1,13 +1,16 @@
 // K1 on the tensor cores: the fused compose pass with its two rank-r products done by warp-level
-// TF32 MMA (mma.sync m16n8k8) in the 3xTF32 form (each fp32 operand x is split into
-// x_hi = tf32(x) and x_lo = tf32(x - x_hi); a*b ~ a_hi b_hi + a_hi b_lo + a_lo b_hi, accumulated in
-// fp32, which keeps fp32-level accuracy).  The products are tiny (K or N = r), so the tensor pipe
-// is far from busy: the point is to replace ~2r FFMA (plus operand loads and index arithmetic)
-// per node-element with a few MMA instructions per warp.
+// TF32 MMA (mma.sync m16n8k8) in the 3xTF32 form (each fp32 operand x is split into x_hi and
+// x_lo; a*b ~ a_hi b_hi + a_hi b_lo + a_lo b_hi, accumulated in fp32, which keeps fp32-level
+// accuracy).  The products are tiny (K or N = r), so the tensor pipe is far from busy: the point
+// is to replace ~2r FFMA (plus operand loads and index arithmetic) per node-element with a few
+// MMA instructions per warp.
 //
 // Per CTA: one strip of 16 columns x all m' (<= 512) rows of one matrix; 16 warps.  A 3-slot
-// cp.async ring holds node i's B and G strips while nodes i+1 and i+2 are in flight; after the
-// last node the two free slots receive Y and Yt for the truncated-basis lambda epilogue.
+// ring holds node i's B and G strips while nodes i+1 and i+2 are in flight; after the last node
+// the two free slots receive Y and Yt for the truncated-basis lambda epilogue.  The ring is
+// filled by the Tensor Memory Accelerator (one thread issues a 2-D/3-D tile copy per operand and
+// node, completion counted on a per-slot mbarrier) when G is read in its stored orientation, and
+// by per-thread 16-byte cp.async otherwise (G read transposed, m > n).
 //   node i:  R_i^T (16 x r) = B_i,strip^T P_prev        K = m' split over the warps
 //            C (m' x 16)    = P_prev R_i                 K = r
 //            M_i = G_i + (B_i - C);  B_i <- M_i;  acc += M_i
@@ -19,18 +22,23 @@
 //   B (8 x 8):  b0 (t, g), b1 (t + 4, g)
 //   C (16 x 8): c0 (g, 2t), c1 (g, 2t + 1), c2 (g + 8, 2t), c3 (g + 8, 2t + 1)
 // Both products are computed transposed, with M = the strip's 16 columns, and their indices are
-// relabelled so that one lane owns the same four elements of every operand: in each 8-row group
-// the lane owns rows t, t + 4 and strip columns 2g, 2g + 1,
-//   e0 = (t, 2g)   e1 = (t, 2g + 1)   e2 = (t + 4, 2g)   e3 = (t + 4, 2g + 1).
+// relabelled so that one lane owns the same four elements of every operand.  With
+// rho(t) = (t % 2) + 4 (t / 2), in each 8-row group the lane owns rows rho(t), rho(t) + 2 and
+// strip columns 2g, 2g + 1:
+//   e0 = (rho, 2g)   e1 = (rho, 2g + 1)   e2 = (rho + 2, 2g)   e3 = (rho + 2, 2g + 1).
 //   R^T = B^T P   (M = columns, K = rows, N = q): M index m <-> column 2 (m % 8) + m / 8, K index
-//                 k <-> row k.  A fragment = (e0, e1, e2, e3); B fragment P(t, q), P(t + 4, q).
-//   C^T = R^T P^T (M = columns, K = q, N = rows): N index n <-> row n / 2 + 4 (n % 2), K index k
-//                 <-> q = 2 (k % 4) + k / 4.  C fragment = (e0, e2, e1, e3); its A fragment is
-//                 the R^T C fragment in the order (c0, c2, c1, c3); B fragment P(row, 2t),
-//                 P(row, 2t + 1) with row = g / 2 + 4 (g % 2).
-// Sums over K are order-free, so the relabelling changes nothing but the rounding order.  B is
+//                 t <-> row rho(t), t + 4 <-> rho(t) + 2.  A fragment = (e0, e1, e2, e3); B
+//                 fragment P(rho, q), P(rho + 2, q).
+//   C^T = R^T P^T (M = columns, K = q, N = rows): N index n <-> row prow(n) = rho(n / 2) +
+//                 2 (n % 2), K index k <-> q = 2 (k % 4) + k / 4.  C fragment = (e0, e2, e1, e3);
+//                 its A fragment is the R^T C fragment in the order (c0, c2, c1, c3); B fragment
+//                 P(prow(g), 2t), P(prow(g), 2t + 1).
+// Sums over K are order-free, so the relabelling changes nothing but the rounding order.  The
+// row labels make the lane's 8-byte loads from the 64-byte-swizzled strips conflict-free.  B is
 // read from shared memory once per node for both products, P's fragments are loaded once per
 // strip into registers, and no operand is re-staged between the products.
+#include <cuda.h>
+
 #include "glr_internal.cuh"
 
 namespace glr {
@@ -40,15 +48,15 @@ namespace {
 constexpr int T = kMmaThreads;         // 512 threads = 16 warps
 constexpr int NW = T / 32;
 constexpr int SW = 16;                 // strip width (columns)
+constexpr int GPW_MAX = 64 / NW;       // row groups per warp for r <= 8 (m' <= 512)
 
-__device__ __forceinline__ uint32_t to_tf32(float x) {
-    uint32_t r;
-    asm("cvt.rna.tf32.f32 %0, %1;" : "=r"(r) : "f"(x));
-    return r;
-}
+// x ~ hi + lo with hi = x rounded to the nearest TF32 value (ties away from zero: add half a unit
+// of the 13 dropped mantissa bits, then clear them) and lo = the TF32 truncation of the exact
+// remainder x - hi; |x - hi| <= 2^-11 |x|, so truncating it costs at most 2^-21 |x|.  Integer
+// operations on the bit pattern; finite inputs below the largest binade.
 __device__ __forceinline__ void split2(float x, uint32_t& hi, uint32_t& lo) {
-    hi = to_tf32(x);
-    lo = to_tf32(x - __uint_as_float(hi));
+    hi = (__float_as_uint(x) + 0x1000u) & 0xffffe000u;
+    lo = __float_as_uint(x - __uint_as_float(hi)) & 0xffffe000u;
 }
 __device__ __forceinline__ void mma_tf32(float (&d)[4], const uint32_t (&a)[4], const uint32_t (&b)[2]) {
     asm volatile("mma.sync.aligned.m16n8k8.row.col.f32.tf32.tf32.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, "
@@ -76,9 +84,8 @@ __device__ __forceinline__ void mma3(float (&d)[4], const FragA& a, const FragB&
     mma_tf32(d, a.hi, b.hi);
 }
 
-__device__ __forceinline__ void cp_async16(void* smem, const void* gmem) {
-    const unsigned s = static_cast<unsigned>(__cvta_generic_to_shared(smem));
-    asm volatile("cp.async.cg.shared.global [%0], [%1], 16;\n" ::"r"(s), "l"(gmem) : "memory");
+__device__ __forceinline__ void cp_async16(uint32_t saddr, const void* gmem) {
+    asm volatile("cp.async.cg.shared.global [%0], [%1], 16;\n" ::"r"(saddr), "l"(gmem) : "memory");
 }
 __device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;\n" ::: "memory"); }
 template <int Pending>
@@ -86,30 +93,78 @@ __device__ __forceinline__ void cp_async_wait() {
     asm volatile("cp.async.wait_group %0;\n" ::"n"(Pending) : "memory");
 }
 
+// ---- Tensor Memory Accelerator and mbarrier ------------------------------------------------
+__device__ __forceinline__ void mbar_init(uint32_t bar, uint32_t count) {
+    asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(bar), "r"(count) : "memory");
+}
+__device__ __forceinline__ void mbar_expect_tx(uint32_t bar, uint32_t bytes) {
+    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar), "r"(bytes) : "memory");
+}
+// Waits for the phase of parity `parity` to complete.  Each poll lets the thread sleep until the
+// phase completes or a time hint (10 ms) passes, so waiting threads issue almost nothing; after
+// 100 polls (about a second) it gives up and returns false.
+__device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity) {
+    for (int it = 0; it < 100; ++it) {
+        uint32_t done;
+        asm volatile("{ .reg .pred p; mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2, %3; selp.u32 %0, 1, 0, p; }"
+                     : "=r"(done) : "r"(bar), "r"(parity), "r"(10000000u) : "memory");
+        if (done) return true;
+    }
+    return false;
+}
+__device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap* map, int x, int y, uint32_t bar) {
+    asm volatile("cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3}], [%4];"
+                 ::"r"(dst), "l"(map), "r"(x), "r"(y), "r"(bar) : "memory");
+}
+__device__ __forceinline__ void tma_load_3d(uint32_t dst, const CUtensorMap* map, int x, int y, int z, uint32_t bar) {
+    asm volatile("cp.async.bulk.tensor.3d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3, %4}], [%5];"
+                 ::"r"(dst), "l"(map), "r"(x), "r"(y), "r"(z), "r"(bar) : "memory");
+}
+__device__ __forceinline__ void bulk_load(uint32_t dst, const void* src, uint32_t bytes, uint32_t bar) {
+    asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];"
+                 ::"r"(dst), "l"(src), "r"(bytes), "r"(bar) : "memory");
+}
+
 __host__ __device__ __forceinline__ int up8(int x) { return (x + 7) & ~7; }
 __host__ __device__ __forceinline__ int up16(int x) { return (x + 15) & ~15; }
 __host__ __device__ __forceinline__ size_t a16(size_t x) { return (x + 15) & ~size_t(15); }
+__host__ __device__ __forceinline__ size_t a1k(size_t x) { return (x + 1023) & ~size_t(1023); }
 
-// Strip rows are 64 bytes = four 16-byte chunks.  fp32 strips (B, and G when it is fp32) store
-// chunk c of row a at position c ^ (2 * ((a >> 1) & 1)), which makes the 8-byte loads of a lane's
-// (row t or t + 4, columns 2g, 2g + 1) hit 32 distinct banks per half-warp.
-__device__ __forceinline__ int sw_elem(int a, int c) {
-    return a * SW + 4 * ((c >> 2) ^ (((a >> 1) & 1) << 1)) + (c & 3);
+// Strip layouts in shared memory (both staging paths write the same ones):
+//   fp32 strips (B, and G when it is fp32): 64-byte rows, 16-byte chunk c of row a at position
+//     c ^ ((a >> 1) & 3)  (the Tensor Memory Accelerator's 64-byte swizzle)
+//   bf16 G strips: 32-byte rows, chunk c of row a at c ^ ((a >> 2) & 1)  (its 32-byte swizzle)
+//   G read transposed (cp.async only): 16 rows (strip columns) of gpt elements.
+__device__ __forceinline__ int sw64(int a, int c) { return a * SW + 4 * ((c >> 2) ^ ((a >> 1) & 3)) + (c & 3); }
+__device__ __forceinline__ int sw32(int a, int c) { return a * SW + 8 * ((c >> 3) ^ ((a >> 2) & 1)) + (c & 7); }
+
+// Tile copies: up8(m') rows in nbox boxes of box_rows rows (a box has at most 256 rows).
+__host__ __device__ __forceinline__ int tma_nbox(int mp) { return (up8(mp) + 255) / 256; }
+__host__ __device__ __forceinline__ int tma_box_rows(int mp) {
+    const int nb = tma_nbox(mp);
+    return up8((up8(mp) + nb - 1) / nb);
 }
-
-// Ring stage layout: [B strip: mp16 x 16 fp32, swizzled][G strip: mp16 x 16 (gradient dtype),
-// or 16 x gpt when G is read transposed (m > n)].
-__host__ __device__ __forceinline__ size_t stage_b_bytes(int mp16) { return (size_t)mp16 * SW * 4; }
+// Rows held by a slot, and the slot's B and G regions (TMA regions start on 1024-byte bounds).
+__host__ __device__ __forceinline__ int slot_rows(int mp, bool tma) {
+    return tma ? tma_nbox(mp) * tma_box_rows(mp) : up16(mp);
+}
 __host__ __device__ __forceinline__ int g_tpitch(int mp16, int gsize) { return mp16 + 16 / gsize; }
-__host__ __device__ __forceinline__ size_t stage_g_bytes(int mp16, int gsize, int transposed) {
-    return a16(transposed ? (size_t)SW * g_tpitch(mp16, gsize) * gsize : (size_t)mp16 * SW * gsize);
+__host__ __device__ __forceinline__ size_t stage_b_bytes(int rows, bool tma) {
+    return tma ? a1k((size_t)rows * SW * 4) : (size_t)rows * SW * 4;
+}
+__host__ __device__ __forceinline__ size_t stage_g_bytes(int mp, int rows, int gsize, int transposed, bool tma) {
+    if (transposed) return a16((size_t)SW * g_tpitch(up16(mp), gsize) * gsize);
+    return tma ? a1k((size_t)rows * SW * gsize) : (size_t)rows * SW * gsize;
 }
 // Warp partials of a 16 x (8 NT) product: one float4 per lane and n-tile; the pitch between
 // warps is = 8 (mod 32) floats so the quarter-sums of the reduction hit distinct banks.
 __host__ __device__ __forceinline__ int part_pitch(int NT) { return NT * 128 + 8; }
+__host__ __device__ __forceinline__ bool lam_partials_in_slot(int KT, size_t stage) {
+    return KT > 0 && (size_t)NW * part_pitch(KT) * 4 <= stage;
+}
 
-// tot[o] = sum over the 16 warps of part[w][o], o < NT * 128, in a fixed order: four threads
-// per output each add four warps (w = q, q + 4, q + 8, q + 12), then two xor-shuffles.
+// tot[o] = sum over the NW warps of part[w][o], o < NT * 128, in a fixed order: four threads
+// per output each add the warps w = q, q + 4, q + 8, ... in turn, then two xor-shuffles.
 __device__ __forceinline__ void reduce_warps(const float* part, int pitch, int NT, float* tot) {
     const int nout = NT * 128;
     for (int base = 0; base < nout * 4; base += T) {
@@ -117,7 +172,8 @@ __device__ __forceinline__ void reduce_warps(const float* part, int pitch, int N
         float a = 0.f;
         if (o < nout) {
             const float* p = part + q * pitch + o;
-            a = ((p[0] + p[4 * pitch]) + p[8 * pitch]) + p[12 * pitch];
+#pragma unroll
+            for (int ww = 0; ww < NW / 4; ++ww) a += p[4 * ww * pitch];
         }
         a += __shfl_xor_sync(0xffffffffu, a, 1);
         a += __shfl_xor_sync(0xffffffffu, a, 2);
@@ -127,23 +183,28 @@ __device__ __forceinline__ void reduce_warps(const float* part, int pitch, int N
 
 template <typename GT> struct GradPair;
 template <> struct GradPair<float> {
-    // (row a, columns 2g, 2g + 1) of a row-major swizzled fp32 strip
+    // (row a, columns c, c + 1) of a 64-byte-swizzled fp32 strip, c even
     static __device__ __forceinline__ float2 row(const float* Gs, int a, int c) {
-        return *reinterpret_cast<const float2*>(Gs + sw_elem(a, c));
+        return *reinterpret_cast<const float2*>(Gs + sw64(a, c));
     }
 };
 template <> struct GradPair<__nv_bfloat16> {
     static __device__ __forceinline__ float2 row(const __nv_bfloat16* Gs, int a, int c) {
-        return __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(Gs + a * SW + c));
+        return __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(Gs + sw32(a, c)));
     }
 };
 
-// NQ = ceil(r / 8) n-tiles over q; each warp owns up to GPW = 4 / NQ groups of 8 rows
-// (group w + 16 j), so m' <= 128 GPW.
-template <typename GT, int NQ>
-__global__ void __launch_bounds__(T, 1) stream_mma_kernel(const __grid_constant__ StreamGroup g) {
-    constexpr int GPW = 4 / NQ;
-    extern __shared__ __align__(16) unsigned char smem[];
+// NQ = ceil(r / 8) n-tiles over q; each warp owns up to GPW = GPW_MAX / NQ groups of 8 rows
+// (group w + NW j), so m' <= 8 NW GPW.  TMA: tile copies (G in its stored orientation), else
+// cp.async.  `maps` holds the tile-copy descriptors (unused without TMA).
+template <typename GT, int NQ, bool TMA>
+__device__ __forceinline__ void compose_strip(const StreamGroup& g, const TmaMaps* maps) {
+    constexpr int GPW = GPW_MAX / NQ;
+    extern __shared__ __align__(16) unsigned char smem_raw[];
+    // tile copies with a 64-byte swizzle need 512-byte aligned destinations: align the base by
+    // an offset within the shared window (pointer arithmetic keeps the shared address space)
+    unsigned char* smem = smem_raw;
+    if constexpr (TMA) smem += (1024u - (static_cast<uint32_t>(__cvta_generic_to_shared(smem_raw)) & 1023u)) & 1023u;
     int mi = 0;
     while (mi + 1 < g.nmat && blockIdx.x >= static_cast<unsigned>(g.mat[mi + 1].strip0)) ++mi;
     const StreamMat& M = g.mat[mi];
@@ -154,111 +215,161 @@ __global__ void __launch_bounds__(T, 1) stream_mma_kernel(const __grid_constant_
     const int tid = threadIdx.x, w = tid >> 5, lane = tid & 31, gg = lane >> 2, t = lane & 3;
     constexpr int GS = sizeof(GT);
     constexpr int EPC = 16 / GS;                      // gradient elements per 16-byte chunk
-    const bool trans = M.transposed != 0;
+    const bool trans = !TMA && M.transposed != 0;
     const int gpt = g_tpitch(mp16, GS);
-    const size_t sb = stage_b_bytes(mp16), sg = stage_g_bytes(mp16, GS, trans), stage = sb + sg;
+    const int rows = slot_rows(mp, TMA);
+    const size_t sb = stage_b_bytes(rows, TMA), sg = stage_g_bytes(mp, rows, GS, trans, TMA), stage = sb + sg;
     const int KT = M.lam ? up8(M.k) >> 3 : 0;        // n-tiles of the lambda epilogue
-    const int pitch = part_pitch(NQ > KT ? NQ : KT);
+    // the epilogue's warp partials go to the last node's ring slot when they fit there
+    const bool wslot = lam_partials_in_slot(KT, stage);
+    const int pitch = part_pitch(wslot || NQ > KT ? NQ : KT);
     unsigned char* ring = smem;
     float* part = reinterpret_cast<float*>(smem + 3 * stage);
-    float* tot = part + NW * pitch;
-    const bool corr = !M.e_zero;
+    float* tot = part + NW * pitch;                   // NQ * 128, and KT * 128 for the epilogue
+    uint64_t* bars = reinterpret_cast<uint64_t*>(tot + (NQ > KT ? NQ : KT) * 128);
+    const bool corr = !M.e_zero, write_B = M.write_B != 0;
     const GT* const* Gp = reinterpret_cast<const GT* const*>(g.G + M.g_off);
+    // the matrix descriptor is indexed by a runtime value: read its pointers once
+    float* const Bst = M.B;
+    const float* const Pprev = M.Pprev;
+    float* const Mbar = M.Mbar;
+    const float* const YFg = M.YF;
+    const float* const YtFg = M.YtF;
+    float* const lam_part = M.part;
+    const uint64_t seed = M.seed;
+    const uint32_t tstep = M.t;
     const int c2 = 2 * gg;                            // the lane's first strip column
     const bool colok = b0 + c2 < np;                  // n' % 4 == 0: both columns or neither
+    const int rho = (t & 1) + 4 * (t >> 1);           // the lane's rows in a group: rho, rho + 2
+    const uint32_t ring_s = static_cast<uint32_t>(__cvta_generic_to_shared(ring));
+    const uint32_t bars_s = static_cast<uint32_t>(__cvta_generic_to_shared(bars));
+    int timed_out = 0;
 
-    // ---- per-thread staging plan (fixed for all nodes): up to 4 chunks of B and 4 of G -------
+    // ---- cp.async staging plan (fixed for all nodes): up to 4 chunks of B and 4 of G -----------
     int boff[4], bdst[4], goff[4], gdst[4];
     unsigned bmask = 0, gmask = 0;
+    if constexpr (!TMA) {
 #pragma unroll
-    for (int j = 0; j < 4; ++j) {
-        const int c = tid + j * T;                    // B chunk: row a, 4 columns
-        const int a = c >> 2, ch = c & 3, col = b0 + 4 * ch;
-        boff[j] = a * np + col;
-        bdst[j] = a * SW + 4 * (ch ^ (((a >> 1) & 1) << 1));
-        if (c < mp * 4) {
-            if (col < np) bmask |= 1u << j;
-            else for (int st = 0; st < 3; ++st)       // columns past n': zero once in every slot
-                *reinterpret_cast<float4*>(reinterpret_cast<float*>(ring + st * stage) + bdst[j]) =
-                    make_float4(0.f, 0.f, 0.f, 0.f);
-        }
-        if (trans) {                                  // G rows b0 + bb, m' contiguous elements
-            const int cpr = mp / EPC;
-            const int bb = c / cpr, gch = c % cpr;
-            goff[j] = (b0 + bb) * mp + gch * EPC;
-            gdst[j] = bb * gpt + gch * EPC;
-            if (c < SW * cpr) {
-                if (b0 + bb < np) gmask |= 1u << j;
-                else for (int st = 0; st < 3; ++st)
-                    *reinterpret_cast<float4*>(reinterpret_cast<GT*>(ring + st * stage + sb) + gdst[j]) =
+        for (int j = 0; j < 4; ++j) {
+            const int c = tid + j * T;                // B chunk: row a, 4 columns
+            const int a = c >> 2, ch = c & 3, col = b0 + 4 * ch;
+            boff[j] = a * np + col;
+            bdst[j] = a * SW + 4 * (ch ^ ((a >> 1) & 3));
+            if (c < mp * 4) {
+                if (col < np) bmask |= 1u << j;
+                else for (int st = 0; st < 3; ++st)   // columns past n': zero once in every slot
+                    *reinterpret_cast<float4*>(reinterpret_cast<float*>(ring + st * stage) + bdst[j]) =
                         make_float4(0.f, 0.f, 0.f, 0.f);
             }
-        } else {                                      // G rows a, SW columns
-            constexpr int CPR = SW / EPC;
-            const int ga = c / CPR, gch = c % CPR, gcol = b0 + gch * EPC;
-            goff[j] = ga * np + gcol;
-            gdst[j] = GS == 4 ? ga * SW + 4 * (gch ^ (((ga >> 1) & 1) << 1)) : ga * SW + gch * EPC;
-            if (c < mp * CPR) {
-                if (gcol < np) gmask |= 1u << j;
-                else for (int st = 0; st < 3; ++st)
-                    *reinterpret_cast<float4*>(reinterpret_cast<GT*>(ring + st * stage + sb) + gdst[j]) =
-                        make_float4(0.f, 0.f, 0.f, 0.f);
+            if (trans) {                              // G rows b0 + bb, m' contiguous elements
+                const int cpr = mp / EPC;
+                const int bb = c / cpr, gch = c % cpr;
+                goff[j] = (b0 + bb) * mp + gch * EPC;
+                gdst[j] = bb * gpt + gch * EPC;
+                if (c < SW * cpr) {
+                    if (b0 + bb < np) gmask |= 1u << j;
+                    else for (int st = 0; st < 3; ++st)
+                        *reinterpret_cast<float4*>(reinterpret_cast<GT*>(ring + st * stage + sb) + gdst[j]) =
+                            make_float4(0.f, 0.f, 0.f, 0.f);
+                }
+            } else {                                  // G rows a, SW columns
+                constexpr int CPR = SW / EPC;
+                const int ga = c / CPR, gch = c % CPR, gcol = b0 + gch * EPC;
+                goff[j] = ga * np + gcol;
+                gdst[j] = GS == 4 ? ga * SW + 4 * (gch ^ ((ga >> 1) & 3)) : ga * SW + 8 * (gch ^ ((ga >> 2) & 1));
+                if (c < mp * CPR) {
+                    if (gcol < np) gmask |= 1u << j;
+                    else for (int st = 0; st < 3; ++st)
+                        *reinterpret_cast<float4*>(reinterpret_cast<GT*>(ring + st * stage + sb) + gdst[j]) =
+                            make_float4(0.f, 0.f, 0.f, 0.f);
+                }
             }
         }
-    }
-    // rows mp..mp16 of every B strip and every (non-transposed) G strip stay zero; transposed
-    // matrices have m' % 8 == 0, so their row groups never reach past m'
-    for (int a = mp + (tid >> 4); a < mp16; a += T / SW) {
-        const int c = tid & (SW - 1);
+        // rows mp..mp16 of every B strip and every (non-transposed) G strip stay zero; transposed
+        // matrices have m' % 8 == 0, so their row groups never reach past m'
+        for (int a = mp + (tid >> 4); a < mp16; a += T / SW) {
+            const int c = tid & (SW - 1);
 #pragma unroll
-        for (int st = 0; st < 3; ++st) {
-            reinterpret_cast<float*>(ring + st * stage)[a * SW + c] = 0.f;
-            if (!trans) reinterpret_cast<GT*>(ring + st * stage + sb)[a * SW + c] = GT(0.f);
+            for (int st = 0; st < 3; ++st) {
+                reinterpret_cast<float*>(ring + st * stage)[a * SW + c] = 0.f;
+                if (!trans) reinterpret_cast<GT*>(ring + st * stage + sb)[a * SW + c] = GT(0.f);
+            }
         }
+    } else {
+        if (tid == 0) {
+#pragma unroll
+            for (int st = 0; st < 3; ++st) mbar_init(bars_s + 8 * st, 1);
+            asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+        }
+        __syncthreads();
     }
 
     // ring item j: node j's B (unless E = 0) and G strips; with the lambda epilogue, items N and
-    // N + 1 are the fragment-ordered Y and Yt (up8(m') x 8 KT floats each)
+    // N + 1 are the fragment-ordered Y and Yt (up8(m') x 8 KT floats each).  With tile copies
+    // thread 0 issues an item (rows past m' and columns past n' arrive as zeros); with cp.async
+    // every thread issues its chunks and commits a group.
+    const int nbox = tma_nbox(mp), brows = tma_box_rows(mp);
     auto stage_item = [&](int j) {
-        if (j < N) {
-            unsigned char* base = ring + (size_t)(j % 3) * stage;
-            if (corr) {
-                float* dst = reinterpret_cast<float*>(base);
-                const float* src = M.B + (int64_t)j * mp * np;
+        const uint32_t base = ring_s + static_cast<uint32_t>((j % 3) * stage);
+        if constexpr (TMA) {
+            if (tid != 0) return;
+            const uint32_t bar = bars_s + 8 * (j % 3);
+            if (j < N) {
+                const uint32_t gbytes = static_cast<uint32_t>(brows * SW * GS);
+                mbar_expect_tx(bar, nbox * ((corr ? brows * SW * 4u : 0u) + gbytes));
+                for (int b = 0; b < nbox; ++b) {
+                    if (corr) tma_load_3d(base + b * brows * SW * 4, &maps->B[mi], b0, b * brows, j, bar);
+                    tma_load_2d(base + static_cast<uint32_t>(sb) + b * gbytes, &maps->G[M.g_off + j], b0, b * brows,
+                                bar);
+                }
+            } else if (j < N + 2 && KT) {
+                const uint32_t bytes = static_cast<uint32_t>(ng * KT * 256);   // 64 floats per (group, n-tile)
+                mbar_expect_tx(bar, bytes);
+                bulk_load(base, j == N ? YFg : YtFg, bytes, bar);
+            }
+        } else {
+            if (j < N) {
+                if (corr) {
+                    const float* src = Bst + (int64_t)j * mp * np;
+#pragma unroll
+                    for (int q = 0; q < 4; ++q)
+                        if (bmask & (1u << q)) cp_async16(base + 4u * bdst[q], src + boff[q]);
+                }
+                const GT* src = Gp[j];
 #pragma unroll
                 for (int q = 0; q < 4; ++q)
-                    if (bmask & (1u << q)) cp_async16(dst + bdst[q], src + boff[q]);
+                    if (gmask & (1u << q)) cp_async16(base + static_cast<uint32_t>(sb) + GS * gdst[q], src + goff[q]);
+            } else if (j < N + 2 && KT) {
+                const float* src = j == N ? YFg : YtFg;
+                const int nch = ng * KT * 16;
+                for (int c = tid; c < nch; c += T) cp_async16(base + 16u * c, src + 4 * c);
             }
-            GT* dst = reinterpret_cast<GT*>(base + sb);
-            const GT* src = Gp[j];
-#pragma unroll
-            for (int q = 0; q < 4; ++q)
-                if (gmask & (1u << q)) cp_async16(dst + gdst[q], src + goff[q]);
-        } else if (j < N + 2 && KT) {
-            float* dst = reinterpret_cast<float*>(ring + (size_t)(j % 3) * stage);
-            const float* src = j == N ? M.YF : M.YtF;
-            const int nch = ng * KT * 16;             // 64 floats per (group, n-tile)
-            for (int c = tid; c < nch; c += T) cp_async16(dst + 4 * c, src + 4 * c);
+            cp_async_commit();
         }
-        cp_async_commit();
+    };
+    // item j has landed for this thread (tile copies: its slot's mbarrier completed item j's phase)
+    auto await_item = [&](int j) {
+        if constexpr (TMA) {
+            if (!mbar_wait(bars_s + 8 * (j % 3), (j / 3) & 1)) timed_out = 1;
+        }
     };
     stage_item(0);
     stage_item(1);
 
     // ---- P_prev fragments of the lane's row groups, once per strip ----------------------------
-    const int prow = (gg >> 1) + 4 * (gg & 1);      // C^T = R^T P^T: N index g -> row
+    const int prow = ((gg >> 1) & 1) + 4 * (gg >> 2) + 2 * (gg & 1);   // C^T = R^T P^T: N index g -> row
     FragB prt[GPW][NQ], pcb[GPW][NQ];
 #pragma unroll
     for (int j = 0; j < GPW; ++j) {
         const int G8 = w + NW * j;
-        const int ra = 8 * G8 + t, rc = 8 * G8 + prow;
+        const int ra = 8 * G8 + rho, rc = 8 * G8 + prow;
 #pragma unroll
         for (int nt = 0; nt < NQ; ++nt) {
             const int q = 8 * nt + gg, q0 = 8 * nt + 2 * t;
             const bool use = corr && G8 < ng;
-            const float* P = M.Pprev;
+            const float* P = Pprev;
             prt[j][nt] = frag_b(use && q < r && ra < mp ? __ldg(P + ra * r + q) : 0.f,
-                                use && q < r && ra + 4 < mp ? __ldg(P + (ra + 4) * r + q) : 0.f);
+                                use && q < r && ra + 2 < mp ? __ldg(P + (ra + 2) * r + q) : 0.f);
             pcb[j][nt] = frag_b(use && q0 < r && rc < mp ? __ldg(P + rc * r + q0) : 0.f,
                                 use && q0 + 1 < r && rc < mp ? __ldg(P + rc * r + q0 + 1) : 0.f);
         }
@@ -271,34 +382,48 @@ __global__ void __launch_bounds__(T, 1) stream_mma_kernel(const __grid_constant_
         for (int e = 0; e < 4; ++e) acc[j][e] = 0.f;
 
     for (int i = 0; i < N; ++i) {
-        cp_async_wait<1>();                // node i has landed; item i + 1 may be in flight
-        __syncthreads();                   // ... for every thread; node i - 1 is finished
-        stage_item(i + 2);                 // into the slot node i - 1 used
+        if constexpr (TMA) {
+            __syncthreads();               // node i - 1 is finished by every thread: its slot is free
+            stage_item(i + 2);
+            await_item(i);
+        } else {
+            cp_async_wait<1>();            // node i has landed; item i + 1 may be in flight
+            __syncthreads();               // ... for every thread; node i - 1 is finished
+            stage_item(i + 2);             // into the slot node i - 1 used
+        }
         const unsigned char* base = ring + (size_t)(i % 3) * stage;
         const float* S = reinterpret_cast<const float*>(base);
         const GT* Gs = reinterpret_cast<const GT*>(base + sb);
         if (corr) {                        // warp partials of R_i^T = B_i^T P_prev
-            float d[NQ][4];
+            // one accumulator per row group, so the groups' MMA chains run side by side
+            float d[GPW][NQ][4];
 #pragma unroll
-            for (int nt = 0; nt < NQ; ++nt)
+            for (int j = 0; j < GPW; ++j)
 #pragma unroll
-                for (int e = 0; e < 4; ++e) d[nt][e] = 0.f;
+                for (int nt = 0; nt < NQ; ++nt)
+#pragma unroll
+                    for (int e = 0; e < 4; ++e) d[j][nt][e] = 0.f;
 #pragma unroll
             for (int j = 0; j < GPW; ++j) {
                 const int G8 = w + NW * j;
                 if (G8 < ng) {
-                    const int ra = 8 * G8 + t;
-                    const float2 x0 = *reinterpret_cast<const float2*>(S + sw_elem(ra, c2));
-                    const float2 x1 = *reinterpret_cast<const float2*>(S + sw_elem(ra + 4, c2));
+                    const int ra = 8 * G8 + rho;
+                    const float2 x0 = *reinterpret_cast<const float2*>(S + sw64(ra, c2));
+                    const float2 x1 = *reinterpret_cast<const float2*>(S + sw64(ra + 2, c2));
                     const FragA A = frag_a(x0.x, x0.y, x1.x, x1.y);
 #pragma unroll
-                    for (int nt = 0; nt < NQ; ++nt) mma3(d[nt], A, prt[j][nt]);
+                    for (int nt = 0; nt < NQ; ++nt) mma3(d[j][nt], A, prt[j][nt]);
                 }
             }
 #pragma unroll
-            for (int nt = 0; nt < NQ; ++nt)
-                *reinterpret_cast<float4*>(part + w * pitch + (nt * 32 + lane) * 4) =
-                    make_float4(d[nt][0], d[nt][1], d[nt][2], d[nt][3]);
+            for (int nt = 0; nt < NQ; ++nt) {
+                float4 v = make_float4(d[0][nt][0], d[0][nt][1], d[0][nt][2], d[0][nt][3]);
+#pragma unroll
+                for (int j = 1; j < GPW; ++j) {
+                    v.x += d[j][nt][0]; v.y += d[j][nt][1]; v.z += d[j][nt][2]; v.w += d[j][nt][3];
+                }
+                *reinterpret_cast<float4*>(part + w * pitch + (nt * 32 + lane) * 4) = v;
+            }
         }
         __syncthreads();
         FragA RA[NQ];
@@ -311,19 +436,19 @@ __global__ void __launch_bounds__(T, 1) stream_mma_kernel(const __grid_constant_
                 RA[nt] = frag_a(R.x, R.z, R.y, R.w);
             }
         }
-        float* Bi = M.B + (int64_t)i * mp * np + b0 + c2;
+        float* Bi = Bst + (int64_t)i * mp * np + b0 + c2;
 #pragma unroll
         for (int j = 0; j < GPW; ++j) {
             const int G8 = w + NW * j;
             if (G8 < ng) {
-                const int ra = 8 * G8 + t, rb = ra + 4;
+                const int ra = 8 * G8 + rho, rb = ra + 2;
                 float c[4] = {0.f, 0.f, 0.f, 0.f};
                 float2 x0 = make_float2(0.f, 0.f), x1 = make_float2(0.f, 0.f);
                 if (corr) {
 #pragma unroll
                     for (int nt = 0; nt < NQ; ++nt) mma3(c, RA[nt], pcb[j][nt]);
-                    x0 = *reinterpret_cast<const float2*>(S + sw_elem(ra, c2));
-                    x1 = *reinterpret_cast<const float2*>(S + sw_elem(rb, c2));
+                    x0 = *reinterpret_cast<const float2*>(S + sw64(ra, c2));
+                    x1 = *reinterpret_cast<const float2*>(S + sw64(rb, c2));
                 }
                 float2 g0, g1;
                 if (trans) {
@@ -337,7 +462,7 @@ __global__ void __launch_bounds__(T, 1) stream_mma_kernel(const __grid_constant_
                 const float m1 = g0.y + (x0.y - c[2]);
                 const float m2 = g1.x + (x1.x - c[1]);
                 const float m3 = g1.y + (x1.y - c[3]);
-                if (M.write_B && colok) {
+                if (write_B && colok) {
                     if (ra < mp) __stcs(reinterpret_cast<float2*>(Bi + (int64_t)ra * np), make_float2(m0, m1));
                     if (rb < mp) __stcs(reinterpret_cast<float2*>(Bi + (int64_t)rb * np), make_float2(m2, m3));
                 }
@@ -345,32 +470,52 @@ __global__ void __launch_bounds__(T, 1) stream_mma_kernel(const __grid_constant_
             }
         }
     }
-    cp_async_wait<0>();
+    if constexpr (!TMA) cp_async_wait<0>();
     const float invN = 1.0f / static_cast<float>(N);
-    float* Mb = M.Mbar + b0 + c2;
+    float* Mb = Mbar + b0 + c2;
 #pragma unroll
     for (int j = 0; j < GPW; ++j) {
         const int G8 = w + NW * j;
 #pragma unroll
         for (int e = 0; e < 4; ++e) acc[j][e] *= invN;
-        const int ra = 8 * G8 + t, rb = ra + 4;
+        const int ra = 8 * G8 + rho, rb = ra + 2;
         if (G8 < ng && colok) {
             if (ra < mp) *reinterpret_cast<float2*>(Mb + (int64_t)ra * np) = make_float2(acc[j][0], acc[j][1]);
             if (rb < mp) *reinterpret_cast<float2*>(Mb + (int64_t)rb * np) = make_float2(acc[j][2], acc[j][3]);
         }
     }
-    if (!KT) return;
+    if (!KT) {
+        if (timed_out && g.err) atomicAdd(g.err, 1);
+        return;
+    }
 
     // ---- truncated-basis Approx-Top-r partial sums: (Mbar - Yt (Y^T Mbar)) v_j ------------------
+    // v_j: the 32 lanes draw the 32 quads (row, 4 columns) of a row group once each: lane (g, t)
+    // draws row rho + 2 (g % 2), quad g / 2 (drawn first: they need no data)
+    float4 vq[GPW];
+#pragma unroll
+    for (int j = 0; j < GPW; ++j) {
+        const int G8 = w + NW * j;
+        if (G8 < ng)
+            vq[j] = gauss4(seed, tstep, static_cast<uint32_t>(8 * G8 + rho + 2 * (gg & 1)),
+                           static_cast<uint32_t>((b0 >> 2) + (gg >> 1)), kTagLambdaV);
+    }
+    await_item(N);
+    await_item(N + 1);
     __syncthreads();                                         // Y, Yt landed for every thread
     const float* YF = reinterpret_cast<const float*>(ring + (size_t)(N % 3) * stage);
     const float* YtF = reinterpret_cast<const float*>(ring + (size_t)((N + 1) % 3) * stage);
+    // the warp partials of W^T (in the slot of the last node, free once every thread is here)
+    float* wpart = wslot ? reinterpret_cast<float*>(ring + (size_t)((N + 2) % 3) * stage) : part;
+    const int wpitch = wslot ? part_pitch(KT) : pitch;
     {
-        float d[4][4];
+        float d[2][4][4];                                    // two accumulators per n-tile
 #pragma unroll
-        for (int nt = 0; nt < 4; ++nt)
+        for (int h = 0; h < 2; ++h)
 #pragma unroll
-            for (int e = 0; e < 4; ++e) d[nt][e] = 0.f;
+            for (int nt = 0; nt < 4; ++nt)
+#pragma unroll
+                for (int e = 0; e < 4; ++e) d[h][nt][e] = 0.f;
 #pragma unroll
         for (int j = 0; j < GPW; ++j) {
             const int G8 = w + NW * j;
@@ -380,18 +525,19 @@ __global__ void __launch_bounds__(T, 1) stream_mma_kernel(const __grid_constant_
                 for (int nt = 0; nt < 4; ++nt)
                     if (nt < KT) {
                         const float2 y = *reinterpret_cast<const float2*>(YF + (G8 * KT + nt) * 64 + 2 * lane);
-                        mma3(d[nt], A, frag_b(y.x, y.y));
+                        mma3(d[j & 1][nt], A, frag_b(y.x, y.y));
                     }
             }
         }
 #pragma unroll
         for (int nt = 0; nt < 4; ++nt)
             if (nt < KT)
-                *reinterpret_cast<float4*>(part + w * pitch + (nt * 32 + lane) * 4) =
-                    make_float4(d[nt][0], d[nt][1], d[nt][2], d[nt][3]);
+                *reinterpret_cast<float4*>(wpart + w * wpitch + (nt * 32 + lane) * 4) =
+                    make_float4(d[0][nt][0] + d[1][nt][0], d[0][nt][1] + d[1][nt][1], d[0][nt][2] + d[1][nt][2],
+                                d[0][nt][3] + d[1][nt][3]);
     }
     __syncthreads();
-    reduce_warps(part, pitch, KT, tot);                      // W^T = Mbar_strip^T Y
+    reduce_warps(wpart, wpitch, KT, tot);                    // W^T = Mbar_strip^T Y
     __syncthreads();
     FragA WA[4];
 #pragma unroll
@@ -414,16 +560,13 @@ __global__ void __launch_bounds__(T, 1) stream_mma_kernel(const __grid_constant_
                 }
             const float d0 = acc[j][0] - c[0], d1 = acc[j][1] - c[2];
             const float d2 = acc[j][2] - c[1], d3 = acc[j][3] - c[3];
-            // v_j: the 32 lanes draw the 32 quads (row, 4 columns) of the group once each: lane
-            // (g, t) draws row t + 4 (g % 2), quad g / 2, keeps the half it needs and trades the
-            // other half with lane g ^ 1
-            const int ra = 8 * G8 + t;
-            const float4 vq = gauss4(M.seed, M.t, static_cast<uint32_t>(ra + 4 * (gg & 1)),
-                                     static_cast<uint32_t>((b0 >> 2) + (gg >> 1)), kTagLambdaV);
-            const float q0 = __shfl_xor_sync(0xffffffffu, odd ? vq.x : vq.z, 4);
-            const float q1 = __shfl_xor_sync(0xffffffffu, odd ? vq.y : vq.w, 4);
-            const float v0 = odd ? q0 : vq.x, v1 = odd ? q1 : vq.y;     // row t
-            const float v2 = odd ? vq.z : q0, v3 = odd ? vq.w : q1;     // row t + 4
+            // each lane keeps the half of its quad it needs and trades the other with lane g ^ 1
+            const int ra = 8 * G8 + rho;
+            const float4 v = vq[j];
+            const float q0 = __shfl_xor_sync(0xffffffffu, odd ? v.x : v.z, 4);
+            const float q1 = __shfl_xor_sync(0xffffffffu, odd ? v.y : v.w, 4);
+            const float v0 = odd ? q0 : v.x, v1 = odd ? q1 : v.y;       // row rho
+            const float v2 = odd ? v.z : q0, v3 = odd ? v.w : q1;       // row rho + 2
             float pa = colok ? d0 * v0 + d1 * v1 : 0.f;
             float pb = colok ? d2 * v2 + d3 * v3 : 0.f;
 #pragma unroll
@@ -432,18 +575,29 @@ __global__ void __launch_bounds__(T, 1) stream_mma_kernel(const __grid_constant_
                 pb += __shfl_xor_sync(0xffffffffu, pb, x);
             }
             if (gg == 0) {
-                if (ra < mp) M.part[(int64_t)s * mp + ra] = pa;
-                if (ra + 4 < mp) M.part[(int64_t)s * mp + ra + 4] = pb;
+                if (ra < mp) lam_part[(int64_t)s * mp + ra] = pa;
+                if (ra + 2 < mp) lam_part[(int64_t)s * mp + ra + 2] = pb;
             }
         }
     }
+    if (timed_out && g.err) atomicAdd(g.err, 1);
+}
+
+template <typename GT, int NQ>
+__global__ void __launch_bounds__(T, 1) stream_mma_kernel(const __grid_constant__ StreamGroup g) {
+    compose_strip<GT, NQ, false>(g, nullptr);
+}
+template <typename GT, int NQ>
+__global__ void __launch_bounds__(T, 1) stream_tma_kernel(const __grid_constant__ StreamGroup g,
+                                                          const __grid_constant__ TmaMaps maps) {
+    compose_strip<GT, NQ, true>(g, &maps);
 }
 
 // dst = src (rows x cols, row-major, ld) in fragment order, up8(rows) x up8(cols) floats:
-// block (group G8, n-tile nt) holds 64 floats, lane L's pair at 2L, 2L + 1.
-//   form 0 (B fragment of X^T Y):  src(8 G8 + t, 8 nt + g), src(8 G8 + t + 4, 8 nt + g)
-//   form 1 (B fragment of W Y^T): src(8 G8 + row, 8 nt + 2t), src(8 G8 + row, 8 nt + 2t + 1),
-//                                  row = g / 2 + 4 (g % 2)
+// block (group G8, n-tile nt) holds 64 floats, lane L = 4g + t's pair at 2L, 2L + 1.
+//   form 0 (B fragment of X^T Y):  src(8 G8 + rho(t), 8 nt + g), src(8 G8 + rho(t) + 2, 8 nt + g)
+//   form 1 (B fragment of W Y^T): src(8 G8 + prow(g), 8 nt + 2t), src(8 G8 + prow(g), 8 nt + 2t + 1)
+// with rho(t) = (t % 2) + 4 (t / 2) and prow(g) = rho(g / 2) + 2 (g % 2).
 __global__ void pack_frag_kernel(float* dst, const float* src, int rows, int cols, int ld, int form) {
     const int KT = up8(cols) >> 3;
     const int total = up8(rows) * KT * 8;
@@ -451,8 +605,8 @@ __global__ void pack_frag_kernel(float* dst, const float* src, int rows, int col
         const int blk = idx >> 6, L = (idx >> 1) & 31, e = idx & 1;
         const int G8 = blk / KT, nt = blk % KT, g = L >> 2, t = L & 3;
         int row, col;
-        if (form == 0) { row = 8 * G8 + t + 4 * e; col = 8 * nt + g; }
-        else { row = 8 * G8 + (g >> 1) + 4 * (g & 1); col = 8 * nt + 2 * t + e; }
+        if (form == 0) { row = 8 * G8 + (t & 1) + 4 * (t >> 1) + 2 * e; col = 8 * nt + g; }
+        else { row = 8 * G8 + ((g >> 1) & 1) + 4 * (g >> 2) + 2 * (g & 1); col = 8 * nt + 2 * t + e; }
         dst[idx] = row < rows && col < cols ? src[(int64_t)row * ld + col] : 0.f;
     }
 }
@@ -463,19 +617,30 @@ int mma_stream_nq(int r) { return (r + 7) / 8; }
 
 bool mma_stream_eligible(int mp, int np, int r, int k, int lam, int transposed, int gsize) {
     const int NQ = mma_stream_nq(r), ng = up8(mp) / 8;
-    if (NQ < 1 || NQ > 2 || (ng + NW - 1) / NW > 4 / NQ) return false;   // groups per warp
+    if (NQ < 1 || NQ > 2 || (ng + NW - 1) / NW > GPW_MAX / NQ) return false;   // groups per warp
     if (lam && (k < 1 || k > 32)) return false;
     if (np % 4 != 0 || (transposed && mp % 8 != 0)) return false;      // 16-byte chunks of G rows
-    return mma_stream_smem_bytes(mp, r, k, lam, gsize, transposed) <= 227 * 1024;
+    return mma_stream_smem_bytes(mp, r, k, lam, gsize, transposed, 0) <= 227 * 1024;
 }
 
-size_t mma_stream_smem_bytes(int mp, int r, int k, int lam, int gsize, int transposed) {
-    const int mp16 = up16(mp), NQ = mma_stream_nq(r), KT = lam ? up8(k) / 8 : 0;
-    const size_t stage = stage_b_bytes(mp16) + stage_g_bytes(mp16, gsize, transposed);
+bool mma_stream_tma_eligible(int mp, int np, int r, int k, int lam, int transposed, int gsize) {
+    if (transposed || !mma_stream_eligible(mp, np, r, k, lam, transposed, gsize)) return false;
+    if (((int64_t)np * gsize) % 16 != 0) return false;                 // row stride of a tile copy
+    return mma_stream_smem_bytes(mp, r, k, lam, gsize, transposed, 1) <= 227 * 1024;
+}
+
+size_t mma_stream_smem_bytes(int mp, int r, int k, int lam, int gsize, int transposed, int tma) {
+    const int NQ = mma_stream_nq(r), KT = lam ? up8(k) / 8 : 0;
+    const int rows = slot_rows(mp, tma != 0);
+    const size_t stage = stage_b_bytes(rows, tma != 0) + stage_g_bytes(mp, rows, gsize, transposed, tma != 0);
     if (lam && (size_t)up8(mp) * KT * 8 * 4 > stage) return ~size_t(0);   // Y, Yt use ring slots
     const int NT = NQ > KT ? NQ : KT;
-    return 3 * stage + (size_t)NW * part_pitch(NT) * 4 + (size_t)NT * 128 * 4;
+    const int PT = lam_partials_in_slot(KT, stage) ? NQ : NT;
+    const size_t bytes = 3 * stage + (size_t)NW * part_pitch(PT) * 4 + (size_t)NT * 128 * 4 + 3 * 8;
+    return tma ? bytes + 1024 : bytes;                 // room to align the base to 1024 bytes
 }
+
+int mma_tma_box_rows(int mp) { return tma_box_rows(mp); }
 
 template <typename GT, int NQ>
 static cudaError_t launch_mma(const StreamGroup& g, size_t smem, cudaStream_t st) {
@@ -489,12 +654,32 @@ static cudaError_t launch_mma(const StreamGroup& g, size_t smem, cudaStream_t st
     stream_mma_kernel<GT, NQ><<<g.total_strips, T, smem, st>>>(g);
     return cudaGetLastError();
 }
+template <typename GT, int NQ>
+static cudaError_t launch_tma(const StreamGroup& g, const TmaMaps& maps, size_t smem, cudaStream_t st) {
+    static bool set = false;
+    if (!set) {
+        cudaError_t e = cudaFuncSetAttribute(stream_tma_kernel<GT, NQ>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                             227 * 1024);
+        if (e != cudaSuccess) return e;
+        set = true;
+    }
+    stream_tma_kernel<GT, NQ><<<g.total_strips, T, smem, st>>>(g, maps);
+    return cudaGetLastError();
+}
 
-cudaError_t stream_group_mma(const StreamGroup& g, size_t smem, cudaStream_t st) {
+cudaError_t stream_group_mma(const StreamGroup& g, const TmaMaps* maps, size_t smem, cudaStream_t st) {
     if (g.total_strips <= 0) return cudaSuccess;
     const int NQ = mma_stream_nq(g.mat[0].r);
     for (int i = 1; i < g.nmat; ++i)
         if (mma_stream_nq(g.mat[i].r) != NQ) return cudaErrorInvalidValue;
+    if (maps) {
+        for (int i = 0; i < g.nmat; ++i)
+            if (g.mat[i].transposed || g.mat[i].g_off + g.mat[i].N > kTmaGMax) return cudaErrorInvalidValue;
+        if (g.grad_dtype == GLR_BF16)
+            return NQ == 1 ? launch_tma<__nv_bfloat16, 1>(g, *maps, smem, st)
+                           : launch_tma<__nv_bfloat16, 2>(g, *maps, smem, st);
+        return NQ == 1 ? launch_tma<float, 1>(g, *maps, smem, st) : launch_tma<float, 2>(g, *maps, smem, st);
+    }
     if (g.grad_dtype == GLR_BF16)
         return NQ == 1 ? launch_mma<__nv_bfloat16, 1>(g, smem, st) : launch_mma<__nv_bfloat16, 2>(g, smem, st);
     return NQ == 1 ? launch_mma<float, 1>(g, smem, st) : launch_mma<float, 2>(g, smem, st);
