@@ -301,7 +301,7 @@ __global__ void __launch_bounds__(NT, 1) stream_kernel(const __grid_constant__ S
             if (ii < nrows) {
                 const int a = a0 + ii;
                 const float4 m = ld4(Ms + a * BN + 4 * cg);
-                const float4 v = gauss4(M.seed, M.t, static_cast<uint32_t>(a), static_cast<uint32_t>(bcol >> 2),
+                const float4 v = gauss4_fast(M.seed, M.t, static_cast<uint32_t>(a), static_cast<uint32_t>(bcol >> 2),
                                         kTagLambdaV);
                 rows[ii] = (m.x - c[ii][0]) * v.x + (m.y - c[ii][1]) * v.y + (m.z - c[ii][2]) * v.z +
                            (m.w - c[ii][3]) * v.w;

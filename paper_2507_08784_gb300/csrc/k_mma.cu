@@ -97,6 +97,9 @@ __device__ __forceinline__ void cp_async_wait() {
 __device__ __forceinline__ void mbar_init(uint32_t bar, uint32_t count) {
     asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(bar), "r"(count) : "memory");
 }
+__device__ __forceinline__ void mbar_arrive(uint32_t bar) {
+    asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(bar) : "memory");
+}
 __device__ __forceinline__ void mbar_expect_tx(uint32_t bar, uint32_t bytes) {
     asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar), "r"(bytes) : "memory");
 }
@@ -194,17 +197,259 @@ template <> struct GradPair<__nv_bfloat16> {
     }
 };
 
+// ---- the pieces of a strip's work, shared by the kernels below ------------------------------
+// Lane geometry (see the header): warp w, lane = 4 gg + t, rows rho and rho + 2 of each group,
+// columns c2 and c2 + 1; prow is the row of the C^T = R^T P^T B fragment.
+struct Lane {
+    int tid, w, lane, gg, t, rho, prow, c2;
+};
+__device__ __forceinline__ Lane lane_geometry() {
+    Lane L;
+    L.tid = threadIdx.x; L.w = L.tid >> 5; L.lane = L.tid & 31; L.gg = L.lane >> 2; L.t = L.lane & 3;
+    L.rho = (L.t & 1) + 4 * (L.t >> 1);
+    L.prow = ((L.gg >> 1) & 1) + 4 * (L.gg >> 2) + 2 * (L.gg & 1);
+    L.c2 = 2 * L.gg;
+    return L;
+}
+
+// P_prev fragments of the lane's row groups (zero where E = 0, past m' or past r).
+template <int NQ, int GPW>
+__device__ __forceinline__ void load_pfrags(const float* P, int mp, int r, int ng, bool use, const Lane& L,
+                                            FragB (&prt)[GPW][NQ], FragB (&pcb)[GPW][NQ]) {
+#pragma unroll
+    for (int j = 0; j < GPW; ++j) {
+        const int G8 = L.w + NW * j;
+        const int ra = 8 * G8 + L.rho, rc = 8 * G8 + L.prow;
+        const bool u = use && G8 < ng;
+#pragma unroll
+        for (int nt = 0; nt < NQ; ++nt) {
+            const int q = 8 * nt + L.gg, q0 = 8 * nt + 2 * L.t;
+            prt[j][nt] = frag_b(u && q < r && ra < mp ? __ldg(P + ra * r + q) : 0.f,
+                                u && q < r && ra + 2 < mp ? __ldg(P + (ra + 2) * r + q) : 0.f);
+            pcb[j][nt] = frag_b(u && q0 < r && rc < mp ? __ldg(P + rc * r + q0) : 0.f,
+                                u && q0 + 1 < r && rc < mp ? __ldg(P + rc * r + q0 + 1) : 0.f);
+        }
+    }
+}
+
+// One node on a strip resident in shared memory (S: B strip, Gs: G strip, transposed with pitch
+// gpt when trans): warp partials of R_i^T = B_i^T P_prev, their reduction, and the combine
+// M_i = G_i + (B_i - P_prev R_i) with B_i <- M_i (Bi: node i's B at the strip's first column)
+// and acc += M_i.  Contains two barriers when corr, one otherwise; the caller's barrier before
+// it made the strip readable.
+template <typename GT, int NQ, int GPW>
+__device__ __forceinline__ void compose_node(const float* S, const GT* Gs, bool trans, int gpt, bool corr,
+                                             const FragB (&prt)[GPW][NQ], const FragB (&pcb)[GPW][NQ],
+                                             float (&acc)[GPW][4], float* part, int pitch, float* tot, float* Bi,
+                                             int mp, int np, int ng, bool write_B, bool colok, const Lane& L) {
+    if (corr) {                            // warp partials of R_i^T = B_i^T P_prev
+        // one accumulator per row group, so the groups' MMA chains run side by side
+        float d[GPW][NQ][4];
+#pragma unroll
+        for (int j = 0; j < GPW; ++j)
+#pragma unroll
+            for (int nt = 0; nt < NQ; ++nt)
+#pragma unroll
+                for (int e = 0; e < 4; ++e) d[j][nt][e] = 0.f;
+#pragma unroll
+        for (int j = 0; j < GPW; ++j) {
+            const int G8 = L.w + NW * j;
+            if (G8 < ng) {
+                const int ra = 8 * G8 + L.rho;
+                const float2 x0 = *reinterpret_cast<const float2*>(S + sw64(ra, L.c2));
+                const float2 x1 = *reinterpret_cast<const float2*>(S + sw64(ra + 2, L.c2));
+                const FragA A = frag_a(x0.x, x0.y, x1.x, x1.y);
+#pragma unroll
+                for (int nt = 0; nt < NQ; ++nt) mma3(d[j][nt], A, prt[j][nt]);
+            }
+        }
+#pragma unroll
+        for (int nt = 0; nt < NQ; ++nt) {
+            float4 v = make_float4(d[0][nt][0], d[0][nt][1], d[0][nt][2], d[0][nt][3]);
+#pragma unroll
+            for (int j = 1; j < GPW; ++j) {
+                v.x += d[j][nt][0]; v.y += d[j][nt][1]; v.z += d[j][nt][2]; v.w += d[j][nt][3];
+            }
+            *reinterpret_cast<float4*>(part + L.w * pitch + (nt * 32 + L.lane) * 4) = v;
+        }
+    }
+    __syncthreads();
+    FragA RA[NQ];
+    if (corr) {
+        reduce_warps(part, pitch, NQ, tot);
+        __syncthreads();
+#pragma unroll
+        for (int nt = 0; nt < NQ; ++nt) {
+            const float4 R = *reinterpret_cast<const float4*>(tot + (nt * 32 + L.lane) * 4);
+            RA[nt] = frag_a(R.x, R.z, R.y, R.w);
+        }
+    }
+#pragma unroll
+    for (int j = 0; j < GPW; ++j) {
+        const int G8 = L.w + NW * j;
+        if (G8 < ng) {
+            const int ra = 8 * G8 + L.rho, rb = ra + 2;
+            float c[4] = {0.f, 0.f, 0.f, 0.f};
+            float2 x0 = make_float2(0.f, 0.f), x1 = make_float2(0.f, 0.f);
+            if (corr) {
+#pragma unroll
+                for (int nt = 0; nt < NQ; ++nt) mma3(c, RA[nt], pcb[j][nt]);
+                x0 = *reinterpret_cast<const float2*>(S + sw64(ra, L.c2));
+                x1 = *reinterpret_cast<const float2*>(S + sw64(rb, L.c2));
+            }
+            float2 g0, g1;
+            if (trans) {
+                g0 = make_float2(static_cast<float>(Gs[L.c2 * gpt + ra]), static_cast<float>(Gs[(L.c2 + 1) * gpt + ra]));
+                g1 = make_float2(static_cast<float>(Gs[L.c2 * gpt + rb]), static_cast<float>(Gs[(L.c2 + 1) * gpt + rb]));
+            } else {
+                g0 = GradPair<GT>::row(Gs, ra, L.c2);
+                g1 = GradPair<GT>::row(Gs, rb, L.c2);
+            }
+            const float m0 = g0.x + (x0.x - c[0]);       // M = G + E, E = B - P_prev R
+            const float m1 = g0.y + (x0.y - c[2]);
+            const float m2 = g1.x + (x1.x - c[1]);
+            const float m3 = g1.y + (x1.y - c[3]);
+            if (write_B && colok) {
+                if (ra < mp) __stcs(reinterpret_cast<float2*>(Bi + (int64_t)ra * np), make_float2(m0, m1));
+                if (rb < mp) __stcs(reinterpret_cast<float2*>(Bi + (int64_t)rb * np), make_float2(m2, m3));
+            }
+            acc[j][0] += m0; acc[j][1] += m1; acc[j][2] += m2; acc[j][3] += m3;
+        }
+    }
+}
+
+// acc <- acc / N, stored as the strip of Mbar (Mb: Mbar at the strip's first column).
+template <int GPW>
+__device__ __forceinline__ void store_mbar(float (&acc)[GPW][4], int N, float* Mb, int mp, int np, int ng, bool colok,
+                                           const Lane& L) {
+    const float invN = 1.0f / static_cast<float>(N);
+#pragma unroll
+    for (int j = 0; j < GPW; ++j) {
+        const int G8 = L.w + NW * j;
+#pragma unroll
+        for (int e = 0; e < 4; ++e) acc[j][e] *= invN;
+        const int ra = 8 * G8 + L.rho, rb = ra + 2;
+        if (G8 < ng && colok) {
+            if (ra < mp) *reinterpret_cast<float2*>(Mb + (int64_t)ra * np) = make_float2(acc[j][0], acc[j][1]);
+            if (rb < mp) *reinterpret_cast<float2*>(Mb + (int64_t)rb * np) = make_float2(acc[j][2], acc[j][3]);
+        }
+    }
+}
+
+// Truncated-basis Approx-Top-r partial sums over the strip: (Mbar - Yt (Y^T Mbar)) v_j.
+// v_j first: the 32 lanes draw the 32 quads (row, 4 columns) of a row group once each: lane
+// (g, t) draws row rho + 2 (g % 2), quad g / 2 (no data needed, so it can run early).
+template <int GPW>
+__device__ __forceinline__ void lam_draw(float4 (&vq)[GPW], uint64_t seed, uint32_t t, int b0, int ng, const Lane& L) {
+#pragma unroll
+    for (int j = 0; j < GPW; ++j) {
+        const int G8 = L.w + NW * j;
+        if (G8 < ng)
+            vq[j] = gauss4_fast(seed, t, static_cast<uint32_t>(8 * G8 + L.rho + 2 * (L.gg & 1)),
+                           static_cast<uint32_t>((b0 >> 2) + (L.gg >> 1)), kTagLambdaV);
+    }
+}
+// Warp partials of W^T = Mbar_strip^T Y (YF: Y in fragment order, KT n-tiles) into wpart.
+template <int GPW>
+__device__ __forceinline__ void lam_w_partials(const float* YF, int KT, const float (&acc)[GPW][4], float* wpart,
+                                               int wpitch, int ng, const Lane& L) {
+    float d[2][4][4];                                        // two accumulators per n-tile
+#pragma unroll
+    for (int h = 0; h < 2; ++h)
+#pragma unroll
+        for (int nt = 0; nt < 4; ++nt)
+#pragma unroll
+            for (int e = 0; e < 4; ++e) d[h][nt][e] = 0.f;
+#pragma unroll
+    for (int j = 0; j < GPW; ++j) {
+        const int G8 = L.w + NW * j;
+        if (G8 < ng) {
+            const FragA A = frag_a(acc[j][0], acc[j][1], acc[j][2], acc[j][3]);
+#pragma unroll
+            for (int nt = 0; nt < 4; ++nt)
+                if (nt < KT) {
+                    const float2 y = *reinterpret_cast<const float2*>(YF + (G8 * KT + nt) * 64 + 2 * L.lane);
+                    mma3(d[j & 1][nt], A, frag_b(y.x, y.y));
+                }
+        }
+    }
+#pragma unroll
+    for (int nt = 0; nt < 4; ++nt)
+        if (nt < KT)
+            *reinterpret_cast<float4*>(wpart + L.w * wpitch + (nt * 32 + L.lane) * 4) =
+                make_float4(d[0][nt][0] + d[1][nt][0], d[0][nt][1] + d[1][nt][1], d[0][nt][2] + d[1][nt][2],
+                            d[0][nt][3] + d[1][nt][3]);
+}
+// With W^T reduced in tot: C = Yt W on the lane's elements (YtF: Yt in fragment order) and the
+// row partial sums of (Mbar - C) v_j, written to part_row[a] (the strip's row of partials).
+template <int GPW>
+__device__ __forceinline__ void lam_finish(const float* YtF, int KT, const float* tot, const float (&acc)[GPW][4],
+                                           const float4 (&vq)[GPW], float* part_row, int mp, int ng, bool colok,
+                                           const Lane& L) {
+    FragA WA[4];
+#pragma unroll
+    for (int nt = 0; nt < 4; ++nt)
+        if (nt < KT) {
+            const float4 W = *reinterpret_cast<const float4*>(tot + (nt * 32 + L.lane) * 4);
+            WA[nt] = frag_a(W.x, W.z, W.y, W.w);
+        }
+    const bool odd = (L.gg & 1) != 0;
+#pragma unroll
+    for (int j = 0; j < GPW; ++j) {
+        const int G8 = L.w + NW * j;                         // warp-uniform: shuffles below are safe
+        if (G8 < ng) {
+            float c[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+            for (int nt = 0; nt < 4; ++nt)
+                if (nt < KT) {
+                    const float2 y = *reinterpret_cast<const float2*>(YtF + (G8 * KT + nt) * 64 + 2 * L.lane);
+                    mma3(c, WA[nt], frag_b(y.x, y.y));
+                }
+            const float d0 = acc[j][0] - c[0], d1 = acc[j][1] - c[2];
+            const float d2 = acc[j][2] - c[1], d3 = acc[j][3] - c[3];
+            // each lane keeps the half of its quad it needs and trades the other with lane g ^ 1
+            const int ra = 8 * G8 + L.rho;
+            const float4 v = vq[j];
+            const float q0 = __shfl_xor_sync(0xffffffffu, odd ? v.x : v.z, 4);
+            const float q1 = __shfl_xor_sync(0xffffffffu, odd ? v.y : v.w, 4);
+            const float v0 = odd ? q0 : v.x, v1 = odd ? q1 : v.y;       // row rho
+            const float v2 = odd ? v.z : q0, v3 = odd ? v.w : q1;       // row rho + 2
+            float pa = colok ? d0 * v0 + d1 * v1 : 0.f;
+            float pb = colok ? d2 * v2 + d3 * v3 : 0.f;
+#pragma unroll
+            for (int x = 4; x < 32; x <<= 1) {
+                pa += __shfl_xor_sync(0xffffffffu, pa, x);
+                pb += __shfl_xor_sync(0xffffffffu, pb, x);
+            }
+            if (L.gg == 0) {
+                if (ra < mp) part_row[ra] = pa;
+                if (ra + 2 < mp) part_row[ra + 2] = pb;
+            }
+        }
+    }
+}
+
+// Base of the dynamic shared memory; tile copies with a 64-byte swizzle need 512-byte aligned
+// destinations, so the TMA kernels align it by an offset within the shared window (pointer
+// arithmetic keeps the shared address space).
+template <bool ALIGN>
+__device__ __forceinline__ unsigned char* smem_base() {
+    extern __shared__ __align__(16) unsigned char smem_raw[];
+    unsigned char* p = smem_raw;
+    if constexpr (ALIGN) p += (1024u - (static_cast<uint32_t>(__cvta_generic_to_shared(smem_raw)) & 1023u)) & 1023u;
+    return p;
+}
+
+// ---- per-strip kernel: one CTA per strip ----------------------------------------------------
 // NQ = ceil(r / 8) n-tiles over q; each warp owns up to GPW = GPW_MAX / NQ groups of 8 rows
 // (group w + NW j), so m' <= 8 NW GPW.  TMA: tile copies (G in its stored orientation), else
 // cp.async.  `maps` holds the tile-copy descriptors (unused without TMA).
 template <typename GT, int NQ, bool TMA>
 __device__ __forceinline__ void compose_strip(const StreamGroup& g, const TmaMaps* maps) {
     constexpr int GPW = GPW_MAX / NQ;
-    extern __shared__ __align__(16) unsigned char smem_raw[];
-    // tile copies with a 64-byte swizzle need 512-byte aligned destinations: align the base by
-    // an offset within the shared window (pointer arithmetic keeps the shared address space)
-    unsigned char* smem = smem_raw;
-    if constexpr (TMA) smem += (1024u - (static_cast<uint32_t>(__cvta_generic_to_shared(smem_raw)) & 1023u)) & 1023u;
+    unsigned char* smem = smem_base<TMA>();
+    const Lane L = lane_geometry();
+    const int tid = L.tid;
     int mi = 0;
     while (mi + 1 < g.nmat && blockIdx.x >= static_cast<unsigned>(g.mat[mi + 1].strip0)) ++mi;
     const StreamMat& M = g.mat[mi];
@@ -212,7 +457,6 @@ __device__ __forceinline__ void compose_strip(const StreamGroup& g, const TmaMap
     const int b0 = s * SW;
     const int mp = M.mp, np = M.np, r = M.r, N = M.N;
     const int mp16 = up16(mp), ng = up8(mp) >> 3;
-    const int tid = threadIdx.x, w = tid >> 5, lane = tid & 31, gg = lane >> 2, t = lane & 3;
     constexpr int GS = sizeof(GT);
     constexpr int EPC = 16 / GS;                      // gradient elements per 16-byte chunk
     const bool trans = !TMA && M.transposed != 0;
@@ -231,18 +475,12 @@ __device__ __forceinline__ void compose_strip(const StreamGroup& g, const TmaMap
     const GT* const* Gp = reinterpret_cast<const GT* const*>(g.G + M.g_off);
     // the matrix descriptor is indexed by a runtime value: read its pointers once
     float* const Bst = M.B;
-    const float* const Pprev = M.Pprev;
-    float* const Mbar = M.Mbar;
     const float* const YFg = M.YF;
     const float* const YtFg = M.YtF;
-    float* const lam_part = M.part;
-    const uint64_t seed = M.seed;
-    const uint32_t tstep = M.t;
-    const int c2 = 2 * gg;                            // the lane's first strip column
-    const bool colok = b0 + c2 < np;                  // n' % 4 == 0: both columns or neither
-    const int rho = (t & 1) + 4 * (t >> 1);           // the lane's rows in a group: rho, rho + 2
+    const bool colok = b0 + L.c2 < np;                // n' % 4 == 0: both columns or neither
     const uint32_t ring_s = static_cast<uint32_t>(__cvta_generic_to_shared(ring));
-    const uint32_t bars_s = static_cast<uint32_t>(__cvta_generic_to_shared(bars));
+    // tile copies: full[3] (copy landed) then empty[3] (every warp is done with the slot)
+    const uint32_t bars_s = static_cast<uint32_t>(__cvta_generic_to_shared(bars)), empty_s = bars_s + 24;
     int timed_out = 0;
 
     // ---- cp.async staging plan (fixed for all nodes): up to 4 chunks of B and 4 of G -----------
@@ -298,7 +536,10 @@ __device__ __forceinline__ void compose_strip(const StreamGroup& g, const TmaMap
     } else {
         if (tid == 0) {
 #pragma unroll
-            for (int st = 0; st < 3; ++st) mbar_init(bars_s + 8 * st, 1);
+            for (int st = 0; st < 3; ++st) {
+                mbar_init(bars_s + 8 * st, 1);
+                mbar_init(empty_s + 8 * st, NW);
+            }
             asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
         }
         __syncthreads();
@@ -312,8 +553,10 @@ __device__ __forceinline__ void compose_strip(const StreamGroup& g, const TmaMap
     auto stage_item = [&](int j) {
         const uint32_t base = ring_s + static_cast<uint32_t>((j % 3) * stage);
         if constexpr (TMA) {
-            if (tid != 0) return;
+            if (tid != 0 || j >= N + (KT ? 2 : 0)) return;
             const uint32_t bar = bars_s + 8 * (j % 3);
+            // the slot's previous item (j - 3) must be released by every warp
+            if (j >= 3 && !mbar_wait(empty_s + 8 * (j % 3), ((j / 3) - 1) & 1)) timed_out = 1;
             if (j < N) {
                 const uint32_t gbytes = static_cast<uint32_t>(brows * SW * GS);
                 mbar_expect_tx(bar, nbox * ((corr ? brows * SW * 4u : 0u) + gbytes));
@@ -322,7 +565,7 @@ __device__ __forceinline__ void compose_strip(const StreamGroup& g, const TmaMap
                     tma_load_2d(base + static_cast<uint32_t>(sb) + b * gbytes, &maps->G[M.g_off + j], b0, b * brows,
                                 bar);
                 }
-            } else if (j < N + 2 && KT) {
+            } else {
                 const uint32_t bytes = static_cast<uint32_t>(ng * KT * 256);   // 64 floats per (group, n-tile)
                 mbar_expect_tx(bar, bytes);
                 bulk_load(base, j == N ? YFg : YtFg, bytes, bar);
@@ -356,25 +599,8 @@ __device__ __forceinline__ void compose_strip(const StreamGroup& g, const TmaMap
     stage_item(0);
     stage_item(1);
 
-    // ---- P_prev fragments of the lane's row groups, once per strip ----------------------------
-    const int prow = ((gg >> 1) & 1) + 4 * (gg >> 2) + 2 * (gg & 1);   // C^T = R^T P^T: N index g -> row
     FragB prt[GPW][NQ], pcb[GPW][NQ];
-#pragma unroll
-    for (int j = 0; j < GPW; ++j) {
-        const int G8 = w + NW * j;
-        const int ra = 8 * G8 + rho, rc = 8 * G8 + prow;
-#pragma unroll
-        for (int nt = 0; nt < NQ; ++nt) {
-            const int q = 8 * nt + gg, q0 = 8 * nt + 2 * t;
-            const bool use = corr && G8 < ng;
-            const float* P = Pprev;
-            prt[j][nt] = frag_b(use && q < r && ra < mp ? __ldg(P + ra * r + q) : 0.f,
-                                use && q < r && ra + 2 < mp ? __ldg(P + (ra + 2) * r + q) : 0.f);
-            pcb[j][nt] = frag_b(use && q0 < r && rc < mp ? __ldg(P + rc * r + q0) : 0.f,
-                                use && q0 + 1 < r && rc < mp ? __ldg(P + rc * r + q0 + 1) : 0.f);
-        }
-    }
-
+    load_pfrags<NQ, GPW>(M.Pprev, mp, r, ng, corr, L, prt, pcb);
     float acc[GPW][4];
 #pragma unroll
     for (int j = 0; j < GPW; ++j)
@@ -383,202 +609,40 @@ __device__ __forceinline__ void compose_strip(const StreamGroup& g, const TmaMap
 
     for (int i = 0; i < N; ++i) {
         if constexpr (TMA) {
-            __syncthreads();               // node i - 1 is finished by every thread: its slot is free
-            stage_item(i + 2);
+            stage_item(i + 2);             // thread 0, once node i - 1's slot is released
             await_item(i);
         } else {
             cp_async_wait<1>();            // node i has landed; item i + 1 may be in flight
             __syncthreads();               // ... for every thread; node i - 1 is finished
             stage_item(i + 2);             // into the slot node i - 1 used
         }
-        const unsigned char* base = ring + (size_t)(i % 3) * stage;
-        const float* S = reinterpret_cast<const float*>(base);
-        const GT* Gs = reinterpret_cast<const GT*>(base + sb);
-        if (corr) {                        // warp partials of R_i^T = B_i^T P_prev
-            // one accumulator per row group, so the groups' MMA chains run side by side
-            float d[GPW][NQ][4];
-#pragma unroll
-            for (int j = 0; j < GPW; ++j)
-#pragma unroll
-                for (int nt = 0; nt < NQ; ++nt)
-#pragma unroll
-                    for (int e = 0; e < 4; ++e) d[j][nt][e] = 0.f;
-#pragma unroll
-            for (int j = 0; j < GPW; ++j) {
-                const int G8 = w + NW * j;
-                if (G8 < ng) {
-                    const int ra = 8 * G8 + rho;
-                    const float2 x0 = *reinterpret_cast<const float2*>(S + sw64(ra, c2));
-                    const float2 x1 = *reinterpret_cast<const float2*>(S + sw64(ra + 2, c2));
-                    const FragA A = frag_a(x0.x, x0.y, x1.x, x1.y);
-#pragma unroll
-                    for (int nt = 0; nt < NQ; ++nt) mma3(d[j][nt], A, prt[j][nt]);
-                }
-            }
-#pragma unroll
-            for (int nt = 0; nt < NQ; ++nt) {
-                float4 v = make_float4(d[0][nt][0], d[0][nt][1], d[0][nt][2], d[0][nt][3]);
-#pragma unroll
-                for (int j = 1; j < GPW; ++j) {
-                    v.x += d[j][nt][0]; v.y += d[j][nt][1]; v.z += d[j][nt][2]; v.w += d[j][nt][3];
-                }
-                *reinterpret_cast<float4*>(part + w * pitch + (nt * 32 + lane) * 4) = v;
-            }
-        }
-        __syncthreads();
-        FragA RA[NQ];
-        if (corr) {
-            reduce_warps(part, pitch, NQ, tot);
-            __syncthreads();
-#pragma unroll
-            for (int nt = 0; nt < NQ; ++nt) {
-                const float4 R = *reinterpret_cast<const float4*>(tot + (nt * 32 + lane) * 4);
-                RA[nt] = frag_a(R.x, R.z, R.y, R.w);
-            }
-        }
-        float* Bi = Bst + (int64_t)i * mp * np + b0 + c2;
-#pragma unroll
-        for (int j = 0; j < GPW; ++j) {
-            const int G8 = w + NW * j;
-            if (G8 < ng) {
-                const int ra = 8 * G8 + rho, rb = ra + 2;
-                float c[4] = {0.f, 0.f, 0.f, 0.f};
-                float2 x0 = make_float2(0.f, 0.f), x1 = make_float2(0.f, 0.f);
-                if (corr) {
-#pragma unroll
-                    for (int nt = 0; nt < NQ; ++nt) mma3(c, RA[nt], pcb[j][nt]);
-                    x0 = *reinterpret_cast<const float2*>(S + sw64(ra, c2));
-                    x1 = *reinterpret_cast<const float2*>(S + sw64(rb, c2));
-                }
-                float2 g0, g1;
-                if (trans) {
-                    g0 = make_float2(static_cast<float>(Gs[c2 * gpt + ra]), static_cast<float>(Gs[(c2 + 1) * gpt + ra]));
-                    g1 = make_float2(static_cast<float>(Gs[c2 * gpt + rb]), static_cast<float>(Gs[(c2 + 1) * gpt + rb]));
-                } else {
-                    g0 = GradPair<GT>::row(Gs, ra, c2);
-                    g1 = GradPair<GT>::row(Gs, rb, c2);
-                }
-                const float m0 = g0.x + (x0.x - c[0]);       // M = G + E, E = B - P_prev R
-                const float m1 = g0.y + (x0.y - c[2]);
-                const float m2 = g1.x + (x1.x - c[1]);
-                const float m3 = g1.y + (x1.y - c[3]);
-                if (write_B && colok) {
-                    if (ra < mp) __stcs(reinterpret_cast<float2*>(Bi + (int64_t)ra * np), make_float2(m0, m1));
-                    if (rb < mp) __stcs(reinterpret_cast<float2*>(Bi + (int64_t)rb * np), make_float2(m2, m3));
-                }
-                acc[j][0] += m0; acc[j][1] += m1; acc[j][2] += m2; acc[j][3] += m3;
-            }
+        const float* S = reinterpret_cast<const float*>(ring + (size_t)(i % 3) * stage);
+        const GT* Gs = reinterpret_cast<const GT*>(ring + (size_t)(i % 3) * stage + sb);
+        compose_node<GT, NQ, GPW>(S, Gs, trans, gpt, corr, prt, pcb, acc, part, pitch, tot,
+                                  Bst + (int64_t)i * mp * np + b0 + L.c2, mp, np, ng, write_B, colok, L);
+        if constexpr (TMA) {               // this warp is done with node i's slot
+            __syncwarp();
+            if (L.lane == 0) mbar_arrive(empty_s + 8 * (i % 3));
         }
     }
     if constexpr (!TMA) cp_async_wait<0>();
-    const float invN = 1.0f / static_cast<float>(N);
-    float* Mb = Mbar + b0 + c2;
-#pragma unroll
-    for (int j = 0; j < GPW; ++j) {
-        const int G8 = w + NW * j;
-#pragma unroll
-        for (int e = 0; e < 4; ++e) acc[j][e] *= invN;
-        const int ra = 8 * G8 + rho, rb = ra + 2;
-        if (G8 < ng && colok) {
-            if (ra < mp) *reinterpret_cast<float2*>(Mb + (int64_t)ra * np) = make_float2(acc[j][0], acc[j][1]);
-            if (rb < mp) *reinterpret_cast<float2*>(Mb + (int64_t)rb * np) = make_float2(acc[j][2], acc[j][3]);
-        }
-    }
-    if (!KT) {
-        if (timed_out && g.err) atomicAdd(g.err, 1);
-        return;
-    }
-
-    // ---- truncated-basis Approx-Top-r partial sums: (Mbar - Yt (Y^T Mbar)) v_j ------------------
-    // v_j: the 32 lanes draw the 32 quads (row, 4 columns) of a row group once each: lane (g, t)
-    // draws row rho + 2 (g % 2), quad g / 2 (drawn first: they need no data)
-    float4 vq[GPW];
-#pragma unroll
-    for (int j = 0; j < GPW; ++j) {
-        const int G8 = w + NW * j;
-        if (G8 < ng)
-            vq[j] = gauss4(seed, tstep, static_cast<uint32_t>(8 * G8 + rho + 2 * (gg & 1)),
-                           static_cast<uint32_t>((b0 >> 2) + (gg >> 1)), kTagLambdaV);
-    }
-    await_item(N);
-    await_item(N + 1);
-    __syncthreads();                                         // Y, Yt landed for every thread
-    const float* YF = reinterpret_cast<const float*>(ring + (size_t)(N % 3) * stage);
-    const float* YtF = reinterpret_cast<const float*>(ring + (size_t)((N + 1) % 3) * stage);
-    // the warp partials of W^T (in the slot of the last node, free once every thread is here)
-    float* wpart = wslot ? reinterpret_cast<float*>(ring + (size_t)((N + 2) % 3) * stage) : part;
-    const int wpitch = wslot ? part_pitch(KT) : pitch;
-    {
-        float d[2][4][4];                                    // two accumulators per n-tile
-#pragma unroll
-        for (int h = 0; h < 2; ++h)
-#pragma unroll
-            for (int nt = 0; nt < 4; ++nt)
-#pragma unroll
-                for (int e = 0; e < 4; ++e) d[h][nt][e] = 0.f;
-#pragma unroll
-        for (int j = 0; j < GPW; ++j) {
-            const int G8 = w + NW * j;
-            if (G8 < ng) {
-                const FragA A = frag_a(acc[j][0], acc[j][1], acc[j][2], acc[j][3]);
-#pragma unroll
-                for (int nt = 0; nt < 4; ++nt)
-                    if (nt < KT) {
-                        const float2 y = *reinterpret_cast<const float2*>(YF + (G8 * KT + nt) * 64 + 2 * lane);
-                        mma3(d[j & 1][nt], A, frag_b(y.x, y.y));
-                    }
-            }
-        }
-#pragma unroll
-        for (int nt = 0; nt < 4; ++nt)
-            if (nt < KT)
-                *reinterpret_cast<float4*>(wpart + w * wpitch + (nt * 32 + lane) * 4) =
-                    make_float4(d[0][nt][0] + d[1][nt][0], d[0][nt][1] + d[1][nt][1], d[0][nt][2] + d[1][nt][2],
-                                d[0][nt][3] + d[1][nt][3]);
-    }
-    __syncthreads();
-    reduce_warps(wpart, wpitch, KT, tot);                    // W^T = Mbar_strip^T Y
-    __syncthreads();
-    FragA WA[4];
-#pragma unroll
-    for (int nt = 0; nt < 4; ++nt)
-        if (nt < KT) {
-            const float4 W = *reinterpret_cast<const float4*>(tot + (nt * 32 + lane) * 4);
-            WA[nt] = frag_a(W.x, W.z, W.y, W.w);
-        }
-    const bool odd = (gg & 1) != 0;
-#pragma unroll
-    for (int j = 0; j < GPW; ++j) {
-        const int G8 = w + NW * j;                           // warp-uniform: shuffles below are safe
-        if (G8 < ng) {
-            float c[4] = {0.f, 0.f, 0.f, 0.f};
-#pragma unroll
-            for (int nt = 0; nt < 4; ++nt)
-                if (nt < KT) {
-                    const float2 y = *reinterpret_cast<const float2*>(YtF + (G8 * KT + nt) * 64 + 2 * lane);
-                    mma3(c, WA[nt], frag_b(y.x, y.y));
-                }
-            const float d0 = acc[j][0] - c[0], d1 = acc[j][1] - c[2];
-            const float d2 = acc[j][2] - c[1], d3 = acc[j][3] - c[3];
-            // each lane keeps the half of its quad it needs and trades the other with lane g ^ 1
-            const int ra = 8 * G8 + rho;
-            const float4 v = vq[j];
-            const float q0 = __shfl_xor_sync(0xffffffffu, odd ? v.x : v.z, 4);
-            const float q1 = __shfl_xor_sync(0xffffffffu, odd ? v.y : v.w, 4);
-            const float v0 = odd ? q0 : v.x, v1 = odd ? q1 : v.y;       // row rho
-            const float v2 = odd ? v.z : q0, v3 = odd ? v.w : q1;       // row rho + 2
-            float pa = colok ? d0 * v0 + d1 * v1 : 0.f;
-            float pb = colok ? d2 * v2 + d3 * v3 : 0.f;
-#pragma unroll
-            for (int x = 4; x < 32; x <<= 1) {
-                pa += __shfl_xor_sync(0xffffffffu, pa, x);
-                pb += __shfl_xor_sync(0xffffffffu, pb, x);
-            }
-            if (gg == 0) {
-                if (ra < mp) lam_part[(int64_t)s * mp + ra] = pa;
-                if (ra + 2 < mp) lam_part[(int64_t)s * mp + ra + 2] = pb;
-            }
-        }
+    store_mbar<GPW>(acc, N, M.Mbar + b0 + L.c2, mp, np, ng, colok, L);
+    if (KT) {
+        float4 vq[GPW];
+        lam_draw<GPW>(vq, M.seed, M.t, b0, ng, L);
+        await_item(N);
+        await_item(N + 1);
+        __syncthreads();                                     // Y, Yt landed for every thread
+        const float* YF = reinterpret_cast<const float*>(ring + (size_t)(N % 3) * stage);
+        const float* YtF = reinterpret_cast<const float*>(ring + (size_t)((N + 1) % 3) * stage);
+        // the warp partials of W^T (in the slot of the last node, free once every thread is here)
+        float* wpart = wslot ? reinterpret_cast<float*>(ring + (size_t)((N + 2) % 3) * stage) : part;
+        const int wpitch = wslot ? part_pitch(KT) : pitch;
+        lam_w_partials<GPW>(YF, KT, acc, wpart, wpitch, ng, L);
+        __syncthreads();
+        reduce_warps(wpart, wpitch, KT, tot);                // W^T = Mbar_strip^T Y
+        __syncthreads();
+        lam_finish<GPW>(YtF, KT, tot, acc, vq, M.part + (int64_t)s * mp, mp, ng, colok, L);
     }
     if (timed_out && g.err) atomicAdd(g.err, 1);
 }
@@ -592,7 +656,6 @@ __global__ void __launch_bounds__(T, 1) stream_tma_kernel(const __grid_constant_
                                                           const __grid_constant__ TmaMaps maps) {
     compose_strip<GT, NQ, true>(g, &maps);
 }
-
 // dst = src (rows x cols, row-major, ld) in fragment order, up8(rows) x up8(cols) floats:
 // block (group G8, n-tile nt) holds 64 floats, lane L = 4g + t's pair at 2L, 2L + 1.
 //   form 0 (B fragment of X^T Y):  src(8 G8 + rho(t), 8 nt + g), src(8 G8 + rho(t) + 2, 8 nt + g)
@@ -637,7 +700,7 @@ size_t mma_stream_smem_bytes(int mp, int r, int k, int lam, int gsize, int trans
     const int NT = NQ > KT ? NQ : KT;
     const int PT = lam_partials_in_slot(KT, stage) ? NQ : NT;
     const size_t bytes = 3 * stage + (size_t)NW * part_pitch(PT) * 4 + (size_t)NT * 128 * 4 + 3 * 8;
-    return tma ? bytes + 1024 : bytes;                 // room to align the base to 1024 bytes
+    return tma ? bytes + 24 + 1024 : bytes;            // empty barriers; room to align the base to 1024 bytes
 }
 
 int mma_tma_box_rows(int mp) { return tma_box_rows(mp); }

@@ -51,7 +51,7 @@ __global__ void __launch_bounds__(256) lambda_kernel(LambdaArgs a) {
         const int j = j0 + ty * 4 + u;
         float s = 0.f;
         if (j < a.mp && bq < a.np) {
-            const float4 g = gauss4(a.seed, a.t, static_cast<uint32_t>(j), static_cast<uint32_t>(bq >> 2), kTagLambdaV);
+            const float4 g = gauss4_fast(a.seed, a.t, static_cast<uint32_t>(j), static_cast<uint32_t>(bq >> 2), kTagLambdaV);
             const float gv[4] = {g.x, g.y, g.z, g.w};
 #pragma unroll
             for (int v = 0; v < 4; ++v) {

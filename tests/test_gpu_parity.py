@@ -239,3 +239,17 @@ def test_fused_kernel_shapes_lockstep(m, n, dtype, k):
     reps = lockstep(m, n, 6, 3, 5, g, dtype=dtype, tau=3, optimizer="msgd", lr=0.05, beta1=0.9, seed=6,
                     basis_rank=k)
     _assert_reports(reps)
+
+
+@pytest.mark.parametrize("m,n,dtype,k,r", [(384, 1536, "bf16", 16, 8), (200, 824, "f32", 24, 6),
+                                           (256, 768, "f32", 16, 16), (768, 256, "f32", 16, 12),
+                                           (64, 4096, "f32", 32, 8)])
+def test_tensor_core_compose_paths_lockstep(m, n, dtype, k, r):
+    """The tensor-core compose kernel's variants: tile copies with bf16 gradients, m' not a
+    multiple of 16 and a partial last strip with k = 24, two q-tiles (r = 16), the cp.async path
+    for transposed gradients with r = 12, and k = 32 at m' = 64 (epilogue partials outside the
+    ring)."""
+    g = _synthetic(m, n, 3, 24, lambda j: 1.0 / j, 0.05, 70 + m + r, dtype=dtype)
+    reps = lockstep(m, n, r, 3, 5, g, dtype=dtype, tau=3, optimizer="msgd", lr=0.05, beta1=0.9, seed=8,
+                    basis_rank=k)
+    _assert_reports(reps)
