@@ -448,6 +448,7 @@ struct StepPlan {
     const void* const* G = nullptr;
     float* X = nullptr;
     bool warm = false, refresh = false, forced = false, lam_fused = false, compressed = false;
+    bool stream_update = false;   // K1 writes Wbar and K3 streams X without re-reading Mbar (k_update.cu)
 };
 
 int check_step_args(glr_handle* h, const void* const* G, float* X) {
@@ -470,6 +471,7 @@ void plan_step(StepPlan& p) {
     h->force_refresh = false;
     p.forced = !p.warm && !p.refresh && h->has_forceJ;
     p.lam_fused = h->fused && !h->exact && !p.warm && !p.refresh && !p.forced;
+    p.stream_update = p.lam_fused && h->mma && update_stream_eligible(h->mp, h->r, h->transposed);
     p.compressed = !p.warm && !(p.refresh && h->s.refresh_mode == GLR_ALG3);
     h->forced_this_step = p.forced;
 }
@@ -529,6 +531,7 @@ int compose_fused(std::vector<StepPlan*>& plans, cudaStream_t st) {
             M.strip0 = g.total_strips; M.nstrips = h->nstrips;
             M.B = h->B; M.Pprev = h->Pprev; M.Mbar = h->Mbar;
             M.YT = h->YT; M.YtT = h->YtT; M.YF = h->YF; M.YtF = h->YtF; M.part = h->lam_part;
+            M.Wbar = p->stream_update ? h->Wbar : nullptr;
             M.seed = h->s.seed; M.t = static_cast<uint32_t>(h->t);
             for (int i = 0; i < h->N; ++i) g.G[M.g_off + i] = p->G[i];
             if (tma) {
@@ -547,6 +550,43 @@ int compose_fused(std::vector<StepPlan*>& plans, cudaStream_t st) {
         {
             PhaseScope ps(f, GLR_PH_COMPOSE, st);
             GLR_LAUNCH(f, 1, mma ? stream_group_mma(g, tma ? &maps : nullptr, smem, st) : stream_group(g, smem, st));
+        }
+        todo.swap(rest);
+    }
+    return GLR_OK;
+}
+
+// K3 for compressed steps of a truncated basis, grouped: Rbar from K1's Wbar, then one pass
+// over X and the optimizer state.
+int update_streamed(std::vector<StepPlan*>& plans, cudaStream_t st) {
+    std::vector<StepPlan*> todo(plans);
+    std::stable_sort(todo.begin(), todo.end(), heavier);
+    while (!todo.empty()) {
+        glr_handle* h0 = todo.front()->h;
+        UpdStreamGroup g{};
+        g.optimizer = h0->s.optimizer;
+        g.lr = h0->s.lr; g.beta1 = h0->s.beta1; g.beta2 = h0->s.beta2; g.eps = h0->s.eps;
+        std::vector<StepPlan*> rest;
+        for (StepPlan* p : todo) {
+            glr_handle* h = p->h;
+            if (h->s.optimizer != g.optimizer || h->s.lr != g.lr || h->s.beta1 != g.beta1 || h->s.beta2 != g.beta2 ||
+                h->s.eps != g.eps || g.nmat == kGroupMax) {
+                rest.push_back(p);
+                continue;
+            }
+            UpdStreamMat& M = g.mat[g.nmat++];
+            M.mp = h->mp; M.np = h->np; M.r = h->r; M.k = h->k; M.transposed = h->transposed;
+            M.tile0 = g.total_tiles; M.ntiles = update_stream_tiles(h->mp, h->np, h->transposed);
+            M.out0 = g.total_out;
+            g.total_out += (int64_t)h->r * h->np;
+            M.J = h->J; M.dsign = h->dsign; M.Yt = h->Yt; M.Wbar = h->Wbar; M.Mbar = h->Mbar; M.P = h->P;
+            M.Rbar = h->Rbar; M.X = p->X; M.Mo = h->Mo; M.Vo = h->Vo;
+            g.total_tiles += M.ntiles;
+        }
+        {
+            PhaseScope ps(h0, GLR_PH_UPDATE, st);
+            GLR_LAUNCH(h0, 1, update_stream_rbar(g, st));
+            GLR_LAUNCH(h0, 1, update_stream_group(g, st));
         }
         todo.swap(rest);
     }
@@ -710,7 +750,10 @@ int step_group(std::vector<StepPlan>& plans, cudaStream_t st) {
         if ((rc = select_phase(p, st)) != GLR_OK) return rc;
     for (glr_handle* h : refreshing) GLR_CK(h, cudaStreamWaitEvent(st, h->rdone, 0));
     if ((rc = select_P_grouped(plans, st)) != GLR_OK) return rc;
-    if (!fused.empty() && (rc = update_fused(fused, st)) != GLR_OK) return rc;
+    std::vector<StepPlan*> streamed, strips;
+    for (StepPlan* p : fused) (p->stream_update ? streamed : strips).push_back(p);
+    if (!streamed.empty() && (rc = update_streamed(streamed, st)) != GLR_OK) return rc;
+    if (!strips.empty() && (rc = update_fused(strips, st)) != GLR_OK) return rc;
     for (StepPlan* p : unfused)
         if ((rc = update_unfused(*p, st)) != GLR_OK) return rc;
     for (StepPlan& p : plans) finish_step(p);

@@ -212,6 +212,7 @@ struct StreamMat {
     float* B; const float* Pprev; float* Mbar;
     const float* YT; const float* YtT; float* part;   // Y^T, Yt^T (k x transposed_pitch(m')); part: nstrips x m'
     const float* YF; const float* YtF;                // Y, Yt in the tensor-core kernel's fragment order
+    float* Wbar;                                      // tensor-core kernel: W = Y^T Mbar written here when set
     uint64_t seed; uint32_t t;
 };
 struct StreamGroup {
@@ -267,6 +268,27 @@ struct UpdateGroup {
 // K3 fused: Rbar_strip = P^T Mbar_strip, Ghat = P Rbar (or Mbar), MSGD / Adam on X.
 cudaError_t update_group(const UpdateGroup& g, size_t smem_bytes, cudaStream_t st);
 size_t update_smem_bytes(int mp, int r, int BN);
+
+// K3 for compressed steps of a truncated basis (k_update.cu): Rbar = D_J (Mbar[J, :] - Yt[J, :] Wbar)
+// from K1's Wbar, then Ghat = P Rbar and MSGD / Adam streamed over X; update_stream_tiles() CTAs
+// per matrix.
+struct UpdStreamMat {
+    int mp, np, r, k, transposed;
+    int tile0, ntiles;                      // update_stream_kernel CTAs of this matrix
+    int64_t out0;                           // first Rbar output of this matrix in rbar_kernel
+    const int32_t* J; const float* dsign; const float* Yt; const float* Wbar; const float* Mbar; const float* P;
+    float* Rbar; float* X; float* Mo; float* Vo;
+};
+struct UpdStreamGroup {
+    int nmat, total_tiles, optimizer;
+    int64_t total_out;
+    float lr, beta1, beta2, eps;
+    UpdStreamMat mat[kGroupMax];
+};
+int update_stream_tiles(int mp, int np, int transposed);
+bool update_stream_eligible(int mp, int r, int transposed);
+cudaError_t update_stream_rbar(const UpdStreamGroup& g, cudaStream_t st);     // Rbar, one thread per output
+cudaError_t update_stream_group(const UpdStreamGroup& g, cudaStream_t st);    // Ghat and the optimizer
 
 // Message reported by glr_last_error(NULL) for entry points that have no handle.
 void set_global_error(const char* msg);

@@ -642,6 +642,16 @@ __device__ __forceinline__ void compose_strip(const StreamGroup& g, const TmaMap
         __syncthreads();
         reduce_warps(wpart, wpitch, KT, tot);                // W^T = Mbar_strip^T Y
         __syncthreads();
+        if (M.Wbar) {
+            // W = Y^T Mbar for K3: tot[(nt 32 + lane) 4 + e] is W[8 nt + 2t + e % 2][b0 + 2g + e / 2]
+            float* Wg = M.Wbar;
+            const int k = M.k;
+            for (int idx = tid; idx < KT * 128; idx += T) {
+                const int ln = (idx >> 2) & 31, e = idx & 3;
+                const int q = 8 * (idx >> 7) + 2 * (ln & 3) + (e & 1), col = b0 + 2 * (ln >> 2) + (e >> 1);
+                if (q < k && col < np) Wg[(int64_t)q * np + col] = tot[idx];
+            }
+        }
         lam_finish<GPW>(YtF, KT, tot, acc, vq, M.part + (int64_t)s * mp, mp, ng, colok, L);
     }
     if (timed_out && g.err) atomicAdd(g.err, 1);
