@@ -577,15 +577,12 @@ int update_streamed(std::vector<StepPlan*>& plans, cudaStream_t st) {
             UpdStreamMat& M = g.mat[g.nmat++];
             M.mp = h->mp; M.np = h->np; M.r = h->r; M.k = h->k; M.transposed = h->transposed;
             M.tile0 = g.total_tiles; M.ntiles = update_stream_tiles(h->mp, h->np, h->transposed);
-            M.out0 = g.total_out;
-            g.total_out += (int64_t)h->r * h->np;
             M.J = h->J; M.dsign = h->dsign; M.Yt = h->Yt; M.Wbar = h->Wbar; M.Mbar = h->Mbar; M.P = h->P;
             M.Rbar = h->Rbar; M.X = p->X; M.Mo = h->Mo; M.Vo = h->Vo;
             g.total_tiles += M.ntiles;
         }
         {
             PhaseScope ps(h0, GLR_PH_UPDATE, st);
-            GLR_LAUNCH(h0, 1, update_stream_rbar(g, st));
             GLR_LAUNCH(h0, 1, update_stream_group(g, st));
         }
         todo.swap(rest);
@@ -672,7 +669,7 @@ int select_P_grouped(std::vector<StepPlan>& plans, cudaStream_t st) {
     auto flush = [&]() -> int {
         if (g.nmat == 0) return GLR_OK;
         PhaseScope ps(h0, GLR_PH_SELECT, st);
-        GLR_LAUNCH(h0, 2, select_group(g, st));
+        GLR_LAUNCH(h0, 3, select_group(g, st));
         g = SelectGroup{};
         h0 = nullptr;
         return GLR_OK;
@@ -687,6 +684,10 @@ int select_P_grouped(std::vector<StepPlan>& plans, cudaStream_t st) {
         M.do_select = (!p.refresh && !p.forced) ? 1 : 0;
         M.dsign = h->exact ? nullptr : h->dsign; M.lam = h->lam; M.J = h->J;
         M.U = h->U; M.Y = h->Y; M.Yt = h->Yt; M.P = h->P;
+        M.rbar = p.stream_update ? 1 : 0; M.np = h->np;
+        M.Mbar = h->Mbar; M.Wbar = h->Wbar; M.Rbar = h->Rbar;
+        M.out0 = g.total_out;
+        g.total_out += (int64_t)h->mp * h->r + (M.rbar ? (int64_t)h->r * h->np : 0);
         if (g.nmat == kGroupMax) {
             int rc = flush();
             if (rc != GLR_OK) return rc;

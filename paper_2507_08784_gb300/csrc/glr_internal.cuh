@@ -143,9 +143,13 @@ struct SelectMat {
     int mp, r, k, mode, do_select;
     const float* dsign; float* lam; int32_t* J;
     const float* U; const float* Y; const float* Yt; float* P;
+    int rbar, np;                           // also form Rbar = P^T Mbar from Wbar (truncated basis)
+    const float* Mbar; const float* Wbar; float* Rbar;
+    int64_t out0;                           // first output of this matrix in pr_kernel
 };
 struct SelectGroup {
     int nmat;
+    int64_t total_out;
     SelectMat mat[kGroupMax];
 };
 cudaError_t select_group(const SelectGroup& g, cudaStream_t st);
@@ -269,25 +273,22 @@ struct UpdateGroup {
 cudaError_t update_group(const UpdateGroup& g, size_t smem_bytes, cudaStream_t st);
 size_t update_smem_bytes(int mp, int r, int BN);
 
-// K3 for compressed steps of a truncated basis (k_update.cu): Rbar = D_J (Mbar[J, :] - Yt[J, :] Wbar)
-// from K1's Wbar, then Ghat = P Rbar and MSGD / Adam streamed over X; update_stream_tiles() CTAs
-// per matrix.
+// K3 for compressed steps of a truncated basis (k_update.cu): with Rbar formed by the selection
+// (pr_kernel, from K1's Wbar), Ghat = P Rbar and MSGD / Adam streamed over X;
+// update_stream_tiles() CTAs per matrix.
 struct UpdStreamMat {
     int mp, np, r, k, transposed;
     int tile0, ntiles;                      // update_stream_kernel CTAs of this matrix
-    int64_t out0;                           // first Rbar output of this matrix in rbar_kernel
     const int32_t* J; const float* dsign; const float* Yt; const float* Wbar; const float* Mbar; const float* P;
     float* Rbar; float* X; float* Mo; float* Vo;
 };
 struct UpdStreamGroup {
     int nmat, total_tiles, optimizer;
-    int64_t total_out;
     float lr, beta1, beta2, eps;
     UpdStreamMat mat[kGroupMax];
 };
 int update_stream_tiles(int mp, int np, int transposed);
 bool update_stream_eligible(int mp, int r, int transposed);
-cudaError_t update_stream_rbar(const UpdStreamGroup& g, cudaStream_t st);     // Rbar, one thread per output
 cudaError_t update_stream_group(const UpdStreamGroup& g, cudaStream_t st);    // Ghat and the optimizer
 
 // Message reported by glr_last_error(NULL) for entry points that have no handle.

@@ -145,84 +145,146 @@ __global__ void build_P_kernel(int mode, int mp, int r, int k, const int32_t* J,
 }  // namespace
 
 // ------------------------------------------------------------------------------------------
-// Grouped selection: one CTA per matrix reduces its partials, runs the arg-top-r (unless J
-// was supplied) and builds P = U[:, J] for its matrix.
+// Grouped selection: lambda_reduce_kernel forms lambda-bar, select_group_kernel (one CTA per
+// matrix) the arg-top-r J, and pr_kernel (one thread per output) P = U[:, J] and, for the
+// matrices whose update streams X, Rbar = P^T Mbar from K1's Wbar.
 // ------------------------------------------------------------------------------------------
 namespace {
+__device__ __forceinline__ unsigned long long shfl_xor_u64(unsigned long long v, int m) {
+    const unsigned lo = __shfl_xor_sync(0xffffffffu, static_cast<unsigned>(v), m);
+    const unsigned hi = __shfl_xor_sync(0xffffffffu, static_cast<unsigned>(v >> 32), m);
+    return (static_cast<unsigned long long>(hi) << 32) | lo;
+}
+
+// Keys (lambda-bar_j^2 bits, ~j): distinct, larger score first and the lower index on ties.
 __global__ void __launch_bounds__(1024) select_group_kernel(const __grid_constant__ SelectGroup g) {
     extern __shared__ unsigned long long keys[];
     const SelectMat& M = g.mat[blockIdx.x];
+    if (!M.do_select) return;                                // J was supplied
     const int tid = threadIdx.x, mp = M.mp, r = M.r, nth = blockDim.x;
-    __shared__ int32_t Js[1024];
-    if (M.do_select) {
-        int npow2 = 1;
-        while (npow2 < mp) npow2 <<= 1;
-        // lambda-bar was reduced from the partials by lambda_reduce_kernel
-        for (int j = tid; j < npow2; j += nth)
-            keys[j] = j < mp ? (static_cast<unsigned long long>(__float_as_uint(M.lam[j] * M.lam[j])) << 32) |
-                                   static_cast<unsigned long long>(0xFFFFFFFFu - static_cast<uint32_t>(j))
-                             : 0ull;
+    auto key_of = [&](int j) -> unsigned long long {
+        return j < mp ? (static_cast<unsigned long long>(__float_as_uint(M.lam[j] * M.lam[j])) << 32) |
+                            static_cast<unsigned long long>(0xFFFFFFFFu - static_cast<uint32_t>(j))
+                      : 0ull;
+    };
+    auto index_of = [](unsigned long long key) { return static_cast<int32_t>(0xFFFFFFFFu - static_cast<uint32_t>(key)); };
+    if (mp <= 1024 && r <= 32) {
+        // each warp sorts its 32 keys (j = 32 w + lane) descending with a bitonic network and
+        // keeps its r largest: the top r of all keys are among these candidates
+        const int lane = tid & 31, w = tid >> 5, nw = (mp + 31) >> 5;
+        unsigned long long key = key_of(tid);
+#pragma unroll
+        for (int size = 2; size <= 32; size <<= 1)
+#pragma unroll
+            for (int stride = size >> 1; stride > 0; stride >>= 1) {
+                const unsigned long long other = shfl_xor_u64(key, stride);
+                const bool keep_max = ((lane & stride) == 0) == ((lane & size) == 0 || size == 32);
+                key = keep_max ? (key > other ? key : other) : (key < other ? key : other);
+            }
+        unsigned long long* cand = keys;                     // nw * r candidates
+        __shared__ int32_t top[32];
+        if (w < nw && lane < r) cand[w * r + lane] = key;
         __syncthreads();
-        if (mp <= 1024) {
-            // keys are distinct: j is among the r largest iff fewer than r keys exceed it
-            __shared__ unsigned char win[1024];
-            for (int j = tid; j < mp; j += nth) {
-                const unsigned long long kj = keys[j];
-                int above = 0;
-                for (int w = 0; w < mp; ++w) above += keys[w] > kj;
-                win[j] = above < r ? 1 : 0;
-            }
-            __syncthreads();
-            for (int j = tid; j < mp; j += nth) {
-                if (!win[j]) continue;
-                int pos = 0;
-                for (int w = 0; w < j; ++w) pos += win[w];
-                M.J[pos] = j;
-                Js[pos] = j;
-            }
-        } else {
-            for (int size = 2; size <= npow2; size <<= 1) {
-                for (int stride = size >> 1; stride > 0; stride >>= 1) {
-                    for (int i = tid; i < npow2; i += nth) {
-                        const int partner = i ^ stride;
-                        if (partner > i) {
-                            const bool desc = (i & size) == 0;
-                            const unsigned long long x = keys[i], y = keys[partner];
-                            if ((x < y) == desc) { keys[i] = y; keys[partner] = x; }
-                        }
-                    }
-                    __syncthreads();
-                }
-            }
-            for (int q = tid; q < r; q += nth) {
-                const uint32_t jq = 0xFFFFFFFFu - static_cast<uint32_t>(keys[q] & 0xFFFFFFFFull);
-                int rank = 0;
-                for (int w = 0; w < r; ++w)
-                    rank += (0xFFFFFFFFu - static_cast<uint32_t>(keys[w] & 0xFFFFFFFFull)) < jq;
-                M.J[rank] = static_cast<int32_t>(jq);
-                Js[rank] = static_cast<int32_t>(jq);
-            }
+        const int C = nw * r;
+        if (tid < C) {
+            const unsigned long long kc = cand[tid];
+            int above = 0;
+            for (int c = 0; c < C; ++c) above += cand[c] > kc;
+            if (above < r) top[above] = index_of(kc);        // descending rank of a winner
+        }
+        __syncthreads();
+        if (tid < r) {                                       // J in ascending index order
+            const int32_t jq = top[tid];
+            int pos = 0;
+            for (int q = 0; q < r; ++q) pos += top[q] < jq;
+            M.J[pos] = jq;
+        }
+        return;
+    }
+    int npow2 = 1;
+    while (npow2 < mp) npow2 <<= 1;
+    for (int j = tid; j < npow2; j += nth) keys[j] = key_of(j);
+    __syncthreads();
+    if (mp <= 1024) {
+        // keys are distinct: j is among the r largest iff fewer than r keys exceed it
+        __shared__ unsigned char win[1024];
+        for (int j = tid; j < mp; j += nth) {
+            const unsigned long long kj = keys[j];
+            int above = 0;
+            for (int w = 0; w < mp; ++w) above += keys[w] > kj;
+            win[j] = above < r ? 1 : 0;
+        }
+        __syncthreads();
+        for (int j = tid; j < mp; j += nth) {
+            if (!win[j]) continue;
+            int pos = 0;
+            for (int w = 0; w < j; ++w) pos += win[w];
+            M.J[pos] = j;
         }
     } else {
-        for (int q = tid; q < r; q += nth) Js[q] = M.J[q];
-    }
-    __syncthreads();
-    const int k = M.k;
-    for (int e = tid; e < mp * r; e += blockDim.x) {
-        const int aa = e / r, q = e % r;
-        const int j = Js[q];
-        float v;
-        if (M.mode == 0) {
-            v = M.U[(int64_t)aa * mp + j];
-        } else {
-            v = (aa == j) ? 1.f : 0.f;
-            const float* ya = M.Y + (int64_t)aa * k;
-            const float* yj = M.Yt + (int64_t)j * k;
-            for (int c = 0; c < k; ++c) v = fmaf(-ya[c], yj[c], v);
-            if (j < k) v *= M.dsign[j];
+        for (int size = 2; size <= npow2; size <<= 1) {
+            for (int stride = size >> 1; stride > 0; stride >>= 1) {
+                for (int i = tid; i < npow2; i += nth) {
+                    const int partner = i ^ stride;
+                    if (partner > i) {
+                        const bool desc = (i & size) == 0;
+                        const unsigned long long x = keys[i], y = keys[partner];
+                        if ((x < y) == desc) { keys[i] = y; keys[partner] = x; }
+                    }
+                }
+                __syncthreads();
+            }
         }
-        M.P[e] = v;
+        for (int q = tid; q < r; q += nth) {
+            const int32_t jq = index_of(keys[q]);
+            int rank = 0;
+            for (int w = 0; w < r; ++w) rank += index_of(keys[w]) < jq;
+            M.J[rank] = jq;
+        }
     }
+}
+
+// Output o of the group: matrix i owns [out0, out0 + m' r) for P (row-major m' x r) and, when
+// rbar is set, the next r n' for Rbar.
+__global__ void __launch_bounds__(256) pr_kernel(const __grid_constant__ SelectGroup g) {
+    const int64_t o = (int64_t)blockIdx.x * 256 + threadIdx.x;
+    int mi = 0;
+    while (mi + 1 < g.nmat && o >= g.mat[mi + 1].out0) ++mi;
+    const SelectMat& M = g.mat[mi];
+    int64_t local = o - M.out0;
+    const int mp = M.mp, r = M.r, k = M.k;
+    if (local < (int64_t)mp * r) {
+        const int aa = static_cast<int>(local / r), q = static_cast<int>(local % r);
+        const int j = M.J[q];
+        if (M.mode == 0) { M.P[local] = M.U[(int64_t)aa * mp + j]; return; }
+        // column j of (I - Y Yt^T), times d_j for the spectral columns j < k
+        float v = (aa == j) ? 1.f : 0.f;
+        const float* ya = M.Y + (int64_t)aa * k;
+        const float* yj = M.Yt + (int64_t)j * k;
+        for (int c = 0; c < k; ++c) v = fmaf(-ya[c], yj[c], v);
+        if (j < k) v *= M.dsign[j];
+        M.P[local] = v;
+        return;
+    }
+    local -= (int64_t)mp * r;
+    if (!M.rbar || local >= (int64_t)r * M.np) return;
+    // Rbar = P^T Mbar = D_J (Mbar[J, :] - Yt[J, :] Wbar) with Wbar = Y^T Mbar (truncated basis)
+    const int np = M.np;
+    const int q = static_cast<int>(local / np), c = static_cast<int>(local % np);
+    const int j = M.J[q];
+    const float* ytj = M.Yt + (int64_t)j * k;
+    const float* wc = M.Wbar + c;
+    float v = M.Mbar[(int64_t)j * np + c];
+    int kk = 0;
+    for (; kk + 4 <= k; kk += 4) {                           // four independent loads per round
+        const float w0 = wc[(int64_t)kk * np], w1 = wc[(int64_t)(kk + 1) * np];
+        const float w2 = wc[(int64_t)(kk + 2) * np], w3 = wc[(int64_t)(kk + 3) * np];
+        v = fmaf(-ytj[kk], w0, v); v = fmaf(-ytj[kk + 1], w1, v);
+        v = fmaf(-ytj[kk + 2], w2, v); v = fmaf(-ytj[kk + 3], w3, v);
+    }
+    for (; kk < k; ++kk) v = fmaf(-ytj[kk], wc[(int64_t)kk * np], v);
+    if (j < k) v *= M.dsign[j];                              // D = diag(d_0..d_{k-1}, 1, ..., 1)
+    M.Rbar[local] = v;
 }
 }  // namespace
 
@@ -250,15 +312,11 @@ __global__ void __launch_bounds__(1024) lambda_reduce_kernel(const __grid_consta
 
 cudaError_t select_group(const SelectGroup& g, cudaStream_t st) {
     if (g.nmat <= 0) return cudaSuccess;
-    {
-        int maxmp = 1;
-        for (int i = 0; i < g.nmat; ++i) maxmp = g.mat[i].mp > maxmp ? g.mat[i].mp : maxmp;
-        lambda_reduce_kernel<<<dim3((maxmp + 31) / 32, g.nmat), 1024, 0, st>>>(g);
-        cudaError_t e = cudaGetLastError();
-        if (e != cudaSuccess) return e;
-    }
     int maxmp = 1;
     for (int i = 0; i < g.nmat; ++i) maxmp = g.mat[i].mp > maxmp ? g.mat[i].mp : maxmp;
+    lambda_reduce_kernel<<<dim3((maxmp + 31) / 32, g.nmat), 1024, 0, st>>>(g);
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
     int npow2 = 1;
     while (npow2 < maxmp) npow2 <<= 1;
     static bool attr_set = false;
@@ -267,6 +325,8 @@ cudaError_t select_group(const SelectGroup& g, cudaStream_t st) {
         attr_set = true;
     }
     select_group_kernel<<<g.nmat, 1024, sizeof(unsigned long long) * npow2, st>>>(g);
+    if ((e = cudaGetLastError()) != cudaSuccess) return e;
+    pr_kernel<<<(unsigned)((g.total_out + 255) / 256), 256, 0, st>>>(g);
     return cudaGetLastError();
 }
 

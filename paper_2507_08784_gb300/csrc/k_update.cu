@@ -102,7 +102,7 @@ __global__ void __launch_bounds__(TU) update_stream_kernel(const __grid_constant
     const int c0 = (tile % ncol) * tcols, row0 = trans ? 0 : (tile / ncol) * RCH;
     const int tid = threadIdx.x;
 
-    // ---- this CTA's columns of Rbar (rbar_kernel's output) ---------------------------------------
+    // ---- this CTA's columns of Rbar (formed by the selection) --------------------------------------
     for (int idx = tid; idx < RM * tcols; idx += TU) {
         const int q = idx / tcols, cc = idx % tcols, c = c0 + cc;
         Rs[q * TC + cc] = q < r && c < np ? M.Rbar[(int64_t)q * np + c] : 0.f;
@@ -175,33 +175,6 @@ __global__ void __launch_bounds__(TU) update_stream_kernel(const __grid_constant
     }
 }
 
-// Rbar[q][c] = d_{J_q} (Mbar[J_q][c] - sum_kk Yt[J_q][kk] Wbar[kk][c]) for every matrix of the
-// group, one thread per output (matrix i owns outputs [out0, out0 + r n')).
-__global__ void __launch_bounds__(TU) rbar_kernel(const __grid_constant__ UpdStreamGroup g) {
-    const int64_t o = (int64_t)blockIdx.x * TU + threadIdx.x;
-    int mi = 0;
-    while (mi + 1 < g.nmat && o >= g.mat[mi + 1].out0) ++mi;
-    const UpdStreamMat& M = g.mat[mi];
-    const int64_t local = o - M.out0;
-    if (local >= (int64_t)M.r * M.np) return;
-    const int np = M.np, k = M.k;
-    const int q = static_cast<int>(local / np), c = static_cast<int>(local % np);
-    const int j = M.J[q];
-    const float* ytj = M.Yt + (int64_t)j * k;
-    const float* wc = M.Wbar + c;
-    float v = M.Mbar[(int64_t)j * np + c];
-    int kk = 0;
-    for (; kk + 4 <= k; kk += 4) {                           // four independent loads per round
-        const float w0 = wc[(int64_t)kk * np], w1 = wc[(int64_t)(kk + 1) * np];
-        const float w2 = wc[(int64_t)(kk + 2) * np], w3 = wc[(int64_t)(kk + 3) * np];
-        v = fmaf(-ytj[kk], w0, v); v = fmaf(-ytj[kk + 1], w1, v);
-        v = fmaf(-ytj[kk + 2], w2, v); v = fmaf(-ytj[kk + 3], w3, v);
-    }
-    for (; kk < k; ++kk) v = fmaf(-ytj[kk], wc[(int64_t)kk * np], v);
-    if (j < k) v *= M.dsign[j];                              // D = diag(d_0..d_{k-1}, 1, ..., 1)
-    M.Rbar[local] = v;
-}
-
 template <int RM>
 cudaError_t launch_update_stream(const UpdStreamGroup& g, cudaStream_t st) {
     if (g.optimizer == GLR_ADAM) update_stream_kernel<RM, true><<<g.total_tiles, TU, 0, st>>>(g);
@@ -217,12 +190,6 @@ int update_stream_tiles(int mp, int np, int transposed) {
 
 bool update_stream_eligible(int mp, int r, int transposed) {
     return r >= 1 && r <= 16 && (!transposed || (mp % 4 == 0 && mp / 4 <= TU / 2));
-}
-
-cudaError_t update_stream_rbar(const UpdStreamGroup& g, cudaStream_t st) {
-    if (g.total_out <= 0) return cudaSuccess;
-    rbar_kernel<<<(unsigned)((g.total_out + TU - 1) / TU), TU, 0, st>>>(g);
-    return cudaGetLastError();
 }
 
 cudaError_t update_stream_group(const UpdStreamGroup& g, cudaStream_t st) {
