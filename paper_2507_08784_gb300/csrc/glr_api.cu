@@ -570,7 +570,7 @@ int update_streamed(std::vector<StepPlan*>& plans, cudaStream_t st) {
         for (StepPlan* p : todo) {
             glr_handle* h = p->h;
             if (h->s.optimizer != g.optimizer || h->s.lr != g.lr || h->s.beta1 != g.beta1 || h->s.beta2 != g.beta2 ||
-                h->s.eps != g.eps || g.nmat == kGroupMax) {
+                h->s.eps != g.eps || h->transposed != h0->transposed || g.nmat == kGroupMax) {
                 rest.push_back(p);
                 continue;
             }

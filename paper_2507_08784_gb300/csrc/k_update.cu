@@ -88,14 +88,14 @@ __device__ __forceinline__ void optimizer_cols(const UpdStreamGroup& g, const Up
 // RM: r rounded up to 4 or 8 or 16 (register arrays); r itself is the matrix's.  A CTA takes a
 // tile of RCH rows x TC columns (X in its stored orientation) or all m' rows x TCT columns (X
 // transposed); each thread issues the loads of four rows (or columns) before using them.
-template <int RM, bool ADAM>
-__global__ void __launch_bounds__(TU) update_stream_kernel(const __grid_constant__ UpdStreamGroup g) {
+template <int RM, bool ADAM, bool TRANS>
+__global__ void __launch_bounds__(TU, TRANS ? 1 : 3) update_stream_kernel(const __grid_constant__ UpdStreamGroup g) {
     __shared__ __align__(16) float Rs[RM * TC];             // Rbar[q][c0 + cc]
     int mi = 0;
     while (mi + 1 < g.nmat && blockIdx.x >= static_cast<unsigned>(g.mat[mi + 1].tile0)) ++mi;
     const UpdStreamMat& M = g.mat[mi];
     const int mp = M.mp, np = M.np, r = M.r, k = M.k;
-    const bool trans = M.transposed != 0;
+    constexpr bool trans = TRANS;
     const int tcols = trans ? TCT : TC;
     const int ncol = (np + tcols - 1) / tcols;
     const int tile = blockIdx.x - M.tile0;
@@ -109,14 +109,12 @@ __global__ void __launch_bounds__(TU) update_stream_kernel(const __grid_constant
     }
     __syncthreads();
 
-    if (!trans) {
+    if constexpr (!TRANS) {
         // X is m' x n' row-major: a thread owns 4 columns of rows row0 + rl + 16 u, u < 4
         const int cq = tid & 15, rl = tid >> 4;
         const int c = c0 + 4 * cq;
         if (c >= np) return;                                 // n' % 4 == 0: the quad is whole
-        float4 rq[RM];
-#pragma unroll
-        for (int q = 0; q < RM; ++q) rq[q] = ld4(Rs + q * TC + 4 * cq);
+        const float* rs = Rs + 4 * cq;                       // Rbar[q][c..c+3] at rs + q TC
         const bool vec = (r % 4) == 0;                       // P rows are 16-byte aligned
         float gh[4][4];
 #pragma unroll
@@ -138,8 +136,9 @@ __global__ void __launch_bounds__(TU) update_stream_kernel(const __grid_constant
             for (int e = 0; e < 4; ++e) gh[u][e] = 0.f;
 #pragma unroll
             for (int q = 0; q < RM; ++q) {
-                gh[u][0] = fmaf(pv[q], rq[q].x, gh[u][0]); gh[u][1] = fmaf(pv[q], rq[q].y, gh[u][1]);
-                gh[u][2] = fmaf(pv[q], rq[q].z, gh[u][2]); gh[u][3] = fmaf(pv[q], rq[q].w, gh[u][3]);
+                const float4 rq = ld4(rs + q * TC);
+                gh[u][0] = fmaf(pv[q], rq.x, gh[u][0]); gh[u][1] = fmaf(pv[q], rq.y, gh[u][1]);
+                gh[u][2] = fmaf(pv[q], rq.z, gh[u][2]); gh[u][3] = fmaf(pv[q], rq.w, gh[u][3]);
             }
         }
         optimizer_rows<ADAM>(g, M, row0 + rl, 16, mp, (int64_t)np, c, gh);
@@ -175,10 +174,10 @@ __global__ void __launch_bounds__(TU) update_stream_kernel(const __grid_constant
     }
 }
 
-template <int RM>
+template <int RM, bool TRANS>
 cudaError_t launch_update_stream(const UpdStreamGroup& g, cudaStream_t st) {
-    if (g.optimizer == GLR_ADAM) update_stream_kernel<RM, true><<<g.total_tiles, TU, 0, st>>>(g);
-    else update_stream_kernel<RM, false><<<g.total_tiles, TU, 0, st>>>(g);
+    if (g.optimizer == GLR_ADAM) update_stream_kernel<RM, true, TRANS><<<g.total_tiles, TU, 0, st>>>(g);
+    else update_stream_kernel<RM, false, TRANS><<<g.total_tiles, TU, 0, st>>>(g);
     return cudaGetLastError();
 }
 
@@ -195,10 +194,14 @@ bool update_stream_eligible(int mp, int r, int transposed) {
 cudaError_t update_stream_group(const UpdStreamGroup& g, cudaStream_t st) {
     if (g.total_tiles <= 0) return cudaSuccess;
     int rmax = 0;
-    for (int i = 0; i < g.nmat; ++i) rmax = g.mat[i].r > rmax ? g.mat[i].r : rmax;
-    if (rmax <= 4) return launch_update_stream<4>(g, st);
-    if (rmax <= 8) return launch_update_stream<8>(g, st);
-    if (rmax <= 16) return launch_update_stream<16>(g, st);
+    for (int i = 0; i < g.nmat; ++i) {
+        rmax = g.mat[i].r > rmax ? g.mat[i].r : rmax;
+        if (g.mat[i].transposed != g.mat[0].transposed) return cudaErrorInvalidValue;   // one orientation per launch
+    }
+    const bool tr = g.mat[0].transposed != 0;
+    if (rmax <= 4) return tr ? launch_update_stream<4, true>(g, st) : launch_update_stream<4, false>(g, st);
+    if (rmax <= 8) return tr ? launch_update_stream<8, true>(g, st) : launch_update_stream<8, false>(g, st);
+    if (rmax <= 16) return tr ? launch_update_stream<16, true>(g, st) : launch_update_stream<16, false>(g, st);
     return cudaErrorInvalidValue;
 }
 
