@@ -45,7 +45,9 @@ struct glr_handle {
                              // [2] bounded device waits of the compose kernel that gave up
     float* gemm_ws = nullptr;   // split-K partial tiles of the refresh GEMMs
     cudaStream_t rstream = nullptr;            // side stream of this handle's refresh
-    cudaEvent_t rfork = nullptr, rdone = nullptr;
+    cudaEvent_t rfork = nullptr, rdone = nullptr, rpow = nullptr;
+    int pow_ok = 0;                            // refresh through the grouped power iteration (k_power.cu)
+    float *powpart = nullptr, *powG = nullptr, *powS = nullptr;
     void* Gstage = nullptr;
     // host state
     int64_t t = 0, refreshes = 0, comm = 0, state_bytes = 0, period_start = 0;
@@ -226,6 +228,71 @@ int wy_from_Q(glr_handle* h, cudaStream_t st) {
     return GLR_OK;
 }
 
+// End of a truncated refresh, with Q orthonormal and H = Q^T Mbar Mbar^T Q in Hk: Rayleigh-Ritz
+// H = W diag W^T, Q <- Q W (columns by descending Ritz value, signs fixed), then the WY form.
+int refresh_tail(glr_handle* h, cudaStream_t st) {
+    const int mp = h->mp, k = h->k;
+    GLR_LAUNCH(h, 1, jacobi_eig(h->Hk, k, h->Vk, h->evals, h->dflags + 1, st));
+    GLR_LAUNCH(h, 1, sort_fix_basis(h->evals, h->Vk, k, k, h->gram, k, h->evals_sorted, st));
+    GLR_LAUNCH(h, 1, gemm_f32(gd(mp, k, k, h->Q, k, 1, h->gram, k, 1, h->Qn, k, 1), st));
+    GLR_LAUNCH(h, 1, fix_column_signs(h->Qn, mp, k, st));
+    std::swap(h->Q, h->Qn);
+    return wy_from_Q(h, st);
+}
+
+// Truncated refreshes of several matrices through the grouped block power iteration
+// (k_power.cu): the same iteration as do_refresh (q power iterations, each half re-normalised by
+// CholeskyQR, then CholeskyQR2 and the Rayleigh-Ritz Gram), one launch per stage for all of
+// them on the first handle's side stream; the k x k tails run on each handle's own stream.
+int refresh_grouped(std::vector<glr_handle*>& hs) {
+    glr_handle* h0 = hs[0];
+    cudaStream_t s0 = h0->rstream;
+    for (glr_handle* h : hs) GLR_CK(h0, cudaStreamWaitEvent(s0, h->rfork, 0));
+    {
+        PhaseScope ps(h0, GLR_PH_REFRESH, s0);
+        PowGroup g{};
+        const int PC = pow_tile(), CH = pow_chunk();
+        int q = h0->s.power_iters;
+        for (glr_handle* h : hs) {
+            if (h->refreshes == 0 && !h->basis_from_user)
+                GLR_LAUNCH(h0, 1, random_block(h->Q, h->mp, h->k, h->s.seed, static_cast<uint32_t>(h->t), s0));
+            PowMat& M = g.mat[g.nmat++];
+            M.mp = h->mp; M.np = h->np; M.k = h->k; M.active = 1;
+            M.t0 = g.tot_t; M.nt = (h->np + PC - 1) / PC; g.tot_t += M.nt;
+            M.r0 = g.tot_r; M.nr = (h->mp + PC - 1) / PC; g.tot_r += M.nr;
+            M.n0 = g.tot_n; M.nn = (h->np + CH - 1) / CH; g.tot_n += M.nn * M.nr;
+            M.Mbar = h->Mbar; M.Q = h->Q; M.Z = h->Z; M.part = h->powpart; M.G = h->powG; M.S = h->powS;
+            M.H = h->Hk; M.flag = h->dflags + 0;
+            q = std::max(q, h->s.power_iters);
+        }
+        // a matrix with fewer power iterations than the group's maximum drops out early
+        for (int it = 0; it < q; ++it) {
+            for (int i = 0; i < g.nmat; ++i) g.mat[i].active = it < hs[i]->s.power_iters ? 1 : 0;
+            GLR_LAUNCH(h0, 1, pow_stage(g, 0, it > 0 ? 1 : 0, s0));   // Z = (Mbar^T Q) S
+            GLR_LAUNCH(h0, 1, pow_stage(g, 4, 1, s0));                // S = chol(Z^T Z)^-T
+            GLR_LAUNCH(h0, 1, pow_stage(g, 1, 0, s0));                // partials of Mbar Z
+            GLR_LAUNCH(h0, 1, pow_stage(g, 2, 0, s0));                // Q = (Mbar Z) S
+            GLR_LAUNCH(h0, 1, pow_stage(g, 4, 0, s0));                // S = chol(Q^T Q)^-T
+        }
+        for (int i = 0; i < g.nmat; ++i) g.mat[i].active = 1;
+        GLR_LAUNCH(h0, 1, pow_stage(g, 3, 1, s0));                    // CholeskyQR2: Q <- Q S ...
+        GLR_LAUNCH(h0, 1, pow_stage(g, 4, 0, s0));
+        GLR_LAUNCH(h0, 1, pow_stage(g, 3, 0, s0));                    // ... twice: orthonormal
+        GLR_LAUNCH(h0, 1, pow_stage(g, 0, 0, s0));                    // Rayleigh-Ritz: Z = Mbar^T Q
+        GLR_LAUNCH(h0, 1, pow_stage(g, 5, 1, s0));                    // H = Z^T Z
+    }
+    GLR_CK(h0, cudaEventRecord(h0->rpow, s0));
+    for (glr_handle* h : hs) {
+        if (h != h0) GLR_CK(h, cudaStreamWaitEvent(h->rstream, h0->rpow, 0));
+        PhaseScope ps(h, GLR_PH_REFRESH, h->rstream);
+        g_ws = h->gemm_ws;
+        const int rc = refresh_tail(h, h->rstream);
+        g_ws = nullptr;
+        if (rc != GLR_OK) return rc;
+    }
+    return GLR_OK;
+}
+
 // Semi-Lazy SVD refresh (Eq. SVD-P1) from Mbar.
 int do_refresh(glr_handle* h, cudaStream_t st) {
     const int mp = h->mp, np = h->np, k = h->k;
@@ -250,15 +317,10 @@ int do_refresh(glr_handle* h, cudaStream_t st) {
         if ((rc = cholqr(h, h->Q, mp, st)) != GLR_OK) return rc;
     }
     if ((rc = cholqr(h, h->Q, mp, st)) != GLR_OK) return rc;   // CholeskyQR2: orthonormal to rounding
-    // Rayleigh-Ritz: Z = Mbar^T Q, H = Z^T Z = Q^T Mbar Mbar^T Q, H = W diag W^T, Q <- Q W
+    // Rayleigh-Ritz: Z = Mbar^T Q, H = Z^T Z = Q^T Mbar Mbar^T Q
     GLR_LAUNCH(h, 1, gemm_f32(gd(np, k, mp, h->Mbar, 1, np, h->Q, k, 1, h->Z, k, 1), st));
     GLR_LAUNCH(h, 1, gemm_f32(gd(k, k, np, h->Z, 1, k, h->Z, k, 1, h->Hk, k, 1), st));
-    GLR_LAUNCH(h, 1, jacobi_eig(h->Hk, k, h->Vk, h->evals, h->dflags + 1, st));
-    GLR_LAUNCH(h, 1, sort_fix_basis(h->evals, h->Vk, k, k, h->gram, k, h->evals_sorted, st));
-    GLR_LAUNCH(h, 1, gemm_f32(gd(mp, k, k, h->Q, k, 1, h->gram, k, 1, h->Qn, k, 1), st));
-    GLR_LAUNCH(h, 1, fix_column_signs(h->Qn, mp, k, st));
-    std::swap(h->Q, h->Qn);
-    return wy_from_Q(h, st);
+    return refresh_tail(h, st);
 }
 
 // Rbar = P^T Mbar; Ghat = P Rbar; optimizer.
@@ -385,6 +447,14 @@ int glr_create(int64_t m, int64_t n, int32_t r, int32_t N, const glr_schedule* s
             const size_t frag = ((MP + 7) & ~size_t(7)) * ((K + 7) & ~size_t(7));
             A(&h->YF, frag); A(&h->YtF, frag);
         }
+        if (k <= 32 && np % 4 == 0) {          // grouped power iteration (k_power.cu)
+            const size_t KM = k <= 16 ? 16 : 32, PC = pow_tile(), CH = pow_chunk();
+            const size_t nt = (NP + PC - 1) / PC, nr = (MP + PC - 1) / PC, nn = (NP + CH - 1) / CH;
+            A(&h->powpart, nn * KM * MP);
+            A(&h->powG, std::max(nt, nr) * KM * KM);
+            A(&h->powS, K * K);
+            h->pow_ok = 1;
+        }
     }
     if (rc != GLR_OK) {
         g_create_err = h->err;
@@ -409,7 +479,8 @@ int glr_create(int64_t m, int64_t n, int32_t r, int32_t N, const glr_schedule* s
     }
     if (cudaStreamCreateWithFlags(&h->rstream, cudaStreamNonBlocking) != cudaSuccess ||
         cudaEventCreateWithFlags(&h->rfork, cudaEventDisableTiming) != cudaSuccess ||
-        cudaEventCreateWithFlags(&h->rdone, cudaEventDisableTiming) != cudaSuccess) {
+        cudaEventCreateWithFlags(&h->rdone, cudaEventDisableTiming) != cudaSuccess ||
+        cudaEventCreateWithFlags(&h->rpow, cudaEventDisableTiming) != cudaSuccess) {
         g_create_err = "could not create the refresh stream";
         free_all(h);
         delete h;
@@ -434,6 +505,7 @@ int glr_destroy(glr_handle* h) {
     if (h->rstream) cudaStreamDestroy(h->rstream);
     if (h->rfork) cudaEventDestroy(h->rfork);
     if (h->rdone) cudaEventDestroy(h->rdone);
+    if (h->rpow) cudaEventDestroy(h->rpow);
     free_all(h);
     delete h;
     return GLR_OK;
@@ -734,18 +806,22 @@ int step_group(std::vector<StepPlan>& plans, cudaStream_t st) {
     // Refreshes (Semi-Lazy SVD) of different matrices are independent: each runs on its
     // handle's side stream after the compose pass, overlapping the others and the selection
     // work of the non-refreshing matrices; the main stream joins them before P is built.
-    std::vector<glr_handle*> refreshing;
+    std::vector<glr_handle*> refreshing, grouped;
     for (StepPlan& p : plans) {
         if (!p.refresh) continue;
         glr_handle* h = p.h;
         GLR_CK(h, cudaEventRecord(h->rfork, st));
         GLR_CK(h, cudaStreamWaitEvent(h->rstream, h->rfork, 0));
-        {
+        refreshing.push_back(h);
+        if (h->pow_ok) grouped.push_back(h);
+    }
+    if (!grouped.empty() && (rc = refresh_grouped(grouped)) != GLR_OK) return rc;
+    for (glr_handle* h : refreshing) {
+        if (!h->pow_ok) {
             PhaseScope ps(h, GLR_PH_REFRESH, h->rstream);
             if ((rc = do_refresh(h, h->rstream)) != GLR_OK) return rc;
         }
         GLR_CK(h, cudaEventRecord(h->rdone, h->rstream));
-        refreshing.push_back(h);
     }
     for (StepPlan& p : plans)
         if ((rc = select_phase(p, st)) != GLR_OK) return rc;

@@ -291,6 +291,29 @@ int update_stream_tiles(int mp, int np, int transposed);
 bool update_stream_eligible(int mp, int r, int transposed);
 cudaError_t update_stream_group(const UpdStreamGroup& g, cudaStream_t st);    // Ghat and the optimizer
 
+// Grouped block power iteration of the truncated-basis refresh (k_power.cu), k <= 32.  Per
+// matrix: t0/nt column tiles of pow_tile() columns (Mbar^T Q), n0 the first of nn x nr CTAs of
+// the split-K product Mbar Z (nn chunks of pow_chunk() columns, nr row tiles of pow_tile() rows),
+// r0/nr row tiles (reduction, apply).  part holds nn x KM x m' floats, G max(nt, nr) x KM x KM
+// (KM = 16 for k <= 16, else 32); S, H are k x k.
+struct PowMat {
+    int mp, np, k, active;
+    int t0, nt, n0, nn, r0, nr;
+    const float* Mbar;
+    float* Q; float* Z; float* part; float* G; float* S; float* H;
+    int* flag;
+};
+struct PowGroup {
+    int nmat, tot_t, tot_n, tot_r;
+    PowMat mat[kGroupMax];
+};
+int pow_tile();
+int pow_chunk();
+// stage 0: Z = (Mbar^T Q) (S if arg) + Gram partials; 1: split-K partials of Mbar Z; 2: Q = (sum)
+// S + Gram partials; 3: Q <- Q S (+ Gram partials if arg); 4: S <- chol(sum of Gram partials)^-T
+// (arg: the partials of stage 0, else of stages 2/3); 5: H <- sum of the stage-0 partials.
+cudaError_t pow_stage(const PowGroup& g, int stage, int arg, cudaStream_t st);
+
 // Message reported by glr_last_error(NULL) for entry points that have no handle.
 void set_global_error(const char* msg);
 

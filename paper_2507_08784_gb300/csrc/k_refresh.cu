@@ -340,7 +340,10 @@ cudaError_t jacobi_eig(float* H, int n, float* V, float* evals, int* sweeps, cud
         attr_set = true;
     }
     const float tol = 4.f * 5.96e-8f * sqrtf(static_cast<float>(n)) + 1e-7f;
-    jacobi_kernel<<<1, 1024, smem, st>>>(H, n, V, evals, sweeps, use_smem, 40, tol);
+    // one thread per 2 x 2 block update of a round, rounded to whole warps (at most 1024)
+    const int work = n * half > half * half ? n * half : half * half;
+    const int nth = work >= 1024 ? 1024 : ((work + 31) / 32) * 32;
+    jacobi_kernel<<<1, nth, smem, st>>>(H, n, V, evals, sweeps, use_smem, 40, tol);
     return cudaGetLastError();
 }
 
