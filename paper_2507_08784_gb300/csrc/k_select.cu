@@ -69,11 +69,122 @@ __global__ void __launch_bounds__(256) lambda_kernel(LambdaArgs a) {
         if (tx == 0 && j < a.mp) a.part[(int64_t)blockIdx.x * a.mp + j] = s;
     }
 }
+
+// ---- the same partial sums for a dense basis on the tensor cores -----------------------------
+// C = U^T Mbar by warp-level TF32 MMA (mma.sync m16n8k8) in the 3xTF32 form (x = hi + lo, hi the
+// TF32 rounding of x, lo the TF32 truncation of x - hi; a b ~ a_hi b_hi + a_hi b_lo + a_lo b_hi),
+// then part[tile][j] = sum over the tile's 64 columns b of C(j, b) v_j[b].  CTA tile 64 j x 64 b,
+// K = m' in chunks of 32 staged in shared memory (row pitch 72: conflict-free fragment loads);
+// 8 warps = 4 m-tiles x 2 column halves of 4 n-tiles each.
+constexpr int LMK = 32;                 // K chunk
+constexpr int LMP = 72;                 // shared row pitch (floats)
+
+__device__ __forceinline__ void lm_split(float x, uint32_t& hi, uint32_t& lo) {
+    hi = (__float_as_uint(x) + 0x1000u) & 0xffffe000u;
+    lo = __float_as_uint(x - __uint_as_float(hi)) & 0xffffe000u;
+}
+__device__ __forceinline__ void lm_mma(float (&d)[4], uint32_t a0, uint32_t a1, uint32_t a2, uint32_t a3, uint32_t b0,
+                                       uint32_t b1) {
+    asm volatile("mma.sync.aligned.m16n8k8.row.col.f32.tf32.tf32.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, "
+                 "{%0,%1,%2,%3};\n"
+                 : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
+                 : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
+}
+
+__global__ void __launch_bounds__(256) lambda_mma_kernel(LambdaArgs a) {
+    __shared__ __align__(16) float As[LMK][LMP];             // U[p][j0 + jj]
+    __shared__ __align__(16) float Bs[LMK][LMP];             // Mbar[p][b0 + bb]
+    __shared__ float half_sum[2][LT];
+    const int j0 = blockIdx.y * LT, b0 = blockIdx.x * LT;
+    const int tid = threadIdx.x, w = tid >> 5, lane = tid & 31, g = lane >> 2, t = lane & 3;
+    const int mt = w & 3, nh = w >> 2;                        // m-tile (16 rows j), column half
+    const int mp = a.mp, np = a.np, K = a.K;
+    constexpr int EPT = LMK * LT / 256;                       // 8 entries of each chunk per thread
+    float na[EPT], nb[EPT];
+    auto fetch = [&](int p0) {
+#pragma unroll
+        for (int l = 0; l < EPT; ++l) {
+            const int e = tid + l * 256, pp = e / LT, cc = e % LT, gp = p0 + pp;
+            na[l] = gp < K && j0 + cc < mp ? a.A[(int64_t)gp * mp + j0 + cc] : 0.f;
+            nb[l] = gp < K && b0 + cc < np ? a.Bm[(int64_t)gp * np + b0 + cc] : 0.f;
+        }
+    };
+    float acc[4][4];
+#pragma unroll
+    for (int nt = 0; nt < 4; ++nt)
+#pragma unroll
+        for (int e = 0; e < 4; ++e) acc[nt][e] = 0.f;
+    fetch(0);
+    for (int p0 = 0; p0 < K; p0 += LMK) {
+        __syncthreads();
+#pragma unroll
+        for (int l = 0; l < EPT; ++l) {
+            const int e = tid + l * 256, pp = e / LT, cc = e % LT;
+            As[pp][cc] = na[l];
+            Bs[pp][cc] = nb[l];
+        }
+        __syncthreads();
+        if (p0 + LMK < K) fetch(p0 + LMK);
+#pragma unroll
+        for (int k0 = 0; k0 < LMK; k0 += 8) {
+            // A (16 j x 8 p): a0 (g, t), a1 (g + 8, t), a2 (g, t + 4), a3 (g + 8, t + 4)
+            uint32_t ah[4], al[4];
+            lm_split(As[k0 + t][mt * 16 + g], ah[0], al[0]);
+            lm_split(As[k0 + t][mt * 16 + g + 8], ah[1], al[1]);
+            lm_split(As[k0 + t + 4][mt * 16 + g], ah[2], al[2]);
+            lm_split(As[k0 + t + 4][mt * 16 + g + 8], ah[3], al[3]);
+#pragma unroll
+            for (int nt = 0; nt < 4; ++nt) {
+                // B (8 p x 8 b): b0 (t, g), b1 (t + 4, g)
+                const int bc = nh * 32 + nt * 8 + g;
+                uint32_t bh0, bl0, bh1, bl1;
+                lm_split(Bs[k0 + t][bc], bh0, bl0);
+                lm_split(Bs[k0 + t + 4][bc], bh1, bl1);
+                lm_mma(acc[nt], al[0], al[1], al[2], al[3], bh0, bh1);
+                lm_mma(acc[nt], ah[0], ah[1], ah[2], ah[3], bl0, bl1);
+                lm_mma(acc[nt], ah[0], ah[1], ah[2], ah[3], bh0, bh1);
+            }
+        }
+    }
+    // C fragment: c0 (g, 2t), c1 (g, 2t + 1), c2 (g + 8, 2t), c3 (g + 8, 2t + 1) of each n-tile
+    float s[2] = {0.f, 0.f};
+#pragma unroll
+    for (int h = 0; h < 2; ++h) {
+        const int j = j0 + mt * 16 + g + 8 * h;
+        if (j < mp) {
+#pragma unroll
+            for (int nt = 0; nt < 4; ++nt) {
+                const int bq = b0 + nh * 32 + nt * 8 + 4 * (t >> 1);   // the quad holding 2t, 2t + 1
+                if (bq < np) {
+                    const float4 v = gauss4_fast(a.seed, a.t, static_cast<uint32_t>(j), static_cast<uint32_t>(bq >> 2),
+                                                 kTagLambdaV);
+                    const bool upper = (t & 1) != 0;            // columns 2, 3 of the quad
+                    const float v0 = upper ? v.z : v.x, v1 = upper ? v.w : v.y;
+                    const int b = bq + 2 * (t & 1);
+                    if (b < np) s[h] = fmaf(acc[nt][2 * h], v0, s[h]);
+                    if (b + 1 < np) s[h] = fmaf(acc[nt][2 * h + 1], v1, s[h]);
+                }
+            }
+        }
+    }
+#pragma unroll
+    for (int h = 0; h < 2; ++h) {                             // the four lanes of a row, in order
+        s[h] += __shfl_xor_sync(0xffffffffu, s[h], 1);
+        s[h] += __shfl_xor_sync(0xffffffffu, s[h], 2);
+        if (t == 0) half_sum[nh][mt * 16 + g + 8 * h] = s[h];
+    }
+    __syncthreads();
+    for (int jj = tid; jj < LT; jj += 256) {
+        const int j = j0 + jj;
+        if (j < mp) a.part[(int64_t)blockIdx.x * mp + j] = half_sum[0][jj] + half_sum[1][jj];
+    }
+}
 }  // namespace
 
 cudaError_t lambda_partials(const LambdaArgs& a, cudaStream_t st) {
     dim3 grid(a.ntiles, (a.mp + LT - 1) / LT);
-    lambda_kernel<<<grid, 256, 0, st>>>(a);
+    if (a.mode == 0) lambda_mma_kernel<<<grid, 256, 0, st>>>(a);   // dense U: a dense contraction
+    else lambda_kernel<<<grid, 256, 0, st>>>(a);
     return cudaGetLastError();
 }
 
