@@ -196,8 +196,10 @@ def bench_mode(torch, glr, cfg, prob, basis_rank, K, Wm, dist_ctx, gsets):
 
 
 def bench_e2e(torch, glr, cfg, K, Wm, dist_ctx):
-    """Same metric through glr_step_host: pinned host gradients copied in and X copied out
-    every step, inside the timed region."""
+    """Same metric through glr_step_group_host: every step copies the N pinned host gradients
+    of every matrix in (on per-matrix copy streams, double-buffered so they overlap the previous
+    step's compute) and the updated X of every matrix out to pinned host memory, inside the
+    timed region, which ends with a device synchronise."""
     prob = W.make_problem(cfg)
     hs = make_handles(glr, cfg, cfg.basis_rank)
     host = [[g.cpu().pin_memory() for g in W.gradients_torch(prob, li, 0)] for li in range(len(cfg.shapes))]
@@ -206,8 +208,7 @@ def bench_e2e(torch, glr, cfg, K, Wm, dist_ctx):
 
     def go(k):
         for _ in range(k):
-            for h, g, x, xh in zip(hs, host, X, Xh):
-                h.step_host(g, x, xh)
+            glr.glr_step_group_host(hs, host, X, Xh)
 
     go(Wm)
     dist_ctx.barrier()

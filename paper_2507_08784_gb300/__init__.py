@@ -18,7 +18,7 @@ from . import _lib
 from ._lib import (GLR_ADAM, GLR_ALG3, GLR_ALG4, GLR_BF16, GLR_F32, GLR_MSGD, GLR_OK,  # noqa: F401
                    PHASE_NAMES, GlrProfile, GlrSchedule, GlrStats, load)
 
-__all__ = ["GlrError", "make_schedule", "glr_create", "glr_destroy", "glr_step", "glr_step_group", "glr_step_host",
+__all__ = ["GlrError", "make_schedule", "glr_create", "glr_destroy", "glr_step", "glr_step_group", "glr_step_group_host", "glr_step_host",
            "glr_refresh", "glr_get_stats", "glr_last_error", "glr_get_error", "glr_get_selection",
            "glr_get_basis", "glr_set_basis", "glr_force_selection", "glr_profile_enable",
            "glr_profile_read", "glr_select_noalloc", "GreedyLore", "load"]
@@ -85,6 +85,18 @@ def glr_step_group(handles: Sequence, G: Sequence[Sequence[torch.Tensor]], X: Se
     garr = (ctypes.c_void_p * n)(*[ctypes.addressof(a) for a in gp])
     xarr = (ctypes.c_void_p * n)(*[x.data_ptr() for x in X])
     _check(load().glr_step_group(hs, n, garr, xarr, _stream_ptr(stream)))
+
+
+def glr_step_group_host(handles: Sequence, G_host: Sequence[Sequence[torch.Tensor]], X: Sequence[torch.Tensor],
+                        X_host_out: Optional[Sequence[torch.Tensor]] = None, stream=None) -> None:
+    """One grouped step from host gradients; only enqueues the work (see glr.h)."""
+    n = len(handles)
+    hs = (ctypes.c_void_p * n)(*[h.handle if isinstance(h, GreedyLore) else h for h in handles])
+    gp = [_ptr_array(g) for g in G_host]
+    garr = (ctypes.c_void_p * n)(*[ctypes.addressof(a) for a in gp])
+    xarr = (ctypes.c_void_p * n)(*[x.data_ptr() for x in X])
+    oarr = None if X_host_out is None else (ctypes.c_void_p * n)(*[o.data_ptr() for o in X_host_out])
+    _check(load().glr_step_group_host(hs, n, garr, xarr, oarr, _stream_ptr(stream)))
 
 
 def glr_step_host(h, G_host: Sequence[torch.Tensor], X: torch.Tensor, X_host_out: Optional[torch.Tensor] = None,

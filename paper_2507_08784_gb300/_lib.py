@@ -77,6 +77,8 @@ _SIGNATURES = {
                                       ctypes.c_void_p]),
     "glr_step_host": (ctypes.c_int, [ctypes.c_void_p, _c_void_pp, ctypes.c_void_p, ctypes.c_void_p,
                                      ctypes.c_void_p]),
+    "glr_step_group_host": (ctypes.c_int, [ctypes.c_void_p, ctypes.c_int32, ctypes.c_void_p, ctypes.c_void_p,
+                                           ctypes.c_void_p, ctypes.c_void_p]),
     "glr_refresh": (ctypes.c_int, [ctypes.c_void_p]),
     "glr_get_stats": (ctypes.c_int, [ctypes.c_void_p, ctypes.POINTER(GlrStats)]),
     "glr_last_error": (ctypes.c_char_p, [ctypes.c_void_p]),

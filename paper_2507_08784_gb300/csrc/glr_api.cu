@@ -49,6 +49,12 @@ struct glr_handle {
     int pow_ok = 0;                            // refresh through the grouped power iteration (k_power.cu)
     float *powpart = nullptr, *powG = nullptr, *powS = nullptr;
     void* Gstage = nullptr;
+    // glr_step_group_host: two device staging buffers of N gradients, filled on a copy stream
+    void* Gstage2[2] = {nullptr, nullptr};
+    cudaStream_t cstream = nullptr;
+    cudaEvent_t cdone = nullptr, sfree[2] = {nullptr, nullptr};
+    bool sfree_set[2] = {false, false};
+    int host_parity = 0;
     // host state
     int64_t t = 0, refreshes = 0, comm = 0, state_bytes = 0, period_start = 0;
     bool e_zero = true, force_refresh = false, last_uncompressed = true, basis_from_user = false;
@@ -506,6 +512,9 @@ int glr_destroy(glr_handle* h) {
     if (h->rfork) cudaEventDestroy(h->rfork);
     if (h->rdone) cudaEventDestroy(h->rdone);
     if (h->rpow) cudaEventDestroy(h->rpow);
+    if (h->cdone) cudaEventDestroy(h->cdone);
+    for (cudaEvent_t e : h->sfree) if (e) cudaEventDestroy(e);
+    if (h->cstream) cudaStreamDestroy(h->cstream);
     free_all(h);
     delete h;
     return GLR_OK;
@@ -876,6 +885,7 @@ int glr_step_host(glr_handle* h, const void* const* G_host, float* X, float* X_h
         int rc = alloc(h, &p, bytes * h->N);
         if (rc != GLR_OK) return rc;
         h->Gstage = p;
+        GLR_CK(h, cudaDeviceSynchronize());      // alloc's zero fill is on the legacy stream
     }
     const void* Gd[GLR_MAX_NODES];
     for (int i = 0; i < h->N; ++i) {
@@ -889,6 +899,63 @@ int glr_step_host(glr_handle* h, const void* const* G_host, float* X, float* X_h
     if (X_host_out) {
         GLR_CK(h, cudaMemcpyAsync(X_host_out, X, sizeof(float) * h->m * h->n, cudaMemcpyDeviceToHost, st));
         GLR_CK(h, cudaStreamSynchronize(st));
+    }
+    return GLR_OK;
+}
+
+int glr_step_group_host(glr_handle* const* handles, int32_t count, const void* const* const* G_host,
+                        float* const* X, float* const* X_host_out, void* stream) {
+    if (!handles || count < 1 || !G_host || !X) return fail(nullptr, GLR_EINVAL, "null arrays or count < 1%s");
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    std::vector<std::vector<const void*>> Gd(count);
+    std::vector<const void* const*> Garr(count);
+    std::vector<int> parity(count);
+    for (int j = 0; j < count; ++j) {
+        glr_handle* h = handles[j];
+        if (!h) return fail(nullptr, GLR_EINVAL, "null handle in the group%s");
+        if (!G_host[j] || !X[j]) return fail(h, GLR_EINVAL, "null host gradient array or X%s");
+        const size_t bytes = static_cast<size_t>(h->m) * h->n * h->gsize;
+        if (!h->cstream) {
+            for (int b = 0; b < 2; ++b) {
+                char* p = nullptr;
+                const int rc = alloc(h, &p, bytes * h->N);
+                if (rc != GLR_OK) return rc;
+                h->Gstage2[b] = p;
+            }
+            if (cudaStreamCreateWithFlags(&h->cstream, cudaStreamNonBlocking) != cudaSuccess ||
+                cudaEventCreateWithFlags(&h->cdone, cudaEventDisableTiming) != cudaSuccess ||
+                cudaEventCreateWithFlags(&h->sfree[0], cudaEventDisableTiming) != cudaSuccess ||
+                cudaEventCreateWithFlags(&h->sfree[1], cudaEventDisableTiming) != cudaSuccess)
+                return fail(h, GLR_ECUDA, "could not create the host-copy stream%s");
+            // alloc's zero fill runs on the legacy default stream, which the non-blocking copy
+            // stream does not wait for: finish it before the first copy
+            GLR_CK(h, cudaDeviceSynchronize());
+        }
+        const int b = h->host_parity;
+        parity[j] = b;
+        // buffer b was last read by this handle's step two calls ago
+        if (h->sfree_set[b]) GLR_CK(h, cudaStreamWaitEvent(h->cstream, h->sfree[b], 0));
+        Gd[j].resize(h->N);
+        for (int i = 0; i < h->N; ++i) {
+            if (!G_host[j][i]) return fail(h, GLR_EINVAL, "host gradient %s is null", std::to_string(i).c_str());
+            char* dst = static_cast<char*>(h->Gstage2[b]) + bytes * i;
+            GLR_CK(h, cudaMemcpyAsync(dst, G_host[j][i], bytes, cudaMemcpyHostToDevice, h->cstream));
+            Gd[j][i] = dst;
+        }
+        GLR_CK(h, cudaEventRecord(h->cdone, h->cstream));
+        GLR_CK(h, cudaStreamWaitEvent(st, h->cdone, 0));
+        Garr[j] = Gd[j].data();
+    }
+    const int rc = glr_step_group(handles, count, Garr.data(), X, stream);
+    if (rc != GLR_OK) return rc;
+    for (int j = 0; j < count; ++j) {
+        glr_handle* h = handles[j];
+        const int b = parity[j];
+        GLR_CK(h, cudaEventRecord(h->sfree[b], st));
+        h->sfree_set[b] = true;
+        h->host_parity = b ^ 1;
+        if (X_host_out && X_host_out[j])
+            GLR_CK(h, cudaMemcpyAsync(X_host_out[j], X[j], sizeof(float) * h->m * h->n, cudaMemcpyDeviceToHost, st));
     }
     return GLR_OK;
 }

@@ -200,6 +200,40 @@ def test_step_host_matches_device_step():
 
 
 @pytest.mark.parametrize("basis_rank", [0, 16])
+def test_step_group_host_matches_step_group(basis_rank):
+    """The asynchronous grouped host step (double-buffered staging on a copy stream) gives the
+    same X, bit for bit, as glr_step_group on device gradients; the host gradient buffers are
+    rewritten between calls only after the stream has passed the step that read them."""
+    import torch
+    import paper_2507_08784_gb300 as glr
+    shapes, r, N = [(256, 128), (64, 576), (128, 1152), (130, 96)], 4, 4
+    kw = dict(tau=3, optimizer="adam", lr=1e-3, basis_rank=basis_rank)
+    dev = [glr.GreedyLore(m, n, r, N, seed=70 + j, **kw) for j, (m, n) in enumerate(shapes)]
+    hst = [glr.GreedyLore(m, n, r, N, seed=70 + j, **kw) for j, (m, n) in enumerate(shapes)]
+    Xd = [torch.zeros(m, n, device="cuda") for m, n in shapes]
+    Xg = [torch.zeros(m, n, device="cuda") for m, n in shapes]
+    Xh = [torch.zeros(m, n).pin_memory() for m, n in shapes]
+    rng = np.random.default_rng(5)
+    # two sets of pinned host gradients, alternated, so a buffer is rewritten only two steps later
+    hbuf = [[[torch.zeros(m, n).pin_memory() for _ in range(N)] for m, n in shapes] for _ in range(2)]
+    for t in range(7):
+        Gs = [[rng.standard_normal((m, n)).astype(np.float32) for _ in range(N)] for m, n in shapes]
+        if t >= 2:
+            torch.cuda.synchronize()                      # buffer t % 2 was read two steps ago
+        for j in range(len(shapes)):
+            for i in range(N):
+                hbuf[t % 2][j][i].copy_(torch.from_numpy(Gs[j][i]))
+        glr.glr_step_group(dev, [[torch.from_numpy(g).cuda() for g in Gs[j]] for j in range(len(shapes))], Xd)
+        glr.glr_step_group_host(hst, hbuf[t % 2], Xg, Xh)
+    torch.cuda.synchronize()
+    for a, b, c in zip(Xd, Xg, Xh):
+        assert torch.equal(a, b)
+        assert torch.equal(a.cpu(), c)
+    for h in dev + hst:
+        h.close()
+
+
+@pytest.mark.parametrize("basis_rank", [0, 16])
 def test_step_group_equals_single_steps(basis_rank):
     """glr_step_group batches the streaming kernels of every matrix into shared launches; the
     results must be bit-identical to stepping each handle alone."""
