@@ -73,8 +73,11 @@ def philox4x32_10(c0, c1, c2, c3, k0: int, k1: int):
 
 
 def _unit_open(x):
-    """Map a 32-bit word to (0, 1): its top 24 bits plus one half, times 2^-24 (exact in fp32)."""
-    return ((np.asarray(x, dtype=np.uint64) >> np.uint64(8)).astype(np.float64) + 0.5) * 2.0 ** -24
+    """Map a 32-bit word to (0, 1): its top 23 bits plus one half, times 2^-23.  Every value
+    (k + 1/2) 2^-23, k < 2^23, has at most 24 significant bits, so it is exact in fp32 as well
+    and lies in [2^-24, 1 - 2^-24]: fp32 and fp64 implementations draw identical uniforms, and
+    neither ever reaches 0 or 1."""
+    return ((np.asarray(x, dtype=np.uint64) >> np.uint64(9)).astype(np.float64) + 0.5) * 2.0 ** -23
 
 
 def gaussian_v(seed: int, t: int, rows: int, cols: int, tag: int = TAG_LAMBDA_V) -> np.ndarray:

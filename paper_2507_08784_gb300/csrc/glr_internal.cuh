@@ -34,8 +34,9 @@ __device__ __forceinline__ U32x4 philox4x32_10(uint32_t c0, uint32_t c1, uint32_
     return {c0, c1, c2, c3};
 }
 
+// (top 23 bits + 1/2) 2^-23: exact in fp32, in [2^-24, 1 - 2^-24]
 __device__ __forceinline__ float unit_open(uint32_t w) {
-    return (static_cast<float>(w >> 8) + 0.5f) * 5.9604644775390625e-8f;  // 2^-24
+    return (static_cast<float>(w >> 9) + 0.5f) * 1.1920928955078125e-7f;  // 2^-23
 }
 
 // The four normals of quad q = b / 4 of row j.
@@ -50,15 +51,19 @@ __device__ __forceinline__ float4 gauss4(uint64_t seed, uint32_t t, uint32_t j, 
     sincospif(2.0f * unit_open(w.w), &s1, &c1);
     return make_float4(r0 * c0, r0 * s0, r1 * c1, r1 * s1);
 }
-// The same four normals with the hardware approximations of log, sin/cos and rsqrt (abs. error
-// of a few 1e-7 per normal): the draw for the v_j of the Approx-Top-r scores, where it runs once
-// per element of every strip.  cos/sin(2 pi u) are taken as -cos/-sin(pi (2u - 1)), whose
-// argument lies in [-pi, pi), the range of the approximations' stated accuracy.
+// The same four normals with the hardware approximations of log, sin/cos and rsqrt: the draw for
+// the v_j of the Approx-Top-r scores, where it runs once per element of every strip.  The
+// approximate log has an absolute error of a few 1e-7 on [1/2, 2], so for u within ~1e-6 of 1
+// -2 log u may come out as 0 or slightly negative; it is clamped to a tiny positive value
+// (radius ~0 instead of at most ~1e-3), which keeps every normal finite.  Elsewhere the error is
+// a few 1e-7 per normal.  cos/sin(2 pi u) are taken as -cos/-sin(pi (2u - 1)), whose argument
+// lies in [-pi, pi), the range of the approximations' stated accuracy.
 __device__ __forceinline__ float4 gauss4_fast(uint64_t seed, uint32_t t, uint32_t j, uint32_t q, uint32_t tag) {
     const U32x4 w = philox4x32_10(q, j, t, tag, static_cast<uint32_t>(seed),
                                   static_cast<uint32_t>(seed >> 32));
     constexpr float kPi = 3.14159265358979323846f;
-    const float e0 = -2.0f * __logf(unit_open(w.x)), e1 = -2.0f * __logf(unit_open(w.z));   // > 0
+    const float e0 = fmaxf(-2.0f * __logf(unit_open(w.x)), 1e-30f);
+    const float e1 = fmaxf(-2.0f * __logf(unit_open(w.z)), 1e-30f);
     const float r0 = e0 * rsqrtf(e0), r1 = e1 * rsqrtf(e1);
     float s0, c0, s1, c1;
     __sincosf(kPi * fmaf(2.0f, unit_open(w.y), -1.0f), &s0, &c0);

@@ -1,0 +1,182 @@
+"""GPU checks at the full matrix sizes of the large workloads (marked gpu).
+
+Algorithm 3 matrices (the d = 2048 decoder's 5632 x 2048 FFN matrix with bf16 gradients and
+Adam; the d = 4096 decoder's 11008 x 4096 FFN matrix, r = 128, k = 256) run three steps through
+the C ABI against expected values from the oracle's building blocks alone, applied to the same
+gradients in the order of Algorithm 3.  The oracle's whole-step routine would form u_j^T M_i for
+every node (about 1.5 TFLOP per step in fp64 at these sizes), so lambda-bar is formed once on the
+node mean instead, which the oracle's pins show equal to the node mean of the per-node lambdas:
+
+* the refresh basis is the oracle's SVD of its own Mbar, completed by its Householder routine,
+  and is copied into the device after the refresh step (glr_set_basis), so both sides select
+  from one U in the compressed steps;
+* lambda-bar by the oracle's Algorithm 2 with its v_j draws, J by its arg-top-r, P = U[:, J],
+  R_i = P^T M_i, E_i = M_i - P R_i, Ghat = P Rbar, and its MSGD / Adam on X.
+
+No device value enters the oracle side.  The device's own refresh (power iteration from a
+random start) is checked for orthonormality and for the energy of Mbar it captures relative to
+the exact top-k singular subspace (the spectra have no gap at k, so the subspace itself is not
+compared).  The refresh-stress matrix (4096 x 11008, a refresh in every step under Algorithm 4)
+compresses with the basis it has just computed, so it is checked by properties that hold for
+any basis: P^T P = I, Rbar = P^T Mbar, the per-step error-feedback balance
+E_i(t) + P R_i(t) = G_i(t) + E_i(t - 1) (Eq. ef1, ef2), and the optimizer applied to Ghat = P Rbar.
+
+Tolerances: 1e-5 relative Frobenius for fp32 arithmetic on bf16-exact inputs, 1e-4 for
+lambda-bar (sums of n' products) and for X under Adam (the update divides by sqrt(V) + eps).
+"""
+import numpy as np
+import pytest
+
+import workloads as W
+from oracle import greedylore as O
+from tests._harness import rel, same_selection
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _lib():
+    torch = pytest.importorskip("torch")
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    import __graft_entry__
+    __graft_entry__.build()
+
+
+def _node_grads(prob, li, t, transposed):
+    """The device gradients of step t and the same values oriented m' x n' in fp64."""
+    Gd = W.gradients_torch(prob, li, t)
+    G = np.stack([g.float().cpu().numpy() for g in Gd]).astype(np.float64)
+    return Gd, (np.swapaxes(G, 1, 2) if transposed else G)
+
+
+def _handle(glr, cfg, li, seed, tau, mode):
+    m, n = cfg.shapes[li]
+    return glr.GreedyLore(m, n, cfg.r, cfg.N, tau=tau, refresh_mode=mode, optimizer=cfg.optimizer, lr=cfg.lr,
+                          beta1=cfg.beta1, beta2=cfg.beta2, eps=cfg.eps, seed=seed, basis_rank=cfg.basis_rank,
+                          power_iters=cfg.power_iters, grad_dtype=cfg.grad_dtype)
+
+
+def _check_refresh(dev, Mbar, s, k, t):
+    """The device's own refresh: an orthogonal U whose first k columns hold nearly all of the
+    top-k energy of Mbar (s: the exact singular values)."""
+    Ud = dev.basis().double().cpu().numpy()
+    mp = Ud.shape[0]
+    assert np.abs(Ud.T @ Ud - np.eye(mp)).max() < 1e-4, f"step {t}: refresh basis not orthogonal"
+    cap = np.linalg.norm(Ud[:, :k].T @ Mbar) ** 2 / np.sum(s[:k] ** 2)
+    assert cap > 0.97, f"step {t}: refresh captures {cap:.4f} of the top-{k} energy"
+    return Ud
+
+
+def _optimizer(cfg, Xo, Mo, Vo, Gh):
+    if cfg.optimizer == "adam":
+        return O.adam_update(Xo, Mo, Vo, Gh, cfg.lr, cfg.beta1, cfg.beta2, cfg.eps)
+    Xo, Mo = O.msgd_update(Xo, Mo, Gh, cfg.lr, cfg.beta1)
+    return Xo, Mo, Vo
+
+
+@pytest.mark.parametrize("name,li", [("cfg3_llama_d2048", 4), ("cfg5_llama_d4096", 4)])
+def test_full_size_algorithm3_steps(name, li):
+    import torch
+    import paper_2507_08784_gb300 as glr
+
+    cfg = W.config(name)
+    prob = W.make_problem(cfg)
+    m, n = cfg.shapes[li]
+    transposed = m > n
+    mp, npr = min(m, n), max(m, n)
+    r, N, k = cfg.r, cfg.N, cfg.basis_rank
+    seed = 4242 + li
+    dev = _handle(glr, cfg, li, seed, cfg.tau, "alg3")
+    x_tol = 1e-4 if cfg.optimizer == "adam" else 1e-5
+    X = torch.zeros(m, n, device="cuda")
+    Xo, Mo, Vo = np.zeros((m, n)), np.zeros((m, n)), np.zeros((m, n))
+    E = np.zeros((N, mp, npr))
+    U = None
+    try:
+        for t in range(3):
+            Gd, G = _node_grads(prob, li, t, transposed)
+            M = G + E                                         # Algorithm 3: G_i + E_i
+            Mbar = M.mean(axis=0)
+            dev.step(Gd, X)
+            torch.cuda.synchronize()
+            J, P, Rbar, lam, Mbar_d = dev.selection()
+            assert rel(Mbar_d.cpu().numpy(), Mbar) <= 1e-5, f"step {t}: Mbar"
+            if t % cfg.tau == 0:                              # refresh: uncompressed mean, E reset
+                U, s = O.left_singular_basis(Mbar)
+                _check_refresh(dev, Mbar, s, k, t)
+                U = O.householder_complement(U[:, :k])
+                dev.set_basis(torch.from_numpy(np.ascontiguousarray(U[:, :k])).float().cuda())
+                assert np.all(J == -1)
+                Ghat = Mbar
+                E = np.zeros_like(E)
+            else:
+                V = O.gaussian_v(seed, t, mp, npr)
+                lam_o = O.approx_top_r_lambda([Mbar], U, V)   # = node mean of u_j^T M_i v_j
+                assert rel(lam.cpu().numpy(), lam_o) <= 1e-4, f"step {t}: lambda-bar"
+                Jo = O.argtop_r(lam_o ** 2, r)
+                ok = same_selection(J, Jo, lam_o, 1e-4)
+                assert ok, f"step {t}: selection differs beyond near-ties"
+                if ok == "tie":
+                    break                                     # the runs legitimately diverge
+                Po = U[:, Jo]
+                assert rel(P.cpu().numpy(), Po) <= 1e-5, f"step {t}: P"
+                R = Po.T @ M                                  # R_i = P^T M_i (batched over i)
+                E = M - Po @ R                                # E_i = M_i - P R_i
+                Rb = R.mean(axis=0)                           # the All-Reduce
+                assert rel(Rbar.cpu().numpy(), Rb) <= 1e-5, f"step {t}: Rbar"
+                for i in (0, N - 1):
+                    Ed = dev.error(i).double().cpu().numpy()
+                    scale = np.linalg.norm(E[i]) + 0.1 * np.linalg.norm(M[i])
+                    assert np.linalg.norm(Ed - E[i]) <= 1e-5 * scale, f"step {t}: E_{i}"
+                Ghat = Po @ Rb
+            Xo, Mo, Vo = _optimizer(cfg, Xo, Mo, Vo, np.swapaxes(Ghat, 0, 1) if transposed else Ghat)
+            assert rel(X.cpu().numpy(), Xo) <= x_tol, f"step {t}: X"
+    finally:
+        dev.close()
+
+
+def test_full_size_refresh_every_step_algorithm4():
+    import torch
+    import paper_2507_08784_gb300 as glr
+
+    cfg = W.config("cfg4_refresh")
+    prob = W.make_problem(cfg)
+    li = 0
+    m, n = cfg.shapes[li]
+    transposed = m > n
+    mp, npr = min(m, n), max(m, n)
+    r, N, k = cfg.r, cfg.N, cfg.basis_rank
+    dev = _handle(glr, cfg, li, 77, 1, "alg4")
+    X = torch.zeros(m, n, device="cuda")
+    Eprev = [np.zeros((mp, npr)) for _ in range(N)]
+    Mo = np.zeros((m, n))
+    try:
+        for t in range(3):
+            Gd, G = _node_grads(prob, li, t, transposed)
+            Xprev = X.double().cpu().numpy()
+            dev.step(Gd, X)
+            torch.cuda.synchronize()
+            J, P, Rbar, lam, Mbar_d = dev.selection()
+            assert np.array_equal(J, np.arange(r)), f"step {t}: Algorithm 4 takes U[:, :r]"
+            Mbar = np.mean([G[i] + Eprev[i] for i in range(N)], axis=0)
+            assert rel(Mbar_d.cpu().numpy(), Mbar) <= 1e-5, f"step {t}: Mbar"
+            _, s, _ = np.linalg.svd(Mbar, full_matrices=False)
+            Ud = _check_refresh(dev, Mbar, s, k, t)
+            Pd = P.double().cpu().numpy()
+            assert rel(Pd, Ud[:, :r]) <= 1e-6, f"step {t}: P = U[:, :r]"
+            assert np.abs(Pd.T @ Pd - np.eye(r)).max() < 1e-4
+            Rb = Pd.T @ Mbar
+            assert rel(Rbar.cpu().numpy(), Rb) <= 1e-5, f"step {t}: Rbar = P^T Mbar"
+            for i in (0, N - 1):                              # E_i(t) + P R_i(t) = G_i(t) + E_i(t-1)
+                Mi = G[i] + Eprev[i]
+                Ed = dev.error(i).double().cpu().numpy()
+                sent = Pd @ (Pd.T @ Mi)
+                assert np.linalg.norm(Ed + sent - Mi) <= 1e-5 * np.linalg.norm(Mi), f"step {t}: EF balance {i}"
+            Eprev = [dev.error(i).double().cpu().numpy() for i in range(N)]
+            Ghat = Pd @ Rb
+            Gh = np.swapaxes(Ghat, 0, 1) if transposed else Ghat
+            Xo, Mo = O.msgd_update(Xprev, Mo, Gh, cfg.lr, cfg.beta1)
+            assert rel(X.cpu().numpy(), Xo) <= 1e-5, f"step {t}: X"
+    finally:
+        dev.close()

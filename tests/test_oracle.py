@@ -36,6 +36,17 @@ def test_philox_known_answers():
         assert [int(x) for x in out] == [int(x, 16) for x in case["out"]]
 
 
+def test_unit_open_is_exact_in_fp32_and_open():
+    """The word-to-uniform map stays inside (0, 1) and every value it takes is an fp32 number,
+    so an fp32 implementation draws the same uniforms (the extremes and a spread of words)."""
+    words = np.array([0, 1, 511, 512, 2 ** 31 - 1, 2 ** 31, 0xFFFFFE00, 0xFFFFFFFE, 0xFFFFFFFF] +
+                     list(np.random.default_rng(3).integers(0, 2 ** 32, 10000, dtype=np.uint64)), dtype=np.uint64)
+    u = O._unit_open(words)
+    assert u.min() == 2.0 ** -24 and u.max() == 1.0 - 2.0 ** -24
+    assert np.all(u.astype(np.float32).astype(np.float64) == u)
+    assert np.all(np.isfinite(np.sqrt(-2.0 * np.log(u)))) and np.all(-2.0 * np.log(u) > 0)
+
+
 def test_gaussian_v_moments_and_freshness():
     V = O.gaussian_v(seed=12345, t=7, rows=400, cols=1001)
     n = V.size
