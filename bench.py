@@ -219,7 +219,7 @@ def bench_e2e(torch, glr, cfg, K, Wm, dist_ctx):
     return {"ms": ms, "h2d": cfg.N * cfg.matrix_elems() * gsz, "d2h": cfg.matrix_elems() * 4}
 
 
-def cpu_oracle_sample(cfg, budget_s=20.0, compressed_steps=6):
+def cpu_oracle_sample(cfg, budget_s=25.0, compressed_steps=20):
     """The oracle as it stands on the host cores: one refresh step and up to `compressed_steps`
     compressed steps of every layer matrix; the per-step time over a tau-step period is
     t_refresh + (tau - 1) * t_compressed."""
