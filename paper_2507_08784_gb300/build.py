@@ -22,6 +22,7 @@ LIB = os.path.join(LIBDIR, "libglr.so")
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-std=c++17", "-lineinfo", "-Xcompiler", "-fPIC", "--expt-relaxed-constexpr",
          "-I", INCLUDE, "-I", CSRC]
+LINK = ["-lcudart", "-lcublas"]
 
 
 def _nvcc() -> str:
@@ -37,7 +38,7 @@ def _sources():
 
 def _digest(nvcc: str) -> str:
     h = hashlib.sha256()
-    h.update(" ".join([nvcc] + ARCH + FLAGS).encode())
+    h.update(" ".join([nvcc] + ARCH + FLAGS + LINK).encode())
     files = _sources() + sorted(os.path.join(CSRC, f) for f in os.listdir(CSRC) if f.endswith((".cuh", ".h")))
     files.append(os.path.join(INCLUDE, "glr.h"))
     for f in files:
@@ -68,7 +69,7 @@ def build(force: bool = False, verbose: bool = False) -> str:
     with cf.ThreadPoolExecutor(max_workers=min(8, os.cpu_count() or 1)) as ex:
         objs = list(ex.map(compile_one, _sources()))
     tmp = LIB + ".tmp"
-    cmd = [nvcc, "-shared", "-o", tmp] + objs + ARCH + ["-lcudart"]
+    cmd = [nvcc, "-shared", "-o", tmp] + objs + ARCH + LINK
     res = subprocess.run(cmd, capture_output=True, text=True)
     if res.returncode != 0:
         raise RuntimeError(f"link failed:\n{res.stdout}\n{res.stderr}")

@@ -7,6 +7,8 @@
 #include <string>
 #include <vector>
 
+#include <cublas_v2.h>
+
 #include "glr_internal.cuh"
 
 using namespace glr;
@@ -44,6 +46,14 @@ struct glr_handle {
     int* dflags = nullptr;   // [0] Cholesky restarts, [1] Jacobi sweeps of the last refresh,
                              // [2] bounded device waits of the compose kernel that gave up
     float* gemm_ws = nullptr;   // split-K partial tiles of the refresh GEMMs
+    // Large plain products (>= 2^30 flops) go to cuBLAS: one library handle for the step stream
+    // and one for the refresh stream (a handle's workspace must not serve two streams at once).
+    cublasHandle_t cb[2] = {nullptr, nullptr};
+    // The first path with its rank-r / rank-k products as library GEMMs (set when those products
+    // are large): E_i = B_i - P_prev (P_prev^T B_i) in place, D = Mbar - Yt W and Ghat = P Rbar
+    // in mn_scratch (m' x n').
+    int tc = 0;
+    float* mn_scratch = nullptr;
     cudaStream_t rstream = nullptr;            // side stream of this handle's refresh
     cudaEvent_t rfork = nullptr, rdone = nullptr, rpow = nullptr;
     int pow_ok = 0;                            // refresh through the grouped power iteration (k_power.cu)
@@ -210,10 +220,66 @@ GemmDesc gd(int M, int N, int K, const float* A, int64_t sAi, int64_t sAp, const
     return d;
 }
 
+// A plain product C = alpha A B + beta C (GemmDesc semantics) through cuBLAS in its fp32-emulating
+// tensor-core mode (CUBLAS_COMPUTE_32F_EMULATED_16BFX9: each fp32 operand split into three bf16
+// parts, the partial products accumulated in fp32; fp32-level accuracy).  Returns 1 when the
+// strides have no column-major reading (the caller then uses gemm_f32).
+int gemm_cublas(glr_handle* h, const GemmDesc& d0, cudaStream_t st) {
+    GemmDesc d = d0;
+    if (d.sCi != 1) {                       // row-major C: form C^T = B^T A^T instead
+        if (d.sCj != 1) return 1;
+        GemmDesc t = d;
+        t.M = d.N; t.N = d.M;
+        t.A = d.B; t.sAi = d.sBj; t.sAp = d.sBp; t.sAz = d.sBz;
+        t.B = d.A; t.sBp = d.sAp; t.sBj = d.sAi; t.sBz = d.sAz;
+        t.sCi = d.sCj; t.sCj = d.sCi;
+        d = t;
+    }
+    cublasOperation_t ta, tb;
+    int64_t lda, ldb;
+    if (d.sAi == 1 && d.sAp >= d.M) { ta = CUBLAS_OP_N; lda = d.sAp; }
+    else if (d.sAp == 1 && d.sAi >= d.K) { ta = CUBLAS_OP_T; lda = d.sAi; }
+    else return 1;
+    if (d.sBp == 1 && d.sBj >= d.K) { tb = CUBLAS_OP_N; ldb = d.sBj; }
+    else if (d.sBj == 1 && d.sBp >= d.N) { tb = CUBLAS_OP_T; ldb = d.sBp; }
+    else return 1;
+    const int64_t ldc = d.sCj;
+    if (ldc < d.M || lda > INT32_MAX || ldb > INT32_MAX || ldc > INT32_MAX) return 1;
+    const int slot = st == h->rstream ? 1 : 0;
+    if (!h->cb[slot] && cublasCreate(&h->cb[slot]) != CUBLAS_STATUS_SUCCESS) {
+        h->cb[slot] = nullptr;
+        return fail(h, GLR_ECUDA, "cublasCreate failed%s");
+    }
+    if (cublasSetStream(h->cb[slot], st) != CUBLAS_STATUS_SUCCESS) return fail(h, GLR_ECUDA, "cublasSetStream failed%s");
+    const float alpha = d.alpha, beta = d.beta;
+    const cublasStatus_t cs = cublasGemmStridedBatchedEx(
+        h->cb[slot], ta, tb, d.M, d.N, d.K, &alpha, d.A, CUDA_R_32F, (int)lda, d.sAz, d.B, CUDA_R_32F, (int)ldb,
+        d.sBz, &beta, d.C, CUDA_R_32F, (int)ldc, d.sCz, d.batch, CUBLAS_COMPUTE_32F_EMULATED_16BFX9, CUBLAS_GEMM_DEFAULT);
+    if (cs != CUBLAS_STATUS_SUCCESS)
+        return fail(h, GLR_ECUDA, "cuBLAS GEMM failed with status %s", std::to_string(static_cast<int>(cs)).c_str());
+    return GLR_OK;
+}
+
+// C = alpha A B + beta C: products of at least 2^30 flops through cuBLAS (above), the rest with
+// gemm_f32 (k_stream.cu).
+int gemm(glr_handle* h, const GemmDesc& d, cudaStream_t st) {
+    if (2.0 * d.M * d.N * (double)d.K * d.batch >= 1073741824.0) {
+        const int rc = gemm_cublas(h, d, st);
+        if (rc != 1) return rc;
+    }
+    GLR_LAUNCH(h, 1, gemm_f32(d, st));
+    return GLR_OK;
+}
+#define GLR_GEMM(h, d, st)                                                                       \
+    do {                                                                                       \
+        const int gemm_rc_ = gemm((h), (d), (st));                                             \
+        if (gemm_rc_ != GLR_OK) return gemm_rc_;                                               \
+    } while (0)
+
 // A (rows x k, row-major) <- A R^{-1} with R from Cholesky of A^T A.
 int cholqr(glr_handle* h, float* A, int rows, cudaStream_t st) {
     const int k = h->k;
-    GLR_LAUNCH(h, 1, gemm_f32(gd(k, k, rows, A, 1, k, A, k, 1, h->gram, k, 1), st));
+    GLR_GEMM(h, gd(k, k, rows, A, 1, k, A, k, 1, h->gram, k, 1), st);
     GLR_LAUNCH(h, 1, cholesky(h->gram, k, h->scratch, h->dflags + 0, st));
     GLR_LAUNCH(h, 1, trsm_right_lt(A, rows, k, h->gram, st));
     return GLR_OK;
@@ -223,7 +289,7 @@ int wy_from_Q(glr_handle* h, cudaStream_t st) {
     const int mp = h->mp, k = h->k;
     GLR_LAUNCH(h, 2, householder_reconstruct(h->Q, mp, k, h->Y, h->T, h->dsign, h->scratch, st));
     // Yt = Y T^T
-    GLR_LAUNCH(h, 1, gemm_f32(gd(mp, k, k, h->Y, k, 1, h->T, 1, k, h->Yt, k, 1), st));
+    GLR_GEMM(h, gd(mp, k, k, h->Y, k, 1, h->T, 1, k, h->Yt, k, 1), st);
     // transposed copies (k x tp, zero-padded) for the fused compose kernel's lambda epilogue
     GLR_LAUNCH(h, 1, transpose_pad(h->YT, transposed_pitch(mp), h->Y, mp, k, st));
     GLR_LAUNCH(h, 1, transpose_pad(h->YtT, transposed_pitch(mp), h->Yt, mp, k, st));
@@ -240,7 +306,7 @@ int refresh_tail(glr_handle* h, cudaStream_t st) {
     const int mp = h->mp, k = h->k;
     GLR_LAUNCH(h, 1, jacobi_eig(h->Hk, k, h->Vk, h->evals, h->dflags + 1, st));
     GLR_LAUNCH(h, 1, sort_fix_basis(h->evals, h->Vk, k, k, h->gram, k, h->evals_sorted, st));
-    GLR_LAUNCH(h, 1, gemm_f32(gd(mp, k, k, h->Q, k, 1, h->gram, k, 1, h->Qn, k, 1), st));
+    GLR_GEMM(h, gd(mp, k, k, h->Q, k, 1, h->gram, k, 1, h->Qn, k, 1), st);
     GLR_LAUNCH(h, 1, fix_column_signs(h->Qn, mp, k, st));
     std::swap(h->Q, h->Qn);
     return wy_from_Q(h, st);
@@ -306,7 +372,7 @@ int do_refresh(glr_handle* h, cudaStream_t st) {
     struct Reset { ~Reset() { g_ws = nullptr; } } reset_ws;
     if (h->exact) {
         // H = Mbar Mbar^T, eigenvectors = left singular vectors, sorted by descending sigma
-        GLR_LAUNCH(h, 1, gemm_f32(gd(mp, mp, np, h->Mbar, np, 1, h->Mbar, 1, np, h->Hbuf, mp, 1), st));
+        GLR_GEMM(h, gd(mp, mp, np, h->Mbar, np, 1, h->Mbar, 1, np, h->Hbuf, mp, 1), st);
         GLR_LAUNCH(h, 1, jacobi_eig(h->Hbuf, mp, h->Vbuf, h->evals, h->dflags + 1, st));
         GLR_LAUNCH(h, 1, sort_fix_basis(h->evals, h->Vbuf, mp, mp, h->U, mp, h->evals_sorted, st));
         return GLR_OK;
@@ -317,15 +383,15 @@ int do_refresh(glr_handle* h, cudaStream_t st) {
     for (int it = 0; it < h->s.power_iters; ++it) {
         // Z = Mbar^T Q (n' x k) and Q = Mbar Z (m' x k), each re-orthonormalised by CholeskyQR
         // (one pass keeps the block well conditioned; the span is what the iteration needs)
-        GLR_LAUNCH(h, 1, gemm_f32(gd(np, k, mp, h->Mbar, 1, np, h->Q, k, 1, h->Z, k, 1), st));
+        GLR_GEMM(h, gd(np, k, mp, h->Mbar, 1, np, h->Q, k, 1, h->Z, k, 1), st);
         if ((rc = cholqr(h, h->Z, np, st)) != GLR_OK) return rc;
-        GLR_LAUNCH(h, 1, gemm_f32(gd(mp, k, np, h->Mbar, np, 1, h->Z, k, 1, h->Q, k, 1), st));
+        GLR_GEMM(h, gd(mp, k, np, h->Mbar, np, 1, h->Z, k, 1, h->Q, k, 1), st);
         if ((rc = cholqr(h, h->Q, mp, st)) != GLR_OK) return rc;
     }
     if ((rc = cholqr(h, h->Q, mp, st)) != GLR_OK) return rc;   // CholeskyQR2: orthonormal to rounding
     // Rayleigh-Ritz: Z = Mbar^T Q, H = Z^T Z = Q^T Mbar Mbar^T Q
-    GLR_LAUNCH(h, 1, gemm_f32(gd(np, k, mp, h->Mbar, 1, np, h->Q, k, 1, h->Z, k, 1), st));
-    GLR_LAUNCH(h, 1, gemm_f32(gd(k, k, np, h->Z, 1, k, h->Z, k, 1, h->Hk, k, 1), st));
+    GLR_GEMM(h, gd(np, k, mp, h->Mbar, 1, np, h->Q, k, 1, h->Z, k, 1), st);
+    GLR_GEMM(h, gd(k, k, np, h->Z, 1, k, h->Z, k, 1, h->Hk, k, 1), st);
     return refresh_tail(h, st);
 }
 
@@ -334,11 +400,21 @@ int project_and_update(glr_handle* h, float* X, cudaStream_t st) {
     const int mp = h->mp, np = h->np, r = h->r;
     {
         PhaseScope ps(h, GLR_PH_PROJECT, st);
-        GLR_LAUNCH(h, 1, gemm_f32(gd(r, np, mp, h->P, 1, r, h->Mbar, np, 1, h->Rbar, np, 1), st));
+        GLR_GEMM(h, gd(r, np, mp, h->P, 1, r, h->Mbar, np, 1, h->Rbar, np, 1), st);
     }
     PhaseScope ps(h, GLR_PH_UPDATE, st);
     UpdateArgs u{};
     u.mp = mp; u.np = np; u.r = r; u.transposed = h->transposed; u.compressed = 1;
+    if (h->tc) {
+        // Ghat = P Rbar as a library product into the scratch, then the optimizer pass reads it
+        // (the update kernel's uncompressed form, with the scratch in place of Mbar)
+        GLR_GEMM(h, gd(mp, np, r, h->P, r, 1, h->Rbar, np, 1, h->mn_scratch, np, 1), st);
+        u.compressed = 0;
+        u.optimizer = h->s.optimizer; u.lr = h->s.lr; u.beta1 = h->s.beta1; u.beta2 = h->s.beta2; u.eps = h->s.eps;
+        u.P = h->P; u.Rbar = h->Rbar; u.Mbar = h->mn_scratch; u.X = X; u.Mo = h->Mo; u.Vo = h->Vo;
+        GLR_LAUNCH(h, 1, update(u, st));
+        return GLR_OK;
+    }
     u.optimizer = h->s.optimizer; u.lr = h->s.lr; u.beta1 = h->s.beta1; u.beta2 = h->s.beta2; u.eps = h->s.eps;
     u.P = h->P; u.Rbar = h->Rbar; u.Mbar = h->Mbar; u.X = X; u.Mo = h->Mo; u.Vo = h->Vo;
     GLR_LAUNCH(h, 1, update(u, st));
@@ -438,6 +514,9 @@ int glr_create(int64_t m, int64_t n, int32_t r, int32_t N, const glr_schedule* s
     if (s->optimizer == GLR_ADAM) A(&h->Vo, (size_t)m * n);
     A(&h->dflags, 4);
     A(&h->gemm_ws, (size_t)kGemmWsFloats);
+    // the first path with library products when the rank-r products are large
+    h->tc = !h->fused && 2.0 * r * (double)mp * (double)np * N >= 1073741824.0 ? 1 : 0;
+    if (h->tc) A(&h->mn_scratch, MP * NP);
     if (exact) {
         A(&h->U, MP * MP); A(&h->Hbuf, MP * MP); A(&h->Vbuf, MP * MP);
         A(&h->evals, MP); A(&h->evals_sorted, MP);
@@ -515,6 +594,7 @@ int glr_destroy(glr_handle* h) {
     if (h->cdone) cudaEventDestroy(h->cdone);
     for (cudaEvent_t e : h->sfree) if (e) cudaEventDestroy(e);
     if (h->cstream) cudaStreamDestroy(h->cstream);
+    for (cublasHandle_t c : h->cb) if (c) cublasDestroy(c);
     free_all(h);
     delete h;
     return GLR_OK;
@@ -565,13 +645,21 @@ int compose_unfused(StepPlan& p, cudaStream_t st) {
         PhaseScope ps(h, GLR_PH_PREV_PROJECT, st);
         GemmDesc d = gd(r, np, mp, h->Pprev, 1, r, h->B, np, 1, h->Rw, np, 1);
         d.batch = N; d.sAz = 0; d.sBz = (int64_t)mp * np; d.sCz = (int64_t)r * np;
-        GLR_LAUNCH(h, 1, gemm_f32(d, st));
+        GLR_GEMM(h, d, st);
+        if (h->tc) {
+            // B_i <- E_i = B_i - P_prev R_w,i in place (one batched library product); the
+            // compose pass below then only adds G_i
+            GemmDesc e = gd(mp, np, r, h->Pprev, r, 1, h->Rw, np, 1, h->B, np, 1, -1.f, 1.f);
+            e.batch = N; e.sAz = 0; e.sBz = (int64_t)r * np; e.sCz = (int64_t)mp * np;
+            GLR_GEMM(h, e, st);
+        }
     }
     PhaseScope ps(h, GLR_PH_COMPOSE, st);
     ComposeArgs ca{};
     for (int i = 0; i < N; ++i) ca.G[i] = p.G[i];
     ca.grad_dtype = h->s.grad_dtype; ca.transposed = h->transposed;
-    ca.mp = mp; ca.np = np; ca.N = N; ca.r = r; ca.e_zero = h->e_zero ? 1 : 0; ca.write_B = p.warm ? 0 : 1;
+    ca.mp = mp; ca.np = np; ca.N = N; ca.r = h->tc ? 0 : r; ca.e_zero = h->e_zero ? 1 : 0;
+    ca.write_B = p.warm ? 0 : 1;
     ca.B = h->B; ca.Pprev = h->Pprev; ca.Rw = h->Rw; ca.Mbar = h->Mbar;
     GLR_LAUNCH(h, 1, compose(ca, st));
     return GLR_OK;
@@ -732,8 +820,15 @@ int select_phase(StepPlan& p, cudaStream_t st) {
             la.mode = 0; la.K = mp; la.A = h->U; la.Bm = h->Mbar; la.Mbar = h->Mbar;
         } else {
             const int k = h->k;
-            GLR_LAUNCH(h, 1, gemm_f32(gd(k, np, mp, h->Y, 1, k, h->Mbar, np, 1, h->Wbar, np, 1), st));  // Wbar = Y^T Mbar
+            GLR_GEMM(h, gd(k, np, mp, h->Y, 1, k, h->Mbar, np, 1, h->Wbar, np, 1), st);  // Wbar = Y^T Mbar
             la.mode = 1; la.K = k; la.A = h->Yt; la.Bm = h->Wbar; la.Mbar = h->Mbar;
+            if (h->tc) {
+                // D = Mbar - Yt Wbar as a library product into the scratch; the score kernel then
+                // only forms the row sums of D against v_j (K = 0)
+                GLR_CK(h, cudaMemcpyAsync(h->mn_scratch, h->Mbar, sizeof(float) * mp * np, cudaMemcpyDeviceToDevice, st));
+                GLR_GEMM(h, gd(mp, np, k, h->Yt, k, 1, h->Wbar, np, 1, h->mn_scratch, np, 1, -1.f, 1.f), st);
+                la.K = 0; la.Mbar = h->mn_scratch;
+            }
         }
         GLR_LAUNCH(h, 1, lambda_partials(la, st));
         h->comm += (int64_t)r * np + mp;
@@ -988,7 +1083,7 @@ int glr_get_error(glr_handle* h, int32_t i, float* E_out, void* stream) {
     const int mp = h->mp, np = h->np, r = h->r;
     float* Bi = h->B + (size_t)i * mp * np;
     float* Rwi = h->Rw + (size_t)i * r * np;
-    if (!h->e_zero) GLR_LAUNCH(h, 1, gemm_f32(gd(r, np, mp, h->Pprev, 1, r, Bi, np, 1, Rwi, np, 1), st));
+    if (!h->e_zero) GLR_GEMM(h, gd(r, np, mp, h->Pprev, 1, r, Bi, np, 1, Rwi, np, 1), st);
     GLR_LAUNCH(h, 1, materialize_error(mp, np, r, h->e_zero ? 1 : 0, Bi, h->Pprev, Rwi, E_out, st));
     return GLR_OK;
 }
