@@ -30,10 +30,14 @@ class GlrError(RuntimeError):
         self.code = code
 
 
-def _check(rc: int, handle=None):
+def _check(rc: int, handle=None, group=()):
     if rc != GLR_OK:
         lib = load()
         msg = lib.glr_last_error(handle)
+        for h in group:                       # a grouped call reports on the failing handle
+            if msg:
+                break
+            msg = lib.glr_last_error(h)
         raise GlrError(rc, msg.decode() if msg else "")
 
 
@@ -84,7 +88,7 @@ def glr_step_group(handles: Sequence, G: Sequence[Sequence[torch.Tensor]], X: Se
     gp = [_ptr_array(g) for g in G]
     garr = (ctypes.c_void_p * n)(*[ctypes.addressof(a) for a in gp])
     xarr = (ctypes.c_void_p * n)(*[x.data_ptr() for x in X])
-    _check(load().glr_step_group(hs, n, garr, xarr, _stream_ptr(stream)))
+    _check(load().glr_step_group(hs, n, garr, xarr, _stream_ptr(stream)), group=list(hs))
 
 
 def glr_step_group_host(handles: Sequence, G_host: Sequence[Sequence[torch.Tensor]], X: Sequence[torch.Tensor],
@@ -96,7 +100,7 @@ def glr_step_group_host(handles: Sequence, G_host: Sequence[Sequence[torch.Tenso
     garr = (ctypes.c_void_p * n)(*[ctypes.addressof(a) for a in gp])
     xarr = (ctypes.c_void_p * n)(*[x.data_ptr() for x in X])
     oarr = None if X_host_out is None else (ctypes.c_void_p * n)(*[o.data_ptr() for o in X_host_out])
-    _check(load().glr_step_group_host(hs, n, garr, xarr, oarr, _stream_ptr(stream)))
+    _check(load().glr_step_group_host(hs, n, garr, xarr, oarr, _stream_ptr(stream)), group=list(hs))
 
 
 def glr_step_host(h, G_host: Sequence[torch.Tensor], X: torch.Tensor, X_host_out: Optional[torch.Tensor] = None,

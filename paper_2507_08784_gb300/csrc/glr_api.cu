@@ -46,7 +46,7 @@ struct glr_handle {
     int* dflags = nullptr;   // [0] Cholesky restarts, [1] Jacobi sweeps of the last refresh,
                              // [2] bounded device waits of the compose kernel that gave up
     float* gemm_ws = nullptr;   // split-K partial tiles of the refresh GEMMs
-    // Large plain products (>= 2^30 flops) go to cuBLAS: one library handle for the step stream
+    // Large plain products (>= 2^26 flops) go to cuBLAS: one library handle for the step stream
     // and one for the refresh stream (a handle's workspace must not serve two streams at once).
     cublasHandle_t cb[2] = {nullptr, nullptr};
     // The first path with its rank-r / rank-k products as library GEMMs (set when those products
@@ -54,6 +54,7 @@ struct glr_handle {
     // in mn_scratch (m' x n').
     int tc = 0;
     float* mn_scratch = nullptr;
+    float* YtJ = nullptr;        // Yt[J, :] (r x k) for P = U[:, J] as a library product
     cudaStream_t rstream = nullptr;            // side stream of this handle's refresh
     cudaEvent_t rfork = nullptr, rdone = nullptr, rpow = nullptr;
     int pow_ok = 0;                            // refresh through the grouped power iteration (k_power.cu)
@@ -260,10 +261,10 @@ int gemm_cublas(glr_handle* h, const GemmDesc& d0, cudaStream_t st) {
     return GLR_OK;
 }
 
-// C = alpha A B + beta C: products of at least 2^30 flops through cuBLAS (above), the rest with
+// C = alpha A B + beta C: products of at least 2^26 flops through cuBLAS (above), the rest with
 // gemm_f32 (k_stream.cu).
 int gemm(glr_handle* h, const GemmDesc& d, cudaStream_t st) {
-    if (2.0 * d.M * d.N * (double)d.K * d.batch >= 1073741824.0) {
+    if (2.0 * d.M * d.N * (double)d.K * d.batch >= 67108864.0) {
         const int rc = gemm_cublas(h, d, st);
         if (rc != 1) return rc;
     }
@@ -406,13 +407,16 @@ int project_and_update(glr_handle* h, float* X, cudaStream_t st) {
     UpdateArgs u{};
     u.mp = mp; u.np = np; u.r = r; u.transposed = h->transposed; u.compressed = 1;
     if (h->tc) {
-        // Ghat = P Rbar as a library product into the scratch, then the optimizer pass reads it
-        // (the update kernel's uncompressed form, with the scratch in place of Mbar)
-        GLR_GEMM(h, gd(mp, np, r, h->P, r, 1, h->Rbar, np, 1, h->mn_scratch, np, 1), st);
+        // Ghat = P Rbar as a library product written straight into X's layout (transposed when
+        // m > n), then one elementwise optimizer pass
+        if (h->transposed)
+            GLR_GEMM(h, gd(mp, np, r, h->P, r, 1, h->Rbar, np, 1, h->mn_scratch, 1, mp), st);
+        else
+            GLR_GEMM(h, gd(mp, np, r, h->P, r, 1, h->Rbar, np, 1, h->mn_scratch, np, 1), st);
         u.compressed = 0;
         u.optimizer = h->s.optimizer; u.lr = h->s.lr; u.beta1 = h->s.beta1; u.beta2 = h->s.beta2; u.eps = h->s.eps;
         u.P = h->P; u.Rbar = h->Rbar; u.Mbar = h->mn_scratch; u.X = X; u.Mo = h->Mo; u.Vo = h->Vo;
-        GLR_LAUNCH(h, 1, update(u, st));
+        GLR_LAUNCH(h, 1, update_streamed_flat(u, st));
         return GLR_OK;
     }
     u.optimizer = h->s.optimizer; u.lr = h->s.lr; u.beta1 = h->s.beta1; u.beta2 = h->s.beta2; u.eps = h->s.eps;
@@ -515,8 +519,9 @@ int glr_create(int64_t m, int64_t n, int32_t r, int32_t N, const glr_schedule* s
     A(&h->dflags, 4);
     A(&h->gemm_ws, (size_t)kGemmWsFloats);
     // the first path with library products when the rank-r products are large
-    h->tc = !h->fused && 2.0 * r * (double)mp * (double)np * N >= 1073741824.0 ? 1 : 0;
+    h->tc = !h->fused && mp % 4 == 0 && np % 4 == 0 && 2.0 * r * (double)mp * (double)np * N >= 67108864.0 ? 1 : 0;
     if (h->tc) A(&h->mn_scratch, MP * NP);
+    if (h->tc && !exact) A(&h->YtJ, (size_t)r * k);
     if (exact) {
         A(&h->U, MP * MP); A(&h->Hbuf, MP * MP); A(&h->Vbuf, MP * MP);
         A(&h->evals, MP); A(&h->evals_sorted, MP);
@@ -661,7 +666,8 @@ int compose_unfused(StepPlan& p, cudaStream_t st) {
     ca.mp = mp; ca.np = np; ca.N = N; ca.r = h->tc ? 0 : r; ca.e_zero = h->e_zero ? 1 : 0;
     ca.write_B = p.warm ? 0 : 1;
     ca.B = h->B; ca.Pprev = h->Pprev; ca.Rw = h->Rw; ca.Mbar = h->Mbar;
-    GLR_LAUNCH(h, 1, compose(ca, st));
+    if (h->tc) GLR_LAUNCH(h, 1, compose_streamed(ca, st));
+    else GLR_LAUNCH(h, 1, compose(ca, st));
     return GLR_OK;
 }
 
@@ -823,11 +829,10 @@ int select_phase(StepPlan& p, cudaStream_t st) {
             GLR_GEMM(h, gd(k, np, mp, h->Y, 1, k, h->Mbar, np, 1, h->Wbar, np, 1), st);  // Wbar = Y^T Mbar
             la.mode = 1; la.K = k; la.A = h->Yt; la.Bm = h->Wbar; la.Mbar = h->Mbar;
             if (h->tc) {
-                // D = Mbar - Yt Wbar as a library product into the scratch; the score kernel then
-                // only forms the row sums of D against v_j (K = 0)
-                GLR_CK(h, cudaMemcpyAsync(h->mn_scratch, h->Mbar, sizeof(float) * mp * np, cudaMemcpyDeviceToDevice, st));
-                GLR_GEMM(h, gd(mp, np, k, h->Yt, k, 1, h->Wbar, np, 1, h->mn_scratch, np, 1, -1.f, 1.f), st);
-                la.K = 0; la.Mbar = h->mn_scratch;
+                // Yt Wbar as a library product into the scratch; the score kernel then forms the
+                // row sums of (Mbar - scratch) against v_j (K = 0)
+                GLR_GEMM(h, gd(mp, np, k, h->Yt, k, 1, h->Wbar, np, 1, h->mn_scratch, np, 1), st);
+                la.K = 0; la.Csub = h->mn_scratch;
             }
         }
         GLR_LAUNCH(h, 1, lambda_partials(la, st));
@@ -862,14 +867,27 @@ int select_P_grouped(std::vector<StepPlan>& plans, cudaStream_t st) {
         M.U = h->U; M.Y = h->Y; M.Yt = h->Yt; M.P = h->P;
         M.rbar = p.stream_update ? 1 : 0; M.np = h->np;
         M.Mbar = h->Mbar; M.Wbar = h->Wbar; M.Rbar = h->Rbar;
+        M.build_p = (h->tc && !h->exact) ? 0 : 1;
         M.out0 = g.total_out;
-        g.total_out += (int64_t)h->mp * h->r + (M.rbar ? (int64_t)h->r * h->np : 0);
+        g.total_out += (M.build_p ? (int64_t)h->mp * h->r : 0) + (M.rbar ? (int64_t)h->r * h->np : 0);
         if (g.nmat == kGroupMax) {
             int rc = flush();
             if (rc != GLR_OK) return rc;
         }
     }
-    return flush();
+    int rc = flush();
+    if (rc != GLR_OK) return rc;
+    // P = U[:, J] of a truncated basis with large products: (E_J - Y Yt[J, :]^T) D_J
+    for (StepPlan& p : plans) {
+        glr_handle* h = p.h;
+        if (!p.compressed || !h->tc || h->exact) continue;
+        PhaseScope ps(h, GLR_PH_SELECT, st);
+        const int mp = h->mp, r = h->r, k = h->k;
+        GLR_LAUNCH(h, 1, wy_columns_gather(h->Yt, h->J, r, k, h->YtJ, st));
+        GLR_GEMM(h, gd(mp, r, k, h->Y, k, 1, h->YtJ, 1, k, h->P, r, 1, -1.f, 0.f), st);
+        GLR_LAUNCH(h, 1, wy_columns_fix(h->P, h->J, h->dsign, mp, r, k, st));
+    }
+    return GLR_OK;
 }
 
 int update_unfused(StepPlan& p, cudaStream_t st) {

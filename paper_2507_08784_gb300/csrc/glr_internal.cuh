@@ -130,6 +130,7 @@ struct LambdaArgs {
     const float* A;         // U (dense) or Yt (wy)
     const float* Bm;        // Mbar (dense) or Wbar (wy)
     const float* Mbar;      // wy only
+    const float* Csub;      // wy only, may be null: subtracted from Mbar as well (a precomputed Yt W)
     uint64_t seed; uint32_t t;
     float* part; int ntiles;
 };
@@ -151,6 +152,7 @@ struct SelectMat {
     int rbar, np;                           // also form Rbar = P^T Mbar from Wbar (truncated basis)
     const float* Mbar; const float* Wbar; float* Rbar;
     int64_t out0;                           // first output of this matrix in pr_kernel
+    int build_p;                            // 0: the caller forms P (wy_columns_*), pr_kernel skips it
 };
 struct SelectGroup {
     int nmat;
@@ -158,6 +160,11 @@ struct SelectGroup {
     SelectMat mat[kGroupMax];
 };
 cudaError_t select_group(const SelectGroup& g, cudaStream_t st);
+// P = U[:, J] of a truncated basis U = (I - Y Yt^T) D formed around a library product:
+// wy_columns_gather writes YtJ = Yt[J, :] (r x k); the caller forms P = -Y YtJ^T (m' x r);
+// wy_columns_fix adds the identity columns e_{J_q} and scales column q by d_{J_q} (J_q < k).
+cudaError_t wy_columns_gather(const float* Yt, const int32_t* J, int r, int k, float* YtJ, cudaStream_t st);
+cudaError_t wy_columns_fix(float* P, const int32_t* J, const float* dsign, int mp, int r, int k, cudaStream_t st);
 
 // P(:, q) = column J[q] of U: dense U (mode 0) or U = (I - Y Yt^T) D (mode 1).
 cudaError_t build_P(int mode, int mp, int r, int k, const int32_t* J, const float* U,
@@ -172,6 +179,12 @@ struct UpdateArgs {
     float* X; float* Mo; float* Vo;
 };
 cudaError_t update(const UpdateArgs& a, cudaStream_t st);
+// The first path's streaming passes when its products run as library GEMMs (k_big.cu):
+// compose_streamed takes B holding E_i (the correction already applied; r unused) and needs
+// m' % 4 == n' % 4 == 0; update_streamed_flat takes Ghat in Mbar laid out like X (a.mp x a.np =
+// X's element count as two factors) and runs the optimizer element by element.
+cudaError_t compose_streamed(const ComposeArgs& a, cudaStream_t st);
+cudaError_t update_streamed_flat(const UpdateArgs& a, cudaStream_t st);
 
 // E_i = B_i - Pprev (Pprev^T B_i) given Rw_i = Pprev^T B_i  (or 0 when e_zero)
 cudaError_t materialize_error(int mp, int np, int r, int e_zero, const float* B, const float* Pprev,

@@ -58,7 +58,10 @@ __global__ void __launch_bounds__(256) lambda_kernel(LambdaArgs a) {
                 const int b = bq + v;
                 if (b < a.np) {
                     float c = acc[u][v];
-                    if (a.mode == 1) c = a.Mbar[(int64_t)j * a.np + b] - c;
+                    if (a.mode == 1) {
+                        c = a.Mbar[(int64_t)j * a.np + b] - c;
+                        if (a.Csub) c -= a.Csub[(int64_t)j * a.np + b];
+                    }
                     s = fmaf(c, gv[v], s);
                 }
             }
@@ -364,7 +367,7 @@ __global__ void __launch_bounds__(256) pr_kernel(const __grid_constant__ SelectG
     const SelectMat& M = g.mat[mi];
     int64_t local = o - M.out0;
     const int mp = M.mp, r = M.r, k = M.k;
-    if (local < (int64_t)mp * r) {
+    if (M.build_p && local < (int64_t)mp * r) {
         const int aa = static_cast<int>(local / r), q = static_cast<int>(local % r);
         const int j = M.J[q];
         if (M.mode == 0) { M.P[local] = M.U[(int64_t)aa * mp + j]; return; }
@@ -377,7 +380,7 @@ __global__ void __launch_bounds__(256) pr_kernel(const __grid_constant__ SelectG
         M.P[local] = v;
         return;
     }
-    local -= (int64_t)mp * r;
+    if (M.build_p) local -= (int64_t)mp * r;
     if (!M.rbar || local >= (int64_t)r * M.np) return;
     // Rbar = P^T Mbar = D_J (Mbar[J, :] - Yt[J, :] Wbar) with Wbar = Y^T Mbar (truncated basis)
     const int np = M.np;
@@ -437,7 +440,37 @@ cudaError_t select_group(const SelectGroup& g, cudaStream_t st) {
     }
     select_group_kernel<<<g.nmat, 1024, sizeof(unsigned long long) * npow2, st>>>(g);
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
+    if (g.total_out <= 0) return cudaSuccess;              // every P formed by the caller
     pr_kernel<<<(unsigned)((g.total_out + 255) / 256), 256, 0, st>>>(g);
+    return cudaGetLastError();
+}
+
+namespace {
+__global__ void wy_gather_kernel(const float* Yt, const int32_t* J, int r, int k, float* YtJ) {
+    const int e = blockIdx.x * blockDim.x + threadIdx.x;
+    if (e >= r * k) return;
+    const int q = e / k, c = e % k;
+    YtJ[e] = Yt[(int64_t)J[q] * k + c];
+}
+__global__ void wy_fix_kernel(float* P, const int32_t* J, const float* dsign, int mp, int r, int k) {
+    const int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+    if (e >= (int64_t)mp * r) return;
+    const int a = static_cast<int>(e / r), q = static_cast<int>(e % r);
+    const int j = J[q];
+    float v = P[e] + (a == j ? 1.f : 0.f);
+    if (j < k) v *= dsign[j];
+    P[e] = v;
+}
+}  // namespace
+
+cudaError_t wy_columns_gather(const float* Yt, const int32_t* J, int r, int k, float* YtJ, cudaStream_t st) {
+    wy_gather_kernel<<<(r * k + 255) / 256, 256, 0, st>>>(Yt, J, r, k, YtJ);
+    return cudaGetLastError();
+}
+
+cudaError_t wy_columns_fix(float* P, const int32_t* J, const float* dsign, int mp, int r, int k, cudaStream_t st) {
+    const int64_t n = (int64_t)mp * r;
+    wy_fix_kernel<<<(unsigned)((n + 255) / 256), 256, 0, st>>>(P, J, dsign, mp, r, k);
     return cudaGetLastError();
 }
 
