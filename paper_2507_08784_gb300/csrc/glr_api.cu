@@ -40,7 +40,7 @@ struct glr_handle {
     float *Mo = nullptr, *Vo = nullptr;
     float *U = nullptr, *Hbuf = nullptr, *Vbuf = nullptr, *evals = nullptr, *evals_sorted = nullptr;
     float *Q = nullptr, *Qn = nullptr, *Y = nullptr, *Yt = nullptr, *T = nullptr, *dsign = nullptr;
-    float *Wbar = nullptr, *Z = nullptr, *Hk = nullptr, *Vk = nullptr, *gram = nullptr, *scratch = nullptr;
+    float *Wbar = nullptr, *Z = nullptr, *Zn = nullptr, *Hk = nullptr, *Vk = nullptr, *gram = nullptr, *scratch = nullptr;
     float *YT = nullptr, *YtT = nullptr;   // k x transposed_pitch(m') copies of Y and Yt for the fused kernel
     float *YF = nullptr, *YtF = nullptr;   // Y and Yt in fragment order for the tensor-core kernel
     int* dflags = nullptr;   // [0] Cholesky restarts, [1] Jacobi sweeps of the last refresh,
@@ -277,12 +277,19 @@ int gemm(glr_handle* h, const GemmDesc& d, cudaStream_t st) {
         if (gemm_rc_ != GLR_OK) return gemm_rc_;                                               \
     } while (0)
 
-// A (rows x k, row-major) <- A R^{-1} with R from Cholesky of A^T A.
-int cholqr(glr_handle* h, float* A, int rows, cudaStream_t st) {
+// A (rows x k, row-major) <- A L^{-T} with L L^T = A^T A (CholeskyQR): the k x k factor and its
+// inverse in one CTA, then one product into tmp; A and tmp trade places.
+int cholqr(glr_handle* h, float*& A, float*& tmp, int rows, cudaStream_t st) {
     const int k = h->k;
     GLR_GEMM(h, gd(k, k, rows, A, 1, k, A, k, 1, h->gram, k, 1), st);
-    GLR_LAUNCH(h, 1, cholesky(h->gram, k, h->scratch, h->dflags + 0, st));
-    GLR_LAUNCH(h, 1, trsm_right_lt(A, rows, k, h->gram, st));
+    if (k > 256) {                           // the factor does not fit one CTA's shared memory
+        GLR_LAUNCH(h, 1, cholesky(h->gram, k, h->scratch, h->dflags + 0, st));
+        GLR_LAUNCH(h, 1, trsm_right_lt(A, rows, k, h->gram, st));
+        return GLR_OK;
+    }
+    GLR_LAUNCH(h, 1, chol_inverse(h->gram, k, h->scratch, h->dflags + 0, st));
+    GLR_GEMM(h, gd(rows, k, k, A, k, 1, h->scratch, k, 1, tmp, k, 1), st);
+    std::swap(A, tmp);
     return GLR_OK;
 }
 
@@ -385,11 +392,11 @@ int do_refresh(glr_handle* h, cudaStream_t st) {
         // Z = Mbar^T Q (n' x k) and Q = Mbar Z (m' x k), each re-orthonormalised by CholeskyQR
         // (one pass keeps the block well conditioned; the span is what the iteration needs)
         GLR_GEMM(h, gd(np, k, mp, h->Mbar, 1, np, h->Q, k, 1, h->Z, k, 1), st);
-        if ((rc = cholqr(h, h->Z, np, st)) != GLR_OK) return rc;
+        if ((rc = cholqr(h, h->Z, h->Zn, np, st)) != GLR_OK) return rc;
         GLR_GEMM(h, gd(mp, k, np, h->Mbar, np, 1, h->Z, k, 1, h->Q, k, 1), st);
-        if ((rc = cholqr(h, h->Q, mp, st)) != GLR_OK) return rc;
+        if ((rc = cholqr(h, h->Q, h->Qn, mp, st)) != GLR_OK) return rc;
     }
-    if ((rc = cholqr(h, h->Q, mp, st)) != GLR_OK) return rc;   // CholeskyQR2: orthonormal to rounding
+    if ((rc = cholqr(h, h->Q, h->Qn, mp, st)) != GLR_OK) return rc;   // CholeskyQR2: orthonormal to rounding
     // Rayleigh-Ritz: Z = Mbar^T Q, H = Z^T Z = Q^T Mbar Mbar^T Q
     GLR_GEMM(h, gd(np, k, mp, h->Mbar, 1, np, h->Q, k, 1, h->Z, k, 1), st);
     GLR_GEMM(h, gd(k, k, np, h->Z, 1, k, h->Z, k, 1, h->Hk, k, 1), st);
@@ -528,7 +535,7 @@ int glr_create(int64_t m, int64_t n, int32_t r, int32_t N, const glr_schedule* s
     } else {
         const size_t K = k;
         A(&h->Q, MP * K); A(&h->Qn, MP * K); A(&h->Y, MP * K); A(&h->Yt, MP * K);
-        A(&h->T, K * K); A(&h->dsign, K); A(&h->Wbar, K * NP); A(&h->Z, NP * K);
+        A(&h->T, K * K); A(&h->dsign, K); A(&h->Wbar, K * NP); A(&h->Z, NP * K); A(&h->Zn, NP * K);
         A(&h->Hk, K * K); A(&h->Vk, K * K); A(&h->gram, K * K); A(&h->scratch, K * K);
         A(&h->evals, K); A(&h->evals_sorted, K);
         A(&h->YT, K * transposed_pitch(static_cast<int>(mp)));

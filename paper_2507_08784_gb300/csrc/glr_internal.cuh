@@ -204,6 +204,9 @@ cudaError_t fix_column_signs(float* A, int rows, int cols, cudaStream_t st);
 // pivot is not positive the diagonal is shifted and the factorisation restarted (*flag =
 // number of restarts).  scratch: n*n floats.
 cudaError_t cholesky(float* A, int n, float* scratch, int* flag, cudaStream_t st);
+// S = L^{-T} for L L^T = G (n x n SPD, n <= 256), one CTA with the factor in shared memory; the
+// same shifted retries as cholesky(), attempts counted in *flag.
+cudaError_t chol_inverse(const float* G, int n, float* S, int* flag, cudaStream_t st);
 // Q <- Q L^{-T} for the rows x n matrix Q (row-major) and lower-triangular L.
 cudaError_t trsm_right_lt(float* Q, int rows, int n, const float* L, cudaStream_t st);
 // Random Gaussian start block (rows x cols) from Philox with the power-iteration tag.

@@ -361,6 +361,95 @@ cudaError_t fix_column_signs(float* A, int rows, int cols, cudaStream_t st) {
     return cudaGetLastError();
 }
 
+namespace {
+// Packed lower triangle: element (i, l), l <= i, at i (i + 1) / 2 + l.
+__device__ __forceinline__ int tri(int i, int l) { return i * (i + 1) / 2 + l; }
+
+// S = L^{-T} with L L^T = G (n x n symmetric positive definite, n <= 256): one CTA, the packed lower
+// triangle in shared memory.  Right-looking Cholesky (a warp per row of the trailing update, lanes
+// along the row); if a pivot is not positive a diagonal shift (1e-7, then x100, times the mean
+// diagonal) is added and the factorisation restarts, at most six attempts, the attempts counted
+// in *flag.  Then L^{-1} in place, column by column from the last: for j = n-1..0 the entries
+// below the diagonal of column j are -(L^{-1}[i, j+1..i] . L[j+1..i, j]) / L_jj, formed for all i
+// before any is written.  S (row-major n x n) is the transpose of L^{-1}.
+__global__ void __launch_bounds__(1024) chol_inverse_kernel(const float* G, int n, float* S, int* flag) {
+    extern __shared__ float L[];                       // n (n + 1) / 2 packed, then n temporaries
+    float* tmp = L + n * (n + 1) / 2;
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5, nw = blockDim.x >> 5;
+    __shared__ int fail;
+    __shared__ float shift, trace;
+    if (tid == 0) {
+        float tr = 0.f;
+        for (int i = 0; i < n; ++i) tr += G[(size_t)i * n + i];
+        trace = tr;
+        shift = 0.f;
+    }
+    __syncthreads();
+    int attempt = 0;
+    for (; attempt < 6; ++attempt) {
+        for (int i = warp; i < n; i += nw)
+            for (int l = lane; l <= i; l += 32) L[tri(i, l)] = G[(size_t)i * n + l] + (l == i ? shift : 0.f);
+        if (tid == 0) fail = 0;
+        __syncthreads();
+        const float thresh = 1e-12f * fmaxf(trace / n, 1e-30f);
+        for (int j = 0; j < n; ++j) {
+            const float d = L[tri(j, j)];
+            if (!(d > thresh)) { fail = 1; break; }      // uniform: every thread reads the same d
+            const float ljj = sqrtf(d);
+            __syncthreads();
+            if (tid == 0) L[tri(j, j)] = ljj;
+            for (int i = j + 1 + tid; i < n; i += blockDim.x) L[tri(i, j)] /= ljj;
+            __syncthreads();
+            for (int i = j + 1 + warp; i < n; i += nw) {
+                const float lij = L[tri(i, j)];
+                for (int l = j + 1 + lane; l <= i; l += 32) L[tri(i, l)] -= lij * L[tri(l, j)];
+            }
+            __syncthreads();
+        }
+        __syncthreads();
+        if (!fail) break;
+        if (tid == 0) shift = (attempt == 0 ? 1e-7f : shift * 100.f) * fmaxf(trace / n, 1e-30f);
+        __syncthreads();
+    }
+    if (tid == 0 && flag) *flag = attempt;
+    for (int j = n - 1; j >= 0; --j) {
+        for (int i = j + 1 + warp; i < n; i += nw) {
+            float t = 0.f;
+            for (int l = j + 1 + lane; l <= i; l += 32) t += L[tri(i, l)] * L[tri(l, j)];
+#pragma unroll
+            for (int o = 16; o > 0; o >>= 1) t += __shfl_xor_sync(0xffffffffu, t, o);
+            if (lane == 0) tmp[i] = t;
+        }
+        __syncthreads();
+        const float ajj = 1.0f / L[tri(j, j)];
+        for (int i = j + 1 + tid; i < n; i += blockDim.x) L[tri(i, j)] = -tmp[i] * ajj;
+        __syncthreads();
+        if (tid == 0) L[tri(j, j)] = ajj;
+        __syncthreads();
+    }
+    for (int e = tid; e < n * n; e += blockDim.x) {
+        const int r = e / n, c = e % n;
+        S[e] = c >= r ? L[tri(c, r)] : 0.f;
+    }
+}
+}  // namespace
+
+cudaError_t chol_inverse(const float* G, int n, float* S, int* flag, cudaStream_t st) {
+    if (n < 1 || n > 256) return cudaErrorInvalidValue;
+    const size_t smem = sizeof(float) * ((size_t)n * (n + 1) / 2 + n);
+    static bool set = false;
+    if (!set) {
+        // the largest factor (n = 256) and its temporaries, below the per-CTA limit with the
+        // kernel's few static bytes
+        const cudaError_t e = cudaFuncSetAttribute(chol_inverse_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                                   (int)(sizeof(float) * (256 * 257 / 2 + 256)));
+        if (e != cudaSuccess) return e;
+        set = true;
+    }
+    chol_inverse_kernel<<<1, 1024, smem, st>>>(G, n, S, flag);
+    return cudaGetLastError();
+}
+
 cudaError_t cholesky(float* A, int n, float* scratch, int* flag, cudaStream_t st) {
     cholesky_kernel<<<1, 1024, 0, st>>>(A, n, scratch, flag);
     return cudaGetLastError();
