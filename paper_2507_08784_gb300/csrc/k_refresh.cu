@@ -370,19 +370,23 @@ __device__ __forceinline__ int tri(int i, int l) { return i * (i + 1) / 2 + l; }
 // along the row); if a pivot is not positive a diagonal shift (1e-7, then x100, times the mean
 // diagonal) is added and the factorisation restarts, at most six attempts, the attempts counted
 // in *flag.  Then L^{-1} in place, column by column from the last: for j = n-1..0 the entries
-// below the diagonal of column j are -(L^{-1}[i, j+1..i] . L[j+1..i, j]) / L_jj, formed for all i
-// before any is written.  S (row-major n x n) is the transpose of L^{-1}.
+// below the diagonal of column j are -(L^{-1}[i, j+1..i] . L[j+1..i, j]) / L_jj.  Each step first
+// copies the column it reads into a contiguous array (a column of the packed triangle is strided
+// by the row lengths, which would make the lanes' reads collide in the banks).  S (row-major
+// n x n) is the transpose of L^{-1}.
 __global__ void __launch_bounds__(1024) chol_inverse_kernel(const float* G, int n, float* S, int* flag) {
-    extern __shared__ float L[];                       // n (n + 1) / 2 packed, then n temporaries
-    float* tmp = L + n * (n + 1) / 2;
+    extern __shared__ float L[];                       // n (n + 1) / 2 packed, then n + n temporaries
+    float* col = L + n * (n + 1) / 2;
+    float* tmp = col + n;
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5, nw = blockDim.x >> 5;
     __shared__ int fail;
     __shared__ float shift, trace;
-    if (tid == 0) {
+    if (warp == 0) {                                   // trace: a warp sum in a fixed order
         float tr = 0.f;
-        for (int i = 0; i < n; ++i) tr += G[(size_t)i * n + i];
-        trace = tr;
-        shift = 0.f;
+        for (int i = lane; i < n; i += 32) tr += G[(size_t)i * n + i];
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) tr += __shfl_xor_sync(0xffffffffu, tr, o);
+        if (lane == 0) { trace = tr; shift = 0.f; }
     }
     __syncthreads();
     int attempt = 0;
@@ -398,11 +402,15 @@ __global__ void __launch_bounds__(1024) chol_inverse_kernel(const float* G, int 
             const float ljj = sqrtf(d);
             __syncthreads();
             if (tid == 0) L[tri(j, j)] = ljj;
-            for (int i = j + 1 + tid; i < n; i += blockDim.x) L[tri(i, j)] /= ljj;
+            for (int i = j + 1 + tid; i < n; i += blockDim.x) {
+                const float v = L[tri(i, j)] / ljj;
+                L[tri(i, j)] = v;
+                col[i] = v;
+            }
             __syncthreads();
             for (int i = j + 1 + warp; i < n; i += nw) {
-                const float lij = L[tri(i, j)];
-                for (int l = j + 1 + lane; l <= i; l += 32) L[tri(i, l)] -= lij * L[tri(l, j)];
+                const float lij = col[i];
+                for (int l = j + 1 + lane; l <= i; l += 32) L[tri(i, l)] -= lij * col[l];
             }
             __syncthreads();
         }
@@ -413,9 +421,11 @@ __global__ void __launch_bounds__(1024) chol_inverse_kernel(const float* G, int 
     }
     if (tid == 0 && flag) *flag = attempt;
     for (int j = n - 1; j >= 0; --j) {
+        for (int l = j + 1 + tid; l < n; l += blockDim.x) col[l] = L[tri(l, j)];
+        __syncthreads();
         for (int i = j + 1 + warp; i < n; i += nw) {
             float t = 0.f;
-            for (int l = j + 1 + lane; l <= i; l += 32) t += L[tri(i, l)] * L[tri(l, j)];
+            for (int l = j + 1 + lane; l <= i; l += 32) t += L[tri(i, l)] * col[l];
 #pragma unroll
             for (int o = 16; o > 0; o >>= 1) t += __shfl_xor_sync(0xffffffffu, t, o);
             if (lane == 0) tmp[i] = t;
@@ -423,7 +433,6 @@ __global__ void __launch_bounds__(1024) chol_inverse_kernel(const float* G, int 
         __syncthreads();
         const float ajj = 1.0f / L[tri(j, j)];
         for (int i = j + 1 + tid; i < n; i += blockDim.x) L[tri(i, j)] = -tmp[i] * ajj;
-        __syncthreads();
         if (tid == 0) L[tri(j, j)] = ajj;
         __syncthreads();
     }
@@ -436,13 +445,13 @@ __global__ void __launch_bounds__(1024) chol_inverse_kernel(const float* G, int 
 
 cudaError_t chol_inverse(const float* G, int n, float* S, int* flag, cudaStream_t st) {
     if (n < 1 || n > 256) return cudaErrorInvalidValue;
-    const size_t smem = sizeof(float) * ((size_t)n * (n + 1) / 2 + n);
+    const size_t smem = sizeof(float) * ((size_t)n * (n + 1) / 2 + 2 * n);
     static bool set = false;
     if (!set) {
         // the largest factor (n = 256) and its temporaries, below the per-CTA limit with the
         // kernel's few static bytes
         const cudaError_t e = cudaFuncSetAttribute(chol_inverse_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                                   (int)(sizeof(float) * (256 * 257 / 2 + 256)));
+                                                   (int)(sizeof(float) * (256 * 257 / 2 + 2 * 256)));
         if (e != cudaSuccess) return e;
         set = true;
     }
