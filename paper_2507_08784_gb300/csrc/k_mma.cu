@@ -103,15 +103,17 @@ __device__ __forceinline__ void mbar_arrive(uint32_t bar) {
 __device__ __forceinline__ void mbar_expect_tx(uint32_t bar, uint32_t bytes) {
     asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar), "r"(bytes) : "memory");
 }
-// Waits for the phase of parity `parity` to complete.  Each poll lets the thread sleep until the
-// phase completes or a time hint (10 ms) passes, so waiting threads issue almost nothing; after
-// 100 polls (about a second) it gives up and returns false.
+// Waits for the phase of parity `parity` to complete, polling with short sleeps in between; after
+// about a second (16 M polls of >= 64 ns) it gives up and returns false.
 __device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity) {
-    for (int it = 0; it < 100; ++it) {
+    uint32_t ns = 16;
+    for (int it = 0; it < 16000000; ++it) {
         uint32_t done;
-        asm volatile("{ .reg .pred p; mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2, %3; selp.u32 %0, 1, 0, p; }"
-                     : "=r"(done) : "r"(bar), "r"(parity), "r"(10000000u) : "memory");
+        asm volatile("{ .reg .pred p; mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2; selp.u32 %0, 1, 0, p; }"
+                     : "=r"(done) : "r"(bar), "r"(parity) : "memory");
         if (done) return true;
+        __nanosleep(ns);                   // back off (16 .. 64 ns) so waiting warps leave the issue slots
+        ns = ns < 64 ? 2 * ns : 64;
     }
     return false;
 }
@@ -190,18 +192,31 @@ template <> struct GradPair<float> {
     static __device__ __forceinline__ float2 row(const float* Gs, int a, int c) {
         return *reinterpret_cast<const float2*>(Gs + sw64(a, c));
     }
+    // the same at a precomputed swizzled offset (Lane::sb0 / sb1 + kGroupStride j)
+    static __device__ __forceinline__ float2 at(const float* Gs, int off, int, int) {
+        return *reinterpret_cast<const float2*>(Gs + off);
+    }
 };
 template <> struct GradPair<__nv_bfloat16> {
     static __device__ __forceinline__ float2 row(const __nv_bfloat16* Gs, int a, int c) {
         return __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(Gs + sw32(a, c)));
+    }
+    static __device__ __forceinline__ float2 at(const __nv_bfloat16* Gs, int, int offg, int) {
+        return __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(Gs + offg));
     }
 };
 
 // ---- the pieces of a strip's work, shared by the kernels below ------------------------------
 // Lane geometry (see the header): warp w, lane = 4 gg + t, rows rho and rho + 2 of each group,
 // columns c2 and c2 + 1; prow is the row of the C^T = R^T P^T B fragment.
+// The lane's rows in row group G8 = w + NW j are ra = 8 G8 + rho and rb = ra + 2; since 8 G8 is a
+// multiple of 8 and rho + 2 < 8, the swizzle terms (ra >> 1) & 3 and (ra >> 2) & 1 depend on rho
+// only, so a row's swizzled offset in a strip is a lane constant plus 128 G8 = 128 w + 2048 j:
+// sb0 / sb1 for the 64-byte swizzle (B, fp32 G), sg0 / sg1 for the 32-byte one (bf16 G), in
+// elements.
 struct Lane {
     int tid, w, lane, gg, t, rho, prow, c2;
+    int sb0, sb1, sg0, sg1;
 };
 __device__ __forceinline__ Lane lane_geometry() {
     Lane L;
@@ -209,8 +224,14 @@ __device__ __forceinline__ Lane lane_geometry() {
     L.rho = (L.t & 1) + 4 * (L.t >> 1);
     L.prow = ((L.gg >> 1) & 1) + 4 * (L.gg >> 2) + 2 * (L.gg & 1);
     L.c2 = 2 * L.gg;
+    const int r0 = L.rho, r1 = L.rho + 2, base = 128 * L.w;
+    L.sb0 = base + SW * r0 + 4 * ((L.c2 >> 2) ^ ((r0 >> 1) & 3)) + (L.c2 & 3);
+    L.sb1 = base + SW * r1 + 4 * ((L.c2 >> 2) ^ ((r1 >> 1) & 3)) + (L.c2 & 3);
+    L.sg0 = base + SW * r0 + 8 * ((L.c2 >> 3) ^ ((r0 >> 2) & 1)) + (L.c2 & 7);
+    L.sg1 = base + SW * r1 + 8 * ((L.c2 >> 3) ^ ((r1 >> 2) & 1)) + (L.c2 & 7);
     return L;
 }
+constexpr int kGroupStride = 128 * NW;   // elements between a lane's rows in groups j and j + 1
 
 // P_prev fragments of the lane's row groups (zero where E = 0, past m' or past r).
 template <int NQ, int GPW>
@@ -255,9 +276,8 @@ __device__ __forceinline__ void compose_node(const float* S, const GT* Gs, bool 
         for (int j = 0; j < GPW; ++j) {
             const int G8 = L.w + NW * j;
             if (G8 < ng) {
-                const int ra = 8 * G8 + L.rho;
-                const float2 x0 = *reinterpret_cast<const float2*>(S + sw64(ra, L.c2));
-                const float2 x1 = *reinterpret_cast<const float2*>(S + sw64(ra + 2, L.c2));
+                const float2 x0 = *reinterpret_cast<const float2*>(S + L.sb0 + kGroupStride * j);
+                const float2 x1 = *reinterpret_cast<const float2*>(S + L.sb1 + kGroupStride * j);
                 const FragA A = frag_a(x0.x, x0.y, x1.x, x1.y);
 #pragma unroll
                 for (int nt = 0; nt < NQ; ++nt) mma3(d[j][nt], A, prt[j][nt]);
@@ -284,6 +304,10 @@ __device__ __forceinline__ void compose_node(const float* S, const GT* Gs, bool 
             RA[nt] = frag_a(R.x, R.z, R.y, R.w);
         }
     }
+    // the lane's first row of group 0 in node i's B, and the distance to group j's (128 rows per
+    // group step) and to row rb (2 rows)
+    float* const Brow = Bi + (int64_t)(8 * L.w + L.rho) * np;
+    const int64_t jstep = (int64_t)(8 * NW) * np;
 #pragma unroll
     for (int j = 0; j < GPW; ++j) {
         const int G8 = L.w + NW * j;
@@ -294,24 +318,25 @@ __device__ __forceinline__ void compose_node(const float* S, const GT* Gs, bool 
             if (corr) {
 #pragma unroll
                 for (int nt = 0; nt < NQ; ++nt) mma3(c, RA[nt], pcb[j][nt]);
-                x0 = *reinterpret_cast<const float2*>(S + sw64(ra, L.c2));
-                x1 = *reinterpret_cast<const float2*>(S + sw64(rb, L.c2));
+                x0 = *reinterpret_cast<const float2*>(S + L.sb0 + kGroupStride * j);
+                x1 = *reinterpret_cast<const float2*>(S + L.sb1 + kGroupStride * j);
             }
             float2 g0, g1;
             if (trans) {
                 g0 = make_float2(static_cast<float>(Gs[L.c2 * gpt + ra]), static_cast<float>(Gs[(L.c2 + 1) * gpt + ra]));
                 g1 = make_float2(static_cast<float>(Gs[L.c2 * gpt + rb]), static_cast<float>(Gs[(L.c2 + 1) * gpt + rb]));
             } else {
-                g0 = GradPair<GT>::row(Gs, ra, L.c2);
-                g1 = GradPair<GT>::row(Gs, rb, L.c2);
+                g0 = GradPair<GT>::at(Gs, L.sb0 + kGroupStride * j, L.sg0 + kGroupStride * j, 0);
+                g1 = GradPair<GT>::at(Gs, L.sb1 + kGroupStride * j, L.sg1 + kGroupStride * j, 0);
             }
             const float m0 = g0.x + (x0.x - c[0]);       // M = G + E, E = B - P_prev R
             const float m1 = g0.y + (x0.y - c[2]);
             const float m2 = g1.x + (x1.x - c[1]);
             const float m3 = g1.y + (x1.y - c[3]);
             if (write_B && colok) {
-                if (ra < mp) __stcs(reinterpret_cast<float2*>(Bi + (int64_t)ra * np), make_float2(m0, m1));
-                if (rb < mp) __stcs(reinterpret_cast<float2*>(Bi + (int64_t)rb * np), make_float2(m2, m3));
+                float* const Ba = Brow + j * jstep;
+                if (ra < mp) __stcs(reinterpret_cast<float2*>(Ba), make_float2(m0, m1));
+                if (rb < mp) __stcs(reinterpret_cast<float2*>(Ba + 2 * (int64_t)np), make_float2(m2, m3));
             }
             acc[j][0] += m0; acc[j][1] += m1; acc[j][2] += m2; acc[j][3] += m3;
         }
