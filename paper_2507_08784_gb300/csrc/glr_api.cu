@@ -54,6 +54,8 @@ struct glr_handle {
     // in mn_scratch (m' x n').
     int tc = 0;
     float* mn_scratch = nullptr;
+    float* jwork = nullptr;      // full basis: the grouped Jacobi's second m' x m' buffer
+    float* jpart = nullptr;      // full basis: its per-CTA norm partials (used by a group's first handle)
     float* YtJ = nullptr;        // Yt[J, :] (r x k) for P = U[:, J] as a library product
     cudaStream_t rstream = nullptr;            // side stream of this handle's refresh
     cudaEvent_t rfork = nullptr, rdone = nullptr, rpow = nullptr;
@@ -373,6 +375,55 @@ int refresh_grouped(std::vector<glr_handle*>& hs) {
     return GLR_OK;
 }
 
+// Full-basis refreshes of several matrices: H = Mbar Mbar^T on each handle's side stream, one
+// cooperative Jacobi launch for all of them on the first handle's side stream (k_jacobi.cu), then
+// each handle sorts its eigenvectors by descending eigenvalue and fixes their signs on its own.
+int refresh_exact_grouped(std::vector<glr_handle*>& hs) {
+    const int grid = jacobi_group_grid();
+    for (size_t c0 = 0; c0 < hs.size(); c0 += kGroupMax) {
+        const size_t c1 = std::min(hs.size(), c0 + kGroupMax);
+        glr_handle* h0 = hs[c0];
+        cudaStream_t s0 = h0->rstream;
+        for (size_t i = c0; i < c1; ++i) {
+            glr_handle* h = hs[i];
+            PhaseScope ps(h, GLR_PH_REFRESH, h->rstream);
+            const int mp = h->mp, np = h->np;
+            GLR_GEMM(h, gd(mp, mp, np, h->Mbar, np, 1, h->Mbar, 1, np, h->Hbuf, mp, 1), h->rstream);
+            if (!grid) {                                         // no cooperative launch: one CTA each
+                GLR_LAUNCH(h, 1, jacobi_eig(h->Hbuf, mp, h->Vbuf, h->evals, h->dflags + 1, h->rstream));
+                GLR_LAUNCH(h, 1, sort_fix_basis(h->evals, h->Vbuf, mp, mp, h->U, mp, h->evals_sorted, h->rstream));
+                continue;
+            }
+            GLR_CK(h, cudaEventRecord(h->rpow, h->rstream));
+            if (h != h0) GLR_CK(h0, cudaStreamWaitEvent(s0, h->rpow, 0));
+        }
+        if (!grid) continue;
+        JacobiGroup g{};
+        g.max_sweeps = 40;
+        g.bar = h0->dflags + 4; g.err = h0->dflags + 2; g.part = h0->jpart;
+        for (size_t i = c0; i < c1; ++i) {
+            glr_handle* h = hs[i];
+            JacobiMat& M = g.mat[g.nmat++];
+            const int n = h->mp;
+            M.n = n; M.tol = 4.f * 5.96e-8f * sqrtf(static_cast<float>(n)) + 1e-7f;
+            M.H = h->Hbuf; M.H2 = h->jwork; M.V = h->Vbuf; M.evals = h->evals;
+            M.sweeps = h->dflags + 1;
+        }
+        {
+            PhaseScope ps(h0, GLR_PH_REFRESH, s0);
+            GLR_LAUNCH(h0, 1, jacobi_group(g, grid, s0));
+        }
+        GLR_CK(h0, cudaEventRecord(h0->rpow, s0));
+        for (size_t i = c0; i < c1; ++i) {
+            glr_handle* h = hs[i];
+            if (h != h0) GLR_CK(h, cudaStreamWaitEvent(h->rstream, h0->rpow, 0));
+            PhaseScope ps(h, GLR_PH_REFRESH, h->rstream);
+            GLR_LAUNCH(h, 1, sort_fix_basis(h->evals, h->Vbuf, h->mp, h->mp, h->U, h->mp, h->evals_sorted, h->rstream));
+        }
+    }
+    return GLR_OK;
+}
+
 // Semi-Lazy SVD refresh (Eq. SVD-P1) from Mbar.
 int do_refresh(glr_handle* h, cudaStream_t st) {
     const int mp = h->mp, np = h->np, k = h->k;
@@ -530,6 +581,8 @@ int glr_create(int64_t m, int64_t n, int32_t r, int32_t N, const glr_schedule* s
     if (h->tc) A(&h->mn_scratch, MP * NP);
     if (h->tc && !exact) A(&h->YtJ, (size_t)r * k);
     if (exact) {
+        A(&h->jwork, MP * MP);
+        A(&h->jpart, (size_t)2 * kGroupMax * kJacobiMaxGrid);
         A(&h->U, MP * MP); A(&h->Hbuf, MP * MP); A(&h->Vbuf, MP * MP);
         A(&h->evals, MP); A(&h->evals_sorted, MP);
     } else {
@@ -935,7 +988,7 @@ int step_group(std::vector<StepPlan>& plans, cudaStream_t st) {
     // Refreshes (Semi-Lazy SVD) of different matrices are independent: each runs on its
     // handle's side stream after the compose pass, overlapping the others and the selection
     // work of the non-refreshing matrices; the main stream joins them before P is built.
-    std::vector<glr_handle*> refreshing, grouped;
+    std::vector<glr_handle*> refreshing, grouped, exact;
     for (StepPlan& p : plans) {
         if (!p.refresh) continue;
         glr_handle* h = p.h;
@@ -943,10 +996,12 @@ int step_group(std::vector<StepPlan>& plans, cudaStream_t st) {
         GLR_CK(h, cudaStreamWaitEvent(h->rstream, h->rfork, 0));
         refreshing.push_back(h);
         if (h->pow_ok) grouped.push_back(h);
+        if (h->exact) exact.push_back(h);
     }
     if (!grouped.empty() && (rc = refresh_grouped(grouped)) != GLR_OK) return rc;
+    if (!exact.empty() && (rc = refresh_exact_grouped(exact)) != GLR_OK) return rc;
     for (glr_handle* h : refreshing) {
-        if (!h->pow_ok) {
+        if (!h->pow_ok && !h->exact) {
             PhaseScope ps(h, GLR_PH_REFRESH, h->rstream);
             if ((rc = do_refresh(h, h->rstream)) != GLR_OK) return rc;
         }

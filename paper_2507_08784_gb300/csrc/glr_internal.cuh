@@ -207,6 +207,25 @@ cudaError_t cholesky(float* A, int n, float* scratch, int* flag, cudaStream_t st
 // S = L^{-T} for L L^T = G (n x n SPD, n <= 256), one CTA with the factor in shared memory; the
 // same shifted retries as cholesky(), attempts counted in *flag.
 cudaError_t chol_inverse(const float* G, int n, float* S, int* flag, cudaStream_t st);
+
+// Full-basis refresh of several matrices at once (k_jacobi.cu): parallel cyclic Jacobi on each
+// n x n Gram matrix H (n <= 1024; H and H2 are overwritten, the eigenvalues end in evals) with
+// eigenvectors in V, spread over one cooperative grid.  part: 2 nmat grid floats; bar: two ints
+// (zeroed by the launcher); err counts barrier waits that gave up; sweeps receives the sweeps
+// each matrix took.  jacobi_group_grid() is 0 where cooperative launches are unavailable.
+struct JacobiMat {
+    int n; float tol;
+    float* H; float* H2; float* V; float* evals;   // H2: a second n x n buffer (rounds alternate)
+    int* sweeps;
+};
+constexpr int kJacobiMaxGrid = 1024;
+struct JacobiGroup {
+    int nmat, max_sweeps;
+    int* bar; int* err; float* part;
+    JacobiMat mat[kGroupMax];
+};
+int jacobi_group_grid();
+cudaError_t jacobi_group(const JacobiGroup& g, int grid, cudaStream_t st);
 // Q <- Q L^{-T} for the rows x n matrix Q (row-major) and lower-triangular L.
 cudaError_t trsm_right_lt(float* Q, int rows, int n, const float* L, cudaStream_t st);
 // Random Gaussian start block (rows x cols) from Philox with the power-iteration tag.
