@@ -380,8 +380,14 @@ int refresh_grouped(std::vector<glr_handle*>& hs) {
 // each handle sorts its eigenvectors by descending eigenvalue and fixes their signs on its own.
 int refresh_exact_grouped(std::vector<glr_handle*>& hs) {
     const int grid = jacobi_group_grid();
-    for (size_t c0 = 0; c0 < hs.size(); c0 += kGroupMax) {
-        const size_t c1 = std::min(hs.size(), c0 + kGroupMax);
+    for (size_t c0 = 0, c1 = 0; c0 < hs.size(); c0 = c1) {
+        // a group: at most kGroupMax matrices whose rotations fit the kernel's shared memory
+        size_t rot = 0;
+        for (c1 = c0; c1 < hs.size() && c1 - c0 < (size_t)kGroupMax; ++c1) {
+            const size_t add = jacobi_rot_floats(hs[c1]->mp) * sizeof(float);
+            if (c1 > c0 && rot + add > kJacobiMaxSmem) break;
+            rot += add;
+        }
         glr_handle* h0 = hs[c0];
         cudaStream_t s0 = h0->rstream;
         for (size_t i = c0; i < c1; ++i) {
@@ -399,6 +405,7 @@ int refresh_exact_grouped(std::vector<glr_handle*>& hs) {
         }
         if (!grid) continue;
         JacobiGroup g{};
+        size_t soff = 0;
         g.max_sweeps = 40;
         g.bar = h0->dflags + 4; g.err = h0->dflags + 2; g.part = h0->jpart;
         for (size_t i = c0; i < c1; ++i) {
@@ -408,6 +415,8 @@ int refresh_exact_grouped(std::vector<glr_handle*>& hs) {
             M.n = n; M.tol = 4.f * 5.96e-8f * sqrtf(static_cast<float>(n)) + 1e-7f;
             M.H = h->Hbuf; M.H2 = h->jwork; M.V = h->Vbuf; M.evals = h->evals;
             M.sweeps = h->dflags + 1;
+            M.soff = (int)soff;
+            soff += jacobi_rot_floats(n);
         }
         {
             PhaseScope ps(h0, GLR_PH_REFRESH, s0);

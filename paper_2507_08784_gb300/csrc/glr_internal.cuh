@@ -217,8 +217,11 @@ struct JacobiMat {
     int n; float tol;
     float* H; float* H2; float* V; float* evals;   // H2: a second n x n buffer (rounds alternate)
     int* sweeps;
+    int soff;               // first float of this matrix's rotations in shared memory (see jacobi_rot_floats)
 };
 constexpr int kJacobiMaxGrid = 1024;
+constexpr size_t kJacobiMaxSmem = 96 * 1024;     // the group's rotations; groups are split to fit
+size_t jacobi_rot_floats(int n);
 struct JacobiGroup {
     int nmat, max_sweeps;
     int* bar; int* err; float* part;
