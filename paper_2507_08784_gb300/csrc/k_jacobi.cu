@@ -58,15 +58,13 @@ __device__ bool grid_barrier(int* count, int* genp, int& gen) {
 // (each entry by one thread).  A check's partial norms are written in one step and decided on at
 // the start of the next, identically by every CTA.  One grid barrier per step.
 enum : int { kCheck = 0, kRound = 1, kPending = 2, kDone = 3 };
-constexpr int kMaxHalf = 512;           // n <= 1024
 
 __global__ void __launch_bounds__(JT) jacobi_group_kernel(const __grid_constant__ JacobiGroup g) {
     const int G = gridDim.x, b = blockIdx.x, t = threadIdx.x;
     const int64_t gtid = (int64_t)b * JT + t, gsz = (int64_t)G * JT;
     __shared__ int sstate[kGroupMax], sround[kGroupMax], ssweep[kGroupMax], sflip[kGroupMax];
-    __shared__ float scs[kMaxHalf], ssn[kMaxHalf];
-    __shared__ int spp[kMaxHalf], sqq[kMaxHalf];
     __shared__ float red[2][JT / 32];
+    extern __shared__ float srot[];                     // per matrix at M.soff: cs, sn, pp, qq (half each)
     int gen = 0;
     bool ok = true;
     for (int mi = 0; mi < g.nmat; ++mi) {
@@ -93,11 +91,11 @@ __global__ void __launch_bounds__(JT) jacobi_group_kernel(const __grid_constant_
         bool any = false;
         for (int mi = 0; mi < g.nmat; ++mi) any = any || sstate[mi] != kDone;
         if (!any) break;
+        // norm checks, and every round's rotations (each matrix in its own shared slice)
         for (int mi = 0; mi < g.nmat; ++mi) {
             const JacobiMat& M = g.mat[mi];
             const int n = M.n;
             const float* Hc = sflip[mi] ? M.H2 : M.H;
-            float* Hn = sflip[mi] ? M.H : M.H2;
             if (sstate[mi] == kCheck) {                 // off-diagonal and total squared norms, per CTA
                 const int64_t nn = (int64_t)n * n;
                 float off = 0.f, tot = 0.f;
@@ -123,6 +121,10 @@ __global__ void __launch_bounds__(JT) jacobi_group_kernel(const __grid_constant_
             }
             if (sstate[mi] != kRound) continue;
             const int npad = n + (n & 1), half = npad / 2, nm1 = npad - 1, r = sround[mi];
+            float* scs = srot + M.soff;
+            float* ssn = scs + half;
+            int* spp = reinterpret_cast<int*>(ssn + half);
+            int* sqq = spp + half;
             for (int i = t; i < half; i += JT) {        // all of the round's rotations, in this CTA
                 int p = (i == 0) ? 0 : circle(r + i, nm1);
                 int q = (i == 0) ? circle(r, nm1) : circle(r - i, nm1);
@@ -142,7 +144,19 @@ __global__ void __launch_bounds__(JT) jacobi_group_kernel(const __grid_constant_
                 }
                 scs[i] = c; ssn[i] = s; spp[i] = p; sqq[i] = q;
             }
-            __syncthreads();
+        }
+        __syncthreads();
+        // every round's updates
+        for (int mi = 0; mi < g.nmat; ++mi) {
+            if (sstate[mi] != kRound) continue;
+            const JacobiMat& M = g.mat[mi];
+            const int n = M.n, half = (n + (n & 1)) / 2;
+            const float* Hc = sflip[mi] ? M.H2 : M.H;
+            float* Hn = sflip[mi] ? M.H : M.H2;
+            const float* scs = srot + M.soff;
+            const float* ssn = scs + half;
+            const int* spp = reinterpret_cast<const int*>(ssn + half);
+            const int* sqq = spp + half;
             const int64_t hh = (int64_t)half * half;
             for (int64_t e = gtid; e < hh; e += gsz) {   // Hn = J^T Hc J, 2 x 2 block by block
                 const int bi = static_cast<int>(e / half), bj = static_cast<int>(e % half);
@@ -177,8 +191,8 @@ __global__ void __launch_bounds__(JT) jacobi_group_kernel(const __grid_constant_
                 M.V[(size_t)a * n + pj] = cj * vp - sj * vq;
                 M.V[(size_t)a * n + qj] = sj * vp + cj * vq;
             }
-            __syncthreads();                             // the rotations' shared arrays are reused next
         }
+        __syncthreads();                                 // the shared rotations are rewritten next step
         if (t < g.nmat) {                               // every CTA advances the same stages
             if (sstate[t] == kCheck) {
                 sstate[t] = kPending;
@@ -210,20 +224,36 @@ int jacobi_group_grid() {
         if (cudaGetDevice(&dev) != cudaSuccess ||
             cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess ||
             cudaDeviceGetAttribute(&coop, cudaDevAttrCooperativeLaunch, dev) != cudaSuccess || !coop ||
-            cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per, jacobi_group_kernel, JT, 0) != cudaSuccess || per < 1)
+            cudaFuncSetAttribute(jacobi_group_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kJacobiMaxSmem) != cudaSuccess ||
+            cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per, jacobi_group_kernel, JT, kJacobiMaxSmem) != cudaSuccess || per < 1)
             return 0;
         grid = sms * (per < 2 ? per : 2);
     }
     return grid;
 }
 
+size_t jacobi_rot_floats(int n) { return 4 * (size_t)((n + (n & 1)) / 2); }
+
 cudaError_t jacobi_group(const JacobiGroup& g, int grid, cudaStream_t st) {
     if (g.nmat <= 0) return cudaSuccess;
     if (grid <= 0 || grid > kJacobiMaxGrid) return cudaErrorInvalidValue;
+    size_t smem = 0;
+    for (int i = 0; i < g.nmat; ++i) {
+        if (g.mat[i].soff != (int)smem) return cudaErrorInvalidValue;
+        smem += jacobi_rot_floats(g.mat[i].n);
+    }
+    smem *= sizeof(float);
+    if (smem > kJacobiMaxSmem) return cudaErrorInvalidValue;
+    static bool set = false;
+    if (!set) {
+        cudaError_t e = cudaFuncSetAttribute(jacobi_group_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kJacobiMaxSmem);
+        if (e != cudaSuccess) return e;
+        set = true;
+    }
     cudaError_t e = cudaMemsetAsync(g.bar, 0, 2 * sizeof(int), st);    // arrivals and generation
     if (e != cudaSuccess) return e;
     void* args[] = {const_cast<JacobiGroup*>(&g)};
-    return cudaLaunchCooperativeKernel(reinterpret_cast<const void*>(jacobi_group_kernel), dim3(grid), dim3(JT), args, 0, st);
+    return cudaLaunchCooperativeKernel(reinterpret_cast<const void*>(jacobi_group_kernel), dim3(grid), dim3(JT), args, smem, st);
 }
 
 }  // namespace glr
