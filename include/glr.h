@@ -182,6 +182,19 @@ int glr_step_host(glr_handle* h, const void* const* G_host, float* X, float* X_h
 int glr_step_group_host(glr_handle* const* handles, int32_t count, const void* const* const* G_host,
                         float* const* X, float* const* X_host_out, void* stream);
 
+/* Checkpoints.  glr_state_size gives the bytes of a checkpoint of h now; glr_save copies the
+ * handle's whole state into host memory host_buf (at least that many bytes): the schedule
+ * position (t, the refresh period, a pending forced selection), the basis, P, the error state
+ * B, the optimizer moments and every other buffer glr_create allocated.  It runs on `stream`
+ * after the work already queued there and synchronises it.  glr_load restores such a checkpoint
+ * into a handle created with the same m, n, r, N, basis rank, gradient dtype, optimizer and
+ * refresh mode (GLR_EINVAL otherwise, or when the buffer is not a checkpoint or is truncated),
+ * also synchronising `stream`; stepping the restored handle continues exactly as the saved one
+ * would have (same results bit for bit).  The format is this library's own (host byte order).  */
+int glr_state_size(const glr_handle* h, int64_t* bytes);
+int glr_save(glr_handle* h, void* host_buf, int64_t bytes, void* stream);
+int glr_load(glr_handle* h, const void* host_buf, int64_t bytes, void* stream);
+
 /* Make the next glr_step a refresh step (Semi-Lazy SVD, Eq. SVD-P1) and restart the tau
  * period there.                                                                          */
 int glr_refresh(glr_handle* h);

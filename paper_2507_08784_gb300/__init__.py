@@ -18,7 +18,7 @@ from . import _lib
 from ._lib import (GLR_ADAM, GLR_ALG3, GLR_ALG4, GLR_BF16, GLR_F32, GLR_MSGD, GLR_OK,  # noqa: F401
                    PHASE_NAMES, GlrProfile, GlrSchedule, GlrStats, load)
 
-__all__ = ["GlrError", "make_schedule", "glr_create", "glr_destroy", "glr_step", "glr_step_group", "glr_step_group_host", "glr_step_host",
+__all__ = ["GlrError", "make_schedule", "glr_create", "glr_destroy", "glr_step", "glr_step_group", "glr_step_group_host", "glr_step_host", "glr_save", "glr_load",
            "glr_refresh", "glr_get_stats", "glr_last_error", "glr_get_error", "glr_get_selection",
            "glr_get_basis", "glr_set_basis", "glr_force_selection", "glr_profile_enable",
            "glr_profile_read", "glr_select_noalloc", "GreedyLore", "load"]
@@ -109,6 +109,22 @@ def glr_step_host(h, G_host: Sequence[torch.Tensor], X: torch.Tensor, X_host_out
                                 None if X_host_out is None else X_host_out.data_ptr(), _stream_ptr(stream)), h)
 
 
+def glr_save(h, stream=None) -> np.ndarray:
+    """The handle's whole state as a host byte array (see glr.h)."""
+    lib = load()
+    size = ctypes.c_int64(0)
+    _check(lib.glr_state_size(h, ctypes.byref(size)), h)
+    buf = np.empty(size.value, dtype=np.uint8)
+    _check(lib.glr_save(h, buf.ctypes.data, size.value, _stream_ptr(stream)), h)
+    return buf
+
+
+def glr_load(h, state, stream=None) -> None:
+    """Restore a checkpoint written by glr_save into a handle of the same shape and schedule."""
+    buf = np.ascontiguousarray(state, dtype=np.uint8)
+    _check(load().glr_load(h, buf.ctypes.data, buf.size, _stream_ptr(stream)), h)
+
+
 def glr_refresh(h) -> None:
     _check(load().glr_refresh(h), h)
 
@@ -184,6 +200,12 @@ class GreedyLore:
 
     def step_host(self, G_host, X, X_host_out=None, stream=None):
         glr_step_host(self.handle, G_host, X, X_host_out, stream)
+
+    def state_dict(self, stream=None) -> np.ndarray:
+        return glr_save(self.handle, stream)
+
+    def load_state_dict(self, state, stream=None):
+        glr_load(self.handle, state, stream)
 
     def refresh(self):
         glr_refresh(self.handle)

@@ -79,6 +79,9 @@ _SIGNATURES = {
                                      ctypes.c_void_p]),
     "glr_step_group_host": (ctypes.c_int, [ctypes.c_void_p, ctypes.c_int32, ctypes.c_void_p, ctypes.c_void_p,
                                            ctypes.c_void_p, ctypes.c_void_p]),
+    "glr_state_size": (ctypes.c_int, [ctypes.c_void_p, ctypes.POINTER(ctypes.c_int64)]),
+    "glr_save": (ctypes.c_int, [ctypes.c_void_p, ctypes.c_void_p, ctypes.c_int64, ctypes.c_void_p]),
+    "glr_load": (ctypes.c_int, [ctypes.c_void_p, ctypes.c_void_p, ctypes.c_int64, ctypes.c_void_p]),
     "glr_refresh": (ctypes.c_int, [ctypes.c_void_p]),
     "glr_get_stats": (ctypes.c_int, [ctypes.c_void_p, ctypes.POINTER(GlrStats)]),
     "glr_last_error": (ctypes.c_char_p, [ctypes.c_void_p]),

@@ -74,6 +74,8 @@ struct glr_handle {
     bool has_forceJ = false, forced_this_step = false;
     std::vector<int32_t> forceJ, iotaJ;
     std::vector<void*> allocs;
+    std::vector<size_t> alloc_bytes;
+    size_t n_state_allocs = 0;       // allocations made by glr_create (the checkpointed state)
     std::string err;
     // launch counting and optional per-phase event timing
     int64_t launches = 0;
@@ -155,6 +157,7 @@ int alloc(glr_handle* h, T** p, size_t count) {
         return fail(h, GLR_ENOMEM, "device allocation of %s bytes failed", std::to_string(bytes).c_str());
     }
     h->allocs.push_back(ptr);
+    h->alloc_bytes.push_back(bytes);
     h->state_bytes += static_cast<int64_t>(bytes);
     if (cudaMemset(ptr, 0, bytes) != cudaSuccess) return fail(h, GLR_ECUDA, "cudaMemset failed%s");
     *p = static_cast<T*>(ptr);
@@ -164,6 +167,7 @@ int alloc(glr_handle* h, T** p, size_t count) {
 void free_all(glr_handle* h) {
     for (void* p : h->allocs) cudaFree(p);
     h->allocs.clear();
+    h->alloc_bytes.clear();
 }
 
 // cuTensorMapEncodeTiled from the driver, looked up once through the runtime (no libcuda link).
@@ -652,6 +656,7 @@ int glr_create(int64_t m, int64_t n, int32_t r, int32_t N, const glr_schedule* s
     }
     h->iotaJ.resize(r);
     for (int q = 0; q < r; ++q) h->iotaJ[q] = q;
+    h->n_state_allocs = h->allocs.size();
     *out = h;
     return GLR_OK;
 }
@@ -1141,6 +1146,105 @@ int glr_step_group_host(glr_handle* const* handles, int32_t count, const void* c
         if (X_host_out && X_host_out[j])
             GLR_CK(h, cudaMemcpyAsync(X_host_out[j], X[j], sizeof(float) * h->m * h->n, cudaMemcpyDeviceToHost, st));
     }
+    return GLR_OK;
+}
+
+// ---- checkpoints ---------------------------------------------------------------------------
+// Layout: a header (magic, version, the handle's shape and schedule identity), the host scalars
+// of the schedule, the allocation index that each role which steps swap between two buffers
+// (P / Pprev, Q / Qn, Z / Zn) currently holds, then every device buffer glr_create allocated,
+// in allocation order.
+namespace {
+constexpr uint64_t kCkptMagic = 0x31544b50524c47ull;   // "GLRPKT1"
+struct CkptHeader {
+    uint64_t magic, version;
+    int64_t m, n;
+    int32_t r, N, k, grad_dtype, optimizer, refresh_mode;
+    uint64_t seed, nbuf, buf_bytes;
+    int64_t t, refreshes, comm, period_start;
+    int32_t e_zero, force_refresh, last_uncompressed, basis_from_user, has_forceJ, pad;
+    int32_t role[6];
+};
+float** role_ptr(glr_handle* h, int i) {
+    float** roles[6] = {&h->P, &h->Pprev, &h->Q, &h->Qn, &h->Z, &h->Zn};
+    return roles[i];
+}
+// bytes of a checkpoint of h; a pending forced selection (r indices) is stored when has_forceJ
+size_t ckpt_bytes(const glr_handle* h, bool has_forceJ) {
+    size_t b = sizeof(CkptHeader) + (has_forceJ ? sizeof(int32_t) * h->r : 0);
+    for (size_t i = 0; i < h->n_state_allocs; ++i) b += h->alloc_bytes[i];
+    return b;
+}
+}  // namespace
+
+int glr_state_size(const glr_handle* h, int64_t* bytes) {
+    if (!h || !bytes) return GLR_EINVAL;
+    *bytes = static_cast<int64_t>(ckpt_bytes(h, h->has_forceJ));
+    return GLR_OK;
+}
+
+int glr_save(glr_handle* h, void* host_buf, int64_t bytes, void* stream) {
+    if (!h) return GLR_EINVAL;
+    if (!host_buf || bytes < static_cast<int64_t>(ckpt_bytes(h, h->has_forceJ)))
+        return fail(h, GLR_EINVAL, "checkpoint buffer is null or smaller than glr_state_size%s");
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    CkptHeader hd{};
+    hd.magic = kCkptMagic; hd.version = 1;
+    hd.m = h->m; hd.n = h->n; hd.r = h->r; hd.N = h->N; hd.k = h->k;
+    hd.grad_dtype = h->s.grad_dtype; hd.optimizer = h->s.optimizer; hd.refresh_mode = h->s.refresh_mode;
+    hd.seed = h->s.seed; hd.nbuf = h->n_state_allocs; hd.buf_bytes = ckpt_bytes(h, h->has_forceJ);
+    hd.t = h->t; hd.refreshes = h->refreshes; hd.comm = h->comm; hd.period_start = h->period_start;
+    hd.e_zero = h->e_zero; hd.force_refresh = h->force_refresh; hd.last_uncompressed = h->last_uncompressed;
+    hd.basis_from_user = h->basis_from_user; hd.has_forceJ = h->has_forceJ;
+    for (int i = 0; i < 6; ++i) {
+        hd.role[i] = -1;
+        float* p = *role_ptr(h, i);
+        for (size_t a = 0; a < h->n_state_allocs; ++a)
+            if (h->allocs[a] == p) hd.role[i] = static_cast<int32_t>(a);
+    }
+    char* out = static_cast<char*>(host_buf);
+    std::memcpy(out, &hd, sizeof(hd));
+    out += sizeof(hd);
+    if (h->has_forceJ) {
+        std::memcpy(out, h->forceJ.data(), sizeof(int32_t) * h->r);
+        out += sizeof(int32_t) * h->r;
+    }
+    for (size_t a = 0; a < h->n_state_allocs; ++a) {
+        GLR_CK(h, cudaMemcpyAsync(out, h->allocs[a], h->alloc_bytes[a], cudaMemcpyDeviceToHost, st));
+        out += h->alloc_bytes[a];
+    }
+    GLR_CK(h, cudaStreamSynchronize(st));
+    return GLR_OK;
+}
+
+int glr_load(glr_handle* h, const void* host_buf, int64_t bytes, void* stream) {
+    if (!h) return GLR_EINVAL;
+    if (!host_buf || bytes < static_cast<int64_t>(sizeof(CkptHeader)))
+        return fail(h, GLR_EINVAL, "checkpoint buffer is null or too small%s");
+    CkptHeader hd;
+    std::memcpy(&hd, host_buf, sizeof(hd));
+    if (hd.magic != kCkptMagic || hd.version != 1) return fail(h, GLR_EINVAL, "not a checkpoint of this library%s");
+    if (hd.m != h->m || hd.n != h->n || hd.r != h->r || hd.N != h->N || hd.k != h->k ||
+        hd.grad_dtype != h->s.grad_dtype || hd.optimizer != h->s.optimizer || hd.refresh_mode != h->s.refresh_mode ||
+        hd.nbuf != h->n_state_allocs || hd.buf_bytes != ckpt_bytes(h, hd.has_forceJ != 0))
+        return fail(h, GLR_EINVAL, "checkpoint of a handle with another shape or schedule%s");
+    if (bytes < static_cast<int64_t>(hd.buf_bytes)) return fail(h, GLR_EINVAL, "checkpoint buffer is truncated%s");
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    const char* in = static_cast<const char*>(host_buf) + sizeof(hd);
+    if (hd.has_forceJ) {
+        h->forceJ.assign(reinterpret_cast<const int32_t*>(in), reinterpret_cast<const int32_t*>(in) + h->r);
+        in += sizeof(int32_t) * h->r;
+    }
+    for (size_t a = 0; a < h->n_state_allocs; ++a) {
+        GLR_CK(h, cudaMemcpyAsync(h->allocs[a], in, h->alloc_bytes[a], cudaMemcpyHostToDevice, st));
+        in += h->alloc_bytes[a];
+    }
+    for (int i = 0; i < 6; ++i)
+        if (hd.role[i] >= 0) *role_ptr(h, i) = static_cast<float*>(h->allocs[hd.role[i]]);
+    h->t = hd.t; h->refreshes = hd.refreshes; h->comm = hd.comm; h->period_start = hd.period_start;
+    h->e_zero = hd.e_zero; h->force_refresh = hd.force_refresh; h->last_uncompressed = hd.last_uncompressed;
+    h->basis_from_user = hd.basis_from_user; h->has_forceJ = hd.has_forceJ;
+    GLR_CK(h, cudaStreamSynchronize(st));
     return GLR_OK;
 }
 

@@ -199,6 +199,44 @@ def test_step_host_matches_device_step():
     b.close()
 
 
+@pytest.mark.parametrize("m,n,basis_rank,opt", [(200, 520, 16, "msgd"), (96, 300, 0, "adam"), (700, 300, 24, "msgd")])
+def test_checkpoint_resume_is_bit_identical(m, n, basis_rank, opt):
+    """glr_save after a few steps, glr_load into a fresh handle: both continue identically, across
+    a refresh, on the tensor-core, paper-exact and transposed fused paths; a handle of another
+    shape refuses the checkpoint."""
+    import torch
+    import paper_2507_08784_gb300 as glr
+    r, N = 6, 3
+    kw = dict(tau=3, optimizer=opt, lr=0.01, beta1=0.9, beta2=0.999, eps=1e-8, seed=31, basis_rank=basis_rank)
+    a = glr.GreedyLore(m, n, r, N, **kw)
+    b = glr.GreedyLore(m, n, r, N, **kw)
+    rng = np.random.default_rng(9)
+    grads = [[torch.from_numpy(rng.standard_normal((m, n)).astype(np.float32)).cuda() for _ in range(N)] for _ in range(8)]
+    Xa = torch.zeros(m, n, device="cuda")
+    for t in range(4):
+        a.step(grads[t], Xa)
+    state = a.state_dict()
+    Xb = Xa.clone()
+    b.load_state_dict(state)
+    for t in range(4, 8):
+        a.step(grads[t], Xa)
+        b.step(grads[t], Xb)
+        torch.cuda.synchronize()
+        assert torch.equal(Xa, Xb), t
+        Ja, *_ = a.selection()
+        Jb, *_ = b.selection()
+        assert np.array_equal(Ja, Jb), t
+        assert torch.equal(a.error(0), b.error(0)), t
+    assert a.stats()["t"] == b.stats()["t"] == 8
+    c = glr.GreedyLore(m, n, r + 1, N, **kw)
+    with pytest.raises(glr.GlrError):
+        c.load_state_dict(state)
+    with pytest.raises(glr.GlrError):
+        b.load_state_dict(state[:100])
+    for h in (a, b, c):
+        h.close()
+
+
 @pytest.mark.parametrize("basis_rank", [0, 16])
 def test_step_group_host_matches_step_group(basis_rank):
     """The asynchronous grouped host step (double-buffered staging on a copy stream) gives the
