@@ -59,6 +59,10 @@ extern "C" {
 #define GLR_MSGD 0   /* Eq. msgd:  M = b1 M + (1 - b1) G;  X -= lr M                          */
 #define GLR_ADAM 1   /* Eq. adam:  M, V EMAs; X -= lr M / (sqrt(V) + eps); no bias correction */
 
+#define GLR_SEL_APPROX 0   /* Algorithm 2 (Approx-Top-r) picks J at every compressed step    */
+#define GLR_SEL_FIXED  1   /* P = U[:, :r] for the whole refresh period: the Lazy-SVD of       *
+                            * Algorithm 1 (with no_error_feedback = 1 it is Algorithm 1)       */
+
 #define GLR_F32  0   /* gradients G_i are float32                                            */
 #define GLR_BF16 1   /* gradients G_i are bfloat16                                           */
 
@@ -78,7 +82,11 @@ extern "C" {
  *   power_iters    q >= 1 (truncated basis only)
  *   grad_dtype     GLR_F32 | GLR_BF16
  *   compress_start the first compress_start steps are uncompressed (plain node mean, no
- *                  error feedback); step compress_start is the first refresh           */
+ *                  error feedback); step compress_start is the first refresh
+ *   no_error_feedback  1 drops error feedback (E_i stays 0, M_i = G_i): the comparison of
+ *                  Sec. 4 / Fig. 2 and, with selection = GLR_SEL_FIXED, Algorithm 1
+ *   selection      GLR_SEL_APPROX (default) | GLR_SEL_FIXED
+ * A zero-initialised schedule with tau set is GreedyLore (Algorithm 3) with MSGD.        */
 typedef struct glr_schedule {
     int32_t  tau;
     int32_t  refresh_mode;
@@ -92,6 +100,8 @@ typedef struct glr_schedule {
     int32_t  power_iters;
     int32_t  grad_dtype;
     int32_t  compress_start;
+    int32_t  no_error_feedback;
+    int32_t  selection;
 } glr_schedule;
 
 typedef struct glr_handle glr_handle;

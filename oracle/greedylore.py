@@ -213,7 +213,9 @@ class GreedyLoreOracle:
 
     refresh_mode "alg3": at t mod tau == 0 the node mean is used uncompressed and E is
     reset to 0 (Algorithm 3); "alg4": every step is compressed, the refresh takes
-    P = U[:, :r], and E is never reset (Algorithm 4).  basis_rank k = 0 keeps the full
+    P = U[:, :r], and E is never reset (Algorithm 4).  selection "fixed" keeps
+    P = U[:, :r] for the whole period (the Lazy-SVD of Algorithm 1); error_feedback False
+    keeps E = 0 (with selection "fixed": Algorithm 1).  basis_rank k = 0 keeps the full
     singular basis (paper-exact); 0 < k < m' keeps the top-k singular vectors and
     completes them with the Householder complement.  selection "approx" is
     Algorithm 2; "exact" is Eq. semi-lazy-svd-2.  compress_start K runs the first K
@@ -222,7 +224,7 @@ class GreedyLoreOracle:
 
     def __init__(self, m, n, r, N, tau, *, refresh_mode="alg3", optimizer="msgd", lr=0.01,
                  beta1=0.9, beta2=0.999, eps=1e-8, seed=0, basis_rank=0, selection="approx",
-                 compress_start=0):
+                 compress_start=0, error_feedback=True):
         self.m, self.n, self.r, self.N, self.tau = m, n, r, N, tau
         self.transposed = m > n                      # Algorithm 4, m > n branch
         self.mp, self.np_ = min(m, n), max(m, n)
@@ -231,6 +233,7 @@ class GreedyLoreOracle:
         self.refresh_mode, self.optimizer = refresh_mode, optimizer
         self.lr, self.beta1, self.beta2, self.eps = lr, beta1, beta2, eps
         self.seed, self.selection, self.compress_start = seed, selection, compress_start
+        self.error_feedback = error_feedback
         self.k = self.mp if basis_rank in (0, None) else basis_rank
         if not (r <= self.k <= self.mp):
             raise ValueError("need r <= basis_rank <= min(m, n)")
@@ -291,6 +294,8 @@ class GreedyLoreOracle:
             J = np.array(sorted(force_J))
         elif self.selection == "exact":
             J = argtop_r(exact_energies(Mbar, self.U), self.r)
+        elif self.selection == "fixed":
+            J = np.arange(self.r)                    # Lazy-SVD (Algorithm 1): P = U[:, :r] all period
         else:
             V = gaussian_v(self.seed, t, self.mp, self.np_)
             lam_bar = approx_top_r_lambda(list(M), self.U, V)
@@ -298,6 +303,8 @@ class GreedyLoreOracle:
         P = self.U[:, J]
         R = P.T @ M                                  # R_i = P^T G^(i)   (for every node i)
         self.E = M - P @ R                           # E_i = G^(i) - P R_i
+        if not self.error_feedback:                  # Algorithm 1 / the no-EF comparison: E_i = 0
+            self.E = np.zeros_like(self.E)
         Rbar = R.mean(axis=0)                        # All-Reduce
         Ghat = P @ Rbar
         X = self.apply_optimizer(X, Ghat)

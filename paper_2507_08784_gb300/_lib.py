@@ -37,6 +37,8 @@ class GlrSchedule(ctypes.Structure):
         ("power_iters", ctypes.c_int32),
         ("grad_dtype", ctypes.c_int32),
         ("compress_start", ctypes.c_int32),
+        ("no_error_feedback", ctypes.c_int32),
+        ("selection", ctypes.c_int32),
     ]
 
 

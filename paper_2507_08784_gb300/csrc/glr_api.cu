@@ -529,6 +529,8 @@ int glr_create(int64_t m, int64_t n, int32_t r, int32_t N, const glr_schedule* s
     if (r < 1 || r > mp || r > kMaxRank) return fail(nullptr, GLR_EINVAL, "need 1 <= r <= min(m, n) and r <= 512%s");
     if (N < 1 || N > GLR_MAX_NODES) return fail(nullptr, GLR_EINVAL, "need 1 <= N <= GLR_MAX_NODES%s");
     if (s->tau < 1) return fail(nullptr, GLR_EINVAL, "need tau >= 1%s");
+    if (s->selection != GLR_SEL_APPROX && s->selection != GLR_SEL_FIXED)
+        return fail(nullptr, GLR_EINVAL, "selection must be GLR_SEL_APPROX or GLR_SEL_FIXED%s");
     if (s->refresh_mode != GLR_ALG3 && s->refresh_mode != GLR_ALG4)
         return fail(nullptr, GLR_EINVAL, "unknown refresh_mode%s");
     if (s->optimizer != GLR_MSGD && s->optimizer != GLR_ADAM) return fail(nullptr, GLR_EINVAL, "unknown optimizer%s");
@@ -688,6 +690,7 @@ struct StepPlan {
     const void* const* G = nullptr;
     float* X = nullptr;
     bool warm = false, refresh = false, forced = false, lam_fused = false, compressed = false;
+    bool fixed = false;             // Lazy-SVD selection: J = 0..r-1 (top-r of the last refresh)
     bool stream_update = false;   // K1 writes Wbar and K3 streams X without re-reading Mbar (k_update.cu)
 };
 
@@ -710,7 +713,8 @@ void plan_step(StepPlan& p) {
     if (p.refresh && h->force_refresh) h->period_start = h->t;
     h->force_refresh = false;
     p.forced = !p.warm && !p.refresh && h->has_forceJ;
-    p.lam_fused = h->fused && !h->exact && !p.warm && !p.refresh && !p.forced;
+    p.fixed = !p.warm && !p.refresh && !p.forced && h->s.selection == GLR_SEL_FIXED;
+    p.lam_fused = h->fused && !h->exact && !p.warm && !p.refresh && !p.forced && !p.fixed;
     p.stream_update = p.lam_fused && h->mma && update_stream_eligible(h->mp, h->r, h->transposed);
     p.compressed = !p.warm && !(p.refresh && h->s.refresh_mode == GLR_ALG3);
     h->forced_this_step = p.forced;
@@ -738,7 +742,7 @@ int compose_unfused(StepPlan& p, cudaStream_t st) {
     for (int i = 0; i < N; ++i) ca.G[i] = p.G[i];
     ca.grad_dtype = h->s.grad_dtype; ca.transposed = h->transposed;
     ca.mp = mp; ca.np = np; ca.N = N; ca.r = h->tc ? 0 : r; ca.e_zero = h->e_zero ? 1 : 0;
-    ca.write_B = p.warm ? 0 : 1;
+    ca.write_B = (p.warm || h->s.no_error_feedback) ? 0 : 1;   // B feeds only the error
     ca.B = h->B; ca.Pprev = h->Pprev; ca.Rw = h->Rw; ca.Mbar = h->Mbar;
     if (h->tc) GLR_LAUNCH(h, 1, compose_streamed(ca, st));
     else GLR_LAUNCH(h, 1, compose(ca, st));
@@ -774,7 +778,7 @@ int compose_fused(std::vector<StepPlan*>& plans, cudaStream_t st) {
             }
             StreamMat& M = g.mat[g.nmat];
             M.mp = h->mp; M.np = h->np; M.N = h->N; M.r = h->r; M.k = h->k;
-            M.transposed = h->transposed; M.e_zero = h->e_zero ? 1 : 0; M.write_B = p->warm ? 0 : 1;
+            M.transposed = h->transposed; M.e_zero = h->e_zero ? 1 : 0; M.write_B = (p->warm || h->s.no_error_feedback) ? 0 : 1;
             M.lam = p->lam_fused ? 1 : 0;
             M.g_off = used;
             M.strip0 = g.total_strips; M.nstrips = h->nstrips;
@@ -887,6 +891,9 @@ int select_phase(StepPlan& p, cudaStream_t st) {
         if (h->s.refresh_mode == GLR_ALG3) return GLR_OK;
         GLR_CK(h, cudaMemcpyAsync(h->J, h->iotaJ.data(), sizeof(int32_t) * r, cudaMemcpyHostToDevice, st));
         h->comm += (int64_t)r * np;
+    } else if (p.fixed) {
+        GLR_CK(h, cudaMemcpyAsync(h->J, h->iotaJ.data(), sizeof(int32_t) * r, cudaMemcpyHostToDevice, st));
+        h->comm += (int64_t)r * np;
     } else if (p.forced) {
         GLR_CK(h, cudaMemcpyAsync(h->J, h->forceJ.data(), sizeof(int32_t) * r, cudaMemcpyHostToDevice, st));
         h->has_forceJ = false;
@@ -936,7 +943,7 @@ int select_P_grouped(std::vector<StepPlan>& plans, cudaStream_t st) {
         SelectMat& M = g.mat[g.nmat++];
         M.part = h->lam_part; M.ntiles = p.lam_fused ? h->nstrips : h->ntiles;
         M.mp = h->mp; M.r = h->r; M.k = h->k; M.mode = h->exact ? 0 : 1;
-        M.do_select = (!p.refresh && !p.forced) ? 1 : 0;
+        M.do_select = (!p.refresh && !p.forced && !p.fixed) ? 1 : 0;
         M.dsign = h->exact ? nullptr : h->dsign; M.lam = h->lam; M.J = h->J;
         M.U = h->U; M.Y = h->Y; M.Yt = h->Yt; M.P = h->P;
         M.rbar = p.stream_update ? 1 : 0; M.np = h->np;
@@ -983,7 +990,7 @@ void finish_step(StepPlan& p) {
         h->has_forceJ = false;
     } else {
         std::swap(h->P, h->Pprev);      // Pprev now holds this step's P (deferred E_i = B_i - P P^T B_i)
-        h->e_zero = false;
+        h->e_zero = h->s.no_error_feedback != 0;   // without error feedback E_i stays 0
         h->last_uncompressed = false;
     }
     h->t++;

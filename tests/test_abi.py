@@ -31,10 +31,31 @@ def test_bindings_cover_every_symbol():
     assert set(_lib.header_symbols()) == set(_lib._SIGNATURES)
 
 
-def test_struct_layouts():
-    assert ctypes.sizeof(_lib.GlrSchedule) == 56
-    assert _lib.GlrSchedule.seed.offset == 32
-    assert ctypes.sizeof(_lib.GlrStats) == 64
+def test_struct_layouts(tmp_path):
+    """The ctypes mirrors match the C layout of glr.h, field by field (a C program compiled
+    against the header prints its sizes and offsets)."""
+    import shutil
+    cc = shutil.which("gcc") or shutil.which("cc")
+    if cc is None:
+        pytest.skip("no C compiler")
+    fields = {"glr_schedule": _lib.GlrSchedule, "glr_stats": _lib.GlrStats}
+    lines = ['#include <stdio.h>', '#include <stddef.h>', '#include "glr.h"', 'int main(void) {']
+    for cname, cls in fields.items():
+        lines.append(f'printf("{cname} %zu\\n", sizeof({cname}));')
+        for f, _ in cls._fields_:
+            lines.append(f'printf("{cname}.{f} %zu\\n", offsetof({cname}, {f}));')
+    lines += ['return 0;', '}']
+    src = tmp_path / "layout.c"
+    src.write_text("\n".join(lines) + "\n")
+    exe = tmp_path / "layout"
+    inc = os.path.join(os.path.dirname(os.path.dirname(os.path.abspath(__file__))), "include")
+    subprocess.run([cc, "-std=c99", "-I", inc, str(src), "-o", str(exe)], check=True)
+    got = dict(line.split() for line in subprocess.run([str(exe)], capture_output=True, text=True,
+                                                        check=True).stdout.splitlines())
+    for cname, cls in fields.items():
+        assert int(got[cname]) == ctypes.sizeof(cls), cname
+        for f, _ in cls._fields_:
+            assert int(got[f"{cname}.{f}"]) == getattr(cls, f).offset, f"{cname}.{f}"
 
 
 @pytest.mark.parametrize("m,n,r,N,kw,frag", [

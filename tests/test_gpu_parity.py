@@ -91,6 +91,18 @@ def test_compress_start_warmup_lockstep():
     assert [r.refresh for r in reps[:4]] == [False, False, False, True]
 
 
+@pytest.mark.parametrize("m,n,k,selection", [(96, 400, 16, "fixed"), (96, 400, 0, "fixed"), (640, 1280, 16, "approx"),
+                                              (300, 130, 24, "fixed"), (200, 824, 24, "approx")])
+def test_without_error_feedback_lockstep(m, n, k, selection):
+    """Algorithm 1 (Lazy-SVD selection, no error feedback) and Approx-Top-r without error
+    feedback (the comparison of Sec. 4), on the tensor-core, FFMA-strip, transposed and
+    paper-exact paths."""
+    g = _synthetic(m, n, 3, 24, lambda j: 1.0 / j, 0.05, 80 + m + k)
+    reps = lockstep(m, n, 5, 3, 6, g, tau=3, optimizer="msgd", lr=0.05, beta1=0.9, seed=11, basis_rank=k,
+                    error_feedback=False, selection=selection)
+    _assert_reports(reps)
+
+
 @pytest.mark.parametrize("m,n,r,N,k", [(1, 5, 1, 1, 0), (7, 7, 7, 1, 0), (9, 40, 1, 3, 0), (40, 9, 2, 2, 3),
                                        (65, 65, 65, 2, 0)])
 def test_edge_shapes(m, n, r, N, k):

@@ -418,3 +418,45 @@ def test_step_selection_is_unbiased_and_takes_the_largest_squares():
         sq[trial] = lam2
     target = O.exact_energies(G.mean(0), base.U)
     assert np.all(np.abs(sq.mean(0) - target) < 5 * sq.std(0) / math.sqrt(T))
+
+
+def test_algorithm1_lazy_svd_sends_the_top_r_projection():
+    """Algorithm 1 (selection fixed, no error feedback): every compressed step of a period sends
+    U_r U_r^T Gbar_t with U_r the top-r left singular vectors (numpy's SVD) of the period's
+    refresh mean, and keeps E = 0."""
+    rng = np.random.default_rng(21)
+    m, n, r, N, tau = 12, 20, 3, 4, 4
+    orc = O.GreedyLoreOracle(m, n, r, N, tau, selection="fixed", error_feedback=False, seed=5)
+    X = np.zeros((m, n))
+    Ur = None
+    for t in range(2 * tau):
+        G = rng.standard_normal((N, m, n))
+        X, info = orc.step(G, X)
+        if t % tau == 0:
+            U, _, _ = np.linalg.svd(G.mean(axis=0))
+            Ur = U[:, :r]
+            assert not info.compressed
+            continue
+        assert np.array_equal(info.J, np.arange(r))
+        np.testing.assert_allclose(np.abs(info.P), np.abs(Ur), atol=1e-10)   # columns up to sign
+        np.testing.assert_allclose(info.Ghat, Ur @ (Ur.T @ G.mean(axis=0)), atol=1e-10)
+        assert np.all(info.E == 0.0)
+
+
+def test_prop1_frozen_subspace_makes_error_feedback_inert():
+    """Prop. 1 through the Lazy-SVD selection: with P = U[:, :r] frozen for the period, E_i stays
+    orthogonal to range(P), so runs with and without error feedback send the same Ghat."""
+    rng = np.random.default_rng(22)
+    m, n, r, N, tau = 10, 16, 2, 3, 5
+    a = O.GreedyLoreOracle(m, n, r, N, tau, selection="fixed", error_feedback=True, seed=1)
+    b = O.GreedyLoreOracle(m, n, r, N, tau, selection="fixed", error_feedback=False, seed=1)
+    Xa = np.zeros((m, n))
+    Xb = np.zeros((m, n))
+    for t in range(tau):
+        G = rng.standard_normal((N, m, n))
+        Xa, ia = a.step(G, Xa)
+        Xb, ib = b.step(G, Xb)
+        np.testing.assert_allclose(ia.Ghat, ib.Ghat, atol=1e-12)
+        if ia.compressed:
+            assert np.abs(ia.P.T @ ia.E[0]).max() < 1e-12       # E_i is orthogonal to range(P)
+            assert np.abs(ia.E).max() > 0.1                     # ... and not zero
