@@ -58,6 +58,8 @@ extern "C" {
 
 #define GLR_MSGD 0   /* Eq. msgd:  M = b1 M + (1 - b1) G;  X -= lr M                          */
 #define GLR_ADAM 1   /* Eq. adam:  M, V EMAs; X -= lr M / (sqrt(V) + eps); no bias correction */
+#define GLR_AMSGRAD 2   /* the analysis' AMSGrad-type Adam (App. A): M, V EMAs as GLR_ADAM,   *
+                         * Vt = max(Vt, max_e V), X -= lr M / sqrt(Vt + eps) (one scalar)    */
 
 #define GLR_SEL_APPROX 0   /* Algorithm 2 (Approx-Top-r) picks J at every compressed step    */
 #define GLR_SEL_FIXED  1   /* P = U[:, :r] for the whole refresh period: the Lazy-SVD of       *
@@ -71,8 +73,8 @@ extern "C" {
 /* Compressor and optimizer settings (Algorithm 3 inputs: tau, r; Sec. 2 optimizers).
  *   tau            refresh period (>= 1)
  *   refresh_mode   GLR_ALG3 | GLR_ALG4
- *   optimizer      GLR_MSGD | GLR_ADAM; lr = gamma; beta1 = beta (MSGD) or beta_1 (Adam);
- *                  beta2, eps used by Adam only
+ *   optimizer      GLR_MSGD | GLR_ADAM | GLR_AMSGRAD; lr = gamma; beta1 = beta (MSGD) or
+ *                  beta_1 (Adam types); beta2, eps used by the Adam types only
  *   seed           64-bit key of the shared random vectors v_j (Eq. random-v): all nodes
  *                  of one matrix draw the same v_j; give every matrix its own seed
  *   basis_rank     k.  0 (or m') keeps the full m' x m' singular basis U of Eq. SVD-P1

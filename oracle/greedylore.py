@@ -16,7 +16,7 @@ with Convergence Guarantees" (arXiv 2507.08784):
 * error feedback Eq. ef1/ef2 as written in Algorithm 3 (E reset at a refresh)
   or Algorithm 4 (no reset, always compressed);
 * the optimizers of Eq. msgd and Eq. adam (no bias correction, eps outside the
-  square root);
+  square root), and the AMSGrad-type Adam of the convergence analysis (Appendix A);
 * the truncated-basis reading: the top-k singular vectors of the refresh
   matrix completed to a full orthogonal U by Householder QR (the proofs of
   Prop. 3 and Lemma 2 only use that U is orthogonal).
@@ -167,6 +167,15 @@ def msgd_update(X, Mo, G, lr, beta):
     return X - lr * Mo, Mo
 
 
+def amsgrad_update(X, Mo, Vo, Vt, G, lr, beta1, beta2, eps):
+    """The AMSGrad-type Adam of the convergence analysis (Appendix A): the EMAs of Eq. adam and one
+    scalar normaliser Vt = max(Vt, ||V||_max), X <- X - lr M / sqrt(Vt + eps)."""
+    Mo = beta1 * Mo + (1.0 - beta1) * G
+    Vo = beta2 * Vo + (1.0 - beta2) * G * G
+    Vt = max(Vt, float(np.max(Vo)))
+    return X - lr * Mo / np.sqrt(Vt + eps), Mo, Vo, Vt
+
+
 def adam_update(X, Mo, Vo, G, lr, beta1, beta2, eps):
     Mo = beta1 * Mo + (1.0 - beta1) * G
     Vo = beta2 * Vo + (1.0 - beta2) * G * G
@@ -242,6 +251,7 @@ class GreedyLoreOracle:
         self.sigma = None
         self.Mo = np.zeros((m, n))
         self.Vo = np.zeros((m, n))
+        self.Vt = 0.0                                # AMSGrad-type scalar normaliser
         self.t = 0
 
     # -- helpers ---------------------------------------------------------------
@@ -259,6 +269,9 @@ class GreedyLoreOracle:
         G = self.orient(Ghat_oriented)               # back to m x n (transpose only when m > n)
         if self.optimizer == "msgd":
             X, self.Mo = msgd_update(X, self.Mo, G, self.lr, self.beta1)
+        elif self.optimizer == "amsgrad":
+            X, self.Mo, self.Vo, self.Vt = amsgrad_update(X, self.Mo, self.Vo, self.Vt, G, self.lr, self.beta1,
+                                                          self.beta2, self.eps)
         else:
             X, self.Mo, self.Vo = adam_update(X, self.Mo, self.Vo, G, self.lr, self.beta1, self.beta2, self.eps)
         return X

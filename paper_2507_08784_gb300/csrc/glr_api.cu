@@ -57,6 +57,7 @@ struct glr_handle {
     float* jwork = nullptr;      // full basis: the grouped Jacobi's second m' x m' buffer
     float* jpart = nullptr;      // full basis: its per-CTA norm partials (used by a group's first handle)
     float* YtJ = nullptr;        // Yt[J, :] (r x k) for P = U[:, J] as a library product
+    float* amsv = nullptr;       // AMSGrad: the scalar normaliser and this step's maximum of V
     cudaStream_t rstream = nullptr;            // side stream of this handle's refresh
     cudaEvent_t rfork = nullptr, rdone = nullptr, rpow = nullptr;
     int pow_ok = 0;                            // refresh through the grouped power iteration (k_power.cu)
@@ -505,6 +506,23 @@ int uncompressed_update(glr_handle* h, float* X, cudaStream_t st) {
     return GLR_OK;
 }
 
+// The AMSGrad-type optimizer step (Appendix A) with Ghat = Mbar (uncompressed) or P Rbar, both
+// products formed here (Rbar = P^T Mbar): one path for every kernel family.
+int amsgrad_step_update(glr_handle* h, float* X, bool compressed, cudaStream_t st) {
+    const int mp = h->mp, np = h->np, r = h->r;
+    const float* Gh = h->Mbar;
+    if (compressed) {
+        PhaseScope ps(h, GLR_PH_PROJECT, st);
+        GLR_GEMM(h, gd(r, np, mp, h->P, 1, r, h->Mbar, np, 1, h->Rbar, np, 1), st);
+        GLR_GEMM(h, gd(mp, np, r, h->P, r, 1, h->Rbar, np, 1, h->mn_scratch, np, 1), st);
+        Gh = h->mn_scratch;
+    }
+    PhaseScope ps(h, GLR_PH_UPDATE, st);
+    GLR_LAUNCH(h, 3, amsgrad_update(Gh, mp, np, h->transposed, X, h->Mo, h->Vo, h->amsv, h->s.lr, h->s.beta1,
+                                    h->s.beta2, h->s.eps, st));
+    return GLR_OK;
+}
+
 int build_selection_P(glr_handle* h, cudaStream_t st) {
     GLR_LAUNCH(h, 1, build_P(h->exact ? 0 : 1, h->mp, h->r, h->k, h->J, h->U, h->Y, h->Yt, h->dsign, h->P, st));
     return GLR_OK;
@@ -533,7 +551,8 @@ int glr_create(int64_t m, int64_t n, int32_t r, int32_t N, const glr_schedule* s
         return fail(nullptr, GLR_EINVAL, "selection must be GLR_SEL_APPROX or GLR_SEL_FIXED%s");
     if (s->refresh_mode != GLR_ALG3 && s->refresh_mode != GLR_ALG4)
         return fail(nullptr, GLR_EINVAL, "unknown refresh_mode%s");
-    if (s->optimizer != GLR_MSGD && s->optimizer != GLR_ADAM) return fail(nullptr, GLR_EINVAL, "unknown optimizer%s");
+    if (s->optimizer != GLR_MSGD && s->optimizer != GLR_ADAM && s->optimizer != GLR_AMSGRAD)
+        return fail(nullptr, GLR_EINVAL, "unknown optimizer%s");
     if (s->grad_dtype != GLR_F32 && s->grad_dtype != GLR_BF16) return fail(nullptr, GLR_EINVAL, "unknown grad_dtype%s");
     if (s->compress_start < 0) return fail(nullptr, GLR_EINVAL, "need compress_start >= 0%s");
     const int k = (s->basis_rank == 0 || s->basis_rank == mp) ? static_cast<int>(mp) : s->basis_rank;
@@ -588,12 +607,13 @@ int glr_create(int64_t m, int64_t n, int32_t r, int32_t N, const glr_schedule* s
     A(&h->lam, MP);
     A(&h->lam_part, MP * std::max(h->ntiles, h->nstrips));
     A(&h->Mo, (size_t)m * n);
-    if (s->optimizer == GLR_ADAM) A(&h->Vo, (size_t)m * n);
+    if (s->optimizer == GLR_ADAM || s->optimizer == GLR_AMSGRAD) A(&h->Vo, (size_t)m * n);
+    if (s->optimizer == GLR_AMSGRAD) A(&h->amsv, 2);
     A(&h->dflags, 4);
     A(&h->gemm_ws, (size_t)kGemmWsFloats);
     // the first path with library products when the rank-r products are large
     h->tc = !h->fused && mp % 4 == 0 && np % 4 == 0 && 2.0 * r * (double)mp * (double)np * N >= 67108864.0 ? 1 : 0;
-    if (h->tc) A(&h->mn_scratch, MP * NP);
+    if (h->tc || s->optimizer == GLR_AMSGRAD) A(&h->mn_scratch, MP * NP);
     if (h->tc && !exact) A(&h->YtJ, (size_t)r * k);
     if (exact) {
         A(&h->jwork, MP * MP);
@@ -715,7 +735,8 @@ void plan_step(StepPlan& p) {
     p.forced = !p.warm && !p.refresh && h->has_forceJ;
     p.fixed = !p.warm && !p.refresh && !p.forced && h->s.selection == GLR_SEL_FIXED;
     p.lam_fused = h->fused && !h->exact && !p.warm && !p.refresh && !p.forced && !p.fixed;
-    p.stream_update = p.lam_fused && h->mma && update_stream_eligible(h->mp, h->r, h->transposed);
+    p.stream_update = p.lam_fused && h->mma && h->s.optimizer != GLR_AMSGRAD &&
+                      update_stream_eligible(h->mp, h->r, h->transposed);
     p.compressed = !p.warm && !(p.refresh && h->s.refresh_mode == GLR_ALG3);
     h->forced_this_step = p.forced;
 }
@@ -1033,11 +1054,17 @@ int step_group(std::vector<StepPlan>& plans, cudaStream_t st) {
     for (glr_handle* h : refreshing) GLR_CK(h, cudaStreamWaitEvent(st, h->rdone, 0));
     if ((rc = select_P_grouped(plans, st)) != GLR_OK) return rc;
     std::vector<StepPlan*> streamed, strips;
-    for (StepPlan* p : fused) (p->stream_update ? streamed : strips).push_back(p);
+    for (StepPlan* p : fused) {
+        if (p->h->s.optimizer == GLR_AMSGRAD) continue;
+        (p->stream_update ? streamed : strips).push_back(p);
+    }
     if (!streamed.empty() && (rc = update_streamed(streamed, st)) != GLR_OK) return rc;
     if (!strips.empty() && (rc = update_fused(strips, st)) != GLR_OK) return rc;
     for (StepPlan* p : unfused)
-        if ((rc = update_unfused(*p, st)) != GLR_OK) return rc;
+        if (p->h->s.optimizer != GLR_AMSGRAD && (rc = update_unfused(*p, st)) != GLR_OK) return rc;
+    for (StepPlan& p : plans)
+        if (p.h->s.optimizer == GLR_AMSGRAD && (rc = amsgrad_step_update(p.h, p.X, p.compressed, st)) != GLR_OK)
+            return rc;
     for (StepPlan& p : plans) finish_step(p);
     return GLR_OK;
 }

@@ -185,6 +185,10 @@ cudaError_t update(const UpdateArgs& a, cudaStream_t st);
 // X's element count as two factors) and runs the optimizer element by element.
 cudaError_t compose_streamed(const ComposeArgs& a, cudaStream_t st);
 cudaError_t update_streamed_flat(const UpdateArgs& a, cudaStream_t st);
+// The AMSGrad-type optimizer step (k_big.cu): Ghat oriented m' x n', X / Mo / Vo in X's layout;
+// vt[0] is the running scalar normaliser, vt[1] scratch for this step's maximum of V.
+cudaError_t amsgrad_update(const float* Ghat, int mp, int np, int transposed, float* X, float* Mo, float* Vo,
+                           float* vt, float lr, float beta1, float beta2, float eps, cudaStream_t st);
 
 // E_i = B_i - Pprev (Pprev^T B_i) given Rw_i = Pprev^T B_i  (or 0 when e_zero)
 cudaError_t materialize_error(int mp, int np, int r, int e_zero, const float* B, const float* Pprev,

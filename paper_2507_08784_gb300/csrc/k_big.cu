@@ -133,6 +133,47 @@ __global__ void __launch_bounds__(TB) update_flat_kernel(UpdateArgs a) {
     }
 }
 
+// The AMSGrad-type Adam of the convergence analysis (Appendix A): M and V are the EMAs of Ghat
+// as in Eq. adam, the normaliser is one scalar, Vt = max(Vt, max over elements of V), and
+// X -= lr M / sqrt(Vt + eps).  Ghat is read oriented (m' x n'); X, M, V are in X's layout
+// (transposed when m > n).  The maximum is taken over non-negative floats, whose bit patterns
+// order like their values, so an integer atomic max gives it exactly, in any order.
+__global__ void __launch_bounds__(TB) amsgrad_moments_kernel(const float* Gh, int mp, int np, int transposed,
+                                                             float* Mo, float* Vo, float b1, float b2,
+                                                             unsigned* vmax_bits) {
+    __shared__ unsigned red[TB / 32];
+    const int64_t total = (int64_t)mp * np;
+    const int xcols = transposed ? mp : np;
+    unsigned local = 0u;
+    for (int64_t e = (int64_t)blockIdx.x * TB + threadIdx.x; e < total; e += (int64_t)gridDim.x * TB) {
+        const int xr = static_cast<int>(e / xcols), xc = static_cast<int>(e % xcols);
+        const int a = transposed ? xc : xr, b = transposed ? xr : xc;
+        const float g = Gh[(int64_t)a * np + b];
+        const float m = fmaf(b1, Mo[e], (1.0f - b1) * g);
+        const float v = fmaf(b2, Vo[e], (1.0f - b2) * g * g);
+        Mo[e] = m;
+        Vo[e] = v;
+        local = max(local, __float_as_uint(v));
+    }
+    for (int o = 16; o > 0; o >>= 1) local = max(local, __shfl_xor_sync(0xffffffffu, local, o));
+    if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = local;
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        unsigned mx = 0u;
+        for (int w = 0; w < TB / 32; ++w) mx = max(mx, red[w]);
+        atomicMax(vmax_bits, mx);
+    }
+}
+__global__ void amsgrad_scalar_kernel(float* vt, const unsigned* vmax_bits) {
+    vt[0] = fmaxf(vt[0], __uint_as_float(*vmax_bits));
+}
+__global__ void __launch_bounds__(TB) amsgrad_apply_kernel(float* X, const float* Mo, const float* vt, int64_t total,
+                                                           float lr, float eps) {
+    const float scale = lr / sqrtf(vt[0] + eps);
+    for (int64_t e = (int64_t)blockIdx.x * TB + threadIdx.x; e < total; e += (int64_t)gridDim.x * TB)
+        X[e] -= scale * Mo[e];
+}
+
 int stream_grid(int64_t quads) {
     static int sms = 0;
     if (!sms) {
@@ -154,6 +195,21 @@ cudaError_t compose_streamed(const ComposeArgs& a, cudaStream_t st) {
     } else {
         compose_rows_kernel<<<stream_grid((int64_t)a.mp * a.np / 4), TB, 0, st>>>(a);
     }
+    return cudaGetLastError();
+}
+
+cudaError_t amsgrad_update(const float* Ghat, int mp, int np, int transposed, float* X, float* Mo, float* Vo,
+                           float* vt, float lr, float beta1, float beta2, float eps, cudaStream_t st) {
+    const int64_t total = (int64_t)mp * np;
+    unsigned* bits = reinterpret_cast<unsigned*>(vt + 1);
+    cudaError_t e = cudaMemsetAsync(bits, 0, sizeof(unsigned), st);
+    if (e != cudaSuccess) return e;
+    const int grid = stream_grid((total + 3) / 4);
+    amsgrad_moments_kernel<<<grid, TB, 0, st>>>(Ghat, mp, np, transposed, Mo, Vo, beta1, beta2, bits);
+    if ((e = cudaGetLastError()) != cudaSuccess) return e;
+    amsgrad_scalar_kernel<<<1, 1, 0, st>>>(vt, bits);
+    if ((e = cudaGetLastError()) != cudaSuccess) return e;
+    amsgrad_apply_kernel<<<grid, TB, 0, st>>>(X, Mo, vt, total, lr, eps);
     return cudaGetLastError();
 }
 

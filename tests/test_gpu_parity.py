@@ -91,6 +91,16 @@ def test_compress_start_warmup_lockstep():
     assert [r.refresh for r in reps[:4]] == [False, False, False, True]
 
 
+@pytest.mark.parametrize("m,n,k", [(96, 400, 16), (96, 400, 0), (300, 130, 24), (640, 1280, 16)])
+def test_amsgrad_lockstep(m, n, k):
+    """The AMSGrad-type optimizer of the analysis (scalar normaliser) on the tensor-core,
+    paper-exact, transposed and FFMA-strip paths."""
+    g = _synthetic(m, n, 3, 24, lambda j: 1.0 / j, 0.05, 90 + m + k)
+    reps = lockstep(m, n, 5, 3, 6, g, tau=3, optimizer="amsgrad", lr=1e-3, beta1=0.9, beta2=0.999, eps=1e-8,
+                    seed=12, basis_rank=k)
+    _assert_reports(reps, tol=1e-4)
+
+
 @pytest.mark.parametrize("m,n,k,selection", [(96, 400, 16, "fixed"), (96, 400, 0, "fixed"), (640, 1280, 16, "approx"),
                                               (300, 130, 24, "fixed"), (200, 824, 24, "approx")])
 def test_without_error_feedback_lockstep(m, n, k, selection):

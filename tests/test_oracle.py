@@ -460,3 +460,23 @@ def test_prop1_frozen_subspace_makes_error_feedback_inert():
         if ia.compressed:
             assert np.abs(ia.P.T @ ia.E[0]).max() < 1e-12       # E_i is orthogonal to range(P)
             assert np.abs(ia.E).max() > 0.1                     # ... and not zero
+
+
+def test_amsgrad_closed_form_and_monotone_normaliser():
+    """The AMSGrad-type step of Appendix A: from a zero state one step gives
+    X = -lr (1 - b1) G / sqrt((1 - b2) max G^2 + eps); with zero gradients afterwards V decays but
+    the scalar normaliser Vt does not, and M keeps decaying geometrically."""
+    rng = np.random.default_rng(23)
+    G = rng.standard_normal((5, 7))
+    lr, b1, b2, eps = 0.01, 0.9, 0.999, 1e-8
+    X, M, V, Vt = O.amsgrad_update(np.zeros((5, 7)), np.zeros((5, 7)), np.zeros((5, 7)), 0.0, G, lr, b1, b2, eps)
+    vt1 = (1 - b2) * float(np.max(G * G))
+    assert Vt == pytest.approx(vt1, rel=1e-15)
+    np.testing.assert_allclose(X, -lr * (1 - b1) * G / np.sqrt(vt1 + eps), rtol=1e-13)
+    prev = Vt
+    for k in range(1, 6):
+        X2, M, V, Vt = O.amsgrad_update(X, M, V, Vt, np.zeros((5, 7)), lr, b1, b2, eps)
+        assert float(np.max(V)) < prev and Vt == prev               # V decays, Vt holds
+        np.testing.assert_allclose(M, (1 - b1) * b1 ** k * G, rtol=1e-13)
+        np.testing.assert_allclose(X2 - X, -lr * M / np.sqrt(vt1 + eps), rtol=1e-12)
+        X = X2
