@@ -60,6 +60,9 @@ extern "C" {
 #define GLR_ADAM 1   /* Eq. adam:  M, V EMAs; X -= lr M / (sqrt(V) + eps); no bias correction */
 #define GLR_AMSGRAD 2   /* the analysis' AMSGrad-type Adam (App. A): M, V EMAs as GLR_ADAM,   *
                          * Vt = max(Vt, max_e V), X -= lr M / sqrt(Vt + eps) (one scalar)    */
+#define GLR_ADAMW 3     /* bias-corrected AdamW: M, V EMAs, X -= lr (Mh / (sqrt(Vh) + eps) +   *
+                         * weight_decay X), Mh = M / (1 - b1^s), Vh = V / (1 - b2^s), s = the  *
+                         * optimizer step (1, 2, ...: every step, refresh and warm-up included)*/
 
 #define GLR_SEL_APPROX 0   /* Algorithm 2 (Approx-Top-r) picks J at every compressed step    */
 #define GLR_SEL_FIXED  1   /* P = U[:, :r] for the whole refresh period: the Lazy-SVD of       *
@@ -73,8 +76,8 @@ extern "C" {
 /* Compressor and optimizer settings (Algorithm 3 inputs: tau, r; Sec. 2 optimizers).
  *   tau            refresh period (>= 1)
  *   refresh_mode   GLR_ALG3 | GLR_ALG4
- *   optimizer      GLR_MSGD | GLR_ADAM | GLR_AMSGRAD; lr = gamma; beta1 = beta (MSGD) or
- *                  beta_1 (Adam types); beta2, eps used by the Adam types only
+ *   optimizer      GLR_MSGD | GLR_ADAM | GLR_AMSGRAD | GLR_ADAMW; lr = gamma; beta1 = beta
+ *                  (MSGD) or beta_1 (Adam types); beta2, eps used by the Adam types only
  *   seed           64-bit key of the shared random vectors v_j (Eq. random-v): all nodes
  *                  of one matrix draw the same v_j; give every matrix its own seed
  *   basis_rank     k.  0 (or m') keeps the full m' x m' singular basis U of Eq. SVD-P1
@@ -88,6 +91,7 @@ extern "C" {
  *   no_error_feedback  1 drops error feedback (E_i stays 0, M_i = G_i): the comparison of
  *                  Sec. 4 / Fig. 2 and, with selection = GLR_SEL_FIXED, Algorithm 1
  *   selection      GLR_SEL_APPROX (default) | GLR_SEL_FIXED
+ *   weight_decay   GLR_ADAMW's decoupled weight decay (ignored by the other optimizers)
  * A zero-initialised schedule with tau set is GreedyLore (Algorithm 3) with MSGD.        */
 typedef struct glr_schedule {
     int32_t  tau;
@@ -104,6 +108,7 @@ typedef struct glr_schedule {
     int32_t  compress_start;
     int32_t  no_error_feedback;
     int32_t  selection;
+    float    weight_decay;
 } glr_schedule;
 
 typedef struct glr_handle glr_handle;

@@ -16,7 +16,8 @@ with Convergence Guarantees" (arXiv 2507.08784):
 * error feedback Eq. ef1/ef2 as written in Algorithm 3 (E reset at a refresh)
   or Algorithm 4 (no reset, always compressed);
 * the optimizers of Eq. msgd and Eq. adam (no bias correction, eps outside the
-  square root), and the AMSGrad-type Adam of the convergence analysis (Appendix A);
+  square root), the AMSGrad-type Adam of the convergence analysis (Appendix A), and
+  bias-corrected AdamW;
 * the truncated-basis reading: the top-k singular vectors of the refresh
   matrix completed to a full orthogonal U by Householder QR (the proofs of
   Prop. 3 and Lemma 2 only use that U is orthogonal).
@@ -176,6 +177,16 @@ def amsgrad_update(X, Mo, Vo, Vt, G, lr, beta1, beta2, eps):
     return X - lr * Mo / np.sqrt(Vt + eps), Mo, Vo, Vt
 
 
+def adamw_update(X, Mo, Vo, s, G, lr, beta1, beta2, eps, weight_decay):
+    """Bias-corrected AdamW with decoupled weight decay (Loshchilov & Hutter) at optimizer step
+    s = 1, 2, ...: Mh = M / (1 - b1^s), Vh = V / (1 - b2^s), X <- X - lr (Mh / (sqrt(Vh) + eps) + wd X)."""
+    Mo = beta1 * Mo + (1.0 - beta1) * G
+    Vo = beta2 * Vo + (1.0 - beta2) * G * G
+    Mh = Mo / (1.0 - beta1 ** s)
+    Vh = Vo / (1.0 - beta2 ** s)
+    return X - lr * (Mh / (np.sqrt(Vh) + eps) + weight_decay * X), Mo, Vo
+
+
 def adam_update(X, Mo, Vo, G, lr, beta1, beta2, eps):
     Mo = beta1 * Mo + (1.0 - beta1) * G
     Vo = beta2 * Vo + (1.0 - beta2) * G * G
@@ -233,7 +244,7 @@ class GreedyLoreOracle:
 
     def __init__(self, m, n, r, N, tau, *, refresh_mode="alg3", optimizer="msgd", lr=0.01,
                  beta1=0.9, beta2=0.999, eps=1e-8, seed=0, basis_rank=0, selection="approx",
-                 compress_start=0, error_feedback=True):
+                 compress_start=0, error_feedback=True, weight_decay=0.0):
         self.m, self.n, self.r, self.N, self.tau = m, n, r, N, tau
         self.transposed = m > n                      # Algorithm 4, m > n branch
         self.mp, self.np_ = min(m, n), max(m, n)
@@ -242,7 +253,7 @@ class GreedyLoreOracle:
         self.refresh_mode, self.optimizer = refresh_mode, optimizer
         self.lr, self.beta1, self.beta2, self.eps = lr, beta1, beta2, eps
         self.seed, self.selection, self.compress_start = seed, selection, compress_start
-        self.error_feedback = error_feedback
+        self.error_feedback, self.weight_decay = error_feedback, weight_decay
         self.k = self.mp if basis_rank in (0, None) else basis_rank
         if not (r <= self.k <= self.mp):
             raise ValueError("need r <= basis_rank <= min(m, n)")
@@ -269,6 +280,9 @@ class GreedyLoreOracle:
         G = self.orient(Ghat_oriented)               # back to m x n (transpose only when m > n)
         if self.optimizer == "msgd":
             X, self.Mo = msgd_update(X, self.Mo, G, self.lr, self.beta1)
+        elif self.optimizer == "adamw":
+            X, self.Mo, self.Vo = adamw_update(X, self.Mo, self.Vo, self.t + 1, G, self.lr, self.beta1, self.beta2,
+                                               self.eps, self.weight_decay)
         elif self.optimizer == "amsgrad":
             X, self.Mo, self.Vo, self.Vt = amsgrad_update(X, self.Mo, self.Vo, self.Vt, G, self.lr, self.beta1,
                                                           self.beta2, self.eps)

@@ -50,13 +50,14 @@ def _stream_ptr(stream) -> int:
 def make_schedule(tau: int, refresh_mode: str = "alg3", optimizer: str = "msgd", lr: float = 0.01,
                   beta1: float = 0.9, beta2: float = 0.999, eps: float = 1e-8, seed: int = 0,
                   basis_rank: int = 0, power_iters: int = 4, grad_dtype: str = "f32",
-                  compress_start: int = 0, error_feedback: bool = True, selection: str = "approx") -> GlrSchedule:
+                  compress_start: int = 0, error_feedback: bool = True, selection: str = "approx",
+                  weight_decay: float = 0.0) -> GlrSchedule:
     return GlrSchedule(tau=tau, refresh_mode={"alg3": GLR_ALG3, "alg4": GLR_ALG4}[refresh_mode],
-                       optimizer={"msgd": GLR_MSGD, "adam": GLR_ADAM, "amsgrad": 2}[optimizer], lr=lr, beta1=beta1,
+                       optimizer={"msgd": GLR_MSGD, "adam": GLR_ADAM, "amsgrad": 2, "adamw": 3}[optimizer], lr=lr, beta1=beta1,
                        beta2=beta2, eps=eps, seed=seed & (2 ** 64 - 1), basis_rank=basis_rank,
                        power_iters=power_iters, grad_dtype={"f32": GLR_F32, "bf16": GLR_BF16}[grad_dtype],
                        compress_start=compress_start, no_error_feedback=0 if error_feedback else 1,
-                       selection={"approx": 0, "fixed": 1}[selection])
+                       selection={"approx": 0, "fixed": 1}[selection], weight_decay=weight_decay)
 
 
 def glr_create(m: int, n: int, r: int, N: int, schedule: GlrSchedule) -> ctypes.c_void_p:

@@ -39,6 +39,7 @@ class GlrSchedule(ctypes.Structure):
         ("compress_start", ctypes.c_int32),
         ("no_error_feedback", ctypes.c_int32),
         ("selection", ctypes.c_int32),
+        ("weight_decay", ctypes.c_float),
     ]
 
 

@@ -2,6 +2,7 @@
 // refresh every tau steps, Approx-Top-r selection otherwise) and the introspection calls.
 // All device work is enqueued on the caller's stream; the host only tracks the schedule.
 #include <algorithm>
+#include <cmath>
 #include <cstdio>
 #include <cstring>
 #include <string>
@@ -506,9 +507,14 @@ int uncompressed_update(glr_handle* h, float* X, cudaStream_t st) {
     return GLR_OK;
 }
 
-// The AMSGrad-type optimizer step (Appendix A) with Ghat = Mbar (uncompressed) or P Rbar, both
-// products formed here (Rbar = P^T Mbar): one path for every kernel family.
-int amsgrad_step_update(glr_handle* h, float* X, bool compressed, cudaStream_t st) {
+// The optimizers outside the fused update kernels — the AMSGrad-type step of Appendix A and
+// bias-corrected AdamW — with Ghat = Mbar (uncompressed) or P Rbar, both products formed here
+// (Rbar = P^T Mbar): one path for every kernel family.
+bool separate_optimizer(const glr_handle* h) {
+    return h->s.optimizer == GLR_AMSGRAD || h->s.optimizer == GLR_ADAMW;
+}
+
+int separate_optimizer_update(glr_handle* h, float* X, bool compressed, cudaStream_t st) {
     const int mp = h->mp, np = h->np, r = h->r;
     const float* Gh = h->Mbar;
     if (compressed) {
@@ -518,6 +524,14 @@ int amsgrad_step_update(glr_handle* h, float* X, bool compressed, cudaStream_t s
         Gh = h->mn_scratch;
     }
     PhaseScope ps(h, GLR_PH_UPDATE, st);
+    if (h->s.optimizer == GLR_ADAMW) {
+        const double s = static_cast<double>(h->t + 1);      // this step's optimizer step, 1-based
+        const float c1 = static_cast<float>(1.0 / (1.0 - std::pow(static_cast<double>(h->s.beta1), s)));
+        const float c2 = static_cast<float>(1.0 / (1.0 - std::pow(static_cast<double>(h->s.beta2), s)));
+        GLR_LAUNCH(h, 1, adamw_update(Gh, mp, np, h->transposed, X, h->Mo, h->Vo, h->s.lr, h->s.beta1, h->s.beta2,
+                                      h->s.eps, h->s.weight_decay, c1, c2, st));
+        return GLR_OK;
+    }
     GLR_LAUNCH(h, 3, amsgrad_update(Gh, mp, np, h->transposed, X, h->Mo, h->Vo, h->amsv, h->s.lr, h->s.beta1,
                                     h->s.beta2, h->s.eps, st));
     return GLR_OK;
@@ -551,7 +565,7 @@ int glr_create(int64_t m, int64_t n, int32_t r, int32_t N, const glr_schedule* s
         return fail(nullptr, GLR_EINVAL, "selection must be GLR_SEL_APPROX or GLR_SEL_FIXED%s");
     if (s->refresh_mode != GLR_ALG3 && s->refresh_mode != GLR_ALG4)
         return fail(nullptr, GLR_EINVAL, "unknown refresh_mode%s");
-    if (s->optimizer != GLR_MSGD && s->optimizer != GLR_ADAM && s->optimizer != GLR_AMSGRAD)
+    if (s->optimizer != GLR_MSGD && s->optimizer != GLR_ADAM && s->optimizer != GLR_AMSGRAD && s->optimizer != GLR_ADAMW)
         return fail(nullptr, GLR_EINVAL, "unknown optimizer%s");
     if (s->grad_dtype != GLR_F32 && s->grad_dtype != GLR_BF16) return fail(nullptr, GLR_EINVAL, "unknown grad_dtype%s");
     if (s->compress_start < 0) return fail(nullptr, GLR_EINVAL, "need compress_start >= 0%s");
@@ -607,13 +621,13 @@ int glr_create(int64_t m, int64_t n, int32_t r, int32_t N, const glr_schedule* s
     A(&h->lam, MP);
     A(&h->lam_part, MP * std::max(h->ntiles, h->nstrips));
     A(&h->Mo, (size_t)m * n);
-    if (s->optimizer == GLR_ADAM || s->optimizer == GLR_AMSGRAD) A(&h->Vo, (size_t)m * n);
+    if (s->optimizer != GLR_MSGD) A(&h->Vo, (size_t)m * n);
     if (s->optimizer == GLR_AMSGRAD) A(&h->amsv, 2);
     A(&h->dflags, 4);
     A(&h->gemm_ws, (size_t)kGemmWsFloats);
     // the first path with library products when the rank-r products are large
     h->tc = !h->fused && mp % 4 == 0 && np % 4 == 0 && 2.0 * r * (double)mp * (double)np * N >= 67108864.0 ? 1 : 0;
-    if (h->tc || s->optimizer == GLR_AMSGRAD) A(&h->mn_scratch, MP * NP);
+    if (h->tc || s->optimizer == GLR_AMSGRAD || s->optimizer == GLR_ADAMW) A(&h->mn_scratch, MP * NP);
     if (h->tc && !exact) A(&h->YtJ, (size_t)r * k);
     if (exact) {
         A(&h->jwork, MP * MP);
@@ -735,7 +749,7 @@ void plan_step(StepPlan& p) {
     p.forced = !p.warm && !p.refresh && h->has_forceJ;
     p.fixed = !p.warm && !p.refresh && !p.forced && h->s.selection == GLR_SEL_FIXED;
     p.lam_fused = h->fused && !h->exact && !p.warm && !p.refresh && !p.forced && !p.fixed;
-    p.stream_update = p.lam_fused && h->mma && h->s.optimizer != GLR_AMSGRAD &&
+    p.stream_update = p.lam_fused && h->mma && !separate_optimizer(h) &&
                       update_stream_eligible(h->mp, h->r, h->transposed);
     p.compressed = !p.warm && !(p.refresh && h->s.refresh_mode == GLR_ALG3);
     h->forced_this_step = p.forced;
@@ -1055,15 +1069,15 @@ int step_group(std::vector<StepPlan>& plans, cudaStream_t st) {
     if ((rc = select_P_grouped(plans, st)) != GLR_OK) return rc;
     std::vector<StepPlan*> streamed, strips;
     for (StepPlan* p : fused) {
-        if (p->h->s.optimizer == GLR_AMSGRAD) continue;
+        if (separate_optimizer(p->h)) continue;
         (p->stream_update ? streamed : strips).push_back(p);
     }
     if (!streamed.empty() && (rc = update_streamed(streamed, st)) != GLR_OK) return rc;
     if (!strips.empty() && (rc = update_fused(strips, st)) != GLR_OK) return rc;
     for (StepPlan* p : unfused)
-        if (p->h->s.optimizer != GLR_AMSGRAD && (rc = update_unfused(*p, st)) != GLR_OK) return rc;
+        if (!separate_optimizer(p->h) && (rc = update_unfused(*p, st)) != GLR_OK) return rc;
     for (StepPlan& p : plans)
-        if (p.h->s.optimizer == GLR_AMSGRAD && (rc = amsgrad_step_update(p.h, p.X, p.compressed, st)) != GLR_OK)
+        if (separate_optimizer(p.h) && (rc = separate_optimizer_update(p.h, p.X, p.compressed, st)) != GLR_OK)
             return rc;
     for (StepPlan& p : plans) finish_step(p);
     return GLR_OK;

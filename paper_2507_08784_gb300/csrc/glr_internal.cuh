@@ -189,6 +189,9 @@ cudaError_t update_streamed_flat(const UpdateArgs& a, cudaStream_t st);
 // vt[0] is the running scalar normaliser, vt[1] scratch for this step's maximum of V.
 cudaError_t amsgrad_update(const float* Ghat, int mp, int np, int transposed, float* X, float* Mo, float* Vo,
                            float* vt, float lr, float beta1, float beta2, float eps, cudaStream_t st);
+// Bias-corrected AdamW step (k_big.cu), same layouts; c1, c2 the bias corrections of this step.
+cudaError_t adamw_update(const float* Ghat, int mp, int np, int transposed, float* X, float* Mo, float* Vo, float lr,
+                         float beta1, float beta2, float eps, float wd, float c1, float c2, cudaStream_t st);
 
 // E_i = B_i - Pprev (Pprev^T B_i) given Rw_i = Pprev^T B_i  (or 0 when e_zero)
 cudaError_t materialize_error(int mp, int np, int r, int e_zero, const float* B, const float* Pprev,

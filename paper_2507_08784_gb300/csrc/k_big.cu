@@ -174,6 +174,27 @@ __global__ void __launch_bounds__(TB) amsgrad_apply_kernel(float* X, const float
         X[e] -= scale * Mo[e];
 }
 
+// Bias-corrected AdamW with decoupled weight decay (Loshchilov & Hutter): M, V as Eq. adam, then
+// X -= lr (c1 M / (sqrt(c2 V) + eps) + wd X) with c1 = 1 / (1 - b1^s), c2 = 1 / (1 - b2^s) for
+// optimizer step s (computed by the caller).  Ghat oriented, X / M / V in X's layout.
+__global__ void __launch_bounds__(TB) adamw_kernel(const float* Gh, int mp, int np, int transposed, float* X,
+                                                   float* Mo, float* Vo, float lr, float b1, float b2, float eps,
+                                                   float wd, float c1, float c2) {
+    const int64_t total = (int64_t)mp * np;
+    const int xcols = transposed ? mp : np;
+    for (int64_t e = (int64_t)blockIdx.x * TB + threadIdx.x; e < total; e += (int64_t)gridDim.x * TB) {
+        const int xr = static_cast<int>(e / xcols), xc = static_cast<int>(e % xcols);
+        const int a = transposed ? xc : xr, b = transposed ? xr : xc;
+        const float g = Gh[(int64_t)a * np + b];
+        const float m = fmaf(b1, Mo[e], (1.0f - b1) * g);
+        const float v = fmaf(b2, Vo[e], (1.0f - b2) * g * g);
+        Mo[e] = m;
+        Vo[e] = v;
+        const float x = X[e];
+        X[e] = x - lr * (c1 * m / (sqrtf(c2 * v) + eps) + wd * x);
+    }
+}
+
 int stream_grid(int64_t quads) {
     static int sms = 0;
     if (!sms) {
@@ -210,6 +231,14 @@ cudaError_t amsgrad_update(const float* Ghat, int mp, int np, int transposed, fl
     amsgrad_scalar_kernel<<<1, 1, 0, st>>>(vt, bits);
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
     amsgrad_apply_kernel<<<grid, TB, 0, st>>>(X, Mo, vt, total, lr, eps);
+    return cudaGetLastError();
+}
+
+cudaError_t adamw_update(const float* Ghat, int mp, int np, int transposed, float* X, float* Mo, float* Vo, float lr,
+                         float beta1, float beta2, float eps, float wd, float c1, float c2, cudaStream_t st) {
+    const int64_t total = (int64_t)mp * np;
+    adamw_kernel<<<stream_grid((total + 3) / 4), TB, 0, st>>>(Ghat, mp, np, transposed, X, Mo, Vo, lr, beta1, beta2,
+                                                              eps, wd, c1, c2);
     return cudaGetLastError();
 }
 

@@ -101,6 +101,16 @@ def test_amsgrad_lockstep(m, n, k):
     _assert_reports(reps, tol=1e-4)
 
 
+@pytest.mark.parametrize("m,n,k", [(96, 400, 16), (300, 130, 0), (640, 1280, 16)])
+def test_adamw_lockstep(m, n, k):
+    """Bias-corrected AdamW with weight decay on the tensor-core, transposed paper-exact and
+    FFMA-strip paths."""
+    g = _synthetic(m, n, 3, 24, lambda j: 1.0 / j, 0.05, 95 + m + k)
+    reps = lockstep(m, n, 5, 3, 6, g, tau=3, optimizer="adamw", lr=1e-3, beta1=0.9, beta2=0.999, eps=1e-8,
+                    weight_decay=0.01, seed=13, basis_rank=k)
+    _assert_reports(reps, tol=1e-4)
+
+
 @pytest.mark.parametrize("m,n,k,selection", [(96, 400, 16, "fixed"), (96, 400, 0, "fixed"), (640, 1280, 16, "approx"),
                                               (300, 130, 24, "fixed"), (200, 824, 24, "approx")])
 def test_without_error_feedback_lockstep(m, n, k, selection):

@@ -480,3 +480,20 @@ def test_amsgrad_closed_form_and_monotone_normaliser():
         np.testing.assert_allclose(M, (1 - b1) * b1 ** k * G, rtol=1e-13)
         np.testing.assert_allclose(X2 - X, -lr * M / np.sqrt(vt1 + eps), rtol=1e-12)
         X = X2
+
+
+def test_adamw_first_step_and_bias_correction():
+    """Bias-corrected AdamW: the first step has Mh = G and Vh = G^2, so from X0 it moves by
+    -lr (G / (|G| + eps) + wd X0); with a constant gradient the corrected moments stay G, G^2."""
+    rng = np.random.default_rng(24)
+    G = rng.standard_normal((4, 6))
+    X0 = rng.standard_normal((4, 6))
+    lr, b1, b2, eps, wd = 0.01, 0.9, 0.999, 1e-8, 0.1
+    X, M, V = O.adamw_update(X0, np.zeros_like(G), np.zeros_like(G), 1, G, lr, b1, b2, eps, wd)
+    np.testing.assert_allclose(X, X0 - lr * (G / (np.abs(G) + eps) + wd * X0), rtol=1e-12)
+    for s in range(2, 6):
+        X2, M, V = O.adamw_update(X, M, V, s, G, lr, b1, b2, eps, wd)
+        np.testing.assert_allclose(M / (1 - b1 ** s), G, rtol=1e-12)
+        np.testing.assert_allclose(V / (1 - b2 ** s), G * G, rtol=1e-12)
+        np.testing.assert_allclose(X2, X - lr * (G / (np.abs(G) + eps) + wd * X), rtol=1e-12)
+        X = X2
