@@ -73,6 +73,17 @@ __device__ __forceinline__ float4 gauss4_fast(uint64_t seed, uint32_t t, uint32_
 
 constexpr int kGroupMax = 32;          // matrices per grouped launch
 
+// Streaming (evict-first) global stores of the error buffers.  Unlike the library's cache-hint
+// store intrinsics these carry no memory clobber, which would make each store a compiler barrier
+// and stop the shared-memory loads of the next rows from being scheduled across it; the kernels
+// that use them never read the stored addresses back.
+__device__ __forceinline__ void st_stream2(float* p, float a, float b) {
+    asm("st.global.cs.v2.f32 [%0], {%1, %2};" ::"l"(p), "f"(a), "f"(b));
+}
+__device__ __forceinline__ void st_stream4(float* p, float a, float b, float c, float d) {
+    asm("st.global.cs.v4.f32 [%0], {%1, %2, %3, %4};" ::"l"(p), "f"(a), "f"(b), "f"(c), "f"(d));
+}
+
 // ------------------------------------------------------------------------------------------
 // Gradient element loads (fp32 or bf16, widened to fp32).
 // ------------------------------------------------------------------------------------------

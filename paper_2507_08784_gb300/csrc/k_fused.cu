@@ -259,7 +259,7 @@ __global__ void __launch_bounds__(NT, 1) stream_kernel(const __grid_constant__ S
                     m[2] += bv.z - c[ii][2]; m[3] += bv.w - c[ii][3];
                 }
                 if (M.write_B)
-                    __stcs(reinterpret_cast<float4*>(Bi + (int64_t)a * np + bcol), make_float4(m[0], m[1], m[2], m[3]));
+                    st_stream4(Bi + (int64_t)a * np + bcol, m[0], m[1], m[2], m[3]);
 #pragma unroll
                 for (int j = 0; j < 4; ++j) acc[ii][j] += m[j];
                 }

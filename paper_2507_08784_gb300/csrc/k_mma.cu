@@ -335,8 +335,8 @@ __device__ __forceinline__ void compose_node(const float* S, const GT* Gs, bool 
             const float m3 = g1.y + (x1.y - c[3]);
             if (write_B && colok) {
                 float* const Ba = Brow + j * jstep;
-                if (ra < mp) __stcs(reinterpret_cast<float2*>(Ba), make_float2(m0, m1));
-                if (rb < mp) __stcs(reinterpret_cast<float2*>(Ba + 2 * (int64_t)np), make_float2(m2, m3));
+                if (ra < mp) st_stream2(Ba, m0, m1);
+                if (rb < mp) st_stream2(Ba + 2 * (int64_t)np, m2, m3);
             }
             acc[j][0] += m0; acc[j][1] += m1; acc[j][2] += m2; acc[j][3] += m3;
         }
