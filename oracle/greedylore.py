@@ -18,6 +18,9 @@ with Convergence Guarantees" (arXiv 2507.08784):
 * the optimizers of Eq. msgd and Eq. adam (no bias correction, eps outside the
   square root), the AMSGrad-type Adam of the convergence analysis (Appendix A), and
   bias-corrected AdamW;
+* the distributed Adam-type GaLore of Algorithm 5 (Appendix E): Adam state on the
+  r x n' projected mean, reset at every refresh, with the Lazy-SVD projector and no
+  error feedback;
 * the truncated-basis reading: the top-k singular vectors of the refresh
   matrix completed to a full orthogonal U by Householder QR (the proofs of
   Prop. 3 and Lemma 2 only use that U is orthogonal).
@@ -240,6 +243,8 @@ class GreedyLoreOracle:
     completes them with the Householder complement.  selection "approx" is
     Algorithm 2; "exact" is Eq. semi-lazy-svd-2.  compress_start K runs the first K
     steps uncompressed (plain mean, no error feedback; Appendix F warm-up).
+    optimizer "galore_adam" is Algorithm 5: it needs refresh_mode "alg4" (the refresh step is
+    compressed with the new P), selection "fixed", error_feedback False and compress_start 0.
     """
 
     def __init__(self, m, n, r, N, tau, *, refresh_mode="alg3", optimizer="msgd", lr=0.01,
@@ -263,6 +268,12 @@ class GreedyLoreOracle:
         self.Mo = np.zeros((m, n))
         self.Vo = np.zeros((m, n))
         self.Vt = 0.0                                # AMSGrad-type scalar normaliser
+        if optimizer == "galore_adam":
+            if refresh_mode != "alg4" or selection != "fixed" or error_feedback or compress_start != 0:
+                raise ValueError("Algorithm 5 needs refresh_mode 'alg4', selection 'fixed', "
+                                 "error_feedback False and compress_start 0")
+        self.Ms = np.zeros((r, self.np_))            # Algorithm 5: subspace Adam state, r x n'
+        self.Vs = np.zeros((r, self.np_))
         self.t = 0
 
     # -- helpers ---------------------------------------------------------------
@@ -289,6 +300,18 @@ class GreedyLoreOracle:
         else:
             X, self.Mo, self.Vo = adam_update(X, self.Mo, self.Vo, G, self.lr, self.beta1, self.beta2, self.eps)
         return X
+
+    def galore_adam(self, X, P, Rbar, refresh):
+        """Algorithm 5's Adam-Update on the projected mean Rbar (r x n'): the state is zeroed at a
+        refresh, M and V are the EMAs of Eq. adam (beta weighting the old state), and X moves by
+        lr P (M / (sqrt(V) + eps)), transposed back when m > n; lr is applied once."""
+        if refresh:
+            self.Ms = np.zeros_like(Rbar)
+            self.Vs = np.zeros_like(Rbar)
+        self.Ms = self.beta1 * self.Ms + (1.0 - self.beta1) * Rbar
+        self.Vs = self.beta2 * self.Vs + (1.0 - self.beta2) * Rbar * Rbar
+        Rhat = self.Ms / (np.sqrt(self.Vs) + self.eps)
+        return X - self.lr * self.orient(P @ Rhat)
 
     # -- one iteration -----------------------------------------------------------
     def step(self, G_nodes: np.ndarray, X: np.ndarray, force_J: Optional[Sequence[int]] = None):
@@ -334,7 +357,10 @@ class GreedyLoreOracle:
             self.E = np.zeros_like(self.E)
         Rbar = R.mean(axis=0)                        # All-Reduce
         Ghat = P @ Rbar
-        X = self.apply_optimizer(X, Ghat)
+        if self.optimizer == "galore_adam":
+            X = self.galore_adam(X, P, Rbar, refresh)
+        else:
+            X = self.apply_optimizer(X, Ghat)
         self.t += 1
         sent = P @ R
         return X, StepInfo(t, refresh, True, J, P, lam_bar, Rbar, Mbar, Ghat, self.E.copy(), sent)

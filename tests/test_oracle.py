@@ -497,3 +497,67 @@ def test_adamw_first_step_and_bias_correction():
         np.testing.assert_allclose(V / (1 - b2 ** s), G * G, rtol=1e-12)
         np.testing.assert_allclose(X2, X - lr * (G / (np.abs(G) + eps) + wd * X), rtol=1e-12)
         X = X2
+
+
+@pytest.mark.parametrize("transposed", [False, True])
+def test_algorithm5_is_adam_on_the_selected_coordinates(transposed):
+    """Algorithm 5 when the refresh means have orthogonal rows: Mbar = diag(s) W (W with orthonormal
+    rows) has U = I up to the order of s, so P holds coordinate vectors e_j, Rbar is those rows of
+    the node mean, and the subspace Adam is Eq. adam on those rows alone, started afresh at every
+    refresh; every other row of X stays put.  The second period's P shares row 1 with the first,
+    so a state carried over the refresh would show."""
+    mp, npr, r, N, tau, lr, b1, b2, eps = 6, 10, 2, 2, 3, 0.01, 0.9, 0.999, 1e-8
+    rng = np.random.default_rng(31)
+    W = np.linalg.qr(rng.standard_normal((npr, npr)))[0][:mp]
+    scale = {0: np.array([5.0, 4.0, 3.0, 2.0, 1.5, 1.0]), 3: np.array([1.0, 5.0, 2.0, 4.0, 1.5, 3.0])}
+    rows = {0: [0, 1], 3: [1, 3]}
+    m, n = (npr, mp) if transposed else (mp, npr)
+    orc = O.GreedyLoreOracle(m, n, r, N, tau, refresh_mode="alg4", optimizer="galore_adam", lr=lr, beta1=b1,
+                             beta2=b2, eps=eps, selection="fixed", error_feedback=False)
+    X0 = rng.standard_normal((mp, npr))
+    X = X0.T.copy() if transposed else X0.copy()
+    Xe = X0.copy()                                   # expected, oriented
+    for t in range(5):
+        if t in scale:
+            Gbar = scale[t][:, None] * W
+            D = rng.standard_normal((mp, npr))
+            G = np.stack([Gbar + D, Gbar - D])
+            sel, Ms, Vs = rows[t], np.zeros((r, npr)), np.zeros((r, npr))
+        else:
+            G = rng.standard_normal((N, mp, npr))
+        Xe[sel], Ms, Vs = O.adam_update(Xe[sel], Ms, Vs, G.mean(axis=0)[sel], lr, b1, b2, eps)
+        X, info = orc.step(np.swapaxes(G, 1, 2) if transposed else G, X)
+        assert info.compressed and info.refresh == (t % tau == 0)
+        assert sorted(np.argmax(np.abs(info.P), axis=0).tolist()) == rows[3 if t >= 3 else 0]
+        np.testing.assert_allclose(X.T if transposed else X, Xe, rtol=0, atol=1e-12)
+        assert np.all(info.E == 0)
+
+
+def test_algorithm5_closed_form_constant_gradient():
+    """A constant gradient in every step and node: P and R = P^T G stay fixed within the period,
+    so M_t = (1 - b1^(t+1)) R and V_t = (1 - b2^(t+1)) R^2 and after T steps
+    X_T = X_0 - lr P sum_t (1 - b1^(t+1)) R / (sqrt(1 - b2^(t+1)) |R| + eps); the weighting of
+    Eq. adam (beta on the old state) is what this checks."""
+    m, n, r, N, T, lr, b1, b2, eps = 7, 5, 2, 3, 6, 0.02, 0.8, 0.95, 1e-3
+    rng = np.random.default_rng(32)
+    G = rng.standard_normal((m, n))
+    orc = O.GreedyLoreOracle(m, n, r, N, 100, refresh_mode="alg4", optimizer="galore_adam", lr=lr, beta1=b1,
+                             beta2=b2, eps=eps, selection="fixed", error_feedback=False)
+    X0 = rng.standard_normal((m, n))
+    X = X0.copy()
+    for _ in range(T):
+        X, info = orc.step(np.stack([G] * N), X)
+    Uo, _, _ = np.linalg.svd(G.T)                    # m > n: the basis lives on the n side
+    P = info.P
+    assert abs(abs(np.linalg.det(P.T @ Uo[:, :r])) - 1.0) < 1e-10   # span of the top-r singular vectors
+    R = P.T @ G.T
+    step = sum((1 - b1 ** (t + 1)) * R / (np.sqrt(1 - b2 ** (t + 1)) * np.abs(R) + eps) for t in range(T))
+    np.testing.assert_allclose(X, X0 - lr * (P @ step).T, rtol=1e-12, atol=1e-14)
+
+
+def test_algorithm5_rejects_other_schedules():
+    for kw in ({"refresh_mode": "alg3"}, {"selection": "approx"}, {"error_feedback": True}, {"compress_start": 2}):
+        args = dict(refresh_mode="alg4", selection="fixed", error_feedback=False, compress_start=0)
+        args.update(kw)
+        with pytest.raises(ValueError):
+            O.GreedyLoreOracle(6, 8, 2, 2, 3, optimizer="galore_adam", **args)
