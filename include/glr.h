@@ -63,6 +63,11 @@ extern "C" {
 #define GLR_ADAMW 3     /* bias-corrected AdamW: M, V EMAs, X -= lr (Mh / (sqrt(Vh) + eps) +   *
                          * weight_decay X), Mh = M / (1 - b1^s), Vh = V / (1 - b2^s), s = the  *
                          * optimizer step (1, 2, ...: every step, refresh and warm-up included)*/
+#define GLR_GALORE_ADAM 4  /* Algorithm 5 (distributed Adam-type GaLore, App. E): Adam state on *
+                            * the projected mean, M, V r x n' (EMAs as GLR_ADAM of Rbar), zeroed *
+                            * at every refresh; X -= lr P (M / (sqrt(V) + eps)), transposed back *
+                            * when m > n.  Needs refresh_mode GLR_ALG4, selection GLR_SEL_FIXED, *
+                            * no_error_feedback 1 and compress_start 0                          */
 
 #define GLR_SEL_APPROX 0   /* Algorithm 2 (Approx-Top-r) picks J at every compressed step    */
 #define GLR_SEL_FIXED  1   /* P = U[:, :r] for the whole refresh period: the Lazy-SVD of       *
@@ -76,7 +81,8 @@ extern "C" {
 /* Compressor and optimizer settings (Algorithm 3 inputs: tau, r; Sec. 2 optimizers).
  *   tau            refresh period (>= 1)
  *   refresh_mode   GLR_ALG3 | GLR_ALG4
- *   optimizer      GLR_MSGD | GLR_ADAM | GLR_AMSGRAD | GLR_ADAMW; lr = gamma; beta1 = beta
+ *   optimizer      GLR_MSGD | GLR_ADAM | GLR_AMSGRAD | GLR_ADAMW | GLR_GALORE_ADAM; lr = gamma;
+ *                  beta1 = beta
  *                  (MSGD) or beta_1 (Adam types); beta2, eps used by the Adam types only
  *   seed           64-bit key of the shared random vectors v_j (Eq. random-v): all nodes
  *                  of one matrix draw the same v_j; give every matrix its own seed
@@ -149,8 +155,9 @@ typedef struct glr_profile {
  * Algorithm 3 inputs).  Requires m, n >= 1, 1 <= r <= min(m, n), 1 <= N <= GLR_MAX_NODES,
  * tau >= 1 and a valid schedule (see glr_schedule).  Allocates all state on the current
  * CUDA device: E_i (N x m' x n' fp32), the basis, optimizer moments (m x n fp32, two for
- * Adam) and workspace.  E starts at 0 and U at I (Algorithm 3 input); t = 0.  On
- * success *out receives the handle.  Errors: GLR_EINVAL, GLR_ENOMEM, GLR_ECUDA.         */
+ * the Adam types; r x n' for GLR_GALORE_ADAM) and workspace.  E starts at 0 and U at I
+ * (Algorithm 3 input); t = 0.  On success *out receives the handle.
+ * Errors: GLR_EINVAL, GLR_ENOMEM, GLR_ECUDA.                                             */
 int glr_create(int64_t m, int64_t n, int32_t r, int32_t N, const glr_schedule* schedule,
                glr_handle** out);
 

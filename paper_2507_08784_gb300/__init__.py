@@ -15,8 +15,8 @@ import numpy as np
 import torch
 
 from . import _lib
-from ._lib import (GLR_ADAM, GLR_ALG3, GLR_ALG4, GLR_BF16, GLR_F32, GLR_MSGD, GLR_OK,  # noqa: F401
-                   PHASE_NAMES, GlrProfile, GlrSchedule, GlrStats, load)
+from ._lib import (GLR_ADAM, GLR_ADAMW, GLR_ALG3, GLR_ALG4, GLR_AMSGRAD, GLR_BF16, GLR_F32,  # noqa: F401
+                   GLR_GALORE_ADAM, GLR_MSGD, GLR_OK, PHASE_NAMES, GlrProfile, GlrSchedule, GlrStats, load)
 
 __all__ = ["GlrError", "make_schedule", "glr_create", "glr_destroy", "glr_step", "glr_step_group", "glr_step_group_host", "glr_step_host", "glr_save", "glr_load",
            "glr_refresh", "glr_get_stats", "glr_last_error", "glr_get_error", "glr_get_selection",
@@ -47,13 +47,19 @@ def _stream_ptr(stream) -> int:
     return int(stream.cuda_stream) if hasattr(stream, "cuda_stream") else int(stream)
 
 
+# "galore_adam" is Algorithm 5; it needs refresh_mode "alg4", selection "fixed" and
+# error_feedback False (glr_create rejects other combinations)
+_OPTIMIZERS = {"msgd": GLR_MSGD, "adam": GLR_ADAM, "amsgrad": GLR_AMSGRAD, "adamw": GLR_ADAMW,
+               "galore_adam": GLR_GALORE_ADAM}
+
+
 def make_schedule(tau: int, refresh_mode: str = "alg3", optimizer: str = "msgd", lr: float = 0.01,
                   beta1: float = 0.9, beta2: float = 0.999, eps: float = 1e-8, seed: int = 0,
                   basis_rank: int = 0, power_iters: int = 4, grad_dtype: str = "f32",
                   compress_start: int = 0, error_feedback: bool = True, selection: str = "approx",
                   weight_decay: float = 0.0) -> GlrSchedule:
     return GlrSchedule(tau=tau, refresh_mode={"alg3": GLR_ALG3, "alg4": GLR_ALG4}[refresh_mode],
-                       optimizer={"msgd": GLR_MSGD, "adam": GLR_ADAM, "amsgrad": 2, "adamw": 3}[optimizer], lr=lr, beta1=beta1,
+                       optimizer=_OPTIMIZERS[optimizer], lr=lr, beta1=beta1,
                        beta2=beta2, eps=eps, seed=seed & (2 ** 64 - 1), basis_rank=basis_rank,
                        power_iters=power_iters, grad_dtype={"f32": GLR_F32, "bf16": GLR_BF16}[grad_dtype],
                        compress_start=compress_start, no_error_feedback=0 if error_feedback else 1,

@@ -15,7 +15,7 @@ HEADER = os.path.join(os.path.dirname(PKG), "include", "glr.h")
 
 GLR_OK, GLR_EINVAL, GLR_ENOMEM, GLR_ECUDA, GLR_ENUMERIC, GLR_ENONFINITE, GLR_ETIMEOUT = 0, -1, -2, -3, -4, -5, -6
 GLR_ALG3, GLR_ALG4 = 0, 1
-GLR_MSGD, GLR_ADAM = 0, 1
+GLR_MSGD, GLR_ADAM, GLR_AMSGRAD, GLR_ADAMW, GLR_GALORE_ADAM = 0, 1, 2, 3, 4
 GLR_F32, GLR_BF16 = 0, 1
 GLR_MAX_NODES = 64
 

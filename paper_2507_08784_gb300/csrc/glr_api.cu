@@ -59,6 +59,7 @@ struct glr_handle {
     float* jpart = nullptr;      // full basis: its per-CTA norm partials (used by a group's first handle)
     float* YtJ = nullptr;        // Yt[J, :] (r x k) for P = U[:, J] as a library product
     float* amsv = nullptr;       // AMSGrad: the scalar normaliser and this step's maximum of V
+    float* galr = nullptr;       // Algorithm 5: the subspace step direction M / (sqrt(V) + eps), r x n'
     cudaStream_t rstream = nullptr;            // side stream of this handle's refresh
     cudaEvent_t rfork = nullptr, rdone = nullptr, rpow = nullptr;
     int pow_ok = 0;                            // refresh through the grouped power iteration (k_power.cu)
@@ -511,11 +512,33 @@ int uncompressed_update(glr_handle* h, float* X, cudaStream_t st) {
 // bias-corrected AdamW — with Ghat = Mbar (uncompressed) or P Rbar, both products formed here
 // (Rbar = P^T Mbar): one path for every kernel family.
 bool separate_optimizer(const glr_handle* h) {
-    return h->s.optimizer == GLR_AMSGRAD || h->s.optimizer == GLR_ADAMW;
+    return h->s.optimizer == GLR_AMSGRAD || h->s.optimizer == GLR_ADAMW || h->s.optimizer == GLR_GALORE_ADAM;
 }
 
-int separate_optimizer_update(glr_handle* h, float* X, bool compressed, cudaStream_t st) {
+// Algorithm 5 (every step compressed with the Lazy-SVD P): the subspace state is zeroed at a
+// refresh, advanced with Rbar = P^T Mbar, and X moves by lr P (M / (sqrt(V) + eps)).
+int galore_update(glr_handle* h, float* X, bool refresh, cudaStream_t st) {
     const int mp = h->mp, np = h->np, r = h->r;
+    const size_t rn = (size_t)r * np;
+    {
+        PhaseScope ps(h, GLR_PH_PROJECT, st);
+        GLR_GEMM(h, gd(r, np, mp, h->P, 1, r, h->Mbar, np, 1, h->Rbar, np, 1), st);
+    }
+    PhaseScope ps(h, GLR_PH_UPDATE, st);
+    if (refresh) {
+        GLR_CK(h, cudaMemsetAsync(h->Mo, 0, rn * 4, st));
+        GLR_CK(h, cudaMemsetAsync(h->Vo, 0, rn * 4, st));
+    }
+    GLR_LAUNCH(h, 1, galore_moments(h->Rbar, (int64_t)rn, h->Mo, h->Vo, h->galr, h->s.beta1, h->s.beta2, h->s.eps,
+                                    st));
+    GLR_GEMM(h, gd(mp, np, r, h->P, r, 1, h->galr, np, 1, h->mn_scratch, np, 1), st);
+    GLR_LAUNCH(h, 1, step_apply(h->mn_scratch, mp, np, h->transposed, X, h->s.lr, st));
+    return GLR_OK;
+}
+
+int separate_optimizer_update(glr_handle* h, float* X, bool compressed, bool refresh, cudaStream_t st) {
+    const int mp = h->mp, np = h->np, r = h->r;
+    if (h->s.optimizer == GLR_GALORE_ADAM) return galore_update(h, X, refresh, st);
     const float* Gh = h->Mbar;
     if (compressed) {
         PhaseScope ps(h, GLR_PH_PROJECT, st);
@@ -565,8 +588,14 @@ int glr_create(int64_t m, int64_t n, int32_t r, int32_t N, const glr_schedule* s
         return fail(nullptr, GLR_EINVAL, "selection must be GLR_SEL_APPROX or GLR_SEL_FIXED%s");
     if (s->refresh_mode != GLR_ALG3 && s->refresh_mode != GLR_ALG4)
         return fail(nullptr, GLR_EINVAL, "unknown refresh_mode%s");
-    if (s->optimizer != GLR_MSGD && s->optimizer != GLR_ADAM && s->optimizer != GLR_AMSGRAD && s->optimizer != GLR_ADAMW)
+    if (s->optimizer != GLR_MSGD && s->optimizer != GLR_ADAM && s->optimizer != GLR_AMSGRAD && s->optimizer != GLR_ADAMW &&
+        s->optimizer != GLR_GALORE_ADAM)
         return fail(nullptr, GLR_EINVAL, "unknown optimizer%s");
+    if (s->optimizer == GLR_GALORE_ADAM && (s->refresh_mode != GLR_ALG4 || s->selection != GLR_SEL_FIXED ||
+                                            !s->no_error_feedback || s->compress_start != 0))
+        return fail(nullptr, GLR_EINVAL,
+                    "GLR_GALORE_ADAM (Algorithm 5) needs refresh_mode GLR_ALG4, selection GLR_SEL_FIXED, "
+                    "no_error_feedback 1 and compress_start 0%s");
     if (s->grad_dtype != GLR_F32 && s->grad_dtype != GLR_BF16) return fail(nullptr, GLR_EINVAL, "unknown grad_dtype%s");
     if (s->compress_start < 0) return fail(nullptr, GLR_EINVAL, "need compress_start >= 0%s");
     const int k = (s->basis_rank == 0 || s->basis_rank == mp) ? static_cast<int>(mp) : s->basis_rank;
@@ -620,14 +649,16 @@ int glr_create(int64_t m, int64_t n, int32_t r, int32_t N, const glr_schedule* s
     A(&h->J, (size_t)r);
     A(&h->lam, MP);
     A(&h->lam_part, MP * std::max(h->ntiles, h->nstrips));
-    A(&h->Mo, (size_t)m * n);
-    if (s->optimizer != GLR_MSGD) A(&h->Vo, (size_t)m * n);
+    const bool galore = s->optimizer == GLR_GALORE_ADAM;
+    A(&h->Mo, galore ? (size_t)r * NP : (size_t)m * n);
+    if (s->optimizer != GLR_MSGD) A(&h->Vo, galore ? (size_t)r * NP : (size_t)m * n);
     if (s->optimizer == GLR_AMSGRAD) A(&h->amsv, 2);
+    if (galore) A(&h->galr, (size_t)r * NP);
     A(&h->dflags, 4);
     A(&h->gemm_ws, (size_t)kGemmWsFloats);
     // the first path with library products when the rank-r products are large
     h->tc = !h->fused && mp % 4 == 0 && np % 4 == 0 && 2.0 * r * (double)mp * (double)np * N >= 67108864.0 ? 1 : 0;
-    if (h->tc || s->optimizer == GLR_AMSGRAD || s->optimizer == GLR_ADAMW) A(&h->mn_scratch, MP * NP);
+    if (h->tc || separate_optimizer(h)) A(&h->mn_scratch, MP * NP);
     if (h->tc && !exact) A(&h->YtJ, (size_t)r * k);
     if (exact) {
         A(&h->jwork, MP * MP);
@@ -1077,7 +1108,7 @@ int step_group(std::vector<StepPlan>& plans, cudaStream_t st) {
     for (StepPlan* p : unfused)
         if (!separate_optimizer(p->h) && (rc = update_unfused(*p, st)) != GLR_OK) return rc;
     for (StepPlan& p : plans)
-        if (separate_optimizer(p.h) && (rc = separate_optimizer_update(p.h, p.X, p.compressed, st)) != GLR_OK)
+        if (separate_optimizer(p.h) && (rc = separate_optimizer_update(p.h, p.X, p.compressed, p.refresh, st)) != GLR_OK)
             return rc;
     for (StepPlan& p : plans) finish_step(p);
     return GLR_OK;

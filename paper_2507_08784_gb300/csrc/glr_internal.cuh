@@ -203,6 +203,11 @@ cudaError_t amsgrad_update(const float* Ghat, int mp, int np, int transposed, fl
 // Bias-corrected AdamW step (k_big.cu), same layouts; c1, c2 the bias corrections of this step.
 cudaError_t adamw_update(const float* Ghat, int mp, int np, int transposed, float* X, float* Mo, float* Vo, float lr,
                          float beta1, float beta2, float eps, float wd, float c1, float c2, cudaStream_t st);
+// Algorithm 5's subspace Adam (k_big.cu): Ms, Vs the EMAs of Rbar (total = r n' elements), Rh the
+// step direction Ms / (sqrt(Vs) + eps); step_apply: X -= lr D, D oriented m' x n', X in its layout.
+cudaError_t galore_moments(const float* Rbar, int64_t total, float* Ms, float* Vs, float* Rh, float beta1, float beta2,
+                           float eps, cudaStream_t st);
+cudaError_t step_apply(const float* D, int mp, int np, int transposed, float* X, float lr, cudaStream_t st);
 
 // E_i = B_i - Pprev (Pprev^T B_i) given Rw_i = Pprev^T B_i  (or 0 when e_zero)
 cudaError_t materialize_error(int mp, int np, int r, int e_zero, const float* B, const float* Pprev,

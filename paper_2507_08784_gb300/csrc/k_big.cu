@@ -195,6 +195,31 @@ __global__ void __launch_bounds__(TB) adamw_kernel(const float* Gh, int mp, int 
     }
 }
 
+// Algorithm 5's Adam-Update on the projected mean (r x n', any layout, e elements): M, V the EMAs
+// of Eq. adam of Rbar, and Rh = M / (sqrt(V) + eps), the step direction in the subspace.
+__global__ void __launch_bounds__(TB) galore_moments_kernel(const float* Rbar, int64_t total, float* Ms, float* Vs,
+                                                            float* Rh, float b1, float b2, float eps) {
+    for (int64_t e = (int64_t)blockIdx.x * TB + threadIdx.x; e < total; e += (int64_t)gridDim.x * TB) {
+        const float g = Rbar[e];
+        const float m = fmaf(b1, Ms[e], (1.0f - b1) * g);
+        const float v = fmaf(b2, Vs[e], (1.0f - b2) * g * g);
+        Ms[e] = m;
+        Vs[e] = v;
+        Rh[e] = m / (sqrtf(v) + eps);
+    }
+}
+// X -= lr D with D oriented (m' x n'); X in its own layout (transposed when m > n).
+__global__ void __launch_bounds__(TB) step_apply_kernel(const float* D, int mp, int np, int transposed, float* X,
+                                                        float lr) {
+    const int64_t total = (int64_t)mp * np;
+    const int xcols = transposed ? mp : np;
+    for (int64_t e = (int64_t)blockIdx.x * TB + threadIdx.x; e < total; e += (int64_t)gridDim.x * TB) {
+        const int xr = static_cast<int>(e / xcols), xc = static_cast<int>(e % xcols);
+        const int a = transposed ? xc : xr, b = transposed ? xr : xc;
+        X[e] -= lr * D[(int64_t)a * np + b];
+    }
+}
+
 int stream_grid(int64_t quads) {
     static int sms = 0;
     if (!sms) {
@@ -239,6 +264,17 @@ cudaError_t adamw_update(const float* Ghat, int mp, int np, int transposed, floa
     const int64_t total = (int64_t)mp * np;
     adamw_kernel<<<stream_grid((total + 3) / 4), TB, 0, st>>>(Ghat, mp, np, transposed, X, Mo, Vo, lr, beta1, beta2,
                                                               eps, wd, c1, c2);
+    return cudaGetLastError();
+}
+
+cudaError_t galore_moments(const float* Rbar, int64_t total, float* Ms, float* Vs, float* Rh, float beta1, float beta2,
+                           float eps, cudaStream_t st) {
+    galore_moments_kernel<<<stream_grid((total + 3) / 4), TB, 0, st>>>(Rbar, total, Ms, Vs, Rh, beta1, beta2, eps);
+    return cudaGetLastError();
+}
+
+cudaError_t step_apply(const float* D, int mp, int np, int transposed, float* X, float lr, cudaStream_t st) {
+    step_apply_kernel<<<stream_grid(((int64_t)mp * np + 3) / 4), TB, 0, st>>>(D, mp, np, transposed, X, lr);
     return cudaGetLastError();
 }
 

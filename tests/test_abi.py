@@ -68,6 +68,11 @@ def test_struct_layouts(tmp_path):
     (8, 20, 4, 1, {"basis_rank": 3}, "basis_rank"),
     (2000, 3000, 4, 1, {"basis_rank": 0}, "full basis"),
     (8, 20, 4, 1, {"power_iters": 0, "basis_rank": 5}, "power_iters"),
+    (8, 20, 4, 1, {"optimizer": "galore_adam", "selection": "fixed", "error_feedback": False}, "Algorithm 5"),
+    (8, 20, 4, 1, {"optimizer": "galore_adam", "refresh_mode": "alg4", "error_feedback": False}, "Algorithm 5"),
+    (8, 20, 4, 1, {"optimizer": "galore_adam", "refresh_mode": "alg4", "selection": "fixed"}, "Algorithm 5"),
+    (8, 20, 4, 1, {"optimizer": "galore_adam", "refresh_mode": "alg4", "selection": "fixed", "error_feedback": False,
+                   "compress_start": 1}, "Algorithm 5"),
 ])
 def test_create_rejects_bad_arguments(lib, m, n, r, N, kw, frag):
     import paper_2507_08784_gb300 as glr

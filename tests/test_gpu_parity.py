@@ -111,6 +111,19 @@ def test_adamw_lockstep(m, n, k):
     _assert_reports(reps, tol=1e-4)
 
 
+@pytest.mark.parametrize("m,n,k", [(64, 100, 0), (96, 400, 16), (300, 130, 24), (640, 1280, 16), (256, 2304, 16)])
+def test_galore_adam_lockstep(m, n, k):
+    """Algorithm 5 (Adam state on the projected mean, zeroed at each refresh; Lazy-SVD P; no error
+    feedback) on the paper-exact, tensor-core, transposed and FFMA-strip paths.  The spectra have
+    clear gaps so the device's own refresh basis matches the oracle's at the refresh step, where
+    Algorithm 5 already compresses with it."""
+    g = _synthetic(m, n, 2, 8, lambda j: 2.0 ** (-j), 0.01, 100 + m + k)
+    reps = lockstep(m, n, 3, 2, 7, g, tau=3, refresh_mode="alg4", optimizer="galore_adam", lr=1e-3, beta1=0.9,
+                    beta2=0.999, eps=1e-8, seed=14, basis_rank=k, selection="fixed", error_feedback=False)
+    _assert_reports(reps, tol=1e-4)
+    assert [r.refresh for r in reps] == [True, False, False, True, False, False, True]
+
+
 @pytest.mark.parametrize("m,n,k,selection", [(96, 400, 16, "fixed"), (96, 400, 0, "fixed"), (640, 1280, 16, "approx"),
                                               (300, 130, 24, "fixed"), (200, 824, 24, "approx")])
 def test_without_error_feedback_lockstep(m, n, k, selection):
