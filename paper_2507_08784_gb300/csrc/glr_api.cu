@@ -45,7 +45,8 @@ struct glr_handle {
     float *YT = nullptr, *YtT = nullptr;   // k x transposed_pitch(m') copies of Y and Yt for the fused kernel
     float *YF = nullptr, *YtF = nullptr;   // Y and Yt in fragment order for the tensor-core kernel
     int* dflags = nullptr;   // [0] Cholesky restarts, [1] Jacobi sweeps of the last refresh,
-                             // [2] bounded device waits of the compose kernel that gave up
+                             // [2] bounded device waits of the compose kernel that gave up,
+                             // [4..5] the cooperative Jacobi's grid barrier
     float* gemm_ws = nullptr;   // split-K partial tiles of the refresh GEMMs
     // Large plain products (>= 2^26 flops) go to cuBLAS: one library handle for the step stream
     // and one for the refresh stream (a handle's workspace must not serve two streams at once).
@@ -654,7 +655,7 @@ int glr_create(int64_t m, int64_t n, int32_t r, int32_t N, const glr_schedule* s
     if (s->optimizer != GLR_MSGD) A(&h->Vo, galore ? (size_t)r * NP : (size_t)m * n);
     if (s->optimizer == GLR_AMSGRAD) A(&h->amsv, 2);
     if (galore) A(&h->galr, (size_t)r * NP);
-    A(&h->dflags, 4);
+    A(&h->dflags, 6);
     A(&h->gemm_ws, (size_t)kGemmWsFloats);
     // the first path with library products when the rank-r products are large
     h->tc = !h->fused && mp % 4 == 0 && np % 4 == 0 && 2.0 * r * (double)mp * (double)np * N >= 67108864.0 ? 1 : 0;
