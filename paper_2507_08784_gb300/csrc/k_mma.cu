@@ -304,10 +304,12 @@ __device__ __forceinline__ void compose_node(const float* S, const GT* Gs, bool 
             RA[nt] = frag_a(R.x, R.z, R.y, R.w);
         }
     }
-    // the lane's first row of group 0 in node i's B, and the distance to group j's (128 rows per
-    // group step) and to row rb (2 rows)
-    float* const Brow = Bi + (int64_t)(8 * L.w + L.rho) * np;
-    const int64_t jstep = (int64_t)(8 * NW) * np;
+    // the lane's element offsets from node i's strip base Bi (warp-uniform): its first row of
+    // group 0 and column c2, the step to group j's rows (128 rows) and to row rb (2 rows); a node
+    // holds fewer than 2^31 elements, so 32 bits suffice and the stores address uniform base +
+    // lane offset
+    const uint32_t orow = static_cast<uint32_t>((8 * L.w + L.rho) * np + L.c2);
+    const uint32_t jstep = static_cast<uint32_t>(8 * NW * np), rstep = static_cast<uint32_t>(2 * np);
 #pragma unroll
     for (int j = 0; j < GPW; ++j) {
         const int G8 = L.w + NW * j;
@@ -334,9 +336,9 @@ __device__ __forceinline__ void compose_node(const float* S, const GT* Gs, bool 
             const float m2 = g1.x + (x1.x - c[1]);
             const float m3 = g1.y + (x1.y - c[3]);
             if (write_B && colok) {
-                float* const Ba = Brow + j * jstep;
-                if (ra < mp) st_stream2(Ba, m0, m1);
-                if (rb < mp) st_stream2(Ba + 2 * (int64_t)np, m2, m3);
+                const uint32_t oa = orow + j * jstep;
+                if (ra < mp) st_stream2(Bi + oa, m0, m1);
+                if (rb < mp) st_stream2(Bi + (oa + rstep), m2, m3);
             }
             acc[j][0] += m0; acc[j][1] += m1; acc[j][2] += m2; acc[j][3] += m3;
         }
@@ -644,7 +646,7 @@ __device__ __forceinline__ void compose_strip(const StreamGroup& g, const TmaMap
         const float* S = reinterpret_cast<const float*>(ring + (size_t)(i % 3) * stage);
         const GT* Gs = reinterpret_cast<const GT*>(ring + (size_t)(i % 3) * stage + sb);
         compose_node<GT, NQ, GPW>(S, Gs, trans, gpt, corr, prt, pcb, acc, part, pitch, tot,
-                                  Bst + (int64_t)i * mp * np + b0 + L.c2, mp, np, ng, write_B, colok, L);
+                                  Bst + (int64_t)i * mp * np + b0, mp, np, ng, write_B, colok, L);
         if constexpr (TMA) {               // this warp is done with node i's slot
             __syncwarp();
             if (L.lane == 0) mbar_arrive(empty_s + 8 * (i % 3));
