@@ -253,16 +253,26 @@ def cpu_oracle_sample(cfg, budget_s=25.0, compressed_steps=20):
 
 
 class DistCtx:
-    def __init__(self):
+    """One rank per GPU (torchrun's RANK / WORLD_SIZE / LOCAL_RANK / MASTER_*): NCCL on GPUs, gloo
+    when the process has no GPU (the host-side tests of the multi-rank path).  Only the barrier
+    and the max of the ranks' timings cross ranks; the data path has no collective."""
+
+    def __init__(self, backend=None):
         self.world = int(os.environ.get("WORLD_SIZE", "1"))
         self.rank = int(os.environ.get("RANK", "0"))
         self.local = int(os.environ.get("LOCAL_RANK", "0"))
+        self.backend = backend
         self.pg = None
 
     def init(self, torch):
         if self.world > 1:
             import torch.distributed as dist
-            dist.init_process_group("nccl", device_id=torch.device("cuda", self.local))
+            if self.backend is None:
+                self.backend = "nccl" if torch.cuda.is_available() else "gloo"
+            if self.backend == "nccl":
+                dist.init_process_group("nccl", device_id=torch.device("cuda", self.local))
+            else:
+                dist.init_process_group(self.backend)
             self.pg = dist
 
     def barrier(self):
@@ -273,9 +283,15 @@ class DistCtx:
         if not self.pg:
             return v
         import torch
-        t = torch.tensor([v], device="cuda", dtype=torch.float64)
+        t = torch.tensor([v], device="cuda" if self.backend == "nccl" else "cpu", dtype=torch.float64)
         self.pg.all_reduce(t, op=self.pg.ReduceOp.MAX)
         return float(t.item())
+
+
+def job_rate(world, units_per_rank, ms_max):
+    """Whole-job throughput of `world` replicas (weak scaling): every rank processed
+    units_per_rank inside its timed region, and the job took as long as its slowest rank."""
+    return world * units_per_rank / (ms_max / 1e3)
 
 
 def run_reference(args):
@@ -352,7 +368,7 @@ def main():
 
     K = args.steps
     elems = cfg.N * cfg.matrix_elems()
-    value = ctx.world * elems * K / (main_run["ms"] / 1e3)
+    value = job_rate(ctx.world, elems * K, main_run["ms"])
     ph = main_run["phases"]
     # the refresh phase runs on one side stream per matrix, concurrently: its summed event time
     # is not wall time, so the dominant phase is taken among the phases on the step's stream and
@@ -402,13 +418,13 @@ def main():
         "phases_note": "refresh = summed event time of the concurrent per-matrix refresh streams",
         "phase_launches": {k: v["launches"] for k, v in ph.items()},
         "paper_exact_basis": None if exact_run is None else {
-            "value": ctx.world * elems * K / (exact_run["ms"] / 1e3),
+            "value": job_rate(ctx.world, elems * K, exact_run["ms"]),
             "ms_per_step": exact_run["ms"] / K,
             "nonrefresh_step_ms_median": exact_run["nonrefresh_step_ms"],
             "refresh_ms_all_matrices": (exact_run["refresh_step_ms"] - exact_run["nonrefresh_step_ms"])
             if exact_run["refresh_step_ms"] else None,
             "phases_ms_per_step": {k: v["ms"] / K for k, v in exact_run["phases"].items()}},
-        "e2e": None if e2e is None else {"value": ctx.world * elems * args.e2e_steps / (e2e["ms"] / 1e3), "unit": UNIT,
+        "e2e": None if e2e is None else {"value": job_rate(ctx.world, elems * args.e2e_steps, e2e["ms"]), "unit": UNIT,
                                          "h2d_bytes_per_step": e2e["h2d"], "d2h_bytes_per_step": e2e["d2h"]},
         "gpu_launches": main_run["launches"],
         "clocks": clk.summary(),
