@@ -2,9 +2,9 @@
 // optimizer update without another pass over Mbar.  With U = (I - Y T Y^T) D and P = U[:, J]
 // (the WY form of the truncated basis),
 //   Rbar = P^T Mbar = D_J (Mbar[J, :] - Yt[J, :] Wbar),   Yt = Y T^T,  Wbar = Y^T Mbar,
-// and Wbar comes out of K1's lambda epilogue.  A CTA forms its TC columns of Rbar from the r
-// rows J of Mbar and of Yt and from Wbar (and writes them out: the projected mean of the step),
-// then streams X and the optimizer state once: Ghat = P Rbar (Alg. 3), MSGD (Eq. msgd) or Adam
+// and Wbar comes out of K1's lambda epilogue; the selection's pr_kernel forms Rbar that way from
+// the r rows J of Mbar and of Yt.  A CTA stages its TC columns of Rbar in shared memory, then
+// streams X and the optimizer state once: Ghat = P Rbar (Alg. 3), MSGD (Eq. msgd) or Adam
 // (Eq. adam).  Bytes per matrix element: X and the moments read and written (16 B MSGD, 24 B Adam);
 // Mbar is touched only in the r selected rows.
 #include "glr_internal.cuh"
