@@ -216,7 +216,24 @@ def bench_e2e(torch, glr, cfg, K, Wm, dist_ctx):
     for h in hs:
         h.close()
     gsz = 4 if cfg.grad_dtype == "f32" else 2
-    return {"ms": ms, "h2d": cfg.N * cfg.matrix_elems() * gsz, "d2h": cfg.matrix_elems() * 4}
+    h2d = cfg.N * cfg.matrix_elems() * gsz
+    return {"ms": ms, "h2d": h2d, "d2h": cfg.matrix_elems() * 4, "link_gbs": h2d_link_gbs(torch, h2d)}
+
+
+def h2d_link_gbs(torch, nbytes, reps=3):
+    """This machine's host-to-device copy rate for one step's worth of gradient bytes: one pinned
+    buffer copied to the device in a single copy, best of `reps` (CUDA events)."""
+    src = torch.empty(nbytes, dtype=torch.uint8).pin_memory()
+    dst = torch.empty(nbytes, dtype=torch.uint8, device="cuda")
+    best = float("inf")
+    for _ in range(reps + 1):
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record()
+        dst.copy_(src, non_blocking=True)
+        e1.record()
+        torch.cuda.synchronize()
+        best = min(best, e0.elapsed_time(e1))
+    return nbytes / (best / 1e3) / 1e9
 
 
 def cpu_oracle_sample(cfg, budget_s=25.0, compressed_steps=20):
@@ -425,7 +442,10 @@ def main():
             if exact_run["refresh_step_ms"] else None,
             "phases_ms_per_step": {k: v["ms"] / K for k, v in exact_run["phases"].items()}},
         "e2e": None if e2e is None else {"value": job_rate(ctx.world, elems * args.e2e_steps, e2e["ms"]), "unit": UNIT,
-                                         "h2d_bytes_per_step": e2e["h2d"], "d2h_bytes_per_step": e2e["d2h"]},
+                                         "h2d_bytes_per_step": e2e["h2d"], "d2h_bytes_per_step": e2e["d2h"],
+                                         "h2d_link_gbs": e2e["link_gbs"],
+                                         "frac_of_link": (e2e["h2d"] / (e2e["ms"] / args.e2e_steps / 1e3) / 1e9)
+                                                         / e2e["link_gbs"]},
         "gpu_launches": main_run["launches"],
         "clocks": clk.summary(),
     }
