@@ -82,14 +82,14 @@ extern "C" {
  *   tau            refresh period (>= 1)
  *   refresh_mode   GLR_ALG3 | GLR_ALG4
  *   optimizer      GLR_MSGD | GLR_ADAM | GLR_AMSGRAD | GLR_ADAMW | GLR_GALORE_ADAM; lr = gamma;
- *                  beta1 = beta
- *                  (MSGD) or beta_1 (Adam types); beta2, eps used by the Adam types only
+ *                  beta1 = beta (MSGD) or beta_1 (Adam types); beta2, eps used by the Adam
+ *                  types only
  *   seed           64-bit key of the shared random vectors v_j (Eq. random-v): all nodes
  *                  of one matrix draw the same v_j; give every matrix its own seed
  *   basis_rank     k.  0 (or m') keeps the full m' x m' singular basis U of Eq. SVD-P1
- *                  (paper-exact).  r <= k < m' keeps the top-k singular vectors and
- *                  completes them to an orthogonal U with Householder reflectors; the
- *                  refresh then uses power_iters block power iterations
+ *                  (paper-exact; m' <= 1024).  r <= k < m', k <= 512, keeps the top-k
+ *                  singular vectors and completes them to an orthogonal U with Householder
+ *                  reflectors; the refresh then uses power_iters block power iterations
  *   power_iters    q >= 1 (truncated basis only)
  *   grad_dtype     GLR_F32 | GLR_BF16
  *   compress_start the first compress_start steps are uncompressed (plain node mean, no
