@@ -1,122 +1,27 @@
-// C ABI of libglr.so: handle lifetime, the per-step schedule of Algorithm 3 (Semi-Lazy SVD
-// refresh every tau steps, Approx-Top-r selection otherwise) and the introspection calls.
-// All device work is enqueued on the caller's stream; the host only tracks the schedule.
-#include <algorithm>
-#include <cmath>
-#include <cstdio>
-#include <cstring>
-#include <string>
-#include <vector>
-
-#include <cublas_v2.h>
-
-#include "glr_internal.cuh"
+// C ABI of libglr.so: handle lifetime and the per-step schedule of Algorithm 3 (Semi-Lazy SVD
+// refresh every tau steps, Approx-Top-r selection otherwise), with the host helpers the library's
+// other host files share (glr_host.cuh).  All device work is enqueued on the caller's stream; the
+// host only tracks the schedule.  The refresh orchestration is in glr_refresh_host.cu, the
+// checkpoints and introspection calls in glr_introspect.cu.
+#include "glr_host.cuh"
 
 using namespace glr;
+using namespace glr::host;
 
-namespace {
-constexpr int kMaxRank = 512;
-constexpr int kMaxFullBasis = 1024;
-constexpr int kMaxTruncBasis = 512;
+namespace glr {
+namespace host {
+
 thread_local std::string g_create_err;
-}  // namespace
+thread_local float* g_ws = nullptr;
 
-struct glr_handle {
-    int64_t m = 0, n = 0;
-    int mp = 0, np = 0, transposed = 0, r = 0, N = 0, k = 0, exact = 0;
-    glr_schedule s{};
-    int device = 0;
-    size_t gsize = 4;
-    // device state
-    float *B = nullptr, *Mbar = nullptr, *Rw = nullptr, *Rbar = nullptr, *P = nullptr, *Pprev = nullptr;
-    int32_t* J = nullptr;
-    float *lam = nullptr, *lam_part = nullptr;
-    int ntiles = 0;                 // lambda tiles of the first-path kernel (64 columns)
-    int fused = 0, BN = 0, nstrips = 0;   // fused strip kernels: strip width, strips per matrix
-    int mma = 0;                          // compose on the tensor cores (k_mma.cu)
-    int tma = 0;                          // ... with its ring filled by tile copies
-    CUtensorMap Bmap{};                   // tile-copy descriptor of B (n' x m' x N)
-    struct GMap { const void* ptr; CUtensorMap map; };
-    std::vector<GMap> gmaps;              // per node: the descriptors of its last two gradient buffers
-    float *Mo = nullptr, *Vo = nullptr;
-    float *U = nullptr, *Hbuf = nullptr, *Vbuf = nullptr, *evals = nullptr, *evals_sorted = nullptr;
-    float *Q = nullptr, *Qn = nullptr, *Y = nullptr, *Yt = nullptr, *T = nullptr, *dsign = nullptr;
-    float *Wbar = nullptr, *Z = nullptr, *Zn = nullptr, *Hk = nullptr, *Vk = nullptr, *gram = nullptr, *scratch = nullptr;
-    float *YT = nullptr, *YtT = nullptr;   // k x transposed_pitch(m') copies of Y and Yt for the fused kernel
-    float *YF = nullptr, *YtF = nullptr;   // Y and Yt in fragment order for the tensor-core kernel
-    int* dflags = nullptr;   // [0] Cholesky restarts, [1] Jacobi sweeps of the last refresh,
-                             // [2] bounded device waits of the compose kernel that gave up,
-                             // [4..5] the cooperative Jacobi's grid barrier
-    float* gemm_ws = nullptr;   // split-K partial tiles of the refresh GEMMs
-    // Large plain products (>= 2^26 flops) go to cuBLAS: one library handle for the step stream
-    // and one for the refresh stream (a handle's workspace must not serve two streams at once).
-    cublasHandle_t cb[2] = {nullptr, nullptr};
-    // The first path with its rank-r / rank-k products as library GEMMs (set when those products
-    // are large): E_i = B_i - P_prev (P_prev^T B_i) in place, D = Mbar - Yt W and Ghat = P Rbar
-    // in mn_scratch (m' x n').
-    int tc = 0;
-    float* mn_scratch = nullptr;
-    float* jwork = nullptr;      // full basis: the grouped Jacobi's second m' x m' buffer
-    float* jpart = nullptr;      // full basis: its per-CTA norm partials (used by a group's first handle)
-    float* YtJ = nullptr;        // Yt[J, :] (r x k) for P = U[:, J] as a library product
-    float* amsv = nullptr;       // AMSGrad: the scalar normaliser and this step's maximum of V
-    float* galr = nullptr;       // Algorithm 5: the subspace step direction M / (sqrt(V) + eps), r x n'
-    cudaStream_t rstream = nullptr;            // side stream of this handle's refresh
-    cudaEvent_t rfork = nullptr, rdone = nullptr, rpow = nullptr;
-    int pow_ok = 0;                            // refresh through the grouped power iteration (k_power.cu)
-    float *powpart = nullptr, *powG = nullptr, *powS = nullptr;
-    void* Gstage = nullptr;
-    // glr_step_group_host: two device staging buffers of N gradients, filled on a copy stream
-    void* Gstage2[2] = {nullptr, nullptr};
-    cudaStream_t cstream = nullptr;
-    cudaEvent_t cdone = nullptr, sfree[2] = {nullptr, nullptr};
-    bool sfree_set[2] = {false, false};
-    int host_parity = 0;
-    // host state
-    int64_t t = 0, refreshes = 0, comm = 0, state_bytes = 0, period_start = 0;
-    bool e_zero = true, force_refresh = false, last_uncompressed = true, basis_from_user = false;
-    bool has_forceJ = false, forced_this_step = false;
-    std::vector<int32_t> forceJ, iotaJ;
-    std::vector<void*> allocs;
-    std::vector<size_t> alloc_bytes;
-    size_t n_state_allocs = 0;       // allocations made by glr_create (the checkpointed state)
-    std::string err;
-    // launch counting and optional per-phase event timing
-    int64_t launches = 0;
-    bool prof = false;
-    struct Rec { int phase; cudaEvent_t a, b; int64_t launches; };
-    std::vector<Rec> recs;
-    std::vector<cudaEvent_t> free_events;
-    double prof_ms[GLR_PHASES] = {};
-    int64_t prof_launch[GLR_PHASES] = {}, prof_count[GLR_PHASES] = {};
-    int cur_phase = -1;
-    cudaEvent_t cur_start = nullptr;
-    int64_t cur_launch0 = 0;
-};
-
-namespace {
-
-int fail(glr_handle* h, int code, const char* fmt, const char* a = "", int line = 0) {
+int fail(glr_handle* h, int code, const char* fmt, const char* a, int line) {
     char buf[512];
     snprintf(buf, sizeof(buf), fmt, a, line);
     if (h) h->err = buf; else g_create_err = buf;
     return code;
 }
 
-#define GLR_CK(h, expr)                                                                        \
-    do {                                                                                       \
-        cudaError_t e__ = (expr);                                                              \
-        if (e__ != cudaSuccess)                                                                \
-            return fail((h), GLR_ECUDA, "CUDA error %s (glr_api.cu:%d)", cudaGetErrorString(e__), \
-                        __LINE__);                                                             \
-    } while (0)
 
-// Count kernels launched by a launcher call and check its status.
-#define GLR_LAUNCH(h, nk, expr)                                                                \
-    do {                                                                                       \
-        (h)->launches += (nk);                                                                 \
-        GLR_CK(h, expr);                                                                       \
-    } while (0)
 
 cudaEvent_t take_event(glr_handle* h) {
     if (!h->free_events.empty()) {
@@ -145,28 +50,7 @@ void phase_end(glr_handle* h, cudaStream_t st) {
     h->cur_phase = -1;
 }
 
-struct PhaseScope {
-    glr_handle* h; cudaStream_t st;
-    PhaseScope(glr_handle* h_, int phase, cudaStream_t st_) : h(h_), st(st_) { phase_begin(h, phase, st); }
-    ~PhaseScope() { phase_end(h, st); }
-};
 
-template <typename T>
-int alloc(glr_handle* h, T** p, size_t count) {
-    if (count == 0) count = 1;
-    void* ptr = nullptr;
-    const size_t bytes = count * sizeof(T);
-    if (cudaMalloc(&ptr, bytes) != cudaSuccess) {
-        cudaGetLastError();
-        return fail(h, GLR_ENOMEM, "device allocation of %s bytes failed", std::to_string(bytes).c_str());
-    }
-    h->allocs.push_back(ptr);
-    h->alloc_bytes.push_back(bytes);
-    h->state_bytes += static_cast<int64_t>(bytes);
-    if (cudaMemset(ptr, 0, bytes) != cudaSuccess) return fail(h, GLR_ECUDA, "cudaMemset failed%s");
-    *p = static_cast<T*>(ptr);
-    return GLR_OK;
-}
 
 void free_all(glr_handle* h) {
     for (void* p : h->allocs) cudaFree(p);
@@ -217,10 +101,9 @@ bool gradient_map(glr_handle* h, int i, const void* ptr, CUtensorMap* out) {
     return true;
 }
 
-thread_local float* g_ws = nullptr;   // split-K workspace of the handle being stepped
 
 GemmDesc gd(int M, int N, int K, const float* A, int64_t sAi, int64_t sAp, const float* B, int64_t sBp,
-            int64_t sBj, float* C, int64_t sCi, int64_t sCj, float alpha = 1.f, float beta = 0.f) {
+            int64_t sBj, float* C, int64_t sCi, int64_t sCj, float alpha, float beta) {
     GemmDesc d{};
     d.ws = g_ws;
     d.ws_floats = g_ws ? kGemmWsFloats : 0;
@@ -281,195 +164,18 @@ int gemm(glr_handle* h, const GemmDesc& d, cudaStream_t st) {
     GLR_LAUNCH(h, 1, gemm_f32(d, st));
     return GLR_OK;
 }
-#define GLR_GEMM(h, d, st)                                                                       \
-    do {                                                                                       \
-        const int gemm_rc_ = gemm((h), (d), (st));                                             \
-        if (gemm_rc_ != GLR_OK) return gemm_rc_;                                               \
-    } while (0)
 
-// A (rows x k, row-major) <- A L^{-T} with L L^T = A^T A (CholeskyQR): the k x k factor and its
-// inverse in one CTA, then one product into tmp; A and tmp trade places.
-int cholqr(glr_handle* h, float*& A, float*& tmp, int rows, cudaStream_t st) {
-    const int k = h->k;
-    GLR_GEMM(h, gd(k, k, rows, A, 1, k, A, k, 1, h->gram, k, 1), st);
-    if (k > 256) {                           // the factor does not fit one CTA's shared memory
-        GLR_LAUNCH(h, 1, cholesky(h->gram, k, h->scratch, h->dflags + 0, st));
-        GLR_LAUNCH(h, 1, trsm_right_lt(A, rows, k, h->gram, st));
-        return GLR_OK;
-    }
-    GLR_LAUNCH(h, 1, chol_inverse(h->gram, k, h->scratch, h->dflags + 0, st));
-    GLR_GEMM(h, gd(rows, k, k, A, k, 1, h->scratch, k, 1, tmp, k, 1), st);
-    std::swap(A, tmp);
-    return GLR_OK;
+int fail_cuda(glr_handle* h, cudaError_t e, const char* file, int line) {
+    const char* base = std::strrchr(file, '/');
+    const std::string where = std::string(cudaGetErrorString(e)) + " (" + (base ? base + 1 : file) + ":" +
+                              std::to_string(line) + ")";
+    return fail(h, GLR_ECUDA, "CUDA error %s", where.c_str());
 }
 
-int wy_from_Q(glr_handle* h, cudaStream_t st) {
-    const int mp = h->mp, k = h->k;
-    GLR_LAUNCH(h, 2, householder_reconstruct(h->Q, mp, k, h->Y, h->T, h->dsign, h->scratch, st));
-    // Yt = Y T^T
-    GLR_GEMM(h, gd(mp, k, k, h->Y, k, 1, h->T, 1, k, h->Yt, k, 1), st);
-    // transposed copies (k x tp, zero-padded) for the fused compose kernel's lambda epilogue
-    GLR_LAUNCH(h, 1, transpose_pad(h->YT, transposed_pitch(mp), h->Y, mp, k, st));
-    GLR_LAUNCH(h, 1, transpose_pad(h->YtT, transposed_pitch(mp), h->Yt, mp, k, st));
-    if (h->mma) {
-        GLR_LAUNCH(h, 1, pack_frag(h->YF, h->Y, mp, k, k, 0, st));
-        GLR_LAUNCH(h, 1, pack_frag(h->YtF, h->Yt, mp, k, k, 1, st));
-    }
-    return GLR_OK;
-}
+}  // namespace host
+}  // namespace glr
 
-// End of a truncated refresh, with Q orthonormal and H = Q^T Mbar Mbar^T Q in Hk: Rayleigh-Ritz
-// H = W diag W^T, Q <- Q W (columns by descending Ritz value, signs fixed), then the WY form.
-int refresh_tail(glr_handle* h, cudaStream_t st) {
-    const int mp = h->mp, k = h->k;
-    GLR_LAUNCH(h, 1, jacobi_eig(h->Hk, k, h->Vk, h->evals, h->dflags + 1, st));
-    GLR_LAUNCH(h, 1, sort_fix_basis(h->evals, h->Vk, k, k, h->gram, k, h->evals_sorted, st));
-    GLR_GEMM(h, gd(mp, k, k, h->Q, k, 1, h->gram, k, 1, h->Qn, k, 1), st);
-    GLR_LAUNCH(h, 1, fix_column_signs(h->Qn, mp, k, st));
-    std::swap(h->Q, h->Qn);
-    return wy_from_Q(h, st);
-}
-
-// Truncated refreshes of several matrices through the grouped block power iteration
-// (k_power.cu): the same iteration as do_refresh (q power iterations, each half re-normalised by
-// CholeskyQR, then CholeskyQR2 and the Rayleigh-Ritz Gram), one launch per stage for all of
-// them on the first handle's side stream; the k x k tails run on each handle's own stream.
-int refresh_grouped(std::vector<glr_handle*>& hs) {
-    glr_handle* h0 = hs[0];
-    cudaStream_t s0 = h0->rstream;
-    for (glr_handle* h : hs) GLR_CK(h0, cudaStreamWaitEvent(s0, h->rfork, 0));
-    {
-        PhaseScope ps(h0, GLR_PH_REFRESH, s0);
-        PowGroup g{};
-        const int PC = pow_tile(), CH = pow_chunk();
-        int q = h0->s.power_iters;
-        for (glr_handle* h : hs) {
-            if (h->refreshes == 0 && !h->basis_from_user)
-                GLR_LAUNCH(h0, 1, random_block(h->Q, h->mp, h->k, h->s.seed, static_cast<uint32_t>(h->t), s0));
-            PowMat& M = g.mat[g.nmat++];
-            M.mp = h->mp; M.np = h->np; M.k = h->k; M.active = 1;
-            M.t0 = g.tot_t; M.nt = (h->np + PC - 1) / PC; g.tot_t += M.nt;
-            M.r0 = g.tot_r; M.nr = (h->mp + PC - 1) / PC; g.tot_r += M.nr;
-            M.n0 = g.tot_n; M.nn = (h->np + CH - 1) / CH; g.tot_n += M.nn * M.nr;
-            M.Mbar = h->Mbar; M.Q = h->Q; M.Z = h->Z; M.part = h->powpart; M.G = h->powG; M.S = h->powS;
-            M.H = h->Hk; M.flag = h->dflags + 0;
-            q = std::max(q, h->s.power_iters);
-        }
-        // a matrix with fewer power iterations than the group's maximum drops out early
-        for (int it = 0; it < q; ++it) {
-            for (int i = 0; i < g.nmat; ++i) g.mat[i].active = it < hs[i]->s.power_iters ? 1 : 0;
-            GLR_LAUNCH(h0, 1, pow_stage(g, 0, it > 0 ? 1 : 0, s0));   // Z = (Mbar^T Q) S
-            GLR_LAUNCH(h0, 1, pow_stage(g, 4, 1, s0));                // S = chol(Z^T Z)^-T
-            GLR_LAUNCH(h0, 1, pow_stage(g, 1, 0, s0));                // partials of Mbar Z
-            GLR_LAUNCH(h0, 1, pow_stage(g, 2, 0, s0));                // Q = (Mbar Z) S
-            GLR_LAUNCH(h0, 1, pow_stage(g, 4, 0, s0));                // S = chol(Q^T Q)^-T
-        }
-        for (int i = 0; i < g.nmat; ++i) g.mat[i].active = 1;
-        GLR_LAUNCH(h0, 1, pow_stage(g, 3, 1, s0));                    // CholeskyQR2: Q <- Q S ...
-        GLR_LAUNCH(h0, 1, pow_stage(g, 4, 0, s0));
-        GLR_LAUNCH(h0, 1, pow_stage(g, 3, 0, s0));                    // ... twice: orthonormal
-        GLR_LAUNCH(h0, 1, pow_stage(g, 0, 0, s0));                    // Rayleigh-Ritz: Z = Mbar^T Q
-        GLR_LAUNCH(h0, 1, pow_stage(g, 5, 1, s0));                    // H = Z^T Z
-    }
-    GLR_CK(h0, cudaEventRecord(h0->rpow, s0));
-    for (glr_handle* h : hs) {
-        if (h != h0) GLR_CK(h, cudaStreamWaitEvent(h->rstream, h0->rpow, 0));
-        PhaseScope ps(h, GLR_PH_REFRESH, h->rstream);
-        g_ws = h->gemm_ws;
-        const int rc = refresh_tail(h, h->rstream);
-        g_ws = nullptr;
-        if (rc != GLR_OK) return rc;
-    }
-    return GLR_OK;
-}
-
-// Full-basis refreshes of several matrices: H = Mbar Mbar^T on each handle's side stream, one
-// cooperative Jacobi launch for all of them on the first handle's side stream (k_jacobi.cu), then
-// each handle sorts its eigenvectors by descending eigenvalue and fixes their signs on its own.
-int refresh_exact_grouped(std::vector<glr_handle*>& hs) {
-    const int grid = jacobi_group_grid();
-    for (size_t c0 = 0, c1 = 0; c0 < hs.size(); c0 = c1) {
-        // a group: at most kGroupMax matrices whose rotations fit the kernel's shared memory
-        size_t rot = 0;
-        for (c1 = c0; c1 < hs.size() && c1 - c0 < (size_t)kGroupMax; ++c1) {
-            const size_t add = jacobi_rot_floats(hs[c1]->mp) * sizeof(float);
-            if (c1 > c0 && rot + add > kJacobiMaxSmem) break;
-            rot += add;
-        }
-        glr_handle* h0 = hs[c0];
-        cudaStream_t s0 = h0->rstream;
-        for (size_t i = c0; i < c1; ++i) {
-            glr_handle* h = hs[i];
-            PhaseScope ps(h, GLR_PH_REFRESH, h->rstream);
-            const int mp = h->mp, np = h->np;
-            GLR_GEMM(h, gd(mp, mp, np, h->Mbar, np, 1, h->Mbar, 1, np, h->Hbuf, mp, 1), h->rstream);
-            if (!grid) {                                         // no cooperative launch: one CTA each
-                GLR_LAUNCH(h, 1, jacobi_eig(h->Hbuf, mp, h->Vbuf, h->evals, h->dflags + 1, h->rstream));
-                GLR_LAUNCH(h, 1, sort_fix_basis(h->evals, h->Vbuf, mp, mp, h->U, mp, h->evals_sorted, h->rstream));
-                continue;
-            }
-            GLR_CK(h, cudaEventRecord(h->rpow, h->rstream));
-            if (h != h0) GLR_CK(h0, cudaStreamWaitEvent(s0, h->rpow, 0));
-        }
-        if (!grid) continue;
-        JacobiGroup g{};
-        size_t soff = 0;
-        g.max_sweeps = 40;
-        g.bar = h0->dflags + 4; g.err = h0->dflags + 2; g.part = h0->jpart;
-        for (size_t i = c0; i < c1; ++i) {
-            glr_handle* h = hs[i];
-            JacobiMat& M = g.mat[g.nmat++];
-            const int n = h->mp;
-            M.n = n; M.tol = 4.f * 5.96e-8f * sqrtf(static_cast<float>(n)) + 1e-7f;
-            M.H = h->Hbuf; M.H2 = h->jwork; M.V = h->Vbuf; M.evals = h->evals;
-            M.sweeps = h->dflags + 1;
-            M.soff = (int)soff;
-            soff += jacobi_rot_floats(n);
-        }
-        {
-            PhaseScope ps(h0, GLR_PH_REFRESH, s0);
-            GLR_LAUNCH(h0, 1, jacobi_group(g, grid, s0));
-        }
-        GLR_CK(h0, cudaEventRecord(h0->rpow, s0));
-        for (size_t i = c0; i < c1; ++i) {
-            glr_handle* h = hs[i];
-            if (h != h0) GLR_CK(h, cudaStreamWaitEvent(h->rstream, h0->rpow, 0));
-            PhaseScope ps(h, GLR_PH_REFRESH, h->rstream);
-            GLR_LAUNCH(h, 1, sort_fix_basis(h->evals, h->Vbuf, h->mp, h->mp, h->U, h->mp, h->evals_sorted, h->rstream));
-        }
-    }
-    return GLR_OK;
-}
-
-// Semi-Lazy SVD refresh (Eq. SVD-P1) from Mbar.
-int do_refresh(glr_handle* h, cudaStream_t st) {
-    const int mp = h->mp, np = h->np, k = h->k;
-    g_ws = h->gemm_ws;
-    struct Reset { ~Reset() { g_ws = nullptr; } } reset_ws;
-    if (h->exact) {
-        // H = Mbar Mbar^T, eigenvectors = left singular vectors, sorted by descending sigma
-        GLR_GEMM(h, gd(mp, mp, np, h->Mbar, np, 1, h->Mbar, 1, np, h->Hbuf, mp, 1), st);
-        GLR_LAUNCH(h, 1, jacobi_eig(h->Hbuf, mp, h->Vbuf, h->evals, h->dflags + 1, st));
-        GLR_LAUNCH(h, 1, sort_fix_basis(h->evals, h->Vbuf, mp, mp, h->U, mp, h->evals_sorted, st));
-        return GLR_OK;
-    }
-    if (h->refreshes == 0 && !h->basis_from_user)
-        GLR_LAUNCH(h, 1, random_block(h->Q, mp, k, h->s.seed, static_cast<uint32_t>(h->t), st));
-    int rc;
-    for (int it = 0; it < h->s.power_iters; ++it) {
-        // Z = Mbar^T Q (n' x k) and Q = Mbar Z (m' x k), each re-orthonormalised by CholeskyQR
-        // (one pass keeps the block well conditioned; the span is what the iteration needs)
-        GLR_GEMM(h, gd(np, k, mp, h->Mbar, 1, np, h->Q, k, 1, h->Z, k, 1), st);
-        if ((rc = cholqr(h, h->Z, h->Zn, np, st)) != GLR_OK) return rc;
-        GLR_GEMM(h, gd(mp, k, np, h->Mbar, np, 1, h->Z, k, 1, h->Q, k, 1), st);
-        if ((rc = cholqr(h, h->Q, h->Qn, mp, st)) != GLR_OK) return rc;
-    }
-    if ((rc = cholqr(h, h->Q, h->Qn, mp, st)) != GLR_OK) return rc;   // CholeskyQR2: orthonormal to rounding
-    // Rayleigh-Ritz: Z = Mbar^T Q, H = Z^T Z = Q^T Mbar Mbar^T Q
-    GLR_GEMM(h, gd(np, k, mp, h->Mbar, 1, np, h->Q, k, 1, h->Z, k, 1), st);
-    GLR_GEMM(h, gd(k, k, np, h->Z, 1, k, h->Z, k, 1, h->Hk, k, 1), st);
-    return refresh_tail(h, st);
-}
+namespace {
 
 // Rbar = P^T Mbar; Ghat = P Rbar; optimizer.
 int project_and_update(glr_handle* h, float* X, cudaStream_t st) {
@@ -1226,223 +932,6 @@ int glr_step_group_host(glr_handle* const* handles, int32_t count, const void* c
         if (X_host_out && X_host_out[j])
             GLR_CK(h, cudaMemcpyAsync(X_host_out[j], X[j], sizeof(float) * h->m * h->n, cudaMemcpyDeviceToHost, st));
     }
-    return GLR_OK;
-}
-
-// ---- checkpoints ---------------------------------------------------------------------------
-// Layout: a header (magic, version, the handle's shape and schedule identity), the host scalars
-// of the schedule, the allocation index that each role which steps swap between two buffers
-// (P / Pprev, Q / Qn, Z / Zn) currently holds, then every device buffer glr_create allocated,
-// in allocation order.
-namespace {
-constexpr uint64_t kCkptMagic = 0x31544b50524c47ull;   // "GLRPKT1"
-struct CkptHeader {
-    uint64_t magic, version;
-    int64_t m, n;
-    int32_t r, N, k, grad_dtype, optimizer, refresh_mode;
-    uint64_t seed, nbuf, buf_bytes;
-    int64_t t, refreshes, comm, period_start;
-    int32_t e_zero, force_refresh, last_uncompressed, basis_from_user, has_forceJ, pad;
-    int32_t role[6];
-};
-float** role_ptr(glr_handle* h, int i) {
-    float** roles[6] = {&h->P, &h->Pprev, &h->Q, &h->Qn, &h->Z, &h->Zn};
-    return roles[i];
-}
-// bytes of a checkpoint of h; a pending forced selection (r indices) is stored when has_forceJ
-size_t ckpt_bytes(const glr_handle* h, bool has_forceJ) {
-    size_t b = sizeof(CkptHeader) + (has_forceJ ? sizeof(int32_t) * h->r : 0);
-    for (size_t i = 0; i < h->n_state_allocs; ++i) b += h->alloc_bytes[i];
-    return b;
-}
-}  // namespace
-
-int glr_state_size(const glr_handle* h, int64_t* bytes) {
-    if (!h || !bytes) return GLR_EINVAL;
-    *bytes = static_cast<int64_t>(ckpt_bytes(h, h->has_forceJ));
-    return GLR_OK;
-}
-
-int glr_save(glr_handle* h, void* host_buf, int64_t bytes, void* stream) {
-    if (!h) return GLR_EINVAL;
-    if (!host_buf || bytes < static_cast<int64_t>(ckpt_bytes(h, h->has_forceJ)))
-        return fail(h, GLR_EINVAL, "checkpoint buffer is null or smaller than glr_state_size%s");
-    cudaStream_t st = static_cast<cudaStream_t>(stream);
-    CkptHeader hd{};
-    hd.magic = kCkptMagic; hd.version = 1;
-    hd.m = h->m; hd.n = h->n; hd.r = h->r; hd.N = h->N; hd.k = h->k;
-    hd.grad_dtype = h->s.grad_dtype; hd.optimizer = h->s.optimizer; hd.refresh_mode = h->s.refresh_mode;
-    hd.seed = h->s.seed; hd.nbuf = h->n_state_allocs; hd.buf_bytes = ckpt_bytes(h, h->has_forceJ);
-    hd.t = h->t; hd.refreshes = h->refreshes; hd.comm = h->comm; hd.period_start = h->period_start;
-    hd.e_zero = h->e_zero; hd.force_refresh = h->force_refresh; hd.last_uncompressed = h->last_uncompressed;
-    hd.basis_from_user = h->basis_from_user; hd.has_forceJ = h->has_forceJ;
-    for (int i = 0; i < 6; ++i) {
-        hd.role[i] = -1;
-        float* p = *role_ptr(h, i);
-        for (size_t a = 0; a < h->n_state_allocs; ++a)
-            if (h->allocs[a] == p) hd.role[i] = static_cast<int32_t>(a);
-    }
-    char* out = static_cast<char*>(host_buf);
-    std::memcpy(out, &hd, sizeof(hd));
-    out += sizeof(hd);
-    if (h->has_forceJ) {
-        std::memcpy(out, h->forceJ.data(), sizeof(int32_t) * h->r);
-        out += sizeof(int32_t) * h->r;
-    }
-    for (size_t a = 0; a < h->n_state_allocs; ++a) {
-        GLR_CK(h, cudaMemcpyAsync(out, h->allocs[a], h->alloc_bytes[a], cudaMemcpyDeviceToHost, st));
-        out += h->alloc_bytes[a];
-    }
-    GLR_CK(h, cudaStreamSynchronize(st));
-    return GLR_OK;
-}
-
-int glr_load(glr_handle* h, const void* host_buf, int64_t bytes, void* stream) {
-    if (!h) return GLR_EINVAL;
-    if (!host_buf || bytes < static_cast<int64_t>(sizeof(CkptHeader)))
-        return fail(h, GLR_EINVAL, "checkpoint buffer is null or too small%s");
-    CkptHeader hd;
-    std::memcpy(&hd, host_buf, sizeof(hd));
-    if (hd.magic != kCkptMagic || hd.version != 1) return fail(h, GLR_EINVAL, "not a checkpoint of this library%s");
-    if (hd.m != h->m || hd.n != h->n || hd.r != h->r || hd.N != h->N || hd.k != h->k ||
-        hd.grad_dtype != h->s.grad_dtype || hd.optimizer != h->s.optimizer || hd.refresh_mode != h->s.refresh_mode ||
-        hd.nbuf != h->n_state_allocs || hd.buf_bytes != ckpt_bytes(h, hd.has_forceJ != 0))
-        return fail(h, GLR_EINVAL, "checkpoint of a handle with another shape or schedule%s");
-    if (bytes < static_cast<int64_t>(hd.buf_bytes)) return fail(h, GLR_EINVAL, "checkpoint buffer is truncated%s");
-    cudaStream_t st = static_cast<cudaStream_t>(stream);
-    const char* in = static_cast<const char*>(host_buf) + sizeof(hd);
-    if (hd.has_forceJ) {
-        h->forceJ.assign(reinterpret_cast<const int32_t*>(in), reinterpret_cast<const int32_t*>(in) + h->r);
-        in += sizeof(int32_t) * h->r;
-    }
-    for (size_t a = 0; a < h->n_state_allocs; ++a) {
-        GLR_CK(h, cudaMemcpyAsync(h->allocs[a], in, h->alloc_bytes[a], cudaMemcpyHostToDevice, st));
-        in += h->alloc_bytes[a];
-    }
-    for (int i = 0; i < 6; ++i)
-        if (hd.role[i] >= 0) *role_ptr(h, i) = static_cast<float*>(h->allocs[hd.role[i]]);
-    h->t = hd.t; h->refreshes = hd.refreshes; h->comm = hd.comm; h->period_start = hd.period_start;
-    h->e_zero = hd.e_zero; h->force_refresh = hd.force_refresh; h->last_uncompressed = hd.last_uncompressed;
-    h->basis_from_user = hd.basis_from_user; h->has_forceJ = hd.has_forceJ;
-    GLR_CK(h, cudaStreamSynchronize(st));
-    return GLR_OK;
-}
-
-int glr_refresh(glr_handle* h) {
-    if (!h) return GLR_EINVAL;
-    h->force_refresh = true;
-    return GLR_OK;
-}
-
-int glr_get_stats(const glr_handle* h, glr_stats* out) {
-    if (!h || !out) return GLR_EINVAL;
-    out->t = h->t; out->refreshes = h->refreshes; out->comm_floats_total = h->comm;
-    out->state_bytes = h->state_bytes;
-    out->m_prime = h->mp; out->n_prime = h->np; out->r = h->r; out->k = h->k;
-    out->transposed = h->transposed;
-    int flags[4] = {0, 0, 0, 0};
-    cudaMemcpy(flags, h->dflags, sizeof(flags), cudaMemcpyDeviceToHost);
-    out->last_refresh_sweeps = flags[1];
-    out->launches = h->launches;
-    return flags[2] ? GLR_ETIMEOUT : GLR_OK;
-}
-
-const char* glr_last_error(const glr_handle* h) { return h ? h->err.c_str() : g_create_err.c_str(); }
-
-int glr_get_error(glr_handle* h, int32_t i, float* E_out, void* stream) {
-    if (!h) return GLR_EINVAL;
-    if (i < 0 || i >= h->N || !E_out) return fail(h, GLR_EINVAL, "bad node index or null output%s");
-    cudaStream_t st = static_cast<cudaStream_t>(stream);
-    const int mp = h->mp, np = h->np, r = h->r;
-    float* Bi = h->B + (size_t)i * mp * np;
-    float* Rwi = h->Rw + (size_t)i * r * np;
-    if (!h->e_zero) GLR_GEMM(h, gd(r, np, mp, h->Pprev, 1, r, Bi, np, 1, Rwi, np, 1), st);
-    GLR_LAUNCH(h, 1, materialize_error(mp, np, r, h->e_zero ? 1 : 0, Bi, h->Pprev, Rwi, E_out, st));
-    return GLR_OK;
-}
-
-int glr_get_selection(glr_handle* h, int32_t* J_host, float* P_out, float* Rbar_out, float* lambda_out,
-                      float* Mbar_out, void* stream) {
-    if (!h) return GLR_EINVAL;
-    cudaStream_t st = static_cast<cudaStream_t>(stream);
-    const size_t mp = h->mp, np = h->np, r = h->r;
-    if (P_out) GLR_CK(h, cudaMemcpyAsync(P_out, h->Pprev, 4 * mp * r, cudaMemcpyDeviceToDevice, st));
-    if (Rbar_out) GLR_CK(h, cudaMemcpyAsync(Rbar_out, h->Rbar, 4 * r * np, cudaMemcpyDeviceToDevice, st));
-    if (lambda_out) GLR_CK(h, cudaMemcpyAsync(lambda_out, h->lam, 4 * mp, cudaMemcpyDeviceToDevice, st));
-    if (Mbar_out) GLR_CK(h, cudaMemcpyAsync(Mbar_out, h->Mbar, 4 * mp * np, cudaMemcpyDeviceToDevice, st));
-    if (J_host) {
-        if (h->last_uncompressed) {
-            for (size_t q = 0; q < r; ++q) J_host[q] = -1;
-        } else {
-            GLR_CK(h, cudaMemcpyAsync(J_host, h->J, 4 * r, cudaMemcpyDeviceToHost, st));
-        }
-    }
-    GLR_CK(h, cudaStreamSynchronize(st));
-    return GLR_OK;
-}
-
-int glr_get_basis(glr_handle* h, float* U_out, void* stream) {
-    if (!h || !U_out) return GLR_EINVAL;
-    cudaStream_t st = static_cast<cudaStream_t>(stream);
-    const size_t mp = h->mp;
-    if (h->exact) GLR_CK(h, cudaMemcpyAsync(U_out, h->U, 4 * mp * mp, cudaMemcpyDeviceToDevice, st));
-    else GLR_LAUNCH(h, 1, materialize_wy_basis(h->mp, h->k, h->Y, h->Yt, h->dsign, U_out, st));
-    return GLR_OK;
-}
-
-int glr_set_basis(glr_handle* h, const float* Q, void* stream) {
-    if (!h || !Q) return GLR_EINVAL;
-    cudaStream_t st = static_cast<cudaStream_t>(stream);
-    const size_t mp = h->mp, k = h->k;
-    if (h->exact) {
-        GLR_CK(h, cudaMemcpyAsync(h->U, Q, 4 * mp * mp, cudaMemcpyDeviceToDevice, st));
-    } else {
-        GLR_CK(h, cudaMemcpyAsync(h->Q, Q, 4 * mp * k, cudaMemcpyDeviceToDevice, st));
-        int rc = wy_from_Q(h, st);
-        if (rc != GLR_OK) return rc;
-    }
-    h->basis_from_user = true;
-    return GLR_OK;
-}
-
-int glr_profile_enable(glr_handle* h, int32_t enable) {
-    if (!h) return GLR_EINVAL;
-    h->prof = enable != 0;
-    return GLR_OK;
-}
-
-int glr_profile_read(glr_handle* h, glr_profile* out, int32_t reset) {
-    if (!h || !out) return GLR_EINVAL;
-    for (auto& rec : h->recs) {
-        GLR_CK(h, cudaEventSynchronize(rec.b));
-        float ms = 0.f;
-        GLR_CK(h, cudaEventElapsedTime(&ms, rec.a, rec.b));
-        h->prof_ms[rec.phase] += ms;
-        h->prof_launch[rec.phase] += rec.launches;
-        h->prof_count[rec.phase] += 1;
-        h->free_events.push_back(rec.a);
-        h->free_events.push_back(rec.b);
-    }
-    h->recs.clear();
-    for (int p = 0; p < GLR_PHASES; ++p) {
-        out->ms[p] = h->prof_ms[p];
-        out->launches[p] = h->prof_launch[p];
-        out->count[p] = h->prof_count[p];
-        if (reset) { h->prof_ms[p] = 0.0; h->prof_launch[p] = 0; h->prof_count[p] = 0; }
-    }
-    return GLR_OK;
-}
-
-int glr_force_selection(glr_handle* h, const int32_t* J_host) {
-    if (!h || !J_host) return GLR_EINVAL;
-    std::vector<int32_t> J(J_host, J_host + h->r);
-    std::sort(J.begin(), J.end());
-    for (int q = 0; q < h->r; ++q) {
-        if (J[q] < 0 || J[q] >= h->mp || (q && J[q] == J[q - 1]))
-            return fail(h, GLR_EINVAL, "forced selection must hold r distinct indices in [0, m')%s");
-    }
-    h->forceJ = J;
-    h->has_forceJ = true;
     return GLR_OK;
 }
 

@@ -1,0 +1,196 @@
+// The Semi-Lazy SVD refresh of Eq. SVD-P1 on the host side: the order of the refresh kernels for
+// a truncated basis (block power iteration with CholeskyQR, Rayleigh-Ritz, the Householder WY
+// form; grouped across matrices through k_power.cu when k <= 32) and for the full basis (the
+// cooperative Jacobi of all refreshing matrices, k_jacobi.cu).  Each handle's refresh runs on its
+// own side stream.
+#include "glr_host.cuh"
+
+namespace glr {
+namespace host {
+
+// A (rows x k, row-major) <- A L^{-T} with L L^T = A^T A (CholeskyQR): the k x k factor and its
+// inverse in one CTA, then one product into tmp; A and tmp trade places.
+int cholqr(glr_handle* h, float*& A, float*& tmp, int rows, cudaStream_t st) {
+    const int k = h->k;
+    GLR_GEMM(h, gd(k, k, rows, A, 1, k, A, k, 1, h->gram, k, 1), st);
+    if (k > 256) {                           // the factor does not fit one CTA's shared memory
+        GLR_LAUNCH(h, 1, cholesky(h->gram, k, h->scratch, h->dflags + 0, st));
+        GLR_LAUNCH(h, 1, trsm_right_lt(A, rows, k, h->gram, st));
+        return GLR_OK;
+    }
+    GLR_LAUNCH(h, 1, chol_inverse(h->gram, k, h->scratch, h->dflags + 0, st));
+    GLR_GEMM(h, gd(rows, k, k, A, k, 1, h->scratch, k, 1, tmp, k, 1), st);
+    std::swap(A, tmp);
+    return GLR_OK;
+}
+
+int wy_from_Q(glr_handle* h, cudaStream_t st) {
+    const int mp = h->mp, k = h->k;
+    GLR_LAUNCH(h, 2, householder_reconstruct(h->Q, mp, k, h->Y, h->T, h->dsign, h->scratch, st));
+    // Yt = Y T^T
+    GLR_GEMM(h, gd(mp, k, k, h->Y, k, 1, h->T, 1, k, h->Yt, k, 1), st);
+    // transposed copies (k x tp, zero-padded) for the fused compose kernel's lambda epilogue
+    GLR_LAUNCH(h, 1, transpose_pad(h->YT, transposed_pitch(mp), h->Y, mp, k, st));
+    GLR_LAUNCH(h, 1, transpose_pad(h->YtT, transposed_pitch(mp), h->Yt, mp, k, st));
+    if (h->mma) {
+        GLR_LAUNCH(h, 1, pack_frag(h->YF, h->Y, mp, k, k, 0, st));
+        GLR_LAUNCH(h, 1, pack_frag(h->YtF, h->Yt, mp, k, k, 1, st));
+    }
+    return GLR_OK;
+}
+
+// End of a truncated refresh, with Q orthonormal and H = Q^T Mbar Mbar^T Q in Hk: Rayleigh-Ritz
+// H = W diag W^T, Q <- Q W (columns by descending Ritz value, signs fixed), then the WY form.
+int refresh_tail(glr_handle* h, cudaStream_t st) {
+    const int mp = h->mp, k = h->k;
+    GLR_LAUNCH(h, 1, jacobi_eig(h->Hk, k, h->Vk, h->evals, h->dflags + 1, st));
+    GLR_LAUNCH(h, 1, sort_fix_basis(h->evals, h->Vk, k, k, h->gram, k, h->evals_sorted, st));
+    GLR_GEMM(h, gd(mp, k, k, h->Q, k, 1, h->gram, k, 1, h->Qn, k, 1), st);
+    GLR_LAUNCH(h, 1, fix_column_signs(h->Qn, mp, k, st));
+    std::swap(h->Q, h->Qn);
+    return wy_from_Q(h, st);
+}
+
+// Truncated refreshes of several matrices through the grouped block power iteration
+// (k_power.cu): the same iteration as do_refresh (q power iterations, each half re-normalised by
+// CholeskyQR, then CholeskyQR2 and the Rayleigh-Ritz Gram), one launch per stage for all of
+// them on the first handle's side stream; the k x k tails run on each handle's own stream.
+int refresh_grouped(std::vector<glr_handle*>& hs) {
+    glr_handle* h0 = hs[0];
+    cudaStream_t s0 = h0->rstream;
+    for (glr_handle* h : hs) GLR_CK(h0, cudaStreamWaitEvent(s0, h->rfork, 0));
+    {
+        PhaseScope ps(h0, GLR_PH_REFRESH, s0);
+        PowGroup g{};
+        const int PC = pow_tile(), CH = pow_chunk();
+        int q = h0->s.power_iters;
+        for (glr_handle* h : hs) {
+            if (h->refreshes == 0 && !h->basis_from_user)
+                GLR_LAUNCH(h0, 1, random_block(h->Q, h->mp, h->k, h->s.seed, static_cast<uint32_t>(h->t), s0));
+            PowMat& M = g.mat[g.nmat++];
+            M.mp = h->mp; M.np = h->np; M.k = h->k; M.active = 1;
+            M.t0 = g.tot_t; M.nt = (h->np + PC - 1) / PC; g.tot_t += M.nt;
+            M.r0 = g.tot_r; M.nr = (h->mp + PC - 1) / PC; g.tot_r += M.nr;
+            M.n0 = g.tot_n; M.nn = (h->np + CH - 1) / CH; g.tot_n += M.nn * M.nr;
+            M.Mbar = h->Mbar; M.Q = h->Q; M.Z = h->Z; M.part = h->powpart; M.G = h->powG; M.S = h->powS;
+            M.H = h->Hk; M.flag = h->dflags + 0;
+            q = std::max(q, h->s.power_iters);
+        }
+        // a matrix with fewer power iterations than the group's maximum drops out early
+        for (int it = 0; it < q; ++it) {
+            for (int i = 0; i < g.nmat; ++i) g.mat[i].active = it < hs[i]->s.power_iters ? 1 : 0;
+            GLR_LAUNCH(h0, 1, pow_stage(g, 0, it > 0 ? 1 : 0, s0));   // Z = (Mbar^T Q) S
+            GLR_LAUNCH(h0, 1, pow_stage(g, 4, 1, s0));                // S = chol(Z^T Z)^-T
+            GLR_LAUNCH(h0, 1, pow_stage(g, 1, 0, s0));                // partials of Mbar Z
+            GLR_LAUNCH(h0, 1, pow_stage(g, 2, 0, s0));                // Q = (Mbar Z) S
+            GLR_LAUNCH(h0, 1, pow_stage(g, 4, 0, s0));                // S = chol(Q^T Q)^-T
+        }
+        for (int i = 0; i < g.nmat; ++i) g.mat[i].active = 1;
+        GLR_LAUNCH(h0, 1, pow_stage(g, 3, 1, s0));                    // CholeskyQR2: Q <- Q S ...
+        GLR_LAUNCH(h0, 1, pow_stage(g, 4, 0, s0));
+        GLR_LAUNCH(h0, 1, pow_stage(g, 3, 0, s0));                    // ... twice: orthonormal
+        GLR_LAUNCH(h0, 1, pow_stage(g, 0, 0, s0));                    // Rayleigh-Ritz: Z = Mbar^T Q
+        GLR_LAUNCH(h0, 1, pow_stage(g, 5, 1, s0));                    // H = Z^T Z
+    }
+    GLR_CK(h0, cudaEventRecord(h0->rpow, s0));
+    for (glr_handle* h : hs) {
+        if (h != h0) GLR_CK(h, cudaStreamWaitEvent(h->rstream, h0->rpow, 0));
+        PhaseScope ps(h, GLR_PH_REFRESH, h->rstream);
+        g_ws = h->gemm_ws;
+        const int rc = refresh_tail(h, h->rstream);
+        g_ws = nullptr;
+        if (rc != GLR_OK) return rc;
+    }
+    return GLR_OK;
+}
+
+// Full-basis refreshes of several matrices: H = Mbar Mbar^T on each handle's side stream, one
+// cooperative Jacobi launch for all of them on the first handle's side stream (k_jacobi.cu), then
+// each handle sorts its eigenvectors by descending eigenvalue and fixes their signs on its own.
+int refresh_exact_grouped(std::vector<glr_handle*>& hs) {
+    const int grid = jacobi_group_grid();
+    for (size_t c0 = 0, c1 = 0; c0 < hs.size(); c0 = c1) {
+        // a group: at most kGroupMax matrices whose rotations fit the kernel's shared memory
+        size_t rot = 0;
+        for (c1 = c0; c1 < hs.size() && c1 - c0 < (size_t)kGroupMax; ++c1) {
+            const size_t add = jacobi_rot_floats(hs[c1]->mp) * sizeof(float);
+            if (c1 > c0 && rot + add > kJacobiMaxSmem) break;
+            rot += add;
+        }
+        glr_handle* h0 = hs[c0];
+        cudaStream_t s0 = h0->rstream;
+        for (size_t i = c0; i < c1; ++i) {
+            glr_handle* h = hs[i];
+            PhaseScope ps(h, GLR_PH_REFRESH, h->rstream);
+            const int mp = h->mp, np = h->np;
+            GLR_GEMM(h, gd(mp, mp, np, h->Mbar, np, 1, h->Mbar, 1, np, h->Hbuf, mp, 1), h->rstream);
+            if (!grid) {                                         // no cooperative launch: one CTA each
+                GLR_LAUNCH(h, 1, jacobi_eig(h->Hbuf, mp, h->Vbuf, h->evals, h->dflags + 1, h->rstream));
+                GLR_LAUNCH(h, 1, sort_fix_basis(h->evals, h->Vbuf, mp, mp, h->U, mp, h->evals_sorted, h->rstream));
+                continue;
+            }
+            GLR_CK(h, cudaEventRecord(h->rpow, h->rstream));
+            if (h != h0) GLR_CK(h0, cudaStreamWaitEvent(s0, h->rpow, 0));
+        }
+        if (!grid) continue;
+        JacobiGroup g{};
+        size_t soff = 0;
+        g.max_sweeps = 40;
+        g.bar = h0->dflags + 4; g.err = h0->dflags + 2; g.part = h0->jpart;
+        for (size_t i = c0; i < c1; ++i) {
+            glr_handle* h = hs[i];
+            JacobiMat& M = g.mat[g.nmat++];
+            const int n = h->mp;
+            M.n = n; M.tol = 4.f * 5.96e-8f * sqrtf(static_cast<float>(n)) + 1e-7f;
+            M.H = h->Hbuf; M.H2 = h->jwork; M.V = h->Vbuf; M.evals = h->evals;
+            M.sweeps = h->dflags + 1;
+            M.soff = (int)soff;
+            soff += jacobi_rot_floats(n);
+        }
+        {
+            PhaseScope ps(h0, GLR_PH_REFRESH, s0);
+            GLR_LAUNCH(h0, 1, jacobi_group(g, grid, s0));
+        }
+        GLR_CK(h0, cudaEventRecord(h0->rpow, s0));
+        for (size_t i = c0; i < c1; ++i) {
+            glr_handle* h = hs[i];
+            if (h != h0) GLR_CK(h, cudaStreamWaitEvent(h->rstream, h0->rpow, 0));
+            PhaseScope ps(h, GLR_PH_REFRESH, h->rstream);
+            GLR_LAUNCH(h, 1, sort_fix_basis(h->evals, h->Vbuf, h->mp, h->mp, h->U, h->mp, h->evals_sorted, h->rstream));
+        }
+    }
+    return GLR_OK;
+}
+
+// Semi-Lazy SVD refresh (Eq. SVD-P1) from Mbar.
+int do_refresh(glr_handle* h, cudaStream_t st) {
+    const int mp = h->mp, np = h->np, k = h->k;
+    g_ws = h->gemm_ws;
+    struct Reset { ~Reset() { g_ws = nullptr; } } reset_ws;
+    if (h->exact) {
+        // H = Mbar Mbar^T, eigenvectors = left singular vectors, sorted by descending sigma
+        GLR_GEMM(h, gd(mp, mp, np, h->Mbar, np, 1, h->Mbar, 1, np, h->Hbuf, mp, 1), st);
+        GLR_LAUNCH(h, 1, jacobi_eig(h->Hbuf, mp, h->Vbuf, h->evals, h->dflags + 1, st));
+        GLR_LAUNCH(h, 1, sort_fix_basis(h->evals, h->Vbuf, mp, mp, h->U, mp, h->evals_sorted, st));
+        return GLR_OK;
+    }
+    if (h->refreshes == 0 && !h->basis_from_user)
+        GLR_LAUNCH(h, 1, random_block(h->Q, mp, k, h->s.seed, static_cast<uint32_t>(h->t), st));
+    int rc;
+    for (int it = 0; it < h->s.power_iters; ++it) {
+        // Z = Mbar^T Q (n' x k) and Q = Mbar Z (m' x k), each re-orthonormalised by CholeskyQR
+        // (one pass keeps the block well conditioned; the span is what the iteration needs)
+        GLR_GEMM(h, gd(np, k, mp, h->Mbar, 1, np, h->Q, k, 1, h->Z, k, 1), st);
+        if ((rc = cholqr(h, h->Z, h->Zn, np, st)) != GLR_OK) return rc;
+        GLR_GEMM(h, gd(mp, k, np, h->Mbar, np, 1, h->Z, k, 1, h->Q, k, 1), st);
+        if ((rc = cholqr(h, h->Q, h->Qn, mp, st)) != GLR_OK) return rc;
+    }
+    if ((rc = cholqr(h, h->Q, h->Qn, mp, st)) != GLR_OK) return rc;   // CholeskyQR2: orthonormal to rounding
+    // Rayleigh-Ritz: Z = Mbar^T Q, H = Z^T Z = Q^T Mbar Mbar^T Q
+    GLR_GEMM(h, gd(np, k, mp, h->Mbar, 1, np, h->Q, k, 1, h->Z, k, 1), st);
+    GLR_GEMM(h, gd(k, k, np, h->Z, 1, k, h->Z, k, 1, h->Hk, k, 1), st);
+    return refresh_tail(h, st);
+}
+
+}  // namespace host
+}  // namespace glr
