@@ -561,3 +561,28 @@ def test_algorithm5_rejects_other_schedules():
         args.update(kw)
         with pytest.raises(ValueError):
             O.GreedyLoreOracle(6, 8, 2, 2, 3, optimizer="galore_adam", **args)
+
+
+@pytest.mark.parametrize("m,n,N,mode,opt", [(1, 5, 3, "alg3", "msgd"), (4, 9, 2, "alg4", "msgd"), (9, 4, 3, "alg3", "adam"),
+                                             (5, 5, 1, "alg4", "adam"), (6, 11, 4, "alg3", "msgd")])
+def test_full_rank_selection_is_uncompressed_data_parallel(m, n, N, mode, opt):
+    """r = m': P is square and orthogonal, so P P^T = I, every E_i stays 0 and Ghat is the plain node
+    mean: GreedyLore reduces to data-parallel MSGD / Adam on the mean gradient (m' = 1, square,
+    transposed and N = 1 cases included)."""
+    rng = np.random.default_rng(41 + m + n)
+    r = min(m, n)
+    kw = dict(lr=0.03, beta1=0.8, beta2=0.95, eps=1e-6, optimizer=opt)
+    orc = O.GreedyLoreOracle(m, n, r, N, 3, refresh_mode=mode, seed=2, **kw)
+    X = rng.standard_normal((m, n))
+    Xe = X.copy()
+    Mo, Vo = np.zeros((m, n)), np.zeros((m, n))
+    for t in range(7):
+        G = rng.standard_normal((N, m, n))
+        X, info = orc.step(G, X)
+        Gbar = G.mean(axis=0)
+        if opt == "msgd":
+            Xe, Mo = O.msgd_update(Xe, Mo, Gbar, kw["lr"], kw["beta1"])
+        else:
+            Xe, Mo, Vo = O.adam_update(Xe, Mo, Vo, Gbar, kw["lr"], kw["beta1"], kw["beta2"], kw["eps"])
+        assert np.abs(info.E).max() < 1e-12
+        np.testing.assert_allclose(X, Xe, rtol=1e-10, atol=1e-12)
