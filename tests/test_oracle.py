@@ -586,3 +586,26 @@ def test_full_rank_selection_is_uncompressed_data_parallel(m, n, N, mode, opt):
             Xe, Mo, Vo = O.adam_update(Xe, Mo, Vo, Gbar, kw["lr"], kw["beta1"], kw["beta2"], kw["eps"])
         assert np.abs(info.E).max() < 1e-12
         np.testing.assert_allclose(X, Xe, rtol=1e-10, atol=1e-12)
+
+
+def test_compress_start_warmup_is_uncompressed_then_refreshes():
+    """Appendix F warm-up: the first K steps use the plain node mean with no error feedback
+    (data-parallel MSGD), step K is the first refresh and the refreshes then follow every tau
+    steps from there."""
+    rng = np.random.default_rng(47)
+    m, n, r, N, tau, K, lr, beta = 5, 8, 2, 3, 4, 3, 0.05, 0.7
+    orc = O.GreedyLoreOracle(m, n, r, N, tau, seed=3, lr=lr, beta1=beta, compress_start=K)
+    X = rng.standard_normal((m, n))
+    Xe, Mo = X.copy(), np.zeros((m, n))
+    refreshes = []
+    for t in range(K + 2 * tau + 1):
+        G = rng.standard_normal((N, m, n))
+        X, info = orc.step(G, X)
+        if info.refresh:
+            refreshes.append(t)
+        if t < K:
+            assert not info.compressed and not info.refresh
+            assert np.all(info.E == 0)
+            Xe, Mo = O.msgd_update(Xe, Mo, G.mean(axis=0), lr, beta)
+            np.testing.assert_allclose(X, Xe, rtol=1e-12, atol=1e-14)
+    assert refreshes == [K, K + tau, K + 2 * tau]
