@@ -46,6 +46,25 @@ def _peaks():
     return 6800.0, "fallback"
 
 
+def tensor_peak_tflops():
+    """The measured sustained dense bf16 tensor rate (the refresh runs inside a long step), else
+    the fallback figure."""
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(path):
+        with open(path) as f:
+            p = json.load(f)
+        if "bf16_tflops_sustained" in p:
+            return float(p["bf16_tflops_sustained"]), "measured"
+    return 1700.0, "fallback"
+
+
+def refresh_flops(cfg, basis_rank):
+    """Algorithmic flops of one truncated-basis refresh of every matrix: q block power iterations,
+    each a pass of Mbar^T Q and of Mbar Z (2 m' n' k flops apiece), and the Rayleigh-Ritz pass
+    (2 m' n' k); the k x k work is negligible beside them."""
+    return sum((2 * cfg.power_iters + 1) * 2 * min(m, n) * max(m, n) * basis_rank for (m, n) in cfg.shapes)
+
+
 def algorithmic_bytes(cfg, e_zero: bool):
     """Bytes a GreedyLore step must move: per node-element G (gsize) + E read/write (8 B; no
     read after an error reset); per matrix element the optimizer state (MSGD 16 B, Adam 24 B)."""
@@ -431,6 +450,13 @@ def main():
         "refresh_ms_all_matrices": refresh_extra_ms,
         "refresh_wall_ms_per_step": (refresh_extra_ms * main_run["refreshes"] / K) if refresh_extra_ms else None,
         "refresh_ms_per_layer": refresh_extra_ms / len(cfg.shapes) if refresh_extra_ms else None,
+        "refresh_tensor": None if not refresh_extra_ms else {
+            "flops": refresh_flops(cfg, cfg.basis_rank),
+            "tflops": refresh_flops(cfg, cfg.basis_rank) / (refresh_extra_ms / 1e3) / 1e12,
+            "frac_of_tensor_peak": refresh_flops(cfg, cfg.basis_rank) / (refresh_extra_ms / 1e3) / 1e12
+                                   / tensor_peak_tflops()[0],
+            "peak": tensor_peak_tflops()[0], "peak_kind": tensor_peak_tflops()[1] + " bf16 sustained",
+            "note": "the truncated refresh runs on the FP32 pipes; bound by HBM and latency, not the tensor cores"},
         "phases_ms_per_step": {k: v["ms"] / K for k, v in ph.items()},
         "phases_note": "refresh = summed event time of the concurrent per-matrix refresh streams",
         "phase_launches": {k: v["launches"] for k, v in ph.items()},

@@ -79,3 +79,14 @@ def test_reference_arm_other_ranks_exit_without_work(monkeypatch):
     with redirect_stdout(buf):
         assert bench.run_reference(Args()) == 0
     assert buf.getvalue() == ""
+
+
+def test_refresh_flops_and_tensor_peak():
+    sys.path.insert(0, ROOT)
+    import bench
+    import workloads as W
+    cfg = W.config("cfg2_resnet")
+    # (2 q + 1) passes of 2 m' n' k flops over the stack's 6,266,880 matrix elements, q = 4, k = 16
+    assert bench.refresh_flops(cfg, 16) == 9 * 2 * 6_266_880 * 16
+    peak, kind = bench.tensor_peak_tflops()
+    assert peak > 100 and kind in ("measured", "fallback")
