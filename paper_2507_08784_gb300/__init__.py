@@ -18,8 +18,8 @@ from . import _lib
 from ._lib import (GLR_ADAM, GLR_ADAMW, GLR_ALG3, GLR_ALG4, GLR_AMSGRAD, GLR_BF16, GLR_F32,  # noqa: F401
                    GLR_GALORE_ADAM, GLR_MSGD, GLR_OK, PHASE_NAMES, GlrProfile, GlrSchedule, GlrStats, load)
 
-__all__ = ["GlrError", "make_schedule", "glr_create", "glr_destroy", "glr_step", "glr_step_group", "glr_step_group_host", "glr_step_host", "glr_save", "glr_load",
-           "glr_refresh", "glr_get_stats", "glr_last_error", "glr_get_error", "glr_get_selection",
+__all__ = ["GlrError", "make_schedule", "glr_create", "glr_destroy", "glr_step", "glr_step_group",
+           "glr_step_group_host", "glr_step_host", "glr_save", "glr_load", "glr_refresh", "glr_get_stats", "glr_last_error", "glr_get_error", "glr_get_selection",
            "glr_get_basis", "glr_set_basis", "glr_force_selection", "glr_profile_enable",
            "glr_profile_read", "glr_select_noalloc", "GreedyLore", "load"]
 
@@ -58,6 +58,24 @@ def make_schedule(tau: int, refresh_mode: str = "alg3", optimizer: str = "msgd",
                   basis_rank: int = 0, power_iters: int = 4, grad_dtype: str = "f32",
                   compress_start: int = 0, error_feedback: bool = True, selection: str = "approx",
                   weight_decay: float = 0.0) -> GlrSchedule:
+    """The glr_schedule of include/glr.h from keyword arguments.
+
+    tau            refresh period of the Semi-Lazy SVD (>= 1)
+    refresh_mode   "alg3" (refresh step uses the uncompressed mean and resets E) or "alg4"
+                   (the refresh step is compressed with P = U[:, :r], E kept)
+    optimizer      "msgd" (Eq. msgd), "adam" (Eq. adam), "amsgrad" (the analysis' AMSGrad-type
+                   rule), "adamw" (bias-corrected, decoupled weight_decay) or "galore_adam"
+                   (Algorithm 5: needs refresh_mode "alg4", selection "fixed",
+                   error_feedback False); lr, beta1, beta2, eps as in those equations
+    seed           key of the shared random vectors v_j (give every matrix its own)
+    basis_rank     0: the full singular basis (paper-exact, min(m, n) <= 1024); r..512: the top-k
+                   singular vectors completed by Householder reflectors, refreshed with
+                   power_iters block power iterations
+    grad_dtype     "f32" or "bf16" (the gradients' storage type)
+    compress_start the first compress_start steps run uncompressed (Appendix F warm-up)
+    error_feedback False drops error feedback (with selection "fixed": Algorithm 1)
+    selection      "approx" (Algorithm 2) or "fixed" (P = U[:, :r] for the whole period)
+    """
     return GlrSchedule(tau=tau, refresh_mode={"alg3": GLR_ALG3, "alg4": GLR_ALG4}[refresh_mode],
                        optimizer=_OPTIMIZERS[optimizer], lr=lr, beta1=beta1,
                        beta2=beta2, eps=eps, seed=seed & (2 ** 64 - 1), basis_rank=basis_rank,
@@ -195,7 +213,12 @@ def glr_select_noalloc(U: torch.Tensor, Mbar: torch.Tensor, seed: int, t: int, r
 
 
 class GreedyLore:
-    """One layer matrix's GreedyLore state (owns a glr handle)."""
+    """One layer matrix's GreedyLore state for N simulated nodes (owns a glr handle).
+
+    GreedyLore(m, n, r, N, **schedule) with the keywords of make_schedule; step(G, X) runs one
+    iteration on the N device gradients G (m x n, the schedule's dtype) and updates the device
+    weights X (m x n float32) in place.  close() frees the device state.
+    """
 
     def __init__(self, m: int, n: int, r: int, N: int, **schedule):
         self.m, self.n, self.r, self.N = m, n, r, N
