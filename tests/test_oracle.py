@@ -609,3 +609,27 @@ def test_compress_start_warmup_is_uncompressed_then_refreshes():
             Xe, Mo = O.msgd_update(Xe, Mo, G.mean(axis=0), lr, beta)
             np.testing.assert_allclose(X, Xe, rtol=1e-12, atol=1e-14)
     assert refreshes == [K, K + tau, K + 2 * tau]
+
+
+def test_lemma2_holds_for_the_truncated_basis():
+    """The truncated-basis reading keeps Lemma 2: its U (top-k singular vectors of an earlier
+    refresh matrix, completed by Householder reflectors) is orthogonal, which is all the lemma
+    uses, so Approx-Top-r on it contracts E||Gbar - P P^T Gbar||^2 <= (1 - r/m) ||Gbar||^2 even
+    though U was computed from a different (stale) matrix."""
+    rng = np.random.default_rng(23)
+    m, n, N, r, k = 8, 10, 2, 2, 3
+    stale = rng.standard_normal((m, n)) * np.linspace(2, 0.5, m)[:, None]
+    Uk, _ = O.left_singular_basis(stale)
+    U = O.householder_complement(Uk[:, :k])
+    np.testing.assert_allclose(U.T @ U, np.eye(m), atol=1e-12)
+    Ms = rng.standard_normal((N, m, n)) * np.linspace(3, 0.2, m)[None, :, None]
+    Gbar = Ms.mean(0)
+    T = 4000
+    errs = np.empty(T)
+    for t in range(T):
+        V = O.gaussian_v(4343, t, m, n)
+        J = O.argtop_r(O.approx_top_r_lambda(list(Ms), U, V) ** 2, r)
+        P = U[:, J]
+        errs[t] = np.linalg.norm(Gbar - P @ P.T @ Gbar) ** 2
+    bound = (1 - r / m) * np.linalg.norm(Gbar) ** 2
+    assert errs.mean() <= bound + 5 * errs.std() / math.sqrt(T)
