@@ -89,6 +89,25 @@ bool encode_strip_map(CUtensorMap* map, const void* base, int rows, int cols, in
               CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+bool encode_map(CUtensorMap* map, CUtensorMapDataType dtype, const void* base, int rank, const uint64_t* dims,
+                const uint64_t* strides, const uint32_t* box, CUtensorMapSwizzle swz) {
+    EncodeTiledFn fn = encode_fn();
+    if (!fn) return false;
+    cuuint64_t d[3], s[2];
+    cuuint32_t b[3], e[3] = {1, 1, 1};
+    for (int i = 0; i < rank; ++i) { d[i] = dims[i]; b[i] = box[i]; }
+    for (int i = 0; i + 1 < rank; ++i) s[i] = strides[i];
+    return fn(map, dtype, rank, const_cast<void*>(base), d, s, b, e, CU_TENSOR_MAP_INTERLEAVE_NONE, swz,
+              CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+// fp32 operand of the tcgen05 path: `rank` dims (innermost first), byte strides of dims 1..,
+// box {32, box[1], 1}, 128-byte swizzle, out-of-range elements read as zero.
+bool encode_f32_map(CUtensorMap* map, const float* base, int rank, const uint64_t* dims, const uint64_t* strides,
+                    const uint32_t* box) {
+    return encode_map(map, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, base, rank, dims, strides, box, CU_TENSOR_MAP_SWIZZLE_128B);
+}
+
 // The descriptor of node i's gradient buffer, re-encoded only when the buffer changes.
 bool gradient_map(glr_handle* h, int i, const void* ptr, CUtensorMap* out) {
     glr_handle::GMap* slots = &h->gmaps[2 * (size_t)i];
@@ -319,7 +338,9 @@ int glr_create(int64_t m, int64_t n, int32_t r, int32_t N, const glr_schedule* s
     h->s = *s; h->gsize = s->grad_dtype == GLR_BF16 ? 2 : 4;
     h->period_start = s->compress_start;
     h->ntiles = static_cast<int>((np + kLambdaTile - 1) / kLambdaTile);
-    {
+    // the tcgen05 path (k_tc.cu) takes the matrices it can; the strip kernels the rest
+    h->tcl = tcl_eligible(mp, np, r, N, k, exact, s) ? 1 : 0;
+    if (!h->tcl) {
         // The fused strip kernels keep a whole m' x BN strip (and P) in shared memory and move
         // rows in 16-byte vectors: they need m' <= 2048, rows of a multiple of 4 elements and
         // room for P.
@@ -344,18 +365,19 @@ int glr_create(int64_t m, int64_t n, int32_t r, int32_t N, const glr_schedule* s
         }
     }
     cudaGetDevice(&h->device);
+    const int rpad_tc = (r + 31) & ~31;
     int rc = GLR_OK;
     const size_t MP = mp, NP = np;
     auto A = [&](auto** p, size_t cnt) { if (rc == GLR_OK) rc = alloc(h, p, cnt); };
     A(&h->B, (size_t)N * MP * NP);
     A(&h->Mbar, MP * NP);
-    A(&h->Rw, (size_t)N * r * NP);
+    A(&h->Rw, (size_t)N * (h->tcl ? rpad_tc : r) * NP);
     A(&h->Rbar, (size_t)r * NP);
     A(&h->P, MP * r);
     A(&h->Pprev, MP * r);
     A(&h->J, (size_t)r);
     A(&h->lam, MP);
-    A(&h->lam_part, MP * std::max(h->ntiles, h->nstrips));
+    A(&h->lam_part, MP * std::max(std::max(h->ntiles, h->nstrips), 2 * ((h->np + 127) / 128)));
     const bool galore = s->optimizer == GLR_GALORE_ADAM;
     A(&h->Mo, galore ? (size_t)r * NP : (size_t)m * n);
     if (s->optimizer != GLR_MSGD) A(&h->Vo, galore ? (size_t)r * NP : (size_t)m * n);
@@ -364,9 +386,10 @@ int glr_create(int64_t m, int64_t n, int32_t r, int32_t N, const glr_schedule* s
     A(&h->dflags, 6);
     A(&h->gemm_ws, (size_t)kGemmWsFloats);
     // the first path with library products when the rank-r products are large
-    h->tc = !h->fused && mp % 4 == 0 && np % 4 == 0 && 2.0 * r * (double)mp * (double)np * N >= 67108864.0 ? 1 : 0;
+    h->tc = !h->fused && !h->tcl && mp % 4 == 0 && np % 4 == 0 &&
+            2.0 * r * (double)mp * (double)np * N >= 67108864.0 ? 1 : 0;
     if (h->tc || separate_optimizer(h)) A(&h->mn_scratch, MP * NP);
-    if (h->tc && !exact) A(&h->YtJ, (size_t)r * k);
+    if ((h->tc || h->tcl) && !exact) A(&h->YtJ, (size_t)r * k);
     if (exact) {
         A(&h->jwork, MP * MP);
         A(&h->jpart, (size_t)2 * kGroupMax * kJacobiMaxGrid);
@@ -384,7 +407,7 @@ int glr_create(int64_t m, int64_t n, int32_t r, int32_t N, const glr_schedule* s
             const size_t frag = ((MP + 7) & ~size_t(7)) * ((K + 7) & ~size_t(7));
             A(&h->YF, frag); A(&h->YtF, frag);
         }
-        if (k <= 32 && np % 4 == 0) {          // grouped power iteration (k_power.cu)
+        if (k <= 32 && np % 4 == 0 && !h->tcl) {   // grouped power iteration (k_power.cu), row-major Mbar
             const size_t KM = k <= 16 ? 16 : 32, PC = pow_tile(), CH = pow_chunk();
             const size_t nt = (NP + PC - 1) / PC, nr = (MP + PC - 1) / PC, nn = (NP + CH - 1) / CH;
             A(&h->powpart, nn * KM * MP);
@@ -393,6 +416,7 @@ int glr_create(int64_t m, int64_t n, int32_t r, int32_t N, const glr_schedule* s
             h->pow_ok = 1;
         }
     }
+    if (rc == GLR_OK && h->tcl) rc = tcl_alloc(h);
     if (rc != GLR_OK) {
         g_create_err = h->err;
         free_all(h);
@@ -431,6 +455,11 @@ int glr_create(int64_t m, int64_t n, int32_t r, int32_t N, const glr_schedule* s
     h->iotaJ.resize(r);
     for (int q = 0; q < r; ++q) h->iotaJ[q] = q;
     h->n_state_allocs = h->allocs.size();
+    if (h->tcl && (rc = tcl_maps(h)) != GLR_OK) {
+        g_create_err = h->err;
+        glr_destroy(h);
+        return rc;
+    }
     *out = h;
     return GLR_OK;
 }
@@ -652,6 +681,155 @@ int update_fused(std::vector<StepPlan*>& plans, cudaStream_t st) {
     return GLR_OK;
 }
 
+// ---- the tcgen05 path (k_tc.cu) -------------------------------------------------------------
+// Every op is one grouped launch over the matrices that take part in it (kTcGroupMax per launch).
+tc::TcMat tc_mat(const glr_handle* h) {
+    tc::TcMat M{};
+    M.mp = h->mp; M.np = h->np; M.N = h->N; M.r = h->r; M.rpad = h->rpad; M.k = h->k; M.kpad = h->kpad;
+    M.transposed = h->transposed; M.gdtype = h->s.grad_dtype;
+    M.seed = h->s.seed; M.t = static_cast<uint32_t>(h->t);
+    return M;
+}
+inline int cdiv(int a, int b) { return (a + b - 1) / b; }
+
+// fill(plan, M, g, first) describes the plan's matrix for the op: 1 = take it, 0 = the plan has
+// no part in this op, -1 = it needs another launch (its optimizer settings differ), -2 = failure
+// (recorded on the plan's handle).
+template <class Fill>
+int tc_run(std::vector<StepPlan*> plans, int phase, cudaError_t (*launch)(tc::TcGroup&, cudaStream_t), cudaStream_t st,
+           Fill fill) {
+    static thread_local tc::TcGroup g;
+    while (!plans.empty()) {
+        g.nmat = 0; g.total_tiles = 0; g.err = nullptr;
+        int gptrs = 0;
+        glr_handle* h0 = nullptr;
+        std::vector<StepPlan*> rest;
+        for (StepPlan* p : plans) {
+            glr_handle* h = p->h;
+            if (g.nmat == tc::kTcGroupMax || gptrs + h->N > tc::kTcGPtrs) { rest.push_back(p); continue; }
+            tc::TcMat M = tc_mat(h);
+            const int take = fill(*p, M, g, h0 == nullptr);
+            if (take == -2) return GLR_ECUDA;         // the fill recorded the failure on h
+            if (take == 0) continue;
+            if (take < 0) { rest.push_back(p); continue; }
+            if (!h0) { h0 = h; g.err = h->dflags + 2; }
+            M.tile0 = g.total_tiles;
+            g.total_tiles += M.ntiles;
+            M.g_off = gptrs;
+            for (int i = 0; i < h->N; ++i) g.G[gptrs + i] = p->G[i];
+            gptrs += h->N;
+            g.mat[g.nmat++] = M;
+        }
+        if (h0 && g.total_tiles > 0) {
+            PhaseScope ps(h0, phase, st);
+            GLR_LAUNCH(h0, 1, launch(g, st));
+        }
+        plans.swap(rest);
+    }
+    return GLR_OK;
+}
+
+bool tc_needs_lambda(const StepPlan& p) { return p.compressed && !p.refresh && !p.forced && !p.fixed; }
+
+// K1: R_w,i^T = (P_prev^T B_i)^T for matrices with a live error, then the compose pass.
+int tcl_compose(std::vector<StepPlan*>& plans, cudaStream_t st) {
+    int rc = tc_run(plans, GLR_PH_PREV_PROJECT, tc::launch_prevproj, st, [](StepPlan& p, tc::TcMat& M, tc::TcGroup&, bool) {
+        glr_handle* h = p.h;
+        if (h->e_zero) return 0;
+        M.na = h->tc_na; M.ng = h->tc_ng; M.tn = cdiv(h->np, 128); M.ntiles = M.tn * M.ng;
+        M.mA = tcl_map(h, kMapBt); M.mB = tcl_map_PT(h, h->Pprev); M.Rw = h->Rw;
+        return 1;
+    });
+    if (rc != GLR_OK) return rc;
+    return tc_run(plans, GLR_PH_COMPOSE, tc::launch_compose, st, [st](StepPlan& p, tc::TcMat& M, tc::TcGroup&, bool) {
+        glr_handle* h = p.h;
+        M.e_zero = h->e_zero ? 1 : 0;
+        M.write_B = (p.warm || h->s.no_error_feedback) ? 0 : 1;
+        M.tm = cdiv(h->mp, 128); M.tn = cdiv(h->np, tc::compose_bn()); M.ntiles = M.tm * M.tn;
+        M.mA = tcl_map_P(h, h->Pprev); M.mB = tcl_map(h, kMapRwT);
+        int rc = GLR_OK;
+        M.mD0 = tcl_map(h, kMapBtD);
+        M.mD1 = tcl_grad_maps(h, p.G, st, &rc);
+        if (rc != GLR_OK) return -2;
+        M.B = h->B; M.Mbar = h->Mbar;
+        return 1;
+    });
+}
+
+auto tc_wbar_fill(bool lam_plans) {
+    return [lam_plans](StepPlan& p, tc::TcMat& M, tc::TcGroup&, bool) {
+        glr_handle* h = p.h;
+        if (!p.compressed || tc_needs_lambda(p) != lam_plans) return 0;
+        M.ntiles = cdiv(h->np, 256);
+        M.mA = tcl_map(h, kMapMbarT); M.mB = tcl_map(h, kMapYT); M.W = h->WT;
+        return 1;
+    };
+}
+
+// Approx-Top-r partials for the matrices that select this step: W = Y^T Mbar, then the scores.
+int tcl_lambda(std::vector<StepPlan*>& plans, cudaStream_t st) {
+    int rc = tc_run(plans, GLR_PH_LAMBDA, tc::launch_wbar, st, tc_wbar_fill(true));
+    if (rc != GLR_OK) return rc;
+    return tc_run(plans, GLR_PH_LAMBDA, tc::launch_lambda, st, [](StepPlan& p, tc::TcMat& M, tc::TcGroup&, bool) {
+        glr_handle* h = p.h;
+        if (!tc_needs_lambda(p)) return 0;
+        M.tm = cdiv(h->mp, 128); M.tn = cdiv(h->np, 128); M.ntiles = M.tm * M.tn;
+        M.mA = tcl_map(h, kMapYt); M.mB = tcl_map(h, kMapWT); M.mD0 = tcl_map(h, kMapMbarL);
+        M.Mbar = h->Mbar; M.part = h->lam_part;
+        return 1;
+    });
+}
+
+// After J: W for the matrices that did not select (a supplied J, or the refresh of Algorithm 4),
+// P = U[:, J] (and P^T), Rbar, then the update pass for every matrix.
+int tcl_project_update(std::vector<StepPlan*>& plans, cudaStream_t st) {
+    int rc = tc_run(plans, GLR_PH_PROJECT, tc::launch_wbar, st, tc_wbar_fill(false));
+    if (rc != GLR_OK) return rc;
+    for (StepPlan* p : plans) {
+        if (!p->compressed) continue;
+        glr_handle* h = p->h;
+        PhaseScope ps(h, GLR_PH_SELECT, st);
+        GLR_LAUNCH(h, 1, wy_columns_gather(h->Yt, h->J, h->r, h->k, h->YtJ, st));
+    }
+    rc = tc_run(plans, GLR_PH_SELECT, tc::launch_pbuild, st, [](StepPlan& p, tc::TcMat& M, tc::TcGroup&, bool) {
+        glr_handle* h = p.h;
+        if (!p.compressed) return 0;
+        M.ntiles = cdiv(h->mp, 128);
+        M.mA = tcl_map(h, kMapY); M.mB = tcl_map(h, kMapYtJn);
+        M.J = h->J; M.dsign = h->dsign; M.Pout = h->P; M.PT = tcl_PT_of(h, h->P);
+        return 1;
+    });
+    if (rc != GLR_OK) return rc;
+    rc = tc_run(plans, GLR_PH_PROJECT, tc::launch_rbar, st, [](StepPlan& p, tc::TcMat& M, tc::TcGroup&, bool) {
+        glr_handle* h = p.h;
+        if (!p.compressed) return 0;
+        M.ntiles = cdiv(h->np, 128);
+        M.mA = tcl_map(h, kMapYtJm); M.mB = tcl_map(h, kMapWT);
+        M.J = h->J; M.dsign = h->dsign; M.Mbar = h->Mbar; M.Rbar = h->Rbar; M.RbarT = h->RbarT;
+        return 1;
+    });
+    if (rc != GLR_OK) return rc;
+    return tc_run(plans, GLR_PH_UPDATE, tc::launch_update, st, [st](StepPlan& p, tc::TcMat& M, tc::TcGroup& g, bool first) {
+        glr_handle* h = p.h;
+        const glr_schedule& s = h->s;
+        if (first) {
+            g.optimizer = s.optimizer; g.lr = s.lr; g.beta1 = s.beta1; g.beta2 = s.beta2; g.eps = s.eps;
+        } else if (g.optimizer != s.optimizer || g.lr != s.lr || g.beta1 != s.beta1 || g.beta2 != s.beta2 ||
+                   g.eps != s.eps) {
+            return -1;
+        }
+        M.compressed = p.compressed ? 1 : 0;
+        M.tm = cdiv(h->mp, 128); M.tn = cdiv(h->np, 128); M.ntiles = M.tm * M.tn;
+        M.mA = tcl_map_P(h, h->P); M.mB = tcl_map(h, kMapRbarT);
+        int rc = GLR_OK;
+        M.mD0 = tcl_x_map(h, p.X, st, &rc);
+        if (rc != GLR_OK) return -2;
+        M.mD1 = tcl_map(h, kMapMo); M.mD2 = tcl_map(h, kMapVo); M.mD3 = tcl_map(h, kMapMbarU);
+        M.Mbar = h->Mbar; M.X = p.X; M.Mo = h->Mo; M.Vo = h->Vo;
+        return 1;
+    });
+}
+
 // Between K1 and K3: refresh, or Approx-Top-r selection and P.
 int select_phase(StepPlan& p, cudaStream_t st) {
     glr_handle* h = p.h;
@@ -671,6 +849,8 @@ int select_phase(StepPlan& p, cudaStream_t st) {
         GLR_CK(h, cudaMemcpyAsync(h->J, h->forceJ.data(), sizeof(int32_t) * r, cudaMemcpyHostToDevice, st));
         h->has_forceJ = false;
         h->comm += (int64_t)r * np + mp;
+    } else if (h->tcl) {
+        h->comm += (int64_t)r * np + mp;           // the scores come from tcl_lambda
     } else if (!p.lam_fused) {
         PhaseScope ps(h, GLR_PH_LAMBDA, st);
         LambdaArgs la{};
@@ -714,14 +894,14 @@ int select_P_grouped(std::vector<StepPlan>& plans, cudaStream_t st) {
         glr_handle* h = p.h;
         if (!h0) h0 = h;
         SelectMat& M = g.mat[g.nmat++];
-        M.part = h->lam_part; M.ntiles = p.lam_fused ? h->nstrips : h->ntiles;
+        M.part = h->lam_part; M.ntiles = h->tcl ? h->tc_lam_tiles : p.lam_fused ? h->nstrips : h->ntiles;
         M.mp = h->mp; M.r = h->r; M.k = h->k; M.mode = h->exact ? 0 : 1;
         M.do_select = (!p.refresh && !p.forced && !p.fixed) ? 1 : 0;
         M.dsign = h->exact ? nullptr : h->dsign; M.lam = h->lam; M.J = h->J;
         M.U = h->U; M.Y = h->Y; M.Yt = h->Yt; M.P = h->P;
         M.rbar = p.stream_update ? 1 : 0; M.np = h->np;
         M.Mbar = h->Mbar; M.Wbar = h->Wbar; M.Rbar = h->Rbar;
-        M.build_p = (h->tc && !h->exact) ? 0 : 1;
+        M.build_p = ((h->tc || h->tcl) && !h->exact) ? 0 : 1;
         M.out0 = g.total_out;
         g.total_out += (M.build_p ? (int64_t)h->mp * h->r : 0) + (M.rbar ? (int64_t)h->r * h->np : 0);
         if (g.nmat == kGroupMax) {
@@ -770,13 +950,14 @@ void finish_step(StepPlan& p) {
 }
 
 int step_group(std::vector<StepPlan>& plans, cudaStream_t st) {
-    std::vector<StepPlan*> fused, unfused;
+    std::vector<StepPlan*> fused, unfused, tcl;
     for (StepPlan& p : plans) {
         plan_step(p);
-        (p.h->fused ? fused : unfused).push_back(&p);
+        (p.h->tcl ? tcl : p.h->fused ? fused : unfused).push_back(&p);
     }
     int rc;
     if (!fused.empty() && (rc = compose_fused(fused, st)) != GLR_OK) return rc;
+    if (!tcl.empty() && (rc = tcl_compose(tcl, st)) != GLR_OK) return rc;
     for (StepPlan* p : unfused)
         if ((rc = compose_unfused(*p, st)) != GLR_OK) return rc;
     // Refreshes (Semi-Lazy SVD) of different matrices are independent: each runs on its
@@ -803,8 +984,10 @@ int step_group(std::vector<StepPlan>& plans, cudaStream_t st) {
     }
     for (StepPlan& p : plans)
         if ((rc = select_phase(p, st)) != GLR_OK) return rc;
+    if (!tcl.empty() && (rc = tcl_lambda(tcl, st)) != GLR_OK) return rc;
     for (glr_handle* h : refreshing) GLR_CK(h, cudaStreamWaitEvent(st, h->rdone, 0));
     if ((rc = select_P_grouped(plans, st)) != GLR_OK) return rc;
+    if (!tcl.empty() && (rc = tcl_project_update(tcl, st)) != GLR_OK) return rc;
     std::vector<StepPlan*> streamed, strips;
     for (StepPlan* p : fused) {
         if (separate_optimizer(p->h)) continue;

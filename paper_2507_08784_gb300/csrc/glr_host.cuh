@@ -54,6 +54,17 @@ struct glr_handle {
     float* YtJ = nullptr;        // Yt[J, :] (r x k) for P = U[:, J] as a library product
     float* amsv = nullptr;       // AMSGrad: the scalar normaliser and this step's maximum of V
     float* galr = nullptr;       // Algorithm 5: the subspace step direction M / (sqrt(V) + eps), r x n'
+    // The tcgen05 large-matrix path (k_tc.cu; truncated basis, bf16 gradients, MSGD / Adam): B
+    // and Mbar are column-major there, P keeps a transposed copy per projector allocation, and
+    // the tensor maps of every operand sit in a device table (not part of the checkpointed state).
+    int tcl = 0, rpad = 0, kpad = 0, tc_na = 0, tc_ng = 0, tc_lam_tiles = 0;
+    float* Pbuf0 = nullptr;                    // the first projector allocation (P and Pprev trade places)
+    float *PT0 = nullptr, *PT1 = nullptr;      // P^T of Pbuf0 / of the other allocation (rpad x m')
+    float *WT = nullptr, *YTk = nullptr, *RbarT = nullptr;   // W^T (n' x kpad), Y^T (kpad x m'), Rbar^T (n' x rpad)
+    CUtensorMap* dmaps = nullptr;
+    const void* tc_gptr[2][GLR_MAX_NODES] = {};   // gradient pointers described in each map slot
+    const float* tc_xptr[2] = {nullptr, nullptr};
+    int tc_glast = 0, tc_xlast = 0;               // the slot used last
     cudaStream_t rstream = nullptr;            // side stream of this handle's refresh
     cudaEvent_t rfork = nullptr, rdone = nullptr, rpow = nullptr;
     int pow_ok = 0;                            // refresh through the grouped power iteration (k_power.cu)
@@ -161,6 +172,26 @@ int gemm(glr_handle* h, const GemmDesc& d, cudaStream_t st);
         const int gemm_rc_ = ::glr::host::gemm((h), (d), (st));                                \
         if (gemm_rc_ != GLR_OK) return gemm_rc_;                                               \
     } while (0)
+
+// The tcgen05 large-matrix path (glr_tc_host.cu): eligibility, buffers, tensor maps.
+enum TcMap { kMapBt, kMapPT0, kMapPT1, kMapP0, kMapP1, kMapRwT, kMapMbarT, kMapYT, kMapYt, kMapWT, kMapY, kMapYtJn,
+             kMapYtJm, kMapRbarT, kMapBtD, kMapMbarL, kMapMbarU, kMapMo, kMapVo, kNumTcMaps };
+// After the fixed maps: two slots of N gradient maps, then two slots for X (the caller's buffers,
+// re-described only when a pointer changes).
+const CUtensorMap* tcl_grad_maps(glr_handle* h, const void* const* G, cudaStream_t st, int* rc);
+const CUtensorMap* tcl_x_map(glr_handle* h, const float* X, cudaStream_t st, int* rc);
+bool tcl_eligible(int64_t mp, int64_t np, int r, int N, int k, bool exact, const glr_schedule* s);
+int tcl_alloc(glr_handle* h);         // state buffers (before n_state_allocs is fixed)
+int tcl_maps(glr_handle* h);          // the device map table (after)
+float* tcl_PT_of(const glr_handle* h, const float* P);
+const CUtensorMap* tcl_map(const glr_handle* h, int which);
+const CUtensorMap* tcl_map_P(const glr_handle* h, const float* P);      // row-major P of that allocation
+const CUtensorMap* tcl_map_PT(const glr_handle* h, const float* P);     // its transpose
+bool encode_f32_map(CUtensorMap* map, const float* base, int rank, const uint64_t* dims, const uint64_t* strides,
+                    const uint32_t* box);
+// Any tiled map: dtype, rank (<= 3), dims innermost first, byte strides of dims 1.., box, swizzle.
+bool encode_map(CUtensorMap* map, CUtensorMapDataType dtype, const void* base, int rank, const uint64_t* dims,
+                const uint64_t* strides, const uint32_t* box, CUtensorMapSwizzle swz);
 
 // The Semi-Lazy SVD refresh (glr_refresh_host.cu).
 int cholqr(glr_handle* h, float*& A, float*& tmp, int rows, cudaStream_t st);

@@ -380,6 +380,57 @@ int pow_chunk();
 // (arg: the partials of stage 0, else of stages 2/3); 5: H <- sum of the stage-0 partials.
 cudaError_t pow_stage(const PowGroup& g, int stage, int arg, cudaStream_t st);
 
+// ------------------------------------------------------------------------------------------
+// The large-matrix path on the tcgen05 tensor cores (k_tc.cu).  Node buffers B_i and Mbar are
+// column-major (B_i^T: n' x m'); P row-major m' x r with P^T (rpad x m'); R_w,i^T (n' x rpad per
+// node), W^T (n' x kpad), Rbar^T (n' x rpad), Y^T (kpad x m'); rpad = r and kpad = k rounded up
+// to 32.  Each launch takes up to kTcGroupMax matrices; a matrix's tiles are [tile0, tile0 +
+// ntiles) of the launch.  Tensor maps live in device memory (one table per handle).
+// ------------------------------------------------------------------------------------------
+namespace tc {
+constexpr int kTcGroupMax = 64;
+constexpr int kTcGPtrs = 512;
+struct TcMat {
+    int mp, np, N, r, rpad, k, kpad;
+    int transposed, gdtype, e_zero, write_B, compressed;
+    int tile0, ntiles, tm, tn;            // this op's tiles of the matrix: tm x tn (or tn x ng node groups)
+    int ng, na;                           // PrevProj: node groups of na nodes
+    int g_off;                            // Compose: first gradient pointer in TcGroup::G
+    const CUtensorMap* mA; const CUtensorMap* mB;      // the MMA operands
+    const CUtensorMap* mD0; const CUtensorMap* mD1;    // epilogue data: Compose B^T, gradients (N maps);
+    const CUtensorMap* mD2; const CUtensorMap* mD3;    // Update X, Mo, Vo, Mbar^T; Lambda Mbar^T
+    float* B; float* Mbar; float* Rw; float* W; float* part;
+    const int32_t* J; const float* dsign;
+    float* Pout; float* PT; float* Rbar; float* RbarT;
+    float* X; float* Mo; float* Vo;
+    uint64_t seed; uint32_t t;
+};
+struct TcGroup {
+    int nmat, total_tiles;
+    int stages; uint32_t stage_bytes; int tbufs;     // set by the launcher: operand ring, accumulators
+    int dstages; uint32_t dstage_bytes;              // ... and the epilogue's data ring
+    int optimizer;                                   // Update: the optimizer of every matrix in the launch
+    float lr, beta1, beta2, eps;
+    int* err;                                        // bounded waits that gave up are counted here
+    TcMat mat[kTcGroupMax];
+    const void* G[kTcGPtrs];
+};
+cudaError_t launch_prevproj(TcGroup& g, cudaStream_t st);
+cudaError_t launch_compose(TcGroup& g, cudaStream_t st);
+cudaError_t launch_wbar(TcGroup& g, cudaStream_t st);
+cudaError_t launch_lambda(TcGroup& g, cudaStream_t st);
+cudaError_t launch_pbuild(TcGroup& g, cudaStream_t st);
+cudaError_t launch_rbar(TcGroup& g, cudaStream_t st);
+cudaError_t launch_update(TcGroup& g, cudaStream_t st);
+int compose_bn();
+// dst (cols x ldd) = src^T rounded to TF32 (src row-major rows x cols, leading dimension lds)
+cudaError_t transpose_round(float* dst, int ldd, const float* src, int rows, int cols, int lds, cudaStream_t st);
+cudaError_t round_tf32(float* p, int64_t n, cudaStream_t st);
+// E (row-major m' x n') = B^T - P Rw with B^T column-major (n' x m'), Rw row-major r x n'
+cudaError_t error_colmajor(const float* Bt, const float* P, const float* Rw, int mp, int np, int r, int e_zero,
+                           float* E, cudaStream_t st);
+}  // namespace tc
+
 // Message reported by glr_last_error(NULL) for entry points that have no handle.
 void set_global_error(const char* msg);
 

@@ -135,6 +135,11 @@ int glr_get_error(glr_handle* h, int32_t i, float* E_out, void* stream) {
     const int mp = h->mp, np = h->np, r = h->r;
     float* Bi = h->B + (size_t)i * mp * np;
     float* Rwi = h->Rw + (size_t)i * r * np;
+    if (h->tcl) {                              // B_i column-major: R_w,i = P_prev^T B_i with strides
+        if (!h->e_zero) GLR_GEMM(h, gd(r, np, mp, h->Pprev, 1, r, Bi, 1, mp, Rwi, np, 1), st);
+        GLR_LAUNCH(h, 1, tc::error_colmajor(Bi, h->Pprev, Rwi, mp, np, r, h->e_zero ? 1 : 0, E_out, st));
+        return GLR_OK;
+    }
     if (!h->e_zero) GLR_GEMM(h, gd(r, np, mp, h->Pprev, 1, r, Bi, np, 1, Rwi, np, 1), st);
     GLR_LAUNCH(h, 1, materialize_error(mp, np, r, h->e_zero ? 1 : 0, Bi, h->Pprev, Rwi, E_out, st));
     return GLR_OK;
@@ -148,7 +153,8 @@ int glr_get_selection(glr_handle* h, int32_t* J_host, float* P_out, float* Rbar_
     if (P_out) GLR_CK(h, cudaMemcpyAsync(P_out, h->Pprev, 4 * mp * r, cudaMemcpyDeviceToDevice, st));
     if (Rbar_out) GLR_CK(h, cudaMemcpyAsync(Rbar_out, h->Rbar, 4 * r * np, cudaMemcpyDeviceToDevice, st));
     if (lambda_out) GLR_CK(h, cudaMemcpyAsync(lambda_out, h->lam, 4 * mp, cudaMemcpyDeviceToDevice, st));
-    if (Mbar_out) GLR_CK(h, cudaMemcpyAsync(Mbar_out, h->Mbar, 4 * mp * np, cudaMemcpyDeviceToDevice, st));
+    if (Mbar_out && h->tcl) GLR_LAUNCH(h, 1, transpose_pad(Mbar_out, (int)np, h->Mbar, (int)np, (int)mp, st));
+    else if (Mbar_out) GLR_CK(h, cudaMemcpyAsync(Mbar_out, h->Mbar, 4 * mp * np, cudaMemcpyDeviceToDevice, st));
     if (J_host) {
         if (h->last_uncompressed) {
             for (size_t q = 0; q < r; ++q) J_host[q] = -1;

@@ -36,6 +36,7 @@ int wy_from_Q(glr_handle* h, cudaStream_t st) {
         GLR_LAUNCH(h, 1, pack_frag(h->YF, h->Y, mp, k, k, 0, st));
         GLR_LAUNCH(h, 1, pack_frag(h->YtF, h->Yt, mp, k, k, 1, st));
     }
+    if (h->tcl) GLR_LAUNCH(h, 1, tc::transpose_round(h->YTk, mp, h->Y, mp, k, k, st));   // Y^T for the W products
     return GLR_OK;
 }
 
@@ -177,17 +178,19 @@ int do_refresh(glr_handle* h, cudaStream_t st) {
     if (h->refreshes == 0 && !h->basis_from_user)
         GLR_LAUNCH(h, 1, random_block(h->Q, mp, k, h->s.seed, static_cast<uint32_t>(h->t), st));
     int rc;
+    // Mbar(a, b) at a * sa + b * sb: row-major, or column-major on the tcgen05 path
+    const int64_t sa = h->tcl ? 1 : np, sb = h->tcl ? mp : 1;
     for (int it = 0; it < h->s.power_iters; ++it) {
         // Z = Mbar^T Q (n' x k) and Q = Mbar Z (m' x k), each re-orthonormalised by CholeskyQR
         // (one pass keeps the block well conditioned; the span is what the iteration needs)
-        GLR_GEMM(h, gd(np, k, mp, h->Mbar, 1, np, h->Q, k, 1, h->Z, k, 1), st);
+        GLR_GEMM(h, gd(np, k, mp, h->Mbar, sb, sa, h->Q, k, 1, h->Z, k, 1), st);
         if ((rc = cholqr(h, h->Z, h->Zn, np, st)) != GLR_OK) return rc;
-        GLR_GEMM(h, gd(mp, k, np, h->Mbar, np, 1, h->Z, k, 1, h->Q, k, 1), st);
+        GLR_GEMM(h, gd(mp, k, np, h->Mbar, sa, sb, h->Z, k, 1, h->Q, k, 1), st);
         if ((rc = cholqr(h, h->Q, h->Qn, mp, st)) != GLR_OK) return rc;
     }
     if ((rc = cholqr(h, h->Q, h->Qn, mp, st)) != GLR_OK) return rc;   // CholeskyQR2: orthonormal to rounding
     // Rayleigh-Ritz: Z = Mbar^T Q, H = Z^T Z = Q^T Mbar Mbar^T Q
-    GLR_GEMM(h, gd(np, k, mp, h->Mbar, 1, np, h->Q, k, 1, h->Z, k, 1), st);
+    GLR_GEMM(h, gd(np, k, mp, h->Mbar, sb, sa, h->Q, k, 1, h->Z, k, 1), st);
     GLR_GEMM(h, gd(k, k, np, h->Z, 1, k, h->Z, k, 1, h->Hk, k, 1), st);
     return refresh_tail(h, st);
 }
