@@ -49,7 +49,7 @@ extern "C" {
 #define GLR_ENOMEM     -2   /* a device or host allocation failed                          */
 #define GLR_ECUDA      -3   /* a CUDA runtime call or kernel launch failed                 */
 #define GLR_ENUMERIC   -4   /* the refresh could not orthonormalise its basis              */
-#define GLR_ENONFINITE -5   /* reserved: non-finite values detected                        */
+#define GLR_ENONFINITE -5   /* a NaN or Inf reached the node-mean gradient (glr_get_stats)  */
 #define GLR_ETIMEOUT   -6   /* a bounded device-side wait gave up (reported by glr_get_stats) */
 
 /* ---- enumerations -------------------------------------------------------------------- */
@@ -130,7 +130,18 @@ typedef struct glr_stats {
     int32_t transposed;             /* 1 when m > n (the handle works on G^T)                */
     int32_t last_refresh_sweeps;    /* eigen-solver sweeps used by the last refresh          */
     int64_t launches;               /* kernels launched by this handle so far                */
+    int32_t path;                   /* kernel family that runs the step: GLR_PATH_*          */
+    int32_t nonfinite;              /* warps of the compose pass that found a NaN or Inf in  *
+                                     * the node-mean gradient since creation (0: all finite) */
 } glr_stats;
+
+/* Kernel families (glr_stats.path), chosen by glr_create from the shape and schedule.       */
+#define GLR_PATH_STRIP   0   /* fused strip kernels, products on the FP32 pipes (m' <= 4096)  */
+#define GLR_PATH_MMA     1   /* fused strip kernels, 3xTF32 mma.sync compose (small m', r)    */
+#define GLR_PATH_TCGEN05 2   /* tcgen05 tensor-core path: TF32 products, TMA-staged epilogues *
+                              * (truncated basis, bf16 gradients, MSGD / Adam, 16 <= r <= 128) */
+#define GLR_PATH_LIBRARY 3   /* unfused passes with cuBLAS products (large fp32 matrices)     */
+#define GLR_PATH_PLAIN   4   /* unfused passes with the library's own FFMA GEMM               */
 
 /* Phases of a step, for glr_profile_read.                                                 */
 #define GLR_PH_PREV_PROJECT 0   /* R_i = P_{t-1}^T B_i for the deferred error                 */
@@ -227,8 +238,10 @@ int glr_refresh(glr_handle* h);
 
 /* Counters (see glr_stats).  Reads the handle's device flags with a blocking copy, so it
  * waits for work already queued on the device.  Returns GLR_ETIMEOUT (with out filled) when a
- * bounded wait inside a compose kernel of this handle's launches has given up since creation:
- * the results of those steps are not valid.                                               */
+ * bounded wait inside a kernel of this handle's launches has given up since creation (the
+ * results of those steps are not valid), else GLR_ENONFINITE when a compose pass found a NaN
+ * or Inf in the node-mean gradient (a node sent a non-finite gradient, or the error state
+ * overflowed), else GLR_OK.                                                                */
 int glr_get_stats(const glr_handle* h, glr_stats* out);
 
 /* Message of the last failure on h (or of the last failed glr_create when h is NULL);

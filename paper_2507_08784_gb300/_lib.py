@@ -56,6 +56,8 @@ class GlrStats(ctypes.Structure):
         ("transposed", ctypes.c_int32),
         ("last_refresh_sweeps", ctypes.c_int32),
         ("launches", ctypes.c_int64),
+        ("path", ctypes.c_int32),
+        ("nonfinite", ctypes.c_int32),
     ]
 
 

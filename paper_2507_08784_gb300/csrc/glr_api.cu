@@ -545,7 +545,7 @@ int compose_unfused(StepPlan& p, cudaStream_t st) {
     ca.grad_dtype = h->s.grad_dtype; ca.transposed = h->transposed;
     ca.mp = mp; ca.np = np; ca.N = N; ca.r = h->tc ? 0 : r; ca.e_zero = h->e_zero ? 1 : 0;
     ca.write_B = (p.warm || h->s.no_error_feedback) ? 0 : 1;   // B feeds only the error
-    ca.B = h->B; ca.Pprev = h->Pprev; ca.Rw = h->Rw; ca.Mbar = h->Mbar;
+    ca.B = h->B; ca.Pprev = h->Pprev; ca.Rw = h->Rw; ca.Mbar = h->Mbar; ca.nonfinite = h->dflags + 3;
     if (h->tc) GLR_LAUNCH(h, 1, compose_streamed(ca, st));
     else GLR_LAUNCH(h, 1, compose(ca, st));
     return GLR_OK;
@@ -587,6 +587,7 @@ int compose_fused(std::vector<StepPlan*>& plans, cudaStream_t st) {
             M.B = h->B; M.Pprev = h->Pprev; M.Mbar = h->Mbar;
             M.YT = h->YT; M.YtT = h->YtT; M.YF = h->YF; M.YtF = h->YtF; M.part = h->lam_part;
             M.Wbar = p->stream_update ? h->Wbar : nullptr;
+            M.nonfinite = h->dflags + 3;
             M.seed = h->s.seed; M.t = static_cast<uint32_t>(h->t);
             for (int i = 0; i < h->N; ++i) g.G[M.g_off + i] = p->G[i];
             if (tma) {
@@ -751,7 +752,7 @@ int tcl_compose(std::vector<StepPlan*>& plans, cudaStream_t st) {
         M.mD0 = tcl_map(h, kMapBtD);
         M.mD1 = tcl_grad_maps(h, p.G, st, &rc);
         if (rc != GLR_OK) return -2;
-        M.B = h->B; M.Mbar = h->Mbar;
+        M.B = h->B; M.Mbar = h->Mbar; M.nonfinite = h->dflags + 3;
         return 1;
     });
 }

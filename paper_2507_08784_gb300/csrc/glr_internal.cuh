@@ -84,6 +84,12 @@ __device__ __forceinline__ void st_stream4(float* p, float a, float b, float c, 
     asm("st.global.cs.v4.f32 [%0], {%1, %2, %3, %4};" ::"l"(p), "f"(a), "f"(b), "f"(c), "f"(d));
 }
 
+// A NaN or Inf in the node-mean gradient: one count per warp that holds any (flag may be null).
+__device__ __forceinline__ void flag_nonfinite(bool bad, int* flag) {
+    const unsigned m = __ballot_sync(__activemask(), bad);
+    if (m && flag && static_cast<int>(threadIdx.x & 31) == __ffs(m) - 1) atomicAdd(flag, 1);
+}
+
 // ------------------------------------------------------------------------------------------
 // Gradient element loads (fp32 or bf16, widened to fp32).
 // ------------------------------------------------------------------------------------------
@@ -129,6 +135,7 @@ struct ComposeArgs {
     const float* Pprev;     // m' x r
     const float* Rw;        // N x r x n'  (Rw_i = Pprev^T B_i)
     float* Mbar;            // m' x n'
+    int* nonfinite;         // counts warps that found a NaN / Inf in Mbar (may be null)
 };
 cudaError_t compose(const ComposeArgs& a, cudaStream_t st);
 
@@ -283,6 +290,7 @@ struct StreamMat {
     const float* YT; const float* YtT; float* part;   // Y^T, Yt^T (k x transposed_pitch(m')); part: nstrips x m'
     const float* YF; const float* YtF;                // Y, Yt in the tensor-core kernel's fragment order
     float* Wbar;                                      // tensor-core kernel: W = Y^T Mbar written here when set
+    int* nonfinite;                                   // counts warps that found a NaN / Inf in Mbar
     uint64_t seed; uint32_t t;
 };
 struct StreamGroup {
@@ -403,6 +411,7 @@ struct TcMat {
     const int32_t* J; const float* dsign;
     float* Pout; float* PT; float* Rbar; float* RbarT;
     float* X; float* Mo; float* Vo;
+    int* nonfinite;                                   // Compose: counts warps that found a NaN / Inf in Mbar
     uint64_t seed; uint32_t t;
 };
 struct TcGroup {

@@ -123,7 +123,10 @@ int glr_get_stats(const glr_handle* h, glr_stats* out) {
     cudaMemcpy(flags, h->dflags, sizeof(flags), cudaMemcpyDeviceToHost);
     out->last_refresh_sweeps = flags[1];
     out->launches = h->launches;
-    return flags[2] ? GLR_ETIMEOUT : GLR_OK;
+    out->path = h->tcl ? GLR_PATH_TCGEN05 : h->mma ? GLR_PATH_MMA : h->fused ? GLR_PATH_STRIP
+              : h->tc ? GLR_PATH_LIBRARY : GLR_PATH_PLAIN;
+    out->nonfinite = flags[3];
+    return flags[2] ? GLR_ETIMEOUT : flags[3] ? GLR_ENONFINITE : GLR_OK;
 }
 
 const char* glr_last_error(const glr_handle* h) { return h ? h->err.c_str() : g_create_err.c_str(); }

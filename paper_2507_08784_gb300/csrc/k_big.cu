@@ -54,6 +54,7 @@ __global__ void __launch_bounds__(TB) compose_rows_kernel(ComposeArgs a) {
             }
         }
         st4(a.Mbar + e, make_float4(acc.x * invN, acc.y * invN, acc.z * invN, acc.w * invN));
+        flag_nonfinite(!isfinite(acc.x) || !isfinite(acc.y) || !isfinite(acc.z) || !isfinite(acc.w), a.nonfinite);
     }
 }
 
@@ -97,13 +98,17 @@ __global__ void __launch_bounds__(TB) compose_cols_kernel(ComposeArgs a) {
         }
     }
     const float invN = 1.0f / static_cast<float>(a.N);
+    bool bad = false;
 #pragma unroll
     for (int u = 0; u < 4; ++u) {
         const int aa = a0 + lr + 16 * u, b = b0 + 4 * lq;
-        if (aa < a.mp && b < a.np)
+        if (aa < a.mp && b < a.np) {
             st4(a.Mbar + (int64_t)aa * a.np + b,
                 make_float4(acc[u].x * invN, acc[u].y * invN, acc[u].z * invN, acc[u].w * invN));
+            bad |= !isfinite(acc[u].x) || !isfinite(acc[u].y) || !isfinite(acc[u].z) || !isfinite(acc[u].w);
+        }
     }
+    flag_nonfinite(bad, a.nonfinite);
 }
 
 // X, Mo (, Vo) and Ghat share X's layout: quads of the flattened m x n array (m n % 4 == 0).

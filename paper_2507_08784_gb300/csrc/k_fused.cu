@@ -273,11 +273,15 @@ __global__ void __launch_bounds__(NT, 1) stream_kernel(const __grid_constant__ S
     for (int ii = 0; ii < 4; ++ii)
 #pragma unroll
         for (int j = 0; j < 4; ++j) acc[ii][j] *= invN;
+    bool bad = false;
     if (mine)
 #pragma unroll
         for (int ii = 0; ii < 4; ++ii)
-            if (ii < nrows)
+            if (ii < nrows) {
                 st4(M.Mbar + (int64_t)(a0 + ii) * np + bcol, make_float4(acc[ii][0], acc[ii][1], acc[ii][2], acc[ii][3]));
+                bad |= !isfinite(acc[ii][0]) || !isfinite(acc[ii][1]) || !isfinite(acc[ii][2]) || !isfinite(acc[ii][3]);
+            }
+    flag_nonfinite(bad, M.nonfinite);
     if (!M.lam) return;
 
     // ---- truncated-basis Approx-Top-r partial sums for this strip ---------------------------

@@ -348,8 +348,9 @@ __device__ __forceinline__ void compose_node(const float* S, const GT* Gs, bool 
 // acc <- acc / N, stored as the strip of Mbar (Mb: Mbar at the strip's first column).
 template <int GPW>
 __device__ __forceinline__ void store_mbar(float (&acc)[GPW][4], int N, float* Mb, int mp, int np, int ng, bool colok,
-                                           const Lane& L) {
+                                           const Lane& L, int* nonfinite) {
     const float invN = 1.0f / static_cast<float>(N);
+    bool bad = false;
 #pragma unroll
     for (int j = 0; j < GPW; ++j) {
         const int G8 = L.w + NW * j;
@@ -357,10 +358,17 @@ __device__ __forceinline__ void store_mbar(float (&acc)[GPW][4], int N, float* M
         for (int e = 0; e < 4; ++e) acc[j][e] *= invN;
         const int ra = 8 * G8 + L.rho, rb = ra + 2;
         if (G8 < ng && colok) {
-            if (ra < mp) *reinterpret_cast<float2*>(Mb + (int64_t)ra * np) = make_float2(acc[j][0], acc[j][1]);
-            if (rb < mp) *reinterpret_cast<float2*>(Mb + (int64_t)rb * np) = make_float2(acc[j][2], acc[j][3]);
+            if (ra < mp) {
+                *reinterpret_cast<float2*>(Mb + (int64_t)ra * np) = make_float2(acc[j][0], acc[j][1]);
+                bad |= !isfinite(acc[j][0]) || !isfinite(acc[j][1]);
+            }
+            if (rb < mp) {
+                *reinterpret_cast<float2*>(Mb + (int64_t)rb * np) = make_float2(acc[j][2], acc[j][3]);
+                bad |= !isfinite(acc[j][2]) || !isfinite(acc[j][3]);
+            }
         }
     }
+    flag_nonfinite(bad, nonfinite);
 }
 
 // Truncated-basis Approx-Top-r partial sums over the strip: (Mbar - Yt (Y^T Mbar)) v_j.
@@ -653,7 +661,7 @@ __device__ __forceinline__ void compose_strip(const StreamGroup& g, const TmaMap
         }
     }
     if constexpr (!TMA) cp_async_wait<0>();
-    store_mbar<GPW>(acc, N, M.Mbar + b0 + L.c2, mp, np, ng, colok, L);
+    store_mbar<GPW>(acc, N, M.Mbar + b0 + L.c2, mp, np, ng, colok, L, M.nonfinite);
     if (KT) {
         float4 vq[GPW];
         lam_draw<GPW>(vq, M.seed, M.t, b0, ng, L);

@@ -175,11 +175,16 @@ __global__ void __launch_bounds__(256) compose_kernel(ComposeArgs a) {
         __syncthreads();
     }
     const float invN = 1.0f / static_cast<float>(a.N);
+    bool bad = false;
 #pragma unroll
     for (int u = 0; u < 4; ++u) {
         const int aa = a0 + ty + 8 * u, b = b0 + tx;
-        if (aa < a.mp && b < a.np) a.Mbar[(int64_t)aa * a.np + b] = sum[u] * invN;
+        if (aa < a.mp && b < a.np) {
+            a.Mbar[(int64_t)aa * a.np + b] = sum[u] * invN;
+            bad |= !isfinite(sum[u]);
+        }
     }
+    flag_nonfinite(bad, a.nonfinite);
 }
 }  // namespace
 

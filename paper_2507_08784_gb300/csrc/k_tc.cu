@@ -168,8 +168,10 @@ __device__ __forceinline__ void bulk_wait_read() { asm volatile("cp.async.bulk.w
 
 // The epilogue's side of the data ring.  acquire() waits for the next stage; release() marks this
 // thread done with it: the last thread to finish (counted on the stage's "done" mbarrier, waited
-// by thread 0 of the epilogue) lets `store` issue the tile copies back to global memory, waits until
-// they have read shared memory and hands the stage back to the data warp.
+// by thread 0 of the epilogue) lets `store` issue the tile copies back to global memory as one
+// bulk group.  A stage goes back to the data warp once its group has read shared memory: with
+// three or more stages the leader checks that one stage later (at most one group pending), so the
+// copies of a stage overlap the work on the next; finish() drains the last one.
 struct DataRing {
     uint8_t* base;
     uint32_t bytes;
@@ -178,6 +180,7 @@ struct DataRing {
     uint64_t *full, *empty, *done;
     volatile int* abort;
     int* err;
+    int pend;                                         // stage whose group may still be reading (leader)
     // warp-uniform: every lane gets the stage, or none (the CTA aborted)
     __device__ __forceinline__ uint8_t* acquire() {
         const bool ok = wait_phase(smem_u32(&full[s]), use, abort, err);
@@ -189,15 +192,27 @@ struct DataRing {
         fence_proxy_async();                          // this thread's writes, before the copies read them
         mbar_arrive(smem_u32(&done[s]));
         if (leader) {
-            if (wait_phase(smem_u32(&done[s]), use, abort, err)) {
-                if (store(smem_u32(base + (size_t)s * bytes))) {
-                    bulk_commit();
-                    bulk_wait_read();
+            if (wait_phase(smem_u32(&done[s]), use, abort, err)) store(smem_u32(base + (size_t)s * bytes));
+            bulk_commit();                            // one group per stage (empty when nothing is stored)
+            if (n < 3) {                              // two stages: hand this one back at once
+                bulk_wait_read();
+                mbar_arrive(smem_u32(&empty[s]));
+            } else {
+                if (pend >= 0) {
+                    asm volatile("cp.async.bulk.wait_group.read 1;" ::: "memory");
+                    mbar_arrive(smem_u32(&empty[pend]));
                 }
+                pend = s;
             }
-            mbar_arrive(smem_u32(&empty[s]));
         }
         if (++s == n) { s = 0; use ^= 1u; }
+    }
+    __device__ __forceinline__ void finish(bool leader) {
+        if (!leader) return;
+        bulk_wait_read();
+        if (pend >= 0) mbar_arrive(smem_u32(&empty[pend]));
+        pend = -1;
+        asm volatile("cp.async.bulk.wait_group 0;" ::: "memory");   // the stores are complete before the CTA ends
     }
 };
 struct NoStore { __device__ bool operator()(uint32_t) const { return false; } };
@@ -315,7 +330,7 @@ __global__ void __launch_bounds__(kThreads, 1) tc_kernel(const __grid_constant__
     } else {
         uint32_t tuse[2] = {0, 0};
         int b = 0;
-        DataRing dr{dring, DB, D, 0, 0u, dfull_bar, dempty_bar, ddone_bar, abort, g.err};
+        DataRing dr{dring, DB, D, 0, 0u, dfull_bar, dempty_bar, ddone_bar, abort, g.err, -1};
         for (int tile = blockIdx.x; tile < g.total_tiles; tile += gridDim.x) {
             Tile t = find_tile(g, tile);
             t.nk = Op::nk(g, t);
@@ -330,6 +345,7 @@ __global__ void __launch_bounds__(kThreads, 1) tc_kernel(const __grid_constant__
             tuse[b] ^= 1u;
             if (nbuf == 2) b ^= 1;
         }
+        if (D > 0) dr.finish(warp == 0 && lane == 0);
     }
     fence_before();
     __syncthreads();
@@ -495,12 +511,18 @@ struct Compose {
                 return true;
             });
         }
+        bool bad = false;
         if (a < M.mp) {
             const float invN = 1.0f / static_cast<float>(M.N);
 #pragma unroll
             for (int j = 0; j < 32; ++j)
-                if (c0 + j < M.np) M.Mbar[(int64_t)(c0 + j) * M.mp + a] = acc[j] * invN;
+                if (c0 + j < M.np) {
+                    const float v = acc[j] * invN;
+                    bad |= !isfinite(v);
+                    M.Mbar[(int64_t)(c0 + j) * M.mp + a] = v;
+                }
         }
+        flag_nonfinite(bad, M.nonfinite);
         return true;
     }
 };
@@ -823,12 +845,16 @@ cudaError_t launch(TcGroup& g, cudaStream_t st) {
         cols = std::max(cols, acc_cols_of<Op>(g.mat[i]));
     }
     if (cols > (int)kTmemCols) return cudaErrorInvalidValue;
-    // two data stages when the op has epilogue data (one if that leaves no room for operands),
-    // then as many operand stages as fit
-    int dstages = db ? 2 : 0;
-    if (db && kSmemBudget < 2 * db + sb) dstages = 1;
-    const size_t left = kSmemBudget - (size_t)dstages * db;
-    int stages = std::min(static_cast<int>(left / sb), kMaxStages);
+    // without epilogue data: as many operand stages as fit; with it: two operand stages (one if
+    // two leave no room for two data stages), then as many data stages as fit (at most four)
+    int stages, dstages = 0;
+    if (!db) {
+        stages = std::min(static_cast<int>(kSmemBudget / sb), kMaxStages);
+    } else {
+        stages = kSmemBudget >= 2 * sb + 2 * db ? 2 : 1;
+        dstages = std::min(static_cast<int>((kSmemBudget - stages * sb) / db), kMaxDStages);
+        if (dstages < 1) return cudaErrorInvalidValue;
+    }
     if (stages < 1) return cudaErrorInvalidValue;
     g.stages = stages;
     g.stage_bytes = static_cast<uint32_t>(sb);

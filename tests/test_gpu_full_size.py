@@ -23,7 +23,11 @@ E_i(t) + P R_i(t) = G_i(t) + E_i(t - 1) (Eq. ef1, ef2), and the optimizer applie
 
 Tolerances: 1e-5 relative Frobenius for fp32 arithmetic on bf16-exact inputs, 1e-4 for
 lambda-bar (sums of n' products) and for X under Adam (the update divides by sqrt(V) + eps).
+Handles on the tcgen05 path (glr_stats.path == GLR_PATH_TCGEN05: these bf16 workloads) form
+their products as TF32 tensor-core MMAs and are held to the bf16 bound instead: 2e-2 relative
+Frobenius, near-ties of the selection within 1e-2 of the largest score.
 """
+
 import numpy as np
 import pytest
 
@@ -88,7 +92,10 @@ def test_full_size_algorithm3_steps(name, li):
     r, N, k = cfg.r, cfg.N, cfg.basis_rank
     seed = 4242 + li
     dev = _handle(glr, cfg, li, seed, cfg.tau, "alg3")
-    x_tol = 1e-4 if cfg.optimizer == "adam" else 1e-5
+    tc = dev.stats()["path"] == 2
+    tol = 2e-2 if tc else 1e-5
+    lam_tol, tie = (2e-2, 1e-2) if tc else (1e-4, 1e-4)
+    x_tol = tol if tc else 1e-4 if cfg.optimizer == "adam" else 1e-5
     X = torch.zeros(m, n, device="cuda")
     Xo, Mo, Vo = np.zeros((m, n)), np.zeros((m, n)), np.zeros((m, n))
     E = np.zeros((N, mp, npr))
@@ -101,7 +108,7 @@ def test_full_size_algorithm3_steps(name, li):
             dev.step(Gd, X)
             torch.cuda.synchronize()
             J, P, Rbar, lam, Mbar_d = dev.selection()
-            assert rel(Mbar_d.cpu().numpy(), Mbar) <= 1e-5, f"step {t}: Mbar"
+            assert rel(Mbar_d.cpu().numpy(), Mbar) <= tol, f"step {t}: Mbar"
             if t % cfg.tau == 0:                              # refresh: uncompressed mean, E reset
                 U, s = O.left_singular_basis(Mbar)
                 _check_refresh(dev, Mbar, s, k, t)
@@ -113,22 +120,22 @@ def test_full_size_algorithm3_steps(name, li):
             else:
                 V = O.gaussian_v(seed, t, mp, npr)
                 lam_o = O.approx_top_r_lambda([Mbar], U, V)   # = node mean of u_j^T M_i v_j
-                assert rel(lam.cpu().numpy(), lam_o) <= 1e-4, f"step {t}: lambda-bar"
+                assert rel(lam.cpu().numpy(), lam_o) <= lam_tol, f"step {t}: lambda-bar"
                 Jo = O.argtop_r(lam_o ** 2, r)
-                ok = same_selection(J, Jo, lam_o, 1e-4)
+                ok = same_selection(J, Jo, lam_o, tie)
                 assert ok, f"step {t}: selection differs beyond near-ties"
                 if ok == "tie":
                     break                                     # the runs legitimately diverge
                 Po = U[:, Jo]
-                assert rel(P.cpu().numpy(), Po) <= 1e-5, f"step {t}: P"
+                assert rel(P.cpu().numpy(), Po) <= tol, f"step {t}: P"
                 R = Po.T @ M                                  # R_i = P^T M_i (batched over i)
                 E = M - Po @ R                                # E_i = M_i - P R_i
                 Rb = R.mean(axis=0)                           # the All-Reduce
-                assert rel(Rbar.cpu().numpy(), Rb) <= 1e-5, f"step {t}: Rbar"
+                assert rel(Rbar.cpu().numpy(), Rb) <= tol, f"step {t}: Rbar"
                 for i in (0, N - 1):
                     Ed = dev.error(i).double().cpu().numpy()
                     scale = np.linalg.norm(E[i]) + 0.1 * np.linalg.norm(M[i])
-                    assert np.linalg.norm(Ed - E[i]) <= 1e-5 * scale, f"step {t}: E_{i}"
+                    assert np.linalg.norm(Ed - E[i]) <= tol * scale, f"step {t}: E_{i}"
                 Ghat = Po @ Rb
             Xo, Mo, Vo = _optimizer(cfg, Xo, Mo, Vo, np.swapaxes(Ghat, 0, 1) if transposed else Ghat)
             assert rel(X.cpu().numpy(), Xo) <= x_tol, f"step {t}: X"
@@ -148,6 +155,8 @@ def test_full_size_refresh_every_step_algorithm4():
     mp, npr = min(m, n), max(m, n)
     r, N, k = cfg.r, cfg.N, cfg.basis_rank
     dev = _handle(glr, cfg, li, 77, 1, "alg4")
+    tc = dev.stats()["path"] == 2
+    tol = 2e-2 if tc else 1e-5
     X = torch.zeros(m, n, device="cuda")
     Eprev = [np.zeros((mp, npr)) for _ in range(N)]
     Mo = np.zeros((m, n))
@@ -160,23 +169,23 @@ def test_full_size_refresh_every_step_algorithm4():
             J, P, Rbar, lam, Mbar_d = dev.selection()
             assert np.array_equal(J, np.arange(r)), f"step {t}: Algorithm 4 takes U[:, :r]"
             Mbar = np.mean([G[i] + Eprev[i] for i in range(N)], axis=0)
-            assert rel(Mbar_d.cpu().numpy(), Mbar) <= 1e-5, f"step {t}: Mbar"
+            assert rel(Mbar_d.cpu().numpy(), Mbar) <= tol, f"step {t}: Mbar"
             _, s, _ = np.linalg.svd(Mbar, full_matrices=False)
             Ud = _check_refresh(dev, Mbar, s, k, t)
             Pd = P.double().cpu().numpy()
-            assert rel(Pd, Ud[:, :r]) <= 1e-6, f"step {t}: P = U[:, :r]"
-            assert np.abs(Pd.T @ Pd - np.eye(r)).max() < 1e-4
+            assert rel(Pd, Ud[:, :r]) <= (tol if tc else 1e-6), f"step {t}: P = U[:, :r]"
+            assert np.abs(Pd.T @ Pd - np.eye(r)).max() < (1e-2 if tc else 1e-4)
             Rb = Pd.T @ Mbar
-            assert rel(Rbar.cpu().numpy(), Rb) <= 1e-5, f"step {t}: Rbar = P^T Mbar"
+            assert rel(Rbar.cpu().numpy(), Rb) <= tol, f"step {t}: Rbar = P^T Mbar"
             for i in (0, N - 1):                              # E_i(t) + P R_i(t) = G_i(t) + E_i(t-1)
                 Mi = G[i] + Eprev[i]
                 Ed = dev.error(i).double().cpu().numpy()
                 sent = Pd @ (Pd.T @ Mi)
-                assert np.linalg.norm(Ed + sent - Mi) <= 1e-5 * np.linalg.norm(Mi), f"step {t}: EF balance {i}"
+                assert np.linalg.norm(Ed + sent - Mi) <= tol * np.linalg.norm(Mi), f"step {t}: EF balance {i}"
             Eprev = [dev.error(i).double().cpu().numpy() for i in range(N)]
             Ghat = Pd @ Rb
             Gh = np.swapaxes(Ghat, 0, 1) if transposed else Ghat
             Xo, Mo = O.msgd_update(Xprev, Mo, Gh, cfg.lr, cfg.beta1)
-            assert rel(X.cpu().numpy(), Xo) <= 1e-5, f"step {t}: X"
+            assert rel(X.cpu().numpy(), Xo) <= tol, f"step {t}: X"
     finally:
         dev.close()
