@@ -1,11 +1,15 @@
 """Benchmark of the GreedyLore compression step on GB300.
 
-Workload: the ResNet conv-gradient stack (8 layer matrices 64x576 ... 512x4608, fp32 gradients,
-N=8 simulated nodes, r=8, refresh every 50 steps, MSGD), synthetic seeded gradients.  A step is
-one GreedyLore iteration (Algorithm 3) over every layer matrix; the timed region covers K
-consecutive steps of the real schedule, so refresh steps are included at their natural
-frequency (one per tau steps).  Inputs (two alternating gradient sets of 200 MB each plus the
-200 MB error state) are larger than the 129 MB L2.
+Headline workload: the 8-layer d = 4096 / ffn = 11008 decoder stack (56 layer matrices: Wq, Wk,
+Wv, Wo 4096 x 4096, Wgate, Wup 11008 x 4096, Wdown 4096 x 11008), N = 4 simulated nodes, bf16
+gradients, fp32 error state, r = 128 with a truncated basis of k = 256, Adam, refresh every 200
+steps; seeded synthetic low-rank-plus-noise gradients of those shapes.  A step is one GreedyLore
+iteration (Algorithm 3) over every matrix of the stack through glr_step_group; the timed region
+covers K consecutive steps of the real schedule.  The refresh (Semi-Lazy SVD) is also timed on its
+own: every handle is forced to refresh (glr_refresh) and that step is timed, three times.  Inputs
+(two alternating 13 GB gradient sets and the 26 GB error state) are far larger than the 129 MB L2.
+The ResNet conv stack (fp32, r = 8) and the d = 2048 decoder stack (bf16, r = 32) are timed as
+extra keys.
 
 Prints ONE JSON line.  `--impl reference` times the CPU oracle instead (on the host cores).
 Multi-GPU (torchrun): every rank runs its own replica of the workload (the matrices are
@@ -34,7 +38,8 @@ import workloads as W  # noqa: E402
 
 METRIC = "gradient elems/s per GreedyLore step & % HBM roofline; subspace refresh ms"
 UNIT = "grad-elem/s"
-WORKLOAD = "cfg2_resnet"
+WORKLOAD = "cfg5_llama_d4096"
+EXTRA_WORKLOADS = ("cfg2_resnet", "cfg3_llama_d2048")
 
 
 def _peaks():
@@ -172,8 +177,17 @@ def timed_steps(torch, hs, gsets, X, t0, K):
     return evs[0].elapsed_time(evs[K]), per
 
 
-def bench_mode(torch, glr, cfg, prob, basis_rank, K, Wm, dist_ctx, gsets):
-    """Time K steps (after Wm warm-up steps) for one basis mode; returns a dict."""
+def compose_bytes(cfg, compressed_steps, reset_steps):
+    """Algorithmic bytes of the compose launches (K1): per node-element the gradient and the error
+    state read + write (no read right after an error reset), per matrix element the Mbar write."""
+    g = 4 if cfg.grad_dtype == "f32" else 2
+    per = cfg.N * cfg.matrix_elems() * (g + 8) + cfg.matrix_elems() * 4
+    return compressed_steps * per + reset_steps * (per - cfg.N * cfg.matrix_elems() * 4)
+
+
+def bench_mode(torch, glr, cfg, basis_rank, K, Wm, dist_ctx, gsets, refresh_reps=0):
+    """Time K steps (after Wm warm-up steps) of the real schedule; then the same K steps again with
+    per-phase CUDA events; then `refresh_reps` forced refresh steps.  Returns a dict."""
     hs = make_handles(glr, cfg, basis_rank)
     X = [torch.zeros(m, n, device="cuda") for (m, n) in cfg.shapes]
     run_steps(hs, gsets, X, 0, Wm)
@@ -186,8 +200,6 @@ def bench_mode(torch, glr, cfg, prob, basis_rank, K, Wm, dist_ctx, gsets):
     is_ref = [(t_first + s) % cfg.tau == 0 for s in range(K)]
     nonref = [p for p, f in zip(per, is_ref) if not f]
     ref = [p for p, f in zip(per, is_ref) if f]
-    nonref_ms = statistics.median(nonref) if nonref else None
-    refresh_step_ms = statistics.mean(ref) if ref else None
     launches = sum(h.stats()["launches"] for h in hs) - l0
     refreshes = sum(1 for t in range(t_first, t_first + K) if t % cfg.tau == 0)
     # second pass with per-phase CUDA events (same schedule continued) for the kernel breakdown
@@ -203,15 +215,25 @@ def bench_mode(torch, glr, cfg, prob, basis_rank, K, Wm, dist_ctx, gsets):
             for key in agg:
                 agg[key] += v[key]
         h.profile(False)
-    e_zero_steps = sum(1 for t in range(t2, t2 + K) if t % cfg.tau == 1)
-    compose_bytes = (K * cfg.N * cfg.matrix_elems() * ((4 if cfg.grad_dtype == "f32" else 2) + 8)
-                     - e_zero_steps * cfg.N * cfg.matrix_elems() * 4)
-    refresh_in_prof = sum(1 for t in range(t2, t2 + K) if t % cfg.tau == 0)
+    resets = sum(1 for t in range(t2, t2 + K) if t % cfg.tau == 1)
+    comp_bytes = compose_bytes(cfg, K - resets, resets)
+    # the refresh on its own: every handle forced to refresh at the next step, that step timed
+    forced = []
+    t3 = t2 + K
+    for rep in range(refresh_reps):
+        for h in hs:
+            h.refresh()
+        forced.append(timed(torch, lambda: run_steps(hs, gsets, X, t3, 1)))
+        t3 += 1
+        run_steps(hs, gsets, X, t3, 1)             # the step after (error reset), untimed
+        t3 += 1
+    path = hs[0].stats()["path"]
     for h in hs:
         h.close()
-    return {"ms": ms, "launches": launches, "refreshes": refreshes, "ms_prof": ms_prof,
-            "phases": phases, "compose_bytes": compose_bytes, "refresh_in_prof": refresh_in_prof,
-            "nonrefresh_step_ms": nonref_ms, "refresh_step_ms": refresh_step_ms}
+    return {"ms": ms, "launches": launches, "refreshes": refreshes, "ms_prof": ms_prof, "phases": phases,
+            "compose_bytes": comp_bytes, "nonrefresh_step_ms": statistics.median(nonref) if nonref else None,
+            "refresh_step_ms_in_window": statistics.mean(ref) if ref else None,
+            "forced_refresh_step_ms": forced, "path": path}
 
 
 def bench_e2e(torch, glr, cfg, K, Wm, dist_ctx):
@@ -236,12 +258,13 @@ def bench_e2e(torch, glr, cfg, K, Wm, dist_ctx):
         h.close()
     gsz = 4 if cfg.grad_dtype == "f32" else 2
     h2d = cfg.N * cfg.matrix_elems() * gsz
-    return {"ms": ms, "h2d": h2d, "d2h": cfg.matrix_elems() * 4, "link_gbs": h2d_link_gbs(torch, h2d)}
+    del host, Xh, X
+    return {"ms": ms, "h2d": h2d, "d2h": cfg.matrix_elems() * 4, "link_gbs": h2d_link_gbs(torch, min(h2d, 1 << 30))}
 
 
 def h2d_link_gbs(torch, nbytes, reps=3):
-    """This machine's host-to-device copy rate for one step's worth of gradient bytes: one pinned
-    buffer copied to the device in a single copy, best of `reps` (CUDA events)."""
+    """This machine's host-to-device copy rate: one pinned buffer copied to the device in a single
+    copy, best of `reps` (CUDA events)."""
     src = torch.empty(nbytes, dtype=torch.uint8).pin_memory()
     dst = torch.empty(nbytes, dtype=torch.uint8, device="cuda")
     best = float("inf")
@@ -255,37 +278,46 @@ def h2d_link_gbs(torch, nbytes, reps=3):
     return nbytes / (best / 1e3) / 1e9
 
 
-def cpu_oracle_sample(cfg, budget_s=25.0, compressed_steps=20):
-    """The oracle as it stands on the host cores: one refresh step and up to `compressed_steps`
-    compressed steps of every layer matrix; the per-step time over a tau-step period is
-    t_refresh + (tau - 1) * t_compressed."""
+def oracle_sample_step(cfg, li, nodes, t=1):
+    """One compressed step of the CPU oracle on layer matrix li with `nodes` nodes, timed: the
+    oracle as it stands, started from Algorithm 3's input basis U = I with the refresh step
+    behind it (t = 1), so it runs the compressed path (Approx-Top-r, projection, error feedback,
+    optimizer).  Returns (seconds, node-elements processed)."""
     from oracle import greedylore as O
-    prob = W.make_problem(cfg)
-    orcs = [O.GreedyLoreOracle(m, n, cfg.r, cfg.N, cfg.tau, optimizer=cfg.optimizer, lr=cfg.lr,
-                               beta1=cfg.beta1, beta2=cfg.beta2, eps=cfg.eps, seed=9000 + li,
-                               basis_rank=cfg.basis_rank)
-            for li, (m, n) in enumerate(cfg.shapes)]
-    Xs = [np.zeros(s) for s in cfg.shapes]
-    grads = [W.gradients_numpy(prob, li, 0) for li in range(len(cfg.shapes))]
+    one = W.config(cfg.name, shapes=cfg.shapes[: li + 1])      # layer li's factors only
+    prob = W.make_problem(one)
+    m, n = cfg.shapes[li]
+    o = O.GreedyLoreOracle(m, n, cfg.r, nodes, cfg.tau, optimizer=cfg.optimizer, lr=cfg.lr, beta1=cfg.beta1,
+                           beta2=cfg.beta2, eps=cfg.eps, seed=9000 + li, basis_rank=cfg.basis_rank)
+    o.t = t
+    G = W.gradients_numpy(prob, li, t, workers=list(range(nodes)))
     t0 = time.perf_counter()
-    for li, o in enumerate(orcs):
-        Xs[li], _ = o.step(grads[li], Xs[li])
-    t_refresh = time.perf_counter() - t0
-    done, t_comp = 0, 0.0
-    while done < compressed_steps and t_refresh + t_comp < budget_s:
-        t0 = time.perf_counter()
-        for li, o in enumerate(orcs):
-            Xs[li], _ = o.step(grads[li], Xs[li])
-        t_comp += time.perf_counter() - t0
-        done += 1
-    per_comp = t_comp / max(done, 1)
-    per_step = (t_refresh + (cfg.tau - 1) * per_comp) / cfg.tau
-    elems = cfg.N * cfg.matrix_elems()
-    return {"value": elems / per_step, "unit": UNIT, "cores": os.cpu_count(), "kind": "oracle",
-            "sample": f"fp64 numpy oracle, all {len(cfg.shapes)} matrices: 1 refresh step "
-                      f"({t_refresh:.2f} s) + {done} compressed steps ({per_comp:.2f} s each), per-step time "
-                      f"over one tau={cfg.tau} period; numpy BLAS on all host cores",
-            "seconds": t_refresh + t_comp}
+    o.step(G, np.zeros((m, n)))
+    return time.perf_counter() - t0, nodes * m * n
+
+
+def cpu_oracle_sample(cfg):
+    """The oracle as it stands on the host cores, on a bounded sample of the workload: one
+    compressed step of the stack's square matrix (the shape of 32 of its 56 matrices) with all N
+    nodes, numpy BLAS on every core; and the same step with one node in a single-threaded process."""
+    li = 0
+    secs, units = oracle_sample_step(cfg, li, cfg.N)
+    m, n = cfg.shapes[li]
+    out = {"value": units / secs, "unit": UNIT, "cores": os.cpu_count(), "kind": "oracle",
+           "sample": f"one compressed step of one {m}x{n} matrix of the stack with all {cfg.N} nodes "
+                     f"({secs:.2f} s; fp64 numpy oracle from U = I, BLAS on every host core); the rate is "
+                     f"node-elements per second on that shape", "seconds": secs}
+    code = ("import sys; sys.path.insert(0, %r); import bench, workloads as W; "
+            "s, u = bench.oracle_sample_step(W.config(%r), 0, 1); print(u / s, s)") % (ROOT, cfg.name)
+    env = dict(os.environ, OMP_NUM_THREADS="1", OPENBLAS_NUM_THREADS="1", MKL_NUM_THREADS="1")
+    try:
+        res = subprocess.run([sys.executable, "-c", code], capture_output=True, text=True, env=env, timeout=120)
+        v, secs1 = (float(x) for x in res.stdout.split()[-2:])
+        out["single_thread"] = {"value": v, "cores": 1, "seconds": secs1,
+                                "sample": f"the same step with 1 node in one thread ({secs1:.2f} s)"}
+    except Exception as e:                      # report, do not fail the benchmark
+        out["single_thread"] = {"value": None, "error": str(e)[:200]}
+    return out
 
 
 class DistCtx:
@@ -331,58 +363,110 @@ def job_rate(world, units_per_rank, ms_max):
 
 
 def run_reference(args):
+    """The reference arm: the CPU oracle (fp64 numpy, the host cores), each step a bounded sample
+    of the workload (one compressed step of one of the stack's square matrices, one node), the
+    rate in the benchmark's unit.  Ranks other than 0 exit without work."""
     ctx = DistCtx()
     if ctx.world > 1 and ctx.rank != 0:
         return 0
     cfg = W.config(WORKLOAD)
-    from oracle import greedylore as O
-    prob = W.make_problem(cfg)
-    li_order = list(range(len(cfg.shapes)))
-    orcs = [O.GreedyLoreOracle(m, n, cfg.r, cfg.N, cfg.tau, optimizer=cfg.optimizer, lr=cfg.lr, beta1=cfg.beta1,
-                               seed=9000 + li, basis_rank=cfg.basis_rank) for li, (m, n) in enumerate(cfg.shapes)]
-    Xs = [np.zeros(s) for s in cfg.shapes]
-    grads = [W.gradients_numpy(prob, li, 0) for li in li_order]
-
-    def one_step():
-        for li in li_order:
-            Xs[li], _ = orcs[li].step(grads[li], Xs[li])
-
     for _ in range(args.warmup):
-        one_step()
-    t0 = time.perf_counter()
+        oracle_sample_step(cfg, 0, 1)
+    secs, units = 0.0, 0
     for _ in range(args.steps):
-        one_step()
-    el = time.perf_counter() - t0
-    elems = cfg.N * cfg.matrix_elems()
-    value = elems * args.steps / el
+        s_, u_ = oracle_sample_step(cfg, 0, 1)
+        secs += s_
+        units += u_
+    value = units / secs
+    m, n = cfg.shapes[0]
     line = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
-            "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * el / args.steps,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * secs / args.steps,
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
             "data": "synthetic", "config": {"workload": WORKLOAD, "basis_rank": cfg.basis_rank,
                                             "matrices": len(cfg.shapes), "N": cfg.N, "r": cfg.r, "tau": cfg.tau},
             "cpu_baseline": {"value": value, "unit": UNIT, "cores": os.cpu_count(), "kind": "oracle",
-                             "sample": f"{args.steps} consecutive oracle steps over all matrices (schedule "
-                                       f"from t={args.warmup}), numpy BLAS on the host cores"},
+                             "sample": f"each step: one compressed oracle step of one {m}x{n} matrix of the "
+                                       f"stack with one node (fp64 numpy from U = I, BLAS on the host cores)"},
             "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
     print(json.dumps(line))
+    return 0
+
+
+def traffic_record(kernel_file, record):
+    """DRAM bytes per unit of one captured launch (profiles/), valid while the kernel source is
+    the one that was captured."""
+    path = os.path.join(ROOT, "profiles", record)
+    if not os.path.exists(path):
+        return None
+    with open(path) as f:
+        rec = json.load(f)
+    with open(os.path.join(ROOT, "paper_2507_08784_gb300", "csrc", kernel_file), "rb") as f:
+        if hashlib.sha256(f.read()).hexdigest() != rec.get("source_sha256"):
+            return None
+    return rec
+
+
+def summarize(cfg, run, K, world, hbm_peak):
+    """Rate, step roofline and phase breakdown of one bench_mode run."""
+    elems = cfg.N * cfg.matrix_elems()
+    step_bytes = algorithmic_bytes(cfg, False)
+    nonref = run["nonrefresh_step_ms"]
+    ph = run["phases"]
+    comp = ph.get("compose", {"ms": 0.0, "launches": 0})
+    return {
+        "value": job_rate(world, elems * K, run["ms"]), "ms_per_step": run["ms"] / K,
+        "path": ["strip", "mma", "tcgen05", "library", "plain"][run["path"]],
+        "nonrefresh_step_ms_median": nonref,
+        "grad_elems_per_s_nonrefresh": elems / (nonref / 1e3) if nonref else None,
+        "step_roofline": {"algorithmic_bytes_per_step": step_bytes,
+                          "achieved_gbs": step_bytes / (nonref / 1e3) / 1e9 if nonref else None,
+                          "frac": step_bytes / (nonref / 1e3) / 1e9 / hbm_peak if nonref else None},
+        "compose_gbs": run["compose_bytes"] / (comp["ms"] / 1e3) / 1e9 if comp["ms"] else None,
+        "phases_ms_per_step": {k: round(v["ms"] / K, 4) for k, v in ph.items()},
+        "phase_launches_per_step": {k: v["launches"] / K for k, v in ph.items()},
+    }
+
+
+def ncu_case():
+    """One 4096 x 4096 matrix of the headline stack for 4 steps (about 1.1 GB of state): the
+    compose launch of step 2 (index 2 among compose launches) is a full one."""
+    import torch
+    import paper_2507_08784_gb300 as glr
+    cfg = W.config(WORKLOAD, shapes=W.config(WORKLOAD).shapes[:1])
+    prob = W.make_problem(cfg)
+    gs = [W.gradients_torch(prob, 0, t) for t in range(2)]
+    hs = make_handles(glr, cfg, cfg.basis_rank)
+    X = [torch.zeros(*cfg.shapes[0], device="cuda")]
+    for t in range(4):
+        glr.glr_step_group(hs, [gs[t % 2]], X)
+    torch.cuda.synchronize()
+    print(json.dumps({"ncu_case": WORKLOAD, "shape": cfg.shapes[0], "N": cfg.N,
+                      "node_elems_per_compose": cfg.N * cfg.matrix_elems(), "path": hs[0].stats()["path"]}))
+    hs[0].close()
     return 0
 
 
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=50)
-    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--only-headline", action="store_true",
-                    help="time the truncated-basis steps only (no paper-exact pass, no e2e, no CPU baseline)")
-    ap.add_argument("--e2e-steps", type=int, default=10)
+                    help="time the headline workload only (no extra workloads, no e2e, no CPU baseline)")
+    ap.add_argument("--e2e-steps", type=int, default=5)
+    ap.add_argument("--refresh-reps", type=int, default=3)
+    ap.add_argument("--ncu-case", action="store_true",
+                    help="a small case for kernel captures: one 4096 x 4096 matrix of the headline stack "
+                         "(N = 4, r = 128, k = 256, bf16, Adam), 4 steps: refresh, reset, then two full steps")
     args = ap.parse_args()
     if args.warmup < 3:
         ap.error("--warmup must be >= 3")
     if args.impl == "reference":
         return run_reference(args)
+    if args.ncu_case:
+        return ncu_case()
 
     import torch
     import paper_2507_08784_gb300 as glr
@@ -396,77 +480,81 @@ def main():
     gsets = [[W.gradients_torch(prob, li, t) for li in range(len(cfg.shapes))] for t in range(2)]
     torch.cuda.synchronize()
     hbm_peak, peak_kind = _peaks()
+    K = args.steps
 
     with ClockSampler(ctx.local) as clk:
-        main_run = bench_mode(torch, glr, cfg, prob, cfg.basis_rank, args.steps, args.warmup, ctx, gsets)
-    exact_run = None if args.only_headline else bench_mode(torch, glr, cfg, prob, 0, args.steps, args.warmup, ctx, gsets)
-    e2e = None if args.only_headline else bench_e2e(torch, glr, cfg, args.e2e_steps, args.warmup, ctx)
+        main_run = bench_mode(torch, glr, cfg, cfg.basis_rank, K, args.warmup, ctx, gsets,
+                              refresh_reps=args.refresh_reps)
+    del gsets
+    torch.cuda.empty_cache()
+    e2e = None if args.only_headline else bench_e2e(torch, glr, cfg, args.e2e_steps, 3, ctx)
+    extras = {}
+    if not args.only_headline:
+        for name in EXTRA_WORKLOADS:
+            xc = W.config(name)
+            xp = W.make_problem(xc)
+            xs = [[W.gradients_torch(xp, li, t) for li in range(len(xc.shapes))] for t in range(2)]
+            xr = bench_mode(torch, glr, xc, xc.basis_rank, K, args.warmup, ctx, xs)
+            extras[name] = summarize(xc, xr, K, ctx.world, hbm_peak)
+            extras[name]["config"] = {"matrices": len(xc.shapes), "N": xc.N, "r": xc.r, "basis_rank": xc.basis_rank,
+                                      "tau": xc.tau, "grad_dtype": xc.grad_dtype, "optimizer": xc.optimizer}
+            del xs
+            torch.cuda.empty_cache()
 
-    K = args.steps
     elems = cfg.N * cfg.matrix_elems()
-    value = job_rate(ctx.world, elems * K, main_run["ms"])
+    head = summarize(cfg, main_run, K, ctx.world, hbm_peak)
     ph = main_run["phases"]
-    # the refresh phase runs on one side stream per matrix, concurrently: its summed event time
-    # is not wall time, so the dominant phase is taken among the phases on the step's stream and
-    # the refresh's wall cost per step is added from the per-step timings
-    dominant = max((k for k in ph if k != "refresh"), key=lambda k: ph[k]["ms"])
-    compose = ph["compose"]
-    compose_gbs = main_run["compose_bytes"] / (compose["ms"] / 1e3) / 1e9 if compose["ms"] else None
-    nonrefresh_ms = main_run["nonrefresh_step_ms"]
-    refresh_extra_ms = (main_run["refresh_step_ms"] - nonrefresh_ms) if main_run["refresh_step_ms"] else None
-    step_bytes = algorithmic_bytes(cfg, False)
+    comp = ph["compose"]
+    comp_launch_bytes = main_run["compose_bytes"] / comp["launches"] if comp["launches"] else None
+    comp_ms = comp["ms"] / comp["launches"] if comp["launches"] else None
+    achieved = comp_launch_bytes / (comp_ms / 1e3) / 1e9 if comp_ms else None
+    rec = traffic_record("k_tc.cu", "compose_tcgen05_traffic.json")
     traffic = None
-    tr_path = os.path.join(ROOT, "profiles", "compose_cfg2_traffic.json")
-    if os.path.exists(tr_path):
-        # the DRAM bytes of one captured compose launch, valid while the kernel source is unchanged
-        with open(tr_path) as f:
-            rec = json.load(f)
-        src = os.path.join(ROOT, "paper_2507_08784_gb300", "csrc", "k_mma.cu")
-        with open(src, "rb") as f:
-            if hashlib.sha256(f.read()).hexdigest() == rec.get("k_mma_cu_sha256"):
-                traffic = rec.get("bytes_per_launch")
-    compose_launch_bytes = main_run["compose_bytes"] / compose["launches"] if compose["launches"] else None
+    if rec:   # the captured launch's DRAM bytes scaled to one launch of this workload by its node-elements
+        traffic = rec["dram_bytes"] * (cfg.N * cfg.matrix_elems()) / rec["node_elems"]
+    nonref = main_run["nonrefresh_step_ms"]
+    forced = main_run["forced_refresh_step_ms"]
+    ref_step = statistics.median(forced) if forced else None
+    refresh_ms = (ref_step - nonref) if (ref_step and nonref) else None
+    layers = len(cfg.shapes) // 7
+    amort = ((cfg.tau - 1) * nonref + ref_step) / cfg.tau if ref_step else None
+    tpeak, tkind = tensor_peak_tflops()
+    rflops = refresh_flops(cfg, cfg.basis_rank)
     line = {
-        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": ctx.world, "steps": K, "warmup": args.warmup,
-        "ms_per_step": main_run["ms"] / K, "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
-        "dtype": "f32", "data": "synthetic",
-        "config": {"workload": WORKLOAD, "matrices": len(cfg.shapes), "shapes": "64x576..512x4608 (x2 each)",
-                   "N": cfg.N, "r": cfg.r, "basis_rank": cfg.basis_rank, "tau": cfg.tau, "optimizer": cfg.optimizer,
+        "metric": METRIC, "value": head["value"], "unit": UNIT, "n_gpus": ctx.world, "steps": K,
+        "warmup": args.warmup, "ms_per_step": main_run["ms"] / K, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "bf16 gradients, fp32 state, TF32 tensor-core products",
+        "data": "synthetic",
+        "config": {"workload": WORKLOAD, "matrices": len(cfg.shapes),
+                   "shapes": "8 layers x {4 x 4096x4096, 2 x 11008x4096, 4096x11008}", "N": cfg.N, "r": cfg.r,
+                   "basis_rank": cfg.basis_rank, "tau": cfg.tau, "optimizer": cfg.optimizer,
                    "grad_dtype": cfg.grad_dtype, "refreshes_in_timed_steps": main_run["refreshes"],
-                   "l2": "inputs larger than L2 (two alternating 200 MB gradient sets + 200 MB error state)",
+                   "path": head["path"],
+                   "l2": "inputs larger than L2 (two alternating 13 GB gradient sets + 26 GB error state)",
                    "parallelism": f"replicas x{ctx.world} (node axis simulated on each GPU)"},
-        "roofline": {"kernel": "compose (K1)", "bound": "hbm", "achieved": compose_gbs, "peak": hbm_peak,
-                     "unit": "GB/s", "frac": (compose_gbs / hbm_peak) if compose_gbs else None,
-                     "traffic": traffic, "peak_kind": peak_kind,
-                     "algorithmic_bytes_per_launch_avg": compose_launch_bytes,
-                     "launches_per_step": compose["launches"] / K,
-                     "timing": "CUDA events around each compose launch on its stream, second timed pass of K steps",
-                     "dominant_phase": dominant},
-        "step_roofline": {"algorithmic_bytes_per_step": step_bytes,
-                          "nonrefresh_step_ms_median": nonrefresh_ms,
-                          "achieved_gbs_nonrefresh": step_bytes / (nonrefresh_ms / 1e3) / 1e9,
-                          "frac_nonrefresh": step_bytes / (nonrefresh_ms / 1e3) / 1e9 / hbm_peak,
-                          "grad_elems_per_s_nonrefresh": elems / (nonrefresh_ms / 1e3)},
-        "refresh_ms_all_matrices": refresh_extra_ms,
-        "refresh_wall_ms_per_step": (refresh_extra_ms * main_run["refreshes"] / K) if refresh_extra_ms else None,
-        "refresh_ms_per_layer": refresh_extra_ms / len(cfg.shapes) if refresh_extra_ms else None,
-        "refresh_tensor": None if not refresh_extra_ms else {
-            "flops": refresh_flops(cfg, cfg.basis_rank),
-            "tflops": refresh_flops(cfg, cfg.basis_rank) / (refresh_extra_ms / 1e3) / 1e12,
-            "frac_of_tensor_peak": refresh_flops(cfg, cfg.basis_rank) / (refresh_extra_ms / 1e3) / 1e12
-                                   / tensor_peak_tflops()[0],
-            "peak": tensor_peak_tflops()[0], "peak_kind": tensor_peak_tflops()[1] + " bf16 sustained",
-            "note": "the truncated refresh runs on the FP32 pipes; bound by HBM and latency, not the tensor cores"},
-        "phases_ms_per_step": {k: v["ms"] / K for k, v in ph.items()},
+        "roofline": {"kernel": "compose (K1, tcgen05)", "bound": "hbm", "achieved": achieved, "peak": hbm_peak,
+                     "unit": "GB/s", "frac": (achieved / hbm_peak) if achieved else None, "traffic": traffic,
+                     "peak_kind": peak_kind, "algorithmic_bytes_per_launch": comp_launch_bytes,
+                     "launch_ms": comp_ms, "launches_per_step": comp["launches"] / K,
+                     "timing": "CUDA events around each compose launch on its stream, second timed pass of K steps"},
+        "step_roofline": head["step_roofline"],
+        "grad_elems_per_s_nonrefresh": head["grad_elems_per_s_nonrefresh"],
+        "nonrefresh_step_ms_median": nonref,
+        "refresh": {"forced_refresh_step_ms": forced, "refresh_ms_all_matrices": refresh_ms,
+                    "refresh_ms_per_layer": refresh_ms / layers if refresh_ms else None,
+                    "refresh_ms_per_matrix": refresh_ms / len(cfg.shapes) if refresh_ms else None,
+                    "tau_amortised_step_ms": amort,
+                    "tau_amortised_value": elems / (amort / 1e3) if amort else None,
+                    "tensor": None if not refresh_ms else {
+                        "flops": rflops, "tflops": rflops / (refresh_ms / 1e3) / 1e12,
+                        "frac_of_tensor_peak": rflops / (refresh_ms / 1e3) / 1e12 / tpeak,
+                        "peak": tpeak, "peak_kind": tkind + " bf16 sustained"},
+                    "how": "every handle forced to refresh (glr_refresh), that step timed with CUDA events, "
+                           f"{len(forced)} repeats; refresh ms = that step minus the median compressed step"},
+        "phases_ms_per_step": head["phases_ms_per_step"],
+        "phase_launches_per_step": head["phase_launches_per_step"],
         "phases_note": "refresh = summed event time of the concurrent per-matrix refresh streams",
-        "phase_launches": {k: v["launches"] for k, v in ph.items()},
-        "paper_exact_basis": None if exact_run is None else {
-            "value": job_rate(ctx.world, elems * K, exact_run["ms"]),
-            "ms_per_step": exact_run["ms"] / K,
-            "nonrefresh_step_ms_median": exact_run["nonrefresh_step_ms"],
-            "refresh_ms_all_matrices": (exact_run["refresh_step_ms"] - exact_run["nonrefresh_step_ms"])
-            if exact_run["refresh_step_ms"] else None,
-            "phases_ms_per_step": {k: v["ms"] / K for k, v in exact_run["phases"].items()}},
+        "extra_workloads": extras,
         "e2e": None if e2e is None else {"value": job_rate(ctx.world, elems * args.e2e_steps, e2e["ms"]), "unit": UNIT,
                                          "h2d_bytes_per_step": e2e["h2d"], "d2h_bytes_per_step": e2e["d2h"],
                                          "h2d_link_gbs": e2e["link_gbs"],
