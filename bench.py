@@ -427,9 +427,10 @@ def summarize(cfg, run, K, world, hbm_peak):
     }
 
 
-def ncu_case():
+def ncu_case(refresh=False):
     """One 4096 x 4096 matrix of the headline stack for 4 steps (about 1.1 GB of state): the
-    compose launch of step 2 (index 2 among compose launches) is a full one."""
+    compose launch of step 2 (index 2 among compose launches) is a full one; with refresh, a
+    fifth step forced to refresh."""
     import torch
     import paper_2507_08784_gb300 as glr
     cfg = W.config(WORKLOAD, shapes=W.config(WORKLOAD).shapes[:1])
@@ -439,6 +440,9 @@ def ncu_case():
     X = [torch.zeros(*cfg.shapes[0], device="cuda")]
     for t in range(4):
         glr.glr_step_group(hs, [gs[t % 2]], X)
+    if refresh:                                    # then one forced refresh step
+        hs[0].refresh()
+        glr.glr_step_group(hs, [gs[0]], X)
     torch.cuda.synchronize()
     print(json.dumps({"ncu_case": WORKLOAD, "shape": cfg.shapes[0], "N": cfg.N,
                       "node_elems_per_compose": cfg.N * cfg.matrix_elems(), "path": hs[0].stats()["path"]}))
@@ -457,16 +461,17 @@ def main():
                     help="time the headline workload only (no extra workloads, no e2e, no CPU baseline)")
     ap.add_argument("--e2e-steps", type=int, default=5)
     ap.add_argument("--refresh-reps", type=int, default=3)
-    ap.add_argument("--ncu-case", action="store_true",
+    ap.add_argument("--ncu-case", nargs="?", const="steps", choices=["steps", "refresh"],
                     help="a small case for kernel captures: one 4096 x 4096 matrix of the headline stack "
-                         "(N = 4, r = 128, k = 256, bf16, Adam), 4 steps: refresh, reset, then two full steps")
+                         "(N = 4, r = 128, k = 256, bf16, Adam), 4 steps: refresh, reset, then two full "
+                         "steps; 'refresh' adds a fifth step forced to refresh")
     args = ap.parse_args()
     if args.warmup < 3:
         ap.error("--warmup must be >= 3")
     if args.impl == "reference":
         return run_reference(args)
     if args.ncu_case:
-        return ncu_case()
+        return ncu_case(args.ncu_case == "refresh")
 
     import torch
     import paper_2507_08784_gb300 as glr

@@ -48,7 +48,7 @@ extern "C" {
 #define GLR_EINVAL     -1   /* bad argument (sizes, null pointer, unknown enum value)      */
 #define GLR_ENOMEM     -2   /* a device or host allocation failed                          */
 #define GLR_ECUDA      -3   /* a CUDA runtime call or kernel launch failed                 */
-#define GLR_ENUMERIC   -4   /* the refresh could not orthonormalise its basis              */
+#define GLR_ENUMERIC   -4   /* the refresh could not orthonormalise its basis (glr_get_stats) */
 #define GLR_ENONFINITE -5   /* a NaN or Inf reached the node-mean gradient (glr_get_stats)  */
 #define GLR_ETIMEOUT   -6   /* a bounded device-side wait gave up (reported by glr_get_stats) */
 
@@ -133,6 +133,8 @@ typedef struct glr_stats {
     int32_t path;                   /* kernel family that runs the step: GLR_PATH_*          */
     int32_t nonfinite;              /* warps of the compose pass that found a NaN or Inf in  *
                                      * the node-mean gradient since creation (0: all finite) */
+    int32_t numeric_failures;       /* refresh factorisations that could not be completed    */
+    int32_t reserved;
 } glr_stats;
 
 /* Kernel families (glr_stats.path), chosen by glr_create from the shape and schedule.       */
@@ -222,8 +224,9 @@ int glr_step_group_host(glr_handle* const* handles, int32_t count, const void* c
  * position (t, the refresh period, a pending forced selection), the basis, P, the error state
  * B, the optimizer moments and every other buffer glr_create allocated.  It runs on `stream`
  * after the work already queued there and synchronises it.  glr_load restores such a checkpoint
- * into a handle created with the same m, n, r, N, basis rank, gradient dtype, optimizer and
- * refresh mode (GLR_EINVAL otherwise, or when the buffer is not a checkpoint or is truncated),
+ * into a handle created with the same m, n, r, N, basis rank, gradient dtype, optimizer,
+ * refresh mode and seed (GLR_EINVAL otherwise, or when the buffer is not a checkpoint, is
+ * truncated, or its header names buffers or a pending selection this handle cannot hold),
  * also synchronising `stream`; stepping the restored handle continues exactly as the saved one
  * would have (same results bit for bit).  The format is this library's own (host byte order).  */
 int glr_state_size(const glr_handle* h, int64_t* bytes);
@@ -239,9 +242,11 @@ int glr_refresh(glr_handle* h);
 /* Counters (see glr_stats).  Reads the handle's device flags with a blocking copy, so it
  * waits for work already queued on the device.  Returns GLR_ETIMEOUT (with out filled) when a
  * bounded wait inside a kernel of this handle's launches has given up since creation (the
- * results of those steps are not valid), else GLR_ENONFINITE when a compose pass found a NaN
- * or Inf in the node-mean gradient (a node sent a non-finite gradient, or the error state
- * overflowed), else GLR_OK.                                                                */
+ * results of those steps are not valid), else GLR_ENUMERIC when a refresh met a Gram matrix it
+ * could not factor (a rank-deficient or zero node mean, e.g. all-zero gradients: the basis of
+ * that refresh is not orthonormal), else GLR_ENONFINITE when a compose pass found a NaN or Inf
+ * in the node-mean gradient (a node sent a non-finite gradient, or the error state overflowed),
+ * else GLR_OK.                                                                             */
 int glr_get_stats(const glr_handle* h, glr_stats* out);
 
 /* Message of the last failure on h (or of the last failed glr_create when h is NULL);
@@ -279,6 +284,13 @@ int glr_profile_read(glr_handle* h, glr_profile* out, int32_t reset);
 /* Override the selection of the next compressed step with J_host (r distinct indices in
  * [0, m')), instead of Algorithm 2.  One-shot.                                           */
 int glr_force_selection(glr_handle* h, const int32_t* J_host);
+
+/* Test aid for the bounded device waits: one kernel on `stream` waits, with the same bounded
+ * polling loop as the pipeline kernels, on an mbarrier that nothing arrives on; after `polls`
+ * polls (1 <= polls <= 2^24) the wait gives up and counts the event in the handle's flags, and
+ * the kernel returns normally (the device stays usable).  glr_get_stats then reports
+ * GLR_ETIMEOUT, as it does after a real stuck wait.  Errors: GLR_EINVAL, GLR_ECUDA.       */
+int glr_test_expire_wait(glr_handle* h, int32_t polls, void* stream);
 
 /* ---- selection without device allocation ------------------------------------------------ */
 

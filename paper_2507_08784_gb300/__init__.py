@@ -20,7 +20,7 @@ from ._lib import (GLR_ADAM, GLR_ADAMW, GLR_ALG3, GLR_ALG4, GLR_AMSGRAD, GLR_BF1
 
 __all__ = ["GlrError", "make_schedule", "glr_create", "glr_destroy", "glr_step", "glr_step_group",
            "glr_step_group_host", "glr_step_host", "glr_save", "glr_load", "glr_refresh", "glr_get_stats", "glr_last_error", "glr_get_error", "glr_get_selection",
-           "glr_get_basis", "glr_set_basis", "glr_force_selection", "glr_profile_enable",
+           "glr_get_basis", "glr_set_basis", "glr_force_selection", "glr_test_expire_wait", "glr_profile_enable",
            "glr_profile_read", "glr_select_noalloc", "GreedyLore", "load"]
 
 
@@ -193,6 +193,11 @@ def glr_force_selection(h, J) -> None:
     _check(load().glr_force_selection(h, arr.ctypes.data), h)
 
 
+def glr_test_expire_wait(h, polls: int, stream=None) -> None:
+    """Let one bounded device wait run out on the handle's flags (test aid, see glr.h)."""
+    _check(load().glr_test_expire_wait(h, int(polls), _stream_ptr(stream)), h)
+
+
 def glr_profile_enable(h, enable: bool = True) -> None:
     _check(load().glr_profile_enable(h, 1 if enable else 0), h)
 
@@ -206,8 +211,22 @@ def glr_profile_read(h, reset: bool = False) -> dict:
 
 def glr_select_noalloc(U: torch.Tensor, Mbar: torch.Tensor, seed: int, t: int, r: int,
                        lambda_out: torch.Tensor, J_out: torch.Tensor, stream=None) -> None:
-    """Approx-Top-r selection into caller buffers; the library allocates nothing (see glr.h)."""
+    """Approx-Top-r selection into caller buffers; the library allocates nothing (see glr.h).
+    The library cannot see the buffers' sizes, so they are checked here: U (m' x m') and Mbar
+    (m' x n') contiguous fp32 on the GPU, lambda_out at least m' fp32, J_out at least r int32."""
+    if Mbar.dim() != 2:
+        raise ValueError("Mbar must be a 2-D m' x n' tensor")
     mp, np_ = Mbar.shape
+    for name, x in (("U", U), ("Mbar", Mbar)):
+        if not (x.is_cuda and x.dtype == torch.float32 and x.is_contiguous()):
+            raise ValueError(f"{name} must be a contiguous float32 CUDA tensor")
+    if tuple(U.shape) != (mp, mp):
+        raise ValueError(f"U must be {mp} x {mp}")
+    if not (lambda_out.is_cuda and lambda_out.dtype == torch.float32 and lambda_out.is_contiguous()
+            and lambda_out.numel() >= mp):
+        raise ValueError(f"lambda_out must be a contiguous float32 CUDA tensor of at least {mp} elements")
+    if not (J_out.is_cuda and J_out.dtype == torch.int32 and J_out.is_contiguous() and J_out.numel() >= r):
+        raise ValueError(f"J_out must be a contiguous int32 CUDA tensor of at least {r} elements")
     _check(load().glr_select_noalloc(mp, np_, r, U.data_ptr(), Mbar.data_ptr(), seed & (2 ** 64 - 1), t,
                                      lambda_out.data_ptr(), J_out.data_ptr(), _stream_ptr(stream)))
 

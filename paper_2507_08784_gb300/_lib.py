@@ -58,6 +58,8 @@ class GlrStats(ctypes.Structure):
         ("launches", ctypes.c_int64),
         ("path", ctypes.c_int32),
         ("nonfinite", ctypes.c_int32),
+        ("numeric_failures", ctypes.c_int32),
+        ("reserved", ctypes.c_int32),
     ]
 
 
@@ -96,6 +98,7 @@ _SIGNATURES = {
     "glr_get_basis": (ctypes.c_int, [ctypes.c_void_p, ctypes.c_void_p, ctypes.c_void_p]),
     "glr_set_basis": (ctypes.c_int, [ctypes.c_void_p, ctypes.c_void_p, ctypes.c_void_p]),
     "glr_force_selection": (ctypes.c_int, [ctypes.c_void_p, ctypes.c_void_p]),
+    "glr_test_expire_wait": (ctypes.c_int, [ctypes.c_void_p, ctypes.c_int32, ctypes.c_void_p]),
     "glr_profile_enable": (ctypes.c_int, [ctypes.c_void_p, ctypes.c_int32]),
     "glr_profile_read": (ctypes.c_int, [ctypes.c_void_p, ctypes.POINTER(GlrProfile), ctypes.c_int32]),
     "glr_select_noalloc": (ctypes.c_int, [ctypes.c_int32, ctypes.c_int32, ctypes.c_int32, ctypes.c_void_p,

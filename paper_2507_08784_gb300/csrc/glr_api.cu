@@ -383,7 +383,7 @@ int glr_create(int64_t m, int64_t n, int32_t r, int32_t N, const glr_schedule* s
     if (s->optimizer != GLR_MSGD) A(&h->Vo, galore ? (size_t)r * NP : (size_t)m * n);
     if (s->optimizer == GLR_AMSGRAD) A(&h->amsv, 2);
     if (galore) A(&h->galr, (size_t)r * NP);
-    A(&h->dflags, 6);
+    A(&h->dflags, 8);
     A(&h->gemm_ws, (size_t)kGemmWsFloats);
     // the first path with library products when the rank-r products are large
     h->tc = !h->fused && !h->tcl && mp % 4 == 0 && np % 4 == 0 &&
@@ -414,6 +414,8 @@ int glr_create(int64_t m, int64_t n, int32_t r, int32_t N, const glr_schedule* s
             A(&h->powG, std::max(nt, nr) * KM * KM);
             A(&h->powS, K * K);
             h->pow_ok = 1;
+        } else {
+            A(&h->jpart, (size_t)2 * kGroupMax * kJacobiMaxGrid);   // the grouped k x k Jacobi (refresh)
         }
     }
     if (rc == GLR_OK && h->tcl) rc = tcl_alloc(h);
@@ -964,25 +966,19 @@ int step_group(std::vector<StepPlan>& plans, cudaStream_t st) {
     // Refreshes (Semi-Lazy SVD) of different matrices are independent: each runs on its
     // handle's side stream after the compose pass, overlapping the others and the selection
     // work of the non-refreshing matrices; the main stream joins them before P is built.
-    std::vector<glr_handle*> refreshing, grouped, exact;
+    std::vector<glr_handle*> refreshing, grouped, exact, trunc;
     for (StepPlan& p : plans) {
         if (!p.refresh) continue;
         glr_handle* h = p.h;
         GLR_CK(h, cudaEventRecord(h->rfork, st));
         GLR_CK(h, cudaStreamWaitEvent(h->rstream, h->rfork, 0));
         refreshing.push_back(h);
-        if (h->pow_ok) grouped.push_back(h);
-        if (h->exact) exact.push_back(h);
+        (h->pow_ok ? grouped : h->exact ? exact : trunc).push_back(h);
     }
     if (!grouped.empty() && (rc = refresh_grouped(grouped)) != GLR_OK) return rc;
     if (!exact.empty() && (rc = refresh_exact_grouped(exact)) != GLR_OK) return rc;
-    for (glr_handle* h : refreshing) {
-        if (!h->pow_ok && !h->exact) {
-            PhaseScope ps(h, GLR_PH_REFRESH, h->rstream);
-            if ((rc = do_refresh(h, h->rstream)) != GLR_OK) return rc;
-        }
-        GLR_CK(h, cudaEventRecord(h->rdone, h->rstream));
-    }
+    if (!trunc.empty() && (rc = refresh_trunc_grouped(trunc)) != GLR_OK) return rc;
+    for (glr_handle* h : refreshing) GLR_CK(h, cudaEventRecord(h->rdone, h->rstream));
     for (StepPlan& p : plans)
         if ((rc = select_phase(p, st)) != GLR_OK) return rc;
     if (!tcl.empty() && (rc = tcl_lambda(tcl, st)) != GLR_OK) return rc;

@@ -38,8 +38,9 @@ struct glr_handle {
     float *YT = nullptr, *YtT = nullptr;   // k x transposed_pitch(m') copies of Y and Yt for the fused kernel
     float *YF = nullptr, *YtF = nullptr;   // Y and Yt in fragment order for the tensor-core kernel
     int* dflags = nullptr;   // [0] Cholesky restarts, [1] Jacobi sweeps of the last refresh,
-                             // [2] bounded device waits of the compose kernel that gave up,
-                             // [4..5] the cooperative Jacobi's grid barrier
+                             // [2] bounded device waits that gave up, [3] warps that found a NaN /
+                             // Inf in Mbar, [4..5] the cooperative Jacobi's grid barrier, [6]
+                             // refresh factorisations that failed (GLR_ENUMERIC), [7] unused
     float* gemm_ws = nullptr;   // split-K partial tiles of the refresh GEMMs
     // Large plain products (>= 2^26 flops) go to cuBLAS: one library handle for the step stream
     // and one for the refresh stream (a handle's workspace must not serve two streams at once).
@@ -197,9 +198,11 @@ bool encode_map(CUtensorMap* map, CUtensorMapDataType dtype, const void* base, i
 int cholqr(glr_handle* h, float*& A, float*& tmp, int rows, cudaStream_t st);
 int wy_from_Q(glr_handle* h, cudaStream_t st);
 int refresh_tail(glr_handle* h, cudaStream_t st);
+int refresh_finish(glr_handle* h, cudaStream_t st);
+int refresh_power(glr_handle* h, cudaStream_t st);
+int refresh_trunc_grouped(std::vector<glr_handle*>& hs);
 int refresh_grouped(std::vector<glr_handle*>& hs);
 int refresh_exact_grouped(std::vector<glr_handle*>& hs);
-int do_refresh(glr_handle* h, cudaStream_t st);
 
 }  // namespace host
 }  // namespace glr

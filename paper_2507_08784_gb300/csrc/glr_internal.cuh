@@ -435,6 +435,8 @@ int compose_bn();
 // dst (cols x ldd) = src^T rounded to TF32 (src row-major rows x cols, leading dimension lds)
 cudaError_t transpose_round(float* dst, int ldd, const float* src, int rows, int cols, int lds, cudaStream_t st);
 cudaError_t round_tf32(float* p, int64_t n, cudaStream_t st);
+// One wait of the pipeline's bounded kind on an mbarrier that never completes, `polls` polls.
+cudaError_t expire_wait(int* err, int polls, cudaStream_t st);
 // E (row-major m' x n') = B^T - P Rw with B^T column-major (n' x m'), Rw row-major r x n'
 cudaError_t error_colmajor(const float* Bt, const float* P, const float* Rw, int mp, int np, int r, int e_zero,
                            float* E, cudaStream_t st);

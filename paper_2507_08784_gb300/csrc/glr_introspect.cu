@@ -88,10 +88,27 @@ int glr_load(glr_handle* h, const void* host_buf, int64_t bytes, void* stream) {
         hd.nbuf != h->n_state_allocs || hd.buf_bytes != ckpt_bytes(h, hd.has_forceJ != 0))
         return fail(h, GLR_EINVAL, "checkpoint of a handle with another shape or schedule%s");
     if (bytes < static_cast<int64_t>(hd.buf_bytes)) return fail(h, GLR_EINVAL, "checkpoint buffer is truncated%s");
+    if (hd.seed != h->s.seed) return fail(h, GLR_EINVAL, "checkpoint of a handle with another seed%s");
+    // each pair of swapped roles (P / Pprev, Q / Qn, Z / Zn) must name the two allocations this
+    // handle uses for that pair, in either order
+    for (int i = 0; i < 6; i += 2) {
+        int cur[2] = {-1, -1};
+        for (int q = 0; q < 2; ++q)
+            for (size_t a = 0; a < h->n_state_allocs; ++a)
+                if (h->allocs[a] == *role_ptr(h, i + q)) cur[q] = static_cast<int>(a);
+        const bool same = hd.role[i] == cur[0] && hd.role[i + 1] == cur[1];
+        const bool swapped = hd.role[i] == cur[1] && hd.role[i + 1] == cur[0];
+        if (!same && !swapped) return fail(h, GLR_EINVAL, "checkpoint roles do not match this handle's buffers%s");
+    }
+    if (hd.has_forceJ != 0 && hd.has_forceJ != 1) return fail(h, GLR_EINVAL, "corrupt checkpoint header%s");
     cudaStream_t st = static_cast<cudaStream_t>(stream);
     const char* in = static_cast<const char*>(host_buf) + sizeof(hd);
     if (hd.has_forceJ) {
-        h->forceJ.assign(reinterpret_cast<const int32_t*>(in), reinterpret_cast<const int32_t*>(in) + h->r);
+        std::vector<int32_t> J(reinterpret_cast<const int32_t*>(in), reinterpret_cast<const int32_t*>(in) + h->r);
+        for (int q = 0; q < h->r; ++q)
+            if (J[q] < 0 || J[q] >= h->mp || (q && J[q] <= J[q - 1]))
+                return fail(h, GLR_EINVAL, "checkpoint's pending selection is not r ascending indices in [0, m')%s");
+        h->forceJ = J;
         in += sizeof(int32_t) * h->r;
     }
     for (size_t a = 0; a < h->n_state_allocs; ++a) {
@@ -119,14 +136,15 @@ int glr_get_stats(const glr_handle* h, glr_stats* out) {
     out->state_bytes = h->state_bytes;
     out->m_prime = h->mp; out->n_prime = h->np; out->r = h->r; out->k = h->k;
     out->transposed = h->transposed;
-    int flags[4] = {0, 0, 0, 0};
+    int flags[8] = {0, 0, 0, 0, 0, 0, 0, 0};
     cudaMemcpy(flags, h->dflags, sizeof(flags), cudaMemcpyDeviceToHost);
     out->last_refresh_sweeps = flags[1];
     out->launches = h->launches;
     out->path = h->tcl ? GLR_PATH_TCGEN05 : h->mma ? GLR_PATH_MMA : h->fused ? GLR_PATH_STRIP
               : h->tc ? GLR_PATH_LIBRARY : GLR_PATH_PLAIN;
     out->nonfinite = flags[3];
-    return flags[2] ? GLR_ETIMEOUT : flags[3] ? GLR_ENONFINITE : GLR_OK;
+    out->numeric_failures = flags[6];
+    return flags[2] ? GLR_ETIMEOUT : flags[6] ? GLR_ENUMERIC : flags[3] ? GLR_ENONFINITE : GLR_OK;
 }
 
 const char* glr_last_error(const glr_handle* h) { return h ? h->err.c_str() : g_create_err.c_str(); }
@@ -218,6 +236,13 @@ int glr_profile_read(glr_handle* h, glr_profile* out, int32_t reset) {
         out->count[p] = h->prof_count[p];
         if (reset) { h->prof_ms[p] = 0.0; h->prof_launch[p] = 0; h->prof_count[p] = 0; }
     }
+    return GLR_OK;
+}
+
+int glr_test_expire_wait(glr_handle* h, int32_t polls, void* stream) {
+    if (!h) return GLR_EINVAL;
+    if (polls < 1 || polls > (1 << 24)) return fail(h, GLR_EINVAL, "need 1 <= polls <= 2^24%s");
+    GLR_LAUNCH(h, 1, tc::expire_wait(h->dflags + 2, polls, static_cast<cudaStream_t>(stream)));
     return GLR_OK;
 }
 

@@ -40,11 +40,10 @@ int wy_from_Q(glr_handle* h, cudaStream_t st) {
     return GLR_OK;
 }
 
-// End of a truncated refresh, with Q orthonormal and H = Q^T Mbar Mbar^T Q in Hk: Rayleigh-Ritz
-// H = W diag W^T, Q <- Q W (columns by descending Ritz value, signs fixed), then the WY form.
-int refresh_tail(glr_handle* h, cudaStream_t st) {
+// Rayleigh-Ritz after the k x k eigen-decomposition H = W diag W^T (eigenvalues in evals, W in
+// Vk): Q <- Q W (columns by descending Ritz value, signs fixed), then the WY form.
+int refresh_finish(glr_handle* h, cudaStream_t st) {
     const int mp = h->mp, k = h->k;
-    GLR_LAUNCH(h, 1, jacobi_eig(h->Hk, k, h->Vk, h->evals, h->dflags + 1, st));
     GLR_LAUNCH(h, 1, sort_fix_basis(h->evals, h->Vk, k, k, h->gram, k, h->evals_sorted, st));
     GLR_GEMM(h, gd(mp, k, k, h->Q, k, 1, h->gram, k, 1, h->Qn, k, 1), st);
     GLR_LAUNCH(h, 1, fix_column_signs(h->Qn, mp, k, st));
@@ -52,8 +51,15 @@ int refresh_tail(glr_handle* h, cudaStream_t st) {
     return wy_from_Q(h, st);
 }
 
+// End of a truncated refresh, with Q orthonormal and H = Q^T Mbar Mbar^T Q in Hk: the k x k
+// Jacobi in one CTA, then refresh_finish.
+int refresh_tail(glr_handle* h, cudaStream_t st) {
+    GLR_LAUNCH(h, 1, jacobi_eig(h->Hk, h->k, h->Vk, h->evals, h->dflags + 1, st));
+    return refresh_finish(h, st);
+}
+
 // Truncated refreshes of several matrices through the grouped block power iteration
-// (k_power.cu): the same iteration as do_refresh (q power iterations, each half re-normalised by
+// (k_power.cu): the same iteration as refresh_power (q power iterations, each half re-normalised by
 // CholeskyQR, then CholeskyQR2 and the Rayleigh-Ritz Gram), one launch per stage for all of
 // them on the first handle's side stream; the k x k tails run on each handle's own stream.
 int refresh_grouped(std::vector<glr_handle*>& hs) {
@@ -163,18 +169,12 @@ int refresh_exact_grouped(std::vector<glr_handle*>& hs) {
     return GLR_OK;
 }
 
-// Semi-Lazy SVD refresh (Eq. SVD-P1) from Mbar.
-int do_refresh(glr_handle* h, cudaStream_t st) {
+// The power-iteration part of a truncated refresh (Eq. SVD-P1 read as the top-k subspace of
+// Mbar): q block power iterations from the previous basis (a seeded Gaussian block at the first
+// refresh), each half re-orthonormalised by CholeskyQR, CholeskyQR2 at the end, then the
+// Rayleigh-Ritz matrix H = Z^T Z = Q^T Mbar Mbar^T Q in Hk.
+int refresh_power(glr_handle* h, cudaStream_t st) {
     const int mp = h->mp, np = h->np, k = h->k;
-    g_ws = h->gemm_ws;
-    struct Reset { ~Reset() { g_ws = nullptr; } } reset_ws;
-    if (h->exact) {
-        // H = Mbar Mbar^T, eigenvectors = left singular vectors, sorted by descending sigma
-        GLR_GEMM(h, gd(mp, mp, np, h->Mbar, np, 1, h->Mbar, 1, np, h->Hbuf, mp, 1), st);
-        GLR_LAUNCH(h, 1, jacobi_eig(h->Hbuf, mp, h->Vbuf, h->evals, h->dflags + 1, st));
-        GLR_LAUNCH(h, 1, sort_fix_basis(h->evals, h->Vbuf, mp, mp, h->U, mp, h->evals_sorted, st));
-        return GLR_OK;
-    }
     if (h->refreshes == 0 && !h->basis_from_user)
         GLR_LAUNCH(h, 1, random_block(h->Q, mp, k, h->s.seed, static_cast<uint32_t>(h->t), st));
     int rc;
@@ -192,7 +192,76 @@ int do_refresh(glr_handle* h, cudaStream_t st) {
     // Rayleigh-Ritz: Z = Mbar^T Q, H = Z^T Z = Q^T Mbar Mbar^T Q
     GLR_GEMM(h, gd(np, k, mp, h->Mbar, sb, sa, h->Q, k, 1, h->Z, k, 1), st);
     GLR_GEMM(h, gd(k, k, np, h->Z, 1, k, h->Z, k, 1, h->Hk, k, 1), st);
-    return refresh_tail(h, st);
+    return GLR_OK;
+}
+
+// Truncated refreshes of several matrices with large k: each handle's power iteration on its
+// own side stream, then the k x k Rayleigh-Ritz eigen-decompositions of all of them in one
+// cooperative Jacobi launch (k_jacobi.cu: every CTA of the grid works on every matrix, where the
+// one-CTA Jacobi of refresh_tail would take k x k rotations in a single SM), then each handle's
+// finish on its own stream.  Without cooperative launches, refresh_tail per handle.
+int refresh_trunc_grouped(std::vector<glr_handle*>& hs) {
+    for (glr_handle* h : hs) {
+        PhaseScope ps(h, GLR_PH_REFRESH, h->rstream);
+        g_ws = h->gemm_ws;
+        const int rc = refresh_power(h, h->rstream);
+        g_ws = nullptr;
+        if (rc != GLR_OK) return rc;
+    }
+    const int grid = jacobi_group_grid();
+    if (!grid) {
+        for (glr_handle* h : hs) {
+            PhaseScope ps(h, GLR_PH_REFRESH, h->rstream);
+            g_ws = h->gemm_ws;
+            const int rc = refresh_tail(h, h->rstream);
+            g_ws = nullptr;
+            if (rc != GLR_OK) return rc;
+        }
+        return GLR_OK;
+    }
+    for (size_t c0 = 0, c1 = 0; c0 < hs.size(); c0 = c1) {
+        size_t rot = 0;
+        for (c1 = c0; c1 < hs.size() && c1 - c0 < (size_t)kGroupMax; ++c1) {
+            const size_t add = jacobi_rot_floats(hs[c1]->k) * sizeof(float);
+            if (c1 > c0 && rot + add > kJacobiMaxSmem) break;
+            rot += add;
+        }
+        glr_handle* h0 = hs[c0];
+        cudaStream_t s0 = h0->rstream;
+        JacobiGroup g{};
+        size_t soff = 0;
+        g.max_sweeps = 40;
+        g.bar = h0->dflags + 4; g.err = h0->dflags + 2; g.part = h0->jpart;
+        for (size_t i = c0; i < c1; ++i) {
+            glr_handle* h = hs[i];
+            if (h != h0) {
+                GLR_CK(h, cudaEventRecord(h->rpow, h->rstream));
+                GLR_CK(h0, cudaStreamWaitEvent(s0, h->rpow, 0));
+            }
+            JacobiMat& M = g.mat[g.nmat++];
+            const int n = h->k;
+            M.n = n; M.tol = 4.f * 5.96e-8f * sqrtf(static_cast<float>(n)) + 1e-7f;
+            M.H = h->Hk; M.H2 = h->scratch; M.V = h->Vk; M.evals = h->evals;
+            M.sweeps = h->dflags + 1;
+            M.soff = (int)soff;
+            soff += jacobi_rot_floats(n);
+        }
+        {
+            PhaseScope ps(h0, GLR_PH_REFRESH, s0);
+            GLR_LAUNCH(h0, 1, jacobi_group(g, grid, s0));
+        }
+        GLR_CK(h0, cudaEventRecord(h0->rpow, s0));
+        for (size_t i = c0; i < c1; ++i) {
+            glr_handle* h = hs[i];
+            if (h != h0) GLR_CK(h, cudaStreamWaitEvent(h->rstream, h0->rpow, 0));
+            PhaseScope ps(h, GLR_PH_REFRESH, h->rstream);
+            g_ws = h->gemm_ws;
+            const int rc = refresh_finish(h, h->rstream);
+            g_ws = nullptr;
+            if (rc != GLR_OK) return rc;
+        }
+    }
+    return GLR_OK;
 }
 
 }  // namespace host

@@ -457,12 +457,10 @@ size_t update_smem_bytes(int mp, int r, int BN) {
 
 template <int BN, typename GT>
 static cudaError_t launch_stream(const StreamGroup& g, size_t smem, cudaStream_t st) {
-    static bool set = false;
-    if (!set) {
-        cudaError_t e = cudaFuncSetAttribute(stream_kernel<BN, GT>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+    {   // per device: set on every call (cheap next to the launch)
+        const cudaError_t ea = cudaFuncSetAttribute(stream_kernel<BN, GT>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                              227 * 1024);
-        if (e != cudaSuccess) return e;
-        set = true;
+        if (ea != cudaSuccess) return ea;
     }
     stream_kernel<BN, GT><<<g.total_strips, NT, smem, st>>>(g);
     return cudaGetLastError();
@@ -482,12 +480,10 @@ cudaError_t stream_group(const StreamGroup& g, size_t smem, cudaStream_t st) {
 
 template <int BN>
 static cudaError_t launch_update(const UpdateGroup& g, size_t smem, cudaStream_t st) {
-    static bool set = false;
-    if (!set) {
-        cudaError_t e = cudaFuncSetAttribute(update_kernel_fused<BN>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+    {   // per device: set on every call (cheap next to the launch)
+        const cudaError_t ea = cudaFuncSetAttribute(update_kernel_fused<BN>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                              227 * 1024);
-        if (e != cudaSuccess) return e;
-        set = true;
+        if (ea != cudaSuccess) return ea;
     }
     update_kernel_fused<BN><<<g.total_strips, NTU, smem, st>>>(g);
     return cudaGetLastError();

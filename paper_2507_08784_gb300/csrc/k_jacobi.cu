@@ -244,11 +244,9 @@ cudaError_t jacobi_group(const JacobiGroup& g, int grid, cudaStream_t st) {
     }
     smem *= sizeof(float);
     if (smem > kJacobiMaxSmem) return cudaErrorInvalidValue;
-    static bool set = false;
-    if (!set) {
-        cudaError_t e = cudaFuncSetAttribute(jacobi_group_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kJacobiMaxSmem);
-        if (e != cudaSuccess) return e;
-        set = true;
+    {   // per device: set on every call (cheap next to the launch)
+        const cudaError_t ea = cudaFuncSetAttribute(jacobi_group_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kJacobiMaxSmem);
+        if (ea != cudaSuccess) return ea;
     }
     cudaError_t e = cudaMemsetAsync(g.bar, 0, 2 * sizeof(int), st);    // arrivals and generation
     if (e != cudaSuccess) return e;

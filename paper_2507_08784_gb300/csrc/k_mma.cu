@@ -752,24 +752,20 @@ int mma_tma_box_rows(int mp) { return tma_box_rows(mp); }
 
 template <typename GT, int NQ>
 static cudaError_t launch_mma(const StreamGroup& g, size_t smem, cudaStream_t st) {
-    static bool set = false;
-    if (!set) {
-        cudaError_t e = cudaFuncSetAttribute(stream_mma_kernel<GT, NQ>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+    {   // per device: set on every call (cheap next to the launch)
+        const cudaError_t ea = cudaFuncSetAttribute(stream_mma_kernel<GT, NQ>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                              227 * 1024);
-        if (e != cudaSuccess) return e;
-        set = true;
+        if (ea != cudaSuccess) return ea;
     }
     stream_mma_kernel<GT, NQ><<<g.total_strips, T, smem, st>>>(g);
     return cudaGetLastError();
 }
 template <typename GT, int NQ>
 static cudaError_t launch_tma(const StreamGroup& g, const TmaMaps& maps, size_t smem, cudaStream_t st) {
-    static bool set = false;
-    if (!set) {
-        cudaError_t e = cudaFuncSetAttribute(stream_tma_kernel<GT, NQ>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+    {   // per device: set on every call (cheap next to the launch)
+        const cudaError_t ea = cudaFuncSetAttribute(stream_tma_kernel<GT, NQ>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                              227 * 1024);
-        if (e != cudaSuccess) return e;
-        set = true;
+        if (ea != cudaSuccess) return ea;
     }
     stream_tma_kernel<GT, NQ><<<g.total_strips, T, smem, st>>>(g, maps);
     return cudaGetLastError();

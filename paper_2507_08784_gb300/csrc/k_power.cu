@@ -321,6 +321,7 @@ __global__ void __launch_bounds__(TCH) pow_chol_kernel(const __grid_constant__ P
     }
     float tr = 0.f;
     for (int i = 0; i < k; ++i) tr += Gs[i][i];
+    if (lane == 0 && M.flag && (!(tr > 0.f) || !isfinite(tr))) atomicAdd(M.flag + 6, 1);   // degenerate block
     float shift = 0.f;
     for (int attempt = 0; attempt < 6; ++attempt) {
         for (int o = lane; o < k * k; o += 32) Ls[o / k][o % k] = Gs[o / k][o % k] + (o / k == o % k ? shift : 0.f);
@@ -361,7 +362,7 @@ __global__ void __launch_bounds__(TCH) pow_chol_kernel(const __grid_constant__ P
     }
     // no factorisation: leave S as identity and count it
     for (int o = lane; o < k * k; o += 32) M.S[o] = o / k == o % k ? 1.f : 0.f;
-    if (lane == 0 && M.flag) atomicAdd(M.flag, 1000);
+    if (lane == 0 && M.flag) { atomicAdd(M.flag, 1000); atomicAdd(M.flag + 6, 1); }
 }
 
 template <int KM>

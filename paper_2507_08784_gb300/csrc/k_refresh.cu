@@ -226,7 +226,12 @@ __global__ void __launch_bounds__(1024) cholesky_kernel(float* A, int n, float* 
     }
     for (int e = tid; e < n * n; e += nth)
         if (e % n > e / n) A[e] = 0.f;
-    if (tid == 0 && flag) *flag = attempt;
+    if (tid == 0 && flag) {
+        *flag = attempt;
+        // no factorisation after every shift, or a Gram matrix with no positive trace (a zero or
+        // non-finite block): the refresh cannot orthonormalise it (flag + 6 counts these)
+        if (attempt == 6 || !(trace > 0.f) || !isfinite(trace)) atomicAdd(flag + 6, 1);
+    }
 }
 
 // Q <- Q L^{-T}: one warp per row, y_j = (x_j - sum_{l<j} y_l L_jl) / L_jj.
@@ -334,10 +339,9 @@ cudaError_t jacobi_eig(float* H, int n, float* V, float* evals, int* sweeps, cud
     const size_t full = 2 * sizeof(float) * (size_t)n * n + pair_bytes;
     const int use_smem = full <= 200 * 1024 ? 1 : 0;
     const size_t smem = use_smem ? full : pair_bytes;
-    static bool attr_set = false;
-    if (!attr_set) {
-        cudaFuncSetAttribute(jacobi_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, 210 * 1024);
-        attr_set = true;
+    {   // per device: set on every call (cheap next to the launch)
+        const cudaError_t ea = cudaFuncSetAttribute(jacobi_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, 210 * 1024);
+        if (ea != cudaSuccess) return ea;
     }
     const float tol = 4.f * 5.96e-8f * sqrtf(static_cast<float>(n)) + 1e-7f;
     // one thread per 2 x 2 block update of a round, rounded to whole warps (at most 1024)
@@ -419,7 +423,12 @@ __global__ void __launch_bounds__(1024) chol_inverse_kernel(const float* G, int 
         if (tid == 0) shift = (attempt == 0 ? 1e-7f : shift * 100.f) * fmaxf(trace / n, 1e-30f);
         __syncthreads();
     }
-    if (tid == 0 && flag) *flag = attempt;
+    if (tid == 0 && flag) {
+        *flag = attempt;
+        // no factorisation after every shift, or a Gram matrix with no positive trace (a zero or
+        // non-finite block): the refresh cannot orthonormalise it (flag + 6 counts these)
+        if (attempt == 6 || !(trace > 0.f) || !isfinite(trace)) atomicAdd(flag + 6, 1);
+    }
     for (int j = n - 1; j >= 0; --j) {
         for (int l = j + 1 + tid; l < n; l += blockDim.x) col[l] = L[tri(l, j)];
         __syncthreads();
@@ -446,14 +455,12 @@ __global__ void __launch_bounds__(1024) chol_inverse_kernel(const float* G, int 
 cudaError_t chol_inverse(const float* G, int n, float* S, int* flag, cudaStream_t st) {
     if (n < 1 || n > 256) return cudaErrorInvalidValue;
     const size_t smem = sizeof(float) * ((size_t)n * (n + 1) / 2 + 2 * n);
-    static bool set = false;
-    if (!set) {
-        // the largest factor (n = 256) and its temporaries, below the per-CTA limit with the
-        // kernel's few static bytes
-        const cudaError_t e = cudaFuncSetAttribute(chol_inverse_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+    // the largest factor (n = 256) and its temporaries, below the per-CTA limit with the
+    // kernel's few static bytes
+    {   // per device: set on every call (cheap next to the launch)
+        const cudaError_t ea = cudaFuncSetAttribute(chol_inverse_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                                    (int)(sizeof(float) * (256 * 257 / 2 + 2 * 256)));
-        if (e != cudaSuccess) return e;
-        set = true;
+        if (ea != cudaSuccess) return ea;
     }
     chol_inverse_kernel<<<1, 1024, smem, st>>>(G, n, S, flag);
     return cudaGetLastError();

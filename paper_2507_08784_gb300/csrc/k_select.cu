@@ -433,10 +433,9 @@ cudaError_t select_group(const SelectGroup& g, cudaStream_t st) {
     if (e != cudaSuccess) return e;
     int npow2 = 1;
     while (npow2 < maxmp) npow2 <<= 1;
-    static bool attr_set = false;
-    if (!attr_set) {
-        cudaFuncSetAttribute(select_group_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, 200 * 1024);
-        attr_set = true;
+    {   // per device: set on every call (cheap next to the launch)
+        const cudaError_t ea = cudaFuncSetAttribute(select_group_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, 200 * 1024);
+        if (ea != cudaSuccess) return ea;
     }
     select_group_kernel<<<g.nmat, 1024, sizeof(unsigned long long) * npow2, st>>>(g);
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
@@ -479,10 +478,9 @@ cudaError_t select_top_r(const float* part, int ntiles, int mp, int r, const flo
     int npow2 = 1;
     while (npow2 < mp) npow2 <<= 1;
     const size_t smem = sizeof(unsigned long long) * npow2;
-    static bool attr_set = false;
-    if (!attr_set) {
-        cudaFuncSetAttribute(select_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, 200 * 1024);
-        attr_set = true;
+    {   // per device: set on every call (cheap next to the launch)
+        const cudaError_t ea = cudaFuncSetAttribute(select_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, 200 * 1024);
+        if (ea != cudaSuccess) return ea;
     }
     select_kernel<<<1, 1024, smem, st>>>(part, ntiles, mp, r, dsign, k, lam, J, npow2);
     return cudaGetLastError();

@@ -191,10 +191,9 @@ __global__ void __launch_bounds__(256) compose_kernel(ComposeArgs a) {
 cudaError_t compose(const ComposeArgs& a, cudaStream_t st) {
     dim3 grid((a.np + CT - 1) / CT, (a.mp + CT - 1) / CT);
     const size_t smem = sizeof(float) * (2 * CT * a.r + CT * (CT + 1));
-    static bool attr_set = false;
-    if (!attr_set) {
-        cudaFuncSetAttribute(compose_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, 160 * 1024);
-        attr_set = true;
+    {   // per device: set on every call (cheap next to the launch)
+        const cudaError_t ea = cudaFuncSetAttribute(compose_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, 160 * 1024);
+        if (ea != cudaSuccess) return ea;
     }
     compose_kernel<<<grid, dim3(CT, 8), smem, st>>>(a);
     return cudaGetLastError();
@@ -280,10 +279,9 @@ __global__ void __launch_bounds__(256) error_kernel(int mp, int np, int r, int e
 cudaError_t update(const UpdateArgs& a, cudaStream_t st) {
     dim3 grid((a.np + CT - 1) / CT, (a.mp + CT - 1) / CT);
     const size_t smem = sizeof(float) * (2 * CT * a.r + CT * (CT + 1));
-    static bool attr_set = false;
-    if (!attr_set) {
-        cudaFuncSetAttribute(update_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, 160 * 1024);
-        attr_set = true;
+    {   // per device: set on every call (cheap next to the launch)
+        const cudaError_t ea = cudaFuncSetAttribute(update_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, 160 * 1024);
+        if (ea != cudaSuccess) return ea;
     }
     update_kernel<<<grid, dim3(CT, 8), smem, st>>>(a);
     return cudaGetLastError();

@@ -69,9 +69,10 @@ __device__ __forceinline__ bool mbar_test(uint32_t bar, uint32_t parity) {
 }
 // Waits for phase `parity` of `bar`; false when the CTA aborted (now or already).  About a second
 // of polling (16 M polls with sleeps of 16..64 ns) before giving up.
-__device__ __forceinline__ bool wait_phase(uint32_t bar, uint32_t parity, volatile int* abort, int* err) {
+__device__ __forceinline__ bool wait_phase(uint32_t bar, uint32_t parity, volatile int* abort, int* err,
+                                           int limit = 16000000) {
     uint32_t ns = 16;
-    for (int it = 0; it < 16000000; ++it) {
+    for (int it = 0; it < limit; ++it) {
         if (mbar_test(bar, parity)) return true;
         if ((it & 255) == 255 && *abort) return false;
         __nanosleep(ns);
@@ -921,6 +922,26 @@ __global__ void error_cm_kernel(const float* Bt, const float* P, const float* Rw
     E[e] = v;
 }
 }  // namespace
+
+namespace {
+// The bounded wait of the pipeline on an mbarrier that nothing arrives on: it gives up after
+// `polls` polls, counts the event in *err (through the abort flag, as a stuck pipeline would)
+// and the kernel returns.
+__global__ void expire_kernel(int* err, int polls) {
+    __shared__ __align__(8) uint64_t bar;
+    __shared__ int abort_flag;
+    if (threadIdx.x != 0) return;
+    abort_flag = 0;
+    mbar_init(smem_u32(&bar), 1);
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    wait_phase(smem_u32(&bar), 0, &abort_flag, err, polls);
+}
+}  // namespace
+
+cudaError_t expire_wait(int* err, int polls, cudaStream_t st) {
+    expire_kernel<<<1, 32, 0, st>>>(err, polls);
+    return cudaGetLastError();
+}
 
 cudaError_t transpose_round(float* dst, int ldd, const float* src, int rows, int cols, int lds, cudaStream_t st) {
     dim3 grid((cols + 31) / 32, (rows + 31) / 32), block(32, 8);
