@@ -42,9 +42,8 @@ namespace tc {
 
 namespace {
 
-constexpr int kEpiWarps = 8;
-constexpr int kThreads = (kEpiWarps + 3) * 32;
-constexpr int kProdWarp = kEpiWarps, kMmaWarp = kEpiWarps + 1, kDataWarp = kEpiWarps + 2;
+// Epilogue warps per op (Op::kEpi); the three role warps follow them.
+template <class Op> constexpr int threads_of() { return (Op::kEpi + 3) * 32; }
 constexpr int kMaxStages = 8;
 constexpr int kMaxDStages = 4;
 constexpr uint32_t kTmemCols = 512;      // every op keeps more than half of shared memory, so one CTA per SM
@@ -117,6 +116,16 @@ __device__ __forceinline__ void tmem_ld16(uint32_t ta, float (&v)[16]) {
     asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
 #pragma unroll
     for (int j = 0; j < 16; ++j) v[j] = __uint_as_float(u[j]);
+}
+// 8 consecutive accumulator columns of this thread's lane.
+__device__ __forceinline__ void tmem_ld8(uint32_t ta, float (&v)[8]) {
+    uint32_t u[8];
+    asm volatile("tcgen05.ld.sync.aligned.32x32b.x8.b32 {%0,%1,%2,%3,%4,%5,%6,%7}, [%8];"
+                 : "=r"(u[0]), "=r"(u[1]), "=r"(u[2]), "=r"(u[3]), "=r"(u[4]), "=r"(u[5]), "=r"(u[6]), "=r"(u[7])
+                 : "r"(ta));
+    asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+#pragma unroll
+    for (int j = 0; j < 8; ++j) v[j] = __uint_as_float(u[j]);
 }
 // x rounded to the nearest TF32 value (ties away from zero), as an fp32 bit pattern.
 __device__ __forceinline__ float rna_tf32(float x) {
@@ -220,13 +229,16 @@ struct NoStore { __device__ bool operator()(uint32_t) const { return false; } };
 
 // Ops without epilogue data.
 struct NoData {
+    static constexpr int kEpi = 8;
     static __device__ __forceinline__ int ndata(const TcGroup&, const Tile&) { return 0; }
     static __device__ __forceinline__ uint32_t data_tx(const TcGroup&, const Tile&, int) { return 0; }
     static __device__ __forceinline__ void data_load(const TcGroup&, const Tile&, int, uint32_t, uint32_t) {}
 };
 
 template <class Op>
-__global__ void __launch_bounds__(kThreads, 1) tc_kernel(const __grid_constant__ TcGroup g) {
+__global__ void __launch_bounds__(threads_of<Op>(), 1) tc_kernel(const __grid_constant__ TcGroup g) {
+    constexpr int kEpiWarps = Op::kEpi;
+    constexpr int kProdWarp = kEpiWarps, kMmaWarp = kEpiWarps + 1, kDataWarp = kEpiWarps + 2;
     extern __shared__ uint8_t dyn_smem[];
     uint8_t* ring = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(dyn_smem) + 1023) & ~uintptr_t(1023));
     __shared__ __align__(8) uint64_t full_bar[kMaxStages], empty_bar[kMaxStages], tfull_bar[2], tempty_bar[2];
@@ -428,6 +440,7 @@ struct PrevProj : NoData {
 // bytes), 16 KiB.  B_i^T is stored back from the stage.
 // ------------------------------------------------------------------------------------------
 struct Compose {
+    static constexpr int kEpi = 16;
     static constexpr int BN = 64;
     static constexpr uint32_t kG = 32768;             // offset of the gradient tile in a data stage
     static __device__ __forceinline__ int nk(const TcGroup& g, const Tile& t) {
@@ -464,21 +477,21 @@ struct Compose {
         const int rt = t.lt / M.tn, ct = t.lt % M.tn;
         const int al = 32 * (warp & 3) + lane;            // row within the tile
         const int a = rt * 128 + al;
-        const int cw = (warp >> 2) * 32;                  // this warp's 32 columns of the tile
+        const int cw = (warp >> 2) * 16;                  // this warp's 16 columns of the tile
         const int c0 = ct * BN + cw;
         const bool leader = warp == 0 && lane == 0;
-        float acc[32];
+        float acc[16];
 #pragma unroll
-        for (int j = 0; j < 32; ++j) acc[j] = 0.f;
+        for (int j = 0; j < 16; ++j) acc[j] = 0.f;
         for (int i = 0; i < M.N; ++i) {
             uint8_t* sm = dr.acquire();
             if (!sm) return false;
             float* Bs = reinterpret_cast<float*>(sm) + al;    // B^T tile: column c at Bs[128 c]
-            float m[32];
+            float m[16];
             if (!M.transposed) {
                 const uint8_t* row = sm + kG + al * 128;
 #pragma unroll
-                for (int q = 0; q < 4; ++q) {
+                for (int q = 0; q < 2; ++q) {
                     const uint4 u = *reinterpret_cast<const uint4*>(row + ((((cw >> 3) + q) ^ (al & 7)) << 4));
                     const uint32_t w[4] = {u.x, u.y, u.z, u.w};
 #pragma unroll
@@ -491,21 +504,20 @@ struct Compose {
             } else {
                 const __nv_bfloat16* col = reinterpret_cast<const __nv_bfloat16*>(sm + kG) + al;
 #pragma unroll
-                for (int j = 0; j < 32; ++j) m[j] = __bfloat162float(col[(cw + j) * 128]);
+                for (int j = 0; j < 16; ++j) m[j] = __bfloat162float(col[(cw + j) * 128]);
             }
             if (!M.e_zero) {
-                float d[32];
-                tmem_ld16(tl + (uint32_t)(i * BN + cw), *reinterpret_cast<float(*)[16]>(d));
-                tmem_ld16(tl + (uint32_t)(i * BN + cw + 16), *reinterpret_cast<float(*)[16]>(d + 16));
+                float d[16];
+                tmem_ld16(tl + (uint32_t)(i * BN + cw), d);
 #pragma unroll
-                for (int j = 0; j < 32; ++j) m[j] += Bs[(cw + j) * 128] - d[j];
+                for (int j = 0; j < 16; ++j) m[j] += Bs[(cw + j) * 128] - d[j];
             }
             if (M.write_B) {
 #pragma unroll
-                for (int j = 0; j < 32; ++j) Bs[(cw + j) * 128] = m[j];
+                for (int j = 0; j < 16; ++j) Bs[(cw + j) * 128] = m[j];
             }
 #pragma unroll
-            for (int j = 0; j < 32; ++j) acc[j] += m[j];
+            for (int j = 0; j < 16; ++j) acc[j] += m[j];
             dr.release(leader, [&](uint32_t st) {
                 if (!M.write_B) return false;
                 tma_store_3d(M.mD0, rt * 128, ct * BN, i, st);
@@ -516,7 +528,7 @@ struct Compose {
         if (a < M.mp) {
             const float invN = 1.0f / static_cast<float>(M.N);
 #pragma unroll
-            for (int j = 0; j < 32; ++j)
+            for (int j = 0; j < 16; ++j)
                 if (c0 + j < M.np) {
                     const float v = acc[j] * invN;
                     bad |= !isfinite(v);
@@ -574,6 +586,7 @@ struct WBar : NoData {
 // the Mbar^T tile (128 columns x 128 rows fp32, 64 KiB).
 // ------------------------------------------------------------------------------------------
 struct Lambda {
+    static constexpr int kEpi = 8;
     static __device__ __forceinline__ int nk(const TcGroup& g, const Tile& t) { return g.mat[t.mat].kpad / 32; }
     static __device__ __forceinline__ uint32_t tx_bytes(const TcGroup&, const Tile&, int) { return 2u * 16384u; }
     static __device__ __forceinline__ void load(const TcGroup& g, const Tile& t, int kc, uint32_t st, uint32_t bar) {
@@ -718,6 +731,7 @@ struct RBar : NoData {
 // bytes), plus Mbar^T's tile when uncompressed; X, Mo, Vo are stored back from the stage.
 // ------------------------------------------------------------------------------------------
 struct Update {
+    static constexpr int kEpi = 16;
     static __device__ __forceinline__ int nk(const TcGroup& g, const Tile& t) {
         const TcMat& M = g.mat[t.mat];
         return M.compressed ? M.rpad / 32 : 0;
@@ -760,13 +774,13 @@ struct Update {
                                                     DataRing& dr) {
         const TcMat& M = g.mat[t.mat];
         const int al = 32 * (warp & 3) + lane;
-        const int h = warp >> 2;
+        const int h = warp >> 2;                                  // this warp's 8 columns of each chunk
         const bool adam = g.optimizer != GLR_MSGD;
         const float lr = g.lr, b1 = g.beta1, b2 = g.beta2, eps = g.eps;
         const bool leader = warp == 0 && lane == 0;
         for (int d = 0; d < 4; ++d) {
-            float gh[16];
-            if (M.compressed) tmem_ld16(tl + (uint32_t)(32 * d + 16 * h), gh);
+            float gh[8];
+            if (M.compressed) tmem_ld8(tl + (uint32_t)(32 * d + 8 * h), gh);
             uint8_t* sm = dr.acquire();
             if (!sm) return false;
             float* Xs = reinterpret_cast<float*>(sm);
@@ -775,21 +789,57 @@ struct Update {
             if (!M.compressed) {
                 const float* Gs = reinterpret_cast<const float*>(sm + (adam ? 49152 : 32768)) + al;
 #pragma unroll
-                for (int e = 0; e < 16; ++e) gh[e] = Gs[(16 * h + e) * 128];
+                for (int e = 0; e < 8; ++e) gh[e] = Gs[(8 * h + e) * 128];
+            }
+            // this thread's 8 elements: row al, columns 8h .. 8h + 7 of the chunk; rows of 128 bytes
+            // with the 128-byte swizzle are read as two 16-byte pieces (conflict-free), the columns
+            // of 512 bytes (m > n) element by element (32 lanes, 32 consecutive floats)
+            float x[8], mo[8], vo[8];
+            int o[8];
+#pragma unroll
+            for (int e = 0; e < 8; ++e) {
+                const int c = 8 * h + e;
+                o[e] = M.transposed ? c * 128 + al : al * 32 + ((((c >> 2) ^ (al & 7)) << 2) | (c & 3));
+            }
+            if (M.transposed) {
+#pragma unroll
+                for (int e = 0; e < 8; ++e) { x[e] = Xs[o[e]]; mo[e] = Ms[o[e]]; if (adam) vo[e] = Vs[o[e]]; }
+            } else {
+#pragma unroll
+                for (int p = 0; p < 2; ++p) {
+                    const float4 a = *reinterpret_cast<const float4*>(Xs + o[4 * p]);
+                    const float4 b = *reinterpret_cast<const float4*>(Ms + o[4 * p]);
+                    x[4 * p] = a.x; x[4 * p + 1] = a.y; x[4 * p + 2] = a.z; x[4 * p + 3] = a.w;
+                    mo[4 * p] = b.x; mo[4 * p + 1] = b.y; mo[4 * p + 2] = b.z; mo[4 * p + 3] = b.w;
+                    if (adam) {
+                        const float4 v = *reinterpret_cast<const float4*>(Vs + o[4 * p]);
+                        vo[4 * p] = v.x; vo[4 * p + 1] = v.y; vo[4 * p + 2] = v.z; vo[4 * p + 3] = v.w;
+                    }
+                }
             }
 #pragma unroll
-            for (int e = 0; e < 16; ++e) {
-                const int c = 16 * h + e;                          // column within the chunk
-                const int o = M.transposed ? c * 128 + al : al * 32 + ((((c >> 2) ^ (al & 7)) << 2) | (c & 3));
+            for (int e = 0; e < 8; ++e) {
                 const float gg = gh[e];
-                const float mo = b1 * Ms[o] + (1.f - b1) * gg;
-                Ms[o] = mo;
+                mo[e] = b1 * mo[e] + (1.f - b1) * gg;
                 if (adam) {
-                    const float vo = b2 * Vs[o] + (1.f - b2) * gg * gg;
-                    Vs[o] = vo;
-                    Xs[o] -= lr * mo / (sqrtf(vo) + eps);
+                    vo[e] = b2 * vo[e] + (1.f - b2) * gg * gg;
+                    x[e] -= lr * mo[e] / (sqrtf(vo[e]) + eps);
                 } else {
-                    Xs[o] -= lr * mo;
+                    x[e] -= lr * mo[e];
+                }
+            }
+            if (M.transposed) {
+#pragma unroll
+                for (int e = 0; e < 8; ++e) { Xs[o[e]] = x[e]; Ms[o[e]] = mo[e]; if (adam) Vs[o[e]] = vo[e]; }
+            } else {
+#pragma unroll
+                for (int p = 0; p < 2; ++p) {
+                    *reinterpret_cast<float4*>(Xs + o[4 * p]) = make_float4(x[4 * p], x[4 * p + 1], x[4 * p + 2], x[4 * p + 3]);
+                    *reinterpret_cast<float4*>(Ms + o[4 * p]) =
+                        make_float4(mo[4 * p], mo[4 * p + 1], mo[4 * p + 2], mo[4 * p + 3]);
+                    if (adam)
+                        *reinterpret_cast<float4*>(Vs + o[4 * p]) =
+                            make_float4(vo[4 * p], vo[4 * p + 1], vo[4 * p + 2], vo[4 * p + 3]);
                 }
             }
             dr.release(leader, [&](uint32_t st) {
@@ -873,7 +923,7 @@ cudaError_t launch(TcGroup& g, cudaStream_t st) {
     cudaError_t e = cudaFuncSetAttribute(tc_kernel<Op>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
     const int grid = std::min(g.total_tiles, g_sms);
-    tc_kernel<Op><<<grid, kThreads, smem, st>>>(g);
+    tc_kernel<Op><<<grid, threads_of<Op>(), smem, st>>>(g);
     return cudaGetLastError();
 }
 
