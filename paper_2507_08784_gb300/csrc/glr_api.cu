@@ -377,7 +377,7 @@ int glr_create(int64_t m, int64_t n, int32_t r, int32_t N, const glr_schedule* s
     A(&h->Pprev, MP * r);
     A(&h->J, (size_t)r);
     A(&h->lam, MP);
-    A(&h->lam_part, MP * std::max(std::max(h->ntiles, h->nstrips), 2 * ((h->np + 127) / 128)));
+    A(&h->lam_part, MP * std::max(std::max(h->ntiles, h->nstrips), 4 * ((h->np + 127) / 128)));
     const bool galore = s->optimizer == GLR_GALORE_ADAM;
     A(&h->Mo, galore ? (size_t)r * NP : (size_t)m * n);
     if (s->optimizer != GLR_MSGD) A(&h->Vo, galore ? (size_t)r * NP : (size_t)m * n);
@@ -788,12 +788,7 @@ int tcl_lambda(std::vector<StepPlan*>& plans, cudaStream_t st) {
 int tcl_project_update(std::vector<StepPlan*>& plans, cudaStream_t st) {
     int rc = tc_run(plans, GLR_PH_PROJECT, tc::launch_wbar, st, tc_wbar_fill(false));
     if (rc != GLR_OK) return rc;
-    for (StepPlan* p : plans) {
-        if (!p->compressed) continue;
-        glr_handle* h = p->h;
-        PhaseScope ps(h, GLR_PH_SELECT, st);
-        GLR_LAUNCH(h, 1, wy_columns_gather(h->Yt, h->J, h->r, h->k, h->YtJ, st));
-    }
+    // YtJ = Yt[J, :] was gathered by the selection launch
     rc = tc_run(plans, GLR_PH_SELECT, tc::launch_pbuild, st, [](StepPlan& p, tc::TcMat& M, tc::TcGroup&, bool) {
         glr_handle* h = p.h;
         if (!p.compressed) return 0;
@@ -905,6 +900,7 @@ int select_P_grouped(std::vector<StepPlan>& plans, cudaStream_t st) {
         M.rbar = p.stream_update ? 1 : 0; M.np = h->np;
         M.Mbar = h->Mbar; M.Wbar = h->Wbar; M.Rbar = h->Rbar;
         M.build_p = ((h->tc || h->tcl) && !h->exact) ? 0 : 1;
+        M.YtJ = (h->tcl && !h->exact) ? h->YtJ : nullptr;
         M.out0 = g.total_out;
         g.total_out += (M.build_p ? (int64_t)h->mp * h->r : 0) + (M.rbar ? (int64_t)h->r * h->np : 0);
         if (g.nmat == kGroupMax) {

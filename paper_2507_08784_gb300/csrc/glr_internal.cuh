@@ -171,6 +171,7 @@ struct SelectMat {
     const float* Mbar; const float* Wbar; float* Rbar;
     int64_t out0;                           // first output of this matrix in pr_kernel
     int build_p;                            // 0: the caller forms P (wy_columns_*), pr_kernel skips it
+    float* YtJ;                             // non-null: also gather YtJ = Yt[J, :] (r x k) after J
 };
 struct SelectGroup {
     int nmat;

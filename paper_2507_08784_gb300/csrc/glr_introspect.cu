@@ -172,7 +172,9 @@ int glr_get_selection(glr_handle* h, int32_t* J_host, float* P_out, float* Rbar_
     cudaStream_t st = static_cast<cudaStream_t>(stream);
     const size_t mp = h->mp, np = h->np, r = h->r;
     if (P_out) GLR_CK(h, cudaMemcpyAsync(P_out, h->Pprev, 4 * mp * r, cudaMemcpyDeviceToDevice, st));
-    if (Rbar_out) GLR_CK(h, cudaMemcpyAsync(Rbar_out, h->Rbar, 4 * r * np, cudaMemcpyDeviceToDevice, st));
+    if (Rbar_out && h->tcl)   // the tcgen05 path keeps only Rbar^T (n' x rpad)
+        GLR_LAUNCH(h, 1, tc::transpose_round(Rbar_out, (int)np, h->RbarT, (int)np, (int)r, h->rpad, st));
+    else if (Rbar_out) GLR_CK(h, cudaMemcpyAsync(Rbar_out, h->Rbar, 4 * r * np, cudaMemcpyDeviceToDevice, st));
     if (lambda_out) GLR_CK(h, cudaMemcpyAsync(lambda_out, h->lam, 4 * mp, cudaMemcpyDeviceToDevice, st));
     if (Mbar_out && h->tcl) GLR_LAUNCH(h, 1, transpose_pad(Mbar_out, (int)np, h->Mbar, (int)np, (int)mp, st));
     else if (Mbar_out) GLR_CK(h, cudaMemcpyAsync(Mbar_out, h->Mbar, 4 * mp * np, cudaMemcpyDeviceToDevice, st));

@@ -32,7 +32,7 @@ int tcl_alloc(glr_handle* h) {
     na_max = std::max(1, std::min(na_max, h->N));
     h->tc_ng = (h->N + na_max - 1) / na_max;
     h->tc_na = (h->N + h->tc_ng - 1) / h->tc_ng;
-    h->tc_lam_tiles = 2 * ((h->np + 127) / 128);
+    h->tc_lam_tiles = 4 * ((h->np + 127) / 128);   // one partial per 32 columns
     int rc = GLR_OK;
     auto A = [&](float** p, size_t cnt) { if (rc == GLR_OK) rc = alloc(h, p, cnt); };
     A(&h->PT0, (size_t)h->rpad * MP);

@@ -271,10 +271,7 @@ __device__ __forceinline__ unsigned long long shfl_xor_u64(unsigned long long v,
 }
 
 // Keys (lambda-bar_j^2 bits, ~j): distinct, larger score first and the lower index on ties.
-__global__ void __launch_bounds__(1024) select_group_kernel(const __grid_constant__ SelectGroup g) {
-    extern __shared__ unsigned long long keys[];
-    const SelectMat& M = g.mat[blockIdx.x];
-    if (!M.do_select) return;                                // J was supplied
+__device__ __forceinline__ void select_top_r_block(const SelectMat& M, unsigned long long* keys) {
     const int tid = threadIdx.x, mp = M.mp, r = M.r, nth = blockDim.x;
     auto key_of = [&](int j) -> unsigned long long {
         return j < mp ? (static_cast<unsigned long long>(__float_as_uint(M.lam[j] * M.lam[j])) << 32) |
@@ -356,6 +353,21 @@ __global__ void __launch_bounds__(1024) select_group_kernel(const __grid_constan
             M.J[rank] = jq;
         }
     }
+}
+
+__global__ void __launch_bounds__(1024) select_group_kernel(const __grid_constant__ SelectGroup g) {
+    extern __shared__ unsigned long long keys[];
+    const SelectMat& M = g.mat[blockIdx.x];
+    if (M.do_select) select_top_r_block(M, keys);           // otherwise J was supplied
+    if (!M.YtJ) return;
+    // YtJ = Yt[J, :] (r x k) for the tcgen05 path's P and Rbar products
+    __syncthreads();
+    const int r = M.r, k = M.k;
+    for (int e = threadIdx.x; e < r * k; e += blockDim.x) {
+        const int q = e / k, c = e - q * k;
+        M.YtJ[e] = M.Yt[(int64_t)M.J[q] * k + c];
+    }
+
 }
 
 // Output o of the group: matrix i owns [out0, out0 + m' r) for P (row-major m' x r) and, when

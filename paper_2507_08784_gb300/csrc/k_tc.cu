@@ -581,12 +581,12 @@ struct WBar : NoData {
 
 // ------------------------------------------------------------------------------------------
 // Lambda: tile = (128 rows j, 128 columns b).  D = Yt[j, :] W[:, b] (K = k); the epilogue adds
-// (Mbar - D)(j, b) v_j[b] over each 64-column half into part[(2 ct + half) m' + j] (the signs D
-// are applied when the partials are reduced).  A = Yt (m' x k), B = W^T (n' x kpad).  Data stage:
+// (Mbar - D)(j, b) v_j[b] over each 32-column quarter into part[(4 ct + quarter) m' + j] (the
+// signs D are applied when the partials are reduced).  A = Yt (m' x k), B = W^T (n' x kpad).  Data stage:
 // the Mbar^T tile (128 columns x 128 rows fp32, 64 KiB).
 // ------------------------------------------------------------------------------------------
 struct Lambda {
-    static constexpr int kEpi = 8;
+    static constexpr int kEpi = 16;
     static __device__ __forceinline__ int nk(const TcGroup& g, const Tile& t) { return g.mat[t.mat].kpad / 32; }
     static __device__ __forceinline__ uint32_t tx_bytes(const TcGroup&, const Tile&, int) { return 2u * 16384u; }
     static __device__ __forceinline__ void load(const TcGroup& g, const Tile& t, int kc, uint32_t st, uint32_t bar) {
@@ -611,15 +611,15 @@ struct Lambda {
         const int rt = t.lt / M.tn, ct = t.lt % M.tn;
         const int al = 32 * (warp & 3) + lane;
         const int j = rt * 128 + al;
-        const int h = warp >> 2;
-        const int b0 = ct * 128 + 64 * h;
+        const int h = warp >> 2;                              // this warp's 32 columns
+        const int b0 = ct * 128 + 32 * h;
         const uint8_t* sm = dr.acquire();
         if (!sm) return false;
-        const float* Ms = reinterpret_cast<const float*>(sm) + al + (64 * h) * 128;   // column b0 + c at Ms[128 c]
+        const float* Ms = reinterpret_cast<const float*>(sm) + al + (32 * h) * 128;   // column b0 + c at Ms[128 c]
         float acc = 0.f;
-        for (int cc = 0; cc < 64; cc += 16) {
+        for (int cc = 0; cc < 32; cc += 16) {
             float d[16];
-            tmem_ld16(tl + (uint32_t)(64 * h + cc), d);
+            tmem_ld16(tl + (uint32_t)(32 * h + cc), d);
             if (j < M.mp) {
 #pragma unroll
                 for (int qq = 0; qq < 4; ++qq) {
@@ -634,7 +634,7 @@ struct Lambda {
             }
         }
         dr.release(warp == 0 && lane == 0, NoStore{});
-        if (j < M.mp) M.part[(int64_t)(2 * ct + h) * M.mp + j] = acc;
+        if (j < M.mp) M.part[(int64_t)(4 * ct + h) * M.mp + j] = acc;
         return true;
     }
 };
@@ -683,10 +683,12 @@ struct PBuild : NoData {
 
 // ------------------------------------------------------------------------------------------
 // RBar: tile = 128 columns b.  D (128 x 128) = Yt[J, :] W[:, b] (K = k, rows q >= r are zero);
-// the epilogue writes Rbar(q, b) = d_{J_q} (Mbar(J_q, b) - D(q, b)) to Rbar (r x n') and Rbar^T
-// (rounded to TF32).  A = YtJ (r x k), B = W^T (n' x kpad).
+// the epilogue writes Rbar^T(b, q) = d_{J_q} (Mbar(J_q, b) - D(q, b)) (rounded to TF32).  A = YtJ
+// (r x k), B = W^T (n' x kpad).  Warp w: rows q = 32 (w % 4) + lane, columns 32 (w / 4) .. + 31;
+// the 32 gathered Mbar(J_q, b) are loaded before any store so that they are all in flight.
 // ------------------------------------------------------------------------------------------
 struct RBar : NoData {
+    static constexpr int kEpi = 16;
     static __device__ __forceinline__ int nk(const TcGroup& g, const Tile& t) { return g.mat[t.mat].kpad / 32; }
     static __device__ __forceinline__ uint32_t tx_bytes(const TcGroup&, const Tile&, int) { return 2u * 16384u; }
     static __device__ __forceinline__ void load(const TcGroup& g, const Tile& t, int kc, uint32_t st, uint32_t bar) {
@@ -700,24 +702,23 @@ struct RBar : NoData {
     static __device__ __forceinline__ bool epilogue(const TcGroup& g, const Tile& t, uint32_t tl, int warp, int lane, DataRing&) {
         const TcMat& M = g.mat[t.mat];
         const int q = 32 * (warp & 3) + lane;
-        const int h = warp >> 2;
-        const int b0 = t.lt * 128 + 64 * h;
-        const bool ok = q < M.r;
-        const int j = ok ? M.J[q] : 0;
-        const float dj = (ok && j < M.k) ? M.dsign[j] : 1.f;
-        for (int cc = 0; cc < 64; cc += 16) {
-            float d[16];
-            tmem_ld16(tl + (uint32_t)(64 * h + cc), d);
-            if (!ok) continue;
+        const int c0 = 32 * (warp >> 2);
+        const int b0 = t.lt * 128 + c0;
+        float d[32];
+        tmem_ld16(tl + (uint32_t)c0, *reinterpret_cast<float(*)[16]>(d));
+        tmem_ld16(tl + (uint32_t)(c0 + 16), *reinterpret_cast<float(*)[16]>(d + 16));
+        if (q >= M.r) return true;
+        const int j = M.J[q];
+        const float dj = j < M.k ? M.dsign[j] : 1.f;
+        const int nb = M.np - b0 < 32 ? M.np - b0 : 32;
+        const float* col = M.Mbar + (int64_t)b0 * M.mp + j;     // Mbar(j, b0 + e) at col[e m']
+        float mb[32];
 #pragma unroll
-            for (int e = 0; e < 16; ++e) {
-                const int b = b0 + cc + e;
-                if (b >= M.np) break;
-                const float v = rna_tf32(dj * (M.Mbar[(int64_t)b * M.mp + j] - d[e]));
-                M.Rbar[(int64_t)q * M.np + b] = v;
-                M.RbarT[(int64_t)b * M.rpad + q] = v;
-            }
-        }
+        for (int e = 0; e < 32; ++e) mb[e] = e < nb ? __ldg(col + (int64_t)e * M.mp) : 0.f;
+        float* out = M.RbarT + (int64_t)b0 * M.rpad + q;
+#pragma unroll
+        for (int e = 0; e < 32; ++e)
+            if (e < nb) out[(int64_t)e * M.rpad] = rna_tf32(dj * (mb[e] - d[e]));
         return true;
     }
 };
