@@ -258,6 +258,19 @@ struct JacobiGroup {
     int* bar; int* err; float* part;
     JacobiMat mat[kGroupMax];
 };
+// The k x k Rayleigh-Ritz eigenproblems of truncated refreshes (k_eig.cu): one CTA per matrix,
+// H (row-major n x n, n <= 256, read only) -> eigenvalues (unsorted) and eigenvectors V (row-major
+// n x n, column j for evals[j]); sweeps done in *sweeps.
+struct EigMat {
+    int n; float tol;
+    const float* H; float* V; float* evals; int* sweeps;
+};
+constexpr int kEigGroupMax = 64;
+struct EigGroup {
+    int nmat, max_sweeps;
+    EigMat mat[kEigGroupMax];
+};
+cudaError_t eig_tmem_group(const EigGroup& g, cudaStream_t st);
 int jacobi_group_grid();
 cudaError_t jacobi_group(const JacobiGroup& g, int grid, cudaStream_t st);
 // Q <- Q L^{-T} for the rows x n matrix Q (row-major) and lower-triangular L.

@@ -208,6 +208,44 @@ int refresh_trunc_grouped(std::vector<glr_handle*>& hs) {
         g_ws = nullptr;
         if (rc != GLR_OK) return rc;
     }
+    // k <= 256: every matrix's eigenproblem in one launch, one CTA each (k_eig.cu)
+    bool small = true;
+    for (glr_handle* h : hs) small = small && h->k <= 256;
+    if (small) {
+        for (size_t c0 = 0; c0 < hs.size(); c0 += kEigGroupMax) {
+            const size_t c1 = std::min(hs.size(), c0 + (size_t)kEigGroupMax);
+            glr_handle* h0 = hs[c0];
+            cudaStream_t s0 = h0->rstream;
+            EigGroup g{};
+            g.max_sweeps = 40;
+            for (size_t i = c0; i < c1; ++i) {
+                glr_handle* h = hs[i];
+                if (h != h0) {
+                    GLR_CK(h, cudaEventRecord(h->rpow, h->rstream));
+                    GLR_CK(h0, cudaStreamWaitEvent(s0, h->rpow, 0));
+                }
+                EigMat& M = g.mat[g.nmat++];
+                const int n = h->k;
+                M.n = n; M.tol = 4.f * 5.96e-8f * sqrtf(static_cast<float>(n)) + 1e-7f;
+                M.H = h->Hk; M.V = h->Vk; M.evals = h->evals; M.sweeps = h->dflags + 1;
+            }
+            {
+                PhaseScope ps(h0, GLR_PH_REFRESH, s0);
+                GLR_LAUNCH(h0, 1, eig_tmem_group(g, s0));
+            }
+            GLR_CK(h0, cudaEventRecord(h0->rpow, s0));
+            for (size_t i = c0; i < c1; ++i) {
+                glr_handle* h = hs[i];
+                if (h != h0) GLR_CK(h, cudaStreamWaitEvent(h->rstream, h0->rpow, 0));
+                PhaseScope ps(h, GLR_PH_REFRESH, h->rstream);
+                g_ws = h->gemm_ws;
+                const int rc = refresh_finish(h, h->rstream);
+                g_ws = nullptr;
+                if (rc != GLR_OK) return rc;
+            }
+        }
+        return GLR_OK;
+    }
     const int grid = jacobi_group_grid();
     if (!grid) {
         for (glr_handle* h : hs) {
