@@ -755,6 +755,7 @@ int tcl_compose(std::vector<StepPlan*>& plans, cudaStream_t st) {
         M.mD1 = tcl_grad_maps(h, p.G, st, &rc);
         if (rc != GLR_OK) return -2;
         M.B = h->B; M.Mbar = h->Mbar; M.nonfinite = h->dflags + 3;
+        M.MbarRow = (p.refresh && h->k <= 256) ? h->Mrow : nullptr;   // the refresh's Mbar Z products
         return 1;
     });
 }
@@ -962,18 +963,19 @@ int step_group(std::vector<StepPlan>& plans, cudaStream_t st) {
     // Refreshes (Semi-Lazy SVD) of different matrices are independent: each runs on its
     // handle's side stream after the compose pass, overlapping the others and the selection
     // work of the non-refreshing matrices; the main stream joins them before P is built.
-    std::vector<glr_handle*> refreshing, grouped, exact, trunc;
+    std::vector<glr_handle*> refreshing, grouped, exact, trunc, tclr;
     for (StepPlan& p : plans) {
         if (!p.refresh) continue;
         glr_handle* h = p.h;
         GLR_CK(h, cudaEventRecord(h->rfork, st));
         GLR_CK(h, cudaStreamWaitEvent(h->rstream, h->rfork, 0));
         refreshing.push_back(h);
-        (h->pow_ok ? grouped : h->exact ? exact : trunc).push_back(h);
+        (h->pow_ok ? grouped : h->exact ? exact : (h->tcl && h->k <= 256) ? tclr : trunc).push_back(h);
     }
     if (!grouped.empty() && (rc = refresh_grouped(grouped)) != GLR_OK) return rc;
     if (!exact.empty() && (rc = refresh_exact_grouped(exact)) != GLR_OK) return rc;
     if (!trunc.empty() && (rc = refresh_trunc_grouped(trunc)) != GLR_OK) return rc;
+    if (!tclr.empty() && (rc = refresh_tcl_grouped(tclr)) != GLR_OK) return rc;
     for (glr_handle* h : refreshing) GLR_CK(h, cudaEventRecord(h->rdone, h->rstream));
     for (StepPlan& p : plans)
         if ((rc = select_phase(p, st)) != GLR_OK) return rc;

@@ -59,6 +59,10 @@ struct glr_handle {
     // and Mbar are column-major there, P keeps a transposed copy per projector allocation, and
     // the tensor maps of every operand sit in a device table (not part of the checkpointed state).
     int tcl = 0, rpad = 0, kpad = 0, tc_na = 0, tc_ng = 0, tc_lam_tiles = 0;
+    // refresh scratch of the tcgen05 path (not checkpointed): Mbar row-major and its TF32 low parts,
+    // TF32 transposes of Q and Z, Gram partials, L^{-1}
+    float *Mrow = nullptr, *Mlo = nullptr, *QTt = nullptr, *ZTt = nullptr, *gpart = nullptr, *Linv = nullptr;
+    float* Qbuf0 = nullptr;                       // Q's first allocation (Q and Qn trade places)
     float* Pbuf0 = nullptr;                    // the first projector allocation (P and Pprev trade places)
     float *PT0 = nullptr, *PT1 = nullptr;      // P^T of Pbuf0 / of the other allocation (rpad x m')
     float *WT = nullptr, *YTk = nullptr, *RbarT = nullptr;   // W^T (n' x kpad), Y^T (kpad x m'), Rbar^T (n' x rpad)
@@ -176,7 +180,8 @@ int gemm(glr_handle* h, const GemmDesc& d, cudaStream_t st);
 
 // The tcgen05 large-matrix path (glr_tc_host.cu): eligibility, buffers, tensor maps.
 enum TcMap { kMapBt, kMapPT0, kMapPT1, kMapP0, kMapP1, kMapRwT, kMapMbarT, kMapYT, kMapYt, kMapWT, kMapY, kMapYtJn,
-             kMapYtJm, kMapRbarT, kMapBtD, kMapMbarL, kMapMbarU, kMapMo, kMapVo, kNumTcMaps };
+             kMapYtJm, kMapRbarT, kMapBtD, kMapMbarL, kMapMbarU, kMapMo, kMapVo,
+             kMapMrow, kMapMlo, kMapQTtA, kMapQTtB, kMapZTtA, kMapZTtB, kMapQA, kMapQA1, kMapZA, kMapLinv, kNumTcMaps };
 // After the fixed maps: two slots of N gradient maps, then two slots for X (the caller's buffers,
 // re-described only when a pointer changes).
 const CUtensorMap* tcl_grad_maps(glr_handle* h, const void* const* G, cudaStream_t st, int* rc);
@@ -201,6 +206,9 @@ int refresh_tail(glr_handle* h, cudaStream_t st);
 int refresh_finish(glr_handle* h, cudaStream_t st);
 int refresh_power(glr_handle* h, cudaStream_t st);
 int refresh_trunc_grouped(std::vector<glr_handle*>& hs);
+int refresh_tcl_grouped(std::vector<glr_handle*>& hs);    // tcgen05 path (k <= 256)
+int cholqr(glr_handle* h, float*& A, float*& tmp, int rows, cudaStream_t st);
+int refresh_finish(glr_handle* h, cudaStream_t st);
 int refresh_grouped(std::vector<glr_handle*>& hs);
 int refresh_exact_grouped(std::vector<glr_handle*>& hs);
 

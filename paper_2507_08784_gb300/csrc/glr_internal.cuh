@@ -238,6 +238,11 @@ cudaError_t cholesky(float* A, int n, float* scratch, int* flag, cudaStream_t st
 // S = L^{-T} for L L^T = G (n x n SPD, n <= 256), one CTA with the factor in shared memory; the
 // same shifted retries as cholesky(), attempts counted in *flag.
 cudaError_t chol_inverse(const float* G, int n, float* S, int* flag, cudaStream_t st);
+// The same factor and inverse for several Gram matrices (one CTA each), each given as the sum of
+// nparts partial matrices (leading dimension ld, ld * ld apart); writes L^{-1} row-major ld x ld.
+struct CholMat { const float* part; int nparts, ld, n; float* out; int* flag; };
+struct CholGroup { int nmat; CholMat mat[64]; };
+cudaError_t chol_group(const CholGroup& g, cudaStream_t st);
 
 // Full-basis refresh of several matrices at once (k_jacobi.cu): parallel cyclic Jacobi on each
 // n x n Gram matrix H (n <= 1024; H and H2 are overwritten, the eigenvalues end in evals) with
@@ -259,11 +264,12 @@ struct JacobiGroup {
     JacobiMat mat[kGroupMax];
 };
 // The k x k Rayleigh-Ritz eigenproblems of truncated refreshes (k_eig.cu): one CTA per matrix,
-// H (row-major n x n, n <= 256, read only) -> eigenvalues (unsorted) and eigenvectors V (row-major
+// H (row-major, n <= 256, read only; summed from partial matrices) -> eigenvalues (unsorted) and eigenvectors V (row-major
 // n x n, column j for evals[j]); sweeps done in *sweeps.
 struct EigMat {
     int n; float tol;
-    const float* H; float* V; float* evals; int* sweeps;
+    const float* H; int nparts, ld;       // H = the sum of nparts matrices (leading dimension ld, ld * ld apart)
+    float* V; float* evals; int* sweeps;
 };
 constexpr int kEigGroupMax = 64;
 struct EigGroup {
@@ -427,6 +433,12 @@ struct TcMat {
     float* X; float* Mo; float* Vo;
     int* nonfinite;                                   // Compose: counts warps that found a NaN / Inf in Mbar
     uint64_t seed; uint32_t t;
+    // refresh products (PowT, PowN, Gram, Apply): a second A operand (PowN split), the rows of the
+    // operand they stream, their outputs (fp32, leading dimension ld_out) and TF32 transposes
+    const CUtensorMap* mA2;
+    int rows, ld_out, split, chunk;
+    float* out; float* outT;
+    float* MbarRow;                                   // Compose on a refresh step: Mbar row-major too
 };
 struct TcGroup {
     int nmat, total_tiles;
@@ -445,6 +457,16 @@ cudaError_t launch_lambda(TcGroup& g, cudaStream_t st);
 cudaError_t launch_pbuild(TcGroup& g, cudaStream_t st);
 cudaError_t launch_rbar(TcGroup& g, cudaStream_t st);
 cudaError_t launch_update(TcGroup& g, cudaStream_t st);
+// Truncated refresh products (k_tc.cu): PowT Z = Mbar^T Q, PowN Q = Mbar Z (TF32, or with the
+// split A = A_hi + A_lo for fp32-level accuracy), Gram partial sums of X^T X over row chunks, Apply
+// X <- X Linv^T.  Each writes its fp32 result and a TF32-rounded transpose.
+cudaError_t launch_powt(TcGroup& g, cudaStream_t st);
+cudaError_t launch_pown(TcGroup& g, cudaStream_t st);
+cudaError_t launch_gram(TcGroup& g, cudaStream_t st);
+cudaError_t launch_apply(TcGroup& g, cudaStream_t st);
+constexpr int kGramChunk = 512;                  // rows per Gram partial
+// Mlo = Mrow - trunc_tf32(Mrow), elementwise over n elements
+cudaError_t split_lo(const float* src, float* lo, int64_t n, cudaStream_t st);
 int compose_bn();
 // dst (cols x ldd) = src^T rounded to TF32 (src row-major rows x cols, leading dimension lds)
 cudaError_t transpose_round(float* dst, int ldd, const float* src, int rows, int cols, int lds, cudaStream_t st);

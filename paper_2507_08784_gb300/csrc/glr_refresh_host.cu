@@ -227,7 +227,7 @@ int refresh_trunc_grouped(std::vector<glr_handle*>& hs) {
                 EigMat& M = g.mat[g.nmat++];
                 const int n = h->k;
                 M.n = n; M.tol = 4.f * 5.96e-8f * sqrtf(static_cast<float>(n)) + 1e-7f;
-                M.H = h->Hk; M.V = h->Vk; M.evals = h->evals; M.sweeps = h->dflags + 1;
+                M.H = h->Hk; M.nparts = 1; M.ld = n; M.V = h->Vk; M.evals = h->evals; M.sweeps = h->dflags + 1;
             }
             {
                 PhaseScope ps(h0, GLR_PH_REFRESH, s0);
@@ -298,6 +298,190 @@ int refresh_trunc_grouped(std::vector<glr_handle*>& hs) {
             g_ws = nullptr;
             if (rc != GLR_OK) return rc;
         }
+    }
+    return GLR_OK;
+}
+
+
+// ---- the tcgen05 path's refresh: every stage one grouped launch for all refreshing matrices ----
+namespace {
+
+tc::TcMat refresh_mat(const glr_handle* h) {
+    tc::TcMat M{};
+    M.mp = h->mp; M.np = h->np; M.N = h->N; M.r = h->r; M.rpad = h->rpad; M.k = h->k; M.kpad = h->kpad;
+    M.transposed = h->transposed; M.gdtype = h->s.grad_dtype;
+    return M;
+}
+
+// One op over the handles for which fill(h, M) returns true, kTcGroupMax matrices per launch, on st.
+template <class Fill>
+int refresh_op(std::vector<glr_handle*>& hs, cudaError_t (*launch)(tc::TcGroup&, cudaStream_t), cudaStream_t st,
+               Fill fill) {
+    static thread_local tc::TcGroup g;
+    size_t i = 0;
+    while (i < hs.size()) {
+        g.nmat = 0; g.total_tiles = 0; g.err = nullptr;
+        glr_handle* h0 = nullptr;
+        for (; i < hs.size() && g.nmat < tc::kTcGroupMax; ++i) {
+            glr_handle* h = hs[i];
+            tc::TcMat M = refresh_mat(h);
+            if (!fill(h, M)) continue;
+            if (!h0) { h0 = h; g.err = h->dflags + 2; }
+            M.tile0 = g.total_tiles;
+            g.total_tiles += M.ntiles;
+            g.mat[g.nmat++] = M;
+        }
+        if (h0 && g.total_tiles > 0) {
+            PhaseScope ps(h0, GLR_PH_REFRESH, st);
+            GLR_LAUNCH(h0, 1, launch(g, st));
+        }
+    }
+    return GLR_OK;
+}
+
+int cdiv(int a, int b) { return (a + b - 1) / b; }
+
+// X^T X (Gram partials over row chunks), its factor L^{-1}, then X <- X L^{-T} (and X^T): the
+// CholeskyQR of X = Z (n' rows) or Q (m' rows) in TF32 products.
+int cholqr_tc(std::vector<glr_handle*>& hs, bool zside, cudaStream_t st, const std::vector<int>& active) {
+    std::vector<glr_handle*> act;
+    for (size_t i = 0; i < hs.size(); ++i) if (active[i]) act.push_back(hs[i]);
+    int rc = refresh_op(act, tc::launch_gram, st, [zside](glr_handle* h, tc::TcMat& M) {
+        M.rows = zside ? h->np : h->mp;
+        M.mA = tcl_map(h, zside ? kMapZTtA : kMapQTtA); M.mB = tcl_map(h, zside ? kMapZTtB : kMapQTtB);
+        M.out = h->gpart; M.ntiles = cdiv(M.rows, tc::kGramChunk);
+        return true;
+    });
+    if (rc != GLR_OK) return rc;
+    for (size_t c0 = 0; c0 < act.size(); c0 += 64) {
+        CholGroup cg{};
+        for (size_t i = c0; i < act.size() && i < c0 + 64; ++i) {
+            glr_handle* h = act[i];
+            CholMat& C = cg.mat[cg.nmat++];
+            C.part = h->gpart; C.nparts = cdiv(zside ? h->np : h->mp, tc::kGramChunk); C.ld = h->kpad; C.n = h->k;
+            C.out = h->Linv; C.flag = h->dflags + 0;
+        }
+        PhaseScope ps(act[c0], GLR_PH_REFRESH, st);
+        GLR_LAUNCH(act[c0], 1, chol_group(cg, st));
+    }
+    return refresh_op(act, tc::launch_apply, st, [zside](glr_handle* h, tc::TcMat& M) {
+        M.rows = zside ? h->np : h->mp;
+        M.mA = tcl_map(h, zside ? kMapZA : (h->Q == h->Qbuf0 ? kMapQA : kMapQA1)); M.mB = tcl_map(h, kMapLinv);
+        M.out = zside ? h->Z : h->Q; M.outT = zside ? h->ZTt : h->QTt; M.ld_out = h->k;
+        M.ntiles = cdiv(M.rows, 128);
+        return true;
+    });
+}
+
+}  // namespace
+
+// Truncated refreshes on the tcgen05 path (k <= 256; Mbar column-major, plus the row-major copy
+// the compose pass wrote on this step).  q block power iterations from the previous basis (a
+// seeded Gaussian block at the first refresh): Z = Mbar^T Q and Q = Mbar Z as TF32 tcgen05
+// products, each re-orthonormalised by a TF32 CholeskyQR (the span is what the iteration needs);
+// the last Q = Mbar Z multiplies Mbar's TF32 low parts too, so the subspace it spans is exact to
+// fp32 level for the iterate it is applied to.  Then CholeskyQR2 in fp32 (orthonormal to
+// rounding), the Rayleigh-Ritz matrix H = (Mbar^T Q)^T (Mbar^T Q), the k x k eigenproblems
+// (k_eig.cu) and each handle's finish (sort, signs, Householder WY form).
+int refresh_tcl_grouped(std::vector<glr_handle*>& hs) {
+    glr_handle* h0 = hs[0];
+    cudaStream_t s0 = h0->rstream;
+    int rc;
+    for (glr_handle* h : hs) GLR_CK(h0, cudaStreamWaitEvent(s0, h->rfork, 0));
+    int q = 0;
+    for (glr_handle* h : hs) {
+        PhaseScope ps(h, GLR_PH_REFRESH, s0);
+        if (h->refreshes == 0 && !h->basis_from_user)
+            GLR_LAUNCH(h, 1, random_block(h->Q, h->mp, h->k, h->s.seed, static_cast<uint32_t>(h->t), s0));
+        GLR_LAUNCH(h, 1, tc::transpose_round(h->QTt, h->mp, h->Q, h->mp, h->k, h->k, s0));
+        q = std::max(q, h->s.power_iters);
+    }
+    std::vector<int> active(hs.size(), 1);
+    for (int it = 0; it < q; ++it) {
+        for (size_t i = 0; i < hs.size(); ++i) active[i] = it < hs[i]->s.power_iters ? 1 : 0;
+        auto is_active = [&](glr_handle* h) {
+            for (size_t i = 0; i < hs.size(); ++i) if (hs[i] == h) return active[i] != 0;
+            return false;
+        };
+        // Z = Mbar^T Q
+        rc = refresh_op(hs, tc::launch_powt, s0, [&](glr_handle* h, tc::TcMat& M) {
+            if (!is_active(h)) return false;
+            M.rows = h->np; M.mA = tcl_map(h, kMapMbarT); M.mB = tcl_map(h, kMapQTtB);
+            M.out = h->Z; M.outT = h->ZTt; M.ld_out = h->k; M.ntiles = cdiv(h->np, 256);
+            return true;
+        });
+        if (rc != GLR_OK) return rc;
+        if ((rc = cholqr_tc(hs, true, s0, active)) != GLR_OK) return rc;
+        // Q = Mbar Z; a handle's last iteration with Mbar's low parts
+        for (size_t i = 0; i < hs.size(); ++i) {
+            glr_handle* h = hs[i];
+            if (!active[i] || it != h->s.power_iters - 1) continue;
+            PhaseScope ps(h, GLR_PH_REFRESH, s0);
+            GLR_LAUNCH(h, 1, tc::split_lo(h->Mrow, h->Mlo, (int64_t)h->mp * h->np, s0));
+        }
+        rc = refresh_op(hs, tc::launch_pown, s0, [&](glr_handle* h, tc::TcMat& M) {
+            if (!is_active(h)) return false;
+            M.rows = h->mp; M.mA = tcl_map(h, kMapMrow); M.mA2 = tcl_map(h, kMapMlo); M.mB = tcl_map(h, kMapZTtB);
+            M.split = it == h->s.power_iters - 1 ? 1 : 0;
+            M.out = h->Q; M.outT = h->QTt; M.ld_out = h->k; M.ntiles = cdiv(h->mp, 256);
+            return true;
+        });
+        if (rc != GLR_OK) return rc;
+        std::vector<int> mid(hs.size(), 0);
+        for (size_t i = 0; i < hs.size(); ++i) mid[i] = active[i] && it < hs[i]->s.power_iters - 1 ? 1 : 0;
+        if ((rc = cholqr_tc(hs, false, s0, mid)) != GLR_OK) return rc;
+    }
+    // CholeskyQR2 in fp32 on each handle's stream, then Q^T for the Rayleigh-Ritz product
+    GLR_CK(h0, cudaEventRecord(h0->rpow, s0));
+    for (glr_handle* h : hs) {
+        if (h != h0) GLR_CK(h, cudaStreamWaitEvent(h->rstream, h0->rpow, 0));
+        PhaseScope ps(h, GLR_PH_REFRESH, h->rstream);
+        g_ws = h->gemm_ws;
+        rc = cholqr(h, h->Q, h->Qn, h->mp, h->rstream);
+        if (rc == GLR_OK) rc = cholqr(h, h->Q, h->Qn, h->mp, h->rstream);
+        g_ws = nullptr;
+        if (rc != GLR_OK) return rc;
+        GLR_LAUNCH(h, 1, tc::transpose_round(h->QTt, h->mp, h->Q, h->mp, h->k, h->k, h->rstream));
+        if (h != h0) {
+            GLR_CK(h, cudaEventRecord(h->rpow, h->rstream));
+            GLR_CK(h0, cudaStreamWaitEvent(s0, h->rpow, 0));
+        }
+    }
+    // Rayleigh-Ritz: Z = Mbar^T Q, H = Z^T Z (Gram partials), the eigenproblems
+    rc = refresh_op(hs, tc::launch_powt, s0, [&](glr_handle* h, tc::TcMat& M) {
+        M.rows = h->np; M.mA = tcl_map(h, kMapMbarT); M.mB = tcl_map(h, kMapQTtB);
+        M.out = h->Z; M.outT = h->ZTt; M.ld_out = h->k; M.ntiles = cdiv(h->np, 256);
+        return true;
+    });
+    if (rc != GLR_OK) return rc;
+    rc = refresh_op(hs, tc::launch_gram, s0, [](glr_handle* h, tc::TcMat& M) {
+        M.rows = h->np; M.mA = tcl_map(h, kMapZTtA); M.mB = tcl_map(h, kMapZTtB);
+        M.out = h->gpart; M.ntiles = cdiv(h->np, tc::kGramChunk);
+        return true;
+    });
+    if (rc != GLR_OK) return rc;
+    for (size_t c0 = 0; c0 < hs.size(); c0 += kEigGroupMax) {
+        EigGroup g{};
+        g.max_sweeps = 40;
+        for (size_t i = c0; i < hs.size() && i < c0 + (size_t)kEigGroupMax; ++i) {
+            glr_handle* h = hs[i];
+            EigMat& M = g.mat[g.nmat++];
+            const int n = h->k;
+            M.n = n; M.tol = 4.f * 5.96e-8f * sqrtf(static_cast<float>(n)) + 1e-7f;
+            M.H = h->gpart; M.nparts = cdiv(h->np, tc::kGramChunk); M.ld = h->kpad;
+            M.V = h->Vk; M.evals = h->evals; M.sweeps = h->dflags + 1;
+        }
+        PhaseScope ps(hs[c0], GLR_PH_REFRESH, s0);
+        GLR_LAUNCH(hs[c0], 1, eig_tmem_group(g, s0));
+    }
+    GLR_CK(h0, cudaEventRecord(h0->rpow, s0));
+    for (glr_handle* h : hs) {
+        if (h != h0) GLR_CK(h, cudaStreamWaitEvent(h->rstream, h0->rpow, 0));
+        PhaseScope ps(h, GLR_PH_REFRESH, h->rstream);
+        g_ws = h->gemm_ws;
+        rc = refresh_finish(h, h->rstream);
+        g_ws = nullptr;
+        if (rc != GLR_OK) return rc;
     }
     return GLR_OK;
 }

@@ -56,6 +56,15 @@ const CUtensorMap* tcl_map_PT(const glr_handle* h, const float* P) {
 int tcl_maps(glr_handle* h) {
     const uint64_t mp = h->mp, np = h->np, N = h->N, r = h->r, k = h->k;
     const uint64_t rp = h->rpad, kp = h->kpad;
+    {   // refresh scratch, allocated after the checkpointed state
+        int rc = GLR_OK;
+        auto A = [&](float** p, size_t cnt) { if (rc == GLR_OK) rc = alloc(h, p, cnt); };
+        const size_t nch = (np + tc::kGramChunk - 1) / tc::kGramChunk;
+        A(&h->Mrow, mp * np); A(&h->Mlo, mp * np);
+        A(&h->QTt, kp * mp); A(&h->ZTt, kp * np);
+        A(&h->gpart, std::max<size_t>(nch, 1) * kp * kp); A(&h->Linv, kp * kp);
+        if (rc != GLR_OK) return rc;
+    }
     std::vector<CUtensorMap> maps(kNumTcMaps);
     float* Pother = h->P == h->Pbuf0 ? h->Pprev : h->P;
     bool ok = true;
@@ -83,6 +92,18 @@ int tcl_maps(glr_handle* h) {
     m2(kMapYtJn, h->YtJ, k, r, k, (uint32_t)rp);           // Yt[J, :] (r x k) as the N operand
     m2(kMapYtJm, h->YtJ, k, r, k, 128);                    // ... and as the M operand
     m2(kMapRbarT, h->RbarT, rp, np, rp, 128);              // Rbar^T: n' x rpad
+    // the refresh products
+    m2(kMapMrow, h->Mrow, np, mp, np, 128);                // Mbar row-major: m' x n'
+    m2(kMapMlo, h->Mlo, np, mp, np, 128);                  // its TF32 low parts
+    m2(kMapQTtA, h->QTt, mp, kp, mp, 128);                 // Q^T (kpad x m') in 128-row slices
+    m2(kMapQTtB, h->QTt, mp, kp, mp, (uint32_t)kp);        // ... and whole (the N operand)
+    m2(kMapZTtA, h->ZTt, np, kp, np, 128);                 // Z^T (kpad x n')
+    m2(kMapZTtB, h->ZTt, np, kp, np, (uint32_t)kp);
+    h->Qbuf0 = h->Q;
+    m2(kMapQA, h->Q, k, mp, k, 128);                       // Q (either allocation), Z row-major (rows x k) as A
+    m2(kMapQA1, h->Qn, k, mp, k, 128);
+    m2(kMapZA, h->Z, k, np, k, 128);
+    m2(kMapLinv, h->Linv, kp, kp, kp, (uint32_t)kp);       // L^{-1}, row-major kpad x kpad
     // epilogue data tiles (no swizzle unless noted)
     auto plain = [&](int idx, const void* base, int rank, const uint64_t* dims, const uint64_t* str, const uint32_t* box,
                      CUtensorMapSwizzle swz) {

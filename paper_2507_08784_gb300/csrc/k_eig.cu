@@ -64,7 +64,11 @@ __global__ void __launch_bounds__(ET, 1) eig_tmem_kernel(const __grid_constant__
     for (int r = t; r <= n; r += ET) off[r] = r * n - r * (r + 1) / 2;
     __syncthreads();
     for (int r = warp; r < n; r += ET / 32)            // H (row-major n x n) -> packed upper triangle
-        for (int c = r + lane; c < n; c += 32) Hs[off[r] + c] = M.H[(size_t)r * n + c];
+        for (int c = r + lane; c < n; c += 32) {
+            float v = 0.f;
+            for (int p = 0; p < M.nparts; ++p) v += M.H[(size_t)p * M.ld * M.ld + (size_t)r * M.ld + c];
+            Hs[off[r] + c] = v;
+        }
     tm_fence_after();
     const uint32_t tmem = tbase;
     // this warp's lane quadrant: W rows a = h 128 + 32 qd + lane of every half h
@@ -205,7 +209,8 @@ cudaError_t eig_tmem_group(const EigGroup& g, cudaStream_t st) {
     if (g.nmat <= 0) return cudaSuccess;
     int nmax = 0;
     for (int i = 0; i < g.nmat; ++i) {
-        if (g.mat[i].n < 2 || g.mat[i].n > kEigMaxN) return cudaErrorInvalidValue;
+        if (g.mat[i].n < 2 || g.mat[i].n > kEigMaxN || g.mat[i].ld < g.mat[i].n || g.mat[i].nparts < 1)
+            return cudaErrorInvalidValue;
         nmax = g.mat[i].n > nmax ? g.mat[i].n : nmax;
     }
     const size_t smem = sizeof(float) * (size_t)nmax * (nmax + 1) / 2;

@@ -378,7 +378,11 @@ __device__ __forceinline__ int tri(int i, int l) { return i * (i + 1) / 2 + l; }
 // copies the column it reads into a contiguous array (a column of the packed triangle is strided
 // by the row lengths, which would make the lanes' reads collide in the banks).  S (row-major
 // n x n) is the transpose of L^{-1}.
-__global__ void __launch_bounds__(1024) chol_inverse_kernel(const float* G, int n, float* S, int* flag) {
+// The Gram matrix is the sum of `nparts` partial matrices (leading dimension ld, spaced ld * ld
+// apart).  Output: S = L^{-T} (row-major n x n), or with out_linv L^{-1} (row-major ld x ld, zero
+// above the diagonal and outside n x n).
+__device__ __forceinline__ void chol_inverse_body(const float* G, int nparts, int ld, int n, float* S, int out_linv,
+                                                  int* flag) {
     extern __shared__ float L[];                       // n (n + 1) / 2 packed, then n + n temporaries
     float* col = L + n * (n + 1) / 2;
     float* tmp = col + n;
@@ -387,7 +391,11 @@ __global__ void __launch_bounds__(1024) chol_inverse_kernel(const float* G, int 
     __shared__ float shift, trace;
     if (warp == 0) {                                   // trace: a warp sum in a fixed order
         float tr = 0.f;
-        for (int i = lane; i < n; i += 32) tr += G[(size_t)i * n + i];
+        for (int i = lane; i < n; i += 32) {
+            float gi = 0.f;
+            for (int p = 0; p < nparts; ++p) gi += G[(size_t)p * ld * ld + (size_t)i * ld + i];
+            tr += gi;
+        }
 #pragma unroll
         for (int o = 16; o > 0; o >>= 1) tr += __shfl_xor_sync(0xffffffffu, tr, o);
         if (lane == 0) { trace = tr; shift = 0.f; }
@@ -396,7 +404,11 @@ __global__ void __launch_bounds__(1024) chol_inverse_kernel(const float* G, int 
     int attempt = 0;
     for (; attempt < 6; ++attempt) {
         for (int i = warp; i < n; i += nw)
-            for (int l = lane; l <= i; l += 32) L[tri(i, l)] = G[(size_t)i * n + l] + (l == i ? shift : 0.f);
+            for (int l = lane; l <= i; l += 32) {
+                float gil = 0.f;
+                for (int p = 0; p < nparts; ++p) gil += G[(size_t)p * ld * ld + (size_t)i * ld + l];
+                L[tri(i, l)] = gil + (l == i ? shift : 0.f);
+            }
         if (tid == 0) fail = 0;
         __syncthreads();
         const float thresh = 1e-12f * fmaxf(trace / n, 1e-30f);
@@ -445,12 +457,44 @@ __global__ void __launch_bounds__(1024) chol_inverse_kernel(const float* G, int 
         if (tid == 0) L[tri(j, j)] = ajj;
         __syncthreads();
     }
+    if (out_linv) {
+        for (int e = tid; e < ld * ld; e += blockDim.x) {
+            const int r = e / ld, c = e % ld;
+            S[e] = (c <= r && r < n) ? L[tri(r, c)] : 0.f;
+        }
+        return;
+    }
     for (int e = tid; e < n * n; e += blockDim.x) {
         const int r = e / n, c = e % n;
         S[e] = c >= r ? L[tri(c, r)] : 0.f;
     }
 }
+
+__global__ void __launch_bounds__(1024) chol_inverse_kernel(const float* G, int n, float* S, int* flag) {
+    chol_inverse_body(G, 1, n, n, S, 0, flag);
+}
+__global__ void __launch_bounds__(1024) chol_group_kernel(const __grid_constant__ CholGroup g) {
+    const CholMat& M = g.mat[blockIdx.x];
+    chol_inverse_body(M.part, M.nparts, M.ld, M.n, M.out, 1, M.flag);
+}
 }  // namespace
+
+cudaError_t chol_group(const CholGroup& g, cudaStream_t st) {
+    if (g.nmat <= 0) return cudaSuccess;
+    int nmax = 0;
+    for (int i = 0; i < g.nmat; ++i) {
+        if (g.mat[i].n < 1 || g.mat[i].n > 256 || g.mat[i].ld < g.mat[i].n) return cudaErrorInvalidValue;
+        nmax = g.mat[i].n > nmax ? g.mat[i].n : nmax;
+    }
+    const size_t smem = sizeof(float) * ((size_t)nmax * (nmax + 1) / 2 + 2 * nmax);
+    {   // per device: set on every call (cheap next to the launch)
+        const cudaError_t ea = cudaFuncSetAttribute(chol_group_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                                   (int)(sizeof(float) * (256 * 257 / 2 + 2 * 256)));
+        if (ea != cudaSuccess) return ea;
+    }
+    chol_group_kernel<<<g.nmat, 1024, smem, st>>>(g);
+    return cudaGetLastError();
+}
 
 cudaError_t chol_inverse(const float* G, int n, float* S, int* flag, cudaStream_t st) {
     if (n < 1 || n > 256) return cudaErrorInvalidValue;

@@ -534,6 +534,14 @@ struct Compose {
                     bad |= !isfinite(v);
                     M.Mbar[(int64_t)(c0 + j) * M.mp + a] = v;
                 }
+            if (M.MbarRow) {                              // a refresh step: Mbar row-major as well
+                float* row = M.MbarRow + (int64_t)a * M.np + c0;
+#pragma unroll
+                for (int j = 0; j < 16; j += 4)
+                    if (c0 + j < M.np)
+                        *reinterpret_cast<float4*>(row + j) =
+                            make_float4(acc[j] * invN, acc[j + 1] * invN, acc[j + 2] * invN, acc[j + 3] * invN);
+            }
         }
         flag_nonfinite(bad, M.nonfinite);
         return true;
@@ -856,6 +864,154 @@ struct Update {
     }
 };
 
+// ------------------------------------------------------------------------------------------
+// Refresh products.  PowT: tile = 256 rows c of n' (two halves of 128); D_h (128 x kpad) =
+// Mbar^T[c, :] Q over K = m' (A = Mbar^T, B = Q^T TF32, kpad x m').  PowN: tile = 256 rows a of
+// m'; D_h = Mbar[a, :] Z over K = n' (A = Mbar row-major, B = Z^T TF32, kpad x n'); with `split`
+// the A slices of Mbar's low parts (Mbar - trunc_tf32(Mbar)) are multiplied too, so the product is
+// exact to fp32 level for the TF32 value of B.  The epilogue writes out[row][q] (fp32, leading
+// dimension ld_out, q < k) and outT[q][row] (TF32).
+// ------------------------------------------------------------------------------------------
+template <int kDir>
+struct Pow : NoData {
+    static __device__ __forceinline__ int nk(const TcGroup& g, const Tile& t) {
+        const TcMat& M = g.mat[t.mat];
+        return ((kDir == 0 ? M.mp : M.np) + 31) / 32;
+    }
+    static __device__ __forceinline__ uint32_t tx_bytes(const TcGroup& g, const Tile& t, int) {
+        const TcMat& M = g.mat[t.mat];
+        return (M.split ? 4u : 2u) * 16384u + (uint32_t)M.kpad * 128u;
+    }
+    static __device__ __forceinline__ void load(const TcGroup& g, const Tile& t, int kc, uint32_t st, uint32_t bar) {
+        const TcMat& M = g.mat[t.mat];
+        tma_load_2d(st, M.mA, kc * 32, t.lt * 256, bar);
+        tma_load_2d(st + 16384u, M.mA, kc * 32, t.lt * 256 + 128, bar);
+        uint32_t o = 32768u;
+        if (M.split) {
+            tma_load_2d(st + o, M.mA2, kc * 32, t.lt * 256, bar);
+            tma_load_2d(st + o + 16384u, M.mA2, kc * 32, t.lt * 256 + 128, bar);
+            o += 32768u;
+        }
+        tma_load_2d(st + o, M.mB, kc * 32, 0, bar);
+    }
+    static __device__ __forceinline__ void mma(const TcGroup& g, const Tile& t, int kc, uint32_t st, uint32_t d) {
+        const TcMat& M = g.mat[t.mat];
+        const uint32_t b = st + (M.split ? 65536u : 32768u);
+        mma_slice(d, st, b, M.kpad, kc == 0);
+        mma_slice(d + (uint32_t)M.kpad, st + 16384u, b, M.kpad, kc == 0);
+        if (M.split) {
+            mma_slice(d, st + 32768u, b, M.kpad, false);
+            mma_slice(d + (uint32_t)M.kpad, st + 49152u, b, M.kpad, false);
+        }
+    }
+    static __device__ __forceinline__ bool epilogue(const TcGroup& g, const Tile& t, uint32_t tl, int warp, int lane, DataRing&) {
+        const TcMat& M = g.mat[t.mat];
+        const int h = warp >> 2;
+        const int c = t.lt * 256 + h * 128 + 32 * (warp & 3) + lane;
+        for (int q = 0; q < M.kpad; q += 16) {
+            float v[16];
+            tmem_ld16(tl + (uint32_t)(h * M.kpad + q), v);
+            if (c >= M.rows) continue;
+#pragma unroll
+            for (int j = 0; j < 16; j += 4)
+                if (q + j < M.k)
+                    *reinterpret_cast<float4*>(M.out + (int64_t)c * M.ld_out + q + j) =
+                        make_float4(v[j], v[j + 1], v[j + 2], v[j + 3]);
+#pragma unroll
+            for (int j = 0; j < 16; ++j) M.outT[(int64_t)(q + j) * M.rows + c] = rna_tf32(v[j]);
+        }
+        return true;
+    }
+};
+using PowT = Pow<0>;
+using PowN = Pow<1>;
+
+// ------------------------------------------------------------------------------------------
+// Gram: tile = (matrix, chunk of kGramChunk rows).  D_h (128 x kpad) = X^T[h 128 .., rows] X over
+// the chunk's rows (A = X^T slices of 128 rows, B = X^T with all kpad rows; X^T is TF32, kpad x
+// rows).  The epilogue writes the chunk's partial Gram matrix out[chunk][l][l'] (kpad x kpad);
+// the consumer sums the chunks in order.
+// ------------------------------------------------------------------------------------------
+struct Gram : NoData {
+    static __device__ __forceinline__ int halves(const TcMat& M) { return (M.kpad + 127) / 128; }
+    static __device__ __forceinline__ int nk(const TcGroup& g, const Tile& t) {
+        const TcMat& M = g.mat[t.mat];
+        const int r0 = t.lt * kGramChunk;
+        const int len = M.rows - r0 < kGramChunk ? M.rows - r0 : kGramChunk;
+        return (len + 31) / 32;
+    }
+    static __device__ __forceinline__ uint32_t tx_bytes(const TcGroup& g, const Tile& t, int) {
+        const TcMat& M = g.mat[t.mat];
+        return (uint32_t)halves(M) * 16384u + (uint32_t)M.kpad * 128u;
+    }
+    static __device__ __forceinline__ void load(const TcGroup& g, const Tile& t, int kc, uint32_t st, uint32_t bar) {
+        const TcMat& M = g.mat[t.mat];
+        const int x = t.lt * kGramChunk + kc * 32;
+        for (int h = 0; h < halves(M); ++h) tma_load_2d(st + h * 16384u, M.mA, x, 128 * h, bar);
+        tma_load_2d(st + 32768u, M.mB, x, 0, bar);
+    }
+    static __device__ __forceinline__ void mma(const TcGroup& g, const Tile& t, int kc, uint32_t st, uint32_t d) {
+        const TcMat& M = g.mat[t.mat];
+        for (int h = 0; h < halves(M); ++h)
+            mma_slice(d + (uint32_t)(h * M.kpad), st + h * 16384u, st + 32768u, M.kpad, kc == 0);
+    }
+    static __device__ __forceinline__ bool epilogue(const TcGroup& g, const Tile& t, uint32_t tl, int warp, int lane, DataRing&) {
+        const TcMat& M = g.mat[t.mat];
+        const int h = warp >> 2;
+        if (h >= halves(M)) return true;
+        const int l = h * 128 + 32 * (warp & 3) + lane;
+        float* out = M.out + ((int64_t)t.lt * M.kpad + l) * M.kpad;
+        for (int q = 0; q < M.kpad; q += 16) {
+            float v[16];
+            tmem_ld16(tl + (uint32_t)(h * M.kpad + q), v);
+            if (l >= M.kpad) continue;
+#pragma unroll
+            for (int j = 0; j < 16; j += 4)
+                *reinterpret_cast<float4*>(out + q + j) = make_float4(v[j], v[j + 1], v[j + 2], v[j + 3]);
+        }
+        return true;
+    }
+};
+
+// ------------------------------------------------------------------------------------------
+// Apply: tile = 128 rows a.  D (128 x kpad) = X[a, :] Linv^T (K = kpad; A = X row-major rows x k,
+// B = Linv row-major kpad x kpad, so that D = X L^{-T}); the epilogue writes X (in place: a tile
+// reads only its own rows, all before the product completes) and X^T (TF32).  Warp w: lanes =
+// rows, w / 4 picks a column half.
+// ------------------------------------------------------------------------------------------
+struct Apply : NoData {
+    static __device__ __forceinline__ int nk(const TcGroup& g, const Tile& t) { return g.mat[t.mat].kpad / 32; }
+    static __device__ __forceinline__ uint32_t tx_bytes(const TcGroup& g, const Tile& t, int) {
+        return 16384u + (uint32_t)g.mat[t.mat].kpad * 128u;
+    }
+    static __device__ __forceinline__ void load(const TcGroup& g, const Tile& t, int kc, uint32_t st, uint32_t bar) {
+        const TcMat& M = g.mat[t.mat];
+        tma_load_2d(st, M.mA, kc * 32, t.lt * 128, bar);
+        tma_load_2d(st + 16384u, M.mB, kc * 32, 0, bar);
+    }
+    static __device__ __forceinline__ void mma(const TcGroup& g, const Tile& t, int kc, uint32_t st, uint32_t d) {
+        mma_slice(d, st, st + 16384u, g.mat[t.mat].kpad, kc == 0);
+    }
+    static __device__ __forceinline__ bool epilogue(const TcGroup& g, const Tile& t, uint32_t tl, int warp, int lane, DataRing&) {
+        const TcMat& M = g.mat[t.mat];
+        const int a = t.lt * 128 + 32 * (warp & 3) + lane;
+        const int hw = M.kpad / 2, q0 = (warp >> 2) * hw;
+        for (int q = q0; q < q0 + hw; q += 16) {
+            float v[16];
+            tmem_ld16(tl + (uint32_t)q, v);
+            if (a >= M.rows) continue;
+#pragma unroll
+            for (int j = 0; j < 16; j += 4)
+                if (q + j < M.k)
+                    *reinterpret_cast<float4*>(M.out + (int64_t)a * M.ld_out + q + j) =
+                        make_float4(v[j], v[j + 1], v[j + 2], v[j + 3]);
+#pragma unroll
+            for (int j = 0; j < 16; ++j) M.outT[(int64_t)(q + j) * M.rows + a] = rna_tf32(v[j]);
+        }
+        return true;
+    }
+};
+
 // Stage bytes of an op for a group (the largest over its matrices).
 template <class Op> size_t stage_bytes_of(const TcMat& M);
 template <> size_t stage_bytes_of<PrevProj>(const TcMat& M) { return (size_t)M.na * 16384 + (size_t)M.rpad * 128; }
@@ -865,6 +1021,10 @@ template <> size_t stage_bytes_of<Lambda>(const TcMat&) { return 2 * 16384; }
 template <> size_t stage_bytes_of<PBuild>(const TcMat& M) { return 16384 + (size_t)M.rpad * 128; }
 template <> size_t stage_bytes_of<RBar>(const TcMat&) { return 2 * 16384; }
 template <> size_t stage_bytes_of<Update>(const TcMat&) { return 2 * 16384; }
+template <> size_t stage_bytes_of<PowT>(const TcMat& M) { return (M.split ? 4 : 2) * 16384 + (size_t)M.kpad * 128; }
+template <> size_t stage_bytes_of<PowN>(const TcMat& M) { return (M.split ? 4 : 2) * 16384 + (size_t)M.kpad * 128; }
+template <> size_t stage_bytes_of<Gram>(const TcMat& M) { return 2 * 16384 + (size_t)M.kpad * 128; }
+template <> size_t stage_bytes_of<Apply>(const TcMat& M) { return 16384 + (size_t)M.kpad * 128; }
 
 // Accumulator columns of one tile (two buffers when two fit in tensor memory).
 template <class Op> int acc_cols_of(const TcMat& M);
@@ -875,6 +1035,10 @@ template <> int acc_cols_of<Lambda>(const TcMat&) { return 128; }
 template <> int acc_cols_of<PBuild>(const TcMat& M) { return M.rpad; }
 template <> int acc_cols_of<RBar>(const TcMat&) { return 128; }
 template <> int acc_cols_of<Update>(const TcMat&) { return 128; }
+template <> int acc_cols_of<PowT>(const TcMat& M) { return 2 * M.kpad; }
+template <> int acc_cols_of<PowN>(const TcMat& M) { return 2 * M.kpad; }
+template <> int acc_cols_of<Gram>(const TcMat& M) { return ((M.kpad + 127) / 128) * M.kpad; }
+template <> int acc_cols_of<Apply>(const TcMat& M) { return M.kpad; }
 
 // Data-stage bytes of an op (0: no data ring).
 template <class Op> size_t dstage_bytes_of(const TcGroup&, const TcMat&) { return 0; }
@@ -937,6 +1101,10 @@ cudaError_t launch_lambda(TcGroup& g, cudaStream_t st) { return launch<Lambda>(g
 cudaError_t launch_pbuild(TcGroup& g, cudaStream_t st) { return launch<PBuild>(g, st); }
 cudaError_t launch_rbar(TcGroup& g, cudaStream_t st) { return launch<RBar>(g, st); }
 cudaError_t launch_update(TcGroup& g, cudaStream_t st) { return launch<Update>(g, st); }
+cudaError_t launch_powt(TcGroup& g, cudaStream_t st) { return launch<PowT>(g, st); }
+cudaError_t launch_pown(TcGroup& g, cudaStream_t st) { return launch<PowN>(g, st); }
+cudaError_t launch_gram(TcGroup& g, cudaStream_t st) { return launch<Gram>(g, st); }
+cudaError_t launch_apply(TcGroup& g, cudaStream_t st) { return launch<Apply>(g, st); }
 
 int compose_bn() { return Compose::BN; }
 
@@ -988,6 +1156,24 @@ __global__ void expire_kernel(int* err, int polls) {
     wait_phase(smem_u32(&bar), 0, &abort_flag, err, polls);
 }
 }  // namespace
+
+namespace {
+// lo = x - (x truncated to TF32): what a TF32 product of x leaves out
+__global__ void split_lo_kernel(const float4* src, float4* lo, int64_t n4) {
+    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n4; i += (int64_t)gridDim.x * blockDim.x) {
+        const float4 v = src[i];
+        auto l = [](float x) { return x - __uint_as_float(__float_as_uint(x) & 0xFFFFE000u); };
+        lo[i] = make_float4(l(v.x), l(v.y), l(v.z), l(v.w));
+    }
+}
+}  // namespace
+
+cudaError_t split_lo(const float* src, float* lo, int64_t n, cudaStream_t st) {
+    if (n % 4) return cudaErrorInvalidValue;
+    split_lo_kernel<<<(unsigned)std::min<int64_t>((n / 4 + 255) / 256, 8 * 152), 256, 0, st>>>(
+        reinterpret_cast<const float4*>(src), reinterpret_cast<float4*>(lo), n / 4);
+    return cudaGetLastError();
+}
 
 cudaError_t expire_wait(int* err, int polls, cudaStream_t st) {
     expire_kernel<<<1, 32, 0, st>>>(err, polls);
