@@ -240,9 +240,32 @@ cudaError_t cholesky(float* A, int n, float* scratch, int* flag, cudaStream_t st
 cudaError_t chol_inverse(const float* G, int n, float* S, int* flag, cudaStream_t st);
 // The same factor and inverse for several Gram matrices (one CTA each), each given as the sum of
 // nparts partial matrices (leading dimension ld, ld * ld apart); writes L^{-1} row-major ld x ld.
-struct CholMat { const float* part; int nparts, ld, n; float* out; int* flag; };
+struct CholMat { const float* part; int nparts, ld, n; float* out; int* flag; int tri_only; };   // tri_only: (U^T)^{-1} of the upper triangle of part (n x n)
 struct CholGroup { int nmat; CholMat mat[64]; };
 cudaError_t chol_group(const CholGroup& g, cudaStream_t st);
+// The end of a truncated refresh for several matrices, one launch per stage: stage 0 sorts each
+// eigenproblem's pairs by descending value and writes W (k x k, unit columns, signs fixed) and the
+// sorted values; 1 fixes the column signs of Q (m' x k); 2 and 3 the Householder reconstruction
+// (top block into Wtop, Y, T, s; then the rows below).
+struct FinishMat {
+    int mp, k;
+    const float* evals; const float* V; float* W; float* evals_sorted;
+    float* Q; float* Wtop; float* Y; float* T; float* s;
+};
+struct FinishGroup { int nmat; FinishMat mat[64]; };
+cudaError_t finish_group(const FinishGroup& g, int stage, cudaStream_t st);
+// C = A B in fp32 (FFMA) for several independent products, one launch: A(i, p) = A[i sAi + p sAp],
+// B(p, j) = B[p sBp + j sBj], C(i, j) = C[i sCi + j sCj]; 64 x 64 output tiles.
+struct GemmMat {
+    int M, N, K;
+    float alpha;                          // C = alpha A B (0 is read as 1)
+    const float* A; int64_t sAi, sAp;
+    const float* B; int64_t sBp, sBj;
+    float* C; int64_t sCi, sCj;
+    int tile0;
+};
+struct GemmGroup { int nmat, total_tiles; GemmMat mat[64]; };
+cudaError_t gemm_group_f32(GemmGroup& g, cudaStream_t st);
 
 // Full-basis refresh of several matrices at once (k_jacobi.cu): parallel cyclic Jacobi on each
 // n x n Gram matrix H (n <= 1024; H and H2 are overwritten, the eigenvalues end in evals) with

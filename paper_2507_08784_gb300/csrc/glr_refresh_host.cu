@@ -341,6 +341,18 @@ int refresh_op(std::vector<glr_handle*>& hs, cudaError_t (*launch)(tc::TcGroup&,
 
 int cdiv(int a, int b) { return (a + b - 1) / b; }
 
+// One grouped fp32 product per handle (fill describes it), 64 per launch.
+template <class Fill>
+int fp32_products(std::vector<glr_handle*>& hs, cudaStream_t st, Fill fill) {
+    for (size_t c0 = 0; c0 < hs.size(); c0 += 64) {
+        GemmGroup gg{};
+        for (size_t i = c0; i < hs.size() && i < c0 + 64; ++i) fill(hs[i], gg.mat[gg.nmat++]);
+        PhaseScope ps(hs[c0], GLR_PH_REFRESH, st);
+        GLR_LAUNCH(hs[c0], 1, gemm_group_f32(gg, st));
+    }
+    return GLR_OK;
+}
+
 // X^T X (Gram partials over row chunks), its factor L^{-1}, then X <- X L^{-T} (and X^T): the
 // CholeskyQR of X = Z (n' rows) or Q (m' rows) in TF32 products.
 int cholqr_tc(std::vector<glr_handle*>& hs, bool zside, cudaStream_t st, const std::vector<int>& active) {
@@ -431,21 +443,36 @@ int refresh_tcl_grouped(std::vector<glr_handle*>& hs) {
         for (size_t i = 0; i < hs.size(); ++i) mid[i] = active[i] && it < hs[i]->s.power_iters - 1 ? 1 : 0;
         if ((rc = cholqr_tc(hs, false, s0, mid)) != GLR_OK) return rc;
     }
-    // CholeskyQR2 in fp32 on each handle's stream, then Q^T for the Rayleigh-Ritz product
-    GLR_CK(h0, cudaEventRecord(h0->rpow, s0));
-    for (glr_handle* h : hs) {
-        if (h != h0) GLR_CK(h, cudaStreamWaitEvent(h->rstream, h0->rpow, 0));
-        PhaseScope ps(h, GLR_PH_REFRESH, h->rstream);
-        g_ws = h->gemm_ws;
-        rc = cholqr(h, h->Q, h->Qn, h->mp, h->rstream);
-        if (rc == GLR_OK) rc = cholqr(h, h->Q, h->Qn, h->mp, h->rstream);
-        g_ws = nullptr;
-        if (rc != GLR_OK) return rc;
-        GLR_LAUNCH(h, 1, tc::transpose_round(h->QTt, h->mp, h->Q, h->mp, h->k, h->k, h->rstream));
-        if (h != h0) {
-            GLR_CK(h, cudaEventRecord(h->rpow, h->rstream));
-            GLR_CK(h0, cudaStreamWaitEvent(s0, h->rpow, 0));
+    // CholeskyQR2 in fp32 (grouped FFMA products and factors), then Q^T for the Rayleigh-Ritz
+    // product
+    for (int pass = 0; pass < 2; ++pass) {
+        if ((rc = fp32_products(hs, s0, [](glr_handle* h, GemmMat& G) {      // Gram Q^T Q
+                 G.M = h->k; G.N = h->k; G.K = h->mp;
+                 G.A = h->Q; G.sAi = 1; G.sAp = h->k; G.B = h->Q; G.sBp = h->k; G.sBj = 1;
+                 G.C = h->gram; G.sCi = h->k; G.sCj = 1;
+             })) != GLR_OK)
+            return rc;
+        for (size_t c0 = 0; c0 < hs.size(); c0 += 64) {
+            CholGroup cg{};
+            for (size_t i = c0; i < hs.size() && i < c0 + 64; ++i) {
+                glr_handle* h = hs[i];
+                CholMat& C = cg.mat[cg.nmat++];
+                C.part = h->gram; C.nparts = 1; C.ld = h->k; C.n = h->k; C.out = h->Linv; C.flag = h->dflags + 0;
+            }
+            PhaseScope ps(hs[c0], GLR_PH_REFRESH, s0);
+            GLR_LAUNCH(hs[c0], 1, chol_group(cg, s0));
         }
+        if ((rc = fp32_products(hs, s0, [](glr_handle* h, GemmMat& G) {      // Qn = Q L^{-T}
+                 G.M = h->mp; G.N = h->k; G.K = h->k;
+                 G.A = h->Q; G.sAi = h->k; G.sAp = 1; G.B = h->Linv; G.sBp = 1; G.sBj = h->k;
+                 G.C = h->Qn; G.sCi = h->k; G.sCj = 1;
+             })) != GLR_OK)
+            return rc;
+        for (glr_handle* h : hs) std::swap(h->Q, h->Qn);
+    }
+    for (glr_handle* h : hs) {
+        PhaseScope ps(h, GLR_PH_REFRESH, s0);
+        GLR_LAUNCH(h, 1, tc::transpose_round(h->QTt, h->mp, h->Q, h->mp, h->k, h->k, s0));
     }
     // Rayleigh-Ritz: Z = Mbar^T Q, H = Z^T Z (Gram partials), the eigenproblems
     rc = refresh_op(hs, tc::launch_powt, s0, [&](glr_handle* h, tc::TcMat& M) {
@@ -474,15 +501,71 @@ int refresh_tcl_grouped(std::vector<glr_handle*>& hs) {
         PhaseScope ps(hs[c0], GLR_PH_REFRESH, s0);
         GLR_LAUNCH(hs[c0], 1, eig_tmem_group(g, s0));
     }
-    GLR_CK(h0, cudaEventRecord(h0->rpow, s0));
-    for (glr_handle* h : hs) {
-        if (h != h0) GLR_CK(h, cudaStreamWaitEvent(h->rstream, h0->rpow, 0));
-        PhaseScope ps(h, GLR_PH_REFRESH, h->rstream);
-        g_ws = h->gemm_ws;
-        rc = refresh_finish(h, h->rstream);
-        g_ws = nullptr;
-        if (rc != GLR_OK) return rc;
+    // the finish, grouped: sorted Ritz pairs, Q <- Q W, column signs, the Householder WY form,
+    // Yt = Y T^T, then Y^T for the W = Y^T Mbar products
+    for (size_t c0 = 0; c0 < hs.size(); c0 += 64) {
+        FinishGroup fg{};
+        for (size_t i = c0; i < hs.size() && i < c0 + 64; ++i) {
+            glr_handle* h = hs[i];
+            FinishMat& F = fg.mat[fg.nmat++];
+            F.mp = h->mp; F.k = h->k; F.evals = h->evals; F.V = h->Vk; F.W = h->gram; F.evals_sorted = h->evals_sorted;
+            F.Wtop = h->scratch; F.Y = h->Y; F.T = h->T; F.s = h->dsign;
+        }
+        PhaseScope ps(hs[c0], GLR_PH_REFRESH, s0);
+        GLR_LAUNCH(hs[c0], 1, finish_group(fg, 0, s0));
     }
+    if ((rc = fp32_products(hs, s0, [](glr_handle* h, GemmMat& G) {          // Qn = Q W
+             G.M = h->mp; G.N = h->k; G.K = h->k;
+             G.A = h->Q; G.sAi = h->k; G.sAp = 1; G.B = h->gram; G.sBp = h->k; G.sBj = 1;
+             G.C = h->Qn; G.sCi = h->k; G.sCj = 1;
+         })) != GLR_OK)
+        return rc;
+    for (glr_handle* h : hs) std::swap(h->Q, h->Qn);
+    for (int stage = 1; stage <= 2; ++stage) {
+        for (size_t c0 = 0; c0 < hs.size(); c0 += 64) {
+            FinishGroup fg{};
+            for (size_t i = c0; i < hs.size() && i < c0 + 64; ++i) {
+                glr_handle* h = hs[i];
+                FinishMat& F = fg.mat[fg.nmat++];
+                F.mp = h->mp; F.k = h->k; F.Q = h->Q; F.Wtop = h->scratch; F.Y = h->Y; F.T = h->T; F.s = h->dsign;
+            }
+            PhaseScope ps(hs[c0], GLR_PH_REFRESH, s0);
+            GLR_LAUNCH(hs[c0], 1, finish_group(fg, stage, s0));
+        }
+    }
+    // rows a >= k of Y: Y[a, :] Utilde = -Q[a, :] with Utilde the upper triangle the top-block
+    // LU left in scratch: Utilde^{-1} (as the inverse of its transpose), then one product
+    for (size_t c0 = 0; c0 < hs.size(); c0 += 64) {
+        CholGroup cg{};
+        for (size_t i = c0; i < hs.size() && i < c0 + 64; ++i) {
+            glr_handle* h = hs[i];
+            CholMat& C = cg.mat[cg.nmat++];
+            C.part = h->scratch; C.nparts = 1; C.ld = h->k; C.n = h->k; C.out = h->Linv; C.tri_only = 1;
+        }
+        PhaseScope ps(hs[c0], GLR_PH_REFRESH, s0);
+        GLR_LAUNCH(hs[c0], 1, chol_group(cg, s0));
+    }
+    if ((rc = fp32_products(hs, s0, [](glr_handle* h, GemmMat& G) {          // Y[k:] = -Q[k:] Utilde^{-1}
+             G.M = h->mp - h->k; G.N = h->k; G.K = h->k; G.alpha = -1.f;
+             G.A = h->Q + (size_t)h->k * h->k; G.sAi = h->k; G.sAp = 1;
+             G.B = h->Linv; G.sBp = 1; G.sBj = h->k;
+             G.C = h->Y + (size_t)h->k * h->k; G.sCi = h->k; G.sCj = 1;
+         })) != GLR_OK)
+        return rc;
+    if ((rc = fp32_products(hs, s0, [](glr_handle* h, GemmMat& G) {          // Yt = Y T^T
+             G.M = h->mp; G.N = h->k; G.K = h->k;
+             G.A = h->Y; G.sAi = h->k; G.sAp = 1; G.B = h->T; G.sBp = 1; G.sBj = h->k;
+             G.C = h->Yt; G.sCi = h->k; G.sCj = 1;
+         })) != GLR_OK)
+        return rc;
+    for (glr_handle* h : hs) {
+        PhaseScope ps(h, GLR_PH_REFRESH, s0);
+        GLR_LAUNCH(h, 1, tc::transpose_round(h->YTk, h->mp, h->Y, h->mp, h->k, h->k, s0));
+    }
+    // every handle's side stream continues after the group's work
+    GLR_CK(h0, cudaEventRecord(h0->rpow, s0));
+    for (glr_handle* h : hs)
+        if (h != h0) GLR_CK(h, cudaStreamWaitEvent(h->rstream, h0->rpow, 0));
     return GLR_OK;
 }
 

@@ -26,14 +26,6 @@ constexpr int kEigMaxN = 256;
 
 __device__ __forceinline__ int circle(int x, int nm1) { return 1 + ((x % nm1) + nm1) % nm1; }
 
-__device__ __forceinline__ void tm_ld2(uint32_t ta, uint32_t tb, float& a, float& b) {
-    uint32_t u, v;
-    asm volatile("tcgen05.ld.sync.aligned.32x32b.x1.b32 {%0}, [%1];" : "=r"(u) : "r"(ta));
-    asm volatile("tcgen05.ld.sync.aligned.32x32b.x1.b32 {%0}, [%1];" : "=r"(v) : "r"(tb));
-    asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
-    a = __uint_as_float(u);
-    b = __uint_as_float(v);
-}
 __device__ __forceinline__ void tm_st1(uint32_t ta, float a) {
     asm volatile("tcgen05.st.sync.aligned.32x32b.x1.b32 [%0], {%1};" ::"r"(ta), "r"(__float_as_uint(a)) : "memory");
 }
@@ -163,18 +155,33 @@ __global__ void __launch_bounds__(ET, 1) eig_tmem_kernel(const __grid_constant__
                 if (vqi) Hs[i10] = cj * a10 - sj * a11;
                 if (vqi && vqj) Hs[i11] = sj * a10 + cj * a11;
             }
-            // W <- W J: the warps of each lane quadrant share the (pair, half) items
-            for (int it = w8; it < half * halves; it += 8) {
-                const int j = it % half, h = it / half;
-                const float sj = ssn[j];
-                if (sj == 0.f) continue;                  // warp-uniform
-                const float cj = scs[j];
-                const uint32_t ap = tmem + lanes + (uint32_t)(h * n + spp[j]);
-                const uint32_t aq = tmem + lanes + (uint32_t)(h * n + sqq[j]);
-                float vp, vq;
-                tm_ld2(ap, aq, vp, vq);
-                tm_st1(ap, cj * vp - sj * vq);
-                tm_st1(aq, sj * vp + cj * vq);
+            // W <- W J: the warps of each lane quadrant share the (pair, half) items, eight at a
+            // time with all sixteen column loads in flight before one wait
+            for (int it0 = w8; it0 < half * halves; it0 += 64) {
+                uint32_t ap[8], aq[8], up[8], uq[8];
+                bool act[8];
+#pragma unroll
+                for (int b = 0; b < 8; ++b) {
+                    const int it = it0 + 8 * b;
+                    const int j = it % half, h = it / half;
+                    act[b] = it < half * halves && ssn[j] != 0.f;   // warp-uniform
+                    ap[b] = tmem + lanes + (uint32_t)(h * n + spp[j]);
+                    aq[b] = tmem + lanes + (uint32_t)(h * n + sqq[j]);
+                    if (act[b]) {
+                        asm volatile("tcgen05.ld.sync.aligned.32x32b.x1.b32 {%0}, [%1];" : "=r"(up[b]) : "r"(ap[b]));
+                        asm volatile("tcgen05.ld.sync.aligned.32x32b.x1.b32 {%0}, [%1];" : "=r"(uq[b]) : "r"(aq[b]));
+                    }
+                }
+                asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+#pragma unroll
+                for (int b = 0; b < 8; ++b) {
+                    if (!act[b]) continue;
+                    const int j = (it0 + 8 * b) % half;
+                    const float cj = scs[j], sj = ssn[j];
+                    const float vp = __uint_as_float(up[b]), vq = __uint_as_float(uq[b]);
+                    tm_st1(ap[b], cj * vp - sj * vq);
+                    tm_st1(aq[b], sj * vp + cj * vq);
+                }
             }
             tm_wait_st();
             tm_fence_before();

@@ -140,8 +140,8 @@ __device__ float warp_column_sign(const float* A, int rows, int ld, int col) {
     return (bidx < rows && A[(size_t)bidx * ld + col] < 0.f) ? -1.f : 1.f;
 }
 
-__global__ void __launch_bounds__(1024) sort_fix_kernel(const float* evals, const float* V, int n, int ncols,
-                                                        float* Out, int ldo, float* evals_sorted, int npow2) {
+__device__ __forceinline__ void sort_fix_body(const float* evals, const float* V, int n, int ncols, float* Out,
+                                              int ldo, float* evals_sorted, int npow2) {
     extern __shared__ unsigned long long keys[];
     const int tid = threadIdx.x;
     for (int i = tid; i < npow2; i += blockDim.x)
@@ -174,7 +174,23 @@ __global__ void __launch_bounds__(1024) sort_fix_kernel(const float* evals, cons
         if (lane == 0 && evals_sorted) evals_sorted[c] = evals[src];
     }
 }
+__global__ void __launch_bounds__(1024) sort_fix_kernel(const float* evals, const float* V, int n, int ncols,
+                                                        float* Out, int ldo, float* evals_sorted, int npow2) {
+    sort_fix_body(evals, V, n, ncols, Out, ldo, evals_sorted, npow2);
+}
+__global__ void __launch_bounds__(1024) sort_fix_group_kernel(const __grid_constant__ FinishGroup g, int npow2) {
+    const FinishMat& M = g.mat[blockIdx.x];
+    sort_fix_body(M.evals, M.V, M.k, M.k, M.W, M.k, M.evals_sorted, npow2);
+}
 
+__global__ void fix_signs_group_kernel(const __grid_constant__ FinishGroup g) {
+    const FinishMat& M = g.mat[blockIdx.y];
+    const int col = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
+    if (col >= M.k) return;
+    const float sg = warp_column_sign(M.Q, M.mp, M.k, col);
+    if (sg < 0.f)
+        for (int a = threadIdx.x & 31; a < M.mp; a += 32) M.Q[(size_t)a * M.k + col] = -M.Q[(size_t)a * M.k + col];
+}
 __global__ void fix_signs_kernel(float* A, int rows, int cols) {
     const int col = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
     if (col >= cols) return;
@@ -265,8 +281,7 @@ __global__ void random_block_kernel(float* Q, int rows, int cols, uint64_t seed,
 // Householder reconstruction, top block: modified LU of S - Q[:k, :k] with s_j = -sign of the
 // current Schur-complement entry of Q (so every pivot has magnitude >= 1); then
 // T Y1^T = Utilde S by forward substitution.  W (k x k scratch) ends holding L1\Utilde.
-__global__ void __launch_bounds__(1024) hh_top_kernel(const float* Q, int k, float* W, float* Y, float* T,
-                                                      float* s) {
+__device__ __forceinline__ void hh_top_body(const float* Q, int k, float* W, float* Y, float* T, float* s) {
     const int tid = threadIdx.x, nth = blockDim.x;
     for (int e = tid; e < k * k; e += nth) W[e] = -Q[e];   // rows 0..k-1 of Q (ld = k)
     __syncthreads();
@@ -302,9 +317,17 @@ __global__ void __launch_bounds__(1024) hh_top_kernel(const float* Q, int k, flo
     }
 }
 
+__global__ void __launch_bounds__(1024) hh_top_kernel(const float* Q, int k, float* W, float* Y, float* T,
+                                                      float* s) {
+    hh_top_body(Q, k, W, Y, T, s);
+}
+__global__ void __launch_bounds__(1024) hh_top_group_kernel(const __grid_constant__ FinishGroup g) {
+    const FinishMat& M = g.mat[blockIdx.x];
+    hh_top_body(M.Q, M.k, M.Wtop, M.Y, M.T, M.s);
+}
+
 // Rows a >= k: Y[a, :] Utilde = -Q[a, :], one warp per row (forward substitution).
-__global__ void hh_rows_kernel(const float* Q, int mp, int k, const float* W, float* Y) {
-    const int warp = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
+__device__ __forceinline__ void hh_rows_body(const float* Q, int mp, int k, const float* W, float* Y, int warp) {
     const int lane = threadIdx.x & 31;
     const int a = k + warp;
     if (a >= mp) return;
@@ -319,6 +342,13 @@ __global__ void hh_rows_kernel(const float* Q, int mp, int k, const float* W, fl
         if (lane == 0) y[l] = val;
         __syncwarp();
     }
+}
+__global__ void hh_rows_kernel(const float* Q, int mp, int k, const float* W, float* Y) {
+    hh_rows_body(Q, mp, k, W, Y, blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5));
+}
+__global__ void hh_rows_group_kernel(const __grid_constant__ FinishGroup g) {
+    const FinishMat& M = g.mat[blockIdx.y];
+    hh_rows_body(M.Q, M.mp, M.k, M.Wtop, M.Y, blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5));
 }
 
 __global__ void wy_basis_kernel(int mp, int k, const float* Y, const float* Yt, const float* dsign, float* U) {
@@ -362,6 +392,28 @@ cudaError_t sort_fix_basis(const float* evals, const float* V, int n, int ncols,
 
 cudaError_t fix_column_signs(float* A, int rows, int cols, cudaStream_t st) {
     fix_signs_kernel<<<(cols + 7) / 8, 256, 0, st>>>(A, rows, cols);
+    return cudaGetLastError();
+}
+
+cudaError_t finish_group(const FinishGroup& g, int stage, cudaStream_t st) {
+    if (g.nmat <= 0) return cudaSuccess;
+    int kmax = 0, rows_max = 0;
+    for (int i = 0; i < g.nmat; ++i) {
+        kmax = g.mat[i].k > kmax ? g.mat[i].k : kmax;
+        rows_max = g.mat[i].mp - g.mat[i].k > rows_max ? g.mat[i].mp - g.mat[i].k : rows_max;
+    }
+    if (stage == 0) {                                   // sort the eigenpairs, normalise, fix signs
+        int npow2 = 1;
+        while (npow2 < kmax) npow2 <<= 1;
+        sort_fix_group_kernel<<<g.nmat, 1024, sizeof(unsigned long long) * npow2, st>>>(g, npow2);
+    } else if (stage == 1) {                            // column signs of Q
+        fix_signs_group_kernel<<<dim3((kmax + 7) / 8, g.nmat), 256, 0, st>>>(g);
+    } else if (stage == 2) {                            // Householder top block
+        hh_top_group_kernel<<<g.nmat, 1024, 0, st>>>(g);
+    } else {                                            // Householder rows below
+        if (rows_max <= 0) return cudaSuccess;
+        hh_rows_group_kernel<<<dim3((rows_max + 7) / 8, g.nmat), 256, 0, st>>>(g);
+    }
     return cudaGetLastError();
 }
 
@@ -473,9 +525,42 @@ __device__ __forceinline__ void chol_inverse_body(const float* G, int nparts, in
 __global__ void __launch_bounds__(1024) chol_inverse_kernel(const float* G, int n, float* S, int* flag) {
     chol_inverse_body(G, 1, n, n, S, 0, flag);
 }
+// L^{-1} of the lower-triangular L = U^T, U the upper triangle of the n x n matrix at A (leading
+// dimension lda): the inverse stage of chol_inverse_body alone.  Output row-major ld x ld.
+__device__ __forceinline__ void tri_inverse_body(const float* A, int lda, int n, float* out, int ld) {
+    extern __shared__ float L[];
+    float* col = L + n * (n + 1) / 2;
+    float* tmp = col + n;
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5, nw = blockDim.x >> 5;
+    for (int i = warp; i < n; i += nw)
+        for (int l = lane; l <= i; l += 32) L[tri(i, l)] = A[(size_t)l * lda + i];
+    __syncthreads();
+    for (int j = n - 1; j >= 0; --j) {
+        for (int l = j + 1 + tid; l < n; l += blockDim.x) col[l] = L[tri(l, j)];
+        __syncthreads();
+        for (int i = j + 1 + warp; i < n; i += nw) {
+            float t = 0.f;
+            for (int l = j + 1 + lane; l <= i; l += 32) t += L[tri(i, l)] * col[l];
+#pragma unroll
+            for (int o = 16; o > 0; o >>= 1) t += __shfl_xor_sync(0xffffffffu, t, o);
+            if (lane == 0) tmp[i] = t;
+        }
+        __syncthreads();
+        const float ajj = 1.0f / L[tri(j, j)];
+        for (int i = j + 1 + tid; i < n; i += blockDim.x) L[tri(i, j)] = -tmp[i] * ajj;
+        if (tid == 0) L[tri(j, j)] = ajj;
+        __syncthreads();
+    }
+    for (int e = tid; e < ld * ld; e += blockDim.x) {
+        const int r = e / ld, c = e % ld;
+        out[e] = (c <= r && r < n) ? L[tri(r, c)] : 0.f;
+    }
+}
+
 __global__ void __launch_bounds__(1024) chol_group_kernel(const __grid_constant__ CholGroup g) {
     const CholMat& M = g.mat[blockIdx.x];
-    chol_inverse_body(M.part, M.nparts, M.ld, M.n, M.out, 1, M.flag);
+    if (M.tri_only) tri_inverse_body(M.part, M.n, M.n, M.out, M.ld);
+    else chol_inverse_body(M.part, M.nparts, M.ld, M.n, M.out, 1, M.flag);
 }
 }  // namespace
 

@@ -295,3 +295,74 @@ cudaError_t materialize_error(int mp, int np, int r, int e_zero, const float* B,
 }
 
 }  // namespace glr
+
+// ------------------------------------------------------------------------------------------
+// Grouped fp32 products (the refresh's k-wide fp32 steps: Gram matrices, CholeskyQR's X L^{-T},
+// the Rayleigh-Ritz rotation Q W, Yt = Y T^T): a 64 x 64 output tile per CTA of 256 threads, each
+// thread a 4 x 4 block, K staged through shared memory 16 at a time; sums in a fixed order.
+// ------------------------------------------------------------------------------------------
+namespace glr {
+namespace {
+
+__global__ void __launch_bounds__(256) gemm_group_kernel(const __grid_constant__ GemmGroup g) {
+    __shared__ float As[16][68], Bs[16][68];
+    const int tile = blockIdx.x;
+    int lo = 0, hi = g.nmat - 1;
+    while (lo < hi) {
+        const int mid = (lo + hi + 1) >> 1;
+        if (g.mat[mid].tile0 <= tile) lo = mid; else hi = mid - 1;
+    }
+    const GemmMat& M = g.mat[lo];
+    const int lt = tile - M.tile0, tn = (M.N + 63) / 64;
+    const int i0 = (lt / tn) * 64, j0 = (lt % tn) * 64;
+    const int tx = threadIdx.x & 15, ty = threadIdx.x >> 4;
+    float acc[4][4] = {};
+    for (int p0 = 0; p0 < M.K; p0 += 16) {
+        for (int e = threadIdx.x; e < 16 * 64; e += 256) {
+            // consecutive threads along the operand's contiguous index
+            const bool pa = M.sAp == 1;
+            const int pp = pa ? (e & 15) : (e >> 6), ii = pa ? (e >> 4) : (e & 63);
+            const int i = i0 + ii, p = p0 + pp;
+            As[pp][ii] = (i < M.M && p < M.K) ? M.A[(int64_t)i * M.sAi + (int64_t)p * M.sAp] : 0.f;
+            const bool jb = M.sBj == 1;
+            const int jj = jb ? (e & 63) : (e >> 4), pq = jb ? (e >> 6) : (e & 15);
+            const int j = j0 + jj, q = p0 + pq;
+            Bs[pq][jj] = (j < M.N && q < M.K) ? M.B[(int64_t)q * M.sBp + (int64_t)j * M.sBj] : 0.f;
+        }
+        __syncthreads();
+#pragma unroll
+        for (int pp = 0; pp < 16; ++pp) {
+            float a[4], b[4];
+#pragma unroll
+            for (int u = 0; u < 4; ++u) { a[u] = As[pp][ty * 4 + u]; b[u] = Bs[pp][tx * 4 + u]; }
+#pragma unroll
+            for (int u = 0; u < 4; ++u)
+#pragma unroll
+                for (int v = 0; v < 4; ++v) acc[u][v] = fmaf(a[u], b[v], acc[u][v]);
+        }
+        __syncthreads();
+    }
+#pragma unroll
+    for (int u = 0; u < 4; ++u)
+#pragma unroll
+        for (int v = 0; v < 4; ++v) {
+            const int i = i0 + ty * 4 + u, j = j0 + tx * 4 + v;
+            if (i < M.M && j < M.N) M.C[(int64_t)i * M.sCi + (int64_t)j * M.sCj] = (M.alpha != 0.f ? M.alpha : 1.f) * acc[u][v];
+        }
+}
+
+}  // namespace
+
+cudaError_t gemm_group_f32(GemmGroup& g, cudaStream_t st) {
+    g.total_tiles = 0;
+    for (int i = 0; i < g.nmat; ++i) {
+        GemmMat& M = g.mat[i];
+        M.tile0 = g.total_tiles;
+        g.total_tiles += ((M.M + 63) / 64) * ((M.N + 63) / 64);
+    }
+    if (g.total_tiles <= 0) return cudaSuccess;
+    gemm_group_kernel<<<g.total_tiles, 256, 0, st>>>(g);
+    return cudaGetLastError();
+}
+
+}  // namespace glr
