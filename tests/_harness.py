@@ -43,7 +43,7 @@ def same_selection(J_dev, J_orc, lam_orc, tie_rel):
 
 
 def lockstep(m, n, r, N, steps, grads: Callable[[int], np.ndarray], *, dtype="f32", inject_basis=True,
-             tie_rel=1e-4, check_errors=True, **schedule) -> List[StepReport]:
+             tie_rel=1e-5, check_errors=True, **schedule) -> List[StepReport]:
     import torch
     import paper_2507_08784_gb300 as glr
 

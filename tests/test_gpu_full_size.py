@@ -21,8 +21,8 @@ compresses with the basis it has just computed, so it is checked by properties t
 any basis: P^T P = I, Rbar = P^T Mbar, the per-step error-feedback balance
 E_i(t) + P R_i(t) = G_i(t) + E_i(t - 1) (Eq. ef1, ef2), and the optimizer applied to Ghat = P Rbar.
 
-Tolerances: 1e-5 relative Frobenius for fp32 arithmetic on bf16-exact inputs, 1e-4 for
-lambda-bar (sums of n' products) and for X under Adam (the update divides by sqrt(V) + eps).
+Tolerances: 1e-5 relative Frobenius for fp32 arithmetic on bf16-exact inputs (X under MSGD and
+Adam, E_i, P, Rbar, lambda-bar; near-ties of the selection within 1e-5 of the largest score).
 Handles on the tcgen05 path (glr_stats.path == GLR_PATH_TCGEN05: these bf16 workloads) form
 their products as TF32 tensor-core MMAs and are held to the bf16 bound instead: 2e-2 relative
 Frobenius, near-ties of the selection within 1e-2 of the largest score.
@@ -94,8 +94,8 @@ def test_full_size_algorithm3_steps(name, li):
     dev = _handle(glr, cfg, li, seed, cfg.tau, "alg3")
     tc = dev.stats()["path"] == 2
     tol = 2e-2 if tc else 1e-5
-    lam_tol, tie = (2e-2, 1e-2) if tc else (1e-4, 1e-4)
-    x_tol = tol if tc else 1e-4 if cfg.optimizer == "adam" else 1e-5
+    lam_tol, tie = (2e-2, 1e-2) if tc else (1e-5, 1e-5)
+    x_tol = tol if tc else 1e-5
     X = torch.zeros(m, n, device="cuda")
     Xo, Mo, Vo = np.zeros((m, n)), np.zeros((m, n)), np.zeros((m, n))
     E = np.zeros((N, mp, npr))
@@ -189,3 +189,39 @@ def test_full_size_refresh_every_step_algorithm4():
             assert rel(X.cpu().numpy(), Xo) <= tol, f"step {t}: X"
     finally:
         dev.close()
+
+
+def test_full_size_refresh_principal_angles_gapped():
+    """The tcgen05 path's refresh at the refresh-stress shape (4096 x 11008, k = 128, bf16 node
+    gradients) on a spectrum with a gap at k (sigma_k / sigma_{k+1} = 10): the largest principal
+    angle between the device's top-k basis and the exact top-k left singular subspace of the same
+    node mean (fp64 eigenvectors of Mbar Mbar^T) is at most 1e-4 rad, and the basis is orthogonal."""
+    import math
+    import torch
+    import paper_2507_08784_gb300 as glr
+
+    m, n, N, k, r, rho = 4096, 11008, 2, 128, 32, 192
+    rng = np.random.default_rng(4242)
+    Ub = np.linalg.qr(rng.standard_normal((m, rho)))[0]
+    Vb = np.linalg.qr(rng.standard_normal((n, rho)))[0]
+    s = np.where(np.arange(rho) < k, 1.0 - 0.002 * np.arange(rho), 0.1 * 0.99 ** np.arange(rho))
+    S = (Ub * s) @ Vb.T
+    G = [S + 1e-3 * rng.standard_normal((m, n)) / np.sqrt(n) for _ in range(N)]
+    Gd = [torch.from_numpy(g.astype(np.float32)).to(torch.bfloat16).cuda().contiguous() for g in G]
+    Mbar = np.mean([g.float().cpu().numpy().astype(np.float64) for g in Gd], axis=0)   # the bf16 values
+    dev = glr.GreedyLore(m, n, r, N, tau=100, optimizer="msgd", lr=0.0, beta1=0.9, seed=7, basis_rank=k,
+                         power_iters=4, grad_dtype="bf16")
+    assert dev.stats()["path"] == 2, "expected the tcgen05 path"
+    X = torch.zeros(m, n, device="cuda")
+    try:
+        dev.step(Gd, X)                                  # step 0 refreshes
+        torch.cuda.synchronize()
+        U = dev.basis().double().cpu().numpy()
+    finally:
+        dev.close()
+    w, V = np.linalg.eigh(Mbar @ Mbar.T)
+    Uo = V[:, np.argsort(w)[::-1][:k]]
+    assert np.abs(U[:, :k].T @ U[:, :k] - np.eye(k)).max() < 1e-4
+    resid = U[:, :k] - Uo @ (Uo.T @ U[:, :k])
+    angle = math.asin(min(1.0, np.linalg.norm(resid, 2)))
+    assert angle <= 1e-4, f"largest principal angle {angle:.3e} rad"

@@ -1,9 +1,10 @@
 """GPU-vs-oracle parity through the C ABI (marked gpu).
 
 Tolerances: relative Frobenius error <= 1e-5 for fp32 arithmetic on fp32 or bf16-exact
-inputs (the oracle works in fp64 on the same values), <= 1e-4 for Adam (its normalised
-update divides by sqrt(V) + eps), selections compared as sets (a difference is accepted
-only between near-tied lambda-bar^2, after which the runs are not compared further).
+inputs (the oracle works in fp64 on the same values) — X under every optimizer, E_i, Mbar,
+P, Rbar and lambda-bar alike; selections compared as sets (a difference is accepted only
+between lambda-bar^2 scores within 1e-5 of the largest, after which the runs are not compared
+further).
 """
 import math
 
@@ -34,7 +35,7 @@ def _synthetic(m, n, N, rho, spectrum, noise, seed, dtype="f32"):
     return lambda t: W.gradients_numpy(prob, 0, t)
 
 
-def _assert_reports(reps, tol=1e-5, lam_tol=1e-4):
+def _assert_reports(reps, tol=1e-5, lam_tol=1e-5):
     assert reps, "no steps compared"
     for rep in reps:
         for key, val in rep.errs.items():
@@ -65,7 +66,7 @@ def test_transposed_adam_bf16_lockstep():
     g = _synthetic(333, 150, 2, 30, lambda k: k ** -1.0, 0.02, 12, dtype="bf16")
     reps = lockstep(333, 150, 6, 2, 8, g, dtype="bf16", tau=3, optimizer="adam", lr=1e-3, beta1=0.9,
                     beta2=0.999, eps=1e-8, seed=9, basis_rank=0)
-    _assert_reports(reps, tol=1e-4)
+    _assert_reports(reps, tol=1e-5)
 
 
 def test_transposed_truncated_lockstep():
@@ -80,7 +81,7 @@ def test_alg4_refresh_compressed_lockstep():
     g = _synthetic(64, 100, 2, 8, lambda k: 2.0 ** (-k), 0.0, 14)
     reps = lockstep(64, 100, 3, 2, 7, g, tau=4, refresh_mode="alg4", optimizer="msgd", lr=0.1, beta1=0.5,
                     seed=3, basis_rank=0)
-    _assert_reports(reps, tol=1e-4)
+    _assert_reports(reps, tol=1e-5)
 
 
 def test_compress_start_warmup_lockstep():
@@ -98,7 +99,7 @@ def test_amsgrad_lockstep(m, n, k):
     g = _synthetic(m, n, 3, 24, lambda j: 1.0 / j, 0.05, 90 + m + k)
     reps = lockstep(m, n, 5, 3, 6, g, tau=3, optimizer="amsgrad", lr=1e-3, beta1=0.9, beta2=0.999, eps=1e-8,
                     seed=12, basis_rank=k)
-    _assert_reports(reps, tol=1e-4)
+    _assert_reports(reps, tol=1e-5)
 
 
 @pytest.mark.parametrize("m,n,k", [(96, 400, 16), (300, 130, 0), (640, 1280, 16)])
@@ -108,7 +109,7 @@ def test_adamw_lockstep(m, n, k):
     g = _synthetic(m, n, 3, 24, lambda j: 1.0 / j, 0.05, 95 + m + k)
     reps = lockstep(m, n, 5, 3, 6, g, tau=3, optimizer="adamw", lr=1e-3, beta1=0.9, beta2=0.999, eps=1e-8,
                     weight_decay=0.01, seed=13, basis_rank=k)
-    _assert_reports(reps, tol=1e-4)
+    _assert_reports(reps, tol=1e-5)
 
 
 @pytest.mark.parametrize("m,n,k", [(64, 100, 0), (96, 400, 16), (300, 130, 24), (640, 1280, 16), (256, 2304, 16)])
@@ -120,7 +121,7 @@ def test_galore_adam_lockstep(m, n, k):
     g = _synthetic(m, n, 2, 8, lambda j: 2.0 ** (-j), 0.01, 100 + m + k)
     reps = lockstep(m, n, 3, 2, 7, g, tau=3, refresh_mode="alg4", optimizer="galore_adam", lr=1e-3, beta1=0.9,
                     beta2=0.999, eps=1e-8, seed=14, basis_rank=k, selection="fixed", error_feedback=False)
-    _assert_reports(reps, tol=1e-4)
+    _assert_reports(reps, tol=1e-5)
     assert [r.refresh for r in reps] == [True, False, False, True, False, False, True]
 
 
