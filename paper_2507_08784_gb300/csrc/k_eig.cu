@@ -36,8 +36,8 @@ __device__ __forceinline__ void tm_fence_after() { asm volatile("tcgen05.fence::
 __global__ void __launch_bounds__(ET, 1) eig_tmem_kernel(const __grid_constant__ EigGroup g) {
     extern __shared__ float Hs[];                      // packed upper triangle, n (n + 1) / 2
     __shared__ int off[kEigMaxN + 1];                  // Hs index of (r, c), r <= c: off[r] + c
-    __shared__ float scs[kEigMaxN / 2], ssn[kEigMaxN / 2];
-    __shared__ int spp[kEigMaxN / 2], sqq[kEigMaxN / 2];
+    __shared__ int4 spq[kEigMaxN / 2];                 // the round's pairs: p, q, off[p], off[q] (q = n: no partner)
+    __shared__ float2 scs[kEigMaxN / 2];               // and their rotations (c, s)
     __shared__ float red[2][ET / 32];
     __shared__ uint32_t tbase;
     __shared__ int s_stop;
@@ -73,6 +73,22 @@ __global__ void __launch_bounds__(ET, 1) eig_tmem_kernel(const __grid_constant__
     tm_wait_st();
     __syncthreads();
     const int items = half * (half + 1) / 2;
+    // this thread's 2 x 2 blocks (bi <= bj) of every round: block row i folded with block row
+    // half - 1 - i so that the enumeration has rows of half + 1 entries
+    constexpr int kItems = (kEigMaxN / 2) * (kEigMaxN / 2 + 1) / 2 / ET + 1;
+    int myblk[kItems];
+#pragma unroll
+    for (int u = 0; u < kItems; ++u) {
+        const int e = t + u * ET;
+        myblk[u] = -1;
+        if (e < items) {
+            const int fr = e / (half + 1), tt = e - fr * (half + 1);
+            int bi, bj;
+            if (tt < half - fr) { bi = fr; bj = fr + tt; }
+            else { bi = half - 1 - fr; bj = bi + (tt - (half - fr)); }
+            myblk[u] = bi | (bj << 16);
+        }
+    }
     int sweep = 0;
     for (;;) {
         // convergence check at the start of a sweep
@@ -115,21 +131,22 @@ __global__ void __launch_bounds__(ET, 1) eig_tmem_kernel(const __grid_constant__
                         s = tt * c;
                     }
                 }
-                scs[t] = c; ssn[t] = s; spp[t] = p; sqq[t] = q;
+                spq[t] = make_int4(p, q, off[p], q < n ? off[q] : 0);
+                scs[t] = make_float2(c, s);
             }
             __syncthreads();
-            for (int e = t; e < items; e += ET) {       // H <- J^T H J, 2 x 2 block by block (bi <= bj)
-                const int fr = e / (half + 1), tt = e - fr * (half + 1);
-                int bi, bj;
-                if (tt < half - fr) { bi = fr; bj = fr + tt; }
-                else { bi = half - 1 - fr; bj = bi + (tt - (half - fr)); }
-                const float si = ssn[bi], sj = ssn[bj];
+#pragma unroll
+            for (int u = 0; u < kItems; ++u) {          // H <- J^T H J, 2 x 2 block by block (bi <= bj)
+                if (myblk[u] < 0) continue;
+                const int bi = myblk[u] & 0xFFFF, bj = myblk[u] >> 16;
+                const float2 rci = scs[bi], rcj = scs[bj];
+                const float ci = rci.x, si = rci.y, cj = rcj.x, sj = rcj.y;
                 if (si == 0.f && sj == 0.f) continue;
-                const float ci = scs[bi], cj = scs[bj];
-                const int pi = spp[bi], qi = sqq[bi], pj = spp[bj], qj = sqq[bj];
+                const int4 pi4 = spq[bi], pj4 = spq[bj];
+                const int pi = pi4.x, qi = pi4.y, pj = pj4.x, qj = pj4.y;
                 const bool vqi = qi < n, vqj = qj < n;
                 if (bi == bj) {                          // diagonal block: the annihilated pair
-                    const int i00 = off[pi] + pi, i01 = off[pi] + qi, i11 = off[qi] + qi;
+                    const int i00 = pi4.z + pi, i01 = pi4.z + qi, i11 = pi4.w + qi;
                     const float h00 = Hs[i00], h01 = Hs[i01], h11 = Hs[i11];
                     const float a00 = ci * h00 - si * h01, a01 = ci * h01 - si * h11;
                     const float a10 = si * h00 + ci * h01, a11 = si * h01 + ci * h11;
@@ -138,12 +155,12 @@ __global__ void __launch_bounds__(ET, 1) eig_tmem_kernel(const __grid_constant__
                     Hs[i01] = 0.f;
                     continue;
                 }
-                // (x, y) of the symmetric matrix at the packed index of (min, max)
-                auto at = [&](int x, int y) { return x <= y ? off[x] + y : off[y] + x; };
-                const int i00 = at(pi, pj);
-                const int i01 = vqj ? at(pi, qj) : -1;
-                const int i10 = vqi ? at(qi, pj) : -1;
-                const int i11 = (vqi && vqj) ? at(qi, qj) : -1;
+                // (x, y) of the symmetric matrix at the packed index of (min, max): offx + y or offy + x
+                // (an index with no partner points at (pi, pj): it is neither read nor written)
+                const int i00 = pi <= pj ? pi4.z + pj : pj4.z + pi;
+                const int i01 = !vqj ? i00 : pi <= qj ? pi4.z + qj : pj4.w + pi;
+                const int i10 = !vqi ? i00 : qi <= pj ? pi4.w + pj : pj4.z + qi;
+                const int i11 = !(vqi && vqj) ? i00 : qi <= qj ? pi4.w + qj : pj4.w + qi;
                 const float h00 = Hs[i00];
                 const float h01 = vqj ? Hs[i01] : 0.f;
                 const float h10 = vqi ? Hs[i10] : 0.f;
@@ -157,30 +174,32 @@ __global__ void __launch_bounds__(ET, 1) eig_tmem_kernel(const __grid_constant__
             }
             // W <- W J: the warps of each lane quadrant share the (pair, half) items, eight at a
             // time with all sixteen column loads in flight before one wait
-            for (int it0 = w8; it0 < half * halves; it0 += 64) {
-                uint32_t ap[8], aq[8], up[8], uq[8];
-                bool act[8];
+            for (int h = 0; h < halves; ++h) {
+                const uint32_t hb = tmem + lanes + (uint32_t)(h * n);
+                for (int j0 = w8; j0 < half; j0 += 64) {
+                    uint32_t ap[8], aq[8], up[8], uq[8];
+                    bool act[8];
 #pragma unroll
-                for (int b = 0; b < 8; ++b) {
-                    const int it = it0 + 8 * b;
-                    const int j = it % half, h = it / half;
-                    act[b] = it < half * halves && ssn[j] != 0.f;   // warp-uniform
-                    ap[b] = tmem + lanes + (uint32_t)(h * n + spp[j]);
-                    aq[b] = tmem + lanes + (uint32_t)(h * n + sqq[j]);
-                    if (act[b]) {
-                        asm volatile("tcgen05.ld.sync.aligned.32x32b.x1.b32 {%0}, [%1];" : "=r"(up[b]) : "r"(ap[b]));
-                        asm volatile("tcgen05.ld.sync.aligned.32x32b.x1.b32 {%0}, [%1];" : "=r"(uq[b]) : "r"(aq[b]));
+                    for (int b = 0; b < 8; ++b) {
+                        const int j = j0 + 8 * b;
+                        act[b] = j < half && scs[j].y != 0.f;   // warp-uniform
+                        const int4 pq = spq[j < half ? j : 0];
+                        ap[b] = hb + (uint32_t)pq.x;
+                        aq[b] = hb + (uint32_t)pq.y;
+                        if (act[b]) {
+                            asm volatile("tcgen05.ld.sync.aligned.32x32b.x1.b32 {%0}, [%1];" : "=r"(up[b]) : "r"(ap[b]));
+                            asm volatile("tcgen05.ld.sync.aligned.32x32b.x1.b32 {%0}, [%1];" : "=r"(uq[b]) : "r"(aq[b]));
+                        }
                     }
-                }
-                asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+                    asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
 #pragma unroll
-                for (int b = 0; b < 8; ++b) {
-                    if (!act[b]) continue;
-                    const int j = (it0 + 8 * b) % half;
-                    const float cj = scs[j], sj = ssn[j];
-                    const float vp = __uint_as_float(up[b]), vq = __uint_as_float(uq[b]);
-                    tm_st1(ap[b], cj * vp - sj * vq);
-                    tm_st1(aq[b], sj * vp + cj * vq);
+                    for (int b = 0; b < 8; ++b) {
+                        if (!act[b]) continue;
+                        const float2 cs = scs[j0 + 8 * b];
+                        const float vp = __uint_as_float(up[b]), vq = __uint_as_float(uq[b]);
+                        tm_st1(ap[b], cs.x * vp - cs.y * vq);
+                        tm_st1(aq[b], cs.y * vp + cs.x * vq);
+                    }
                 }
             }
             tm_wait_st();
