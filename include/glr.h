@@ -219,6 +219,42 @@ int glr_step_host(glr_handle* h, const void* const* G_host, float* X, float* X_h
 int glr_step_group_host(glr_handle* const* handles, int32_t count, const void* const* const* G_host,
                         float* const* X, float* const* X_host_out, void* stream);
 
+/* Data-parallel steps across processes: Algorithm 3's All-Reduce lines (Sec. 4.3; the per-step
+ * traffic of Table 2) made explicit for nodes that live in different processes.  Each rank
+ * creates a handle for its own shard of the N nodes of the data-parallel group (the same shard
+ * size, m, n, r, schedule and seed on every rank) and runs every step in three calls; between them
+ * the caller averages each buffer a call exposes over the ranks (an all-reduce of the sum divided
+ * by the number of ranks, in place, in device memory, ordered after `stream`):
+ *
+ *   glr_dp_begin   M_i = G_i + E_i for the local nodes (Eq. ef1).  Exposes the shard's
+ *                  Approx-Top-r scores lambda-bar (m' floats; Algorithm 2, Eq. lambda-bar: linear
+ *                  in the node mean, so the average over shards is the group's), or on a refresh
+ *                  or warm-up step the shard's node mean Mbar (m' x n' floats).
+ *   glr_dp_select  With the averaged buffers: the refresh of the averaged Mbar (Eq. SVD-P1) or the
+ *                  arg-top-r of the averaged lambda-bar, P = U[:, J], and the shard's projected
+ *                  mean Rbar = P^T Mbar (exposed as Rbar^T, n' x rpad floats, rpad = r rounded up to
+ *                  32; Eq. 8zhb2we09).  Nothing is exposed when the step is uncompressed.
+ *   glr_dp_finish  With the averaged Rbar: Ghat = P Rbar (Mbar when uncompressed), the optimizer on
+ *                  X (Eq. msgd / adam), and the error feedback E_i = M_i - P R_i of the local nodes
+ *                  (deferred to the next step's compose pass, as in glr_step).
+ *
+ * The floats exchanged per step are Table 2's: m' + r n' on a compressed step (plus the padding
+ * columns of Rbar^T when r is not a multiple of 32), m' n' on an Algorithm 3 refresh;
+ * glr_stats.comm_floats_* count them.  G's pointers must stay valid until glr_dp_finish.  Only
+ * handles on the tcgen05 path (glr_stats.path == GLR_PATH_TCGEN05) take these calls; others,
+ * out-of-order calls (a begin before the last finish, a select without a begin, a finish without
+ * a select), null or misaligned pointers return GLR_EINVAL.  `out` receives device pointers into
+ * the handle's state (valid until the next call on the handle) and their sizes; count is 0..1. */
+typedef struct {
+    int32_t count;          /* buffers to average */
+    int32_t pad_;
+    float* ptr[2];          /* device pointers into the handle's state */
+    int64_t floats[2];      /* floats in each */
+} glr_dp_exchange;
+int glr_dp_begin(glr_handle* h, const void* const* G, void* stream, glr_dp_exchange* out);
+int glr_dp_select(glr_handle* h, void* stream, glr_dp_exchange* out);
+int glr_dp_finish(glr_handle* h, float* X, void* stream);
+
 /* Checkpoints.  glr_state_size gives the bytes of a checkpoint of h now; glr_save copies the
  * handle's whole state into host memory host_buf (at least that many bytes): the schedule
  * position (t, the refresh period, a pending forced selection), the basis, P, the error state

@@ -106,6 +106,29 @@ def glr_step(h, G: Sequence[torch.Tensor], X: torch.Tensor, stream=None) -> None
     _check(load().glr_step(h, _ptr_array(G), X.data_ptr(), _stream_ptr(stream)), h)
 
 
+def _exchange(ex) -> list:
+    return [(int(ex.ptr[i]), int(ex.floats[i])) for i in range(ex.count)]
+
+
+def glr_dp_begin(h, G: Sequence[torch.Tensor], stream=None) -> list:
+    """First phase of a data-parallel step (see glr.h): [(device pointer, floats)] to average."""
+    ex = _lib.GlrDpExchange()
+    _check(load().glr_dp_begin(h, _ptr_array(G), _stream_ptr(stream), ctypes.byref(ex)), h)
+    return _exchange(ex)
+
+
+def glr_dp_select(h, stream=None) -> list:
+    """Second phase: the selection (or refresh) on the averaged buffers; returns Rbar^T to average."""
+    ex = _lib.GlrDpExchange()
+    _check(load().glr_dp_select(h, _stream_ptr(stream), ctypes.byref(ex)), h)
+    return _exchange(ex)
+
+
+def glr_dp_finish(h, X: torch.Tensor, stream=None) -> None:
+    """Third phase: the update of X with the averaged Rbar and the local error feedback."""
+    _check(load().glr_dp_finish(h, X.data_ptr(), _stream_ptr(stream)), h)
+
+
 def glr_step_group(handles: Sequence, G: Sequence[Sequence[torch.Tensor]], X: Sequence[torch.Tensor],
                    stream=None) -> None:
     """One step of several handles with batched launches (see glr.h)."""

@@ -63,6 +63,16 @@ class GlrStats(ctypes.Structure):
     ]
 
 
+class GlrDpExchange(ctypes.Structure):
+    """glr_dp_exchange: the device buffers a data-parallel phase exposes for averaging."""
+    _fields_ = [
+        ("count", ctypes.c_int32),
+        ("pad_", ctypes.c_int32),
+        ("ptr", ctypes.c_void_p * 2),
+        ("floats", ctypes.c_int64 * 2),
+    ]
+
+
 GLR_PHASES = 7
 PHASE_NAMES = ["prev_project", "compose", "lambda", "select", "project", "update", "refresh"]
 
@@ -101,6 +111,9 @@ _SIGNATURES = {
     "glr_test_expire_wait": (ctypes.c_int, [ctypes.c_void_p, ctypes.c_int32, ctypes.c_void_p]),
     "glr_profile_enable": (ctypes.c_int, [ctypes.c_void_p, ctypes.c_int32]),
     "glr_profile_read": (ctypes.c_int, [ctypes.c_void_p, ctypes.POINTER(GlrProfile), ctypes.c_int32]),
+    "glr_dp_begin": (ctypes.c_int, [ctypes.c_void_p, _c_void_pp, ctypes.c_void_p, ctypes.POINTER(GlrDpExchange)]),
+    "glr_dp_select": (ctypes.c_int, [ctypes.c_void_p, ctypes.c_void_p, ctypes.POINTER(GlrDpExchange)]),
+    "glr_dp_finish": (ctypes.c_int, [ctypes.c_void_p, ctypes.c_void_p, ctypes.c_void_p]),
     "glr_select_noalloc": (ctypes.c_int, [ctypes.c_int32, ctypes.c_int32, ctypes.c_int32, ctypes.c_void_p,
                                           ctypes.c_void_p, ctypes.c_uint64, ctypes.c_int64, ctypes.c_void_p,
                                           ctypes.c_void_p, ctypes.c_void_p]),

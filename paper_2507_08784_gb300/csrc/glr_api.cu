@@ -786,7 +786,7 @@ int tcl_lambda(std::vector<StepPlan*>& plans, cudaStream_t st) {
 
 // After J: W for the matrices that did not select (a supplied J, or the refresh of Algorithm 4),
 // P = U[:, J] (and P^T), Rbar, then the update pass for every matrix.
-int tcl_project_update(std::vector<StepPlan*>& plans, cudaStream_t st) {
+int tcl_project(std::vector<StepPlan*>& plans, cudaStream_t st) {
     int rc = tc_run(plans, GLR_PH_PROJECT, tc::launch_wbar, st, tc_wbar_fill(false));
     if (rc != GLR_OK) return rc;
     // YtJ = Yt[J, :] was gathered by the selection launch
@@ -807,7 +807,11 @@ int tcl_project_update(std::vector<StepPlan*>& plans, cudaStream_t st) {
         M.J = h->J; M.dsign = h->dsign; M.Mbar = h->Mbar; M.Rbar = h->Rbar; M.RbarT = h->RbarT;
         return 1;
     });
-    if (rc != GLR_OK) return rc;
+    return rc;
+}
+
+// The update pass (K3) of every matrix.
+int tcl_update(std::vector<StepPlan*>& plans, cudaStream_t st) {
     return tc_run(plans, GLR_PH_UPDATE, tc::launch_update, st, [st](StepPlan& p, tc::TcMat& M, tc::TcGroup& g, bool first) {
         glr_handle* h = p.h;
         const glr_schedule& s = h->s;
@@ -827,6 +831,11 @@ int tcl_project_update(std::vector<StepPlan*>& plans, cudaStream_t st) {
         M.Mbar = h->Mbar; M.X = p.X; M.Mo = h->Mo; M.Vo = h->Vo;
         return 1;
     });
+}
+
+int tcl_project_update(std::vector<StepPlan*>& plans, cudaStream_t st) {
+    const int rc = tcl_project(plans, st);
+    return rc != GLR_OK ? rc : tcl_update(plans, st);
 }
 
 // Between K1 and K3: refresh, or Approx-Top-r selection and P.
@@ -877,13 +886,13 @@ int select_phase(StepPlan& p, cudaStream_t st) {
 }
 
 // arg-top-r (unless J was supplied) and P = U[:, J] for every compressed matrix, grouped.
-int select_P_grouped(std::vector<StepPlan>& plans, cudaStream_t st) {
+int select_P_grouped(std::vector<StepPlan>& plans, cudaStream_t st, int stages = 3) {
     SelectGroup g{};
     glr_handle* h0 = nullptr;
     auto flush = [&]() -> int {
         if (g.nmat == 0) return GLR_OK;
         PhaseScope ps(h0, GLR_PH_SELECT, st);
-        GLR_LAUNCH(h0, 3, select_group(g, st));
+        GLR_LAUNCH(h0, (stages & 1) + 2 * ((stages >> 1) & 1), select_group(g, st, stages));
         g = SelectGroup{};
         h0 = nullptr;
         return GLR_OK;
@@ -911,6 +920,7 @@ int select_P_grouped(std::vector<StepPlan>& plans, cudaStream_t st) {
     }
     int rc = flush();
     if (rc != GLR_OK) return rc;
+    if (!(stages & 2)) return GLR_OK;
     // P = U[:, J] of a truncated basis with large products: (E_J - Y Yt[J, :]^T) D_J
     for (StepPlan& p : plans) {
         glr_handle* h = p.h;
@@ -999,6 +1009,82 @@ int step_group(std::vector<StepPlan>& plans, cudaStream_t st) {
     return GLR_OK;
 }
 
+// ---- data-parallel steps across processes (glr_dp_*) ------------------------------------------
+enum : int { kDpWarm = 1, kDpRefresh = 2, kDpForced = 4, kDpFixed = 8, kDpCompressed = 16 };
+
+StepPlan dp_plan(glr_handle* h) {
+    StepPlan p;
+    p.h = h; p.G = h->dp_G; p.X = nullptr;
+    p.warm = h->dp_flags & kDpWarm; p.refresh = h->dp_flags & kDpRefresh; p.forced = h->dp_flags & kDpForced;
+    p.fixed = h->dp_flags & kDpFixed; p.compressed = h->dp_flags & kDpCompressed;
+    return p;
+}
+
+void dp_expose(glr_dp_exchange* ex, float* ptr, int64_t floats) {
+    ex->ptr[ex->count] = ptr;
+    ex->floats[ex->count] = floats;
+    ex->count++;
+}
+
+int dp_begin(glr_handle* h, const void* const* G, cudaStream_t st, glr_dp_exchange* ex) {
+    for (int i = 0; i < h->N; ++i) h->dp_G[i] = G[i];
+    std::vector<StepPlan> plans(1);
+    StepPlan& p = plans[0];
+    p.h = h; p.G = h->dp_G;
+    plan_step(p);
+    h->dp_flags = (p.warm ? kDpWarm : 0) | (p.refresh ? kDpRefresh : 0) | (p.forced ? kDpForced : 0) |
+                  (p.fixed ? kDpFixed : 0) | (p.compressed ? kDpCompressed : 0);
+    std::vector<StepPlan*> v{&p};
+    int rc = tcl_compose(v, st);
+    if (rc != GLR_OK) return rc;
+    if (p.warm || p.refresh) {                 // the node mean: the refresh's input, or Ghat
+        dp_expose(ex, h->Mbar, (int64_t)h->mp * h->np);
+        return GLR_OK;
+    }
+    if ((rc = select_phase(p, st)) != GLR_OK) return rc;     // J of a forced / fixed selection
+    if (tc_needs_lambda(p)) {                  // this shard's lambda-bar (linear in Mbar)
+        if ((rc = tcl_lambda(v, st)) != GLR_OK) return rc;
+        if ((rc = select_P_grouped(plans, st, 1)) != GLR_OK) return rc;
+        dp_expose(ex, h->lam, h->mp);
+    }
+    return GLR_OK;
+}
+
+int dp_select(glr_handle* h, cudaStream_t st, glr_dp_exchange* ex) {
+    std::vector<StepPlan> plans(1, dp_plan(h));
+    StepPlan& p = plans[0];
+    std::vector<StepPlan*> v{&p};
+    int rc;
+    if (p.refresh) {                           // the Semi-Lazy SVD of the averaged node mean
+        if (h->k <= 256)
+            GLR_LAUNCH(h, 1, transpose_pad(h->Mrow, h->np, h->Mbar, h->np, h->mp, st));   // its row-major copy
+        GLR_CK(h, cudaEventRecord(h->rfork, st));
+        GLR_CK(h, cudaStreamWaitEvent(h->rstream, h->rfork, 0));
+        std::vector<glr_handle*> hs{h};
+        rc = h->k <= 256 ? refresh_tcl_grouped(hs) : refresh_trunc_grouped(hs);
+        if (rc != GLR_OK) return rc;
+        GLR_CK(h, cudaEventRecord(h->rdone, h->rstream));
+        GLR_CK(h, cudaStreamWaitEvent(st, h->rdone, 0));
+        if ((rc = select_phase(p, st)) != GLR_OK) return rc;
+    }
+    if (!p.compressed) return GLR_OK;          // Ghat = Mbar: nothing more to average
+    if ((rc = select_P_grouped(plans, st, 2)) != GLR_OK) return rc;   // lambda-bar came from glr_dp_begin
+    if ((rc = tcl_project(v, st)) != GLR_OK) return rc;
+    dp_expose(ex, h->RbarT, (int64_t)h->np * h->rpad);       // this shard's Rbar (as Rbar^T)
+    return GLR_OK;
+}
+
+int dp_finish(glr_handle* h, float* X, cudaStream_t st) {
+    std::vector<StepPlan> plans(1, dp_plan(h));
+    StepPlan& p = plans[0];
+    p.X = X;
+    std::vector<StepPlan*> v{&p};
+    const int rc = tcl_update(v, st);
+    if (rc != GLR_OK) return rc;
+    finish_step(p);
+    return GLR_OK;
+}
+
 }  // namespace
 
 extern "C" {
@@ -1054,6 +1140,39 @@ int glr_step_host(glr_handle* h, const void* const* G_host, float* X, float* X_h
         GLR_CK(h, cudaStreamSynchronize(st));
     }
     return GLR_OK;
+}
+
+int glr_dp_begin(glr_handle* h, const void* const* G, void* stream, glr_dp_exchange* out) {
+    if (!h || !out) return fail(h, GLR_EINVAL, "null handle or exchange descriptor%s");
+    h->err.clear();
+    *out = glr_dp_exchange{};
+    if (!h->tcl) return fail(h, GLR_EINVAL, "data-parallel steps need the tcgen05 path (bf16 gradients, truncated basis)%s");
+    if (h->dp_stage != 0) return fail(h, GLR_EINVAL, "glr_dp_begin: the previous data-parallel step is not finished%s");
+    if (!G) return fail(h, GLR_EINVAL, "null gradient array%s");
+    for (int i = 0; i < h->N; ++i)
+        if (!G[i] || !aligned16(G[i]))
+            return fail(h, GLR_EINVAL, "gradient %s is null or not 16-byte aligned", std::to_string(i).c_str());
+    const int rc = dp_begin(h, G, static_cast<cudaStream_t>(stream), out);
+    if (rc == GLR_OK) h->dp_stage = 1;
+    return rc;
+}
+
+int glr_dp_select(glr_handle* h, void* stream, glr_dp_exchange* out) {
+    if (!h || !out) return fail(h, GLR_EINVAL, "null handle or exchange descriptor%s");
+    *out = glr_dp_exchange{};
+    if (h->dp_stage != 1) return fail(h, GLR_EINVAL, "glr_dp_select needs a step begun by glr_dp_begin%s");
+    const int rc = dp_select(h, static_cast<cudaStream_t>(stream), out);
+    if (rc == GLR_OK) h->dp_stage = 2;
+    return rc;
+}
+
+int glr_dp_finish(glr_handle* h, float* X, void* stream) {
+    if (!h) return GLR_EINVAL;
+    if (h->dp_stage != 2) return fail(h, GLR_EINVAL, "glr_dp_finish needs a step selected by glr_dp_select%s");
+    if (!X || !aligned16(X)) return fail(h, GLR_EINVAL, "X is null or not 16-byte aligned%s");
+    const int rc = dp_finish(h, X, static_cast<cudaStream_t>(stream));
+    h->dp_stage = 0;
+    return rc;
 }
 
 int glr_step_group_host(glr_handle* const* handles, int32_t count, const void* const* const* G_host,

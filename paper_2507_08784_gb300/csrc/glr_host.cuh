@@ -63,6 +63,10 @@ struct glr_handle {
     // TF32 transposes of Q and Z, Gram partials, L^{-1}
     float *Mrow = nullptr, *Mlo = nullptr, *QTt = nullptr, *ZTt = nullptr, *gpart = nullptr, *Linv = nullptr;
     float* Qbuf0 = nullptr;                       // Q's first allocation (Q and Qn trade places)
+    // a data-parallel step in progress (glr_dp_begin / glr_dp_select / glr_dp_finish): 0 idle,
+    // 1 begun, 2 selected; the step's plan and the caller's gradient pointers
+    int dp_stage = 0, dp_flags = 0;
+    const void* dp_G[GLR_MAX_NODES] = {};
     float* Pbuf0 = nullptr;                    // the first projector allocation (P and Pprev trade places)
     float *PT0 = nullptr, *PT1 = nullptr;      // P^T of Pbuf0 / of the other allocation (rpad x m')
     float *WT = nullptr, *YTk = nullptr, *RbarT = nullptr;   // W^T (n' x kpad), Y^T (kpad x m'), Rbar^T (n' x rpad)

@@ -178,7 +178,8 @@ struct SelectGroup {
     int64_t total_out;
     SelectMat mat[kGroupMax];
 };
-cudaError_t select_group(const SelectGroup& g, cudaStream_t st);
+// stages: 1 = lambda-bar from the partials, 2 = arg-top-r, P and Rbar (3: both)
+cudaError_t select_group(const SelectGroup& g, cudaStream_t st, int stages = 3);
 // P = U[:, J] of a truncated basis U = (I - Y Yt^T) D formed around a library product:
 // wy_columns_gather writes YtJ = Yt[J, :] (r x k); the caller forms P = -Y YtJ^T (m' x r);
 // wy_columns_fix adds the identity columns e_{J_q} and scales column q by d_{J_q} (J_q < k).

@@ -436,13 +436,16 @@ __global__ void __launch_bounds__(1024) lambda_reduce_kernel(const __grid_consta
     }
 }
 
-cudaError_t select_group(const SelectGroup& g, cudaStream_t st) {
+cudaError_t select_group(const SelectGroup& g, cudaStream_t st, int stages) {
     if (g.nmat <= 0) return cudaSuccess;
     int maxmp = 1;
     for (int i = 0; i < g.nmat; ++i) maxmp = g.mat[i].mp > maxmp ? g.mat[i].mp : maxmp;
-    lambda_reduce_kernel<<<dim3((maxmp + 31) / 32, g.nmat), 1024, 0, st>>>(g);
-    cudaError_t e = cudaGetLastError();
-    if (e != cudaSuccess) return e;
+    cudaError_t e = cudaSuccess;
+    if (stages & 1) {
+        lambda_reduce_kernel<<<dim3((maxmp + 31) / 32, g.nmat), 1024, 0, st>>>(g);
+        if ((e = cudaGetLastError()) != cudaSuccess) return e;
+    }
+    if (!(stages & 2)) return cudaSuccess;
     int npow2 = 1;
     while (npow2 < maxmp) npow2 <<= 1;
     {   // per device: set on every call (cheap next to the launch)

@@ -38,7 +38,7 @@ def test_struct_layouts(tmp_path):
     cc = shutil.which("gcc") or shutil.which("cc")
     if cc is None:
         pytest.skip("no C compiler")
-    fields = {"glr_schedule": _lib.GlrSchedule, "glr_stats": _lib.GlrStats}
+    fields = {"glr_schedule": _lib.GlrSchedule, "glr_stats": _lib.GlrStats, "glr_dp_exchange": _lib.GlrDpExchange}
     lines = ['#include <stdio.h>', '#include <stddef.h>', '#include "glr.h"', 'int main(void) {']
     for cname, cls in fields.items():
         lines.append(f'printf("{cname} %zu\\n", sizeof({cname}));')
