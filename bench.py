@@ -437,12 +437,26 @@ def summarize(cfg, run, K, world, hbm_peak):
     }
 
 
-def ncu_case(refresh=False):
+def ncu_case(refresh=False, stress=False):
     """One 4096 x 4096 matrix of the headline stack for 4 steps (about 1.1 GB of state): the
     compose launch of step 2 (index 2 among compose launches) is a full one; with refresh, a
-    fifth step forced to refresh."""
+    fifth step forced to refresh.  With stress: the refresh-stress matrix (4096 x 11008, N = 8,
+    k = 128, Algorithm 4) for 3 steps, each a refresh (about 4 GB of state)."""
     import torch
     import paper_2507_08784_gb300 as glr
+    if stress:
+        cfg = W.config("cfg4_refresh")
+        prob = W.make_problem(cfg)
+        gs = [W.gradients_torch(prob, 0, t) for t in range(2)]
+        hs = make_handles(glr, cfg, cfg.basis_rank)
+        X = [torch.zeros(*cfg.shapes[0], device="cuda")]
+        for t in range(3):
+            glr.glr_step_group(hs, [gs[t % 2]], X)
+        torch.cuda.synchronize()
+        print(json.dumps({"ncu_case": "cfg4_refresh", "shape": cfg.shapes[0], "N": cfg.N, "k": cfg.basis_rank,
+                          "path": hs[0].stats()["path"]}))
+        hs[0].close()
+        return 0
     cfg = W.config(WORKLOAD, shapes=W.config(WORKLOAD).shapes[:1])
     prob = W.make_problem(cfg)
     gs = [W.gradients_torch(prob, 0, t) for t in range(2)]
@@ -471,17 +485,18 @@ def main():
                     help="time the headline workload only (no extra workloads, no e2e, no CPU baseline)")
     ap.add_argument("--e2e-steps", type=int, default=5)
     ap.add_argument("--refresh-reps", type=int, default=3)
-    ap.add_argument("--ncu-case", nargs="?", const="steps", choices=["steps", "refresh"],
+    ap.add_argument("--ncu-case", nargs="?", const="steps", choices=["steps", "refresh", "stress"],
                     help="a small case for kernel captures: one 4096 x 4096 matrix of the headline stack "
                          "(N = 4, r = 128, k = 256, bf16, Adam), 4 steps: refresh, reset, then two full "
-                         "steps; 'refresh' adds a fifth step forced to refresh")
+                         "steps; 'refresh' adds a fifth step forced to refresh; 'stress' runs the refresh-stress "
+                         "matrix (4096 x 11008, N = 8, k = 128) for 3 refresh steps")
     args = ap.parse_args()
     if args.warmup < 3:
         ap.error("--warmup must be >= 3")
     if args.impl == "reference":
         return run_reference(args)
     if args.ncu_case:
-        return ncu_case(args.ncu_case == "refresh")
+        return ncu_case(args.ncu_case == "refresh", args.ncu_case == "stress")
 
     import torch
     import paper_2507_08784_gb300 as glr
