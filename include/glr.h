@@ -87,7 +87,11 @@ extern "C" {
  *   seed           64-bit key of the shared random vectors v_j (Eq. random-v): all nodes
  *                  of one matrix draw the same v_j; give every matrix its own seed
  *   basis_rank     k.  0 (or m') keeps the full m' x m' singular basis U of Eq. SVD-P1
- *                  (paper-exact; m' <= 1024).  r <= k < m', k <= 512, keeps the top-k
+ *                  (paper-exact): any m' <= 1024; above that m' a multiple of 128 up to 4096
+ *                  with n' a multiple of 8, bf16 gradients, MSGD or Adam, 16 <= r <= 128 (a
+ *                  multiple of 4) and N <= 8 (the tcgen05 path; its refresh is a blocked
+ *                  Jacobi eigen-solve of Mbar Mbar^T, GLR_ENUMERIC from glr_get_stats when it
+ *                  has not converged in 30 sweeps).  r <= k < m', k <= 512, keeps the top-k
  *                  singular vectors and completes them to an orthogonal U with Householder
  *                  reflectors; the refresh then uses power_iters block power iterations
  *   power_iters    q >= 1 (truncated basis only)

@@ -327,8 +327,11 @@ int glr_create(int64_t m, int64_t n, int32_t r, int32_t N, const glr_schedule* s
     const int k = (s->basis_rank == 0 || s->basis_rank == mp) ? static_cast<int>(mp) : s->basis_rank;
     const bool exact = k == mp;
     if (!exact && (k < r || k > mp)) return fail(nullptr, GLR_EINVAL, "need r <= basis_rank <= min(m, n)%s");
-    if (exact && mp > kMaxFullBasis)
-        return fail(nullptr, GLR_EINVAL, "the full basis is supported up to min(m, n) = 1024; set basis_rank%s");
+    if (exact && mp > kMaxFullBasis && !tcl_eligible(mp, np, r, N, k, exact, s))
+        return fail(nullptr, GLR_EINVAL,
+                    "the full basis above min(m, n) = 1024 needs min(m, n) a multiple of 128 up to 4096, "
+                    "max(m, n) a multiple of 8, bf16 gradients, MSGD or Adam, 16 <= r <= 128 (r a multiple of 4) "
+                    "and N <= 8; or set basis_rank%s");
     if (!exact && k > kMaxTruncBasis) return fail(nullptr, GLR_EINVAL, "basis_rank above 512 is not supported%s");
     if (!exact && (s->power_iters < 1 || s->power_iters > 64)) return fail(nullptr, GLR_EINVAL, "need 1 <= power_iters <= 64%s");
 
@@ -428,7 +431,10 @@ int glr_create(int64_t m, int64_t n, int32_t r, int32_t N, const glr_schedule* s
     // U = I (Algorithm 3 input): dense identity, or Q = I[:, :k], Y = T = 0, d = 1.
     std::vector<float> ones(static_cast<size_t>(mp), 1.f);
     cudaError_t e = cudaSuccess;
-    if (exact) e = cudaMemcpy2D(h->U, (MP + 1) * 4, ones.data(), 4, 4, MP, cudaMemcpyHostToDevice);
+    if (exact) {
+        e = cudaMemcpy2D(h->U, (MP + 1) * 4, ones.data(), 4, 4, MP, cudaMemcpyHostToDevice);
+        if (e == cudaSuccess && h->UT) e = cudaMemcpy2D(h->UT, (MP + 1) * 4, ones.data(), 4, 4, MP, cudaMemcpyHostToDevice);
+    }
     else {
         e = cudaMemcpy2D(h->Q, ((size_t)k + 1) * 4, ones.data(), 4, 4, k, cudaMemcpyHostToDevice);
         if (e == cudaSuccess) e = cudaMemcpy(h->dsign, ones.data(), 4 * (size_t)k, cudaMemcpyHostToDevice);
@@ -763,7 +769,7 @@ int tcl_compose(std::vector<StepPlan*>& plans, cudaStream_t st) {
 auto tc_wbar_fill(bool lam_plans) {
     return [lam_plans](StepPlan& p, tc::TcMat& M, tc::TcGroup&, bool) {
         glr_handle* h = p.h;
-        if (!p.compressed || tc_needs_lambda(p) != lam_plans) return 0;
+        if (!p.compressed || h->exact || tc_needs_lambda(p) != lam_plans) return 0;
         M.ntiles = cdiv(h->np, 256);
         M.mA = tcl_map(h, kMapMbarT); M.mB = tcl_map(h, kMapYT); M.W = h->WT;
         return 1;
@@ -774,12 +780,21 @@ auto tc_wbar_fill(bool lam_plans) {
 int tcl_lambda(std::vector<StepPlan*>& plans, cudaStream_t st) {
     int rc = tc_run(plans, GLR_PH_LAMBDA, tc::launch_wbar, st, tc_wbar_fill(true));
     if (rc != GLR_OK) return rc;
-    return tc_run(plans, GLR_PH_LAMBDA, tc::launch_lambda, st, [](StepPlan& p, tc::TcMat& M, tc::TcGroup&, bool) {
+    rc = tc_run(plans, GLR_PH_LAMBDA, tc::launch_lambda, st, [](StepPlan& p, tc::TcMat& M, tc::TcGroup&, bool) {
         glr_handle* h = p.h;
-        if (!tc_needs_lambda(p)) return 0;
+        if (!tc_needs_lambda(p) || h->exact) return 0;
         M.tm = cdiv(h->mp, 128); M.tn = cdiv(h->np, 128); M.ntiles = M.tm * M.tn;
         M.mA = tcl_map(h, kMapYt); M.mB = tcl_map(h, kMapWT); M.mD0 = tcl_map(h, kMapMbarL);
         M.Mbar = h->Mbar; M.part = h->lam_part;
+        return 1;
+    });
+    if (rc != GLR_OK) return rc;
+    // the full basis: the dense scores U^T Mbar with v_j in the epilogue
+    return tc_run(plans, GLR_PH_LAMBDA, tc::launch_lambda_u, st, [](StepPlan& p, tc::TcMat& M, tc::TcGroup&, bool) {
+        glr_handle* h = p.h;
+        if (!tc_needs_lambda(p) || !h->exact) return 0;
+        M.tm = cdiv(h->mp, 128); M.tn = cdiv(h->np, 128); M.ntiles = M.tm * M.tn;
+        M.mA = tcl_map(h, kMapUT); M.mB = tcl_map(h, kMapMbarT); M.part = h->lam_part;
         return 1;
     });
 }
@@ -790,18 +805,33 @@ int tcl_project(std::vector<StepPlan*>& plans, cudaStream_t st) {
     int rc = tc_run(plans, GLR_PH_PROJECT, tc::launch_wbar, st, tc_wbar_fill(false));
     if (rc != GLR_OK) return rc;
     // YtJ = Yt[J, :] was gathered by the selection launch
+    for (StepPlan* p : plans) {                 // a full basis: P = U[:, J] and P^T, gathered
+        glr_handle* h = p->h;
+        if (!p->compressed || !h->exact) continue;
+        PhaseScope ps(h, GLR_PH_SELECT, st);
+        GLR_LAUNCH(h, 1, tc::gather_p(h->U, h->mp, h->J, h->r, h->P, tcl_PT_of(h, h->P), st));
+    }
     rc = tc_run(plans, GLR_PH_SELECT, tc::launch_pbuild, st, [](StepPlan& p, tc::TcMat& M, tc::TcGroup&, bool) {
         glr_handle* h = p.h;
-        if (!p.compressed) return 0;
+        if (!p.compressed || h->exact) return 0;
         M.ntiles = cdiv(h->mp, 128);
         M.mA = tcl_map(h, kMapY); M.mB = tcl_map(h, kMapYtJn);
         M.J = h->J; M.dsign = h->dsign; M.Pout = h->P; M.PT = tcl_PT_of(h, h->P);
         return 1;
     });
     if (rc != GLR_OK) return rc;
+    // a full basis: Rbar^T = (P^T Mbar)^T by the R_w product on Mbar as a single node
+    rc = tc_run(plans, GLR_PH_PROJECT, tc::launch_prevproj, st, [](StepPlan& p, tc::TcMat& M, tc::TcGroup&, bool) {
+        glr_handle* h = p.h;
+        if (!p.compressed || !h->exact) return 0;
+        M.N = 1; M.na = 1; M.ng = 1; M.tn = cdiv(h->np, 128); M.ntiles = M.tn;
+        M.mA = tcl_map(h, kMapMbar3); M.mB = tcl_map_PT(h, h->P); M.Rw = h->RbarT;
+        return 1;
+    });
+    if (rc != GLR_OK) return rc;
     rc = tc_run(plans, GLR_PH_PROJECT, tc::launch_rbar, st, [](StepPlan& p, tc::TcMat& M, tc::TcGroup&, bool) {
         glr_handle* h = p.h;
-        if (!p.compressed) return 0;
+        if (!p.compressed || h->exact) return 0;
         M.ntiles = cdiv(h->np, 128);
         M.mA = tcl_map(h, kMapYtJm); M.mB = tcl_map(h, kMapWT);
         M.J = h->J; M.dsign = h->dsign; M.Mbar = h->Mbar; M.Rbar = h->Rbar; M.RbarT = h->RbarT;
@@ -909,7 +939,7 @@ int select_P_grouped(std::vector<StepPlan>& plans, cudaStream_t st, int stages =
         M.U = h->U; M.Y = h->Y; M.Yt = h->Yt; M.P = h->P;
         M.rbar = p.stream_update ? 1 : 0; M.np = h->np;
         M.Mbar = h->Mbar; M.Wbar = h->Wbar; M.Rbar = h->Rbar;
-        M.build_p = ((h->tc || h->tcl) && !h->exact) ? 0 : 1;
+        M.build_p = (h->tcl || (h->tc && !h->exact)) ? 0 : 1;   // the tcgen05 path builds its own P
         M.YtJ = (h->tcl && !h->exact) ? h->YtJ : nullptr;
         M.out0 = g.total_out;
         g.total_out += (M.build_p ? (int64_t)h->mp * h->r : 0) + (M.rbar ? (int64_t)h->r * h->np : 0);
@@ -1061,7 +1091,7 @@ int dp_select(glr_handle* h, cudaStream_t st, glr_dp_exchange* ex) {
         GLR_CK(h, cudaEventRecord(h->rfork, st));
         GLR_CK(h, cudaStreamWaitEvent(h->rstream, h->rfork, 0));
         std::vector<glr_handle*> hs{h};
-        rc = h->k <= 256 ? refresh_tcl_grouped(hs) : refresh_trunc_grouped(hs);
+        rc = h->exact ? refresh_exact_grouped(hs) : h->k <= 256 ? refresh_tcl_grouped(hs) : refresh_trunc_grouped(hs);
         if (rc != GLR_OK) return rc;
         GLR_CK(h, cudaEventRecord(h->rdone, h->rstream));
         GLR_CK(h, cudaStreamWaitEvent(st, h->rdone, 0));

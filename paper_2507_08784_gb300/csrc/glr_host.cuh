@@ -63,6 +63,11 @@ struct glr_handle {
     // TF32 transposes of Q and Z, Gram partials, L^{-1}
     float *Mrow = nullptr, *Mlo = nullptr, *QTt = nullptr, *ZTt = nullptr, *gpart = nullptr, *Linv = nullptr;
     float* Qbuf0 = nullptr;                       // Q's first allocation (Q and Qn trade places)
+    // the full basis on the tcgen05 path (m' > 1024): U^T rounded to TF32 (the score operand, part
+    // of the state), and the blocked Jacobi's scratch (not checkpointed): the second V buffer, the
+    // pair rotations (m' x 128), the pair solver's eigenvalues, the norm partials, the sweep count
+    float *UT = nullptr, *Vbuf2 = nullptr, *bjJ = nullptr, *bjev = nullptr, *bjpart = nullptr;
+    int bj_sweeps = 0, numeric_failures_host = 0;
     // a data-parallel step in progress (glr_dp_begin / glr_dp_select / glr_dp_finish): 0 idle,
     // 1 begun, 2 selected; the step's plan and the caller's gradient pointers
     int dp_stage = 0, dp_flags = 0;
@@ -185,7 +190,8 @@ int gemm(glr_handle* h, const GemmDesc& d, cudaStream_t st);
 // The tcgen05 large-matrix path (glr_tc_host.cu): eligibility, buffers, tensor maps.
 enum TcMap { kMapBt, kMapPT0, kMapPT1, kMapP0, kMapP1, kMapRwT, kMapMbarT, kMapYT, kMapYt, kMapWT, kMapY, kMapYtJn,
              kMapYtJm, kMapRbarT, kMapBtD, kMapMbarL, kMapMbarU, kMapMo, kMapVo,
-             kMapMrow, kMapMlo, kMapQTtA, kMapQTtB, kMapZTtA, kMapZTtB, kMapQA, kMapQA1, kMapZA, kMapLinv, kNumTcMaps };
+             kMapMrow, kMapMlo, kMapQTtA, kMapQTtB, kMapZTtA, kMapZTtB, kMapQA, kMapQA1, kMapZA, kMapLinv,
+             kMapUT, kMapMbar3, kNumTcMaps };
 // After the fixed maps: two slots of N gradient maps, then two slots for X (the caller's buffers,
 // re-described only when a pointer changes).
 const CUtensorMap* tcl_grad_maps(glr_handle* h, const void* const* G, cudaStream_t st, int* rc);
@@ -215,6 +221,7 @@ int cholqr(glr_handle* h, float*& A, float*& tmp, int rows, cudaStream_t st);
 int refresh_finish(glr_handle* h, cudaStream_t st);
 int refresh_grouped(std::vector<glr_handle*>& hs);
 int refresh_exact_grouped(std::vector<glr_handle*>& hs);
+int refresh_exact_blocked(std::vector<glr_handle*>& hs);   // m' > 1024, sorted by m'
 
 }  // namespace host
 }  // namespace glr

@@ -14,7 +14,7 @@ namespace glr {
 // Philox4x32-10 (Salmon, Moraes, Dror, Shaw, SC'11) and Box-Muller: the random vectors
 // v_j ~ N(0, I) of Eq. random-v.  Element (j, b) of the stacked m' x n' matrix uses counter
 // (b / 4, j, t, tag) and key (seed lo, seed hi); the four output words give two Box-Muller
-// pairs and v_j[b] = z_{b mod 4}.  Uniforms are (top 24 bits + 0.5) * 2^-24, exact in fp32.
+// pairs and v_j[b] = z_{b mod 4}.  Uniforms are (top 23 bits + 0.5) * 2^-23, exact in fp32.
 // ------------------------------------------------------------------------------------------
 constexpr uint32_t kTagLambdaV = 0x4C414D56u;   // v_j of Algorithm 2
 constexpr uint32_t kTagPowerInit = 0x50574954u; // random start block of the power iteration
@@ -301,6 +301,30 @@ struct EigGroup {
     EigMat mat[kEigGroupMax];
 };
 cudaError_t eig_tmem_group(const EigGroup& g, cudaStream_t st);
+
+// Blocked Jacobi rounds of the full-basis refresh above m' = 1024 (k_bjac.cu).  H, V: this
+// round's n x n matrices in the round's storage order; H2, V2 receive J^T H J and V J in the next
+// round's order; J: the round's n / 128 pair rotations, 128 x 128 row-major each.
+constexpr int kBjacMaxN = 4096;
+constexpr int kBjacGroupMax = 32;
+constexpr int kBjacNormCtas = 64;
+struct BjacMat {
+    int n, round;
+    const float* H; float* H2;
+    const float* V; float* V2;
+    const float* J;
+    int tile0h, tile0v;
+};
+struct BjacGroup {
+    int nmat, tiles_h, tiles_v;
+    BjacMat mat[kBjacGroupMax];
+};
+cudaError_t bjac_apply(BjacGroup& g, cudaStream_t st);
+// part[2 (i kBjacNormCtas + c) + {0, 1}]: CTA c's squared diagonal / off-diagonal sums of H_i
+cudaError_t bjac_norms(const BjacGroup& g, float* part, cudaStream_t st);
+cudaError_t bjac_eye(float* V, int n, cudaStream_t st);
+cudaError_t bjac_diag(const float* H, int n, float* evals, cudaStream_t st);
+cudaError_t count_flag(int* flag, int v, cudaStream_t st);   // *flag += v on the device
 int jacobi_group_grid();
 cudaError_t jacobi_group(const JacobiGroup& g, int grid, cudaStream_t st);
 // Q <- Q L^{-T} for the rows x n matrix Q (row-major) and lower-triangular L.
@@ -478,6 +502,7 @@ cudaError_t launch_prevproj(TcGroup& g, cudaStream_t st);
 cudaError_t launch_compose(TcGroup& g, cudaStream_t st);
 cudaError_t launch_wbar(TcGroup& g, cudaStream_t st);
 cudaError_t launch_lambda(TcGroup& g, cudaStream_t st);
+cudaError_t launch_lambda_u(TcGroup& g, cudaStream_t st);   // full basis: the scores from U^T Mbar
 cudaError_t launch_pbuild(TcGroup& g, cudaStream_t st);
 cudaError_t launch_rbar(TcGroup& g, cudaStream_t st);
 cudaError_t launch_update(TcGroup& g, cudaStream_t st);
@@ -494,6 +519,8 @@ cudaError_t split_lo(const float* src, float* lo, int64_t n, cudaStream_t st);
 int compose_bn();
 // dst (cols x ldd) = src^T rounded to TF32 (src row-major rows x cols, leading dimension lds)
 cudaError_t transpose_round(float* dst, int ldd, const float* src, int rows, int cols, int lds, cudaStream_t st);
+// P = U[:, J] (m' x r) and P^T (r x m') rounded to TF32, U row-major m' x m'
+cudaError_t gather_p(const float* U, int mp, const int32_t* J, int r, float* P, float* PT, cudaStream_t st);
 cudaError_t round_tf32(float* p, int64_t n, cudaStream_t st);
 // One wait of the pipeline's bounded kind on an mbarrier that never completes, `polls` polls.
 cudaError_t expire_wait(int* err, int polls, cudaStream_t st);

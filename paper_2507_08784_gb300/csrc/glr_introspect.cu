@@ -204,6 +204,7 @@ int glr_set_basis(glr_handle* h, const float* Q, void* stream) {
     const size_t mp = h->mp, k = h->k;
     if (h->exact) {
         GLR_CK(h, cudaMemcpyAsync(h->U, Q, 4 * mp * mp, cudaMemcpyDeviceToDevice, st));
+        if (h->UT) GLR_LAUNCH(h, 1, tc::transpose_round(h->UT, (int)mp, h->U, (int)mp, (int)mp, (int)mp, st));
     } else {
         GLR_CK(h, cudaMemcpyAsync(h->Q, Q, 4 * mp * k, cudaMemcpyDeviceToDevice, st));
         int rc = wy_from_Q(h, st);

@@ -115,6 +115,17 @@ int refresh_grouped(std::vector<glr_handle*>& hs) {
 // cooperative Jacobi launch for all of them on the first handle's side stream (k_jacobi.cu), then
 // each handle sorts its eigenvectors by descending eigenvalue and fixes their signs on its own.
 int refresh_exact_grouped(std::vector<glr_handle*>& hs) {
+    {   // above m' = 1024: the blocked solver (tcgen05 path only)
+        std::vector<glr_handle*> big, small;
+        for (glr_handle* h : hs) (h->mp > kMaxFullBasis ? big : small).push_back(h);
+        if (!big.empty()) {
+            std::stable_sort(big.begin(), big.end(), [](const glr_handle* a, const glr_handle* b) { return a->mp < b->mp; });
+            const int rc = refresh_exact_blocked(big);
+            if (rc != GLR_OK) return rc;
+        }
+        if (small.empty()) return GLR_OK;
+        hs.swap(small);
+    }
     const int grid = jacobi_group_grid();
     for (size_t c0 = 0, c1 = 0; c0 < hs.size(); c0 = c1) {
         // a group: at most kGroupMax matrices whose rotations fit the kernel's shared memory
@@ -166,6 +177,135 @@ int refresh_exact_grouped(std::vector<glr_handle*>& hs) {
             GLR_LAUNCH(h, 1, sort_fix_basis(h->evals, h->Vbuf, h->mp, h->mp, h->U, h->mp, h->evals_sorted, h->rstream));
         }
     }
+    return GLR_OK;
+}
+
+// Full-basis refreshes above m' = 1024 (k_bjac.cu), all on the first handle's side stream:
+// H = Mbar Mbar^T by the grouped FFMA product (Mbar is column-major on the tcgen05 path), V = I,
+// then the blocked Jacobi rounds of every matrix of the same size together, one sweep at a time,
+// each sweep opened by the norm check (summed on the host in a fixed order, so that the decision
+// does not depend on the grouping); finally each handle's sorted, sign-fixed U and its TF32
+// transpose.  A matrix that has not converged after kBjacMaxSweeps sweeps keeps its last basis
+// and counts a numeric failure (GLR_ENUMERIC from glr_get_stats).
+constexpr int kBjacMaxSweeps = 30;
+
+int refresh_exact_blocked(std::vector<glr_handle*>& hs) {
+    glr_handle* h0 = hs[0];
+    cudaStream_t s0 = h0->rstream;
+    for (glr_handle* h : hs) {
+        if (h == h0) continue;
+        GLR_CK(h, cudaEventRecord(h->rpow, h->rstream));
+        GLR_CK(h0, cudaStreamWaitEvent(s0, h->rpow, 0));
+    }
+    PhaseScope ps(h0, GLR_PH_REFRESH, s0);
+    {   // H = Mbar Mbar^T: Mbar^T is n' x m' row-major
+        GemmGroup gg{};
+        auto flush = [&]() -> int {
+            if (gg.nmat) GLR_LAUNCH(h0, 1, gemm_group_f32(gg, s0));
+            gg.nmat = 0;
+            return GLR_OK;
+        };
+        for (glr_handle* h : hs) {
+            GemmMat& G = gg.mat[gg.nmat++];
+            G = GemmMat{};
+            G.M = h->mp; G.N = h->mp; G.K = h->np; G.alpha = 1.f;
+            G.A = h->Mbar; G.sAi = 1; G.sAp = h->mp;
+            G.B = h->Mbar; G.sBp = h->mp; G.sBj = 1;
+            G.C = h->Hbuf; G.sCi = h->mp; G.sCj = 1;
+            if (gg.nmat == 64 && flush() != GLR_OK) return GLR_ECUDA;
+            GLR_LAUNCH(h, 1, bjac_eye(h->Vbuf, h->mp, s0));
+        }
+        if (flush() != GLR_OK) return GLR_ECUDA;
+    }
+    struct State { glr_handle* h; float *H, *H2, *V, *V2; int rd; bool done; };
+    std::vector<State> all;
+    for (glr_handle* h : hs) all.push_back(State{h, h->Hbuf, h->jwork, h->Vbuf, h->Vbuf2, 0, false});
+    std::vector<float> part;
+    for (size_t a0 = 0; a0 < all.size();) {
+        // the matrices of one size
+        size_t a1 = a0;
+        while (a1 < all.size() && all[a1].h->mp == all[a0].h->mp) ++a1;
+        const int n = all[a0].h->mp, m = n / 64, P = n / 128;
+        const double tol = 4.0 * 5.96e-8 * std::sqrt((double)n) + 1e-7;
+        for (int sweep = 0;; ++sweep) {
+            // the norm check of every unfinished matrix
+            std::vector<State*> act;
+            for (size_t a = a0; a < a1; ++a)
+                if (!all[a].done) act.push_back(&all[a]);
+            for (size_t c0 = 0; c0 < act.size(); c0 += kBjacGroupMax) {
+                BjacGroup g{};
+                for (size_t c = c0; c < act.size() && c < c0 + kBjacGroupMax; ++c) {
+                    BjacMat& M = g.mat[g.nmat++];
+                    M.n = n; M.H = act[c]->H;
+                }
+                GLR_LAUNCH(h0, 1, bjac_norms(g, h0->bjpart, s0));
+                part.resize((size_t)2 * kBjacNormCtas * g.nmat);
+                GLR_CK(h0, cudaMemcpyAsync(part.data(), h0->bjpart, sizeof(float) * part.size(), cudaMemcpyDeviceToHost, s0));
+                GLR_CK(h0, cudaStreamSynchronize(s0));
+                for (int i = 0; i < g.nmat; ++i) {
+                    double d = 0.0, o = 0.0;
+                    for (int c = 0; c < kBjacNormCtas; ++c) {
+                        d += part[2 * ((size_t)i * kBjacNormCtas + c)];
+                        o += part[2 * ((size_t)i * kBjacNormCtas + c) + 1];
+                    }
+                    State* S = act[c0 + i];
+                    if (o <= tol * tol * (o + d)) S->done = true;
+                    else if (sweep == kBjacMaxSweeps) {
+                        S->done = true;
+                        S->h->numeric_failures_host++;
+                    }
+                    if (S->done) S->h->bj_sweeps = sweep;
+                }
+            }
+            act.erase(std::remove_if(act.begin(), act.end(), [](State* S) { return S->done; }), act.end());
+            if (act.empty()) break;
+            for (int round = 0; round < m - 1; ++round) {
+                EigGroup eg{};
+                eg.max_sweeps = 1;
+                for (State* S : act)
+                    for (int k = 0; k < P; ++k) {
+                        EigMat& E = eg.mat[eg.nmat++];
+                        E.n = 128; E.tol = 0.f; E.H = S->H + (size_t)128 * k * (n + 1); E.nparts = 1; E.ld = n;
+                        E.V = S->h->bjJ + (size_t)k * 16384; E.evals = S->h->bjev + 128 * k; E.sweeps = nullptr;
+                        if (eg.nmat == kEigGroupMax) {
+                            GLR_LAUNCH(h0, 1, eig_tmem_group(eg, s0));
+                            eg.nmat = 0;
+                        }
+                    }
+                if (eg.nmat) GLR_LAUNCH(h0, 1, eig_tmem_group(eg, s0));
+                for (size_t c0 = 0; c0 < act.size(); c0 += kBjacGroupMax) {
+                    BjacGroup g{};
+                    for (size_t c = c0; c < act.size() && c < c0 + kBjacGroupMax; ++c) {
+                        State* S = act[c];
+                        BjacMat& M = g.mat[g.nmat++];
+                        M.n = n; M.round = S->rd; M.H = S->H; M.H2 = S->H2; M.V = S->V; M.V2 = S->V2; M.J = S->h->bjJ;
+                    }
+                    GLR_LAUNCH(h0, 2, bjac_apply(g, s0));
+                }
+                for (State* S : act) {
+                    std::swap(S->H, S->H2);
+                    std::swap(S->V, S->V2);
+                    S->rd = (S->rd + 1) % (m - 1);
+                }
+            }
+        }
+        a0 = a1;
+    }
+    for (State& S : all) {
+        glr_handle* h = S.h;
+        const int n = h->mp;
+        GLR_LAUNCH(h, 1, bjac_diag(S.H, n, h->evals, s0));
+        GLR_LAUNCH(h, 1, sort_fix_basis(h->evals, S.V, n, n, h->U, n, h->evals_sorted, s0));
+        GLR_LAUNCH(h, 1, tc::transpose_round(h->UT, n, h->U, n, n, n, s0));
+        GLR_CK(h, cudaMemcpyAsync(h->dflags + 1, &h->bj_sweeps, sizeof(int), cudaMemcpyHostToDevice, s0));
+        if (h->numeric_failures_host) {
+            GLR_LAUNCH(h, 1, count_flag(h->dflags + 6, h->numeric_failures_host, s0));
+            h->numeric_failures_host = 0;
+        }
+    }
+    GLR_CK(h0, cudaEventRecord(h0->rpow, s0));
+    for (glr_handle* h : hs)
+        if (h != h0) GLR_CK(h, cudaStreamWaitEvent(h->rstream, h0->rpow, 0));
     return GLR_OK;
 }
 

@@ -15,10 +15,12 @@ inline int up32(int x) { return (x + 31) & ~31; }
 // columns), 16 <= r <= 128 (the projected mean takes one 128-row tile), k <= 256 (one MMA's N)
 // and m' >= 128 (one MMA's M).
 bool tcl_eligible(int64_t mp, int64_t np, int r, int N, int k, bool exact, const glr_schedule* s) {
-    if (exact || s->grad_dtype != GLR_BF16) return false;
+    if (s->grad_dtype != GLR_BF16) return false;
+    // the full basis takes this path above m' = 1024 only (the blocked Jacobi's 128-index pairs)
+    if (exact && (mp <= kMaxFullBasis || mp > kBjacMaxN || mp % 128)) return false;
     if (s->optimizer != GLR_MSGD && s->optimizer != GLR_ADAM) return false;
     if (mp % 8 || np % 8 || r % 4 || k % 4) return false;   // bf16 rows of 16-byte multiples too
-    if (N > 8 || r < 16 || r > 128 || k > 256) return false;
+    if (N > 8 || r < 16 || r > 128 || (!exact && k > 256)) return false;
     return mp >= 128;
 }
 
@@ -37,8 +39,12 @@ int tcl_alloc(glr_handle* h) {
     auto A = [&](float** p, size_t cnt) { if (rc == GLR_OK) rc = alloc(h, p, cnt); };
     A(&h->PT0, (size_t)h->rpad * MP);
     A(&h->PT1, (size_t)h->rpad * MP);
-    A(&h->WT, NP * h->kpad);
-    A(&h->YTk, (size_t)h->kpad * MP);
+    if (h->exact) {
+        A(&h->UT, MP * MP);
+    } else {
+        A(&h->WT, NP * h->kpad);
+        A(&h->YTk, (size_t)h->kpad * MP);
+    }
     A(&h->RbarT, NP * h->rpad);
     h->Pbuf0 = h->P;
     return rc;
@@ -59,10 +65,15 @@ int tcl_maps(glr_handle* h) {
     {   // refresh scratch, allocated after the checkpointed state
         int rc = GLR_OK;
         auto A = [&](float** p, size_t cnt) { if (rc == GLR_OK) rc = alloc(h, p, cnt); };
-        const size_t nch = (np + tc::kGramChunk - 1) / tc::kGramChunk;
-        A(&h->Mrow, mp * np); A(&h->Mlo, mp * np);
-        A(&h->QTt, kp * mp); A(&h->ZTt, kp * np);
-        A(&h->gpart, std::max<size_t>(nch, 1) * kp * kp); A(&h->Linv, kp * kp);
+        if (h->exact) {
+            A(&h->Vbuf2, mp * mp); A(&h->bjJ, mp * 128); A(&h->bjev, mp);
+            A(&h->bjpart, (size_t)2 * kBjacNormCtas * kBjacGroupMax);
+        } else {
+            const size_t nch = (np + tc::kGramChunk - 1) / tc::kGramChunk;
+            A(&h->Mrow, mp * np); A(&h->Mlo, mp * np);
+            A(&h->QTt, kp * mp); A(&h->ZTt, kp * np);
+            A(&h->gpart, std::max<size_t>(nch, 1) * kp * kp); A(&h->Linv, kp * kp);
+        }
         if (rc != GLR_OK) return rc;
     }
     std::vector<CUtensorMap> maps(kNumTcMaps);
@@ -85,13 +96,17 @@ int tcl_maps(glr_handle* h) {
     m2(kMapP1, Pother, r, mp, r, 128);
     m3(kMapRwT, h->Rw, rp, np, N, (uint32_t)tc::compose_bn());   // R_w,i^T: n' x rpad per node
     m2(kMapMbarT, h->Mbar, mp, np, mp, 128);               // Mbar^T: n' x m'
+    m2(kMapRbarT, h->RbarT, rp, np, rp, 128);              // Rbar^T: n' x rpad
+    if (h->exact) {
+        m2(kMapUT, h->UT, mp, mp, mp, 128);                // U^T (TF32), row-major m' x m'
+        m3(kMapMbar3, h->Mbar, mp, np, 1, 128);            // Mbar^T as a one-node B^T
+    } else {
     m2(kMapYT, h->YTk, mp, kp, mp, (uint32_t)kp);          // Y^T: kpad x m'
     m2(kMapYt, h->Yt, k, mp, k, 128);                      // Yt, row-major m' x k
     m2(kMapWT, h->WT, kp, np, kp, 128);                    // W^T: n' x kpad
     m2(kMapY, h->Y, k, mp, k, 128);                        // Y, row-major m' x k
     m2(kMapYtJn, h->YtJ, k, r, k, (uint32_t)rp);           // Yt[J, :] (r x k) as the N operand
     m2(kMapYtJm, h->YtJ, k, r, k, 128);                    // ... and as the M operand
-    m2(kMapRbarT, h->RbarT, rp, np, rp, 128);              // Rbar^T: n' x rpad
     // the refresh products
     m2(kMapMrow, h->Mrow, np, mp, np, 128);                // Mbar row-major: m' x n'
     m2(kMapMlo, h->Mlo, np, mp, np, 128);                  // its TF32 low parts
@@ -104,6 +119,7 @@ int tcl_maps(glr_handle* h) {
     m2(kMapQA1, h->Qn, k, mp, k, 128);
     m2(kMapZA, h->Z, k, np, k, 128);
     m2(kMapLinv, h->Linv, kp, kp, kp, (uint32_t)kp);       // L^{-1}, row-major kpad x kpad
+    }
     // epilogue data tiles (no swizzle unless noted)
     auto plain = [&](int idx, const void* base, int rank, const uint64_t* dims, const uint64_t* str, const uint32_t* box,
                      CUtensorMapSwizzle swz) {

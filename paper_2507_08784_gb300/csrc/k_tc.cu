@@ -648,6 +648,54 @@ struct Lambda {
 };
 
 // ------------------------------------------------------------------------------------------
+// LambdaU (full basis): tile = (128 rows j, 128 columns b).  D = U^T[j, :] Mbar[:, b] (K = m'),
+// and the epilogue adds D(j, b) v_j[b] over each warp's 32 columns into part[(4 ct + h) m' + j]
+// (Algorithm 2's u_j^T Mbar v_j, the dense form of the scores).  A = U^T (m' x m', TF32),
+// B = Mbar^T (n' x m').
+// ------------------------------------------------------------------------------------------
+struct LambdaU : NoData {
+    static constexpr int kEpi = 16;
+    static __device__ __forceinline__ int nk(const TcGroup& g, const Tile& t) { return (g.mat[t.mat].mp + 31) / 32; }
+    static __device__ __forceinline__ uint32_t tx_bytes(const TcGroup&, const Tile&, int) { return 2u * 16384u; }
+    static __device__ __forceinline__ void load(const TcGroup& g, const Tile& t, int kc, uint32_t st, uint32_t bar) {
+        const TcMat& M = g.mat[t.mat];
+        const int rt = t.lt / M.tn, ct = t.lt % M.tn;
+        tma_load_2d(st, M.mA, kc * 32, rt * 128, bar);
+        tma_load_2d(st + 16384u, M.mB, kc * 32, ct * 128, bar);
+    }
+    static __device__ __forceinline__ void mma(const TcGroup&, const Tile&, int kc, uint32_t st, uint32_t d) {
+        mma_slice(d, st, st + 16384u, 128, kc == 0);
+    }
+    static __device__ __forceinline__ bool epilogue(const TcGroup& g, const Tile& t, uint32_t tl, int warp, int lane,
+                                                    DataRing&) {
+        const TcMat& M = g.mat[t.mat];
+        const int rt = t.lt / M.tn, ct = t.lt % M.tn;
+        const int j = rt * 128 + 32 * (warp & 3) + lane;
+        const int h = warp >> 2;                              // this warp's 32 columns
+        const int b0 = ct * 128 + 32 * h;
+        float acc = 0.f;
+        for (int cc = 0; cc < 32; cc += 16) {
+            float d[16];
+            tmem_ld16(tl + (uint32_t)(32 * h + cc), d);
+            if (j < M.mp) {
+#pragma unroll
+                for (int qq = 0; qq < 4; ++qq) {
+                    const int b = b0 + cc + 4 * qq;
+                    if (b >= M.np) break;
+                    const float4 v = gauss4_fast(M.seed, M.t, (uint32_t)j, (uint32_t)(b >> 2), kTagLambdaV);
+                    const float vv[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+                    for (int e = 0; e < 4; ++e)
+                        if (b + e < M.np) acc += d[4 * qq + e] * vv[e];
+                }
+            }
+        }
+        if (j < M.mp) M.part[(int64_t)(4 * ct + h) * M.mp + j] = acc;
+        return true;
+    }
+};
+
+// ------------------------------------------------------------------------------------------
 // PBuild: tile = 128 rows a.  D (128 x rpad) = Y[a, :] Yt[J, :]^T (K = k); the epilogue writes
 // P(a, q) = d_{J_q} ([a == J_q] - D(a, q)) (rounded to TF32) and P^T.  A = Y (m' x k), B = YtJ
 // (r x k, rows past r read as zeros).
@@ -1018,6 +1066,7 @@ template <> size_t stage_bytes_of<PrevProj>(const TcMat& M) { return (size_t)M.n
 template <> size_t stage_bytes_of<Compose>(const TcMat& M) { return 16384 + (size_t)M.N * Compose::BN * 128; }
 template <> size_t stage_bytes_of<WBar>(const TcMat& M) { return 2 * 16384 + (size_t)M.kpad * 128; }
 template <> size_t stage_bytes_of<Lambda>(const TcMat&) { return 2 * 16384; }
+template <> size_t stage_bytes_of<LambdaU>(const TcMat&) { return 2 * 16384; }
 template <> size_t stage_bytes_of<PBuild>(const TcMat& M) { return 16384 + (size_t)M.rpad * 128; }
 template <> size_t stage_bytes_of<RBar>(const TcMat&) { return 2 * 16384; }
 template <> size_t stage_bytes_of<Update>(const TcMat&) { return 2 * 16384; }
@@ -1032,6 +1081,7 @@ template <> int acc_cols_of<PrevProj>(const TcMat& M) { return M.na * M.rpad; }
 template <> int acc_cols_of<Compose>(const TcMat& M) { return M.N * Compose::BN; }
 template <> int acc_cols_of<WBar>(const TcMat& M) { return 2 * M.kpad; }
 template <> int acc_cols_of<Lambda>(const TcMat&) { return 128; }
+template <> int acc_cols_of<LambdaU>(const TcMat&) { return 128; }
 template <> int acc_cols_of<PBuild>(const TcMat& M) { return M.rpad; }
 template <> int acc_cols_of<RBar>(const TcMat&) { return 128; }
 template <> int acc_cols_of<Update>(const TcMat&) { return 128; }
@@ -1098,6 +1148,7 @@ cudaError_t launch_prevproj(TcGroup& g, cudaStream_t st) { return launch<PrevPro
 cudaError_t launch_compose(TcGroup& g, cudaStream_t st) { return launch<Compose>(g, st); }
 cudaError_t launch_wbar(TcGroup& g, cudaStream_t st) { return launch<WBar>(g, st); }
 cudaError_t launch_lambda(TcGroup& g, cudaStream_t st) { return launch<Lambda>(g, st); }
+cudaError_t launch_lambda_u(TcGroup& g, cudaStream_t st) { return launch<LambdaU>(g, st); }
 cudaError_t launch_pbuild(TcGroup& g, cudaStream_t st) { return launch<PBuild>(g, st); }
 cudaError_t launch_rbar(TcGroup& g, cudaStream_t st) { return launch<RBar>(g, st); }
 cudaError_t launch_update(TcGroup& g, cudaStream_t st) { return launch<Update>(g, st); }
@@ -1112,6 +1163,17 @@ int compose_bn() { return Compose::BN; }
 namespace {
 // dst (cols x ldd) = src^T rounded to TF32, src row-major rows x cols (leading dim lds); rows of
 // dst past `rows` are left alone (zero from allocation).
+// P = U[:, J] (m' x r, row-major) and P^T (r x m'), rounded to TF32: the projector of a full basis.
+__global__ void gather_p_kernel(const float* __restrict__ U, int mp, const int32_t* __restrict__ J, int r,
+                                float* __restrict__ P, float* __restrict__ PT) {
+    const int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+    if (e >= (int64_t)mp * r) return;
+    const int q = (int)(e / mp), a = (int)(e % mp);
+    const float v = rna_tf32(U[(int64_t)a * mp + J[q]]);
+    P[(int64_t)a * r + q] = v;
+    PT[(int64_t)q * mp + a] = v;
+}
+
 __global__ void transpose_round_kernel(float* dst, int ldd, const float* src, int rows, int cols, int lds) {
     __shared__ float tile[32][33];
     const int r0 = blockIdx.y * 32, c0 = blockIdx.x * 32;
@@ -1177,6 +1239,12 @@ cudaError_t split_lo(const float* src, float* lo, int64_t n, cudaStream_t st) {
 
 cudaError_t expire_wait(int* err, int polls, cudaStream_t st) {
     expire_kernel<<<1, 32, 0, st>>>(err, polls);
+    return cudaGetLastError();
+}
+
+cudaError_t gather_p(const float* U, int mp, const int32_t* J, int r, float* P, float* PT, cudaStream_t st) {
+    const int64_t n = (int64_t)mp * r;
+    gather_p_kernel<<<(unsigned)((n + 255) / 256), 256, 0, st>>>(U, mp, J, r, P, PT);
     return cudaGetLastError();
 }
 
