@@ -40,6 +40,15 @@ METRIC = "gradient elems/s per GreedyLore step & % HBM roofline; subspace refres
 UNIT = "grad-elem/s"
 WORKLOAD = "cfg5_llama_d4096"
 EXTRA_WORKLOADS = ("cfg2_resnet", "cfg3_llama_d2048", "cfg4_refresh")
+PAPER_EXACT = "cfg5_layer_paper_exact"     # one d = 4096 decoder layer with the full m' x m' basis
+
+
+def paper_exact_config():
+    """One layer of the d = 4096 decoder stack (Wq, Wk, Wv, Wo, Wgate, Wup, Wdown; N = 4, bf16,
+    Adam, r = 128) with basis_rank = 0: the paper-exact basis of Eq. SVD-P1, refreshed by the
+    blocked Jacobi eigen-solve, its scores the dense U^T Mbar."""
+    base = W.config("cfg5_llama_d4096")
+    return W.config("cfg5_llama_d4096", name=PAPER_EXACT, shapes=base.shapes[:7], basis_rank=0)
 
 
 def _peaks():
@@ -238,12 +247,13 @@ def bench_mode(torch, glr, cfg, basis_rank, K, Wm, dist_ctx, gsets, refresh_reps
         run_steps(hs, gsets, X, t3, 1)             # the step after (error reset), untimed
         t3 += 1
     path = hs[0].stats()["path"]
+    sweeps = [h.stats()["last_refresh_sweeps"] for h in hs]
     for h in hs:
         h.close()
     return {"ms": ms, "launches": launches, "refreshes": refreshes, "ms_prof": ms_prof, "phases": phases,
             "compose_bytes": comp_bytes, "nonrefresh_step_ms": statistics.median(nonref) if nonref else None,
             "refresh_step_ms_in_window": statistics.mean(ref) if ref else None,
-            "forced_refresh_step_ms": forced, "path": path}
+            "forced_refresh_step_ms": forced, "path": path, "sweeps": sweeps}
 
 
 def bench_e2e(torch, glr, cfg, K, Wm, dist_ctx):
@@ -437,6 +447,38 @@ def summarize(cfg, run, K, world, hbm_peak):
     }
 
 
+def bench_paper_exact(torch, glr, K, Wm, ctx, hbm_peak):
+    """The paper-exact basis on one d = 4096 decoder layer: compressed steps with the dense scores
+    U^T Mbar (TF32 tcgen05, 2 m'^2 n' flops per matrix) and one forced refresh step (the blocked
+    Jacobi eigen-solve of Mbar Mbar^T for all 7 matrices)."""
+    xc = paper_exact_config()
+    xp = W.make_problem(xc)
+    xs = [[W.gradients_torch(xp, li, t) for li in range(len(xc.shapes))] for t in range(2)]
+    xr = bench_mode(torch, glr, xc, 0, K, Wm, ctx, xs, refresh_reps=1)
+    out = summarize(xc, xr, K, ctx.world, hbm_peak)
+    out["config"] = {"matrices": len(xc.shapes), "shapes": "4 x 4096x4096, 2 x 11008x4096, 4096x11008",
+                     "N": xc.N, "r": xc.r, "basis_rank": 0, "tau": xc.tau, "grad_dtype": xc.grad_dtype,
+                     "optimizer": xc.optimizer, "refresh_mode": refresh_mode_of(xc)}
+    flops = sum(2.0 * min(m, n) ** 2 * max(m, n) for (m, n) in xc.shapes)
+    lam_ms = xr["phases"]["lambda"]["ms"] / K
+    tpeak, tkind = tensor_peak_tflops()
+    out["scores_tensor"] = {
+        "kernel": "tc_kernel<LambdaU> (U^T Mbar, v_j in the epilogue)", "flops_per_step": flops, "ms": lam_ms,
+        "tflops": flops / (lam_ms / 1e3) / 1e12, "tf32_peak": tpeak * TF32_OVER_BF16,
+        "frac_of_tf32_peak": flops / (lam_ms / 1e3) / 1e12 / (tpeak * TF32_OVER_BF16),
+        "peak_kind": tkind + " bf16 sustained x nominal TF32/BF16 ratio (1.1 / 2.25)"}
+    forced, nonref = xr["forced_refresh_step_ms"], xr["nonrefresh_step_ms"]
+    ref = statistics.median(forced) - nonref if forced and nonref else None
+    out["refresh"] = {"forced_refresh_step_ms": forced, "refresh_ms_per_layer": ref,
+                      "refresh_ms_per_matrix": ref / len(xc.shapes) if ref else None,
+                      "jacobi_sweeps": xr["sweeps"],
+                      "method": "H = Mbar Mbar^T (FFMA), blocked two-sided Jacobi: 128-index pair blocks "
+                                "solved by one scalar-Jacobi sweep each, block rotations as FFMA products"}
+    del xs
+    torch.cuda.empty_cache()
+    return out
+
+
 def ncu_case(refresh=False, stress=False):
     """One 4096 x 4096 matrix of the headline stack for 4 steps (about 1.1 GB of state): the
     compose launch of step 2 (index 2 among compose launches) is a full one; with refresh, a
@@ -540,6 +582,7 @@ def main():
                     "peak_kind": tkind + " bf16 sustained x nominal TF32/BF16 ratio (1.1 / 2.25)"}
             del xs
             torch.cuda.empty_cache()
+        extras[PAPER_EXACT] = bench_paper_exact(torch, glr, K, args.warmup, ctx, hbm_peak)
 
     elems = cfg.N * cfg.matrix_elems()
     head = summarize(cfg, main_run, K, ctx.world, hbm_peak)

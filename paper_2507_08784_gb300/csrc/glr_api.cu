@@ -793,7 +793,7 @@ int tcl_lambda(std::vector<StepPlan*>& plans, cudaStream_t st) {
     return tc_run(plans, GLR_PH_LAMBDA, tc::launch_lambda_u, st, [](StepPlan& p, tc::TcMat& M, tc::TcGroup&, bool) {
         glr_handle* h = p.h;
         if (!tc_needs_lambda(p) || !h->exact) return 0;
-        M.tm = cdiv(h->mp, 128); M.tn = cdiv(h->np, 128); M.ntiles = M.tm * M.tn;
+        M.tm = cdiv(h->mp, 128); M.tn = cdiv(h->np, 256); M.ntiles = M.tm * M.tn;
         M.mA = tcl_map(h, kMapUT); M.mB = tcl_map(h, kMapMbarT); M.part = h->lam_part;
         return 1;
     });
@@ -932,7 +932,8 @@ int select_P_grouped(std::vector<StepPlan>& plans, cudaStream_t st, int stages =
         glr_handle* h = p.h;
         if (!h0) h0 = h;
         SelectMat& M = g.mat[g.nmat++];
-        M.part = h->lam_part; M.ntiles = h->tcl ? h->tc_lam_tiles : p.lam_fused ? h->nstrips : h->ntiles;
+        M.part = h->lam_part;
+        M.ntiles = h->tcl ? (h->exact ? 4 * cdiv(h->np, 256) : h->tc_lam_tiles) : p.lam_fused ? h->nstrips : h->ntiles;
         M.mp = h->mp; M.r = h->r; M.k = h->k; M.mode = h->exact ? 0 : 1;
         M.do_select = (!p.refresh && !p.forced && !p.fixed) ? 1 : 0;
         M.dsign = h->exact ? nullptr : h->dsign; M.lam = h->lam; M.J = h->J;

@@ -648,35 +648,36 @@ struct Lambda {
 };
 
 // ------------------------------------------------------------------------------------------
-// LambdaU (full basis): tile = (128 rows j, 128 columns b).  D = U^T[j, :] Mbar[:, b] (K = m'),
-// and the epilogue adds D(j, b) v_j[b] over each warp's 32 columns into part[(4 ct + h) m' + j]
-// (Algorithm 2's u_j^T Mbar v_j, the dense form of the scores).  A = U^T (m' x m', TF32),
-// B = Mbar^T (n' x m').
+// LambdaU (full basis): tile = (128 rows j, 256 columns b).  D = U^T[j, :] Mbar[:, b] (K = m',
+// N = 256: each U^T slice serves 256 columns), and the epilogue adds D(j, b) v_j[b] over each
+// warp's 64 columns into part[(4 ct + h) m' + j] (Algorithm 2's u_j^T Mbar v_j, the dense form of
+// the scores).  A = U^T (m' x m', TF32), B = Mbar^T (n' x m') in two 128-row boxes.
 // ------------------------------------------------------------------------------------------
 struct LambdaU : NoData {
     static constexpr int kEpi = 16;
     static __device__ __forceinline__ int nk(const TcGroup& g, const Tile& t) { return (g.mat[t.mat].mp + 31) / 32; }
-    static __device__ __forceinline__ uint32_t tx_bytes(const TcGroup&, const Tile&, int) { return 2u * 16384u; }
+    static __device__ __forceinline__ uint32_t tx_bytes(const TcGroup&, const Tile&, int) { return 3u * 16384u; }
     static __device__ __forceinline__ void load(const TcGroup& g, const Tile& t, int kc, uint32_t st, uint32_t bar) {
         const TcMat& M = g.mat[t.mat];
         const int rt = t.lt / M.tn, ct = t.lt % M.tn;
         tma_load_2d(st, M.mA, kc * 32, rt * 128, bar);
-        tma_load_2d(st + 16384u, M.mB, kc * 32, ct * 128, bar);
+        tma_load_2d(st + 16384u, M.mB, kc * 32, ct * 256, bar);
+        tma_load_2d(st + 32768u, M.mB, kc * 32, ct * 256 + 128, bar);
     }
     static __device__ __forceinline__ void mma(const TcGroup&, const Tile&, int kc, uint32_t st, uint32_t d) {
-        mma_slice(d, st, st + 16384u, 128, kc == 0);
+        mma_slice(d, st, st + 16384u, 256, kc == 0);
     }
     static __device__ __forceinline__ bool epilogue(const TcGroup& g, const Tile& t, uint32_t tl, int warp, int lane,
                                                     DataRing&) {
         const TcMat& M = g.mat[t.mat];
         const int rt = t.lt / M.tn, ct = t.lt % M.tn;
         const int j = rt * 128 + 32 * (warp & 3) + lane;
-        const int h = warp >> 2;                              // this warp's 32 columns
-        const int b0 = ct * 128 + 32 * h;
+        const int h = warp >> 2;                              // this warp's 64 columns
+        const int b0 = ct * 256 + 64 * h;
         float acc = 0.f;
-        for (int cc = 0; cc < 32; cc += 16) {
+        for (int cc = 0; cc < 64; cc += 16) {
             float d[16];
-            tmem_ld16(tl + (uint32_t)(32 * h + cc), d);
+            tmem_ld16(tl + (uint32_t)(64 * h + cc), d);
             if (j < M.mp) {
 #pragma unroll
                 for (int qq = 0; qq < 4; ++qq) {
@@ -1066,7 +1067,7 @@ template <> size_t stage_bytes_of<PrevProj>(const TcMat& M) { return (size_t)M.n
 template <> size_t stage_bytes_of<Compose>(const TcMat& M) { return 16384 + (size_t)M.N * Compose::BN * 128; }
 template <> size_t stage_bytes_of<WBar>(const TcMat& M) { return 2 * 16384 + (size_t)M.kpad * 128; }
 template <> size_t stage_bytes_of<Lambda>(const TcMat&) { return 2 * 16384; }
-template <> size_t stage_bytes_of<LambdaU>(const TcMat&) { return 2 * 16384; }
+template <> size_t stage_bytes_of<LambdaU>(const TcMat&) { return 3 * 16384; }
 template <> size_t stage_bytes_of<PBuild>(const TcMat& M) { return 16384 + (size_t)M.rpad * 128; }
 template <> size_t stage_bytes_of<RBar>(const TcMat&) { return 2 * 16384; }
 template <> size_t stage_bytes_of<Update>(const TcMat&) { return 2 * 16384; }
@@ -1081,7 +1082,7 @@ template <> int acc_cols_of<PrevProj>(const TcMat& M) { return M.na * M.rpad; }
 template <> int acc_cols_of<Compose>(const TcMat& M) { return M.N * Compose::BN; }
 template <> int acc_cols_of<WBar>(const TcMat& M) { return 2 * M.kpad; }
 template <> int acc_cols_of<Lambda>(const TcMat&) { return 128; }
-template <> int acc_cols_of<LambdaU>(const TcMat&) { return 128; }
+template <> int acc_cols_of<LambdaU>(const TcMat&) { return 256; }
 template <> int acc_cols_of<PBuild>(const TcMat& M) { return M.rpad; }
 template <> int acc_cols_of<RBar>(const TcMat&) { return 128; }
 template <> int acc_cols_of<Update>(const TcMat&) { return 128; }
