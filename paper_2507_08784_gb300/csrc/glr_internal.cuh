@@ -312,14 +312,16 @@ struct BjacMat {
     int n, round;
     const float* H; float* H2;
     const float* V; float* V2;
-    const float* J;
-    int tile0h, tile0v;
+    float* J;
+    int tile0h, tile0v, tile0p;
 };
 struct BjacGroup {
     int nmat, tiles_h, tiles_v;
     BjacMat mat[kBjacGroupMax];
 };
 cudaError_t bjac_apply(BjacGroup& g, cudaStream_t st);
+// J_k of every pair of every matrix: one Jacobi sweep on H's 128 x 128 diagonal pair blocks
+cudaError_t bjac_pairs(BjacGroup& g, cudaStream_t st);
 // part[2 (i kBjacNormCtas + c) + {0, 1}]: CTA c's squared diagonal / off-diagonal sums of H_i
 cudaError_t bjac_norms(const BjacGroup& g, float* part, cudaStream_t st);
 cudaError_t bjac_eye(float* V, int n, cudaStream_t st);

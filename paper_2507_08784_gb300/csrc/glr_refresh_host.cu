@@ -260,19 +260,14 @@ int refresh_exact_blocked(std::vector<glr_handle*>& hs) {
             act.erase(std::remove_if(act.begin(), act.end(), [](State* S) { return S->done; }), act.end());
             if (act.empty()) break;
             for (int round = 0; round < m - 1; ++round) {
-                EigGroup eg{};
-                eg.max_sweeps = 1;
-                for (State* S : act)
-                    for (int k = 0; k < P; ++k) {
-                        EigMat& E = eg.mat[eg.nmat++];
-                        E.n = 128; E.tol = 0.f; E.H = S->H + (size_t)128 * k * (n + 1); E.nparts = 1; E.ld = n;
-                        E.V = S->h->bjJ + (size_t)k * 16384; E.evals = S->h->bjev + 128 * k; E.sweeps = nullptr;
-                        if (eg.nmat == kEigGroupMax) {
-                            GLR_LAUNCH(h0, 1, eig_tmem_group(eg, s0));
-                            eg.nmat = 0;
-                        }
+                for (size_t c0 = 0; c0 < act.size(); c0 += kBjacGroupMax) {
+                    BjacGroup g{};
+                    for (size_t c = c0; c < act.size() && c < c0 + kBjacGroupMax; ++c) {
+                        BjacMat& M = g.mat[g.nmat++];
+                        M.n = n; M.H = act[c]->H; M.J = act[c]->h->bjJ;
                     }
-                if (eg.nmat) GLR_LAUNCH(h0, 1, eig_tmem_group(eg, s0));
+                    GLR_LAUNCH(h0, 1, bjac_pairs(g, s0));
+                }
                 for (size_t c0 = 0; c0 < act.size(); c0 += kBjacGroupMax) {
                     BjacGroup g{};
                     for (size_t c = c0; c < act.size() && c < c0 + kBjacGroupMax; ++c) {

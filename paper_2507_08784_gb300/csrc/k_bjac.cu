@@ -7,9 +7,10 @@
 // slot per round, so that every two blocks meet once in m - 1 rounds, one sweep), and the pairs
 // of a round are stored next to each other: pair k holds rows and columns 128 k .. 128 k + 127.
 // A round
-//   1. takes each pair's 128 x 128 diagonal block S_k and forms J_k, one cyclic sweep of scalar
-//      Jacobi on S_k started from the identity (eig_tmem_kernel with one sweep), so that J_k
-//      stays close to the identity and no reordering inside the pair is needed;
+//   1. takes each pair's 128 x 128 diagonal block S_k and forms J_k, one sweep of parallel cyclic
+//      scalar Jacobi on S_k started from the identity (bjac_pair_kernel; the rotation formula
+//      and circle ordering of the k x k eigen-solver), so that J_k stays close to the identity and
+//      no reordering inside the pair is needed;
 //   2. applies the block-diagonal J = diag(J_k): H <- J^T H J (each 128 x 128 pair block
 //      J_i^T H_ij J_j, the upper ones formed and mirrored) and V <- V J, writing every 64-block
 //      straight to its place in the next round's storage order;
@@ -207,6 +208,120 @@ __global__ void __launch_bounds__(256) bjac_norms_kernel(const __grid_constant__
     }
 }
 
+// One sweep of parallel cyclic two-sided Jacobi on the 128 x 128 diagonal pair block S_k of H,
+// from W = I: 127 rounds of 64 disjoint rotations (circle ordering; Golub & Van Loan sym.schur2),
+// each round's rotations formed from the round's own 2 x 2 diagonal blocks, then S <- R^T S R and
+// W <- W R in one barrier-separated phase.  S is packed (upper triangle by rows), W padded to 129
+// columns; J_k = W is written row-major.  512 threads, two CTAs per SM.
+constexpr int PT = 512;
+constexpr int PN = 128, PH = 64, PLD = 129;
+constexpr int kPairItems = PH * (PH + 1) / 2;                 // 2 x 2 blocks (bi <= bj) of a round
+constexpr size_t kPairSmem = sizeof(float) * (PN * (PN + 1) / 2 + PN * PLD);
+
+__device__ __forceinline__ int pcircle(int x) { return 1 + ((x % (PN - 1)) + (PN - 1)) % (PN - 1); }
+
+__global__ void __launch_bounds__(PT, 2) bjac_pair_kernel(const __grid_constant__ BjacGroup g) {
+    extern __shared__ float psm[];
+    float* Ss = psm;                                   // packed upper triangle: (r, c >= r) at off[r] + c
+    float* Ws = psm + PN * (PN + 1) / 2;               // W[a][j] at a PLD + j
+    __shared__ int off[PN + 1];
+    __shared__ int4 spq[PH];
+    __shared__ float2 scs[PH];
+    int mi = 0;
+    while (mi + 1 < g.nmat && g.mat[mi + 1].tile0p <= (int)blockIdx.x) ++mi;
+    const BjacMat& M = g.mat[mi];
+    const int n = M.n, k = blockIdx.x - M.tile0p, t = threadIdx.x;
+    const float* S0 = M.H + (int64_t)(PN * k) * (n + 1);
+    for (int r = t; r <= PN; r += PT) off[r] = r * PN - r * (r + 1) / 2;
+    __syncthreads();
+    for (int e = t; e < PN * PN; e += PT) {
+        const int r = e >> 7, c = e & 127;
+        if (c >= r) Ss[off[r] + c] = S0[(int64_t)r * n + c];
+        Ws[r * PLD + c] = r == c ? 1.f : 0.f;
+    }
+    // this thread's 2 x 2 blocks: block row i folded with block row PH - 1 - i (equal counts)
+    constexpr int kItems = (kPairItems + PT - 1) / PT;
+    int myblk[kItems];
+#pragma unroll
+    for (int u = 0; u < kItems; ++u) {
+        const int e = t + u * PT;
+        myblk[u] = -1;
+        if (e < kPairItems) {
+            const int fr = e / (PH + 1), tt = e - fr * (PH + 1);
+            int bi, bj;
+            if (tt < PH - fr) { bi = fr; bj = fr + tt; }
+            else { bi = PH - 1 - fr; bj = bi + (tt - (PH - fr)); }
+            myblk[u] = bi | (bj << 16);
+        }
+    }
+    const int wa = t & (PN - 1), wj0 = t >> 7;         // W: row wa, rotations wj0, wj0 + 4, ...
+    __syncthreads();
+    for (int rd = 0; rd < PN - 1; ++rd) {
+        if (t < PH) {
+            int p = (t == 0) ? 0 : pcircle(rd + t);
+            int q = (t == 0) ? pcircle(rd) : pcircle(rd - t);
+            if (p > q) { const int tmp = p; p = q; q = tmp; }
+            float c = 1.f, s = 0.f;
+            const float hpq = Ss[off[p] + q], hpp = Ss[off[p] + p], hqq = Ss[off[q] + q];
+            if (fabsf(hpq) > 1e-30f && fabsf(hpq) > 1e-9f * sqrtf(fabsf(hpp * hqq))) {
+                const float theta = (hqq - hpp) / (2.f * hpq);
+                float tt;
+                if (fabsf(theta) > 1e15f) tt = 0.5f / theta;
+                else tt = copysignf(1.f, theta) / (fabsf(theta) + sqrtf(theta * theta + 1.f));
+                c = 1.f / sqrtf(tt * tt + 1.f);
+                s = tt * c;
+            }
+            spq[t] = make_int4(p, q, off[p], off[q]);
+            scs[t] = make_float2(c, s);
+        }
+        __syncthreads();
+#pragma unroll
+        for (int u = 0; u < kItems; ++u) {              // S <- R^T S R, 2 x 2 block by block
+            if (myblk[u] < 0) continue;
+            const int bi = myblk[u] & 0xFFFF, bj = myblk[u] >> 16;
+            const float2 rci = scs[bi], rcj = scs[bj];
+            const float ci = rci.x, si = rci.y, cj = rcj.x, sj = rcj.y;
+            if (si == 0.f && sj == 0.f) continue;
+            const int4 pi4 = spq[bi], pj4 = spq[bj];
+            const int pi = pi4.x, qi = pi4.y, pj = pj4.x, qj = pj4.y;
+            if (bi == bj) {
+                const int i00 = pi4.z + pi, i01 = pi4.z + qi, i11 = pi4.w + qi;
+                const float h00 = Ss[i00], h01 = Ss[i01], h11 = Ss[i11];
+                const float a00 = ci * h00 - si * h01, a01 = ci * h01 - si * h11;
+                const float a10 = si * h00 + ci * h01, a11 = si * h01 + ci * h11;
+                Ss[i00] = cj * a00 - sj * a01;
+                Ss[i11] = sj * a10 + cj * a11;
+                Ss[i01] = 0.f;
+                continue;
+            }
+            const int i00 = pi <= pj ? pi4.z + pj : pj4.z + pi;
+            const int i01 = pi <= qj ? pi4.z + qj : pj4.w + pi;
+            const int i10 = qi <= pj ? pi4.w + pj : pj4.z + qi;
+            const int i11 = qi <= qj ? pi4.w + qj : pj4.w + qi;
+            const float h00 = Ss[i00], h01 = Ss[i01], h10 = Ss[i10], h11 = Ss[i11];
+            const float a00 = ci * h00 - si * h10, a01 = ci * h01 - si * h11;
+            const float a10 = si * h00 + ci * h10, a11 = si * h01 + ci * h11;
+            Ss[i00] = cj * a00 - sj * a01;
+            Ss[i01] = sj * a00 + cj * a01;
+            Ss[i10] = cj * a10 - sj * a11;
+            Ss[i11] = sj * a10 + cj * a11;
+        }
+        float* wr = Ws + wa * PLD;                      // W <- W R
+#pragma unroll 4
+        for (int j = wj0; j < PH; j += PT / PN) {
+            const float2 cs = scs[j];
+            if (cs.y == 0.f) continue;
+            const int4 pq = spq[j];
+            const float vp = wr[pq.x], vq = wr[pq.y];
+            wr[pq.x] = cs.x * vp - cs.y * vq;
+            wr[pq.y] = cs.y * vp + cs.x * vq;
+        }
+        __syncthreads();
+    }
+    float* J = M.J + (int64_t)k * PN * PN;
+    for (int e = t; e < PN * PN; e += PT) J[e] = Ws[(e >> 7) * PLD + (e & 127)];
+}
+
 __global__ void count_flag_kernel(int* flag, int v) { atomicAdd(flag, v); }
 
 __global__ void bjac_eye_kernel(float* V, int n) {
@@ -237,6 +352,21 @@ cudaError_t bjac_apply(BjacGroup& g, cudaStream_t st) {
     bjac_apply_h_kernel<<<g.tiles_h, BT, kApplyHSmem, st>>>(g);
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
     bjac_apply_v_kernel<<<g.tiles_v, BT, kApplyVSmem, st>>>(g);
+    return cudaGetLastError();
+}
+
+cudaError_t bjac_pairs(BjacGroup& g, cudaStream_t st) {
+    if (g.nmat <= 0) return cudaSuccess;
+    int tiles = 0;
+    for (int i = 0; i < g.nmat; ++i) {
+        BjacMat& M = g.mat[i];
+        if (M.n < 256 || M.n % 128 || M.n > kBjacMaxN) return cudaErrorInvalidValue;
+        M.tile0p = tiles;
+        tiles += M.n / 128;
+    }
+    cudaError_t e = cudaFuncSetAttribute(bjac_pair_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kPairSmem);
+    if (e != cudaSuccess) return e;
+    bjac_pair_kernel<<<tiles, PT, kPairSmem, st>>>(g);
     return cudaGetLastError();
 }
 
