@@ -19,6 +19,7 @@ from __future__ import annotations
 
 import argparse
 import hashlib
+import dataclasses
 import json
 import math
 import os
@@ -48,7 +49,7 @@ def paper_exact_config():
     Adam, r = 128) with basis_rank = 0: the paper-exact basis of Eq. SVD-P1, refreshed by the
     blocked Jacobi eigen-solve, its scores the dense U^T Mbar."""
     base = W.config("cfg5_llama_d4096")
-    return W.config("cfg5_llama_d4096", name=PAPER_EXACT, shapes=base.shapes[:7], basis_rank=0)
+    return dataclasses.replace(base, name=PAPER_EXACT, shapes=base.shapes[:7], basis_rank=0)
 
 
 def _peaks():
@@ -479,6 +480,27 @@ def bench_paper_exact(torch, glr, K, Wm, ctx, hbm_peak):
     return out
 
 
+def ncu_case_exact():
+    """One 4096 x 4096 matrix of the headline stack with the full basis (basis_rank = 0) for 4
+    steps: step 0 is the blocked Jacobi refresh (about 15 sweeps of 63 rounds, each round one pair
+    sweep launch and two block-product launches), steps 1-3 run the dense scores (LambdaU)."""
+    import torch
+    import paper_2507_08784_gb300 as glr
+    base = W.config(WORKLOAD)
+    cfg = dataclasses.replace(base, shapes=base.shapes[:1], basis_rank=0)
+    prob = W.make_problem(cfg)
+    gs = [W.gradients_torch(prob, 0, t) for t in range(2)]
+    hs = make_handles(glr, cfg, 0)
+    X = [torch.zeros(*cfg.shapes[0], device="cuda")]
+    for t in range(4):
+        glr.glr_step_group(hs, [gs[t % 2]], X)
+    torch.cuda.synchronize()
+    print(json.dumps({"ncu_case": "paper_exact", "shape": cfg.shapes[0], "N": cfg.N, "r": cfg.r,
+                      "sweeps": hs[0].stats()["last_refresh_sweeps"], "path": hs[0].stats()["path"]}))
+    hs[0].close()
+    return 0
+
+
 def ncu_case(refresh=False, stress=False):
     """One 4096 x 4096 matrix of the headline stack for 4 steps (about 1.1 GB of state): the
     compose launch of step 2 (index 2 among compose launches) is a full one; with refresh, a
@@ -527,7 +549,7 @@ def main():
                     help="time the headline workload only (no extra workloads, no e2e, no CPU baseline)")
     ap.add_argument("--e2e-steps", type=int, default=5)
     ap.add_argument("--refresh-reps", type=int, default=3)
-    ap.add_argument("--ncu-case", nargs="?", const="steps", choices=["steps", "refresh", "stress"],
+    ap.add_argument("--ncu-case", nargs="?", const="steps", choices=["steps", "refresh", "stress", "exact"],
                     help="a small case for kernel captures: one 4096 x 4096 matrix of the headline stack "
                          "(N = 4, r = 128, k = 256, bf16, Adam), 4 steps: refresh, reset, then two full "
                          "steps; 'refresh' adds a fifth step forced to refresh; 'stress' runs the refresh-stress "
@@ -537,6 +559,8 @@ def main():
         ap.error("--warmup must be >= 3")
     if args.impl == "reference":
         return run_reference(args)
+    if args.ncu_case == "exact":
+        return ncu_case_exact()
     if args.ncu_case:
         return ncu_case(args.ncu_case == "refresh", args.ncu_case == "stress")
 
