@@ -212,14 +212,17 @@ int glr_step_host(glr_handle* h, const void* const* G_host, float* X, float* X_h
 
 /* glr_step_group with host gradients, for a training loop that produces them on the host:
  * G_host[j][i] is node i's gradient of handles[j] (host memory, m x n of the gradient dtype;
- * pinned memory makes the copies asynchronous).  Each handle copies them on its own copy
- * stream into one of two library-owned device staging buffers (alternating per call, so the
- * copies of one call overlap the compute of the previous one) and the step waits for them on
- * `stream`.  X[j] is the device weight matrix (updated in place); when X_host_out is not NULL
- * and X_host_out[j] is not NULL the updated X[j] is copied back to it on `stream`.  The call
- * only enqueues work: X_host_out holds the result once `stream` has passed this step
- * (synchronise it or record an event), and the gradient host buffers must stay valid until
- * then.  Errors as glr_step_group.                                                         */
+ * pinned memory makes the copies asynchronous).  They are copied on one library copy stream
+ * (the first handle's) into one of two library-owned device staging buffers per handle
+ * (alternating per call, so the copies of one call overlap the compute of the previous one) and
+ * the step waits for them on `stream`.  X[j] is the device weight matrix (updated in place);
+ * when X_host_out is not NULL and X_host_out[j] is not NULL the updated X[j] is copied back to
+ * it after the step on a second library stream (the first handle's read-back stream, so the
+ * next call's gradient copies and compute run beside it; only that call's update, which
+ * rewrites X, waits for it).  The call only enqueues work: X_host_out holds the
+ * result after cudaDeviceSynchronize, or once `stream` has passed the next call on the same
+ * handles; the gradient host buffers must stay valid until `stream` has passed this step.
+ * Errors as glr_step_group.                                                                 */
 int glr_step_group_host(glr_handle* const* handles, int32_t count, const void* const* const* G_host,
                         float* const* X, float* const* X_host_out, void* stream);
 

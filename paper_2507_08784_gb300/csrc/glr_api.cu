@@ -484,6 +484,9 @@ int glr_destroy(glr_handle* h) {
     if (h->cdone) cudaEventDestroy(h->cdone);
     for (cudaEvent_t e : h->sfree) if (e) cudaEventDestroy(e);
     if (h->cstream) cudaStreamDestroy(h->cstream);
+    if (h->xready) cudaEventDestroy(h->xready);
+    if (h->xdone) cudaEventDestroy(h->xdone);
+    if (h->xstream) cudaStreamDestroy(h->xstream);
     for (cublasHandle_t c : h->cb) if (c) cublasDestroy(c);
     free_all(h);
     delete h;
@@ -1023,6 +1026,12 @@ int step_group(std::vector<StepPlan>& plans, cudaStream_t st) {
     if (!tcl.empty() && (rc = tcl_lambda(tcl, st)) != GLR_OK) return rc;
     for (glr_handle* h : refreshing) GLR_CK(h, cudaStreamWaitEvent(st, h->rdone, 0));
     if ((rc = select_P_grouped(plans, st)) != GLR_OK) return rc;
+    // X is written from here on: a read-back of the previous step's X (glr_step_group_host) ends first
+    for (StepPlan& p : plans)
+        if (p.h->x_pending) {
+            GLR_CK(p.h, cudaStreamWaitEvent(st, p.h->xdone, 0));
+            p.h->x_pending = false;
+        }
     if (!tcl.empty() && (rc = tcl_project_update(tcl, st)) != GLR_OK) return rc;
     std::vector<StepPlan*> streamed, strips;
     for (StepPlan* p : fused) {
@@ -1110,6 +1119,10 @@ int dp_finish(glr_handle* h, float* X, cudaStream_t st) {
     StepPlan& p = plans[0];
     p.X = X;
     std::vector<StepPlan*> v{&p};
+    if (h->x_pending) {                        // a host read-back of X still in flight
+        GLR_CK(h, cudaStreamWaitEvent(st, h->xdone, 0));
+        h->x_pending = false;
+    }
     const int rc = tcl_update(v, st);
     if (rc != GLR_OK) return rc;
     finish_step(p);
@@ -1213,12 +1226,14 @@ int glr_step_group_host(glr_handle* const* handles, int32_t count, const void* c
     std::vector<std::vector<const void*>> Gd(count);
     std::vector<const void* const*> Garr(count);
     std::vector<int> parity(count);
-    for (int j = 0; j < count; ++j) {
+    for (int j = 0; j < count; ++j) {           // staging, streams and events on first use
         glr_handle* h = handles[j];
         if (!h) return fail(nullptr, GLR_EINVAL, "null handle in the group%s");
         if (!G_host[j] || !X[j]) return fail(h, GLR_EINVAL, "null host gradient array or X%s");
-        const size_t bytes = static_cast<size_t>(h->m) * h->n * h->gsize;
+        for (int i = 0; i < h->N; ++i)
+            if (!G_host[j][i]) return fail(h, GLR_EINVAL, "host gradient %s is null", std::to_string(i).c_str());
         if (!h->cstream) {
+            const size_t bytes = static_cast<size_t>(h->m) * h->n * h->gsize;
             for (int b = 0; b < 2; ++b) {
                 char* p = nullptr;
                 const int rc = alloc(h, &p, bytes * h->N);
@@ -1228,37 +1243,59 @@ int glr_step_group_host(glr_handle* const* handles, int32_t count, const void* c
             if (cudaStreamCreateWithFlags(&h->cstream, cudaStreamNonBlocking) != cudaSuccess ||
                 cudaEventCreateWithFlags(&h->cdone, cudaEventDisableTiming) != cudaSuccess ||
                 cudaEventCreateWithFlags(&h->sfree[0], cudaEventDisableTiming) != cudaSuccess ||
-                cudaEventCreateWithFlags(&h->sfree[1], cudaEventDisableTiming) != cudaSuccess)
-                return fail(h, GLR_ECUDA, "could not create the host-copy stream%s");
+                cudaEventCreateWithFlags(&h->sfree[1], cudaEventDisableTiming) != cudaSuccess ||
+                cudaStreamCreateWithFlags(&h->xstream, cudaStreamNonBlocking) != cudaSuccess ||
+                cudaEventCreateWithFlags(&h->xready, cudaEventDisableTiming) != cudaSuccess ||
+                cudaEventCreateWithFlags(&h->xdone, cudaEventDisableTiming) != cudaSuccess)
+                return fail(h, GLR_ECUDA, "could not create the host-copy streams%s");
             // alloc's zero fill runs on the legacy default stream, which the non-blocking copy
             // stream does not wait for: finish it before the first copy
             GLR_CK(h, cudaDeviceSynchronize());
         }
+    }
+    // every gradient copy of the call on one stream (the first handle's) and every read-back on
+    // another: one stream per direction keeps the two directions on separate copy engines, so
+    // the read-back of this step runs beside the next step's gradient copies
+    glr_handle* h0 = handles[0];
+    cudaStream_t cs = h0->cstream, xs = h0->xstream;
+    for (int j = 0; j < count; ++j) {
+        glr_handle* h = handles[j];
+        const size_t bytes = static_cast<size_t>(h->m) * h->n * h->gsize;
         const int b = h->host_parity;
         parity[j] = b;
         // buffer b was last read by this handle's step two calls ago
-        if (h->sfree_set[b]) GLR_CK(h, cudaStreamWaitEvent(h->cstream, h->sfree[b], 0));
+        if (h->sfree_set[b]) GLR_CK(h, cudaStreamWaitEvent(cs, h->sfree[b], 0));
         Gd[j].resize(h->N);
         for (int i = 0; i < h->N; ++i) {
-            if (!G_host[j][i]) return fail(h, GLR_EINVAL, "host gradient %s is null", std::to_string(i).c_str());
             char* dst = static_cast<char*>(h->Gstage2[b]) + bytes * i;
-            GLR_CK(h, cudaMemcpyAsync(dst, G_host[j][i], bytes, cudaMemcpyHostToDevice, h->cstream));
+            GLR_CK(h, cudaMemcpyAsync(dst, G_host[j][i], bytes, cudaMemcpyHostToDevice, cs));
             Gd[j][i] = dst;
         }
-        GLR_CK(h, cudaEventRecord(h->cdone, h->cstream));
-        GLR_CK(h, cudaStreamWaitEvent(st, h->cdone, 0));
         Garr[j] = Gd[j].data();
     }
+    GLR_CK(h0, cudaEventRecord(h0->cdone, cs));
+    GLR_CK(h0, cudaStreamWaitEvent(st, h0->cdone, 0));
     const int rc = glr_step_group(handles, count, Garr.data(), X, stream);
     if (rc != GLR_OK) return rc;
+    bool out = false;
     for (int j = 0; j < count; ++j) {
         glr_handle* h = handles[j];
         const int b = parity[j];
         GLR_CK(h, cudaEventRecord(h->sfree[b], st));
         h->sfree_set[b] = true;
         h->host_parity = b ^ 1;
-        if (X_host_out && X_host_out[j])
-            GLR_CK(h, cudaMemcpyAsync(X_host_out[j], X[j], sizeof(float) * h->m * h->n, cudaMemcpyDeviceToHost, st));
+        out = out || (X_host_out && X_host_out[j]);
+    }
+    if (!out) return GLR_OK;
+    // the read-back after the step; only the next step's update (which rewrites X) waits for it
+    GLR_CK(h0, cudaEventRecord(h0->xready, st));
+    GLR_CK(h0, cudaStreamWaitEvent(xs, h0->xready, 0));
+    for (int j = 0; j < count; ++j) {
+        glr_handle* h = handles[j];
+        if (!X_host_out[j]) continue;
+        GLR_CK(h, cudaMemcpyAsync(X_host_out[j], X[j], sizeof(float) * h->m * h->n, cudaMemcpyDeviceToHost, xs));
+        GLR_CK(h, cudaEventRecord(h->xdone, xs));
+        h->x_pending = true;
     }
     return GLR_OK;
 }

@@ -90,6 +90,11 @@ struct glr_handle {
     cudaEvent_t cdone = nullptr, sfree[2] = {nullptr, nullptr};
     bool sfree_set[2] = {false, false};
     int host_parity = 0;
+    // the read-back of X to the host (glr_step_group_host) on its own stream: xready marks X final
+    // on the step's stream, xdone the copy's end; x_pending makes the next step's update wait
+    cudaStream_t xstream = nullptr;
+    cudaEvent_t xready = nullptr, xdone = nullptr;
+    bool x_pending = false;
     // host state
     int64_t t = 0, refreshes = 0, comm = 0, state_bytes = 0, period_start = 0;
     bool e_zero = true, force_refresh = false, last_uncompressed = true, basis_from_user = false;
