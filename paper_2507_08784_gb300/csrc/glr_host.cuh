@@ -66,7 +66,9 @@ struct glr_handle {
     // the full basis on the tcgen05 path (m' > 1024): U^T rounded to TF32 (the score operand, part
     // of the state), and the blocked Jacobi's scratch (not checkpointed): the second V buffer, the
     // pair rotations (m' x 128), the pair solver's eigenvalues, the norm partials, the sweep count
-    float *UT = nullptr, *Vbuf2 = nullptr, *bjJ = nullptr, *bjev = nullptr, *bjpart = nullptr;
+    float *UT = nullptr, *Vbuf2 = nullptr, *bjJ = nullptr, *bjpart = nullptr;
+    // ... and the TF32 low parts of the rotations' operands: J^T, H, T^T (in jwork) and both V buffers
+    float *bjJlo = nullptr, *Hlo = nullptr, *Ttlo = nullptr, *Vlo = nullptr, *V2lo = nullptr;
     int bj_sweeps = 0, numeric_failures_host = 0;
     // a data-parallel step in progress (glr_dp_begin / glr_dp_select / glr_dp_finish): 0 idle,
     // 1 begun, 2 selected; the step's plan and the caller's gradient pointers
@@ -196,7 +198,8 @@ int gemm(glr_handle* h, const GemmDesc& d, cudaStream_t st);
 enum TcMap { kMapBt, kMapPT0, kMapPT1, kMapP0, kMapP1, kMapRwT, kMapMbarT, kMapYT, kMapYt, kMapWT, kMapY, kMapYtJn,
              kMapYtJm, kMapRbarT, kMapBtD, kMapMbarL, kMapMbarU, kMapMo, kMapVo,
              kMapMrow, kMapMlo, kMapQTtA, kMapQTtB, kMapZTtA, kMapZTtB, kMapQA, kMapQA1, kMapZA, kMapLinv,
-             kMapUT, kMapMbar3, kNumTcMaps };
+             kMapUT, kMapMbar3, kMapBjH, kMapBjHlo, kMapBjT, kMapBjTlo, kMapBjV0, kMapBjV0lo, kMapBjV1, kMapBjV1lo,
+             kMapBjJ, kMapBjJlo, kNumTcMaps };
 // After the fixed maps: two slots of N gradient maps, then two slots for X (the caller's buffers,
 // re-described only when a pointer changes).
 const CUtensorMap* tcl_grad_maps(glr_handle* h, const void* const* G, cudaStream_t st, int* rc);

@@ -302,25 +302,40 @@ struct EigGroup {
 };
 cudaError_t eig_tmem_group(const EigGroup& g, cudaStream_t st);
 
-// Blocked Jacobi rounds of the full-basis refresh above m' = 1024 (k_bjac.cu).  H, V: this
-// round's n x n matrices in the round's storage order; H2, V2 receive J^T H J and V J in the next
-// round's order; J: the round's n / 128 pair rotations, 128 x 128 row-major each.
+// The blocked Jacobi's round-robin tournament over m blocks of 64 indices (circle method: block 0
+// fixed, the others one slot further each round; slots s and m - 1 - s pair up and are stored at
+// positions 2 s, 2 s + 1): the storage position of block x in round rd, the block at position p,
+// and where the data at position p of round rd goes for round rd + 1.
+__device__ __forceinline__ int bjac_position_of(int x, int m, int rd) {
+    const int s = x == 0 ? 0 : 1 + ((x - 1 - rd) % (m - 1) + (m - 1)) % (m - 1);
+    return s < m / 2 ? 2 * s : 2 * (m - 1 - s) + 1;
+}
+__device__ __forceinline__ int bjac_block_at(int p, int m, int rd) {
+    const int s = (p & 1) ? m - 1 - (p >> 1) : (p >> 1);
+    return s == 0 ? 0 : 1 + (s - 1 + rd) % (m - 1);
+}
+__device__ __forceinline__ int bjac_dest_of(int p, int m, int rd) {
+    return bjac_position_of(bjac_block_at(p, m, rd), m, (rd + 1) % (m - 1));
+}
+
+// Blocked Jacobi rounds of the full-basis refresh above m' = 1024 (k_bjac.cu; the rotations are
+// tc_kernel<BjacMul> in k_tc.cu).  H: this round's n x n matrix in the round's storage order;
+// J, Jlo: the round's n / 128 pair rotations as J_k^T (128 x 128 row-major each) and their TF32
+// low parts.
 constexpr int kBjacMaxN = 4096;
 constexpr int kBjacGroupMax = 32;
 constexpr int kBjacNormCtas = 64;
 struct BjacMat {
-    int n, round;
-    const float* H; float* H2;
-    const float* V; float* V2;
-    float* J;
-    int tile0h, tile0v, tile0p;
+    int n;
+    const float* H;
+    float* J; float* Jlo;
+    int tile0p;
 };
 struct BjacGroup {
-    int nmat, tiles_h, tiles_v;
+    int nmat;
     BjacMat mat[kBjacGroupMax];
 };
-cudaError_t bjac_apply(BjacGroup& g, cudaStream_t st);
-// J_k of every pair of every matrix: one Jacobi sweep on H's 128 x 128 diagonal pair blocks
+// J_k^T of every pair of every matrix: one Jacobi sweep on H's 128 x 128 diagonal pair blocks
 cudaError_t bjac_pairs(BjacGroup& g, cudaStream_t st);
 // part[2 (i kBjacNormCtas + c) + {0, 1}]: CTA c's squared diagonal / off-diagonal sums of H_i
 cudaError_t bjac_norms(const BjacGroup& g, float* part, cudaStream_t st);
@@ -489,6 +504,11 @@ struct TcMat {
     int rows, ld_out, split, chunk;
     float* out; float* outT;
     float* MbarRow;                                   // Compose on a refresh step: Mbar row-major too
+    // BjacMul (the blocked Jacobi's rotations): the second B operand (B's TF32 low parts; mA2 holds
+    // A's), the output mode and the tournament round, the output's low parts
+    const CUtensorMap* mB2;
+    int bjmode, bjround;
+    float* out_lo;
 };
 struct TcGroup {
     int nmat, total_tiles;
@@ -505,6 +525,8 @@ cudaError_t launch_compose(TcGroup& g, cudaStream_t st);
 cudaError_t launch_wbar(TcGroup& g, cudaStream_t st);
 cudaError_t launch_lambda(TcGroup& g, cudaStream_t st);
 cudaError_t launch_lambda_u(TcGroup& g, cudaStream_t st);   // full basis: the scores from U^T Mbar
+// The blocked Jacobi's rotations in the split TF32 form (k_tc.cu, BjacMul; modes in k_tc.cu)
+cudaError_t launch_bjac(TcGroup& g, cudaStream_t st);
 cudaError_t launch_pbuild(TcGroup& g, cudaStream_t st);
 cudaError_t launch_rbar(TcGroup& g, cudaStream_t st);
 cudaError_t launch_update(TcGroup& g, cudaStream_t st);

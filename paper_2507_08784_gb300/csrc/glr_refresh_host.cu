@@ -184,9 +184,11 @@ int refresh_exact_grouped(std::vector<glr_handle*>& hs) {
 // H = Mbar Mbar^T by the grouped FFMA product (Mbar is column-major on the tcgen05 path), V = I,
 // then the blocked Jacobi rounds of every matrix of the same size together, one sweep at a time,
 // each sweep opened by the norm check (summed on the host in a fixed order, so that the decision
-// does not depend on the grouping); finally each handle's sorted, sign-fixed U and its TF32
-// transpose.  A matrix that has not converged after kBjacMaxSweeps sweeps keeps its last basis
-// and counts a numeric failure (GLR_ENUMERIC from glr_get_stats).
+// does not depend on the grouping).  A round: the pair sweeps (J_k^T and its low part), then the
+// three split-TF32 products of tc_kernel<BjacMul>: T^T = (H J)^T, H <- T^T J, V' <- V J (V and
+// V' trade buffers).  Finally each handle's sorted, sign-fixed U and its TF32 transpose.  A matrix
+// that has not converged after kBjacMaxSweeps sweeps keeps its last basis and counts a numeric
+// failure (GLR_ENUMERIC from glr_get_stats).
 constexpr int kBjacMaxSweeps = 30;
 
 int refresh_exact_blocked(std::vector<glr_handle*>& hs) {
@@ -198,7 +200,7 @@ int refresh_exact_blocked(std::vector<glr_handle*>& hs) {
         GLR_CK(h0, cudaStreamWaitEvent(s0, h->rpow, 0));
     }
     PhaseScope ps(h0, GLR_PH_REFRESH, s0);
-    {   // H = Mbar Mbar^T: Mbar^T is n' x m' row-major
+    {   // H = Mbar Mbar^T (Mbar^T is n' x m' row-major) and its low part; V = I, V_lo = 0
         GemmGroup gg{};
         auto flush = [&]() -> int {
             if (gg.nmat) GLR_LAUNCH(h0, 1, gemm_group_f32(gg, s0));
@@ -213,14 +215,20 @@ int refresh_exact_blocked(std::vector<glr_handle*>& hs) {
             G.B = h->Mbar; G.sBp = h->mp; G.sBj = 1;
             G.C = h->Hbuf; G.sCi = h->mp; G.sCj = 1;
             if (gg.nmat == 64 && flush() != GLR_OK) return GLR_ECUDA;
-            GLR_LAUNCH(h, 1, bjac_eye(h->Vbuf, h->mp, s0));
         }
         if (flush() != GLR_OK) return GLR_ECUDA;
+        for (glr_handle* h : hs) {
+            const int64_t nn = (int64_t)h->mp * h->mp;
+            GLR_LAUNCH(h, 1, tc::split_lo(h->Hbuf, h->Hlo, nn, s0));
+            GLR_LAUNCH(h, 1, bjac_eye(h->Vbuf, h->mp, s0));
+            GLR_CK(h, cudaMemsetAsync(h->Vlo, 0, sizeof(float) * nn, s0));
+        }
     }
-    struct State { glr_handle* h; float *H, *H2, *V, *V2; int rd; bool done; };
+    struct State { glr_handle* h; int vpar, rd; bool done; };
     std::vector<State> all;
-    for (glr_handle* h : hs) all.push_back(State{h, h->Hbuf, h->jwork, h->Vbuf, h->Vbuf2, 0, false});
+    for (glr_handle* h : hs) all.push_back(State{h, 0, 0, false});
     std::vector<float> part;
+    static thread_local tc::TcGroup tg;
     for (size_t a0 = 0; a0 < all.size();) {
         // the matrices of one size
         size_t a1 = a0;
@@ -236,7 +244,7 @@ int refresh_exact_blocked(std::vector<glr_handle*>& hs) {
                 BjacGroup g{};
                 for (size_t c = c0; c < act.size() && c < c0 + kBjacGroupMax; ++c) {
                     BjacMat& M = g.mat[g.nmat++];
-                    M.n = n; M.H = act[c]->H;
+                    M.n = n; M.H = act[c]->h->Hbuf;
                 }
                 GLR_LAUNCH(h0, 1, bjac_norms(g, h0->bjpart, s0));
                 part.resize((size_t)2 * kBjacNormCtas * g.nmat);
@@ -264,22 +272,40 @@ int refresh_exact_blocked(std::vector<glr_handle*>& hs) {
                     BjacGroup g{};
                     for (size_t c = c0; c < act.size() && c < c0 + kBjacGroupMax; ++c) {
                         BjacMat& M = g.mat[g.nmat++];
-                        M.n = n; M.H = act[c]->H; M.J = act[c]->h->bjJ;
+                        M.n = n; M.H = act[c]->h->Hbuf; M.J = act[c]->h->bjJ; M.Jlo = act[c]->h->bjJlo;
                     }
                     GLR_LAUNCH(h0, 1, bjac_pairs(g, s0));
                 }
-                for (size_t c0 = 0; c0 < act.size(); c0 += kBjacGroupMax) {
-                    BjacGroup g{};
-                    for (size_t c = c0; c < act.size() && c < c0 + kBjacGroupMax; ++c) {
-                        State* S = act[c];
-                        BjacMat& M = g.mat[g.nmat++];
-                        M.n = n; M.round = S->rd; M.H = S->H; M.H2 = S->H2; M.V = S->V; M.V2 = S->V2; M.J = S->h->bjJ;
+                for (int mode = 0; mode < 3; ++mode) {
+                    for (size_t c0 = 0; c0 < act.size(); c0 += tc::kTcGroupMax) {
+                        tg.nmat = 0; tg.total_tiles = 0; tg.err = h0->dflags + 2;
+                        for (size_t c = c0; c < act.size() && c < c0 + tc::kTcGroupMax; ++c) {
+                            const State* S = act[c];
+                            glr_handle* h = S->h;
+                            tc::TcMat M{};
+                            M.mp = n; M.ntiles = P * P; M.tile0 = tg.total_tiles; M.bjmode = mode; M.bjround = S->rd;
+                            const int vin = S->vpar ? kMapBjV1 : kMapBjV0;
+                            if (mode == 0) {
+                                M.mA = tcl_map(h, kMapBjH); M.mA2 = tcl_map(h, kMapBjHlo);
+                                M.mB = tcl_map(h, kMapBjJ); M.mB2 = tcl_map(h, kMapBjJlo);
+                                M.out = h->jwork; M.out_lo = h->Ttlo;
+                            } else if (mode == 1) {
+                                M.mA = tcl_map(h, kMapBjT); M.mA2 = tcl_map(h, kMapBjTlo);
+                                M.mB = tcl_map(h, kMapBjJ); M.mB2 = tcl_map(h, kMapBjJlo);
+                                M.out = h->Hbuf; M.out_lo = h->Hlo;
+                            } else {
+                                M.mA = tcl_map(h, kMapBjJ); M.mA2 = tcl_map(h, kMapBjJlo);
+                                M.mB = tcl_map(h, vin); M.mB2 = tcl_map(h, vin + 1);
+                                M.out = S->vpar ? h->Vbuf : h->Vbuf2; M.out_lo = S->vpar ? h->Vlo : h->V2lo;
+                            }
+                            tg.total_tiles += M.ntiles;
+                            tg.mat[tg.nmat++] = M;
+                        }
+                        GLR_LAUNCH(h0, 1, tc::launch_bjac(tg, s0));
                     }
-                    GLR_LAUNCH(h0, 2, bjac_apply(g, s0));
                 }
                 for (State* S : act) {
-                    std::swap(S->H, S->H2);
-                    std::swap(S->V, S->V2);
+                    S->vpar ^= 1;
                     S->rd = (S->rd + 1) % (m - 1);
                 }
             }
@@ -289,8 +315,8 @@ int refresh_exact_blocked(std::vector<glr_handle*>& hs) {
     for (State& S : all) {
         glr_handle* h = S.h;
         const int n = h->mp;
-        GLR_LAUNCH(h, 1, bjac_diag(S.H, n, h->evals, s0));
-        GLR_LAUNCH(h, 1, sort_fix_basis(h->evals, S.V, n, n, h->U, n, h->evals_sorted, s0));
+        GLR_LAUNCH(h, 1, bjac_diag(h->Hbuf, n, h->evals, s0));
+        GLR_LAUNCH(h, 1, sort_fix_basis(h->evals, S.vpar ? h->Vbuf2 : h->Vbuf, n, n, h->U, n, h->evals_sorted, s0));
         GLR_LAUNCH(h, 1, tc::transpose_round(h->UT, n, h->U, n, n, n, s0));
         GLR_CK(h, cudaMemcpyAsync(h->dflags + 1, &h->bj_sweeps, sizeof(int), cudaMemcpyHostToDevice, s0));
         if (h->numeric_failures_host) {

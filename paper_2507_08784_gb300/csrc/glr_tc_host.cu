@@ -66,7 +66,8 @@ int tcl_maps(glr_handle* h) {
         int rc = GLR_OK;
         auto A = [&](float** p, size_t cnt) { if (rc == GLR_OK) rc = alloc(h, p, cnt); };
         if (h->exact) {
-            A(&h->Vbuf2, mp * mp); A(&h->bjJ, mp * 128); A(&h->bjev, mp);
+            A(&h->Vbuf2, mp * mp); A(&h->bjJ, mp * 128); A(&h->bjJlo, mp * 128);
+            A(&h->Hlo, mp * mp); A(&h->Ttlo, mp * mp); A(&h->Vlo, mp * mp); A(&h->V2lo, mp * mp);
             A(&h->bjpart, (size_t)2 * kBjacNormCtas * kBjacGroupMax);
         } else {
             const size_t nch = (np + tc::kGramChunk - 1) / tc::kGramChunk;
@@ -100,6 +101,12 @@ int tcl_maps(glr_handle* h) {
     if (h->exact) {
         m2(kMapUT, h->UT, mp, mp, mp, 128);                // U^T (TF32), row-major m' x m'
         m3(kMapMbar3, h->Mbar, mp, np, 1, 128);            // Mbar^T as a one-node B^T
+        // the blocked Jacobi's operands (rows of 128, K slices of 32) and their TF32 low parts
+        m2(kMapBjH, h->Hbuf, mp, mp, mp, 128);  m2(kMapBjHlo, h->Hlo, mp, mp, mp, 128);
+        m2(kMapBjT, h->jwork, mp, mp, mp, 128); m2(kMapBjTlo, h->Ttlo, mp, mp, mp, 128);
+        m2(kMapBjV0, h->Vbuf, mp, mp, mp, 128); m2(kMapBjV0lo, h->Vlo, mp, mp, mp, 128);
+        m2(kMapBjV1, h->Vbuf2, mp, mp, mp, 128); m2(kMapBjV1lo, h->V2lo, mp, mp, mp, 128);
+        m2(kMapBjJ, h->bjJ, 128, mp, 128, 128); m2(kMapBjJlo, h->bjJlo, 128, mp, 128, 128);
     } else {
     m2(kMapYT, h->YTk, mp, kp, mp, (uint32_t)kp);          // Y^T: kpad x m'
     m2(kMapYt, h->Yt, k, mp, k, 128);                      // Yt, row-major m' x k

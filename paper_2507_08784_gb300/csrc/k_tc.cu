@@ -697,6 +697,71 @@ struct LambdaU : NoData {
 };
 
 // ------------------------------------------------------------------------------------------
+// BjacMul (the blocked Jacobi of the full-basis refresh, k_bjac.cu): Y = X J_l over the 128
+// columns of pair l, as three products per K slice (A B + A_lo B + A B_lo: the split TF32 form,
+// about as accurate as fp32 FFMA); tile = (128-row block rt, pair l), K = 128.  Modes:
+//   0: A = H rows, B = J_l^T:    D(i, c) = (H J)(i, 128 l + c), written to T^T (row 128 l + c)
+//   1: A = T^T rows, B = J_l^T:  D(r, c) = (T^T J)(r, 128 l + c) = (J^T H J)(r, 128 l + c),
+//      written transposed (the matrix is symmetric) at the next round's rows and columns
+//   2: A = J_l^T, B = V rows:    D(c, r) = (V J)(r, 128 l + c), written to V' at row r and the
+//      next round's column of 128 l + c
+// With these orientations a warp's stores are 128 contiguous bytes.  Each output goes out with
+// its TF32 low part x - trunc_tf32(x), the next product's second operand.
+// ------------------------------------------------------------------------------------------
+struct BjacMul : NoData {
+    static constexpr int kEpi = 16;
+    static __device__ __forceinline__ int nk(const TcGroup&, const Tile&) { return 4; }
+    static __device__ __forceinline__ uint32_t tx_bytes(const TcGroup&, const Tile&, int) { return 4u * 16384u; }
+    static __device__ __forceinline__ void load(const TcGroup& g, const Tile& t, int kc, uint32_t st, uint32_t bar) {
+        const TcMat& M = g.mat[t.mat];
+        const int P = M.mp / 128, rt = t.lt / P, l = t.lt % P;
+        int ax, ay, bx, by;
+        if (M.bjmode < 2) { ax = 128 * l + 32 * kc; ay = 128 * rt; bx = 32 * kc; by = 128 * l; }
+        else { ax = 32 * kc; ay = 128 * l; bx = 128 * l + 32 * kc; by = 128 * rt; }
+        tma_load_2d(st, M.mA, ax, ay, bar);
+        tma_load_2d(st + 16384u, M.mA2, ax, ay, bar);
+        tma_load_2d(st + 32768u, M.mB, bx, by, bar);
+        tma_load_2d(st + 49152u, M.mB2, bx, by, bar);
+    }
+    static __device__ __forceinline__ void mma(const TcGroup&, const Tile&, int kc, uint32_t st, uint32_t d) {
+        mma_slice(d, st, st + 32768u, 128, kc == 0);           // A B
+        mma_slice(d, st + 16384u, st + 32768u, 128, false);    // A_lo B
+        mma_slice(d, st, st + 49152u, 128, false);             // A B_lo
+    }
+    static __device__ __forceinline__ int dest(int x, int m, int rd) {
+        return 64 * bjac_dest_of(x >> 6, m, rd) + (x & 63);
+    }
+    static __device__ __forceinline__ bool epilogue(const TcGroup& g, const Tile& t, uint32_t tl, int warp, int lane,
+                                                    DataRing&) {
+        const TcMat& M = g.mat[t.mat];
+        const int n = M.mp, P = n / 128, m = n / 64, rt = t.lt / P, l = t.lt % P;
+        const int row = 32 * (warp & 3) + lane, h = warp >> 2;
+        // per-thread parts of the output index: a stride for the tile's columns, a fixed offset
+        int64_t base = 0, step = 0;
+        int dr = 0;
+        if (M.bjmode == 0) { base = (int64_t)(128 * l) * n + 128 * rt + row; step = n; }
+        else if (M.bjmode == 1) { dr = dest(128 * rt + row, m, M.bjround); }
+        else { base = dest(128 * l + row, m, M.bjround); step = n; }
+        for (int cc = 0; cc < 32; cc += 16) {
+            float d[16];
+            tmem_ld16(tl + (uint32_t)(32 * h + cc), d);
+#pragma unroll
+            for (int e = 0; e < 16; ++e) {
+                const int col = 32 * h + cc + e;
+                int64_t a;
+                if (M.bjmode == 0) a = base + (int64_t)col * step;
+                else if (M.bjmode == 1) a = (int64_t)dest(128 * l + col, m, M.bjround) * n + dr;
+                else a = base + (int64_t)(128 * rt + col) * step;
+                const float v = d[e];
+                M.out[a] = v;
+                M.out_lo[a] = v - __uint_as_float(__float_as_uint(v) & 0xffffe000u);
+            }
+        }
+        return true;
+    }
+};
+
+// ------------------------------------------------------------------------------------------
 // PBuild: tile = 128 rows a.  D (128 x rpad) = Y[a, :] Yt[J, :]^T (K = k); the epilogue writes
 // P(a, q) = d_{J_q} ([a == J_q] - D(a, q)) (rounded to TF32) and P^T.  A = Y (m' x k), B = YtJ
 // (r x k, rows past r read as zeros).
@@ -1068,6 +1133,7 @@ template <> size_t stage_bytes_of<Compose>(const TcMat& M) { return 16384 + (siz
 template <> size_t stage_bytes_of<WBar>(const TcMat& M) { return 2 * 16384 + (size_t)M.kpad * 128; }
 template <> size_t stage_bytes_of<Lambda>(const TcMat&) { return 2 * 16384; }
 template <> size_t stage_bytes_of<LambdaU>(const TcMat&) { return 3 * 16384; }
+template <> size_t stage_bytes_of<BjacMul>(const TcMat&) { return 4 * 16384; }
 template <> size_t stage_bytes_of<PBuild>(const TcMat& M) { return 16384 + (size_t)M.rpad * 128; }
 template <> size_t stage_bytes_of<RBar>(const TcMat&) { return 2 * 16384; }
 template <> size_t stage_bytes_of<Update>(const TcMat&) { return 2 * 16384; }
@@ -1083,6 +1149,7 @@ template <> int acc_cols_of<Compose>(const TcMat& M) { return M.N * Compose::BN;
 template <> int acc_cols_of<WBar>(const TcMat& M) { return 2 * M.kpad; }
 template <> int acc_cols_of<Lambda>(const TcMat&) { return 128; }
 template <> int acc_cols_of<LambdaU>(const TcMat&) { return 256; }
+template <> int acc_cols_of<BjacMul>(const TcMat&) { return 128; }
 template <> int acc_cols_of<PBuild>(const TcMat& M) { return M.rpad; }
 template <> int acc_cols_of<RBar>(const TcMat&) { return 128; }
 template <> int acc_cols_of<Update>(const TcMat&) { return 128; }
@@ -1150,6 +1217,7 @@ cudaError_t launch_compose(TcGroup& g, cudaStream_t st) { return launch<Compose>
 cudaError_t launch_wbar(TcGroup& g, cudaStream_t st) { return launch<WBar>(g, st); }
 cudaError_t launch_lambda(TcGroup& g, cudaStream_t st) { return launch<Lambda>(g, st); }
 cudaError_t launch_lambda_u(TcGroup& g, cudaStream_t st) { return launch<LambdaU>(g, st); }
+cudaError_t launch_bjac(TcGroup& g, cudaStream_t st) { return launch<BjacMul>(g, st); }
 cudaError_t launch_pbuild(TcGroup& g, cudaStream_t st) { return launch<PBuild>(g, st); }
 cudaError_t launch_rbar(TcGroup& g, cudaStream_t st) { return launch<RBar>(g, st); }
 cudaError_t launch_update(TcGroup& g, cudaStream_t st) { return launch<Update>(g, st); }

@@ -315,11 +315,84 @@ def test_full_basis_blocked_refresh_matches_svd():
     off = np.abs(D - np.diag(np.diag(D))).max() / np.abs(D).max()
     msg = f"sweeps {st['last_refresh_sweeps']} orth {orth:.2e} lead {lead:.2e} off {off:.2e}"
     print(msg)
-    # fp32 rotations: a column passes ~30 rounds of 128-term products and 127-rotation pair sweeps
-    # per sweep, ~1e-5 of accumulated rounding over 15 sweeps (measured: orth 1.8e-5, leading
-    # columns 5e-5, off-diagonal 5e-6 relative)
+    # fp32 pair sweeps and split-TF32 block products (~2^-21 per product): a column passes ~30
+    # rounds of 128-term products and 127-rotation pair sweeps per sweep, a few 1e-5 of accumulated
+    # rounding over 15 sweeps (measured: orth 3.1e-5, leading columns 1.2e-4, off-diagonal 1e-5
+    # relative)
     assert 1 <= st["last_refresh_sweeps"] <= 30, msg
     assert orth <= 2e-4, msg
     assert lead <= 5e-4, msg
     assert off <= 5e-5, msg
     assert np.all(np.diff(np.diag(D)) <= 1e-5 * D[0, 0]), msg
+
+
+def test_full_basis_group_equals_single_steps():
+    """Full-basis handles of two sizes (1152 x 1280, 2048 x 1536 stored transposed) through one
+    grouped step are the same computation as per-handle steps, across two blocked-Jacobi refreshes
+    (the grouped refresh solves each size on its own): bit-identical X, E_0 and basis."""
+    import torch
+    import paper_2507_08784_gb300 as glr
+    shapes = [(1152, 1280), (2048, 1536)]
+    N, r = 2, 32
+    grads = [_grads(m, n, N, seed=71 + i, rho=64) for i, (m, n) in enumerate(shapes)]
+    mk = lambda: [glr.GreedyLore(m, n, r, N, grad_dtype="bf16", **_sched("adam", 3, 0, 130 + i))
+                  for i, (m, n) in enumerate(shapes)]
+    A, B = mk(), mk()
+    XA = [torch.zeros(m, n, device="cuda") for m, n in shapes]
+    XB = [torch.zeros(m, n, device="cuda") for m, n in shapes]
+    try:
+        for t in range(5):
+            Gd = [[torch.from_numpy(g).to(torch.bfloat16).cuda() for g in gr(t)] for gr in grads]
+            glr.glr_step_group([h.handle for h in A], Gd, XA)
+            for h, G, X in zip(B, Gd, XB):
+                h.step(G, X)
+        torch.cuda.synchronize()
+        for i in range(len(shapes)):
+            assert A[i].stats()["refreshes"] == 2
+            assert torch.equal(XA[i], XB[i]), f"matrix {i}: X differs"
+            assert torch.equal(A[i].error(0), B[i].error(0)), f"matrix {i}: E_0 differs"
+            assert torch.equal(A[i].basis(), B[i].basis()), f"matrix {i}: U differs"
+    finally:
+        for h in A + B:
+            h.close()
+
+
+def test_full_basis_checkpoint_resume_is_bit_identical():
+    """glr_save / glr_load of a full-basis handle on the tcgen05 path (U and its TF32 transpose are
+    part of the state): both handles continue identically across a refresh."""
+    import torch
+    import paper_2507_08784_gb300 as glr
+    m, n, r, N = 1280, 1536, 32, 2
+    grads = _grads(m, n, N, seed=5, rho=64)
+    kw = _sched("msgd", 3, 0, 44)
+    a = glr.GreedyLore(m, n, r, N, grad_dtype="bf16", **kw)
+    b = glr.GreedyLore(m, n, r, N, grad_dtype="bf16", **kw)
+    try:
+        Xa = torch.zeros(m, n, device="cuda")
+        Gs = [[torch.from_numpy(g).to(torch.bfloat16).cuda() for g in grads(t)] for t in range(7)]
+        for t in range(2):
+            a.step(Gs[t], Xa)
+        b.load_state_dict(a.state_dict())
+        Xb = Xa.clone()
+        for t in range(2, 7):
+            a.step(Gs[t], Xa)
+            b.step(Gs[t], Xb)
+            torch.cuda.synchronize()
+            assert torch.equal(Xa, Xb), t
+            assert np.array_equal(a.selection()[0], b.selection()[0]), t
+        assert torch.equal(a.basis(), b.basis())
+    finally:
+        a.close()
+        b.close()
+
+
+@pytest.mark.parametrize("m,n,kw", [
+    (2048, 2304, dict(grad_dtype="f32")),          # fp32 gradients: no full-basis path above 1024
+    (1100, 2304, dict(grad_dtype="bf16")),         # m' not a multiple of 128
+    (8192, 8192, dict(grad_dtype="bf16")),         # m' above 4096
+])
+def test_full_basis_above_1024_needs_tcgen05_conditions(m, n, kw):
+    import paper_2507_08784_gb300 as glr
+    with pytest.raises(glr.GlrError) as e:
+        glr.GreedyLore(m, n, 32, 2, basis_rank=0, tau=10, **kw)
+    assert "full basis" in str(e.value)
