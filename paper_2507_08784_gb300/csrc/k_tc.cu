@@ -736,22 +736,23 @@ struct BjacMul : NoData {
         const TcMat& M = g.mat[t.mat];
         const int n = M.mp, P = n / 128, m = n / 64, rt = t.lt / P, l = t.lt % P;
         const int row = 32 * (warp & 3) + lane, h = warp >> 2;
-        // per-thread parts of the output index: a stride for the tile's columns, a fixed offset
+        // per-thread parts of the output index: a stride for the tile's columns, a fixed offset;
+        // mode 1: a warp's 32 columns lie in one 64-block, whose next place is found once
         int64_t base = 0, step = 0;
-        int dr = 0;
         if (M.bjmode == 0) { base = (int64_t)(128 * l) * n + 128 * rt + row; step = n; }
-        else if (M.bjmode == 1) { dr = dest(128 * rt + row, m, M.bjround); }
-        else { base = dest(128 * l + row, m, M.bjround); step = n; }
+        else if (M.bjmode == 1) {
+            const int x0 = 128 * l + 32 * h;
+            base = (int64_t)(64 * bjac_dest_of(x0 >> 6, m, M.bjround) + (x0 & 63)) * n + dest(128 * rt + row, m, M.bjround);
+            step = n;
+        } else { base = dest(128 * l + row, m, M.bjround); step = n; }
         for (int cc = 0; cc < 32; cc += 16) {
             float d[16];
             tmem_ld16(tl + (uint32_t)(32 * h + cc), d);
 #pragma unroll
             for (int e = 0; e < 16; ++e) {
                 const int col = 32 * h + cc + e;
-                int64_t a;
-                if (M.bjmode == 0) a = base + (int64_t)col * step;
-                else if (M.bjmode == 1) a = (int64_t)dest(128 * l + col, m, M.bjround) * n + dr;
-                else a = base + (int64_t)(128 * rt + col) * step;
+                const int64_t a = M.bjmode == 2 ? base + (int64_t)(128 * rt + col) * step
+                                                : base + (int64_t)(cc + e + (M.bjmode == 0 ? 32 * h : 0)) * step;
                 const float v = d[e];
                 M.out[a] = v;
                 M.out_lo[a] = v - __uint_as_float(__float_as_uint(v) & 0xffffe000u);
