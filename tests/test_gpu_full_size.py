@@ -1,15 +1,16 @@
 """GPU checks at the full matrix sizes of the large workloads (marked gpu).
 
 Algorithm 3 matrices (the d = 2048 decoder's 5632 x 2048 FFN matrix with bf16 gradients and
-Adam; the d = 4096 decoder's 11008 x 4096 FFN matrix, r = 128, k = 256) run three steps through
-the C ABI against expected values from the oracle's building blocks alone, applied to the same
-gradients in the order of Algorithm 3.  The oracle's whole-step routine would form u_j^T M_i for
+Adam; the d = 4096 decoder's 11008 x 4096 FFN matrix, r = 128, k = 256, and the same matrix with
+the paper-exact full basis, k = m' = 4096) run three steps through the C ABI against expected
+values from the oracle's building blocks alone, applied to the same gradients in the order of
+Algorithm 3.  The oracle's whole-step routine would form u_j^T M_i for
 every node (about 1.5 TFLOP per step in fp64 at these sizes), so lambda-bar is formed once on the
 node mean instead, which the oracle's pins show equal to the node mean of the per-node lambdas:
 
-* the refresh basis is the oracle's SVD of its own Mbar, completed by its Householder routine,
-  and is copied into the device after the refresh step (glr_set_basis), so both sides select
-  from one U in the compressed steps;
+* the refresh basis is the oracle's SVD of its own Mbar, completed by its Householder routine
+  (the full basis: all m' left singular vectors), and is copied into the device after the refresh
+  step (glr_set_basis), so both sides select from one U in the compressed steps;
 * lambda-bar by the oracle's Algorithm 2 with its v_j draws, J by its arg-top-r, P = U[:, J],
   R_i = P^T M_i, E_i = M_i - P R_i, Ghat = P Rbar, and its MSGD / Adam on X.
 
@@ -54,10 +55,11 @@ def _node_grads(prob, li, t, transposed):
     return Gd, (np.swapaxes(G, 1, 2) if transposed else G)
 
 
-def _handle(glr, cfg, li, seed, tau, mode):
+def _handle(glr, cfg, li, seed, tau, mode, basis_rank=None):
     m, n = cfg.shapes[li]
+    k = cfg.basis_rank if basis_rank is None else basis_rank
     return glr.GreedyLore(m, n, cfg.r, cfg.N, tau=tau, refresh_mode=mode, optimizer=cfg.optimizer, lr=cfg.lr,
-                          beta1=cfg.beta1, beta2=cfg.beta2, eps=cfg.eps, seed=seed, basis_rank=cfg.basis_rank,
+                          beta1=cfg.beta1, beta2=cfg.beta2, eps=cfg.eps, seed=seed, basis_rank=k,
                           power_iters=cfg.power_iters, grad_dtype=cfg.grad_dtype)
 
 
@@ -79,8 +81,11 @@ def _optimizer(cfg, Xo, Mo, Vo, Gh):
     return Xo, Mo, Vo
 
 
-@pytest.mark.parametrize("name,li", [("cfg3_llama_d2048", 4), ("cfg5_llama_d4096", 4)])
-def test_full_size_algorithm3_steps(name, li):
+@pytest.mark.parametrize("name,li,full", [("cfg3_llama_d2048", 4, False), ("cfg5_llama_d4096", 4, False),
+                                          ("cfg5_llama_d4096", 4, True)])
+def test_full_size_algorithm3_steps(name, li, full):
+    """full: the paper-exact basis (basis_rank = 0; the blocked Jacobi refresh and the dense
+    scores U^T Mbar), U the oracle's full SVD basis of its own Mbar."""
     import torch
     import paper_2507_08784_gb300 as glr
 
@@ -89,9 +94,11 @@ def test_full_size_algorithm3_steps(name, li):
     m, n = cfg.shapes[li]
     transposed = m > n
     mp, npr = min(m, n), max(m, n)
-    r, N, k = cfg.r, cfg.N, cfg.basis_rank
+    r, N = cfg.r, cfg.N
+    k = mp if full else cfg.basis_rank
     seed = 4242 + li
-    dev = _handle(glr, cfg, li, seed, cfg.tau, "alg3")
+    dev = _handle(glr, cfg, li, seed, cfg.tau, "alg3", 0 if full else None)
+    assert dev.stats()["k"] == k
     tc = dev.stats()["path"] == 2
     tol = 2e-2 if tc else 1e-5
     lam_tol, tie = (2e-2, 1e-2) if tc else (1e-5, 1e-5)
@@ -112,7 +119,8 @@ def test_full_size_algorithm3_steps(name, li):
             if t % cfg.tau == 0:                              # refresh: uncompressed mean, E reset
                 U, s = O.left_singular_basis(Mbar)
                 _check_refresh(dev, Mbar, s, k, t)
-                U = O.householder_complement(U[:, :k])
+                if not full:
+                    U = O.householder_complement(U[:, :k])
                 dev.set_basis(torch.from_numpy(np.ascontiguousarray(U[:, :k])).float().cuda())
                 assert np.all(J == -1)
                 Ghat = Mbar
