@@ -37,13 +37,14 @@ def _grads(m, n, N, seed, rho=48, noise=0.01):
     return at
 
 
-@pytest.mark.parametrize("m,n,mode", [(256, 704, "alg3"), (704, 256, "alg3"), (256, 640, "alg4")])
-def test_dp_shards_match_single_handle(m, n, mode):
+@pytest.mark.parametrize("m,n,mode,k", [(256, 704, "alg3", 64), (704, 256, "alg3", 64), (256, 640, "alg4", 64),
+                                        (1152, 1280, "alg3", 0)])      # the full basis (blocked Jacobi)
+def test_dp_shards_match_single_handle(m, n, mode, k):
     import torch
     import paper_2507_08784_gb300 as glr
     from paper_2507_08784_gb300.dp import DataParallelGreedyLore, ShardEngine
 
-    r, N, k, steps = 32, 4, 64, 7
+    r, N, steps = 32, 4, 7
     sched = dict(tau=3, refresh_mode=mode, optimizer="adam", lr=1e-3, beta1=0.9, beta2=0.999, eps=1e-8, seed=5,
                  basis_rank=k, grad_dtype="bf16")
     grads = _grads(m, n, N, seed=m + n)
