@@ -547,7 +547,7 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--only-headline", action="store_true",
                     help="time the headline workload only (no extra workloads, no e2e, no CPU baseline)")
-    ap.add_argument("--e2e-steps", type=int, default=5)
+    ap.add_argument("--e2e-steps", type=int, default=10)
     ap.add_argument("--refresh-reps", type=int, default=3)
     ap.add_argument("--ncu-case", nargs="?", const="steps", choices=["steps", "refresh", "stress", "exact"],
                     help="a small case for kernel captures: one 4096 x 4096 matrix of the headline stack "
