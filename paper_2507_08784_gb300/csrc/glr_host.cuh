@@ -70,6 +70,7 @@ struct glr_handle {
     // ... and the TF32 low parts of the rotations' operands: J^T, H, T^T (in jwork) and both V buffers
     float *bjJlo = nullptr, *Hlo = nullptr, *Ttlo = nullptr, *Vlo = nullptr, *V2lo = nullptr;
     int bj_sweeps = 0, numeric_failures_host = 0;
+    const float* bj_V = nullptr;       // the blocked Jacobi's final V (after a refresh that used it)
     // a data-parallel step in progress (glr_dp_begin / glr_dp_select / glr_dp_finish): 0 idle,
     // 1 begun, 2 selected; the step's plan and the caller's gradient pointers
     int dp_stage = 0, dp_flags = 0;
@@ -205,6 +206,7 @@ enum TcMap { kMapBt, kMapPT0, kMapPT1, kMapP0, kMapP1, kMapRwT, kMapMbarT, kMapY
 const CUtensorMap* tcl_grad_maps(glr_handle* h, const void* const* G, cudaStream_t st, int* rc);
 const CUtensorMap* tcl_x_map(glr_handle* h, const float* X, cudaStream_t st, int* rc);
 bool tcl_eligible(int64_t mp, int64_t np, int r, int N, int k, bool exact, const glr_schedule* s);
+bool tcl_rr_blocked(const glr_handle* h);
 int tcl_alloc(glr_handle* h);         // state buffers (before n_state_allocs is fixed)
 int tcl_maps(glr_handle* h);          // the device map table (after)
 float* tcl_PT_of(const glr_handle* h, const float* P);

@@ -337,6 +337,17 @@ struct BjacGroup {
 };
 // J_k^T of every pair of every matrix: one Jacobi sweep on H's 128 x 128 diagonal pair blocks
 cudaError_t bjac_pairs(BjacGroup& g, cudaStream_t st);
+// The start of a solve: H = sum of nparts partials (leading dimension ld; nparts = 0: H given),
+// H_lo = H - trunc_tf32(H), V = I, V_lo = 0 (all n x n row-major)
+struct BjacPrep {
+    const float* part; int nparts, ld, n;
+    float *H, *Hlo, *V, *Vlo;
+};
+struct BjacPrepGroup {
+    int nmat;
+    BjacPrep mat[kBjacGroupMax];
+};
+cudaError_t bjac_prep(const BjacPrepGroup& g, cudaStream_t st);
 // part[2 (i kBjacNormCtas + c) + {0, 1}]: CTA c's squared diagonal / off-diagonal sums of H_i
 cudaError_t bjac_norms(const BjacGroup& g, float* part, cudaStream_t st);
 cudaError_t bjac_eye(float* V, int n, cudaStream_t st);

@@ -180,66 +180,38 @@ int refresh_exact_grouped(std::vector<glr_handle*>& hs) {
     return GLR_OK;
 }
 
-// Full-basis refreshes above m' = 1024 (k_bjac.cu), all on the first handle's side stream:
-// H = Mbar Mbar^T by the grouped FFMA product (Mbar is column-major on the tcgen05 path), V = I,
-// then the blocked Jacobi rounds of every matrix of the same size together, one sweep at a time,
-// each sweep opened by the norm check (summed on the host in a fixed order, so that the decision
-// does not depend on the grouping).  A round: the pair sweeps (J_k^T and its low part), then the
-// three split-TF32 products of tc_kernel<BjacMul>: T^T = (H J)^T, H <- T^T J, V' <- V J (V and
-// V' trade buffers).  Finally each handle's sorted, sign-fixed U and its TF32 transpose.  A matrix
-// that has not converged after kBjacMaxSweeps sweeps keeps its last basis and counts a numeric
-// failure (GLR_ENUMERIC from glr_get_stats).
+// The blocked Jacobi (k_bjac.cu) for a set of symmetric n x n problems, n a multiple of 128 from
+// 256 to 4096: the full basis's m' x m' eigenproblem, or a truncated refresh's k x k Rayleigh-Ritz
+// problem.  Each problem lives in its handle's buffers (H in Hbuf with its low part in Hlo, T^T in
+// jwork / Ttlo, V in Vbuf / Vbuf2 with Vlo / V2lo, the rotations in bjJ / bjJlo) and the kMapBj*
+// tensor maps over them; bjac_prep has set H, H_lo, V = I, V_lo = 0.  The problems of one size run
+// together, one sweep at a time, each sweep opened by the norm check (per-CTA partials summed on
+// the host in a fixed order, so that the decision does not depend on the grouping); a round is the
+// pair sweeps (J_k^T and its low part), then the three split-TF32 products of tc_kernel<BjacMul>:
+// T^T = (H J)^T, H <- T^T J, V' <- V J.  A problem that has not converged after kBjacMaxSweeps
+// sweeps keeps its last V and counts a numeric failure (GLR_ENUMERIC from glr_get_stats).
 constexpr int kBjacMaxSweeps = 30;
 
-int refresh_exact_blocked(std::vector<glr_handle*>& hs) {
-    glr_handle* h0 = hs[0];
-    cudaStream_t s0 = h0->rstream;
-    for (glr_handle* h : hs) {
-        if (h == h0) continue;
-        GLR_CK(h, cudaEventRecord(h->rpow, h->rstream));
-        GLR_CK(h0, cudaStreamWaitEvent(s0, h->rpow, 0));
-    }
-    PhaseScope ps(h0, GLR_PH_REFRESH, s0);
-    {   // H = Mbar Mbar^T (Mbar^T is n' x m' row-major) and its low part; V = I, V_lo = 0
-        GemmGroup gg{};
-        auto flush = [&]() -> int {
-            if (gg.nmat) GLR_LAUNCH(h0, 1, gemm_group_f32(gg, s0));
-            gg.nmat = 0;
-            return GLR_OK;
-        };
-        for (glr_handle* h : hs) {
-            GemmMat& G = gg.mat[gg.nmat++];
-            G = GemmMat{};
-            G.M = h->mp; G.N = h->mp; G.K = h->np; G.alpha = 1.f;
-            G.A = h->Mbar; G.sAi = 1; G.sAp = h->mp;
-            G.B = h->Mbar; G.sBp = h->mp; G.sBj = 1;
-            G.C = h->Hbuf; G.sCi = h->mp; G.sCj = 1;
-            if (gg.nmat == 64 && flush() != GLR_OK) return GLR_ECUDA;
-        }
-        if (flush() != GLR_OK) return GLR_ECUDA;
-        for (glr_handle* h : hs) {
-            const int64_t nn = (int64_t)h->mp * h->mp;
-            GLR_LAUNCH(h, 1, tc::split_lo(h->Hbuf, h->Hlo, nn, s0));
-            GLR_LAUNCH(h, 1, bjac_eye(h->Vbuf, h->mp, s0));
-            GLR_CK(h, cudaMemsetAsync(h->Vlo, 0, sizeof(float) * nn, s0));
-        }
-    }
-    struct State { glr_handle* h; int vpar, rd; bool done; };
-    std::vector<State> all;
-    for (glr_handle* h : hs) all.push_back(State{h, 0, 0, false});
+struct BjItem {
+    glr_handle* h;
+    int n, vpar, rd;
+    bool done;
+    const float* V() const { return vpar ? h->Vbuf2 : h->Vbuf; }
+};
+
+int bjac_run(std::vector<BjItem>& all, glr_handle* h0, cudaStream_t s0) {
+    std::stable_sort(all.begin(), all.end(), [](const BjItem& a, const BjItem& b) { return a.n < b.n; });
     std::vector<float> part;
     static thread_local tc::TcGroup tg;
     for (size_t a0 = 0; a0 < all.size();) {
-        // the matrices of one size
-        size_t a1 = a0;
-        while (a1 < all.size() && all[a1].h->mp == all[a0].h->mp) ++a1;
-        const int n = all[a0].h->mp, m = n / 64, P = n / 128;
+        size_t a1 = a0;                                         // the problems of one size
+        while (a1 < all.size() && all[a1].n == all[a0].n) ++a1;
+        const int n = all[a0].n, m = n / 64, P = n / 128;
         const double tol = 4.0 * 5.96e-8 * std::sqrt((double)n) + 1e-7;
         for (int sweep = 0;; ++sweep) {
-            // the norm check of every unfinished matrix
-            std::vector<State*> act;
-            for (size_t a = a0; a < a1; ++a)
-                if (!all[a].done) act.push_back(&all[a]);
+            std::vector<BjItem*> act;
+            for (size_t i = a0; i < a1; ++i)
+                if (!all[i].done) act.push_back(&all[i]);
             for (size_t c0 = 0; c0 < act.size(); c0 += kBjacGroupMax) {
                 BjacGroup g{};
                 for (size_t c = c0; c < act.size() && c < c0 + kBjacGroupMax; ++c) {
@@ -256,7 +228,7 @@ int refresh_exact_blocked(std::vector<glr_handle*>& hs) {
                         d += part[2 * ((size_t)i * kBjacNormCtas + c)];
                         o += part[2 * ((size_t)i * kBjacNormCtas + c) + 1];
                     }
-                    State* S = act[c0 + i];
+                    BjItem* S = act[c0 + i];
                     if (o <= tol * tol * (o + d)) S->done = true;
                     else if (sweep == kBjacMaxSweeps) {
                         S->done = true;
@@ -265,7 +237,7 @@ int refresh_exact_blocked(std::vector<glr_handle*>& hs) {
                     if (S->done) S->h->bj_sweeps = sweep;
                 }
             }
-            act.erase(std::remove_if(act.begin(), act.end(), [](State* S) { return S->done; }), act.end());
+            act.erase(std::remove_if(act.begin(), act.end(), [](BjItem* S) { return S->done; }), act.end());
             if (act.empty()) break;
             for (int round = 0; round < m - 1; ++round) {
                 for (size_t c0 = 0; c0 < act.size(); c0 += kBjacGroupMax) {
@@ -280,7 +252,7 @@ int refresh_exact_blocked(std::vector<glr_handle*>& hs) {
                     for (size_t c0 = 0; c0 < act.size(); c0 += tc::kTcGroupMax) {
                         tg.nmat = 0; tg.total_tiles = 0; tg.err = h0->dflags + 2;
                         for (size_t c = c0; c < act.size() && c < c0 + tc::kTcGroupMax; ++c) {
-                            const State* S = act[c];
+                            const BjItem* S = act[c];
                             glr_handle* h = S->h;
                             tc::TcMat M{};
                             M.mp = n; M.ntiles = P * P; M.tile0 = tg.total_tiles; M.bjmode = mode; M.bjround = S->rd;
@@ -304,7 +276,7 @@ int refresh_exact_blocked(std::vector<glr_handle*>& hs) {
                         GLR_LAUNCH(h0, 1, tc::launch_bjac(tg, s0));
                     }
                 }
-                for (State* S : act) {
+                for (BjItem* S : act) {
                     S->vpar ^= 1;
                     S->rd = (S->rd + 1) % (m - 1);
                 }
@@ -312,17 +284,75 @@ int refresh_exact_blocked(std::vector<glr_handle*>& hs) {
         }
         a0 = a1;
     }
-    for (State& S : all) {
+    for (BjItem& S : all) {
         glr_handle* h = S.h;
-        const int n = h->mp;
-        GLR_LAUNCH(h, 1, bjac_diag(h->Hbuf, n, h->evals, s0));
-        GLR_LAUNCH(h, 1, sort_fix_basis(h->evals, S.vpar ? h->Vbuf2 : h->Vbuf, n, n, h->U, n, h->evals_sorted, s0));
-        GLR_LAUNCH(h, 1, tc::transpose_round(h->UT, n, h->U, n, n, n, s0));
         GLR_CK(h, cudaMemcpyAsync(h->dflags + 1, &h->bj_sweeps, sizeof(int), cudaMemcpyHostToDevice, s0));
         if (h->numeric_failures_host) {
             GLR_LAUNCH(h, 1, count_flag(h->dflags + 6, h->numeric_failures_host, s0));
             h->numeric_failures_host = 0;
         }
+    }
+    return GLR_OK;
+}
+
+// bjac_prep over the items (in groups); part(h) gives a problem's partials and their count and
+// leading dimension (count 0: H is already in Hbuf).
+template <class Parts>
+int bjac_prepare(const std::vector<BjItem>& items, glr_handle* h0, cudaStream_t s0, Parts parts) {
+    for (size_t c0 = 0; c0 < items.size(); c0 += kBjacGroupMax) {
+        BjacPrepGroup g{};
+        for (size_t c = c0; c < items.size() && c < c0 + kBjacGroupMax; ++c) {
+            glr_handle* h = items[c].h;
+            BjacPrep& P = g.mat[g.nmat++];
+            P.n = items[c].n; P.H = h->Hbuf; P.Hlo = h->Hlo; P.V = h->Vbuf; P.Vlo = h->Vlo;
+            parts(h, P);
+        }
+        GLR_LAUNCH(h0, 1, bjac_prep(g, s0));
+    }
+    return GLR_OK;
+}
+
+// Full-basis refreshes above m' = 1024, all on the first handle's side stream: H = Mbar Mbar^T by
+// the grouped FFMA product (Mbar is column-major on the tcgen05 path), the blocked Jacobi, then
+// each handle's sorted, sign-fixed U and its TF32 transpose.
+int refresh_exact_blocked(std::vector<glr_handle*>& hs) {
+    glr_handle* h0 = hs[0];
+    cudaStream_t s0 = h0->rstream;
+    for (glr_handle* h : hs) {
+        if (h == h0) continue;
+        GLR_CK(h, cudaEventRecord(h->rpow, h->rstream));
+        GLR_CK(h0, cudaStreamWaitEvent(s0, h->rpow, 0));
+    }
+    PhaseScope ps(h0, GLR_PH_REFRESH, s0);
+    {   // H = Mbar Mbar^T (Mbar^T is n' x m' row-major)
+        GemmGroup gg{};
+        auto flush = [&]() -> int {
+            if (gg.nmat) GLR_LAUNCH(h0, 1, gemm_group_f32(gg, s0));
+            gg.nmat = 0;
+            return GLR_OK;
+        };
+        for (glr_handle* h : hs) {
+            GemmMat& G = gg.mat[gg.nmat++];
+            G = GemmMat{};
+            G.M = h->mp; G.N = h->mp; G.K = h->np; G.alpha = 1.f;
+            G.A = h->Mbar; G.sAi = 1; G.sAp = h->mp;
+            G.B = h->Mbar; G.sBp = h->mp; G.sBj = 1;
+            G.C = h->Hbuf; G.sCi = h->mp; G.sCj = 1;
+            if (gg.nmat == 64 && flush() != GLR_OK) return GLR_ECUDA;
+        }
+        if (flush() != GLR_OK) return GLR_ECUDA;
+    }
+    std::vector<BjItem> items;
+    for (glr_handle* h : hs) items.push_back(BjItem{h, h->mp, 0, 0, false});
+    int rc = bjac_prepare(items, h0, s0, [](glr_handle*, BjacPrep& P) { P.nparts = 0; });
+    if (rc == GLR_OK) rc = bjac_run(items, h0, s0);
+    if (rc != GLR_OK) return rc;
+    for (const BjItem& S : items) {
+        glr_handle* h = S.h;
+        const int n = h->mp;
+        GLR_LAUNCH(h, 1, bjac_diag(h->Hbuf, n, h->evals, s0));
+        GLR_LAUNCH(h, 1, sort_fix_basis(h->evals, S.V(), n, n, h->U, n, h->evals_sorted, s0));
+        GLR_LAUNCH(h, 1, tc::transpose_round(h->UT, n, h->U, n, n, n, s0));
     }
     GLR_CK(h0, cudaEventRecord(h0->rpow, s0));
     for (glr_handle* h : hs)
@@ -648,19 +678,40 @@ int refresh_tcl_grouped(std::vector<glr_handle*>& hs) {
         return true;
     });
     if (rc != GLR_OK) return rc;
-    for (size_t c0 = 0; c0 < hs.size(); c0 += kEigGroupMax) {
+    // the k x k problems: the blocked Jacobi for k a multiple of 128 from 256, else one CTA each
+    std::vector<glr_handle*> small;
+    std::vector<BjItem> big;
+    for (glr_handle* h : hs) {
+        if (tcl_rr_blocked(h)) big.push_back(BjItem{h, h->k, 0, 0, false});
+        else small.push_back(h);
+        h->bj_V = nullptr;
+    }
+    for (size_t c0 = 0; c0 < small.size(); c0 += kEigGroupMax) {
         EigGroup g{};
         g.max_sweeps = 40;
-        for (size_t i = c0; i < hs.size() && i < c0 + (size_t)kEigGroupMax; ++i) {
-            glr_handle* h = hs[i];
+        for (size_t i = c0; i < small.size() && i < c0 + (size_t)kEigGroupMax; ++i) {
+            glr_handle* h = small[i];
             EigMat& M = g.mat[g.nmat++];
             const int n = h->k;
             M.n = n; M.tol = 4.f * 5.96e-8f * sqrtf(static_cast<float>(n)) + 1e-7f;
             M.H = h->gpart; M.nparts = cdiv(h->np, tc::kGramChunk); M.ld = h->kpad;
             M.V = h->Vk; M.evals = h->evals; M.sweeps = h->dflags + 1;
         }
-        PhaseScope ps(hs[c0], GLR_PH_REFRESH, s0);
-        GLR_LAUNCH(hs[c0], 1, eig_tmem_group(g, s0));
+        PhaseScope ps(small[c0], GLR_PH_REFRESH, s0);
+        GLR_LAUNCH(small[c0], 1, eig_tmem_group(g, s0));
+    }
+    if (!big.empty()) {
+        glr_handle* b0 = big[0].h;
+        PhaseScope ps(b0, GLR_PH_REFRESH, s0);
+        rc = bjac_prepare(big, b0, s0, [](glr_handle* h, BjacPrep& P) {
+            P.part = h->gpart; P.nparts = cdiv(h->np, tc::kGramChunk); P.ld = h->kpad;
+        });
+        if (rc == GLR_OK) rc = bjac_run(big, b0, s0);
+        if (rc != GLR_OK) return rc;
+        for (const BjItem& S : big) {
+            GLR_LAUNCH(S.h, 1, bjac_diag(S.h->Hbuf, S.n, S.h->evals, s0));
+            S.h->bj_V = S.V();
+        }
     }
     // the finish, grouped: sorted Ritz pairs, Q <- Q W, column signs, the Householder WY form,
     // Yt = Y T^T, then Y^T for the W = Y^T Mbar products
@@ -669,7 +720,8 @@ int refresh_tcl_grouped(std::vector<glr_handle*>& hs) {
         for (size_t i = c0; i < hs.size() && i < c0 + 64; ++i) {
             glr_handle* h = hs[i];
             FinishMat& F = fg.mat[fg.nmat++];
-            F.mp = h->mp; F.k = h->k; F.evals = h->evals; F.V = h->Vk; F.W = h->gram; F.evals_sorted = h->evals_sorted;
+            F.mp = h->mp; F.k = h->k; F.evals = h->evals; F.V = h->bj_V ? h->bj_V : h->Vk; F.W = h->gram;
+            F.evals_sorted = h->evals_sorted;
             F.Wtop = h->scratch; F.Y = h->Y; F.T = h->T; F.s = h->dsign;
         }
         PhaseScope ps(hs[c0], GLR_PH_REFRESH, s0);

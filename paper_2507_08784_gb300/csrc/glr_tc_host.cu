@@ -14,6 +14,10 @@ inline int up32(int x) { return (x + 31) & ~31; }
 // multiples for every tile copy (m', n' multiples of 8, r, k of 4), at most 8 nodes (N x 64 accumulator
 // columns), 16 <= r <= 128 (the projected mean takes one 128-row tile), k <= 256 (one MMA's N)
 // and m' >= 128 (one MMA's M).
+// A truncated refresh's k x k Rayleigh-Ritz eigenproblem goes to the blocked Jacobi when k is a
+// multiple of 128 from 256 (its pairs are 128 x 128); smaller k stay on the one-CTA solver.
+bool tcl_rr_blocked(const glr_handle* h) { return !h->exact && h->k >= 256 && h->k % 128 == 0; }
+
 bool tcl_eligible(int64_t mp, int64_t np, int r, int N, int k, bool exact, const glr_schedule* s) {
     if (s->grad_dtype != GLR_BF16) return false;
     // the full basis takes this path above m' = 1024 only (the blocked Jacobi's 128-index pairs)
@@ -74,6 +78,12 @@ int tcl_maps(glr_handle* h) {
             A(&h->Mrow, mp * np); A(&h->Mlo, mp * np);
             A(&h->QTt, kp * mp); A(&h->ZTt, kp * np);
             A(&h->gpart, std::max<size_t>(nch, 1) * kp * kp); A(&h->Linv, kp * kp);
+            if (tcl_rr_blocked(h)) {        // the k x k Rayleigh-Ritz problem by the blocked Jacobi
+                A(&h->Hbuf, k * k); A(&h->Hlo, k * k); A(&h->jwork, k * k); A(&h->Ttlo, k * k);
+                A(&h->Vbuf, k * k); A(&h->Vlo, k * k); A(&h->Vbuf2, k * k); A(&h->V2lo, k * k);
+                A(&h->bjJ, k * 128); A(&h->bjJlo, k * 128);
+                A(&h->bjpart, (size_t)2 * kBjacNormCtas * kBjacGroupMax);
+            }
         }
         if (rc != GLR_OK) return rc;
     }
@@ -101,13 +111,18 @@ int tcl_maps(glr_handle* h) {
     if (h->exact) {
         m2(kMapUT, h->UT, mp, mp, mp, 128);                // U^T (TF32), row-major m' x m'
         m3(kMapMbar3, h->Mbar, mp, np, 1, 128);            // Mbar^T as a one-node B^T
-        // the blocked Jacobi's operands (rows of 128, K slices of 32) and their TF32 low parts
-        m2(kMapBjH, h->Hbuf, mp, mp, mp, 128);  m2(kMapBjHlo, h->Hlo, mp, mp, mp, 128);
-        m2(kMapBjT, h->jwork, mp, mp, mp, 128); m2(kMapBjTlo, h->Ttlo, mp, mp, mp, 128);
-        m2(kMapBjV0, h->Vbuf, mp, mp, mp, 128); m2(kMapBjV0lo, h->Vlo, mp, mp, mp, 128);
-        m2(kMapBjV1, h->Vbuf2, mp, mp, mp, 128); m2(kMapBjV1lo, h->V2lo, mp, mp, mp, 128);
-        m2(kMapBjJ, h->bjJ, 128, mp, 128, 128); m2(kMapBjJlo, h->bjJlo, 128, mp, 128, 128);
-    } else {
+    }
+    if (h->bjJ) {
+        // the blocked Jacobi's operands (rows of 128, K slices of 32) and their TF32 low parts; its
+        // problem is n = m' for the full basis, k for a truncated refresh's Rayleigh-Ritz step
+        const uint64_t bn = h->exact ? mp : k;
+        m2(kMapBjH, h->Hbuf, bn, bn, bn, 128);  m2(kMapBjHlo, h->Hlo, bn, bn, bn, 128);
+        m2(kMapBjT, h->jwork, bn, bn, bn, 128); m2(kMapBjTlo, h->Ttlo, bn, bn, bn, 128);
+        m2(kMapBjV0, h->Vbuf, bn, bn, bn, 128); m2(kMapBjV0lo, h->Vlo, bn, bn, bn, 128);
+        m2(kMapBjV1, h->Vbuf2, bn, bn, bn, 128); m2(kMapBjV1lo, h->V2lo, bn, bn, bn, 128);
+        m2(kMapBjJ, h->bjJ, 128, bn, 128, 128); m2(kMapBjJlo, h->bjJlo, 128, bn, 128, 128);
+    }
+    if (!h->exact) {
     m2(kMapYT, h->YTk, mp, kp, mp, (uint32_t)kp);          // Y^T: kpad x m'
     m2(kMapYt, h->Yt, k, mp, k, 128);                      // Yt, row-major m' x k
     m2(kMapWT, h->WT, kp, np, kp, 128);                    // W^T: n' x kpad

@@ -175,6 +175,27 @@ __global__ void __launch_bounds__(PT, 2) bjac_pair_kernel(const __grid_constant_
     }
 }
 
+// Before the first round, per problem: H = the sum of nparts partial matrices (leading dimension
+// ld; none when H is already formed), H's TF32 low part, V = I and V's low part 0.
+__global__ void bjac_prep_kernel(const __grid_constant__ BjacPrepGroup g) {
+    const BjacPrep& P = g.mat[blockIdx.y];
+    const int n = P.n;
+    for (int64_t q = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; q < (int64_t)n * n; q += (int64_t)gridDim.x * blockDim.x) {
+        const int r = (int)(q / n), c = (int)(q % n);
+        float h;
+        if (P.nparts > 0) {
+            h = 0.f;
+            for (int p = 0; p < P.nparts; ++p) h += P.part[(int64_t)p * P.ld * P.ld + (int64_t)r * P.ld + c];
+            P.H[q] = h;
+        } else {
+            h = P.H[q];
+        }
+        P.Hlo[q] = h - __uint_as_float(__float_as_uint(h) & 0xffffe000u);
+        P.V[q] = r == c ? 1.f : 0.f;
+        P.Vlo[q] = 0.f;
+    }
+}
+
 __global__ void count_flag_kernel(int* flag, int v) { atomicAdd(flag, v); }
 
 __global__ void bjac_eye_kernel(float* V, int n) {
@@ -206,6 +227,12 @@ cudaError_t bjac_pairs(BjacGroup& g, cudaStream_t st) {
 cudaError_t bjac_norms(const BjacGroup& g, float* part, cudaStream_t st) {
     if (g.nmat <= 0) return cudaSuccess;
     bjac_norms_kernel<<<dim3(kBjacNormCtas, g.nmat), 256, 0, st>>>(g, part);
+    return cudaGetLastError();
+}
+
+cudaError_t bjac_prep(const BjacPrepGroup& g, cudaStream_t st) {
+    if (g.nmat <= 0) return cudaSuccess;
+    bjac_prep_kernel<<<dim3(64, g.nmat), 256, 0, st>>>(g);
     return cudaGetLastError();
 }
 
