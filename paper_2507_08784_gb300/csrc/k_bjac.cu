@@ -59,15 +59,17 @@ __global__ void __launch_bounds__(256) bjac_norms_kernel(const __grid_constant__
 // from W = I: 127 rounds of 64 disjoint rotations (circle ordering; Golub & Van Loan sym.schur2),
 // each round's rotations formed from the round's own 2 x 2 diagonal blocks, then S <- R^T S R and
 // W <- W R in one barrier-separated phase.  S is packed (upper triangle by rows), W padded to 129
-// columns; J_k^T is written row-major with its TF32 low part.  512 threads, two CTAs per SM.
-constexpr int PT = 512;
+// columns; J_k^T is written row-major with its TF32 low part.  PT = 512 threads with two CTAs per
+// SM when a launch has more pairs than SMs, else PT = 1024 (half the work per thread and round:
+// each update's arithmetic is the same, so the results are too).
 constexpr int PN = 128, PH = 64, PLD = 129;
 constexpr int kPairItems = PH * (PH + 1) / 2;                 // 2 x 2 blocks (bi <= bj) of a round
 constexpr size_t kPairSmem = sizeof(float) * (PN * (PN + 1) / 2 + PN * PLD);
 
 __device__ __forceinline__ int pcircle(int x) { return 1 + ((x % (PN - 1)) + (PN - 1)) % (PN - 1); }
 
-__global__ void __launch_bounds__(PT, 2) bjac_pair_kernel(const __grid_constant__ BjacGroup g) {
+template <int PT>
+__global__ void __launch_bounds__(PT, 1024 / PT) bjac_pair_kernel(const __grid_constant__ BjacGroup g) {
     extern __shared__ float psm[];
     float* Ss = psm;                                   // packed upper triangle: (r, c >= r) at off[r] + c
     float* Ws = psm + PN * (PN + 1) / 2;               // W[a][j] at a PLD + j
@@ -218,9 +220,21 @@ cudaError_t bjac_pairs(BjacGroup& g, cudaStream_t st) {
         M.tile0p = tiles;
         tiles += M.n / 128;
     }
-    cudaError_t e = cudaFuncSetAttribute(bjac_pair_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kPairSmem);
-    if (e != cudaSuccess) return e;
-    bjac_pair_kernel<<<tiles, PT, kPairSmem, st>>>(g);
+    static int sms = 0;
+    if (!sms) {
+        int dev = 0;
+        cudaGetDevice(&dev);
+        cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+    }
+    if (tiles <= sms) {
+        cudaError_t e = cudaFuncSetAttribute(bjac_pair_kernel<1024>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kPairSmem);
+        if (e != cudaSuccess) return e;
+        bjac_pair_kernel<1024><<<tiles, 1024, kPairSmem, st>>>(g);
+    } else {
+        cudaError_t e = cudaFuncSetAttribute(bjac_pair_kernel<512>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kPairSmem);
+        if (e != cudaSuccess) return e;
+        bjac_pair_kernel<512><<<tiles, 512, kPairSmem, st>>>(g);
+    }
     return cudaGetLastError();
 }
 
