@@ -306,15 +306,15 @@ cudaError_t eig_tmem_group(const EigGroup& g, cudaStream_t st);
 // fixed, the others one slot further each round; slots s and m - 1 - s pair up and are stored at
 // positions 2 s, 2 s + 1): the storage position of block x in round rd, the block at position p,
 // and where the data at position p of round rd goes for round rd + 1.
-__device__ __forceinline__ int bjac_position_of(int x, int m, int rd) {
+__host__ __device__ __forceinline__ int bjac_position_of(int x, int m, int rd) {
     const int s = x == 0 ? 0 : 1 + ((x - 1 - rd) % (m - 1) + (m - 1)) % (m - 1);
     return s < m / 2 ? 2 * s : 2 * (m - 1 - s) + 1;
 }
-__device__ __forceinline__ int bjac_block_at(int p, int m, int rd) {
+__host__ __device__ __forceinline__ int bjac_block_at(int p, int m, int rd) {
     const int s = (p & 1) ? m - 1 - (p >> 1) : (p >> 1);
     return s == 0 ? 0 : 1 + (s - 1 + rd) % (m - 1);
 }
-__device__ __forceinline__ int bjac_dest_of(int p, int m, int rd) {
+__host__ __device__ __forceinline__ int bjac_dest_of(int p, int m, int rd) {
     return bjac_position_of(bjac_block_at(p, m, rd), m, (rd + 1) % (m - 1));
 }
 
